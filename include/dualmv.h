@@ -1,0 +1,162 @@
+/*
+ * dualmv — fused dual matrix-vector product for NVIDIA GB300 (sm_103a).
+ *
+ *     q = A * p        (q_i = sum_j A_ij p_j,  i < M)
+ *     s = A^T * r      (s_j = sum_i A_ij r_i,  j < N)
+ *
+ * both from a single pass over A.  This is the BICG kernel that the paper
+ * tunes (Table 1 and Table 2, row "BICG", Section 4.2); the paper names it
+ * without printing a formula, and the definition above is PolyBench's BiCG
+ * sub-kernel.
+ *
+ * Conventions shared by every entry point below
+ * ---------------------------------------------
+ * Layout.  A is M x N, row-major, element (i, j) at A[i * lda + j], with
+ *   lda >= max(1, N).  Columns N..lda-1 of each row are padding and are never
+ *   read.  p has N elements, r has M, q has M, s has N; all are contiguous.
+ * Memory.  Every pointer is caller-owned DEVICE memory on the current CUDA
+ *   device (cudaSetDevice).  Nothing is copied to or from the host.  Outputs
+ *   must not alias inputs or each other (not checked; undefined if they do).
+ * Streams.  Each call is asynchronous on `stream` (0 is the legacy default
+ *   stream): it enqueues its kernels and returns.  The library takes a
+ *   stream-ordered workspace from its own per-device memory pool
+ *   (cudaMallocFromPoolAsync) and returns it on the same stream.
+ * Results.  Floating-point outputs are deterministic run to run for a given
+ *   shape on a given GPU (fixed summation order, no atomics).  Integer
+ *   outputs are exact modulo 2^64 in any order.
+ * Errors.  Every call returns a dualmv_status and never prints or aborts.
+ *   DUALMV_ERR_INVALID_VALUE: M < 0, N < 0, batch < 0, lda < max(1, N), a
+ *     NULL pointer whose extent is nonzero, or batch strides that make
+ *     outputs of different problems overlap.  Nothing is enqueued.
+ *   DUALMV_ERR_ALLOC: the workspace could not be allocated.  Nothing ran.
+ *   DUALMV_ERR_LAUNCH: a CUDA call failed; dualmv_last_cuda_error() gives
+ *     the cudaError_t value.
+ *   Empty problems succeed: when N == 0, q is set to zero; when M == 0, s is
+ *   set to zero; when batch == 0 nothing happens.
+ *   Faults that happen on the device after the call returned (a bounded wait
+ *   that timed out) are reported by dualmv_device_fault().
+ * Alignment.  The fast path streams A with the Tensor Memory Accelerator and
+ *   needs A 16-byte aligned and lda * sizeof(element) (and, batched,
+ *   strideA * sizeof(element)) a multiple of 16 bytes.  Other inputs take a
+ *   slower plain-load path with the same results contract; this is not an
+ *   error.
+ */
+#ifndef DUALMV_H
+#define DUALMV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum dualmv_status {
+    DUALMV_SUCCESS = 0,
+    DUALMV_ERR_INVALID_VALUE = 1,
+    DUALMV_ERR_ALLOC = 2,
+    DUALMV_ERR_LAUNCH = 3,
+    DUALMV_ERR_TIMEOUT = 4,
+    DUALMV_ERR_UNSUPPORTED = 5
+} dualmv_status;
+
+/* Opaque CUDA stream handle (the same pointer as cudaStream_t). */
+typedef struct CUstream_st *dualmv_stream_t;
+
+/* ---- single problem ----------------------------------------------------
+ * BICG (Table 1 / Table 2): q = A p and s = A^T r from one read of A.
+ * f32: float inputs, float accumulation and outputs.
+ * f64: double inputs, double accumulation and outputs.
+ * i32: int32 inputs, products and sums in 64 bits with wrap-around modulo
+ *      2^64, int64 outputs (bit-exact in any summation order). */
+dualmv_status dualmv_f32(int64_t M, int64_t N, const float *A, int64_t lda,
+                         const float *p, const float *r, float *q, float *s,
+                         dualmv_stream_t stream);
+dualmv_status dualmv_f64(int64_t M, int64_t N, const double *A, int64_t lda,
+                         const double *p, const double *r, double *q,
+                         double *s, dualmv_stream_t stream);
+dualmv_status dualmv_i32(int64_t M, int64_t N, const int32_t *A, int64_t lda,
+                         const int32_t *p, const int32_t *r, int64_t *q,
+                         int64_t *s, dualmv_stream_t stream);
+
+/* ---- strided batch -----------------------------------------------------
+ * `batch` independent problems of the same shape (BICG, Table 1 / Table 2,
+ * applied to each).  Problem b uses A + b*strideA, p + b*strideP,
+ * r + b*strideR and writes q + b*strideQ, s + b*strideS (strides in
+ * elements).  Input strides may be 0 (the same operand for every problem).
+ * When batch > 1, strideQ >= M and strideS >= N are required so that the
+ * outputs of different problems do not overlap. */
+dualmv_status dualmv_f32_strided_batched(
+    int64_t M, int64_t N, const float *A, int64_t lda, int64_t strideA,
+    const float *p, int64_t strideP, const float *r, int64_t strideR,
+    float *q, int64_t strideQ, float *s, int64_t strideS, int64_t batch,
+    dualmv_stream_t stream);
+dualmv_status dualmv_f64_strided_batched(
+    int64_t M, int64_t N, const double *A, int64_t lda, int64_t strideA,
+    const double *p, int64_t strideP, const double *r, int64_t strideR,
+    double *q, int64_t strideQ, double *s, int64_t strideS, int64_t batch,
+    dualmv_stream_t stream);
+dualmv_status dualmv_i32_strided_batched(
+    int64_t M, int64_t N, const int32_t *A, int64_t lda, int64_t strideA,
+    const int32_t *p, int64_t strideP, const int32_t *r, int64_t strideR,
+    int64_t *q, int64_t strideQ, int64_t *s, int64_t strideS, int64_t batch,
+    dualmv_stream_t stream);
+
+/* ---- diagnostics and control ------------------------------------------ */
+
+/* Static English text for a status code ("unknown status" otherwise). */
+const char *dualmv_status_string(dualmv_status status);
+
+/* cudaError_t value of the most recent CUDA failure seen by this thread
+ * (0 if none).  Reading it does not clear it. */
+int dualmv_last_cuda_error(void);
+
+/* Synchronises `stream`, then reads and clears the current device's fault
+ * word.  Returns DUALMV_ERR_TIMEOUT if any kernel of this library gave up a
+ * bounded wait (a pipeline barrier that never completed) since the last
+ * read, DUALMV_ERR_LAUNCH if the synchronisation itself failed, and
+ * DUALMV_SUCCESS otherwise.  A kernel that gives up writes no output it has
+ * not finished; the outputs of that call are then unspecified. */
+dualmv_status dualmv_device_fault(dualmv_stream_t stream);
+
+/* Which kernel streams A.  DUALMV_PATH_AUTO (default) uses the TMA pipeline
+ * when the alignment rules above hold and the plain-load kernel otherwise;
+ * the other values force one of them (FORCE_TMA falls back to plain loads
+ * when the alignment rules do not hold).  Process-wide; meant for tests and
+ * tuning.  Returns the previous setting, or -1 for an unknown value. */
+enum { DUALMV_PATH_AUTO = 0, DUALMV_PATH_TMA = 1, DUALMV_PATH_DIRECT = 2 };
+int dualmv_set_path(int path);
+
+/* ---- planner (pure host code, no CUDA call) ----------------------------
+ * The work decomposition a call would use.  A is cut into column bands of
+ * `band_cols` columns and row stripes of `tile_rows` rows; a tile is one
+ * stripe of one band of one problem.  Tiles are numbered band-major
+ * (problem, band, stripe) and CTA c of `grid` owns the contiguous range
+ * [floor(c*tiles/grid), floor((c+1)*tiles/grid)).  A band split between
+ * CTAs leaves one column partial per CTA ("segment"); row partials of
+ * different bands are combined by a second kernel in ascending band order,
+ * column partials in ascending CTA order.  `num_sms` is the SM count to plan
+ * for.  Returns DUALMV_ERR_INVALID_VALUE for bad shapes or elem_bytes not
+ * in {4, 8}. */
+typedef struct dualmv_plan_t {
+    int64_t band_cols;      /* columns per band (tile width)              */
+    int64_t tile_rows;      /* rows per tile (stripe height)              */
+    int64_t bands;          /* column bands per problem                   */
+    int64_t stripes;        /* row stripes per problem                    */
+    int64_t tiles;          /* batch * bands * stripes                    */
+    int64_t grid;           /* CTAs launched (persistent)                 */
+    int64_t max_segments;   /* most band segments one CTA can own         */
+    int64_t workspace_bytes;/* stream-ordered scratch the call allocates  */
+    int64_t smem_bytes;     /* dynamic shared memory per CTA              */
+    int64_t threads;        /* threads per CTA                            */
+} dualmv_plan_t;
+
+dualmv_status dualmv_plan(int64_t M, int64_t N, int64_t batch,
+                          int64_t elem_bytes, int64_t acc_bytes,
+                          int64_t num_sms, dualmv_plan_t *out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DUALMV_H */

@@ -1,0 +1,132 @@
+"""Seeded synthetic inputs for the dual matrix-vector product.
+
+This module holds no arithmetic of the method: it only draws random operands
+and names the workloads.  Both the CUDA path (tests, benchmark) and the CPU
+oracle take their inputs from here, so both sides see the same numbers.
+
+Recipe: one ``torch.Generator`` on the target device, seeded with the
+workload's seed, fills A, then p, then r, in that order.  Floats are drawn
+with ``uniform_(-1, 1)`` (half-open [-1, 1)) or ``normal_(0, 1)``; integers
+with ``randint(-8, 9)`` (inclusive [-8, 8]).  Batched workloads draw each
+operand for the whole batch in one call.  Padding columns (``lda > N``) are
+filled with a sentinel the kernels must never read: NaN for floats,
+INT32_MIN for integers.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, replace
+
+import torch
+
+DTYPES = {"f32": torch.float32, "f64": torch.float64, "i32": torch.int32}
+OUT_DTYPES = {"f32": torch.float32, "f64": torch.float64, "i32": torch.int64}
+ELEM_BYTES = {"f32": 4, "f64": 8, "i32": 4}
+OUT_BYTES = {"f32": 4, "f64": 8, "i32": 8}
+
+
+@dataclass(frozen=True)
+class Workload:
+    """One synthetic problem (or strided batch of problems)."""
+
+    name: str
+    dtype: str          # "f32" | "f64" | "i32"
+    M: int
+    N: int
+    lda: int
+    dist: str           # "uniform" | "normal" | "int8"
+    seed: int
+    batch: int = 0      # 0 = single problem; >= 1 = strided batch
+
+    @property
+    def batched(self) -> bool:
+        return self.batch > 0
+
+    @property
+    def nbatch(self) -> int:
+        return max(1, self.batch)
+
+    def bytes_counted(self) -> int:
+        """Bytes of the logical A (padding excluded), of p and r read, and of
+        q and s written: the numerator of the effective-bandwidth metric."""
+        e, o = ELEM_BYTES[self.dtype], OUT_BYTES[self.dtype]
+        per = (self.M * self.N * e + (self.M + self.N) * e
+               + (self.M + self.N) * o)
+        return per * self.nbatch
+
+    def scaled(self, **kw) -> "Workload":
+        return replace(self, **kw)
+
+
+# The five workloads: a small square problem, a 1 GiB square fp32 matrix, a
+# 2 GiB tall-skinny fp64 matrix, a wide int32 matrix with a padded, ragged
+# row, and a strided batch of 256 square fp32 problems (4 GiB).
+WORKLOADS = {
+    w.name: w for w in (
+        Workload("f32_1024x1024", "f32", 1024, 1024, 1024, "uniform", 0),
+        Workload("f32_16384x16384", "f32", 16384, 16384, 16384, "uniform", 1),
+        Workload("f64_65536x4096", "f64", 65536, 4096, 4096, "normal", 2),
+        Workload("i32_4001x100003_lda100008", "i32", 4001, 100003, 100008,
+                 "int8", 3),
+        Workload("f32_batch256_2048x2048", "f32", 2048, 2048, 2048, "uniform",
+                 4, batch=256),
+    )
+}
+
+
+def _sentinel(dtype: str):
+    return float("nan") if dtype != "i32" else -(2 ** 31)
+
+
+def _fill(t: torch.Tensor, dist: str, g: torch.Generator) -> None:
+    if dist == "uniform":
+        t.uniform_(-1.0, 1.0, generator=g)
+    elif dist == "normal":
+        t.normal_(0.0, 1.0, generator=g)
+    elif dist == "int8":
+        t.copy_(torch.randint(-8, 9, t.shape, generator=g, device=t.device,
+                              dtype=t.dtype))
+    else:
+        raise ValueError(f"unknown distribution {dist!r}")
+
+
+def generate(w: Workload, device: str | torch.device = "cpu"):
+    """Return ``(A, p, r)`` on ``device``.
+
+    ``A`` has shape ``(M, lda)`` (or ``(batch, M, lda)``) and holds the
+    matrix in its first N columns and the padding sentinel after them.
+    ``p`` is ``(N,)`` / ``(batch, N)`` and ``r`` is ``(M,)`` /
+    ``(batch, M)``.
+    """
+    dev = torch.device(device)
+    g = torch.Generator(device=dev)
+    g.manual_seed(w.seed)
+    t = DTYPES[w.dtype]
+    lead = (w.batch,) if w.batched else ()
+    A = torch.empty(lead + (w.M, w.lda), dtype=t, device=dev)
+    if w.lda > w.N:
+        A[..., w.N:] = _sentinel(w.dtype)
+    view = A[..., : w.N]
+    if view.numel():
+        if view.is_contiguous():
+            _fill(view, w.dist, g)
+        else:
+            tmp = torch.empty(view.shape, dtype=t, device=dev)
+            _fill(tmp, w.dist, g)
+            view.copy_(tmp)
+            del tmp
+    p = torch.empty(lead + (w.N,), dtype=t, device=dev)
+    r = torch.empty(lead + (w.M,), dtype=t, device=dev)
+    if p.numel():
+        _fill(p, w.dist, g)
+    if r.numel():
+        _fill(r, w.dist, g)
+    return A, p, r
+
+
+def empty_outputs(w: Workload, device: str | torch.device = "cpu"):
+    """Output buffers ``(q, s)`` of the right dtype and shape."""
+    t = OUT_DTYPES[w.dtype]
+    lead = (w.batch,) if w.batched else ()
+    q = torch.empty(lead + (w.M,), dtype=t, device=device)
+    s = torch.empty(lead + (w.N,), dtype=t, device=device)
+    return q, s

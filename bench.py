@@ -1,0 +1,434 @@
+#!/usr/bin/env python3
+"""Benchmark of the fused dual matrix-vector product (BICG: q = A p, s = A^T r).
+
+One step = one dualmv call over the whole workload (default: the 16384 x
+16384 fp32 matrix, 1 GiB, seeded uniform[-1, 1)).  Prints ONE JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   (the CPU oracle, timed on the host)
+
+Metric: effective bandwidth = (bytes of the logical A, of p and r read and of
+q and s written) / device time, in GB/s (1e9 B/s).  The inputs (1 GiB) are
+larger than L2 (129 MB), so consecutive steps cannot hit in L2.  Device time
+comes from CUDA events on the launching stream, bracketed by a barrier and a
+device synchronisation; with several ranks the slowest rank's time counts.
+Per-step times are also summarised with the trimmed mean of Eq. 3
+(R timings sorted, k lowest and k highest dropped).
+
+Multi-GPU: each rank runs its own copy of the workload on its own GPU (the
+problems are independent; no data-path collective) and ``value`` counts the
+bytes of all ranks: weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "dualmv effective HBM GB/s (bytes of A+vectors / device time) and % of GB300 peak"
+DEFAULT_WORKLOAD = "f32_16384x16384"
+FALLBACK_HBM_GBS = 6800.0
+KERNEL_SOURCES = ("paper_2512_22147_gb300/csrc/dualmv_kernels.cuh",
+                  "paper_2512_22147_gb300/csrc/dualmv.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+
+
+# ------------------------------------------------------------- helpers ----
+
+def trimmed_mean(times, k: int) -> float:
+    """Eq. 3: sort the R timings, drop the k lowest and k highest, average."""
+    t = sorted(times)
+    if k < 0 or len(t) <= 2 * k:
+        raise ValueError("trimmed mean needs R > 2k")
+    mid = t[k:len(t) - k]
+    return sum(mid) / len(mid)
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def measured_peak():
+    """(GB/s, source) from the generated MEASURED_PEAKS.json, else the
+    fallback figure."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            v = float(json.load(f)["hbm_gbs"])
+        return v, "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch of the streaming kernel from a committed ncu
+    capture, if it was taken on the current kernel source; else None."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    ent = rec.get(workload)
+    if not ent or ent.get("kernel_source_hash") != kernel_source_hash():
+        return None
+    return ent.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clock and throttle-reason samples while the timed region runs."""
+
+    QUERY = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        import tempfile
+        fd, self.path = tempfile.mkstemp(prefix="dualmv_clocks_", suffix=".csv")
+        os.close(fd)
+        cmd = ["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+               "-lms", "100"]
+        if self.uuid:
+            cmd += ["-i", self.uuid]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=open(self.path, "w"),
+                                         stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"],
+                    "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 10:
+                    rows.append(parts)
+        os.unlink(self.path)
+        sm = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        mx = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[6:10]) if v == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def gpu_uuid(torch, dev):
+    try:
+        u = str(torch.cuda.get_device_properties(dev).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:  # noqa: BLE001 - older torch: sample the default GPU
+        return None
+
+
+# ---------------------------------------------------------- distributed ---
+
+def dist_setup(torch, backend):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def max_over_ranks(torch, value: float, world: int, device) -> float:
+    if world == 1:
+        return value
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# --------------------------------------------------------------- native ---
+
+def run_native(args):
+    import torch
+
+    world, rank, local = dist_setup(torch, "nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    import paper_2512_22147_gb300 as dm
+    from paper_2512_22147_gb300 import inputs
+
+    w = inputs.WORKLOADS[args.workload]
+    A, p, r = inputs.generate(w, dev)
+    Av = A[..., : w.N]
+    q, s = inputs.empty_outputs(w, dev)
+    stream = torch.cuda.current_stream(dev)
+    nbytes = w.bytes_counted()
+
+    for _ in range(args.warmup):
+        dm.dualmv(Av, p, r, q=q, s=s)
+    torch.cuda.synchronize(dev)
+    if dm.device_fault() != dm.DUALMV_SUCCESS:
+        raise RuntimeError("device fault during warm-up")
+
+    K = args.steps
+    call_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(K)]
+    kern_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(K)]
+    region = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+
+    sampler = ClockSampler(gpu_uuid(torch, dev))
+    sampler.start()
+    time.sleep(0.3)  # let the sampler start before the timed region
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    region[0].record(stream)
+    for i in range(K):
+        ks, ke = kern_ev[i]
+        dm.dualmv_record_kernel_events(ks.cuda_event, ke.cuda_event)
+        call_ev[i][0].record(stream)
+        dm.dualmv(Av, p, r, q=q, s=s)
+        call_ev[i][1].record(stream)
+    region[1].record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clocks = sampler.stop()
+    fault = dm.device_fault()
+    if fault != dm.DUALMV_SUCCESS:
+        raise RuntimeError("device fault during the timed region")
+
+    region_ms = region[0].elapsed_time(region[1])
+    region_ms = max_over_ranks(torch, region_ms, world, dev)
+    step_ms = [a.elapsed_time(b) for a, b in call_ev]
+    kern_ms = [a.elapsed_time(b) for a, b in kern_ev]
+    ms_per_step = region_ms / K
+    value = world * nbytes * K / (region_ms * 1e-3) / 1e9
+
+    peak, peak_src = measured_peak()
+    kern_avg_ms = sum(kern_ms) / len(kern_ms)
+    achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9
+    traffic = recorded_traffic(args.workload)
+
+    # End to end through the same public call with host buffers: pinned host
+    # inputs copied in, the call, results copied out, every step.
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(torch, dm, w, A, p, r, dev, stream, args.e2e_steps)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, A, p, r, args.cpu_seconds)
+
+    out = {
+        "metric": METRIC,
+        "value": round(value, 2),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": w.dtype,
+        "data": "synthetic",
+        "config": {
+            "workload": w.name, "M": w.M, "N": w.N, "lda": w.lda,
+            "batch": w.batch, "dtype": w.dtype, "distribution": w.dist, "seed": w.seed,
+            "bytes_per_step": nbytes,
+            "l2": "inputs larger than L2 (no flush needed)",
+            "parallelism": f"replicas x{world}",
+        },
+        "pct_of_peak": round(100.0 * value / (world * peak), 2),
+        "trimmed_mean_ms": round(trimmed_mean(step_ms, 3) if K > 6 else ms_per_step, 5),
+        "median_step_ms": round(statistics.median(step_ms), 5),
+        "roofline": {
+            "bound": "hbm",
+            "kernel": "dualmv_stream_kernel",
+            "achieved": round(achieved, 2),
+            "peak": peak,
+            "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
+            else "fallback 6.8 TB/s",
+            "unit": "GB/s",
+            "frac": round(achieved / peak, 4),
+            "traffic": traffic,
+            "algorithmic_bytes_per_launch": nbytes,
+            "kernel_avg_ms": round(kern_avg_ms, 5),
+        },
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": 2 * K,
+        "clocks": clocks,
+    }
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_e2e(torch, dm, w, A, p, r, dev, stream, steps):
+    Ah = A.cpu().pin_memory()
+    ph = p.cpu().pin_memory()
+    rh = r.cpu().pin_memory()
+    Ad = torch.empty_like(A)
+    pd = torch.empty_like(p)
+    rd = torch.empty_like(r)
+    q, s = dm.dualmv(Ad[..., : w.N].copy_(A[..., : w.N]), pd.copy_(p), rd.copy_(r))
+    qh = torch.empty(q.shape, dtype=q.dtype).pin_memory()
+    sh = torch.empty(s.shape, dtype=s.dtype).pin_memory()
+    torch.cuda.synchronize(dev)
+    start = torch.cuda.Event(enable_timing=True)
+    stop = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for _ in range(steps):
+        Ad.copy_(Ah, non_blocking=True)
+        pd.copy_(ph, non_blocking=True)
+        rd.copy_(rh, non_blocking=True)
+        dm.dualmv(Ad[..., : w.N], pd, rd, q=q, s=s)
+        qh.copy_(q, non_blocking=True)
+        sh.copy_(s, non_blocking=True)
+    stop.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = start.elapsed_time(stop) / steps
+    h2d = Ah.numel() * Ah.element_size() + ph.numel() * ph.element_size() \
+        + rh.numel() * rh.element_size()
+    d2h = qh.numel() * qh.element_size() + sh.numel() * sh.element_size()
+    return {"value": round(w.bytes_counted() / (ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+            "ms_per_step": round(ms, 4), "steps": steps,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "how": "pinned host A, p, r copied to the GPU, dualmv through the C ABI, q and s "
+                   "copied back, all on one stream inside CUDA events"}
+
+
+# ------------------------------------------------------- CPU (oracle) ----
+
+def oracle_sample(w, A_np, p_np, r_np, budget_s: float):
+    """Times the oracle on leading rows of the workload (of each problem,
+    batched: leading problems), growing the sample until it takes about
+    ``budget_s`` seconds or covers the whole workload.  Returns
+    (bytes per second, seconds, description)."""
+    import oracle
+    from paper_2512_22147_gb300 import inputs
+
+    e, o = inputs.ELEM_BYTES[w.dtype], inputs.OUT_BYTES[w.dtype]
+    if w.batched:
+        units, per_unit = w.batch, None
+    else:
+        units, per_unit = w.M, None
+    n = max(1, min(units, 64))
+    while True:
+        t0 = time.perf_counter()
+        if w.batched:
+            oracle.dualmv_batched(A_np[:n], p_np[:n], r_np[:n], N=w.N)
+            nbytes = n * (w.M * w.N * e + (w.M + w.N) * (e + o))
+        else:
+            oracle.dualmv(A_np[:n], p_np, r_np[:n], N=w.N)
+            nbytes = n * w.N * e + (n + w.N) * (e + o)
+        dt = time.perf_counter() - t0
+        if dt >= budget_s or n >= units:
+            break
+        grow = max(2.0, min(8.0, budget_s / max(dt, 1e-3)))
+        n = min(units, int(math.ceil(n * grow)))
+    what = (f"first {n} of {units} {'problems' if w.batched else 'rows'} of {w.name}, "
+            f"single-threaded C oracle (double/Dot2/int64 sums)")
+    return nbytes / dt / 1e9, dt, what
+
+
+def cpu_baseline(w, A, p, r, budget_s):
+    A_np = A.cpu().numpy()
+    p_np, r_np = p.cpu().numpy(), r.cpu().numpy()
+    gbs, dt, what = oracle_sample(w, A_np, p_np, r_np, budget_s)
+    return {"value": round(gbs, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": what, "seconds": round(dt, 3), "host_cpus": os.cpu_count()}
+
+
+def run_reference(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import torch
+
+    from paper_2512_22147_gb300 import inputs
+    w = inputs.WORKLOADS[args.workload]
+    A, p, r = inputs.generate(w, "cpu")
+    A_np, p_np, r_np = A.numpy(), p.numpy(), r.numpy()
+    budget = args.cpu_seconds / max(1, args.steps + args.warmup)
+    vals, secs = [], []
+    what = ""
+    for i in range(args.warmup + args.steps):
+        gbs, dt, what = oracle_sample(w, A_np, p_np, r_np, budget)
+        if i >= args.warmup:
+            vals.append(gbs)
+            secs.append(dt)
+    value = statistics.mean(vals)
+    del torch
+    out = {
+        "impl": "reference",
+        "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(1e3 * statistics.mean(secs), 4), "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+        "config": {"workload": w.name, "M": w.M, "N": w.N, "lda": w.lda, "batch": w.batch,
+                   "dtype": w.dtype, "distribution": w.dist, "seed": w.seed},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1,
+                         "kind": "oracle", "sample": what},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--impl", choices=["native", "reference"], default="native")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_native(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -127,6 +127,14 @@ dualmv_status dualmv_device_fault(dualmv_stream_t stream);
 enum { DUALMV_PATH_AUTO = 0, DUALMV_PATH_TMA = 1, DUALMV_PATH_DIRECT = 2 };
 int dualmv_set_path(int path);
 
+/* Instrumentation for benchmarks: the next dualmv call made by this thread
+ * records `start` (a cudaEvent_t) on its stream just before it launches its
+ * streaming kernel and `stop` just after, so that the streaming kernel can be
+ * timed on the stream it runs on.  The events are used once and forgotten;
+ * pass NULL, NULL to cancel.  Calls that launch no streaming kernel (empty
+ * problems, invalid arguments) leave the request pending. */
+void dualmv_record_kernel_events(void *start, void *stop);
+
 /* ---- planner (pure host code, no CUDA call) ----------------------------
  * The work decomposition a call would use.  A is cut into column bands of
  * `band_cols` columns and row stripes of `tile_rows` rows; a tile is one

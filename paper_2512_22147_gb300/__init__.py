@@ -1,0 +1,37 @@
+"""GB300-native fused dual matrix-vector product (BICG: q = A p, s = A^T r).
+
+The computation is the BICG kernel that the paper tunes (Table 1 and
+Table 2).  It runs in hand-written CUDA for sm_103a behind the C ABI of
+``include/dualmv.h``; this package holds the in-tree build script, the
+ctypes binding (``_binding``), a tensor-level wrapper (``api.dualmv``) and
+the seeded workload generator (``inputs``).
+
+The CUDA library is loaded on first use of any binding name (for example
+``paper_2512_22147_gb300.dualmv``); if ``libdualmv.so`` has not been built
+that first use raises ImportError.  There is no CPU fallback.
+"""
+import importlib
+
+_BINDING_NAMES = {
+    "DUALMV_ERR_ALLOC", "DUALMV_ERR_INVALID_VALUE", "DUALMV_ERR_LAUNCH",
+    "DUALMV_ERR_TIMEOUT", "DUALMV_ERR_UNSUPPORTED", "DUALMV_PATH_AUTO",
+    "DUALMV_PATH_DIRECT", "DUALMV_PATH_TMA", "DUALMV_SUCCESS", "EXPORTED",
+    "LIBRARY_PATH", "DualmvError", "Plan", "dualmv_device_fault", "dualmv_f32",
+    "dualmv_f32_strided_batched", "dualmv_f64", "dualmv_f64_strided_batched",
+    "dualmv_i32", "dualmv_i32_strided_batched", "dualmv_last_cuda_error",
+    "dualmv_plan", "dualmv_record_kernel_events", "dualmv_set_path",
+    "dualmv_status_string", "library",
+}
+_API_NAMES = {"dualmv", "device_fault"}
+
+
+def __getattr__(name):
+    if name in _BINDING_NAMES:
+        return getattr(importlib.import_module("._binding", __name__), name)
+    if name in _API_NAMES:
+        return getattr(importlib.import_module(".api", __name__), name)
+    raise AttributeError(f"module {__name__!r} has no attribute {name!r}")
+
+
+def __dir__():
+    return sorted(set(globals()) | _BINDING_NAMES | _API_NAMES)

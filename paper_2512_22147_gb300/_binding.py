@@ -1,0 +1,157 @@
+"""ctypes binding of the C ABI in ``include/dualmv.h``.
+
+Argument marshalling only: every step of the computation runs in the CUDA
+library.  There is no fallback: if ``libdualmv.so`` has not been built, the
+import fails with an error that says how to build it.
+
+Two layers:
+  * the raw entry points under their C names (``dualmv_f32``,
+    ``dualmv_f32_strided_batched``, ...), taking integers and raw pointers
+    exactly like the C functions;
+  * ``dualmv(A, p, r)``, which takes CUDA torch tensors, derives the sizes,
+    leading dimension and strides from them, picks the entry point by dtype
+    and runs on the current torch stream.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+from . import build as _build
+
+DUALMV_SUCCESS = 0
+DUALMV_ERR_INVALID_VALUE = 1
+DUALMV_ERR_ALLOC = 2
+DUALMV_ERR_LAUNCH = 3
+DUALMV_ERR_TIMEOUT = 4
+DUALMV_ERR_UNSUPPORTED = 5
+
+DUALMV_PATH_AUTO = 0
+DUALMV_PATH_TMA = 1
+DUALMV_PATH_DIRECT = 2
+
+EXPORTED = (
+    "dualmv_f32", "dualmv_f64", "dualmv_i32",
+    "dualmv_f32_strided_batched", "dualmv_f64_strided_batched",
+    "dualmv_i32_strided_batched",
+    "dualmv_status_string", "dualmv_last_cuda_error", "dualmv_device_fault",
+    "dualmv_set_path", "dualmv_plan", "dualmv_record_kernel_events",
+)
+
+
+class DualmvError(RuntimeError):
+    """A dualmv entry point returned a status other than success."""
+
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {status_string(status)} (status {status}, "
+                         f"cuda error {_lib.dualmv_last_cuda_error()})")
+
+
+class Plan(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int64) for n in (
+        "band_cols", "tile_rows", "bands", "stripes", "tiles", "grid",
+        "max_segments", "workspace_bytes", "smem_bytes", "threads")]
+
+
+def _load() -> ctypes.CDLL:
+    path = _build.LIB_PATH
+    if not os.path.exists(path):
+        raise ImportError(
+            f"{path} is missing: build it with `python -m "
+            "paper_2512_22147_gb300.build` (nvcc for sm_103a); there is no "
+            "CPU fallback")
+    lib = ctypes.CDLL(path)
+    i64, vp, st = ctypes.c_int64, ctypes.c_void_p, ctypes.c_int
+    single = [i64, i64, vp, i64, vp, vp, vp, vp, vp]
+    batched = [i64, i64, vp, i64, i64, vp, i64, vp, i64, vp, i64, vp, i64, i64, vp]
+    for t in ("f32", "f64", "i32"):
+        f = getattr(lib, f"dualmv_{t}")
+        f.argtypes, f.restype = single, st
+        f = getattr(lib, f"dualmv_{t}_strided_batched")
+        f.argtypes, f.restype = batched, st
+    lib.dualmv_status_string.argtypes = [st]
+    lib.dualmv_status_string.restype = ctypes.c_char_p
+    lib.dualmv_last_cuda_error.argtypes = []
+    lib.dualmv_last_cuda_error.restype = st
+    lib.dualmv_device_fault.argtypes = [vp]
+    lib.dualmv_device_fault.restype = st
+    lib.dualmv_set_path.argtypes = [st]
+    lib.dualmv_set_path.restype = st
+    lib.dualmv_record_kernel_events.argtypes = [vp, vp]
+    lib.dualmv_record_kernel_events.restype = None
+    lib.dualmv_plan.argtypes = [i64, i64, i64, i64, i64, i64, ctypes.POINTER(Plan)]
+    lib.dualmv_plan.restype = st
+    return lib
+
+
+_lib = _load()
+LIBRARY_PATH = _build.LIB_PATH
+
+
+def library() -> ctypes.CDLL:
+    return _lib
+
+
+# --------------------------------------------------- raw C entry points ----
+
+def dualmv_f32(M, N, A, lda, p, r, q, s, stream):
+    return _lib.dualmv_f32(M, N, A, lda, p, r, q, s, stream)
+
+
+def dualmv_f64(M, N, A, lda, p, r, q, s, stream):
+    return _lib.dualmv_f64(M, N, A, lda, p, r, q, s, stream)
+
+
+def dualmv_i32(M, N, A, lda, p, r, q, s, stream):
+    return _lib.dualmv_i32(M, N, A, lda, p, r, q, s, stream)
+
+
+def dualmv_f32_strided_batched(M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS, batch, stream):
+    return _lib.dualmv_f32_strided_batched(M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS,
+                                           batch, stream)
+
+
+def dualmv_f64_strided_batched(M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS, batch, stream):
+    return _lib.dualmv_f64_strided_batched(M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS,
+                                           batch, stream)
+
+
+def dualmv_i32_strided_batched(M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS, batch, stream):
+    return _lib.dualmv_i32_strided_batched(M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS,
+                                           batch, stream)
+
+
+def dualmv_status_string(status: int) -> str:
+    return _lib.dualmv_status_string(status).decode()
+
+
+status_string = dualmv_status_string
+
+
+def dualmv_last_cuda_error() -> int:
+    return _lib.dualmv_last_cuda_error()
+
+
+def dualmv_device_fault(stream=None) -> int:
+    return _lib.dualmv_device_fault(stream)
+
+
+def dualmv_set_path(path: int) -> int:
+    old = _lib.dualmv_set_path(path)
+    if old < 0:
+        raise ValueError(f"unknown path {path}")
+    return old
+
+
+def dualmv_record_kernel_events(start, stop) -> None:
+    """Raw cudaEvent_t handles (ints) or None; see include/dualmv.h."""
+    _lib.dualmv_record_kernel_events(start, stop)
+
+
+def dualmv_plan(M, N, batch, elem_bytes, acc_bytes, num_sms) -> Plan:
+    out = Plan()
+    rc = _lib.dualmv_plan(M, N, batch, elem_bytes, acc_bytes, num_sms, ctypes.byref(out))
+    if rc != DUALMV_SUCCESS:
+        raise DualmvError(rc, "dualmv_plan")
+    return out

@@ -1,0 +1,105 @@
+"""Tensor-level entry point: ``dualmv(A, p, r)`` on CUDA torch tensors.
+
+PyTorch only provides device memory and the current stream; the work runs
+in the CUDA library through the C ABI (``_binding``).
+
+Shapes (BICG, Tables 1-2 of the paper: q = A p, s = A^T r):
+  single:  A (M, N) with A.stride(1) == 1 and leading dimension A.stride(0);
+           p (N,), r (M,)  ->  q (M,), s (N,)
+  batched: A (B, M, N) with A.stride(2) == 1; lda = A.stride(1),
+           strideA = A.stride(0); p (B, N) or (N,) (shared), r (B, M) or
+           (M,) (shared)  ->  q (B, M), s (B, N)
+dtype float32 -> float32 outputs, float64 -> float64, int32 -> int64
+(exact modulo 2^64).  A may be a column slice of a wider buffer (its row
+stride is the leading dimension).
+"""
+from __future__ import annotations
+
+import torch
+
+from . import _binding as B
+
+_OUT = {torch.float32: torch.float32, torch.float64: torch.float64,
+        torch.int32: torch.int64}
+_TAG = {torch.float32: "f32", torch.float64: "f64", torch.int32: "i32"}
+
+
+def _vec_stride(v: torch.Tensor, length: int, batch: int, name: str) -> int:
+    """Element stride between problems for a per-problem vector (0 = shared)."""
+    if v.dim() == 1:
+        if v.shape[0] != length or (length > 1 and v.stride(0) != 1):
+            raise ValueError(f"{name} must be a contiguous vector of length {length}")
+        return 0
+    if v.dim() != 2 or v.shape[0] != batch or v.shape[1] != length:
+        raise ValueError(f"{name} must have shape ({batch}, {length})")
+    if length > 1 and v.stride(1) != 1:
+        raise ValueError(f"{name} rows must be contiguous")
+    return v.stride(0)
+
+
+def dualmv(A: torch.Tensor, p: torch.Tensor, r: torch.Tensor,
+           q: torch.Tensor | None = None, s: torch.Tensor | None = None,
+           stream: torch.cuda.Stream | None = None):
+    """Compute ``q = A p`` and ``s = A^T r`` (per problem when batched).
+
+    Returns ``(q, s)``; pass ``q``/``s`` to write into existing buffers.
+    Runs asynchronously on ``stream`` (default: the current stream).
+    """
+    if A.dtype not in _TAG:
+        raise TypeError(f"unsupported dtype {A.dtype}; use float32, float64 or int32")
+    if not A.is_cuda:
+        raise ValueError("A must be a CUDA tensor (the library has no CPU path)")
+    for t, n in ((p, "p"), (r, "r")):
+        if t.dtype != A.dtype or t.device != A.device:
+            raise ValueError(f"{n} must match A's dtype and device")
+    batched = A.dim() == 3
+    if A.dim() not in (2, 3):
+        raise ValueError("A must be 2-D (M, N) or 3-D (B, M, N)")
+    Bn = A.shape[0] if batched else 1
+    M, N = A.shape[-2], A.shape[-1]
+    if N > 1 and A.stride(-1) != 1:
+        raise ValueError("A's last dimension must be contiguous")
+    if M > 1 and A.stride(-2) < N:
+        raise ValueError("A's rows overlap (row stride smaller than N)")
+    lda = max(A.stride(-2), N, 1) if M > 1 else max(N, 1)
+    strideA = A.stride(0) if batched else 0
+    out_t = _OUT[A.dtype]
+    shape_q = (Bn, M) if batched else (M,)
+    shape_s = (Bn, N) if batched else (N,)
+    if q is None:
+        q = torch.empty(shape_q, dtype=out_t, device=A.device)
+    if s is None:
+        s = torch.empty(shape_s, dtype=out_t, device=A.device)
+    if q.dtype != out_t or s.dtype != out_t:
+        raise ValueError(f"outputs must be {out_t}")
+    if tuple(q.shape) != shape_q or tuple(s.shape) != shape_s:
+        raise ValueError("output shapes do not match")
+    strm = stream if stream is not None else torch.cuda.current_stream(A.device)
+    h = strm.cuda_stream
+    tag = _TAG[A.dtype]
+    with torch.cuda.device(A.device):
+        if batched:
+            sP = _vec_stride(p, N, Bn, "p")
+            sR = _vec_stride(r, M, Bn, "r")
+            sQ = _vec_stride(q, M, Bn, "q") if q.dim() == 2 else M
+            sS = _vec_stride(s, N, Bn, "s") if s.dim() == 2 else N
+            fn = getattr(B, f"dualmv_{tag}_strided_batched")
+            rc = fn(M, N, A.data_ptr(), lda, strideA, p.data_ptr(), sP, r.data_ptr(), sR,
+                    q.data_ptr(), sQ, s.data_ptr(), sS, Bn, h)
+        else:
+            _vec_stride(p, N, 1, "p")
+            _vec_stride(r, M, 1, "r")
+            if not (q.is_contiguous() and s.is_contiguous()):
+                raise ValueError("q and s must be contiguous")
+            fn = getattr(B, f"dualmv_{tag}")
+            rc = fn(M, N, A.data_ptr(), lda, p.data_ptr(), r.data_ptr(), q.data_ptr(),
+                    s.data_ptr(), h)
+    if rc != B.DUALMV_SUCCESS:
+        raise B.DualmvError(rc, f"dualmv_{tag}")
+    return q, s
+
+
+def device_fault(stream: torch.cuda.Stream | None = None) -> int:
+    """Synchronise ``stream`` and return (and clear) the device fault status."""
+    strm = stream if stream is not None else torch.cuda.current_stream()
+    return B.dualmv_device_fault(strm.cuda_stream)

@@ -1,0 +1,425 @@
+// Host side of the dualmv library: argument checks, the work planner, TMA
+// descriptors, the stream-ordered workspace and the C ABI declared in
+// include/dualmv.h.  The operation is the BICG kernel of the paper (Table 1
+// and Table 2): q = A p and s = A^T r from a single pass over A.
+#include "dualmv.h"
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "dualmv_kernels.cuh"
+
+namespace {
+
+using dmv::kBandCols;
+using dmv::Params;
+
+// Tile shape per element width: W consumer warps x RPW rows per warp, and
+// the ring depth.  Every tile is 32 KiB of A.
+constexpr int kWarps = 8;
+constexpr int kRpw4 = 4;   // 4-byte elements: 32 rows x 1 KiB
+constexpr int kRpw8 = 2;   // 8-byte elements: 16 rows x 2 KiB
+constexpr int kStages = 6;
+constexpr int kDirectCtasPerSm = 4;
+
+thread_local int g_last_cuda_error = 0;
+thread_local cudaEvent_t g_kernel_ev_start = nullptr;
+thread_local cudaEvent_t g_kernel_ev_stop = nullptr;
+int g_path = DUALMV_PATH_AUTO;
+
+dualmv_status cuda_fail(cudaError_t e) {
+    g_last_cuda_error = static_cast<int>(e);
+    return DUALMV_ERR_LAUNCH;
+}
+
+// ------------------------------------------------------- per-device state --
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceState {
+    std::once_flag once;
+    cudaError_t init_error = cudaSuccess;
+    int sms = 0;
+    cudaMemPool_t pool = nullptr;
+};
+DeviceState g_dev[kMaxDevices];
+
+cudaError_t device_state(int dev, DeviceState **out) {
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    DeviceState &st = g_dev[dev];
+    std::call_once(st.once, [&]() {
+        cudaError_t e = cudaDeviceGetAttribute(&st.sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) { st.init_error = e; return; }
+        cudaMemPoolProps props;
+        std::memset(&props, 0, sizeof props);
+        props.allocType = cudaMemAllocationTypePinned;
+        props.handleTypes = cudaMemHandleTypeNone;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = dev;
+        e = cudaMemPoolCreate(&st.pool, &props);
+        if (e != cudaSuccess) { st.init_error = e; return; }
+        // Keep freed workspace cached in the pool between calls.
+        uint64_t keep = UINT64_MAX;
+        e = cudaMemPoolSetAttribute(st.pool, cudaMemPoolAttrReleaseThreshold, &keep);
+        if (e != cudaSuccess) { st.init_error = e; return; }
+    });
+    *out = &st;
+    return st.init_error;
+}
+
+// ------------------------------------------------------------ TMA encode --
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t,
+                                   void *, const cuuint64_t *, const cuuint64_t *,
+                                   const cuuint32_t *, const cuuint32_t *,
+                                   CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = []() -> EncodeTiledFn {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return nullptr;
+        return reinterpret_cast<EncodeTiledFn>(p);
+    }();
+    return fn;
+}
+
+template <typename T> CUtensorMapDataType tma_dtype();
+template <> CUtensorMapDataType tma_dtype<float>() { return CU_TENSOR_MAP_DATA_TYPE_FLOAT32; }
+template <> CUtensorMapDataType tma_dtype<double>() { return CU_TENSOR_MAP_DATA_TYPE_FLOAT64; }
+template <> CUtensorMapDataType tma_dtype<int32_t>() { return CU_TENSOR_MAP_DATA_TYPE_INT32; }
+
+// Encodes A as a 2-D (N, M) or 3-D (N, M, batch) tiled tensor with a box of
+// kBandCols x tile_rows (x 1).  Columns >= N and rows >= M read as zero.
+template <typename T>
+bool encode_a(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
+              int64_t strideA, int64_t batch, int tile_rows, bool three_d) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const int64_t es = sizeof(T);
+    cuuint64_t dims[3] = {(cuuint64_t)N, (cuuint64_t)M, (cuuint64_t)batch};
+    cuuint64_t strides[2] = {(cuuint64_t)(lda * es), (cuuint64_t)(strideA * es)};
+    cuuint32_t box[3] = {(cuuint32_t)kBandCols, (cuuint32_t)tile_rows, 1u};
+    cuuint32_t estr[3] = {1u, 1u, 1u};
+    CUresult rc = fn(map, tma_dtype<T>(), three_d ? 3u : 2u, const_cast<T *>(A), dims,
+                     strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return rc == CUDA_SUCCESS;
+}
+
+// ------------------------------------------------------------------ plan --
+
+dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
+                        int64_t acc_bytes, int64_t ctas, bool tma, dualmv_plan_t *pl) {
+    if (M <= 0 || N <= 0 || batch <= 0 || ctas <= 0 || pl == nullptr)
+        return DUALMV_ERR_INVALID_VALUE;
+    if ((elem_bytes != 4 && elem_bytes != 8) || (acc_bytes != 4 && acc_bytes != 8) ||
+        acc_bytes < elem_bytes)
+        return DUALMV_ERR_INVALID_VALUE;
+    const int64_t rpw = elem_bytes == 4 ? kRpw4 : kRpw8;
+    const int64_t bm = kWarps * rpw;
+    dualmv_plan_t p;
+    std::memset(&p, 0, sizeof p);
+    p.band_cols = kBandCols;
+    p.tile_rows = bm;
+    p.bands = (N + kBandCols - 1) / kBandCols;
+    p.stripes = (M + bm - 1) / bm;
+    if (p.bands > INT64_MAX / p.stripes / batch) return DUALMV_ERR_INVALID_VALUE;
+    p.tiles = batch * p.bands * p.stripes;
+    p.grid = p.tiles < ctas ? p.tiles : ctas;
+    // Most segments (bands touched) of any CTA.
+    int64_t most = 0;
+    for (int64_t c = 0; c < p.grid; ++c) {
+        const int64_t t0 = dmv::cta_first_tile(c, p.tiles, p.grid);
+        const int64_t t1 = dmv::cta_first_tile(c + 1, p.tiles, p.grid);
+        const int64_t nseg = (t1 - 1) / p.stripes - t0 / p.stripes + 1;
+        if (nseg > most) most = nseg;
+    }
+    p.max_segments = most;
+    const int64_t q_ws = p.bands > 1 ? batch * p.bands * M * acc_bytes : 0;
+    const int64_t s_ws = p.grid * p.max_segments * kBandCols * acc_bytes;
+    p.workspace_bytes = ((q_ws + 255) / 256) * 256 + s_ws;
+    const int64_t tile_bytes = bm * kBandCols * elem_bytes;
+    const int64_t scratch = kWarps * kBandCols * acc_bytes;
+    p.smem_bytes = tma ? 1024 + kStages * tile_bytes + scratch + 2 * kStages * 8 : scratch;
+    p.threads = (kWarps + (tma ? 1 : 0)) * 32;
+    *pl = p;
+    return DUALMV_SUCCESS;
+}
+
+// ------------------------------------------------------------ validation --
+
+dualmv_status validate(int64_t M, int64_t N, const void *A, int64_t lda, int64_t strideA,
+                       const void *p, int64_t strideP, const void *r, int64_t strideR,
+                       const void *q, int64_t strideQ, const void *s, int64_t strideS,
+                       int64_t batch) {
+    if (M < 0 || N < 0 || batch < 0) return DUALMV_ERR_INVALID_VALUE;
+    if (lda < (N > 1 ? N : 1)) return DUALMV_ERR_INVALID_VALUE;
+    if (strideA < 0 || strideP < 0 || strideR < 0 || strideQ < 0 || strideS < 0)
+        return DUALMV_ERR_INVALID_VALUE;
+    if (batch == 0) return DUALMV_SUCCESS;
+    if (M > 0 && N > 0 && (A == nullptr || p == nullptr || r == nullptr))
+        return DUALMV_ERR_INVALID_VALUE;
+    if (M > 0 && q == nullptr) return DUALMV_ERR_INVALID_VALUE;
+    if (N > 0 && s == nullptr) return DUALMV_ERR_INVALID_VALUE;
+    if (batch > 1 && (strideQ < M || strideS < N)) return DUALMV_ERR_INVALID_VALUE;
+    // Index arithmetic stays in int64: the last element of A must be addressable.
+    if (M > 0 && N > 0) {
+        const int64_t lim = INT64_MAX / 4;
+        if (M > lim / lda) return DUALMV_ERR_INVALID_VALUE;
+        if (batch > 1 && strideA > 0 && batch - 1 > (lim - M * lda) / strideA)
+            return DUALMV_ERR_INVALID_VALUE;
+    }
+    return DUALMV_SUCCESS;
+}
+
+bool fault_injected_alloc() {
+    const char *v = std::getenv("DUALMV_FAULT_INJECT");
+    return v != nullptr && std::strcmp(v, "alloc") == 0;
+}
+
+// ------------------------------------------------------------- launching --
+
+template <typename T, bool kTma, bool k3d>
+cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
+                          cudaStream_t stream) {
+    constexpr int rpw = sizeof(T) == 4 ? kRpw4 : kRpw8;
+    auto kern = dmv::dualmv_stream_kernel<T, kWarps, rpw, kStages, kTma, k3d>;
+    // Setting the attribute is idempotent and cheap; doing it per call keeps
+    // it correct on every device without extra bookkeeping.
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)pl.smem_bytes);
+    if (e != cudaSuccess) return e;
+    kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(map, prm);
+    return cudaGetLastError();
+}
+
+template <typename Acc>
+cudaError_t launch_combine(const Params &prm, int sms, cudaStream_t stream) {
+    const int64_t total = (prm.bands > 1 ? prm.batch * prm.M : 0) + prm.batch * prm.N;
+    int64_t blocks = (total + 255) / 256;
+    const int64_t cap = (int64_t)sms * 8;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    cudaLaunchConfig_t cfg;
+    std::memset(&cfg, 0, sizeof cfg);
+    cfg.gridDim = dim3((unsigned)blocks);
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, dmv::dualmv_combine_kernel<Acc>, prm);
+}
+
+template <typename Acc>
+cudaError_t zero_fill(Acc *out, int64_t len, int64_t stride, int64_t batch,
+                      cudaStream_t stream) {
+    if (len <= 0 || batch <= 0) return cudaSuccess;
+    const int64_t total = len * batch;
+    int64_t blocks = (total + 255) / 256;
+    if (blocks > 4096) blocks = 4096;
+    dmv::dualmv_zero_kernel<Acc><<<(unsigned)blocks, 256, 0, stream>>>(out, len, stride, batch);
+    return cudaGetLastError();
+}
+
+template <typename T, typename Out>
+dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA,
+                  const T *p, int64_t strideP, const T *r, int64_t strideR, Out *q,
+                  int64_t strideQ, Out *s, int64_t strideS, int64_t batch,
+                  cudaStream_t stream) {
+    using Acc = typename dmv::Traits<T>::Acc;
+    static_assert(sizeof(Acc) == sizeof(Out), "accumulator and output widths differ");
+    dualmv_status st = validate(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ,
+                                s, strideS, batch);
+    if (st != DUALMV_SUCCESS || batch == 0) return st;
+    if (batch == 1) {  // strides are irrelevant for one problem
+        strideA = M * lda; strideP = N; strideR = M; strideQ = M; strideS = N;
+    }
+
+    if (M == 0 || N == 0) {
+        cudaError_t e = zero_fill(reinterpret_cast<Acc *>(q), M, strideQ, batch, stream);
+        if (e == cudaSuccess)
+            e = zero_fill(reinterpret_cast<Acc *>(s), N, strideS, batch, stream);
+        return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
+    }
+    if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
+
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e);
+    DeviceState *ds = nullptr;
+    e = device_state(dev, &ds);
+    if (e != cudaSuccess) return cuda_fail(e);
+
+    // Path choice: TMA needs a 16-byte aligned base, 16-byte multiple
+    // strides and 32-bit coordinates.
+    const int64_t es = sizeof(T);
+    const bool three_d = batch > 1;
+    bool tma = g_path != DUALMV_PATH_DIRECT &&
+               (reinterpret_cast<uintptr_t>(A) % 16 == 0) && ((lda * es) % 16 == 0) &&
+               M < INT32_MAX && N < INT32_MAX && batch < INT32_MAX &&
+               (!three_d || (strideA > 0 && (strideA * es) % 16 == 0));
+    CUtensorMap map;
+    std::memset(&map, 0, sizeof map);
+    const int tile_rows = kWarps * (es == 4 ? kRpw4 : kRpw8);
+    if (tma) tma = encode_a<T>(&map, A, M, N, lda, strideA, batch, tile_rows, three_d);
+
+    dualmv_plan_t pl;
+    st = make_plan(M, N, batch, es, sizeof(Acc),
+                   (int64_t)ds->sms * (tma ? 1 : kDirectCtasPerSm), tma, &pl);
+    if (st != DUALMV_SUCCESS) return st;
+
+    void *ws = nullptr;
+    e = cudaMallocFromPoolAsync(&ws, (size_t)pl.workspace_bytes, ds->pool, stream);
+    if (e != cudaSuccess) {
+        g_last_cuda_error = static_cast<int>(e);
+        return DUALMV_ERR_ALLOC;
+    }
+    Params prm;
+    prm.A = A; prm.lda = lda; prm.strideA = strideA;
+    prm.p = p; prm.strideP = strideP;
+    prm.r = r; prm.strideR = strideR;
+    prm.q = q; prm.strideQ = strideQ;
+    prm.s = s; prm.strideS = strideS;
+    prm.M = M; prm.N = N; prm.batch = batch;
+    prm.bands = pl.bands; prm.stripes = pl.stripes; prm.tiles = pl.tiles;
+    prm.grid = pl.grid; prm.max_seg = pl.max_segments;
+    const int64_t q_ws_bytes = pl.bands > 1 ? batch * pl.bands * M * (int64_t)sizeof(Acc) : 0;
+    prm.q_ws = pl.bands > 1 ? ws : nullptr;
+    prm.s_ws = static_cast<unsigned char *>(ws) + ((q_ws_bytes + 255) / 256) * 256;
+
+    cudaEvent_t ev_start = g_kernel_ev_start, ev_stop = g_kernel_ev_stop;
+    g_kernel_ev_start = g_kernel_ev_stop = nullptr;
+    e = ev_start ? cudaEventRecord(ev_start, stream) : cudaSuccess;
+    if (e == cudaSuccess) {
+        if (tma) {
+            e = three_d ? launch_stream<T, true, true>(map, prm, pl, stream)
+                        : launch_stream<T, true, false>(map, prm, pl, stream);
+        } else {
+            e = launch_stream<T, false, false>(map, prm, pl, stream);
+        }
+    }
+    if (e == cudaSuccess && ev_stop) e = cudaEventRecord(ev_stop, stream);
+    if (e == cudaSuccess && (pl.bands > 1 || pl.grid > 1))
+        e = launch_combine<Acc>(prm, ds->sms, stream);
+    cudaError_t ef = cudaFreeAsync(ws, stream);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (ef != cudaSuccess) return cuda_fail(ef);
+    return DUALMV_SUCCESS;
+}
+
+}  // namespace
+
+// ================================================================ C ABI ===
+
+extern "C" {
+
+dualmv_status dualmv_f32(int64_t M, int64_t N, const float *A, int64_t lda, const float *p,
+                         const float *r, float *q, float *s, dualmv_stream_t stream) {
+    return run<float, float>(M, N, A, lda, 0, p, 0, r, 0, q, 0, s, 0, 1,
+                             reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_f64(int64_t M, int64_t N, const double *A, int64_t lda,
+                         const double *p, const double *r, double *q, double *s,
+                         dualmv_stream_t stream) {
+    return run<double, double>(M, N, A, lda, 0, p, 0, r, 0, q, 0, s, 0, 1,
+                               reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_i32(int64_t M, int64_t N, const int32_t *A, int64_t lda,
+                         const int32_t *p, const int32_t *r, int64_t *q, int64_t *s,
+                         dualmv_stream_t stream) {
+    return run<int32_t, int64_t>(M, N, A, lda, 0, p, 0, r, 0, q, 0, s, 0, 1,
+                                 reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_f32_strided_batched(int64_t M, int64_t N, const float *A, int64_t lda,
+                                         int64_t strideA, const float *p, int64_t strideP,
+                                         const float *r, int64_t strideR, float *q,
+                                         int64_t strideQ, float *s, int64_t strideS,
+                                         int64_t batch, dualmv_stream_t stream) {
+    return run<float, float>(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ, s,
+                             strideS, batch, reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_f64_strided_batched(int64_t M, int64_t N, const double *A, int64_t lda,
+                                         int64_t strideA, const double *p, int64_t strideP,
+                                         const double *r, int64_t strideR, double *q,
+                                         int64_t strideQ, double *s, int64_t strideS,
+                                         int64_t batch, dualmv_stream_t stream) {
+    return run<double, double>(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ, s,
+                               strideS, batch, reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_i32_strided_batched(int64_t M, int64_t N, const int32_t *A,
+                                         int64_t lda, int64_t strideA, const int32_t *p,
+                                         int64_t strideP, const int32_t *r, int64_t strideR,
+                                         int64_t *q, int64_t strideQ, int64_t *s,
+                                         int64_t strideS, int64_t batch,
+                                         dualmv_stream_t stream) {
+    return run<int32_t, int64_t>(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ,
+                                 s, strideS, batch, reinterpret_cast<cudaStream_t>(stream));
+}
+
+const char *dualmv_status_string(dualmv_status status) {
+    switch (status) {
+    case DUALMV_SUCCESS: return "success";
+    case DUALMV_ERR_INVALID_VALUE: return "invalid argument";
+    case DUALMV_ERR_ALLOC: return "workspace allocation failed";
+    case DUALMV_ERR_LAUNCH: return "CUDA launch or runtime error";
+    case DUALMV_ERR_TIMEOUT: return "a device-side bounded wait timed out";
+    case DUALMV_ERR_UNSUPPORTED: return "unsupported configuration";
+    }
+    return "unknown status";
+}
+
+int dualmv_last_cuda_error(void) { return g_last_cuda_error; }
+
+dualmv_status dualmv_device_fault(dualmv_stream_t stream) {
+    cudaError_t e = cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e);
+    unsigned int word = 0, zero = 0;
+    e = cudaMemcpyFromSymbol(&word, dmv::g_fault_word, sizeof word);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (word != 0) {
+        e = cudaMemcpyToSymbol(dmv::g_fault_word, &zero, sizeof zero);
+        if (e != cudaSuccess) return cuda_fail(e);
+        return DUALMV_ERR_TIMEOUT;
+    }
+    return DUALMV_SUCCESS;
+}
+
+void dualmv_record_kernel_events(void *start, void *stop) {
+    g_kernel_ev_start = static_cast<cudaEvent_t>(start);
+    g_kernel_ev_stop = static_cast<cudaEvent_t>(stop);
+}
+
+int dualmv_set_path(int path) {
+    if (path != DUALMV_PATH_AUTO && path != DUALMV_PATH_TMA && path != DUALMV_PATH_DIRECT)
+        return -1;
+    const int old = g_path;
+    g_path = path;
+    return old;
+}
+
+dualmv_status dualmv_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
+                          int64_t acc_bytes, int64_t num_sms, dualmv_plan_t *out) {
+    return make_plan(M, N, batch, elem_bytes, acc_bytes, num_sms, true, out);
+}
+
+}  // extern "C"

@@ -1,0 +1,580 @@
+// Device code of the fused dual matrix-vector product (BICG, Tables 1-2):
+//     q = A p,  s = A^T r,  one pass over a row-major A.
+//
+// Work decomposition
+//   A (one problem, or each problem of a strided batch) is cut into column
+//   bands of kBandCols = 256 columns and row stripes of BM rows; a tile is
+//   one stripe of one band.  Tiles are numbered band-major
+//   (problem, band, stripe) and CTA c of a persistent grid of G CTAs owns the
+//   contiguous range [c*T/G, (c+1)*T/G), so every CTA streams the same number
+//   of tiles to within one.
+//
+// Inside a CTA (TMA path)
+//   one producer warp issues one 2-D/3-D TMA box (256 columns x BM rows) per
+//   tile into a ring of kStages shared-memory buffers, tracked by mbarriers;
+//   W consumer warps each take RPW consecutive rows of every tile.  Lane l
+//   holds 8 columns of the band (two or four 16-byte vectors) and the
+//   matching 8 entries of p in registers.
+//     * q: each row's 8-term partial is reduced across the warp with a
+//       reduce-scatter butterfly (RPW rows share log2 steps), which yields
+//       the complete band partial of that row; it goes to q directly when
+//       the matrix is one band wide, else to the band-partial workspace.
+//     * s: each lane accumulates its 8 columns over the rows of the tile,
+//       then over a group of tiles, then over the segment (the run of
+//       stripes of one band that this CTA owns).  At a segment end the W
+//       warps' partials are summed in warp order through shared memory and
+//       written to s (segment covers the whole band) or to the segment
+//       workspace.
+//   A second kernel adds band partials (q) in ascending band order and
+//   segment partials (s) in ascending CTA order.  Every sum has a fixed
+//   order, so floating-point results are identical run to run.
+//
+// Plain-load path: the same schedule and arithmetic, but each consumer warp
+// reads its rows straight from global memory with bounds checks.  It serves
+// inputs the TMA unit cannot address (unaligned base or leading dimension).
+//
+// Every wait on an mbarrier is bounded in time.  A warp that gives up sets
+// the device fault word and stops waiting, but keeps the same control flow
+// (so no named barrier is left short of a participant) and the producer
+// still waits, bounded, for the copies it issued before the CTA exits.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace dmv {
+
+constexpr int kBandCols = 256;          // columns per band = TMA box width
+constexpr int kLaneCols = kBandCols / 32;  // columns per lane = 8
+constexpr int kGroupTiles = 16;         // tiles summed before the segment sum
+constexpr unsigned long long kWaitTimeoutNs = 2000000000ull;  // 2 s
+
+// Device fault word: bit 0 = a bounded wait timed out.  Read and cleared by
+// the host through dualmv_device_fault().
+__device__ unsigned int g_fault_word;
+
+template <typename T> struct Traits;
+template <> struct Traits<float> {
+    using Acc = float;
+    using Vec = float4;
+    static constexpr int kVecElems = 4;
+};
+template <> struct Traits<double> {
+    using Acc = double;
+    using Vec = double2;
+    static constexpr int kVecElems = 2;
+};
+// int32 inputs: exact 64-bit products, sums modulo 2^64 (unsigned, so the
+// wrap-around is defined), reinterpreted as int64 on output.
+template <> struct Traits<int32_t> {
+    using Acc = unsigned long long;
+    using Vec = int4;
+    static constexpr int kVecElems = 4;
+};
+
+// ------------------------------------------------------------ arithmetic --
+
+__device__ __forceinline__ float mul_acc(float a, float x, float acc) {
+    return fmaf(a, x, acc);
+}
+__device__ __forceinline__ double mul_acc(double a, double x, double acc) {
+    return fma(a, x, acc);
+}
+__device__ __forceinline__ unsigned long long mul_acc(int32_t a, int32_t x,
+                                                      unsigned long long acc) {
+    return acc + (unsigned long long)((long long)a * (long long)x);
+}
+
+template <typename Acc>
+__device__ __forceinline__ Acc shfl_xor(Acc v, int off) {
+    return __shfl_xor_sync(0xffffffffu, v, off);
+}
+
+// Element e of a 16-byte vector.
+__device__ __forceinline__ float vget(const float4 &v, int e) {
+    return e == 0 ? v.x : e == 1 ? v.y : e == 2 ? v.z : v.w;
+}
+__device__ __forceinline__ double vget(const double2 &v, int e) {
+    return e == 0 ? v.x : v.y;
+}
+__device__ __forceinline__ int32_t vget(const int4 &v, int e) {
+    return e == 0 ? v.x : e == 1 ? v.y : e == 2 ? v.z : v.w;
+}
+
+// Band-relative column of element e of vector v held by `lane`.
+template <typename T>
+__device__ __forceinline__ int lane_col(int v, int lane, int e) {
+    return (v * 32 + lane) * Traits<T>::kVecElems + e;
+}
+
+// Reduce-scatter butterfly over RPW row partials held by every lane.  On
+// return, v[0] of lane l is the full warp sum of row
+// (l >> (5 - log2 RPW)) & (RPW - 1).  Step k exchanges half of the
+// remaining values across lane bit (4 - k); the remaining bits are summed
+// with plain xor steps.  Fixed order, so deterministic.
+template <int RPW, typename Acc>
+__device__ __forceinline__ void warp_rows_reduce(Acc (&v)[RPW], int lane) {
+    int off = 16;
+#pragma unroll
+    for (int h = RPW / 2; h >= 1; h /= 2) {
+        const bool upper = (lane & off) != 0;
+#pragma unroll
+        for (int k = 0; k < h; ++k) {
+            const Acc send = upper ? v[k] : v[k + h];
+            const Acc keep = upper ? v[k + h] : v[k];
+            v[k] = keep + shfl_xor(send, off);
+        }
+        off >>= 1;
+    }
+#pragma unroll
+    for (; off >= 1; off >>= 1) v[0] = v[0] + shfl_xor(v[0], off);
+}
+
+template <int RPW>
+__device__ __forceinline__ int butterfly_row(int lane) {
+    constexpr int L = RPW == 1 ? 0 : RPW == 2 ? 1 : RPW == 4 ? 2 : RPW == 8 ? 3 : 4;
+    return (lane >> (5 - L)) & (RPW - 1);
+}
+template <int RPW>
+__device__ __forceinline__ bool butterfly_writer(int lane) {
+    constexpr int L = RPW == 1 ? 0 : RPW == 2 ? 1 : RPW == 4 ? 2 : RPW == 8 ? 3 : 4;
+    return (lane & ((32 >> L) - 1)) == 0;
+}
+
+// --------------------------------------------------- mbarrier and TMA ----
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile(
+        "{\n\t.reg .b64 st;\n\t"
+        "mbarrier.arrive.shared::cta.b64 st, [%0];\n\t}" ::"r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile(
+        "{\n\t.reg .b64 st;\n\t"
+        "mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n\t}" ::"r"(bar),
+        "r"(bytes)
+        : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Slow path of mbar_wait_bounded: keeps polling for at most kWaitTimeoutNs,
+// then sets the device fault word and returns false.
+__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity) {
+    const unsigned long long t0 = global_ns();
+    for (;;) {
+        for (int i = 0; i < 64; ++i)
+            if (mbar_try_wait(bar, parity)) return true;
+        if (global_ns() - t0 > kWaitTimeoutNs) {
+            atomicOr(&g_fault_word, 1u);
+            return false;
+        }
+    }
+}
+
+// Wait for the phase of `bar` with parity `parity`, bounded in time.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    return mbar_wait_slow(bar, parity);
+}
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map,
+                                            int x, int y, uint32_t bar, uint64_t pol) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(pol)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map,
+                                            int x, int y, int z, uint32_t bar,
+                                            uint64_t pol) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar),
+        "l"(pol)
+        : "memory");
+}
+
+__device__ __forceinline__ void named_barrier(int id, int threads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
+__device__ __forceinline__ void pdl_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// ------------------------------------------------------------ parameters --
+
+struct Params {
+    const void *A;
+    int64_t lda, strideA;
+    const void *p;
+    int64_t strideP;
+    const void *r;
+    int64_t strideR;
+    void *q;
+    int64_t strideQ;
+    void *s;
+    int64_t strideS;
+    int64_t M, N, batch;
+    int64_t bands, stripes, tiles, grid, max_seg;
+    void *q_ws;  // [batch][bands][M] band partials of q (bands > 1 only)
+    void *s_ws;  // [grid][max_seg][kBandCols] segment partials of s
+};
+
+// First tile of CTA c, and the CTA that owns tile t (inverse of the split).
+__host__ __device__ __forceinline__ int64_t cta_first_tile(int64_t c, int64_t T,
+                                                           int64_t G) {
+    return (c * T) / G;
+}
+__host__ __device__ __forceinline__ int64_t cta_of_tile(int64_t t, int64_t T,
+                                                        int64_t G) {
+    return ((t + 1) * G - 1) / T;
+}
+
+template <int W, int RPW, int STAGES, int TILE_BYTES, typename Acc>
+struct SmemLayout {
+    static constexpr int kRing = STAGES * TILE_BYTES;
+    static constexpr int kScratch = W * kBandCols * (int)sizeof(Acc);
+    static constexpr int kBars = 2 * STAGES * 8;
+    static constexpr int kTotal = 1024 + kRing + kScratch + kBars;  // + align slack
+};
+
+// ------------------------------------------------------------ main kernel --
+//
+// Template: element type T, W consumer warps, RPW rows per warp per tile,
+// STAGES ring depth, kTma = TMA producer (else plain loads), kBatched3d =
+// 3-D tensor map (batch as the outer coordinate).
+template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d>
+__global__ void __launch_bounds__((W + (kTma ? 1 : 0)) * 32, 1)
+dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
+    using Acc = typename Traits<T>::Acc;
+    using Vec = typename Traits<T>::Vec;
+    constexpr int VE = Traits<T>::kVecElems;
+    constexpr int VPL = kLaneCols / VE;  // 16-byte vectors per lane per row
+    constexpr int BM = W * RPW;
+    constexpr int ROW_BYTES = kBandCols * (int)sizeof(T);
+    constexpr int TILE_BYTES = BM * ROW_BYTES;
+    using L = SmemLayout<W, RPW, STAGES, TILE_BYTES, Acc>;
+
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    unsigned char *ring = smem;
+    Acc *scratch = reinterpret_cast<Acc *>(smem + L::kRing);
+    uint64_t *full_bar = reinterpret_cast<uint64_t *>(smem + L::kRing + L::kScratch);
+    uint64_t *empty_bar = full_bar + STAGES;
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t T_ = prm.tiles, G = prm.grid, S = prm.stripes;
+    const int64_t c = blockIdx.x;
+    const int64_t t0 = cta_first_tile(c, T_, G);
+    const int64_t t1 = cta_first_tile(c + 1, T_, G);
+    const int64_t ntiles = t1 - t0;
+    const int64_t g_first = t0 / S;
+
+    if constexpr (kTma) {
+        if (threadIdx.x == 0) {
+            for (int i = 0; i < STAGES; ++i) {
+                mbar_init(smem_u32(&full_bar[i]), 1);
+                mbar_init(smem_u32(&empty_bar[i]), W);
+            }
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        }
+        __syncthreads();
+    }
+    // Dependent grids (the combine kernel) may start launching now; they
+    // wait for this grid's completion before reading anything it writes.
+    pdl_launch_dependents();
+
+    // ------------------------------------------------------ producer ----
+    if constexpr (kTma) {
+        if (warp == W) {
+            if (lane == 0) {
+                const uint64_t pol = policy_evict_first();
+                bool ok = true;
+                int64_t issued = 0;
+                for (int64_t k = 0; k < ntiles; ++k) {
+                    const int stage = (int)(k % STAGES);
+                    const uint32_t round = (uint32_t)(k / STAGES);
+                    if (ok && round > 0)
+                        ok = mbar_wait_bounded(smem_u32(&empty_bar[stage]),
+                                               (round - 1) & 1u);
+                    if (!ok) break;
+                    const int64_t t = t0 + k;
+                    const int64_t g = t / S;
+                    const int stripe = (int)(t - g * S);
+                    const int band = (int)(g % prm.bands);
+                    const int b = (int)(g / prm.bands);
+                    const uint32_t fb = smem_u32(&full_bar[stage]);
+                    mbar_arrive_expect_tx(fb, TILE_BYTES);
+                    const uint32_t dst = smem_u32(ring + (size_t)stage * TILE_BYTES);
+                    if constexpr (kBatched3d)
+                        tma_load_3d(dst, &tmap, band * kBandCols, stripe * BM, b, fb, pol);
+                    else
+                        tma_load_2d(dst, &tmap, band * kBandCols, stripe * BM, fb, pol);
+                    issued = k + 1;
+                }
+                // Before the CTA exits, every copy it issued must have landed
+                // (bounded): the last min(STAGES, ntiles) issued stages.
+                for (int64_t k = issued > STAGES ? issued - STAGES : 0; k < issued; ++k) {
+                    const int stage = (int)(k % STAGES);
+                    mbar_wait_bounded(smem_u32(&full_bar[stage]),
+                                      (uint32_t)(k / STAGES) & 1u);
+                }
+            }
+            return;
+        }
+    }
+
+    // ----------------------------------------------------- consumers ----
+    const T *__restrict__ Ag = static_cast<const T *>(prm.A);
+    const T *__restrict__ pg = static_cast<const T *>(prm.p);
+    const T *__restrict__ rg = static_cast<const T *>(prm.r);
+    const int nthreads_c = W * 32;
+
+    T pv[kLaneCols];
+    Acc grp[kLaneCols], seg[kLaneCols];
+#pragma unroll
+    for (int e = 0; e < kLaneCols; ++e) {
+        pv[e] = T(0);
+        grp[e] = Acc(0);
+        seg[e] = Acc(0);
+    }
+    int ngrp = 0;
+    int64_t seg_start_stripe = 0;
+    bool ok = true;
+
+    for (int64_t k = 0; k < ntiles; ++k) {
+        const int64_t t = t0 + k;
+        const int64_t g = t / S;
+        const int64_t stripe = t - g * S;
+        const int64_t band = g % prm.bands;
+        const int64_t b = g / prm.bands;
+        const int64_t col0 = band * kBandCols;
+        const int64_t row0 = stripe * BM + (int64_t)warp * RPW;
+
+        if (k == 0 || stripe == 0) {  // a new segment: this band's p
+            seg_start_stripe = stripe;
+            const T *pb = pg + b * prm.strideP;
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) {
+                    const int64_t col = col0 + lane_col<T>(v, lane, e);
+                    pv[v * VE + e] = col < prm.N ? pb[col] : T(0);
+                }
+        }
+
+        // r for this warp's RPW rows (lane i < RPW holds row row0 + i).
+        T rmine = T(0);
+        if (lane < RPW && row0 + lane < prm.M) rmine = rg[b * prm.strideR + row0 + lane];
+
+        Acc qp[RPW];
+        Acc tacc[kLaneCols];
+#pragma unroll
+        for (int e = 0; e < kLaneCols; ++e) tacc[e] = Acc(0);
+
+        const int stage = (int)(k % STAGES);
+        if constexpr (kTma) {
+            if (ok) ok = mbar_wait_bounded(smem_u32(&full_bar[stage]),
+                                           (uint32_t)(k / STAGES) & 1u);
+        }
+#pragma unroll
+        for (int i = 0; i < RPW; ++i) {
+            Vec a[VPL];
+            if constexpr (kTma) {
+                const Vec *rowp = reinterpret_cast<const Vec *>(
+                    ring + (size_t)stage * TILE_BYTES +
+                    (size_t)(warp * RPW + i) * ROW_BYTES);
+#pragma unroll
+                for (int v = 0; v < VPL; ++v) a[v] = rowp[v * 32 + lane];
+            } else {
+                const int64_t row = row0 + i;
+                const T *arow = Ag + b * prm.strideA + row * prm.lda;
+#pragma unroll
+                for (int v = 0; v < VPL; ++v) {
+                    T tmp[VE];
+#pragma unroll
+                    for (int e = 0; e < VE; ++e) {
+                        const int64_t col = col0 + lane_col<T>(v, lane, e);
+                        tmp[e] = (row < prm.M && col < prm.N) ? arow[col] : T(0);
+                    }
+                    if constexpr (VE == 4) a[v] = Vec{tmp[0], tmp[1], tmp[2], tmp[3]};
+                    else a[v] = Vec{tmp[0], tmp[1]};
+                }
+            }
+            const T ri = __shfl_sync(0xffffffffu, rmine, i);
+            Acc dot = Acc(0);
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) {
+                    const T av = vget(a[v], e);
+                    dot = mul_acc(av, pv[v * VE + e], dot);
+                    tacc[v * VE + e] = mul_acc(av, ri, tacc[v * VE + e]);
+                }
+            qp[i] = dot;
+        }
+        if constexpr (kTma) {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[stage]));
+        }
+
+        // q: complete band partial of each of this warp's rows.
+        warp_rows_reduce<RPW>(qp, lane);
+        if (butterfly_writer<RPW>(lane)) {
+            const int64_t row = row0 + butterfly_row<RPW>(lane);
+            if (row < prm.M) {
+                if (prm.bands == 1) {
+                    Acc *qo = static_cast<Acc *>(prm.q);
+                    qo[b * prm.strideQ + row] = qp[0];
+                } else {
+                    Acc *qw = static_cast<Acc *>(prm.q_ws);
+                    qw[(b * prm.bands + band) * prm.M + row] = qp[0];
+                }
+            }
+        }
+
+        // s: tile -> group -> segment accumulation.
+#pragma unroll
+        for (int e = 0; e < kLaneCols; ++e) grp[e] = grp[e] + tacc[e];
+        if (++ngrp == kGroupTiles) {
+#pragma unroll
+            for (int e = 0; e < kLaneCols; ++e) {
+                seg[e] = seg[e] + grp[e];
+                grp[e] = Acc(0);
+            }
+            ngrp = 0;
+        }
+
+        if (stripe == S - 1 || k == ntiles - 1) {  // segment end: flush s
+#pragma unroll
+            for (int e = 0; e < kLaneCols; ++e) seg[e] = seg[e] + grp[e];
+            Acc *sw = scratch + warp * kBandCols;
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) sw[lane_col<T>(v, lane, e)] = seg[v * VE + e];
+            named_barrier(1, nthreads_c);
+            const bool whole_band = (seg_start_stripe == 0 && stripe == S - 1);
+            for (int col = threadIdx.x; col < kBandCols; col += nthreads_c) {
+                Acc acc = scratch[col];
+#pragma unroll
+                for (int w = 1; w < W; ++w) acc = acc + scratch[w * kBandCols + col];
+                if (whole_band) {
+                    if (col0 + col < prm.N) {
+                        Acc *so = static_cast<Acc *>(prm.s);
+                        so[b * prm.strideS + col0 + col] = acc;
+                    }
+                } else {
+                    Acc *sws = static_cast<Acc *>(prm.s_ws);
+                    sws[((c * prm.max_seg) + (g - g_first)) * kBandCols + col] = acc;
+                }
+            }
+            named_barrier(1, nthreads_c);
+#pragma unroll
+            for (int e = 0; e < kLaneCols; ++e) {
+                grp[e] = Acc(0);
+                seg[e] = Acc(0);
+            }
+            ngrp = 0;
+        }
+    }
+}
+
+// --------------------------------------------------------- combine kernel --
+//
+// Adds the band partials of q (ascending band) and the segment partials of
+// s (ascending CTA) for every band that more than one CTA touched.  Launched
+// as a programmatic dependent of the stream kernel: it waits for that grid
+// to complete before reading the workspace.
+template <typename Acc>
+__global__ void __launch_bounds__(256) dualmv_combine_kernel(const Params prm) {
+    pdl_wait();
+    const int64_t T_ = prm.tiles, G = prm.grid, S = prm.stripes;
+    const int64_t nq = prm.bands > 1 ? prm.batch * prm.M : 0;
+    const int64_t ns = prm.batch * prm.N;
+    const int64_t total = nq + ns;
+    const Acc *qw = static_cast<const Acc *>(prm.q_ws);
+    const Acc *sw = static_cast<const Acc *>(prm.s_ws);
+    for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        if (idx < nq) {
+            const int64_t b = idx / prm.M, i = idx - b * prm.M;
+            Acc acc = qw[(b * prm.bands) * prm.M + i];
+            for (int64_t band = 1; band < prm.bands; ++band)
+                acc = acc + qw[(b * prm.bands + band) * prm.M + i];
+            static_cast<Acc *>(prm.q)[b * prm.strideQ + i] = acc;
+        } else {
+            const int64_t js = idx - nq;
+            const int64_t b = js / prm.N, j = js - b * prm.N;
+            const int64_t band = j / kBandCols, col = j - band * kBandCols;
+            const int64_t g = b * prm.bands + band;
+            const int64_t c_lo = cta_of_tile(g * S, T_, G);
+            const int64_t c_hi = cta_of_tile(g * S + S - 1, T_, G);
+            if (c_lo == c_hi) continue;  // written directly by the stream kernel
+            Acc acc = Acc(0);
+            for (int64_t cc = c_lo; cc <= c_hi; ++cc) {
+                const int64_t seg = g - cta_first_tile(cc, T_, G) / S;
+                const Acc v = sw[(cc * prm.max_seg + seg) * kBandCols + col];
+                acc = (cc == c_lo) ? v : acc + v;
+            }
+            static_cast<Acc *>(prm.s)[b * prm.strideS + j] = acc;
+        }
+    }
+}
+
+// Zero-fill of strided outputs (empty problems).
+template <typename Acc>
+__global__ void dualmv_zero_kernel(Acc *out, int64_t len, int64_t stride, int64_t batch) {
+    const int64_t total = len * batch;
+    for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t b = idx / len, i = idx - b * len;
+        out[b * stride + i] = Acc(0);
+    }
+}
+
+}  // namespace dmv

@@ -205,6 +205,12 @@ def run_native(args):
     kern_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                for _ in range(K)]
     region = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    # torch creates the CUDA event lazily on its first record; the library
+    # records the kernel events itself, so make them exist first.
+    for ks, ke in kern_ev:
+        ks.record(stream)
+        ke.record(stream)
+    torch.cuda.synchronize(dev)
 
     sampler = ClockSampler(gpu_uuid(torch, dev))
     sampler.start()

@@ -119,6 +119,19 @@ bool encode_a(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
 
 // ------------------------------------------------------------------ plan --
 
+template <typename T>
+int64_t smem_of(bool tma) {
+    constexpr int rpw = sizeof(T) == 4 ? kRpw4 : kRpw8;
+    return tma ? dmv::SmemLayout<T, kWarps, rpw, kStages, true>::kTotal
+               : dmv::SmemLayout<T, kWarps, rpw, kStages, false>::kTotal;
+}
+
+// Shared memory of the stream kernel for an element / accumulator width.
+int64_t smem_bytes_for(int64_t elem_bytes, int64_t acc_bytes, bool tma) {
+    if (elem_bytes == 8) return smem_of<double>(tma);
+    return acc_bytes == 8 ? smem_of<int32_t>(tma) : smem_of<float>(tma);
+}
+
 dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
                         int64_t acc_bytes, int64_t ctas, bool tma, dualmv_plan_t *pl) {
     if (M <= 0 || N <= 0 || batch <= 0 || ctas <= 0 || pl == nullptr)
@@ -149,9 +162,7 @@ dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
     const int64_t q_ws = p.bands > 1 ? batch * p.bands * M * acc_bytes : 0;
     const int64_t s_ws = p.grid * p.max_segments * kBandCols * acc_bytes;
     p.workspace_bytes = ((q_ws + 255) / 256) * 256 + s_ws;
-    const int64_t tile_bytes = bm * kBandCols * elem_bytes;
-    const int64_t scratch = kWarps * kBandCols * acc_bytes;
-    p.smem_bytes = tma ? 1024 + kStages * tile_bytes + scratch + 2 * kStages * 8 : scratch;
+    p.smem_bytes = smem_bytes_for(elem_bytes, acc_bytes, tma);
     p.threads = (kWarps + (tma ? 1 : 0)) * 32;
     *pl = p;
     return DUALMV_SUCCESS;

@@ -272,12 +272,20 @@ __host__ __device__ __forceinline__ int64_t cta_of_tile(int64_t t, int64_t T,
     return ((t + 1) * G - 1) / T;
 }
 
-template <int W, int RPW, int STAGES, int TILE_BYTES, typename Acc>
+// Dynamic shared memory of the stream kernel, the single definition used by
+// both the kernel (offsets) and the host (launch size).  TMA path: a
+// 1024-byte-aligned ring of STAGES tiles, the warp scratch for the s flush,
+// then the full/empty mbarriers.  Plain-load path: the scratch only.
+template <typename T, int W, int RPW, int STAGES, bool kTma>
 struct SmemLayout {
-    static constexpr int kRing = STAGES * TILE_BYTES;
+    using Acc = typename Traits<T>::Acc;
+    static constexpr int kTileBytes = W * RPW * kBandCols * (int)sizeof(T);
+    static constexpr int kAlign = kTma ? 1024 : 16;
+    static constexpr int kRing = kTma ? STAGES * kTileBytes : 0;
     static constexpr int kScratch = W * kBandCols * (int)sizeof(Acc);
-    static constexpr int kBars = 2 * STAGES * 8;
-    static constexpr int kTotal = 1024 + kRing + kScratch + kBars;  // + align slack
+    static constexpr int kBars = kTma ? 2 * STAGES * 8 : 0;
+    // kAlign bytes of slack let the kernel round the dynamic base up.
+    static constexpr int kTotal = kAlign + kRing + kScratch + kBars;
 };
 
 // ------------------------------------------------------------ main kernel --
@@ -295,11 +303,13 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
     constexpr int BM = W * RPW;
     constexpr int ROW_BYTES = kBandCols * (int)sizeof(T);
     constexpr int TILE_BYTES = BM * ROW_BYTES;
-    using L = SmemLayout<W, RPW, STAGES, TILE_BYTES, Acc>;
+    using L = SmemLayout<T, W, RPW, STAGES, kTma>;
+    static_assert(L::kTileBytes == TILE_BYTES, "tile size mismatch");
 
     extern __shared__ unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+        (reinterpret_cast<uintptr_t>(smem_raw) + (L::kAlign - 1)) &
+        ~uintptr_t(L::kAlign - 1));
     unsigned char *ring = smem;
     Acc *scratch = reinterpret_cast<Acc *>(smem + L::kRing);
     uint64_t *full_bar = reinterpret_cast<uint64_t *>(smem + L::kRing + L::kScratch);

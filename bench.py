@@ -146,6 +146,22 @@ def gpu_uuid(torch, dev):
         return None
 
 
+def workload_from_args(inputs, args):
+    """The named workload, optionally resized (for small profiling cases)."""
+    w = inputs.WORKLOADS[args.workload]
+    kw = {}
+    for k in ("M", "N", "lda", "batch"):
+        v = getattr(args, k)
+        if v is not None:
+            kw[k] = v
+    if "N" in kw and "lda" not in kw:
+        kw["lda"] = kw["N"]
+    if kw:
+        w = w.scaled(name=w.name + "_resized_" + "_".join(f"{k}{v}" for k, v in kw.items()),
+                     **kw)
+    return w
+
+
 # ---------------------------------------------------------- distributed ---
 
 def dist_setup(torch, backend):
@@ -186,7 +202,7 @@ def run_native(args):
     import paper_2512_22147_gb300 as dm
     from paper_2512_22147_gb300 import inputs
 
-    w = inputs.WORKLOADS[args.workload]
+    w = workload_from_args(inputs, args)
     A, p, r = inputs.generate(w, dev)
     Av = A[..., : w.N]
     q, s = inputs.empty_outputs(w, dev)
@@ -200,45 +216,59 @@ def run_native(args):
         raise RuntimeError("device fault during warm-up")
 
     K = args.steps
-    call_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(K)]
-    kern_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(K)]
     region = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-    # torch creates the CUDA event lazily on its first record; the library
-    # records the kernel events itself, so make them exist first.
-    for ks, ke in kern_ev:
-        ks.record(stream)
-        ke.record(stream)
-    torch.cuda.synchronize(dev)
 
+    # Timed region: K back-to-back calls, nothing recorded between them.
     sampler = ClockSampler(gpu_uuid(torch, dev))
     sampler.start()
     time.sleep(0.3)  # let the sampler start before the timed region
     barrier(world)
     torch.cuda.synchronize(dev)
     region[0].record(stream)
-    for i in range(K):
+    for _ in range(K):
+        dm.dualmv(Av, p, r, q=q, s=s)
+    region[1].record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clocks = sampler.stop()
+    if dm.device_fault() != dm.DUALMV_SUCCESS:
+        raise RuntimeError("device fault during the timed region")
+    region_ms = region[0].elapsed_time(region[1])
+    region_ms = max_over_ranks(torch, region_ms, world, dev)
+    ms_per_step = region_ms / K
+    value = world * nbytes * K / (region_ms * 1e-3) / 1e9
+
+    # Instrumented region: the same calls, each bracketed by events, and the
+    # streaming kernel bracketed by events the library records on its own
+    # stream (dualmv_record_kernel_events).  Gives the per-call times for the
+    # trimmed mean of Eq. 3 and the kernel time for the roofline.
+    Ki = min(K, args.instrumented_steps)
+    call_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(Ki)]
+    kern_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(Ki)]
+    # torch creates the CUDA event lazily on its first record; the library
+    # records the kernel events itself, so make them exist first.
+    for ks, ke in kern_ev:
+        ks.record(stream)
+        ke.record(stream)
+    torch.cuda.synchronize(dev)
+    for i in range(Ki):
         ks, ke = kern_ev[i]
         dm.dualmv_record_kernel_events(ks.cuda_event, ke.cuda_event)
         call_ev[i][0].record(stream)
         dm.dualmv(Av, p, r, q=q, s=s)
         call_ev[i][1].record(stream)
-    region[1].record(stream)
     torch.cuda.synchronize(dev)
-    barrier(world)
-    clocks = sampler.stop()
-    fault = dm.device_fault()
-    if fault != dm.DUALMV_SUCCESS:
-        raise RuntimeError("device fault during the timed region")
-
-    region_ms = region[0].elapsed_time(region[1])
-    region_ms = max_over_ranks(torch, region_ms, world, dev)
+    if dm.device_fault() != dm.DUALMV_SUCCESS:
+        raise RuntimeError("device fault during the instrumented region")
     step_ms = [a.elapsed_time(b) for a, b in call_ev]
     kern_ms = [a.elapsed_time(b) for a, b in kern_ev]
-    ms_per_step = region_ms / K
-    value = world * nbytes * K / (region_ms * 1e-3) / 1e9
 
+    plan = dm.dualmv_plan(w.M, w.N, w.nbatch, inputs.ELEM_BYTES[w.dtype],
+                          inputs.OUT_BYTES[w.dtype],
+                          torch.cuda.get_device_properties(dev).multi_processor_count)
+    launches_per_call = 1 + (1 if (plan.bands > 1 or plan.grid > 1) else 0)
     peak, peak_src = measured_peak()
     kern_avg_ms = sum(kern_ms) / len(kern_ms)
     achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9
@@ -275,7 +305,7 @@ def run_native(args):
             "parallelism": f"replicas x{world}",
         },
         "pct_of_peak": round(100.0 * value / (world * peak), 2),
-        "trimmed_mean_ms": round(trimmed_mean(step_ms, 3) if K > 6 else ms_per_step, 5),
+        "trimmed_mean_ms": round(trimmed_mean(step_ms, 3) if Ki > 6 else statistics.mean(step_ms), 5),
         "median_step_ms": round(statistics.median(step_ms), 5),
         "roofline": {
             "bound": "hbm",
@@ -292,7 +322,8 @@ def run_native(args):
         },
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": 2 * K,
+        "gpu_launches": launches_per_call * K,
+        "instrumented_steps": Ki,
         "clocks": clocks,
     }
     if rank == 0:
@@ -386,7 +417,7 @@ def run_reference(args):
     import torch
 
     from paper_2512_22147_gb300 import inputs
-    w = inputs.WORKLOADS[args.workload]
+    w = workload_from_args(inputs, args)
     A, p, r = inputs.generate(w, "cpu")
     A_np, p_np, r_np = A.numpy(), p.numpy(), r.numpy()
     budget = args.cpu_seconds / max(1, args.steps + args.warmup)
@@ -423,6 +454,11 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
+    ap.add_argument("--instrumented-steps", type=int, default=300)
+    ap.add_argument("--M", type=int, default=None, help="resize the workload (profiling)")
+    ap.add_argument("--N", type=int, default=None)
+    ap.add_argument("--lda", type=int, default=None)
+    ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-e2e", action="store_true")

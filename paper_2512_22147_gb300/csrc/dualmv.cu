@@ -7,6 +7,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstdint>
 #include <cstdlib>
 #include <cstring>
@@ -203,25 +204,40 @@ bool fault_injected_alloc() {
 
 template <typename T, bool kTma, bool k3d>
 cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
-                          cudaStream_t stream) {
+                          int dev, cudaStream_t stream) {
     constexpr int rpw = sizeof(T) == 4 ? kRpw4 : kRpw8;
     auto kern = dmv::dualmv_stream_kernel<T, kWarps, rpw, kStages, kTma, k3d>;
-    // Setting the attribute is idempotent and cheap; doing it per call keeps
-    // it correct on every device without extra bookkeeping.
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)pl.smem_bytes);
-    if (e != cudaSuccess) return e;
+    // The shared-memory opt-in is per device and per kernel; set it once.
+    static std::atomic<uint64_t> opted_in{0};
+    const uint64_t bit = 1ull << (dev & 63);
+    if (!(opted_in.load(std::memory_order_acquire) & bit)) {
+        cudaError_t e = cudaFuncSetAttribute(
+            kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem_bytes);
+        if (e != cudaSuccess) return e;
+        opted_in.fetch_or(bit, std::memory_order_acq_rel);
+    }
     kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(map, prm);
     return cudaGetLastError();
 }
 
+// Chunks per q output in the combine kernel: the smallest power of two
+// giving at most about 8 band partials per thread, at most 32.
+int combine_chunks(int64_t bands) {
+    int c = 1;
+    while (c < 32 && (int64_t)c * 8 < bands) c *= 2;
+    return c;
+}
+
 template <typename Acc>
-cudaError_t launch_combine(const Params &prm, int sms, cudaStream_t stream) {
-    const int64_t total = (prm.bands > 1 ? prm.batch * prm.M : 0) + prm.batch * prm.N;
-    int64_t blocks = (total + 255) / 256;
-    const int64_t cap = (int64_t)sms * 8;
-    if (blocks > cap) blocks = cap;
-    if (blocks < 1) blocks = 1;
+cudaError_t launch_combine(const Params &prm, cudaStream_t stream) {
+    const int chunks = combine_chunks(prm.bands);
+    const int64_t rows_per_block = 256 / chunks;
+    const int64_t q_blocks =
+        prm.bands > 1 ? (prm.batch * prm.M + rows_per_block - 1) / rows_per_block : 0;
+    const int64_t s_blocks = prm.grid > 1 ? prm.batch * prm.bands : 0;
+    const int64_t blocks = q_blocks + s_blocks;
+    if (blocks == 0) return cudaSuccess;
+    if (blocks > INT32_MAX) return cudaErrorInvalidConfiguration;
     cudaLaunchConfig_t cfg;
     std::memset(&cfg, 0, sizeof cfg);
     cfg.gridDim = dim3((unsigned)blocks);
@@ -233,7 +249,7 @@ cudaError_t launch_combine(const Params &prm, int sms, cudaStream_t stream) {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, dmv::dualmv_combine_kernel<Acc>, prm);
+    return cudaLaunchKernelEx(&cfg, dmv::dualmv_combine_kernel<Acc>, prm, q_blocks, chunks);
 }
 
 template <typename Acc>
@@ -318,15 +334,14 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     e = ev_start ? cudaEventRecord(ev_start, stream) : cudaSuccess;
     if (e == cudaSuccess) {
         if (tma) {
-            e = three_d ? launch_stream<T, true, true>(map, prm, pl, stream)
-                        : launch_stream<T, true, false>(map, prm, pl, stream);
+            e = three_d ? launch_stream<T, true, true>(map, prm, pl, dev, stream)
+                        : launch_stream<T, true, false>(map, prm, pl, dev, stream);
         } else {
-            e = launch_stream<T, false, false>(map, prm, pl, stream);
+            e = launch_stream<T, false, false>(map, prm, pl, dev, stream);
         }
     }
     if (e == cudaSuccess && ev_stop) e = cudaEventRecord(ev_stop, stream);
-    if (e == cudaSuccess && (pl.bands > 1 || pl.grid > 1))
-        e = launch_combine<Acc>(prm, ds->sms, stream);
+    if (e == cudaSuccess) e = launch_combine<Acc>(prm, stream);
     cudaError_t ef = cudaFreeAsync(ws, stream);
     if (e != cudaSuccess) return cuda_fail(e);
     if (ef != cudaSuccess) return cuda_fail(ef);

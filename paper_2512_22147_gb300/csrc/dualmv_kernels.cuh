@@ -536,44 +536,68 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
 
 // --------------------------------------------------------- combine kernel --
 //
-// Adds the band partials of q (ascending band) and the segment partials of
-// s (ascending CTA) for every band that more than one CTA touched.  Launched
-// as a programmatic dependent of the stream kernel: it waits for that grid
-// to complete before reading the workspace.
+// Adds the band partials of q and the segment partials of s in a fixed
+// order, for the outputs the stream kernel could not finish alone.  Launched
+// as a programmatic dependent of the stream kernel: it waits for that grid to
+// complete before reading the workspace.  256 threads per block.
+//   Blocks [0, q_blocks): rows of q.  A block takes R = 256 / C consecutive
+//     outputs (over batch * M) and C chunks; chunk y adds bands y, y + C,
+//     y + 2C, ... in ascending order, then the C chunk sums are added in
+//     ascending chunk order.  C depends only on the band count, so the
+//     order (and the rounding) is the same on every call.
+//   Blocks [q_blocks, q_blocks + batch * bands): one band of s each; the
+//     segments of a band split between CTAs are added in ascending CTA order.
 template <typename Acc>
-__global__ void __launch_bounds__(256) dualmv_combine_kernel(const Params prm) {
+__global__ void __launch_bounds__(256)
+dualmv_combine_kernel(const Params prm, int64_t q_blocks, int q_chunks) {
     pdl_wait();
-    const int64_t T_ = prm.tiles, G = prm.grid, S = prm.stripes;
-    const int64_t nq = prm.bands > 1 ? prm.batch * prm.M : 0;
-    const int64_t ns = prm.batch * prm.N;
-    const int64_t total = nq + ns;
+    __shared__ Acc part[256];
     const Acc *qw = static_cast<const Acc *>(prm.q_ws);
     const Acc *sw = static_cast<const Acc *>(prm.s_ws);
-    for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-         idx += (int64_t)gridDim.x * blockDim.x) {
-        if (idx < nq) {
-            const int64_t b = idx / prm.M, i = idx - b * prm.M;
-            Acc acc = qw[(b * prm.bands) * prm.M + i];
-            for (int64_t band = 1; band < prm.bands; ++band)
-                acc = acc + qw[(b * prm.bands + band) * prm.M + i];
-            static_cast<Acc *>(prm.q)[b * prm.strideQ + i] = acc;
-        } else {
-            const int64_t js = idx - nq;
-            const int64_t b = js / prm.N, j = js - b * prm.N;
-            const int64_t band = j / kBandCols, col = j - band * kBandCols;
-            const int64_t g = b * prm.bands + band;
-            const int64_t c_lo = cta_of_tile(g * S, T_, G);
-            const int64_t c_hi = cta_of_tile(g * S + S - 1, T_, G);
-            if (c_lo == c_hi) continue;  // written directly by the stream kernel
-            Acc acc = Acc(0);
-            for (int64_t cc = c_lo; cc <= c_hi; ++cc) {
-                const int64_t seg = g - cta_first_tile(cc, T_, G) / S;
-                const Acc v = sw[(cc * prm.max_seg + seg) * kBandCols + col];
-                acc = (cc == c_lo) ? v : acc + v;
+    if ((int64_t)blockIdx.x < q_blocks) {
+        const int C = q_chunks, R = 256 / C;
+        const int x = threadIdx.x % R, y = threadIdx.x / R;
+        const int64_t idx = (int64_t)blockIdx.x * R + x;
+        const bool valid = idx < prm.batch * prm.M;
+        int64_t b = 0, i = 0;
+        Acc acc = Acc(0);
+        if (valid) {
+            b = idx / prm.M;
+            i = idx - b * prm.M;
+            const Acc *base = qw + (b * prm.bands) * prm.M + i;
+            int64_t k = y;
+            if (k < prm.bands) {
+                acc = base[k * prm.M];
+                k += C;
             }
-            static_cast<Acc *>(prm.s)[b * prm.strideS + j] = acc;
+#pragma unroll 4
+            for (; k < prm.bands; k += C) acc = acc + base[k * prm.M];
         }
+        part[threadIdx.x] = acc;
+        __syncthreads();
+        if (y == 0 && valid) {
+            Acc tot = part[x];
+            for (int yy = 1; yy < C; ++yy) tot = tot + part[yy * R + x];
+            static_cast<Acc *>(prm.q)[b * prm.strideQ + i] = tot;
+        }
+        return;
     }
+    const int64_t T_ = prm.tiles, G = prm.grid, S = prm.stripes;
+    const int64_t g = (int64_t)blockIdx.x - q_blocks;  // b * bands + band
+    const int64_t b = g / prm.bands, band = g - b * prm.bands;
+    const int64_t c_lo = cta_of_tile(g * S, T_, G);
+    const int64_t c_hi = cta_of_tile(g * S + S - 1, T_, G);
+    if (c_lo == c_hi) return;  // written directly by the stream kernel
+    const int col = threadIdx.x;
+    const int64_t j = band * kBandCols + col;
+    if (j >= prm.N) return;
+    Acc acc = Acc(0);
+    for (int64_t cc = c_lo; cc <= c_hi; ++cc) {
+        const int64_t seg = g - cta_first_tile(cc, T_, G) / S;
+        const Acc v = sw[(cc * prm.max_seg + seg) * kBandCols + col];
+        acc = (cc == c_lo) ? v : acc + v;
+    }
+    static_cast<Acc *>(prm.s)[b * prm.strideS + j] = acc;
 }
 
 // Zero-fill of strided outputs (empty problems).

@@ -276,6 +276,31 @@ __host__ __device__ __forceinline__ int64_t cta_of_tile(int64_t t, int64_t T,
 // both the kernel (offsets) and the host (launch size).  TMA path: a
 // 1024-byte-aligned ring of STAGES tiles, the warp scratch for the s flush,
 // then the full/empty mbarriers.  Plain-load path: the scratch only.
+// Coordinates of a tile in band-major order, advanced one tile at a time so
+// that the per-tile loop does no 64-bit division.
+struct TileCursor {
+    int64_t g;       // global band index: b * bands + band
+    int64_t b;       // problem
+    int64_t band;    // band within the problem
+    int64_t stripe;  // stripe within the band
+    __device__ __forceinline__ void init(int64_t t, int64_t S, int64_t bands) {
+        g = t / S;
+        stripe = t - g * S;
+        b = g / bands;
+        band = g - b * bands;
+    }
+    __device__ __forceinline__ void advance(int64_t S, int64_t bands) {
+        if (++stripe == S) {
+            stripe = 0;
+            ++g;
+            if (++band == bands) {
+                band = 0;
+                ++b;
+            }
+        }
+    }
+};
+
 template <typename T, int W, int RPW, int STAGES, bool kTma>
 struct SmemLayout {
     using Acc = typename Traits<T>::Acc;
@@ -345,26 +370,30 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
                 const uint64_t pol = policy_evict_first();
                 bool ok = true;
                 int64_t issued = 0;
+                TileCursor cur;
+                cur.init(t0, S, prm.bands);
+                int stage = 0;
+                uint32_t phase = 0;  // parity of the ring pass, flips each pass
                 for (int64_t k = 0; k < ntiles; ++k) {
-                    const int stage = (int)(k % STAGES);
-                    const uint32_t round = (uint32_t)(k / STAGES);
-                    if (ok && round > 0)
-                        ok = mbar_wait_bounded(smem_u32(&empty_bar[stage]),
-                                               (round - 1) & 1u);
+                    // Before the second pass over the ring, wait until the
+                    // consumers released the previous tile in this stage.
+                    if (ok && k >= STAGES)
+                        ok = mbar_wait_bounded(smem_u32(&empty_bar[stage]), phase ^ 1u);
                     if (!ok) break;
-                    const int64_t t = t0 + k;
-                    const int64_t g = t / S;
-                    const int stripe = (int)(t - g * S);
-                    const int band = (int)(g % prm.bands);
-                    const int b = (int)(g / prm.bands);
                     const uint32_t fb = smem_u32(&full_bar[stage]);
                     mbar_arrive_expect_tx(fb, TILE_BYTES);
                     const uint32_t dst = smem_u32(ring + (size_t)stage * TILE_BYTES);
+                    const int x = (int)(cur.band * kBandCols), y = (int)(cur.stripe * BM);
                     if constexpr (kBatched3d)
-                        tma_load_3d(dst, &tmap, band * kBandCols, stripe * BM, b, fb, pol);
+                        tma_load_3d(dst, &tmap, x, y, (int)cur.b, fb, pol);
                     else
-                        tma_load_2d(dst, &tmap, band * kBandCols, stripe * BM, fb, pol);
+                        tma_load_2d(dst, &tmap, x, y, fb, pol);
                     issued = k + 1;
+                    cur.advance(S, prm.bands);
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
                 }
                 // Before the CTA exits, every copy it issued must have landed
                 // (bounded): the last min(STAGES, ntiles) issued stages.
@@ -396,14 +425,31 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
     int64_t seg_start_stripe = 0;
     bool ok = true;
 
+    TileCursor cur;
+    cur.init(t0, S, prm.bands);
+    // r for this warp's RPW rows of the next tile (lane i < RPW holds row
+    // row0 + i), loaded one tile ahead so its latency hides behind a tile.
+    T r_next = T(0);
+    {
+        const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
+        if (lane < RPW && row < prm.M) r_next = rg[cur.b * prm.strideR + row];
+    }
+    int stage = 0;
+    uint32_t phase = 0;
+
     for (int64_t k = 0; k < ntiles; ++k) {
-        const int64_t t = t0 + k;
-        const int64_t g = t / S;
-        const int64_t stripe = t - g * S;
-        const int64_t band = g % prm.bands;
-        const int64_t b = g / prm.bands;
+        const int64_t g = cur.g;
+        const int64_t stripe = cur.stripe;
+        const int64_t band = cur.band;
+        const int64_t b = cur.b;
         const int64_t col0 = band * kBandCols;
         const int64_t row0 = stripe * BM + (int64_t)warp * RPW;
+        const T rmine = r_next;
+        cur.advance(S, prm.bands);
+        if (k + 1 < ntiles) {
+            const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
+            r_next = (lane < RPW && row < prm.M) ? rg[cur.b * prm.strideR + row] : T(0);
+        }
 
         if (k == 0 || stripe == 0) {  // a new segment: this band's p
             seg_start_stripe = stripe;
@@ -417,19 +463,13 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
                 }
         }
 
-        // r for this warp's RPW rows (lane i < RPW holds row row0 + i).
-        T rmine = T(0);
-        if (lane < RPW && row0 + lane < prm.M) rmine = rg[b * prm.strideR + row0 + lane];
-
         Acc qp[RPW];
         Acc tacc[kLaneCols];
 #pragma unroll
         for (int e = 0; e < kLaneCols; ++e) tacc[e] = Acc(0);
 
-        const int stage = (int)(k % STAGES);
         if constexpr (kTma) {
-            if (ok) ok = mbar_wait_bounded(smem_u32(&full_bar[stage]),
-                                           (uint32_t)(k / STAGES) & 1u);
+            if (ok) ok = mbar_wait_bounded(smem_u32(&full_bar[stage]), phase);
         }
 #pragma unroll
         for (int i = 0; i < RPW; ++i) {
@@ -470,6 +510,10 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
         if constexpr (kTma) {
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&empty_bar[stage]));
+        }
+        if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
         }
 
         // q: complete band partial of each of this warp's rows.

@@ -57,7 +57,8 @@ typedef enum dualmv_status {
     DUALMV_ERR_ALLOC = 2,
     DUALMV_ERR_LAUNCH = 3,
     DUALMV_ERR_TIMEOUT = 4,
-    DUALMV_ERR_UNSUPPORTED = 5
+    DUALMV_ERR_UNSUPPORTED = 5,
+    DUALMV_ERR_TOO_LARGE = 6
 } dualmv_status;
 
 /* Opaque CUDA stream handle (the same pointer as cudaStream_t). */
@@ -101,6 +102,39 @@ dualmv_status dualmv_i32_strided_batched(
     const int32_t *p, int64_t strideP, const int32_t *r, int64_t strideR,
     int64_t *q, int64_t strideQ, int64_t *s, int64_t strideS, int64_t batch,
     dualmv_stream_t stream);
+
+/* ---- single problem without allocation --------------------------------
+ * The paper has no counterpart to this entry point; it exists for callers
+ * that cannot allocate device memory during the call: code inside a
+ * framework that owns every device allocation (a fixed memory budget or an
+ * allocator dualmv cannot see), real-time loops that must not enter an
+ * allocator, and hot streams that must not gain pool-growing calls.
+ *
+ * Same operation, arguments and results contract as dualmv_f32, but the
+ * scratch that holds partial sums between the two kernels is a fixed
+ * device array inside the library (dualmv_f32_noalloc_scratch_bytes(),
+ * 8 MiB), held by every GPU that loads the library until the process
+ * exits.  The call makes no cudaMalloc, cudaFree or pool allocation.
+ * The caller still passes A, p, r, q and s.
+ *
+ * Limit: the partial sums need about ceil(N / 256) * M * 4 bytes (none
+ * when N <= 256) plus under 1 MiB; a 16384 x 16384 matrix fits, a
+ * 32768 x 16384 one does not.  Larger problems return DUALMV_ERR_TOO_LARGE
+ * and enqueue nothing.
+ * Set-up: the first call on each device looks up the SM count and the
+ * device address of the array (cudaGetSymbolAddress) with that device
+ * current; make that first call before any stream capture.
+ * Sharing: every call on a device uses the same array, and each call fully
+ * rewrites the part it reads, so nothing carries over from one call to the
+ * next.  Calls that can overlap on the GPU (different streams without
+ * ordering between them) race on the array and give wrong results; order
+ * them on one stream or with events. */
+dualmv_status dualmv_f32_noalloc(int64_t M, int64_t N, const float *A,
+                                 int64_t lda, const float *p, const float *r,
+                                 float *q, float *s, dualmv_stream_t stream);
+
+/* Size in bytes of the fixed scratch array used by dualmv_f32_noalloc. */
+int64_t dualmv_f32_noalloc_scratch_bytes(void);
 
 /* ---- diagnostics and control ------------------------------------------ */
 

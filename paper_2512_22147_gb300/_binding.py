@@ -25,6 +25,7 @@ DUALMV_ERR_ALLOC = 2
 DUALMV_ERR_LAUNCH = 3
 DUALMV_ERR_TIMEOUT = 4
 DUALMV_ERR_UNSUPPORTED = 5
+DUALMV_ERR_TOO_LARGE = 6
 
 DUALMV_PATH_AUTO = 0
 DUALMV_PATH_TMA = 1
@@ -36,6 +37,7 @@ EXPORTED = (
     "dualmv_i32_strided_batched",
     "dualmv_status_string", "dualmv_last_cuda_error", "dualmv_device_fault",
     "dualmv_set_path", "dualmv_plan", "dualmv_record_kernel_events",
+    "dualmv_f32_noalloc", "dualmv_f32_noalloc_scratch_bytes",
 )
 
 
@@ -70,6 +72,9 @@ def _load() -> ctypes.CDLL:
         f.argtypes, f.restype = single, st
         f = getattr(lib, f"dualmv_{t}_strided_batched")
         f.argtypes, f.restype = batched, st
+    lib.dualmv_f32_noalloc.argtypes, lib.dualmv_f32_noalloc.restype = single, st
+    lib.dualmv_f32_noalloc_scratch_bytes.argtypes = []
+    lib.dualmv_f32_noalloc_scratch_bytes.restype = i64
     lib.dualmv_status_string.argtypes = [st]
     lib.dualmv_status_string.restype = ctypes.c_char_p
     lib.dualmv_last_cuda_error.argtypes = []
@@ -105,6 +110,16 @@ def dualmv_f64(M, N, A, lda, p, r, q, s, stream):
 
 def dualmv_i32(M, N, A, lda, p, r, q, s, stream):
     return _lib.dualmv_i32(M, N, A, lda, p, r, q, s, stream)
+
+
+def dualmv_f32_noalloc(M, N, A, lda, p, r, q, s, stream):
+    """dualmv_f32 without any device allocation: scratch is a fixed array
+    inside the library (see include/dualmv.h for who needs this and why)."""
+    return _lib.dualmv_f32_noalloc(M, N, A, lda, p, r, q, s, stream)
+
+
+def dualmv_f32_noalloc_scratch_bytes() -> int:
+    return _lib.dualmv_f32_noalloc_scratch_bytes()
 
 
 def dualmv_f32_strided_batched(M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS, batch, stream):

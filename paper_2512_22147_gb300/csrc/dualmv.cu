@@ -348,6 +348,98 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     return DUALMV_SUCCESS;
 }
 
+// ------------------------------------------------- no-allocation variant --
+//
+// Some callers cannot allocate device memory while they run dualmv: code
+// inside a framework that owns every device allocation (a fixed memory
+// budget, or a custom allocator that dualmv cannot see), real-time loops
+// that must not call into the allocator, and code that must not add
+// synchronising or pool-growing calls on a hot stream.  dualmv_f32_noalloc
+// serves them: its scratch (the band partials of q and segment partials of s
+// that the combine kernel reads) lives in this fixed device array, which
+// every GPU that loads the library holds until the process exits.
+constexpr int64_t kNoallocScratchBytes = 8ll << 20;  // 8 MiB
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
+
+struct NoallocDevice {
+    std::once_flag once;
+    cudaError_t error = cudaSuccess;
+    int sms = 0;
+    void *scratch = nullptr;  // device address of g_noalloc_scratch
+};
+NoallocDevice g_noalloc_dev[kMaxDevices];
+
+// Once per device, with that device current: the SM count and the device
+// address of the scratch array (in host code the array's name is only a
+// stand-in, never a device address).
+cudaError_t noalloc_setup(int dev, NoallocDevice **out) {
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    NoallocDevice &nd = g_noalloc_dev[dev];
+    std::call_once(nd.once, [&]() {
+        cudaError_t e = cudaDeviceGetAttribute(&nd.sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) { nd.error = e; return; }
+        void *ptr = nullptr;
+        e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+        if (e != cudaSuccess) { nd.error = e; return; }
+        nd.scratch = ptr;
+    });
+    *out = &nd;
+    return nd.error;
+}
+
+dualmv_status run_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,
+                              const float *p, const float *r, float *q, float *s,
+                              cudaStream_t stream) {
+    using T = float;
+    using Acc = float;
+    dualmv_status st = validate(M, N, A, lda, 0, p, 0, r, 0, q, 0, s, 0, 1);
+    if (st != DUALMV_SUCCESS) return st;
+    if (M == 0 || N == 0) {
+        cudaError_t e = zero_fill(q, M, M, 1, stream);
+        if (e == cudaSuccess) e = zero_fill(s, N, N, 1, stream);
+        return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
+    }
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e);
+    NoallocDevice *nd = nullptr;
+    e = noalloc_setup(dev, &nd);
+    if (e != cudaSuccess) return cuda_fail(e);
+
+    const int64_t es = sizeof(T);
+    bool tma = g_path != DUALMV_PATH_DIRECT &&
+               (reinterpret_cast<uintptr_t>(A) % 16 == 0) && ((lda * es) % 16 == 0) &&
+               M < INT32_MAX && N < INT32_MAX;
+    CUtensorMap map;
+    std::memset(&map, 0, sizeof map);
+    if (tma) tma = encode_a<T>(&map, A, M, N, lda, M * lda, 1, kWarps * kRpw4, false);
+    dualmv_plan_t pl;
+    st = make_plan(M, N, 1, es, sizeof(Acc),
+                   (int64_t)nd->sms * (tma ? 1 : kDirectCtasPerSm), tma, &pl);
+    if (st != DUALMV_SUCCESS) return st;
+    if (pl.workspace_bytes > kNoallocScratchBytes) return DUALMV_ERR_TOO_LARGE;
+
+    // Every scratch word the combine kernel reads is written earlier in the
+    // same call, so nothing needs clearing between calls.
+    Params prm;
+    prm.A = A; prm.lda = lda; prm.strideA = M * lda;
+    prm.p = p; prm.strideP = N;
+    prm.r = r; prm.strideR = M;
+    prm.q = q; prm.strideQ = M;
+    prm.s = s; prm.strideS = N;
+    prm.M = M; prm.N = N; prm.batch = 1;
+    prm.bands = pl.bands; prm.stripes = pl.stripes; prm.tiles = pl.tiles;
+    prm.grid = pl.grid; prm.max_seg = pl.max_segments;
+    const int64_t q_ws_bytes = pl.bands > 1 ? pl.bands * M * (int64_t)sizeof(Acc) : 0;
+    prm.q_ws = pl.bands > 1 ? nd->scratch : nullptr;
+    prm.s_ws = static_cast<unsigned char *>(nd->scratch) + ((q_ws_bytes + 255) / 256) * 256;
+
+    e = tma ? launch_stream<T, true, false>(map, prm, pl, dev, stream)
+            : launch_stream<T, false, false>(map, prm, pl, dev, stream);
+    if (e == cudaSuccess) e = launch_combine<Acc>(prm, stream);
+    return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
+}
+
 }  // namespace
 
 // ================================================================ C ABI ===
@@ -402,6 +494,14 @@ dualmv_status dualmv_i32_strided_batched(int64_t M, int64_t N, const int32_t *A,
                                  s, strideS, batch, reinterpret_cast<cudaStream_t>(stream));
 }
 
+dualmv_status dualmv_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,
+                                 const float *p, const float *r, float *q, float *s,
+                                 dualmv_stream_t stream) {
+    return run_f32_noalloc(M, N, A, lda, p, r, q, s, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int64_t dualmv_f32_noalloc_scratch_bytes(void) { return kNoallocScratchBytes; }
+
 const char *dualmv_status_string(dualmv_status status) {
     switch (status) {
     case DUALMV_SUCCESS: return "success";
@@ -410,6 +510,8 @@ const char *dualmv_status_string(dualmv_status status) {
     case DUALMV_ERR_LAUNCH: return "CUDA launch or runtime error";
     case DUALMV_ERR_TIMEOUT: return "a device-side bounded wait timed out";
     case DUALMV_ERR_UNSUPPORTED: return "unsupported configuration";
+    case DUALMV_ERR_TOO_LARGE:
+        return "problem needs more scratch than the no-allocation entry point holds";
     }
     return "unknown status";
 }

@@ -99,6 +99,27 @@ template <> CUtensorMapDataType tma_dtype<float>() { return CU_TENSOR_MAP_DATA_T
 template <> CUtensorMapDataType tma_dtype<double>() { return CU_TENSOR_MAP_DATA_TYPE_FLOAT64; }
 template <> CUtensorMapDataType tma_dtype<int32_t>() { return CU_TENSOR_MAP_DATA_TYPE_INT32; }
 
+// L2 promotion for the TMA loads of A: the largest of 256, 128 and 64 bytes
+// that divides the base address and every row (and problem) stride, else
+// none.  Each box row starts a whole number of bands (1 or 2 KiB) into its
+// matrix row, so with this choice no promoted chunk reaches into a
+// neighbouring band; a larger promotion on misaligned rows would make both
+// bands fetch the shared chunk, and the second fetch comes long after the
+// first has left L2.
+CUtensorMapL2promotion l2_promotion(uintptr_t base, int64_t row_bytes, int64_t batch_bytes,
+                                    bool three_d) {
+    const int64_t sizes[3] = {256, 128, 64};
+    const CUtensorMapL2promotion kinds[3] = {CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                             CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                                             CU_TENSOR_MAP_L2_PROMOTION_L2_64B};
+    for (int i = 0; i < 3; ++i) {
+        const int64_t s = sizes[i];
+        if (base % (uintptr_t)s == 0 && row_bytes % s == 0 && (!three_d || batch_bytes % s == 0))
+            return kinds[i];
+    }
+    return CU_TENSOR_MAP_L2_PROMOTION_NONE;
+}
+
 // Encodes A as a 2-D (N, M) or 3-D (N, M, batch) tiled tensor with a box of
 // kBandCols x tile_rows (x 1).  Columns >= N and rows >= M read as zero.
 template <typename T>
@@ -107,13 +128,15 @@ bool encode_a(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     const int64_t es = sizeof(T);
+    const CUtensorMapL2promotion promo =
+        l2_promotion(reinterpret_cast<uintptr_t>(A), lda * es, strideA * es, three_d);
     cuuint64_t dims[3] = {(cuuint64_t)N, (cuuint64_t)M, (cuuint64_t)batch};
     cuuint64_t strides[2] = {(cuuint64_t)(lda * es), (cuuint64_t)(strideA * es)};
     cuuint32_t box[3] = {(cuuint32_t)kBandCols, (cuuint32_t)tile_rows, 1u};
     cuuint32_t estr[3] = {1u, 1u, 1u};
     CUresult rc = fn(map, tma_dtype<T>(), three_d ? 3u : 2u, const_cast<T *>(A), dims,
                      strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                     CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_SWIZZLE_NONE, promo,
                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return rc == CUDA_SUCCESS;
 }

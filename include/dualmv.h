@@ -155,10 +155,20 @@ dualmv_status dualmv_device_fault(dualmv_stream_t stream);
 
 /* Which kernel streams A.  DUALMV_PATH_AUTO (default) uses the TMA pipeline
  * when the alignment rules above hold and the plain-load kernel otherwise;
- * the other values force one of them (FORCE_TMA falls back to plain loads
- * when the alignment rules do not hold).  Process-wide; meant for tests and
- * tuning.  Returns the previous setting, or -1 for an unknown value. */
-enum { DUALMV_PATH_AUTO = 0, DUALMV_PATH_TMA = 1, DUALMV_PATH_DIRECT = 2 };
+ * DUALMV_PATH_TMA and DUALMV_PATH_DIRECT force one of them (TMA falls back
+ * to plain loads when the alignment rules do not hold).  On the TMA path,
+ * fp64 products and sums run in double-float arithmetic on the FP32 pipes
+ * (GB300's FP64 pipe is far slower than its HBM), with native fp64 FMA for
+ * any rows holding values outside [2^-40, 2^40) (zero excepted);
+ * DUALMV_PATH_TMA_NATIVE_F64 makes the TMA path use native fp64 FMA for
+ * all of them.  Process-wide; meant for tests and tuning.  Returns the
+ * previous setting, or -1 for an unknown value. */
+enum {
+    DUALMV_PATH_AUTO = 0,
+    DUALMV_PATH_TMA = 1,
+    DUALMV_PATH_DIRECT = 2,
+    DUALMV_PATH_TMA_NATIVE_F64 = 3
+};
 int dualmv_set_path(int path);
 
 /* Instrumentation for benchmarks: the next dualmv call made by this thread

@@ -15,7 +15,7 @@ import importlib
 _BINDING_NAMES = {
     "DUALMV_ERR_ALLOC", "DUALMV_ERR_INVALID_VALUE", "DUALMV_ERR_LAUNCH",
     "DUALMV_ERR_TIMEOUT", "DUALMV_ERR_UNSUPPORTED", "DUALMV_ERR_TOO_LARGE", "DUALMV_PATH_AUTO",
-    "DUALMV_PATH_DIRECT", "DUALMV_PATH_TMA", "DUALMV_SUCCESS", "EXPORTED",
+    "DUALMV_PATH_DIRECT", "DUALMV_PATH_TMA", "DUALMV_PATH_TMA_NATIVE_F64", "DUALMV_SUCCESS", "EXPORTED",
     "LIBRARY_PATH", "DualmvError", "Plan", "dualmv_device_fault", "dualmv_f32",
     "dualmv_f32_strided_batched", "dualmv_f64", "dualmv_f64_strided_batched",
     "dualmv_i32", "dualmv_i32_strided_batched", "dualmv_last_cuda_error",

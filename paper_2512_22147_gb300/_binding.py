@@ -30,6 +30,7 @@ DUALMV_ERR_TOO_LARGE = 6
 DUALMV_PATH_AUTO = 0
 DUALMV_PATH_TMA = 1
 DUALMV_PATH_DIRECT = 2
+DUALMV_PATH_TMA_NATIVE_F64 = 3
 
 EXPORTED = (
     "dualmv_f32", "dualmv_f64", "dualmv_i32",

@@ -14,6 +14,7 @@
 #include <mutex>
 
 #include "dualmv_kernels.cuh"
+#include "dualmv_f64e.cuh"
 
 namespace {
 
@@ -21,12 +22,28 @@ using dmv::kBandCols;
 using dmv::Params;
 
 // Tile shape per element width: W consumer warps x RPW rows per warp, and
-// the ring depth.  Every tile is 32 KiB of A.
+// the ring depth.  Every tile of the generic kernel is 32 KiB of A.
 constexpr int kWarps = 8;
 constexpr int kRpw4 = 4;   // 4-byte elements: 32 rows x 1 KiB
 constexpr int kRpw8 = 2;   // 8-byte elements: 16 rows x 2 KiB
 constexpr int kStages = 6;
 constexpr int kDirectCtasPerSm = 4;
+// fp64 on the FP32 pipes (dualmv_f64e.cuh).
+#ifndef DUALMV_F64E_WARPS
+#define DUALMV_F64E_WARPS 7
+#endif
+#ifndef DUALMV_F64E_RPW
+#define DUALMV_F64E_RPW 4
+#endif
+#ifndef DUALMV_F64E_STAGES
+#define DUALMV_F64E_STAGES 3
+#endif
+constexpr int kF64eWarps = DUALMV_F64E_WARPS;
+constexpr int kF64eRpw = DUALMV_F64E_RPW;
+constexpr int kF64eStages = DUALMV_F64E_STAGES;
+
+// Which stream kernel a call uses.
+enum class Kind { kTma, kDirect, kF64e };
 
 thread_local int g_last_cuda_error = 0;
 thread_local cudaEvent_t g_kernel_ev_start = nullptr;
@@ -143,28 +160,47 @@ bool encode_a(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
 
 // ------------------------------------------------------------------ plan --
 
+// Warps, rows per warp and shared memory of each stream kernel.
+struct Geometry {
+    int64_t tile_rows;
+    int64_t smem;
+    int64_t threads;
+};
+
 template <typename T>
-int64_t smem_of(bool tma) {
+Geometry generic_geometry(bool tma) {
     constexpr int rpw = sizeof(T) == 4 ? kRpw4 : kRpw8;
-    return tma ? dmv::SmemLayout<T, kWarps, rpw, kStages, true>::kTotal
-               : dmv::SmemLayout<T, kWarps, rpw, kStages, false>::kTotal;
+    Geometry g;
+    g.tile_rows = kWarps * rpw;
+    g.smem = tma ? dmv::SmemLayout<T, kWarps, rpw, kStages, true>::kTotal
+                 : dmv::SmemLayout<T, kWarps, rpw, kStages, false>::kTotal;
+    g.threads = (kWarps + (tma ? 1 : 0)) * 32;
+    return g;
 }
 
-// Shared memory of the stream kernel for an element / accumulator width.
-int64_t smem_bytes_for(int64_t elem_bytes, int64_t acc_bytes, bool tma) {
-    if (elem_bytes == 8) return smem_of<double>(tma);
-    return acc_bytes == 8 ? smem_of<int32_t>(tma) : smem_of<float>(tma);
+Geometry geometry(int64_t elem_bytes, int64_t acc_bytes, Kind kind) {
+    if (kind == Kind::kF64e) {
+        Geometry g;
+        g.tile_rows = kF64eWarps * kF64eRpw;
+        g.smem = dmv::SmemLayout<double, kF64eWarps, kF64eRpw, kF64eStages, true>::kTotal;
+        g.threads = (kF64eWarps + 1) * 32;
+        return g;
+    }
+    const bool tma = kind == Kind::kTma;
+    if (elem_bytes == 8) return generic_geometry<double>(tma);
+    return acc_bytes == 8 ? generic_geometry<int32_t>(tma) : generic_geometry<float>(tma);
 }
 
 dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
-                        int64_t acc_bytes, int64_t ctas, bool tma, dualmv_plan_t *pl) {
+                        int64_t acc_bytes, int64_t ctas, Kind kind, dualmv_plan_t *pl) {
     if (M <= 0 || N <= 0 || batch <= 0 || ctas <= 0 || pl == nullptr)
         return DUALMV_ERR_INVALID_VALUE;
     if ((elem_bytes != 4 && elem_bytes != 8) || (acc_bytes != 4 && acc_bytes != 8) ||
         acc_bytes < elem_bytes)
         return DUALMV_ERR_INVALID_VALUE;
-    const int64_t rpw = elem_bytes == 4 ? kRpw4 : kRpw8;
-    const int64_t bm = kWarps * rpw;
+    if (kind == Kind::kF64e && elem_bytes != 8) return DUALMV_ERR_INVALID_VALUE;
+    const Geometry geo = geometry(elem_bytes, acc_bytes, kind);
+    const int64_t bm = geo.tile_rows;
     dualmv_plan_t p;
     std::memset(&p, 0, sizeof p);
     p.band_cols = kBandCols;
@@ -186,8 +222,8 @@ dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
     const int64_t q_ws = p.bands > 1 ? batch * p.bands * M * acc_bytes : 0;
     const int64_t s_ws = p.grid * p.max_segments * kBandCols * acc_bytes;
     p.workspace_bytes = ((q_ws + 255) / 256) * 256 + s_ws;
-    p.smem_bytes = smem_bytes_for(elem_bytes, acc_bytes, tma);
-    p.threads = (kWarps + (tma ? 1 : 0)) * 32;
+    p.smem_bytes = geo.smem;
+    p.threads = geo.threads;
     *pl = p;
     return DUALMV_SUCCESS;
 }
@@ -249,6 +285,22 @@ int combine_chunks(int64_t bands) {
     int c = 1;
     while (c < 32 && (int64_t)c * 8 < bands) c *= 2;
     return c;
+}
+
+template <bool k3d>
+cudaError_t launch_f64e(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
+                        int dev, cudaStream_t stream) {
+    auto kern = dmv::dualmv_stream_f64e_kernel<kF64eWarps, kF64eRpw, kF64eStages, k3d>;
+    static std::atomic<uint64_t> opted_in{0};
+    const uint64_t bit = 1ull << (dev & 63);
+    if (!(opted_in.load(std::memory_order_acquire) & bit)) {
+        cudaError_t e = cudaFuncSetAttribute(
+            kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem_bytes);
+        if (e != cudaSuccess) return e;
+        opted_in.fetch_or(bit, std::memory_order_acq_rel);
+    }
+    kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(map, prm);
+    return cudaGetLastError();
 }
 
 template <typename Acc>
@@ -323,14 +375,20 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                (reinterpret_cast<uintptr_t>(A) % 16 == 0) && ((lda * es) % 16 == 0) &&
                M < INT32_MAX && N < INT32_MAX && batch < INT32_MAX &&
                (!three_d || (strideA > 0 && (strideA * es) % 16 == 0));
+    // fp64 runs on the FP32 pipes unless native fp64 FMA is requested.
+    Kind kind = Kind::kDirect;
+    if (tma) kind = (es == 8 && g_path != DUALMV_PATH_TMA_NATIVE_F64) ? Kind::kF64e : Kind::kTma;
     CUtensorMap map;
     std::memset(&map, 0, sizeof map);
-    const int tile_rows = kWarps * (es == 4 ? kRpw4 : kRpw8);
-    if (tma) tma = encode_a<T>(&map, A, M, N, lda, strideA, batch, tile_rows, three_d);
+    if (tma) {
+        const int tile_rows = (int)geometry(es, sizeof(Acc), kind).tile_rows;
+        tma = encode_a<T>(&map, A, M, N, lda, strideA, batch, tile_rows, three_d);
+        if (!tma) kind = Kind::kDirect;
+    }
 
     dualmv_plan_t pl;
     st = make_plan(M, N, batch, es, sizeof(Acc),
-                   (int64_t)ds->sms * (tma ? 1 : kDirectCtasPerSm), tma, &pl);
+                   (int64_t)ds->sms * (tma ? 1 : kDirectCtasPerSm), kind, &pl);
     if (st != DUALMV_SUCCESS) return st;
 
     void *ws = nullptr;
@@ -356,7 +414,10 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     g_kernel_ev_start = g_kernel_ev_stop = nullptr;
     e = ev_start ? cudaEventRecord(ev_start, stream) : cudaSuccess;
     if (e == cudaSuccess) {
-        if (tma) {
+        if (kind == Kind::kF64e) {
+            e = three_d ? launch_f64e<true>(map, prm, pl, dev, stream)
+                        : launch_f64e<false>(map, prm, pl, dev, stream);
+        } else if (kind == Kind::kTma) {
             e = three_d ? launch_stream<T, true, true>(map, prm, pl, dev, stream)
                         : launch_stream<T, true, false>(map, prm, pl, dev, stream);
         } else {
@@ -438,7 +499,8 @@ dualmv_status run_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,
     if (tma) tma = encode_a<T>(&map, A, M, N, lda, M * lda, 1, kWarps * kRpw4, false);
     dualmv_plan_t pl;
     st = make_plan(M, N, 1, es, sizeof(Acc),
-                   (int64_t)nd->sms * (tma ? 1 : kDirectCtasPerSm), tma, &pl);
+                   (int64_t)nd->sms * (tma ? 1 : kDirectCtasPerSm),
+                   tma ? Kind::kTma : Kind::kDirect, &pl);
     if (st != DUALMV_SUCCESS) return st;
     if (pl.workspace_bytes > kNoallocScratchBytes) return DUALMV_ERR_TOO_LARGE;
 
@@ -561,7 +623,8 @@ void dualmv_record_kernel_events(void *start, void *stop) {
 }
 
 int dualmv_set_path(int path) {
-    if (path != DUALMV_PATH_AUTO && path != DUALMV_PATH_TMA && path != DUALMV_PATH_DIRECT)
+    if (path != DUALMV_PATH_AUTO && path != DUALMV_PATH_TMA && path != DUALMV_PATH_DIRECT &&
+        path != DUALMV_PATH_TMA_NATIVE_F64)
         return -1;
     const int old = g_path;
     g_path = path;
@@ -570,7 +633,8 @@ int dualmv_set_path(int path) {
 
 dualmv_status dualmv_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
                           int64_t acc_bytes, int64_t num_sms, dualmv_plan_t *out) {
-    return make_plan(M, N, batch, elem_bytes, acc_bytes, num_sms, true, out);
+    return make_plan(M, N, batch, elem_bytes, acc_bytes, num_sms,
+                     elem_bytes == 8 ? Kind::kF64e : Kind::kTma, out);
 }
 
 }  // extern "C"

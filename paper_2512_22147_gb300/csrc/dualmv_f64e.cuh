@@ -1,0 +1,458 @@
+// fp64 dual matrix-vector product (BICG, Tables 1-2) on the FP32 pipes.
+//
+// GB300's FP64 pipe retires about 1.6 DFMA per clock per SM, and float <->
+// double conversions run on the same narrow pipe, so two DFMAs per element
+// of A cap a native fp64 kernel near a quarter of HBM bandwidth.  This
+// kernel streams A exactly like the generic one (same TMA ring, tile
+// schedule, workspace layout and combine kernel) but forms both products in
+// "double-float" arithmetic: each double is split, with integer bit
+// operations only, into an unevaluated sum of two floats, and products and
+// sums use error-free FP32 transformations.
+//
+//   split   a = a_hi + a_lo + d, a_hi the top 24 significant bits of a, a_lo
+//           the next 23, |d| < 2^-46 |a| (truncation, same sign as a).
+//   product a*x ~ a_hi x_hi + (err(a_hi x_hi) + a_hi x_lo + a_lo x_hi); the
+//           first term and its rounding error come from FMUL and FFMA
+//           exactly; the dropped a_lo x_lo is below 2^-46 |a x|.
+//   sum     Knuth's TwoSum on the high parts, the low parts and the TwoSum
+//           errors summed in a second float ("sloppy" double-float
+//           accumulation), in three levels: the RPW rows of a tile (or the 8
+//           columns of a lane), groups of kGroupTiles tiles, then fp64 for
+//           the segment.  Every level sums few terms, so the bound stays
+//           near (terms per level) * 2^-47 * sum |a x|, far below 1e-12.
+//
+// Range.  The split and the FP32 arithmetic are exact only while every
+// |a|, |p_j|, |r_i| lies in [2^-40, 2^40) or is zero (products then stay
+// inside FP32's normal range).  Each element costs two integer ops of range
+// bookkeeping; a warp whose rows of a tile hold anything else re-checks
+// them exactly (zeros are fine) and, if a value really is out of range,
+// recomputes those rows with native fp64 FMA.  Results are the same
+// arithmetic on every call, so they are deterministic.
+#pragma once
+
+#include "dualmv_kernels.cuh"
+
+namespace dmv {
+
+// Bits of |a| as the high word of a double: 2^-40 has biased exponent 983,
+// 2^40 has 1063.
+constexpr uint32_t kF64eLoBits = 983u << 20;
+constexpr uint32_t kF64eSpanBits = (1063u - 983u) << 20;
+
+struct DF {
+    float s;  // high part
+    float c;  // low part (sum of everything below s)
+};
+
+// Split a double into hi + lo floats with integer operations only.  Zero
+// (either sign) gives two zeros; values outside [2^-40, 2^40) give garbage
+// and must be caught by the range check.
+__device__ __forceinline__ void split_f64(double a, float &hi, float &lo, uint32_t &habs) {
+    const uint32_t h = (uint32_t)__double2hiint(a);
+    const uint32_t l = (uint32_t)__double2loint(a);
+    habs = h & 0x7FFFFFFFu;
+    // Rebias the exponent from 1023 to 127 (896 << 20); zero keeps zero.
+    const uint32_t t = h - min(habs, 896u << 20);
+    // (t << 3) | (l >> 29): exponent and top 23 mantissa bits of a float.
+    const uint32_t hb = __funnelshift_l(l, t, 3);
+    const uint32_t hi_bits = (hb & 0x7FFFFFFFu) | (h & 0x80000000u);
+    hi = __uint_as_float(hi_bits);
+    // lo = 0.m28..m6 * 2^(e-23): a float 1.m28..m6 * 2^(e-23) minus 2^(e-23).
+    const uint32_t e_lo = (hi_bits & 0xFF800000u) - (23u << 23);
+    lo = __fsub_rn(__uint_as_float(e_lo | ((l >> 6) & 0x7FFFFFu)), __uint_as_float(e_lo));
+}
+
+// Exact range test: |a| in [2^-40, 2^40) or a == 0.
+__device__ __forceinline__ bool f64e_in_range(double a) {
+    const uint32_t h = (uint32_t)__double2hiint(a), l = (uint32_t)__double2loint(a);
+    const uint32_t habs = h & 0x7FFFFFFFu;
+    return (habs - kF64eLoBits) < kF64eSpanBits || (habs | l) == 0u;
+}
+
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
+    s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+
+// a * x as (p, q) with p + q within 2^-46 |a x| of the exact product.
+__device__ __forceinline__ void df_prod(float ah, float al, float xh, float xl, float &p,
+                                        float &q) {
+    p = __fmul_rn(ah, xh);
+    q = __fmaf_rn(ah, xh, -p);  // exact rounding error of p
+    q = __fmaf_rn(ah, xl, q);
+    q = __fmaf_rn(al, xh, q);
+}
+
+// acc += (p, q)
+__device__ __forceinline__ void df_acc(DF &acc, float p, float q) {
+    float s, e;
+    two_sum(acc.s, p, s, e);
+    acc.s = s;
+    acc.c = __fadd_rn(acc.c, __fadd_rn(e, q));
+}
+
+__device__ __forceinline__ DF df_add(DF x, DF y) {
+    DF r;
+    float e;
+    two_sum(x.s, y.s, r.s, e);
+    r.c = __fadd_rn(__fadd_rn(x.c, y.c), e);
+    return r;
+}
+
+__device__ __forceinline__ double df_to_double(DF x) {
+    return __dadd_rn((double)x.s, (double)x.c);
+}
+
+// Reduce-scatter butterfly (as warp_rows_reduce) on double-float values,
+// written on the two float components so that every select stays in
+// registers.
+template <int RPW>
+__device__ __forceinline__ void warp_rows_reduce_df(DF (&v)[RPW], int lane) {
+    int off = 16;
+#pragma unroll
+    for (int h = RPW / 2; h >= 1; h /= 2) {
+        const bool upper = (lane & off) != 0;
+#pragma unroll
+        for (int k = 0; k < h; ++k) {
+            const float send_s = upper ? v[k].s : v[k + h].s;
+            const float send_c = upper ? v[k].c : v[k + h].c;
+            DF keep;
+            keep.s = upper ? v[k + h].s : v[k].s;
+            keep.c = upper ? v[k + h].c : v[k].c;
+            DF recv;
+            recv.s = __shfl_xor_sync(0xffffffffu, send_s, off);
+            recv.c = __shfl_xor_sync(0xffffffffu, send_c, off);
+            v[k] = df_add(keep, recv);
+        }
+        off >>= 1;
+    }
+#pragma unroll
+    for (; off >= 1; off >>= 1) {
+        DF recv;
+        recv.s = __shfl_xor_sync(0xffffffffu, v[0].s, off);
+        recv.c = __shfl_xor_sync(0xffffffffu, v[0].c, off);
+        v[0] = df_add(v[0], recv);
+    }
+}
+
+// ---------------------------------------------------------------- kernel --
+//
+// W consumer warps x RPW rows per warp per tile; lane l holds columns
+// 2l, 2l+1 (+64, +128, +192) of the 256-column band (four double2 vectors).
+template <int W, int RPW, int STAGES, bool kBatched3d>
+__global__ void __launch_bounds__((W + 1) * 32, 1)
+dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
+    using T = double;
+    using Acc = double;
+    using Vec = double2;
+    constexpr int VE = 2;
+    constexpr int VPL = kLaneCols / VE;  // 4 vectors per lane per row
+    constexpr int BM = W * RPW;
+    constexpr int ROW_BYTES = kBandCols * (int)sizeof(T);
+    constexpr int TILE_BYTES = BM * ROW_BYTES;
+    using L = SmemLayout<T, W, RPW, STAGES, true>;
+    static_assert(L::kTileBytes == TILE_BYTES, "tile size mismatch");
+
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + (L::kAlign - 1)) &
+        ~uintptr_t(L::kAlign - 1));
+    unsigned char *ring = smem;
+    Acc *scratch = reinterpret_cast<Acc *>(smem + L::kRing);
+    uint64_t *full_bar = reinterpret_cast<uint64_t *>(smem + L::kRing + L::kScratch);
+    uint64_t *empty_bar = full_bar + STAGES;
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t T_ = prm.tiles, G = prm.grid, S = prm.stripes;
+    const int64_t c = blockIdx.x;
+    const int64_t t0 = cta_first_tile(c, T_, G);
+    const int64_t t1 = cta_first_tile(c + 1, T_, G);
+    const int64_t ntiles = t1 - t0;
+    const int64_t g_first = t0 / S;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < STAGES; ++i) {
+            mbar_init(smem_u32(&full_bar[i]), 1);
+            mbar_init(smem_u32(&empty_bar[i]), W);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    pdl_launch_dependents();
+
+    // ------------------------------------------------------ producer ----
+    if (warp == W) {
+        if (lane == 0) {
+            const uint64_t pol = policy_evict_first();
+            bool ok = true;
+            int64_t issued = 0;
+            TileCursor cur;
+            cur.init(t0, S, prm.bands);
+            int stage = 0;
+            uint32_t phase = 0;
+            for (int64_t k = 0; k < ntiles; ++k) {
+                if (ok && k >= STAGES)
+                    ok = mbar_wait_bounded(smem_u32(&empty_bar[stage]), phase ^ 1u);
+                if (!ok) break;
+                const uint32_t fb = smem_u32(&full_bar[stage]);
+                mbar_arrive_expect_tx(fb, TILE_BYTES);
+                const uint32_t dst = smem_u32(ring + (size_t)stage * TILE_BYTES);
+                const int x = (int)(cur.band * kBandCols), y = (int)(cur.stripe * BM);
+                if constexpr (kBatched3d)
+                    tma_load_3d(dst, &tmap, x, y, (int)cur.b, fb, pol);
+                else
+                    tma_load_2d(dst, &tmap, x, y, fb, pol);
+                issued = k + 1;
+                cur.advance(S, prm.bands);
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            for (int64_t k = issued > STAGES ? issued - STAGES : 0; k < issued; ++k) {
+                const int st = (int)(k % STAGES);
+                mbar_wait_bounded(smem_u32(&full_bar[st]), (uint32_t)(k / STAGES) & 1u);
+            }
+        }
+        return;
+    }
+
+    // ----------------------------------------------------- consumers ----
+    const T *__restrict__ pg = static_cast<const T *>(prm.p);
+    const T *__restrict__ rg = static_cast<const T *>(prm.r);
+    const int nthreads_c = W * 32;
+
+    float ph[kLaneCols], pl[kLaneCols];  // split p of this lane's columns
+    bool p_bad = false;                  // some p of this lane out of range
+    DF grp[kLaneCols];                   // group sums of s (double-float)
+    // Segment sums of s (fp64) live in this warp's row of the flush scratch;
+    // each lane owns its 8 columns there, so no synchronisation is needed
+    // until the segment flush.
+    Acc *segp = scratch + warp * kBandCols;
+#pragma unroll
+    for (int e = 0; e < kLaneCols; ++e) {
+        ph[e] = pl[e] = 0.f;
+        grp[e].s = grp[e].c = 0.f;
+    }
+#pragma unroll
+    for (int v = 0; v < VPL; ++v)
+#pragma unroll
+        for (int e = 0; e < VE; ++e) segp[lane_col<T>(v, lane, e)] = 0.0;
+    int ngrp = 0;
+    int64_t seg_start_stripe = 0;
+    bool ok = true;
+
+    TileCursor cur;
+    cur.init(t0, S, prm.bands);
+    T r_next = T(0);
+    {
+        const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
+        if (lane < RPW && row < prm.M) r_next = rg[cur.b * prm.strideR + row];
+    }
+    int stage = 0;
+    uint32_t phase = 0;
+
+    for (int64_t k = 0; k < ntiles; ++k) {
+        const int64_t g = cur.g;
+        const int64_t stripe = cur.stripe;
+        const int64_t band = cur.band;
+        const int64_t b = cur.b;
+        const int64_t col0 = band * kBandCols;
+        const int64_t row0 = stripe * BM + (int64_t)warp * RPW;
+        const T rmine = r_next;
+        cur.advance(S, prm.bands);
+        if (k + 1 < ntiles) {
+            const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
+            r_next = (lane < RPW && row < prm.M) ? rg[cur.b * prm.strideR + row] : T(0);
+        }
+
+        if (k == 0 || stripe == 0) {  // new segment: split this band's p
+            seg_start_stripe = stripe;
+            const T *pb = pg + b * prm.strideP;
+            p_bad = false;
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) {
+                    const int64_t col = col0 + lane_col<T>(v, lane, e);
+                    const T pv = col < prm.N ? pb[col] : T(0);
+                    uint32_t habs;
+                    split_f64(pv, ph[v * VE + e], pl[v * VE + e], habs);
+                    p_bad |= !f64e_in_range(pv);
+                }
+        }
+        // r of this warp's rows, split by its owner lane.
+        float rh_mine, rl_mine;
+        uint32_t r_habs;
+        split_f64(rmine, rh_mine, rl_mine, r_habs);
+        const bool r_bad = !f64e_in_range(rmine);
+
+        if (ok) ok = mbar_wait_bounded(smem_u32(&full_bar[stage]), phase);
+        const Vec *tile = reinterpret_cast<const Vec *>(ring + (size_t)stage * TILE_BYTES);
+
+        // Fast path: double-float arithmetic with a cheap range bound.
+        DF q[RPW];
+        DF tacc[kLaneCols];
+        uint32_t span = 0;  // max over elements of (|a| bits - 2^-40 bits)
+#pragma unroll
+        for (int i = 0; i < RPW; ++i) {
+            const Vec *rowp = tile + (size_t)(warp * RPW + i) * (ROW_BYTES / 16);
+            Vec a[VPL];
+#pragma unroll
+            for (int v = 0; v < VPL; ++v) a[v] = rowp[v * 32 + lane];
+            const float rh = __shfl_sync(0xffffffffu, rh_mine, i);
+            const float rl = __shfl_sync(0xffffffffu, rl_mine, i);
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) {
+                    const int ce = v * VE + e;
+                    float ah, al;
+                    uint32_t habs;
+                    split_f64(vget(a[v], e), ah, al, habs);
+                    span = max(span, habs - kF64eLoBits);
+                    float p0, p1;
+                    df_prod(ah, al, rh, rl, p0, p1);
+                    if (i == 0) {
+                        tacc[ce].s = p0;
+                        tacc[ce].c = p1;
+                    } else {
+                        df_acc(tacc[ce], p0, p1);
+                    }
+                    df_prod(ah, al, ph[ce], pl[ce], p0, p1);
+                    if (ce == 0) {
+                        q[i].s = p0;
+                        q[i].c = p1;
+                    } else {
+                        df_acc(q[i], p0, p1);
+                    }
+                }
+        }
+        // Anything suspicious in this warp's rows (zeros included)?
+        const bool rows_r_bad = __any_sync(0xffffffffu, lane < RPW && r_bad);
+        bool need_fp64 = rows_r_bad || __any_sync(0xffffffffu, p_bad);
+        if (!need_fp64 && __any_sync(0xffffffffu, span >= kF64eSpanBits)) {
+            // Exact re-check: zeros are fine, anything else out of range is not.
+            bool bad = false;
+#pragma unroll
+            for (int i = 0; i < RPW; ++i) {
+                const Vec *rowp = tile + (size_t)(warp * RPW + i) * (ROW_BYTES / 16);
+#pragma unroll
+                for (int v = 0; v < VPL; ++v) {
+                    const Vec av = rowp[v * 32 + lane];
+                    bad |= !f64e_in_range(av.x) || !f64e_in_range(av.y);
+                }
+            }
+            need_fp64 = __any_sync(0xffffffffu, bad);
+        }
+
+        if (!need_fp64) {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[stage]));
+            warp_rows_reduce_df<RPW>(q, lane);
+            if (butterfly_writer<RPW>(lane)) {
+                const int64_t row = row0 + butterfly_row<RPW>(lane);
+                if (row < prm.M) {
+                    const double qv = df_to_double(q[0]);
+                    if (prm.bands == 1)
+                        static_cast<Acc *>(prm.q)[b * prm.strideQ + row] = qv;
+                    else
+                        static_cast<Acc *>(prm.q_ws)[(b * prm.bands + band) * prm.M + row] = qv;
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < kLaneCols; ++e) grp[e] = df_add(grp[e], tacc[e]);
+        } else {
+            // Out-of-range values in these rows: native fp64 for them.
+            double pd[kLaneCols];
+            const T *pb = pg + b * prm.strideP;
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) {
+                    const int64_t col = col0 + lane_col<T>(v, lane, e);
+                    pd[v * VE + e] = col < prm.N ? pb[col] : 0.0;
+                }
+            double qd[RPW];
+            double td[kLaneCols];
+#pragma unroll
+            for (int e = 0; e < kLaneCols; ++e) td[e] = 0.0;
+#pragma unroll
+            for (int i = 0; i < RPW; ++i) {
+                const Vec *rowp = tile + (size_t)(warp * RPW + i) * (ROW_BYTES / 16);
+                const double ri = __shfl_sync(0xffffffffu, rmine, i);
+                double dot = 0.0;
+#pragma unroll
+                for (int v = 0; v < VPL; ++v) {
+                    const Vec av = rowp[v * 32 + lane];
+#pragma unroll
+                    for (int e = 0; e < VE; ++e) {
+                        const double x = vget(av, e);
+                        dot = fma(x, pd[v * VE + e], dot);
+                        td[v * VE + e] = fma(x, ri, td[v * VE + e]);
+                    }
+                }
+                qd[i] = dot;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[stage]));
+            warp_rows_reduce<RPW>(qd, lane);
+            if (butterfly_writer<RPW>(lane)) {
+                const int64_t row = row0 + butterfly_row<RPW>(lane);
+                if (row < prm.M) {
+                    if (prm.bands == 1)
+                        static_cast<Acc *>(prm.q)[b * prm.strideQ + row] = qd[0];
+                    else
+                        static_cast<Acc *>(prm.q_ws)[(b * prm.bands + band) * prm.M + row] =
+                            qd[0];
+                }
+            }
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) segp[lane_col<T>(v, lane, e)] += td[v * VE + e];
+        }
+        if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+        }
+
+        const bool seg_end = (stripe == S - 1 || k == ntiles - 1);
+        if (++ngrp == kGroupTiles || seg_end) {
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) {
+                    segp[lane_col<T>(v, lane, e)] += df_to_double(grp[v * VE + e]);
+                    grp[v * VE + e].s = grp[v * VE + e].c = 0.f;
+                }
+            ngrp = 0;
+        }
+
+        if (seg_end) {  // segment end: flush s
+            named_barrier(1, nthreads_c);
+            const bool whole_band = (seg_start_stripe == 0 && stripe == S - 1);
+            for (int col = threadIdx.x; col < kBandCols; col += nthreads_c) {
+                Acc acc = scratch[col];
+#pragma unroll
+                for (int w = 1; w < W; ++w) acc = acc + scratch[w * kBandCols + col];
+                if (whole_band) {
+                    if (col0 + col < prm.N)
+                        static_cast<Acc *>(prm.s)[b * prm.strideS + col0 + col] = acc;
+                } else {
+                    static_cast<Acc *>(prm.s_ws)[((c * prm.max_seg) + (g - g_first)) *
+                                                     kBandCols + col] = acc;
+                }
+            }
+            named_barrier(1, nthreads_c);
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) segp[lane_col<T>(v, lane, e)] = 0.0;
+        }
+    }
+}
+
+}  // namespace dmv

@@ -188,7 +188,7 @@ __device__ __forceinline__ unsigned long long global_ns() {
 
 // Slow path of mbar_wait_bounded: keeps polling for at most kWaitTimeoutNs,
 // then sets the device fault word and returns false.
-__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity) {
     const unsigned long long t0 = global_ns();
     for (;;) {
         for (int i = 0; i < 64; ++i)

@@ -155,9 +155,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     static_assert(L::kTileBytes == TILE_BYTES, "tile size mismatch");
 
     extern __shared__ unsigned char smem_raw[];
-    unsigned char *smem = reinterpret_cast<unsigned char *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + (L::kAlign - 1)) &
-        ~uintptr_t(L::kAlign - 1));
+    unsigned char *smem = smem_raw + shared_align_pad<L::kAlign>(smem_raw);
     unsigned char *ring = smem;
     Acc *scratch = reinterpret_cast<Acc *>(smem + L::kRing);
     uint64_t *full_bar = reinterpret_cast<uint64_t *>(smem + L::kRing + L::kScratch);
@@ -304,6 +302,8 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             for (int v = 0; v < VPL; ++v) a[v] = rowp[v * 32 + lane];
             const float rh = __shfl_sync(0xffffffffu, rh_mine, i);
             const float rl = __shfl_sync(0xffffffffu, rl_mine, i);
+            // Row products with p, summed pairwise (depth 3, not a chain of 7).
+            DF qp[kLaneCols];
 #pragma unroll
             for (int v = 0; v < VPL; ++v)
 #pragma unroll
@@ -321,14 +321,10 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                     } else {
                         df_acc(tacc[ce], p0, p1);
                     }
-                    df_prod(ah, al, ph[ce], pl[ce], p0, p1);
-                    if (ce == 0) {
-                        q[i].s = p0;
-                        q[i].c = p1;
-                    } else {
-                        df_acc(q[i], p0, p1);
-                    }
+                    df_prod(ah, al, ph[ce], pl[ce], qp[ce].s, qp[ce].c);
                 }
+            q[i] = df_add(df_add(df_add(qp[0], qp[1]), df_add(qp[2], qp[3])),
+                          df_add(df_add(qp[4], qp[5]), df_add(qp[6], qp[7])));
         }
         // Anything suspicious in this warp's rows (zeros included)?
         const bool rows_r_bad = __any_sync(0xffffffffu, lane < RPW && r_bad);

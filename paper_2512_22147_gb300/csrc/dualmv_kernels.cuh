@@ -148,6 +148,15 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// Bytes to skip so that the dynamic shared memory base is kAlign-aligned.
+// Callers offset the __shared__ array itself by this amount (pointer
+// arithmetic keeps the shared address space visible to the compiler, so
+// tile reads stay shared-memory loads rather than generic ones).
+template <int kAlign>
+__device__ __forceinline__ uint32_t shared_align_pad(const void *base) {
+    return (uint32_t)(kAlign - (smem_u32(base) & (kAlign - 1))) & (uint32_t)(kAlign - 1);
+}
+
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count)
                  : "memory");
@@ -332,9 +341,7 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
     static_assert(L::kTileBytes == TILE_BYTES, "tile size mismatch");
 
     extern __shared__ unsigned char smem_raw[];
-    unsigned char *smem = reinterpret_cast<unsigned char *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + (L::kAlign - 1)) &
-        ~uintptr_t(L::kAlign - 1));
+    unsigned char *smem = smem_raw + shared_align_pad<L::kAlign>(smem_raw);
     unsigned char *ring = smem;
     Acc *scratch = reinterpret_cast<Acc *>(smem + L::kRing);
     uint64_t *full_bar = reinterpret_cast<uint64_t *>(smem + L::kRing + L::kScratch);

@@ -9,11 +9,15 @@
 // operations only, into an unevaluated sum of two floats, and products and
 // sums use error-free FP32 transformations.
 //
-//   split   a = a_hi + a_lo + d, a_hi the top 24 significant bits of a, a_lo
-//           the next 23, |d| < 2^-46 |a| (truncation, same sign as a).
+//   split   a = a_hi + a_lo + d, a_hi the top 21 significant bits of a, a_lo
+//           the remaining 32 rounded to 24, |d| <= 2^-45 |a|.
 //   product a*x ~ a_hi x_hi + (err(a_hi x_hi) + a_hi x_lo + a_lo x_hi); the
 //           first term and its rounding error come from FMUL and FFMA
-//           exactly; the dropped a_lo x_lo is below 2^-46 |a x|.
+//           exactly; the dropped a_lo x_lo is below 2^-44 |a x|.
+//   native  two of each lane's eight columns (kNativeCols) take their
+//           column sums from native fp64 FMA instead: GB300's FP64 pipe is
+//           otherwise idle here, and this moves a quarter of the s work off
+//           the FP32 pipes at about a third of the FP64 pipe's rate.
 //   sum     Knuth's TwoSum on the high parts, the low parts and the TwoSum
 //           errors summed in a second float ("sloppy" double-float
 //           accumulation), in three levels: the RPW rows of a tile (or the 8
@@ -34,6 +38,10 @@
 
 namespace dmv {
 
+#ifndef DUALMV_F64E_NATIVE_COLS
+#define DUALMV_F64E_NATIVE_COLS 2
+#endif
+
 // Bits of |a| as the high word of a double: 2^-40 has biased exponent 983,
 // 2^40 has 1063.
 constexpr uint32_t kF64eLoBits = 983u << 20;
@@ -44,22 +52,23 @@ struct DF {
     float c;  // low part (sum of everything below s)
 };
 
-// Split a double into hi + lo floats with integer operations only.  Zero
-// (either sign) gives two zeros; values outside [2^-40, 2^40) give garbage
-// and must be caught by the range check.
+// Split a double into hi + lo floats without touching the FP64 pipe.
+// a_hi keeps the sign, exponent and top 20 mantissa bits (the double's high
+// word, rebiased); a_lo is the low word converted to float (rounded to 24 of
+// its 32 bits) and scaled by 2^(e-52).  |a - a_hi - a_lo| <= 2^-45 |a|.
+// Zero (either sign) gives two zeros; values outside [2^-40, 2^40) give
+// garbage and must be caught by the range check.
 __device__ __forceinline__ void split_f64(double a, float &hi, float &lo, uint32_t &habs) {
     const uint32_t h = (uint32_t)__double2hiint(a);
     const uint32_t l = (uint32_t)__double2loint(a);
     habs = h & 0x7FFFFFFFu;
     // Rebias the exponent from 1023 to 127 (896 << 20); zero keeps zero.
     const uint32_t t = h - min(habs, 896u << 20);
-    // (t << 3) | (l >> 29): exponent and top 23 mantissa bits of a float.
-    const uint32_t hb = __funnelshift_l(l, t, 3);
-    const uint32_t hi_bits = (hb & 0x7FFFFFFFu) | (h & 0x80000000u);
+    const uint32_t hi_bits = ((t << 3) & 0x7FFFFFFFu) | (h & 0x80000000u);
     hi = __uint_as_float(hi_bits);
-    // lo = 0.m28..m6 * 2^(e-23): a float 1.m28..m6 * 2^(e-23) minus 2^(e-23).
-    const uint32_t e_lo = (hi_bits & 0xFF800000u) - (23u << 23);
-    lo = __fsub_rn(__uint_as_float(e_lo | ((l >> 6) & 0x7FFFFFu)), __uint_as_float(e_lo));
+    // 2^(e-52) with the sign of a.
+    const float scale = __uint_as_float((hi_bits & 0xFF800000u) - (52u << 23));
+    lo = __fmul_rn(__uint2float_rn(l), scale);
 }
 
 // Exact range test: |a| in [2^-40, 2^40) or a == 0.
@@ -222,6 +231,12 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     const T *__restrict__ rg = static_cast<const T *>(prm.r);
     const int nthreads_c = W * 32;
 
+    // Lane columns kLaneCols - kNativeCols .. kLaneCols - 1 sum s in fp64.
+    constexpr int kNativeCols = DUALMV_F64E_NATIVE_COLS;
+    constexpr int kFirstNative = kLaneCols - kNativeCols;
+    double snat[kNativeCols > 0 ? kNativeCols : 1];  // fp64 segment sums of s
+#pragma unroll
+    for (int j = 0; j < kNativeCols; ++j) snat[j] = 0.0;
     float ph[kLaneCols], pl[kLaneCols];  // split p of this lane's columns
     bool p_bad = false;                  // some p of this lane out of range
     DF grp[kLaneCols];                   // group sums of s (double-float)
@@ -293,6 +308,9 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         // Fast path: double-float arithmetic with a cheap range bound.
         DF q[RPW];
         DF tacc[kLaneCols];
+        double tnat[kNativeCols > 0 ? kNativeCols : 1];
+#pragma unroll
+        for (int j = 0; j < kNativeCols; ++j) tnat[j] = 0.0;
         uint32_t span = 0;  // max over elements of (|a| bits - 2^-40 bits)
 #pragma unroll
         for (int i = 0; i < RPW; ++i) {
@@ -302,6 +320,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             for (int v = 0; v < VPL; ++v) a[v] = rowp[v * 32 + lane];
             const float rh = __shfl_sync(0xffffffffu, rh_mine, i);
             const float rl = __shfl_sync(0xffffffffu, rl_mine, i);
+            const double rd = __shfl_sync(0xffffffffu, rmine, i);
             // Row products with p, summed pairwise (depth 3, not a chain of 7).
             DF qp[kLaneCols];
 #pragma unroll
@@ -313,13 +332,18 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                     uint32_t habs;
                     split_f64(vget(a[v], e), ah, al, habs);
                     span = max(span, habs - kF64eLoBits);
-                    float p0, p1;
-                    df_prod(ah, al, rh, rl, p0, p1);
-                    if (i == 0) {
-                        tacc[ce].s = p0;
-                        tacc[ce].c = p1;
+                    if (ce < kFirstNative) {
+                        float p0, p1;
+                        df_prod(ah, al, rh, rl, p0, p1);
+                        if (i == 0) {
+                            tacc[ce].s = p0;
+                            tacc[ce].c = p1;
+                        } else {
+                            df_acc(tacc[ce], p0, p1);
+                        }
                     } else {
-                        df_acc(tacc[ce], p0, p1);
+                        tnat[ce - kFirstNative] =
+                            fma(vget(a[v], e), rd, tnat[ce - kFirstNative]);
                     }
                     df_prod(ah, al, ph[ce], pl[ce], qp[ce].s, qp[ce].c);
                 }
@@ -359,7 +383,9 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                 }
             }
 #pragma unroll
-            for (int e = 0; e < kLaneCols; ++e) grp[e] = df_add(grp[e], tacc[e]);
+            for (int e = 0; e < kFirstNative; ++e) grp[e] = df_add(grp[e], tacc[e]);
+#pragma unroll
+            for (int j = 0; j < kNativeCols; ++j) snat[j] += tnat[j];
         } else {
             // Out-of-range values in these rows: native fp64 for them.
             double pd[kLaneCols];
@@ -421,10 +447,25 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             for (int v = 0; v < VPL; ++v)
 #pragma unroll
                 for (int e = 0; e < VE; ++e) {
-                    segp[lane_col<T>(v, lane, e)] += df_to_double(grp[v * VE + e]);
-                    grp[v * VE + e].s = grp[v * VE + e].c = 0.f;
+                    const int ce = v * VE + e;
+                    if (ce < kFirstNative) {
+                        segp[lane_col<T>(v, lane, e)] += df_to_double(grp[ce]);
+                        grp[ce].s = grp[ce].c = 0.f;
+                    }
                 }
             ngrp = 0;
+        }
+        if (seg_end) {
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) {
+                    const int ce = v * VE + e;
+                    if (ce >= kFirstNative) {
+                        segp[lane_col<T>(v, lane, e)] += snat[ce - kFirstNative];
+                        snat[ce - kFirstNative] = 0.0;
+                    }
+                }
         }
 
         if (seg_end) {  // segment end: flush s

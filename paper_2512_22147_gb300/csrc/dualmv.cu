@@ -38,9 +38,13 @@ constexpr int kDirectCtasPerSm = 4;
 #ifndef DUALMV_F64E_STAGES
 #define DUALMV_F64E_STAGES 3
 #endif
+#ifndef DUALMV_F64E_BAND
+#define DUALMV_F64E_BAND 256
+#endif
 constexpr int kF64eWarps = DUALMV_F64E_WARPS;
 constexpr int kF64eRpw = DUALMV_F64E_RPW;
 constexpr int kF64eStages = DUALMV_F64E_STAGES;
+constexpr int kF64eBand = DUALMV_F64E_BAND;
 
 // Which stream kernel a call uses.
 enum class Kind { kTma, kDirect, kF64e };
@@ -141,7 +145,7 @@ CUtensorMapL2promotion l2_promotion(uintptr_t base, int64_t row_bytes, int64_t b
 // kBandCols x tile_rows (x 1).  Columns >= N and rows >= M read as zero.
 template <typename T>
 bool encode_a(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
-              int64_t strideA, int64_t batch, int tile_rows, bool three_d) {
+              int64_t strideA, int64_t batch, int box_cols, int tile_rows, bool three_d) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     const int64_t es = sizeof(T);
@@ -149,7 +153,7 @@ bool encode_a(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
         l2_promotion(reinterpret_cast<uintptr_t>(A), lda * es, strideA * es, three_d);
     cuuint64_t dims[3] = {(cuuint64_t)N, (cuuint64_t)M, (cuuint64_t)batch};
     cuuint64_t strides[2] = {(cuuint64_t)(lda * es), (cuuint64_t)(strideA * es)};
-    cuuint32_t box[3] = {(cuuint32_t)kBandCols, (cuuint32_t)tile_rows, 1u};
+    cuuint32_t box[3] = {(cuuint32_t)box_cols, (cuuint32_t)tile_rows, 1u};
     cuuint32_t estr[3] = {1u, 1u, 1u};
     CUresult rc = fn(map, tma_dtype<T>(), three_d ? 3u : 2u, const_cast<T *>(A), dims,
                      strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -162,7 +166,9 @@ bool encode_a(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
 
 // Warps, rows per warp and shared memory of each stream kernel.
 struct Geometry {
-    int64_t tile_rows;
+    int64_t band_cols;  // columns per band (tile width)
+    int64_t tile_rows;  // rows per tile (stripe height)
+    int64_t box_rows;   // rows per TMA box
     int64_t smem;
     int64_t threads;
 };
@@ -171,7 +177,9 @@ template <typename T>
 Geometry generic_geometry(bool tma) {
     constexpr int rpw = sizeof(T) == 4 ? kRpw4 : kRpw8;
     Geometry g;
+    g.band_cols = kBandCols;
     g.tile_rows = kWarps * rpw;
+    g.box_rows = g.tile_rows;
     g.smem = tma ? dmv::SmemLayout<T, kWarps, rpw, kStages, true>::kTotal
                  : dmv::SmemLayout<T, kWarps, rpw, kStages, false>::kTotal;
     g.threads = (kWarps + (tma ? 1 : 0)) * 32;
@@ -181,8 +189,10 @@ Geometry generic_geometry(bool tma) {
 Geometry geometry(int64_t elem_bytes, int64_t acc_bytes, Kind kind) {
     if (kind == Kind::kF64e) {
         Geometry g;
+        g.band_cols = kF64eBand;
         g.tile_rows = kF64eWarps * kF64eRpw;
-        g.smem = dmv::SmemLayout<double, kF64eWarps, kF64eRpw, kF64eStages, true>::kTotal;
+        g.box_rows = kF64eRpw;  // one box per consumer warp
+        g.smem = dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand>::kTotal;
         g.threads = (kF64eWarps + 1) * 32;
         return g;
     }
@@ -203,9 +213,9 @@ dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
     const int64_t bm = geo.tile_rows;
     dualmv_plan_t p;
     std::memset(&p, 0, sizeof p);
-    p.band_cols = kBandCols;
+    p.band_cols = geo.band_cols;
     p.tile_rows = bm;
-    p.bands = (N + kBandCols - 1) / kBandCols;
+    p.bands = (N + p.band_cols - 1) / p.band_cols;
     p.stripes = (M + bm - 1) / bm;
     if (p.bands > INT64_MAX / p.stripes / batch) return DUALMV_ERR_INVALID_VALUE;
     p.tiles = batch * p.bands * p.stripes;
@@ -220,7 +230,7 @@ dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
     }
     p.max_segments = most;
     const int64_t q_ws = p.bands > 1 ? batch * p.bands * M * acc_bytes : 0;
-    const int64_t s_ws = p.grid * p.max_segments * kBandCols * acc_bytes;
+    const int64_t s_ws = p.grid * p.max_segments * p.band_cols * acc_bytes;
     p.workspace_bytes = ((q_ws + 255) / 256) * 256 + s_ws;
     p.smem_bytes = geo.smem;
     p.threads = geo.threads;
@@ -290,7 +300,7 @@ int combine_chunks(int64_t bands) {
 template <bool k3d>
 cudaError_t launch_f64e(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                         int dev, cudaStream_t stream) {
-    auto kern = dmv::dualmv_stream_f64e_kernel<kF64eWarps, kF64eRpw, kF64eStages, k3d>;
+    auto kern = dmv::dualmv_stream_f64e_kernel<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand, k3d>;
     static std::atomic<uint64_t> opted_in{0};
     const uint64_t bit = 1ull << (dev & 63);
     if (!(opted_in.load(std::memory_order_acquire) & bit)) {
@@ -381,8 +391,9 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     CUtensorMap map;
     std::memset(&map, 0, sizeof map);
     if (tma) {
-        const int tile_rows = (int)geometry(es, sizeof(Acc), kind).tile_rows;
-        tma = encode_a<T>(&map, A, M, N, lda, strideA, batch, tile_rows, three_d);
+        const Geometry geo = geometry(es, sizeof(Acc), kind);
+        tma = encode_a<T>(&map, A, M, N, lda, strideA, batch, (int)geo.band_cols,
+                          (int)geo.box_rows, three_d);
         if (!tma) kind = Kind::kDirect;
     }
 
@@ -404,6 +415,7 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     prm.q = q; prm.strideQ = strideQ;
     prm.s = s; prm.strideS = strideS;
     prm.M = M; prm.N = N; prm.batch = batch;
+    prm.band_cols = pl.band_cols;
     prm.bands = pl.bands; prm.stripes = pl.stripes; prm.tiles = pl.tiles;
     prm.grid = pl.grid; prm.max_seg = pl.max_segments;
     const int64_t q_ws_bytes = pl.bands > 1 ? batch * pl.bands * M * (int64_t)sizeof(Acc) : 0;
@@ -496,7 +508,7 @@ dualmv_status run_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,
                M < INT32_MAX && N < INT32_MAX;
     CUtensorMap map;
     std::memset(&map, 0, sizeof map);
-    if (tma) tma = encode_a<T>(&map, A, M, N, lda, M * lda, 1, kWarps * kRpw4, false);
+    if (tma) tma = encode_a<T>(&map, A, M, N, lda, M * lda, 1, kBandCols, kWarps * kRpw4, false);
     dualmv_plan_t pl;
     st = make_plan(M, N, 1, es, sizeof(Acc),
                    (int64_t)nd->sms * (tma ? 1 : kDirectCtasPerSm),
@@ -513,6 +525,7 @@ dualmv_status run_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,
     prm.q = q; prm.strideQ = M;
     prm.s = s; prm.strideS = N;
     prm.M = M; prm.N = N; prm.batch = 1;
+    prm.band_cols = pl.band_cols;
     prm.bands = pl.bands; prm.stripes = pl.stripes; prm.tiles = pl.tiles;
     prm.grid = pl.grid; prm.max_seg = pl.max_segments;
     const int64_t q_ws_bytes = pl.bands > 1 ? pl.bands * M * (int64_t)sizeof(Acc) : 0;

@@ -145,30 +145,47 @@ __device__ __forceinline__ void warp_rows_reduce_df(DF (&v)[RPW], int lane) {
     }
 }
 
+// Dynamic shared memory of the fp64 kernel: every consumer warp has its own
+// ring of STAGES boxes (its RPW rows of a tile), so warps wait only for
+// their own rows and drift apart instead of finishing every tile together;
+// then the warp scratch for the s flush and one full/empty mbarrier pair
+// per (warp, stage).
+template <int W, int RPW, int STAGES, int BAND>
+struct F64eLayout {
+    static constexpr int kBoxBytes = RPW * BAND * (int)sizeof(double);
+    static constexpr int kAlign = 1024;
+    static constexpr int kRing = W * STAGES * kBoxBytes;
+    static constexpr int kScratch = W * BAND * (int)sizeof(double);
+    static constexpr int kBars = 2 * W * STAGES * 8;
+    static constexpr int kTotal = kAlign + kRing + kScratch + kBars;
+};
+
 // ---------------------------------------------------------------- kernel --
 //
 // W consumer warps x RPW rows per warp per tile; lane l holds columns
 // 2l, 2l+1 (+64, +128, +192) of the 256-column band (four double2 vectors).
-template <int W, int RPW, int STAGES, bool kBatched3d>
+template <int W, int RPW, int STAGES, int BAND, bool kBatched3d>
 __global__ void __launch_bounds__((W + 1) * 32, 1)
 dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
     using T = double;
     using Acc = double;
     using Vec = double2;
     constexpr int VE = 2;
-    constexpr int VPL = kLaneCols / VE;  // 4 vectors per lane per row
+    constexpr int LANE_COLS = BAND / 32;  // columns per lane
+    constexpr int VPL = LANE_COLS / VE;   // 16-byte vectors per lane per row
     constexpr int BM = W * RPW;
-    constexpr int ROW_BYTES = kBandCols * (int)sizeof(T);
-    constexpr int TILE_BYTES = BM * ROW_BYTES;
-    using L = SmemLayout<T, W, RPW, STAGES, true>;
-    static_assert(L::kTileBytes == TILE_BYTES, "tile size mismatch");
+    constexpr int ROW_BYTES = BAND * (int)sizeof(T);
+    using L = F64eLayout<W, RPW, STAGES, BAND>;
+    static_assert(LANE_COLS == 4 || LANE_COLS == 8, "band of 128 or 256 columns");
+    constexpr int BOX_BYTES = L::kBoxBytes;
+    static_assert(BOX_BYTES == RPW * ROW_BYTES, "box size mismatch");
 
     extern __shared__ unsigned char smem_raw[];
     unsigned char *smem = smem_raw + shared_align_pad<L::kAlign>(smem_raw);
     unsigned char *ring = smem;
     Acc *scratch = reinterpret_cast<Acc *>(smem + L::kRing);
     uint64_t *full_bar = reinterpret_cast<uint64_t *>(smem + L::kRing + L::kScratch);
-    uint64_t *empty_bar = full_bar + STAGES;
+    uint64_t *empty_bar = full_bar + W * STAGES;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -180,9 +197,9 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     const int64_t g_first = t0 / S;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < STAGES; ++i) {
+        for (int i = 0; i < W * STAGES; ++i) {
             mbar_init(smem_u32(&full_bar[i]), 1);
-            mbar_init(smem_u32(&empty_bar[i]), W);
+            mbar_init(smem_u32(&empty_bar[i]), 1);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -195,22 +212,31 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             const uint64_t pol = policy_evict_first();
             bool ok = true;
             int64_t issued = 0;
+            int partial_w = 0;
             TileCursor cur;
             cur.init(t0, S, prm.bands);
             int stage = 0;
             uint32_t phase = 0;
             for (int64_t k = 0; k < ntiles; ++k) {
-                if (ok && k >= STAGES)
-                    ok = mbar_wait_bounded(smem_u32(&empty_bar[stage]), phase ^ 1u);
+                const int x = (int)(cur.band * BAND), y = (int)(cur.stripe * BM);
+                // One box of RPW rows per consumer warp, into that warp's ring.
+                for (int w = 0; w < W && ok; ++w) {
+                    const int slot = w * STAGES + stage;
+                    if (k >= STAGES)
+                        ok = mbar_wait_bounded(smem_u32(&empty_bar[slot]), phase ^ 1u);
+                    if (!ok) {
+                        partial_w = w;  // boxes 0..w-1 of tile k are in flight
+                        break;
+                    }
+                    const uint32_t fb = smem_u32(&full_bar[slot]);
+                    mbar_arrive_expect_tx(fb, BOX_BYTES);
+                    const uint32_t dst = smem_u32(ring + (size_t)slot * BOX_BYTES);
+                    if constexpr (kBatched3d)
+                        tma_load_3d(dst, &tmap, x, y + w * RPW, (int)cur.b, fb, pol);
+                    else
+                        tma_load_2d(dst, &tmap, x, y + w * RPW, fb, pol);
+                }
                 if (!ok) break;
-                const uint32_t fb = smem_u32(&full_bar[stage]);
-                mbar_arrive_expect_tx(fb, TILE_BYTES);
-                const uint32_t dst = smem_u32(ring + (size_t)stage * TILE_BYTES);
-                const int x = (int)(cur.band * kBandCols), y = (int)(cur.stripe * BM);
-                if constexpr (kBatched3d)
-                    tma_load_3d(dst, &tmap, x, y, (int)cur.b, fb, pol);
-                else
-                    tma_load_2d(dst, &tmap, x, y, fb, pol);
                 issued = k + 1;
                 cur.advance(S, prm.bands);
                 if (++stage == STAGES) {
@@ -218,9 +244,15 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                     phase ^= 1u;
                 }
             }
-            for (int64_t k = issued > STAGES ? issued - STAGES : 0; k < issued; ++k) {
+            // Every box issued must land before the CTA exits (bounded): the
+            // last STAGES whole tiles, and the first partial_w boxes of a
+            // tile abandoned half way by a timeout.
+            for (int64_t k = issued > STAGES ? issued - STAGES : 0; k <= issued; ++k) {
                 const int st = (int)(k % STAGES);
-                mbar_wait_bounded(smem_u32(&full_bar[st]), (uint32_t)(k / STAGES) & 1u);
+                const int nw = k < issued ? W : partial_w;
+                for (int w = 0; w < nw; ++w)
+                    mbar_wait_bounded(smem_u32(&full_bar[w * STAGES + st]),
+                                      (uint32_t)(k / STAGES) & 1u);
             }
         }
         return;
@@ -231,21 +263,21 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     const T *__restrict__ rg = static_cast<const T *>(prm.r);
     const int nthreads_c = W * 32;
 
-    // Lane columns kLaneCols - kNativeCols .. kLaneCols - 1 sum s in fp64.
-    constexpr int kNativeCols = DUALMV_F64E_NATIVE_COLS;
-    constexpr int kFirstNative = kLaneCols - kNativeCols;
+    // Lane columns LANE_COLS - kNativeCols .. LANE_COLS - 1 sum s in fp64.
+    constexpr int kNativeCols = DUALMV_F64E_NATIVE_COLS * LANE_COLS / 8;
+    constexpr int kFirstNative = LANE_COLS - kNativeCols;
     double snat[kNativeCols > 0 ? kNativeCols : 1];  // fp64 segment sums of s
 #pragma unroll
     for (int j = 0; j < kNativeCols; ++j) snat[j] = 0.0;
-    float ph[kLaneCols], pl[kLaneCols];  // split p of this lane's columns
+    float ph[LANE_COLS], pl[LANE_COLS];  // split p of this lane's columns
     bool p_bad = false;                  // some p of this lane out of range
-    DF grp[kLaneCols];                   // group sums of s (double-float)
+    DF grp[LANE_COLS];                   // group sums of s (double-float)
     // Segment sums of s (fp64) live in this warp's row of the flush scratch;
     // each lane owns its 8 columns there, so no synchronisation is needed
     // until the segment flush.
-    Acc *segp = scratch + warp * kBandCols;
+    Acc *segp = scratch + warp * BAND;
 #pragma unroll
-    for (int e = 0; e < kLaneCols; ++e) {
+    for (int e = 0; e < LANE_COLS; ++e) {
         ph[e] = pl[e] = 0.f;
         grp[e].s = grp[e].c = 0.f;
     }
@@ -272,7 +304,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         const int64_t stripe = cur.stripe;
         const int64_t band = cur.band;
         const int64_t b = cur.b;
-        const int64_t col0 = band * kBandCols;
+        const int64_t col0 = band * BAND;
         const int64_t row0 = stripe * BM + (int64_t)warp * RPW;
         const T rmine = r_next;
         cur.advance(S, prm.bands);
@@ -302,19 +334,21 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         split_f64(rmine, rh_mine, rl_mine, r_habs);
         const bool r_bad = !f64e_in_range(rmine);
 
-        if (ok) ok = mbar_wait_bounded(smem_u32(&full_bar[stage]), phase);
-        const Vec *tile = reinterpret_cast<const Vec *>(ring + (size_t)stage * TILE_BYTES);
+        const int slot = warp * STAGES + stage;
+        if (ok) ok = mbar_wait_bounded(smem_u32(&full_bar[slot]), phase);
+        // This warp's RPW rows of the tile.
+        const Vec *tile = reinterpret_cast<const Vec *>(ring + (size_t)slot * BOX_BYTES);
 
         // Fast path: double-float arithmetic with a cheap range bound.
         DF q[RPW];
-        DF tacc[kLaneCols];
+        DF tacc[LANE_COLS];
         double tnat[kNativeCols > 0 ? kNativeCols : 1];
 #pragma unroll
         for (int j = 0; j < kNativeCols; ++j) tnat[j] = 0.0;
         uint32_t span = 0;  // max over elements of (|a| bits - 2^-40 bits)
 #pragma unroll
         for (int i = 0; i < RPW; ++i) {
-            const Vec *rowp = tile + (size_t)(warp * RPW + i) * (ROW_BYTES / 16);
+            const Vec *rowp = tile + (size_t)i * (ROW_BYTES / 16);
             Vec a[VPL];
 #pragma unroll
             for (int v = 0; v < VPL; ++v) a[v] = rowp[v * 32 + lane];
@@ -322,7 +356,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             const float rl = __shfl_sync(0xffffffffu, rl_mine, i);
             const double rd = __shfl_sync(0xffffffffu, rmine, i);
             // Row products with p, summed pairwise (depth 3, not a chain of 7).
-            DF qp[kLaneCols];
+            DF qp[LANE_COLS];
 #pragma unroll
             for (int v = 0; v < VPL; ++v)
 #pragma unroll
@@ -347,8 +381,11 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                     }
                     df_prod(ah, al, ph[ce], pl[ce], qp[ce].s, qp[ce].c);
                 }
-            q[i] = df_add(df_add(df_add(qp[0], qp[1]), df_add(qp[2], qp[3])),
-                          df_add(df_add(qp[4], qp[5]), df_add(qp[6], qp[7])));
+            if constexpr (LANE_COLS == 8)
+                q[i] = df_add(df_add(df_add(qp[0], qp[1]), df_add(qp[2], qp[3])),
+                              df_add(df_add(qp[4], qp[5]), df_add(qp[6], qp[7])));
+            else
+                q[i] = df_add(df_add(qp[0], qp[1]), df_add(qp[2], qp[3]));
         }
         // Anything suspicious in this warp's rows (zeros included)?
         const bool rows_r_bad = __any_sync(0xffffffffu, lane < RPW && r_bad);
@@ -358,7 +395,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             bool bad = false;
 #pragma unroll
             for (int i = 0; i < RPW; ++i) {
-                const Vec *rowp = tile + (size_t)(warp * RPW + i) * (ROW_BYTES / 16);
+                const Vec *rowp = tile + (size_t)i * (ROW_BYTES / 16);
 #pragma unroll
                 for (int v = 0; v < VPL; ++v) {
                     const Vec av = rowp[v * 32 + lane];
@@ -370,7 +407,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
 
         if (!need_fp64) {
             __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[stage]));
+            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[slot]));
             warp_rows_reduce_df<RPW>(q, lane);
             if (butterfly_writer<RPW>(lane)) {
                 const int64_t row = row0 + butterfly_row<RPW>(lane);
@@ -388,7 +425,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             for (int j = 0; j < kNativeCols; ++j) snat[j] += tnat[j];
         } else {
             // Out-of-range values in these rows: native fp64 for them.
-            double pd[kLaneCols];
+            double pd[LANE_COLS];
             const T *pb = pg + b * prm.strideP;
 #pragma unroll
             for (int v = 0; v < VPL; ++v)
@@ -398,12 +435,12 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                     pd[v * VE + e] = col < prm.N ? pb[col] : 0.0;
                 }
             double qd[RPW];
-            double td[kLaneCols];
+            double td[LANE_COLS];
 #pragma unroll
-            for (int e = 0; e < kLaneCols; ++e) td[e] = 0.0;
+            for (int e = 0; e < LANE_COLS; ++e) td[e] = 0.0;
 #pragma unroll
             for (int i = 0; i < RPW; ++i) {
-                const Vec *rowp = tile + (size_t)(warp * RPW + i) * (ROW_BYTES / 16);
+                const Vec *rowp = tile + (size_t)i * (ROW_BYTES / 16);
                 const double ri = __shfl_sync(0xffffffffu, rmine, i);
                 double dot = 0.0;
 #pragma unroll
@@ -419,7 +456,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                 qd[i] = dot;
             }
             __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[stage]));
+            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[slot]));
             warp_rows_reduce<RPW>(qd, lane);
             if (butterfly_writer<RPW>(lane)) {
                 const int64_t row = row0 + butterfly_row<RPW>(lane);
@@ -471,16 +508,16 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         if (seg_end) {  // segment end: flush s
             named_barrier(1, nthreads_c);
             const bool whole_band = (seg_start_stripe == 0 && stripe == S - 1);
-            for (int col = threadIdx.x; col < kBandCols; col += nthreads_c) {
+            for (int col = threadIdx.x; col < BAND; col += nthreads_c) {
                 Acc acc = scratch[col];
 #pragma unroll
-                for (int w = 1; w < W; ++w) acc = acc + scratch[w * kBandCols + col];
+                for (int w = 1; w < W; ++w) acc = acc + scratch[w * BAND + col];
                 if (whole_band) {
                     if (col0 + col < prm.N)
                         static_cast<Acc *>(prm.s)[b * prm.strideS + col0 + col] = acc;
                 } else {
                     static_cast<Acc *>(prm.s_ws)[((c * prm.max_seg) + (g - g_first)) *
-                                                     kBandCols + col] = acc;
+                                                     BAND + col] = acc;
                 }
             }
             named_barrier(1, nthreads_c);

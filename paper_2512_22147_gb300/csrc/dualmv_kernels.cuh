@@ -266,6 +266,7 @@ struct Params {
     void *s;
     int64_t strideS;
     int64_t M, N, batch;
+    int64_t band_cols;  // columns per band (the stream kernel's tile width)
     int64_t bands, stripes, tiles, grid, max_seg;
     void *q_ws;  // [batch][bands][M] band partials of q (bands > 1 only)
     void *s_ws;  // [grid][max_seg][kBandCols] segment partials of s
@@ -596,8 +597,9 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
 //     y + 2C, ... in ascending order, then the C chunk sums are added in
 //     ascending chunk order.  C depends only on the band count, so the
 //     order (and the rounding) is the same on every call.
-//   Blocks [q_blocks, q_blocks + batch * bands): one band of s each; the
-//     segments of a band split between CTAs are added in ascending CTA order.
+//   Blocks [q_blocks, q_blocks + batch * bands): one band of s each (band
+//     width prm.band_cols <= 256); the segments of a band split between
+//     CTAs are added in ascending CTA order.
 template <typename Acc>
 __global__ void __launch_bounds__(256)
 dualmv_combine_kernel(const Params prm, int64_t q_blocks, int q_chunks) {
@@ -640,12 +642,13 @@ dualmv_combine_kernel(const Params prm, int64_t q_blocks, int q_chunks) {
     const int64_t c_hi = cta_of_tile(g * S + S - 1, T_, G);
     if (c_lo == c_hi) return;  // written directly by the stream kernel
     const int col = threadIdx.x;
-    const int64_t j = band * kBandCols + col;
+    if (col >= prm.band_cols) return;
+    const int64_t j = band * prm.band_cols + col;
     if (j >= prm.N) return;
     Acc acc = Acc(0);
     for (int64_t cc = c_lo; cc <= c_hi; ++cc) {
         const int64_t seg = g - cta_first_tile(cc, T_, G) / S;
-        const Acc v = sw[(cc * prm.max_seg + seg) * kBandCols + col];
+        const Acc v = sw[(cc * prm.max_seg + seg) * prm.band_cols + col];
         acc = (cc == c_lo) ? v : acc + v;
     }
     static_cast<Acc *>(prm.s)[b * prm.strideS + j] = acc;

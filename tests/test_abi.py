@@ -122,9 +122,10 @@ def _ref_first(c, T, G):
 ])
 def test_plan_covers_every_tile_once(M, N, batch, eb, ab, sms):
     pl = dm.dualmv_plan(M, N, batch, eb, ab, sms)
-    rows = 32 if eb == 4 else 28     # fp64: 7 warps x 4 rows (FP32-pipe kernel)
-    assert pl.band_cols == 256 and pl.tile_rows == rows
-    assert pl.bands == -(-N // 256) and pl.stripes == -(-M // rows)
+    # fp64: 7 warps x 4 rows of 256-column bands (FP32-pipe kernel)
+    rows, width = (32, 256) if eb == 4 else (28, 256)
+    assert pl.band_cols == width and pl.tile_rows == rows
+    assert pl.bands == -(-N // width) and pl.stripes == -(-M // rows)
     assert pl.tiles == batch * pl.bands * pl.stripes
     assert pl.grid == min(pl.tiles, sms)
     T, G, S = pl.tiles, pl.grid, pl.stripes
@@ -135,7 +136,7 @@ def test_plan_covers_every_tile_once(M, N, batch, eb, ab, sms):
             for c in range(G)]
     assert pl.max_segments == max(nseg)
     q_ws = batch * pl.bands * M * ab if pl.bands > 1 else 0
-    s_ws = G * pl.max_segments * 256 * ab
+    s_ws = G * pl.max_segments * width * ab
     assert pl.workspace_bytes == -(-q_ws // 256) * 256 + s_ws
     assert pl.smem_bytes <= 227 * 1024 and pl.threads == (288 if eb == 4 else 256)
 

@@ -23,7 +23,8 @@
  *   (cudaMallocFromPoolAsync) and returns it on the same stream.
  * Results.  Floating-point outputs are deterministic run to run for a given
  *   shape on a given GPU (fixed summation order, no atomics).  Integer
- *   outputs are exact modulo 2^64 in any order.
+ *   outputs are exact modulo 2^64 in any order, so the int32 path adds its
+ *   partial sums into q and s with atomics and takes no workspace.
  * Errors.  Every call returns a dualmv_status and never prints or aborts.
  *   DUALMV_ERR_INVALID_VALUE: M < 0, N < 0, batch < 0, lda < max(1, N), a
  *     NULL pointer whose extent is nonzero, or batch strides that make

@@ -12,6 +12,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <type_traits>
 
 #include "dualmv_kernels.cuh"
 #include "dualmv_f64e.cuh"
@@ -231,7 +232,10 @@ dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
     p.max_segments = most;
     const int64_t q_ws = p.bands > 1 ? batch * p.bands * M * acc_bytes : 0;
     const int64_t s_ws = p.grid * p.max_segments * p.band_cols * acc_bytes;
-    p.workspace_bytes = ((q_ws + 255) / 256) * 256 + s_ws;
+    // int32 inputs (4-byte elements, 8-byte sums) accumulate atomically into
+    // q and s and take no workspace.
+    const bool atomic_out = elem_bytes == 4 && acc_bytes == 8;
+    p.workspace_bytes = atomic_out ? 0 : ((q_ws + 255) / 256) * 256 + s_ws;
     p.smem_bytes = geo.smem;
     p.threads = geo.threads;
     *pl = p;
@@ -285,8 +289,25 @@ cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualm
         if (e != cudaSuccess) return e;
         opted_in.fetch_or(bit, std::memory_order_acq_rel);
     }
-    kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(map, prm);
-    return cudaGetLastError();
+    if constexpr (std::is_same<T, int32_t>::value) {
+        // Programmatic dependent of the zeroing kernel launched just before.
+        cudaLaunchConfig_t cfg;
+        std::memset(&cfg, 0, sizeof cfg);
+        cfg.gridDim = dim3((unsigned)pl.grid);
+        cfg.blockDim = dim3((unsigned)pl.threads);
+        cfg.dynamicSmemBytes = (size_t)pl.smem_bytes;
+        cfg.stream = stream;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(&cfg, kern, map, prm);
+    } else {
+        kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(map,
+                                                                                       prm);
+        return cudaGetLastError();
+    }
 }
 
 // Chunks per q output in the combine kernel: the smallest power of two
@@ -402,11 +423,16 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                    (int64_t)ds->sms * (tma ? 1 : kDirectCtasPerSm), kind, &pl);
     if (st != DUALMV_SUCCESS) return st;
 
+    // The int32 path accumulates into q and s atomically (exact, so still
+    // deterministic) and needs no workspace.
+    constexpr bool kAtomicOut = std::is_same<T, int32_t>::value;
     void *ws = nullptr;
-    e = cudaMallocFromPoolAsync(&ws, (size_t)pl.workspace_bytes, ds->pool, stream);
-    if (e != cudaSuccess) {
-        g_last_cuda_error = static_cast<int>(e);
-        return DUALMV_ERR_ALLOC;
+    if (!kAtomicOut) {
+        e = cudaMallocFromPoolAsync(&ws, (size_t)pl.workspace_bytes, ds->pool, stream);
+        if (e != cudaSuccess) {
+            g_last_cuda_error = static_cast<int>(e);
+            return DUALMV_ERR_ALLOC;
+        }
     }
     Params prm;
     prm.A = A; prm.lda = lda; prm.strideA = strideA;
@@ -419,8 +445,19 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     prm.bands = pl.bands; prm.stripes = pl.stripes; prm.tiles = pl.tiles;
     prm.grid = pl.grid; prm.max_seg = pl.max_segments;
     const int64_t q_ws_bytes = pl.bands > 1 ? batch * pl.bands * M * (int64_t)sizeof(Acc) : 0;
-    prm.q_ws = pl.bands > 1 ? ws : nullptr;
-    prm.s_ws = static_cast<unsigned char *>(ws) + ((q_ws_bytes + 255) / 256) * 256;
+    prm.q_ws = (pl.bands > 1 && ws) ? ws : nullptr;
+    prm.s_ws = ws ? static_cast<unsigned char *>(ws) + ((q_ws_bytes + 255) / 256) * 256 : nullptr;
+
+    if (kAtomicOut) {
+        const int64_t total = (M + N) * batch;
+        int64_t blocks = (total + 255) / 256;
+        if (blocks > (int64_t)ds->sms * 4) blocks = (int64_t)ds->sms * 4;
+        dmv::dualmv_zero_outputs_kernel<Acc><<<(unsigned)blocks, 256, 0, stream>>>(
+            reinterpret_cast<Acc *>(q), M, strideQ, reinterpret_cast<Acc *>(s), N, strideS,
+            batch);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return cuda_fail(e);
+    }
 
     cudaEvent_t ev_start = g_kernel_ev_start, ev_stop = g_kernel_ev_stop;
     g_kernel_ev_start = g_kernel_ev_stop = nullptr;
@@ -437,8 +474,8 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
         }
     }
     if (e == cudaSuccess && ev_stop) e = cudaEventRecord(ev_stop, stream);
-    if (e == cudaSuccess) e = launch_combine<Acc>(prm, stream);
-    cudaError_t ef = cudaFreeAsync(ws, stream);
+    if (e == cudaSuccess && !kAtomicOut) e = launch_combine<Acc>(prm, stream);
+    cudaError_t ef = ws ? cudaFreeAsync(ws, stream) : cudaSuccess;
     if (e != cudaSuccess) return cuda_fail(e);
     if (ef != cudaSuccess) return cuda_fail(ef);
     return DUALMV_SUCCESS;

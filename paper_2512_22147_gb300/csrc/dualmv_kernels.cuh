@@ -43,6 +43,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <type_traits>
+
 namespace dmv {
 
 constexpr int kBandCols = 256;          // columns per band = TMA box width
@@ -332,6 +334,13 @@ template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d>
 __global__ void __launch_bounds__((W + (kTma ? 1 : 0)) * 32, 1)
 dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
     using Acc = typename Traits<T>::Acc;
+    // Integer sums are exact modulo 2^64 in any order, so the int32 path adds
+    // its band and segment partials straight into q and s with atomics (the
+    // result is the same bits on every run) and needs no workspace and no
+    // combine kernel.  q and s are zeroed by a preceding kernel, whose
+    // completion the consumers await (programmatic dependent launch) before
+    // their first write.
+    constexpr bool kAtomicOut = std::is_same<T, int32_t>::value;
     using Vec = typename Traits<T>::Vec;
     constexpr int VE = Traits<T>::kVecElems;
     constexpr int VPL = kLaneCols / VE;  // 16-byte vectors per lane per row
@@ -444,6 +453,7 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
     }
     int stage = 0;
     uint32_t phase = 0;
+    if constexpr (kAtomicOut) pdl_wait();  // q and s zeroed before any add
 
     for (int64_t k = 0; k < ntiles; ++k) {
         const int64_t g = cur.g;
@@ -532,6 +542,8 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
                 if (prm.bands == 1) {
                     Acc *qo = static_cast<Acc *>(prm.q);
                     qo[b * prm.strideQ + row] = qp[0];
+                } else if constexpr (kAtomicOut) {
+                    atomicAdd(static_cast<Acc *>(prm.q) + b * prm.strideQ + row, qp[0]);
                 } else {
                     Acc *qw = static_cast<Acc *>(prm.q_ws);
                     qw[(b * prm.bands + band) * prm.M + row] = qp[0];
@@ -570,6 +582,9 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
                         Acc *so = static_cast<Acc *>(prm.s);
                         so[b * prm.strideS + col0 + col] = acc;
                     }
+                } else if constexpr (kAtomicOut) {
+                    if (col0 + col < prm.N)
+                        atomicAdd(static_cast<Acc *>(prm.s) + b * prm.strideS + col0 + col, acc);
                 } else {
                     Acc *sws = static_cast<Acc *>(prm.s_ws);
                     sws[((c * prm.max_seg) + (g - g_first)) * kBandCols + col] = acc;
@@ -652,6 +667,27 @@ dualmv_combine_kernel(const Params prm, int64_t q_blocks, int q_chunks) {
         acc = (cc == c_lo) ? v : acc + v;
     }
     static_cast<Acc *>(prm.s)[b * prm.strideS + j] = acc;
+}
+
+// Zeroes q and s (strided batches) ahead of a stream kernel that adds into
+// them atomically; lets that kernel launch at once (programmatic dependent
+// launch) so its prologue and first copies overlap this one.
+template <typename Acc>
+__global__ void dualmv_zero_outputs_kernel(Acc *q, int64_t M, int64_t strideQ, Acc *s,
+                                           int64_t N, int64_t strideS, int64_t batch) {
+    pdl_launch_dependents();
+    const int64_t nq = M * batch, total = nq + N * batch;
+    for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        if (idx < nq) {
+            const int64_t b = idx / M, i = idx - b * M;
+            q[b * strideQ + i] = Acc(0);
+        } else {
+            const int64_t js = idx - nq;
+            const int64_t b = js / N, j = js - b * N;
+            s[b * strideS + j] = Acc(0);
+        }
+    }
 }
 
 // Zero-fill of strided outputs (empty problems).

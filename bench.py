@@ -148,7 +148,7 @@ def gpu_uuid(torch, dev):
 
 def workload_from_args(inputs, args):
     """The named workload, optionally resized (for small profiling cases)."""
-    w = inputs.WORKLOADS[args.workload]
+    w = inputs.WORKLOADS.get(args.workload) or inputs.OP_WORKLOADS[args.workload]
     kw = {}
     for k in ("M", "N", "lda", "batch"):
         v = getattr(args, k)
@@ -203,14 +203,30 @@ def run_native(args):
     from paper_2512_22147_gb300 import inputs
 
     w = workload_from_args(inputs, args)
-    A, p, r = inputs.generate(w, dev)
-    Av = A[..., : w.N]
-    q, s = inputs.empty_outputs(w, dev)
     stream = torch.cuda.current_stream(dev)
     nbytes = w.bytes_counted()
+    if w.op == "bicg":
+        A, p, r = inputs.generate(w, dev)
+        Av = A[..., : w.N]
+        q, s = inputs.empty_outputs(w, dev)
+
+        def call():
+            dm.dualmv(Av, p, r, q=q, s=s)
+    elif w.op == "gesummv":
+        A, Bm, x = inputs.generate_gesummv(w, dev)
+        y = torch.empty(w.M, dtype=A.dtype, device=dev)
+
+        def call():
+            dm.gesummv(A[:, : w.N], Bm[:, : w.N], x, alpha=1.5, beta=1.2, y=y)
+    else:
+        A, x = inputs.generate_atax(w, dev)
+        y = torch.empty(w.N, dtype=A.dtype, device=dev)
+
+        def call():
+            dm.atax(A[:, : w.N], x, y=y)
 
     for _ in range(args.warmup):
-        dm.dualmv(Av, p, r, q=q, s=s)
+        call()
     torch.cuda.synchronize(dev)
     if dm.device_fault() != dm.DUALMV_SUCCESS:
         raise RuntimeError("device fault during warm-up")
@@ -226,7 +242,7 @@ def run_native(args):
     torch.cuda.synchronize(dev)
     region[0].record(stream)
     for _ in range(K):
-        dm.dualmv(Av, p, r, q=q, s=s)
+        call()
     region[1].record(stream)
     torch.cuda.synchronize(dev)
     barrier(world)
@@ -255,10 +271,15 @@ def run_native(args):
     torch.cuda.synchronize(dev)
     for i in range(Ki):
         ks, ke = kern_ev[i]
-        dm.dualmv_record_kernel_events(ks.cuda_event, ke.cuda_event)
+        if w.op == "bicg":
+            dm.dualmv_record_kernel_events(ks.cuda_event, ke.cuda_event)
+        else:  # several streaming passes per call: time the whole call
+            ks.record(stream)
         call_ev[i][0].record(stream)
-        dm.dualmv(Av, p, r, q=q, s=s)
+        call()
         call_ev[i][1].record(stream)
+        if w.op != "bicg":
+            ke.record(stream)
     torch.cuda.synchronize(dev)
     if dm.device_fault() != dm.DUALMV_SUCCESS:
         raise RuntimeError("device fault during the instrumented region")
@@ -269,6 +290,10 @@ def run_native(args):
                           inputs.OUT_BYTES[w.dtype],
                           torch.cuda.get_device_properties(dev).multi_processor_count)
     launches_per_call = 1 + (1 if (plan.bands > 1 or plan.grid > 1) else 0)
+    if w.op == "gesummv":   # two row passes (stream + combine each) + epilogue
+        launches_per_call = 2 * launches_per_call + 1
+    elif w.op == "atax":    # a row pass and a column pass
+        launches_per_call = 2 * launches_per_call
     peak, peak_src = measured_peak()
     kern_avg_ms = sum(kern_ms) / len(kern_ms)
     achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9
@@ -277,11 +302,11 @@ def run_native(args):
     # End to end through the same public call with host buffers: pinned host
     # inputs copied in, the call, results copied out, every step.
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and w.op == "bicg":
         e2e = run_e2e(torch, dm, w, A, p, r, dev, stream, args.e2e_steps)
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and w.op == "bicg":
         cpu = cpu_baseline(w, A, p, r, args.cpu_seconds)
 
     out = {
@@ -298,7 +323,7 @@ def run_native(args):
         "dtype": w.dtype,
         "data": "synthetic",
         "config": {
-            "workload": w.name, "M": w.M, "N": w.N, "lda": w.lda,
+            "workload": w.name, "op": w.op, "M": w.M, "N": w.N, "lda": w.lda,
             "batch": w.batch, "dtype": w.dtype, "distribution": w.dist, "seed": w.seed,
             "bytes_per_step": nbytes,
             "l2": "inputs larger than L2 (no flush needed)",
@@ -309,7 +334,7 @@ def run_native(args):
         "median_step_ms": round(statistics.median(step_ms), 5),
         "roofline": {
             "bound": "hbm",
-            "kernel": "dualmv_stream_kernel",
+            "kernel": "dualmv_stream_kernel" if w.op == "bicg" else f"whole {w.op} call",
             "achieved": round(achieved, 2),
             "peak": peak,
             "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"

@@ -104,6 +104,35 @@ dualmv_status dualmv_i32_strided_batched(
     int64_t *q, int64_t strideQ, int64_t *s, int64_t strideS, int64_t batch,
     dualmv_stream_t stream);
 
+/* ---- operations built on the same streaming kernels --------------------
+ * Two more kernels the paper tunes (Table 1 and Table 2), each a short
+ * sequence of single-sided passes of the dual product's streaming kernel
+ * (rows only or columns only), so every pass reads its matrix once.
+ * Conventions as above (row-major, caller-owned device memory, asynchronous
+ * on `stream`, stream-ordered scratch from the library's pool).
+ *
+ * GESUMMV (Table 1 / Table 2, row "GESUMMV"): with A and B both M x N
+ * (leading dimensions lda, ldb >= max(1, N)), x of length N and y of
+ * length M:  tmp = A x;  y = B x;  y = alpha * tmp + beta * y.
+ * Floating-point sums have a fixed order (deterministic).  Errors as for
+ * dualmv_f32: DUALMV_ERR_INVALID_VALUE for bad sizes or NULL pointers with
+ * nonzero extents; N == 0 sets y to zero. */
+dualmv_status dualmv_gesummv_f32(int64_t M, int64_t N, float alpha, const float *A,
+                                 int64_t lda, float beta, const float *B, int64_t ldb,
+                                 const float *x, float *y, dualmv_stream_t stream);
+dualmv_status dualmv_gesummv_f64(int64_t M, int64_t N, double alpha, const double *A,
+                                 int64_t lda, double beta, const double *B, int64_t ldb,
+                                 const double *x, double *y, dualmv_stream_t stream);
+
+/* ATAX (Table 1, row "ATAX"): with A M x N (lda >= max(1, N)), x of length
+ * N and y of length N:  tmp = A x (length M);  y = A^T tmp.  The second
+ * product needs all of tmp, so A is streamed twice (rows, then columns).
+ * M == 0 sets y to zero. */
+dualmv_status dualmv_atax_f32(int64_t M, int64_t N, const float *A, int64_t lda,
+                              const float *x, float *y, dualmv_stream_t stream);
+dualmv_status dualmv_atax_f64(int64_t M, int64_t N, const double *A, int64_t lda,
+                              const double *x, double *y, dualmv_stream_t stream);
+
 /* ---- single problem without allocation --------------------------------
  * The paper has no counterpart to this entry point; it exists for callers
  * that cannot allocate device memory during the call: code inside a

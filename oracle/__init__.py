@@ -85,6 +85,15 @@ def _declare(lib):
         fn.restype = ctypes.c_int
     lib.oracle_trimmed_mean.argtypes = [vp, i64, i64, vp]
     lib.oracle_trimmed_mean.restype = ctypes.c_int
+    dbl = ctypes.c_double
+    for name in ("oracle_gesummv_f32", "oracle_gesummv_f64"):
+        fn = getattr(lib, name)
+        fn.argtypes = [i64, i64, dbl, vp, i64, dbl, vp, i64, vp, vp]
+        fn.restype = ctypes.c_int
+    for name in ("oracle_atax_f32", "oracle_atax_f64"):
+        fn = getattr(lib, name)
+        fn.argtypes = [i64, i64, vp, i64, vp, vp]
+        fn.restype = ctypes.c_int
     return lib
 
 
@@ -183,3 +192,57 @@ def trimmed_mean(times, k: int, lib=None) -> float:
     if rc != 0:
         raise ValueError("trimmed mean needs R > 2k and k >= 0")
     return float(out[0])
+
+
+def _float_tag(A: np.ndarray) -> str:
+    if A.dtype == np.float32:
+        return "f32"
+    if A.dtype == np.float64:
+        return "f64"
+    raise TypeError(f"unsupported dtype {A.dtype}")
+
+
+def gesummv(A: np.ndarray, B: np.ndarray, x: np.ndarray, alpha: float, beta: float,
+            N: int | None = None, lib=None) -> np.ndarray:
+    """GESUMMV (Table 1 / Table 2): y = alpha (A x) + beta (B x), in float64.
+
+    A and B are M x lda and M x ldb C-contiguous storage; only their first
+    N columns (default: all of A's) belong to the matrices."""
+    lib = lib or load()
+    tag = _float_tag(A)
+    if B.dtype != A.dtype or A.ndim != 2 or B.ndim != 2 or A.shape[0] != B.shape[0]:
+        raise ValueError("A and B must be 2-D with the same dtype and row count")
+    if not (A.flags.c_contiguous and B.flags.c_contiguous):
+        raise ValueError("A and B must be C-contiguous")
+    M = A.shape[0]
+    N = A.shape[1] if N is None else int(N)
+    if N > A.shape[1] or N > B.shape[1]:
+        raise ValueError("N exceeds a leading dimension")
+    x = np.ascontiguousarray(x, dtype=A.dtype)
+    if x.shape != (N,):
+        raise ValueError("x must have N elements")
+    y = np.zeros(M, dtype=np.float64)
+    rc = getattr(lib, f"oracle_gesummv_{tag}")(M, N, float(alpha), _ptr(A), max(A.shape[1], 1),
+                                               float(beta), _ptr(B), max(B.shape[1], 1),
+                                               _ptr(x), _ptr(y))
+    if rc != 0:
+        raise RuntimeError(f"oracle_gesummv_{tag} returned {rc}")
+    return y
+
+
+def atax(A: np.ndarray, x: np.ndarray, N: int | None = None, lib=None) -> np.ndarray:
+    """ATAX (Table 1): y = A^T (A x), in float64 (A is M x lda storage)."""
+    lib = lib or load()
+    tag = _float_tag(A)
+    if A.ndim != 2 or not A.flags.c_contiguous:
+        raise ValueError("A must be a C-contiguous 2-D buffer")
+    M = A.shape[0]
+    N = A.shape[1] if N is None else int(N)
+    x = np.ascontiguousarray(x, dtype=A.dtype)
+    if x.shape != (N,) or N > A.shape[1]:
+        raise ValueError("x must have N elements, N <= lda")
+    y = np.zeros(N, dtype=np.float64)
+    rc = getattr(lib, f"oracle_atax_{tag}")(M, N, _ptr(A), max(A.shape[1], 1), _ptr(x), _ptr(y))
+    if rc != 0:
+        raise RuntimeError(f"oracle_atax_{tag} returned {rc}")
+    return y

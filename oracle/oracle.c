@@ -36,7 +36,10 @@
  *
  * Also provided: the magnitude sums  sum_j |A_ij||p_j|  and
  * sum_i |A_ij||r_i|  in double, the denominators of the parity metric
- * max |err| / sum |A||x|.
+ * max |err| / sum |A||x|; and two more PolyBench kernels of the paper's
+ * tables built from the same products, with the same precision rules:
+ *     GESUMMV  y = alpha (A x) + beta (B x)       (Table 1, Table 2)
+ *     ATAX     y = A^T (A x)                      (Table 1)
  *
  * Build: plain C99, -O2 -fno-fast-math -ffp-contract=off, so the compiler
  * neither reassociates the sums nor fuses a multiply into an add.
@@ -234,5 +237,106 @@ int oracle_trimmed_mean(double *t, int64_t R, int64_t k, double *out)
     double sum = 0.0;
     for (int64_t i = k; i < R - k; ++i) sum += t[i];
     *out = sum / (double)(R - 2 * k);
+    return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------- GESUMMV --- */
+
+/* GESUMMV (Table 1 / Table 2): tmp = A x, yb = B x, y = alpha tmp + beta yb,
+ * with A and B M x N (leading dimensions lda, ldb >= N).  Float inputs:
+ * exact double products summed in double, result in double. */
+int oracle_gesummv_f32(int64_t M, int64_t N, double alpha, const float *A, int64_t lda,
+                       double beta, const float *B, int64_t ldb, const float *x, double *y)
+{
+    if (M < 0 || N < 0 || lda < N || ldb < N || lda < 1 || ldb < 1) return ORACLE_EINVAL;
+    if (M > 0 && (y == NULL || (N > 0 && (A == NULL || B == NULL || x == NULL))))
+        return ORACLE_EINVAL;
+    for (int64_t i = 0; i < M; ++i) {
+        double ta = 0.0, tb = 0.0;
+        for (int64_t j = 0; j < N; ++j) {
+            ta += (double)A[i * lda + j] * (double)x[j];
+            tb += (double)B[i * ldb + j] * (double)x[j];
+        }
+        y[i] = alpha * ta + beta * tb;
+    }
+    return ORACLE_OK;
+}
+
+/* Double inputs: each dot product with Dot2, then alpha tmp + beta yb. */
+int oracle_gesummv_f64(int64_t M, int64_t N, double alpha, const double *A, int64_t lda,
+                       double beta, const double *B, int64_t ldb, const double *x, double *y)
+{
+    if (M < 0 || N < 0 || lda < N || ldb < N || lda < 1 || ldb < 1) return ORACLE_EINVAL;
+    if (M > 0 && (y == NULL || (N > 0 && (A == NULL || B == NULL || x == NULL))))
+        return ORACLE_EINVAL;
+    for (int64_t i = 0; i < M; ++i) {
+        double a_hi = 0.0, a_lo = 0.0, b_hi = 0.0, b_lo = 0.0;
+        for (int64_t j = 0; j < N; ++j) {
+            double prod, perr, sum, serr;
+            two_prod(A[i * lda + j], x[j], &prod, &perr);
+            two_sum(a_hi, prod, &sum, &serr);
+            a_hi = sum;
+            a_lo = a_lo + (perr + serr);
+            two_prod(B[i * ldb + j], x[j], &prod, &perr);
+            two_sum(b_hi, prod, &sum, &serr);
+            b_hi = sum;
+            b_lo = b_lo + (perr + serr);
+        }
+        y[i] = alpha * (a_hi + a_lo) + beta * (b_hi + b_lo);
+    }
+    return ORACLE_OK;
+}
+
+/* ---------------------------------------------------------------- ATAX --- */
+
+/* ATAX (Table 1): tmp = A x (length M), y = A^T tmp (length N).  Float
+ * inputs: both products in double, tmp kept in double. */
+int oracle_atax_f32(int64_t M, int64_t N, const float *A, int64_t lda, const float *x,
+                    double *y)
+{
+    if (M < 0 || N < 0 || lda < N || lda < 1) return ORACLE_EINVAL;
+    if (N > 0 && (y == NULL || (M > 0 && (A == NULL || x == NULL)))) return ORACLE_EINVAL;
+    for (int64_t j = 0; j < N; ++j) y[j] = 0.0;
+    for (int64_t i = 0; i < M; ++i) {
+        double tmp = 0.0;
+        for (int64_t j = 0; j < N; ++j) tmp += (double)A[i * lda + j] * (double)x[j];
+        for (int64_t j = 0; j < N; ++j) y[j] += (double)A[i * lda + j] * tmp;
+    }
+    return ORACLE_OK;
+}
+
+/* Double inputs: tmp_i with Dot2 (rounded to double), then each y_j with
+ * Dot2 over i of A_ij tmp_i. */
+int oracle_atax_f64(int64_t M, int64_t N, const double *A, int64_t lda, const double *x,
+                    double *y)
+{
+    if (M < 0 || N < 0 || lda < N || lda < 1) return ORACLE_EINVAL;
+    if (N > 0 && (y == NULL || (M > 0 && (A == NULL || x == NULL)))) return ORACLE_EINVAL;
+    double *y_lo = NULL;
+    if (N > 0) {
+        y_lo = (double *)malloc((size_t)N * sizeof(double));
+        if (y_lo == NULL) return ORACLE_ENOMEM;
+        for (int64_t j = 0; j < N; ++j) { y[j] = 0.0; y_lo[j] = 0.0; }
+    }
+    for (int64_t i = 0; i < M; ++i) {
+        double t_hi = 0.0, t_lo = 0.0;
+        for (int64_t j = 0; j < N; ++j) {
+            double prod, perr, sum, serr;
+            two_prod(A[i * lda + j], x[j], &prod, &perr);
+            two_sum(t_hi, prod, &sum, &serr);
+            t_hi = sum;
+            t_lo = t_lo + (perr + serr);
+        }
+        const double tmp = t_hi + t_lo;
+        for (int64_t j = 0; j < N; ++j) {
+            double prod, perr, sum, serr;
+            two_prod(A[i * lda + j], tmp, &prod, &perr);
+            two_sum(y[j], prod, &sum, &serr);
+            y[j] = sum;
+            y_lo[j] = y_lo[j] + (perr + serr);
+        }
+    }
+    for (int64_t j = 0; j < N; ++j) y[j] = y[j] + y_lo[j];
+    free(y_lo);
     return ORACLE_OK;
 }

@@ -21,9 +21,10 @@ _BINDING_NAMES = {
     "dualmv_i32", "dualmv_i32_strided_batched", "dualmv_last_cuda_error",
     "dualmv_plan", "dualmv_record_kernel_events", "dualmv_set_path",
     "dualmv_status_string", "library", "dualmv_f32_noalloc",
-    "dualmv_f32_noalloc_scratch_bytes",
+    "dualmv_f32_noalloc_scratch_bytes", "dualmv_gesummv_f32", "dualmv_gesummv_f64",
+    "dualmv_atax_f32", "dualmv_atax_f64",
 }
-_API_NAMES = {"dualmv", "device_fault"}
+_API_NAMES = {"dualmv", "device_fault", "gesummv", "atax"}
 
 
 def __getattr__(name):

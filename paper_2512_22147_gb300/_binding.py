@@ -39,6 +39,7 @@ EXPORTED = (
     "dualmv_status_string", "dualmv_last_cuda_error", "dualmv_device_fault",
     "dualmv_set_path", "dualmv_plan", "dualmv_record_kernel_events",
     "dualmv_f32_noalloc", "dualmv_f32_noalloc_scratch_bytes",
+    "dualmv_gesummv_f32", "dualmv_gesummv_f64", "dualmv_atax_f32", "dualmv_atax_f64",
 )
 
 
@@ -76,6 +77,13 @@ def _load() -> ctypes.CDLL:
     lib.dualmv_f32_noalloc.argtypes, lib.dualmv_f32_noalloc.restype = single, st
     lib.dualmv_f32_noalloc_scratch_bytes.argtypes = []
     lib.dualmv_f32_noalloc_scratch_bytes.restype = i64
+    for tag, real in (("f32", ctypes.c_float), ("f64", ctypes.c_double)):
+        f = getattr(lib, f"dualmv_gesummv_{tag}")
+        f.argtypes = [i64, i64, real, vp, i64, real, vp, i64, vp, vp, vp]
+        f.restype = st
+        f = getattr(lib, f"dualmv_atax_{tag}")
+        f.argtypes = [i64, i64, vp, i64, vp, vp, vp]
+        f.restype = st
     lib.dualmv_status_string.argtypes = [st]
     lib.dualmv_status_string.restype = ctypes.c_char_p
     lib.dualmv_last_cuda_error.argtypes = []
@@ -136,6 +144,22 @@ def dualmv_f64_strided_batched(M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS, bat
 def dualmv_i32_strided_batched(M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS, batch, stream):
     return _lib.dualmv_i32_strided_batched(M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS,
                                            batch, stream)
+
+
+def dualmv_gesummv_f32(M, N, alpha, A, lda, beta, B, ldb, x, y, stream):
+    return _lib.dualmv_gesummv_f32(M, N, alpha, A, lda, beta, B, ldb, x, y, stream)
+
+
+def dualmv_gesummv_f64(M, N, alpha, A, lda, beta, B, ldb, x, y, stream):
+    return _lib.dualmv_gesummv_f64(M, N, alpha, A, lda, beta, B, ldb, x, y, stream)
+
+
+def dualmv_atax_f32(M, N, A, lda, x, y, stream):
+    return _lib.dualmv_atax_f32(M, N, A, lda, x, y, stream)
+
+
+def dualmv_atax_f64(M, N, A, lda, x, y, stream):
+    return _lib.dualmv_atax_f64(M, N, A, lda, x, y, stream)
 
 
 def dualmv_status_string(status: int) -> str:

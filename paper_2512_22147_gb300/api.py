@@ -19,6 +19,8 @@ import torch
 
 from . import _binding as B
 
+B_ = B  # the binding, where a parameter is named B
+
 _OUT = {torch.float32: torch.float32, torch.float64: torch.float64,
         torch.int32: torch.int64}
 _TAG = {torch.float32: "f32", torch.float64: "f64", torch.int32: "i32"}
@@ -103,3 +105,68 @@ def device_fault(stream: torch.cuda.Stream | None = None) -> int:
     """Synchronise ``stream`` and return (and clear) the device fault status."""
     strm = stream if stream is not None else torch.cuda.current_stream()
     return B.dualmv_device_fault(strm.cuda_stream)
+
+
+def _matrix(A: torch.Tensor, name: str):
+    if A.dim() != 2:
+        raise ValueError(f"{name} must be 2-D")
+    M, N = A.shape
+    if N > 1 and A.stride(1) != 1:
+        raise ValueError(f"{name}'s last dimension must be contiguous")
+    if M > 1 and A.stride(0) < N:
+        raise ValueError(f"{name}'s rows overlap")
+    return M, N, (max(A.stride(0), N, 1) if M > 1 else max(N, 1))
+
+
+def _vector(v: torch.Tensor, n: int, like: torch.Tensor, name: str):
+    if v.dtype != like.dtype or v.device != like.device or v.dim() != 1 or v.shape[0] != n:
+        raise ValueError(f"{name} must be a {like.dtype} vector of length {n} on {like.device}")
+    if n > 1 and v.stride(0) != 1:
+        raise ValueError(f"{name} must be contiguous")
+
+
+def gesummv(A: torch.Tensor, B: torch.Tensor, x: torch.Tensor, alpha: float = 1.0,
+            beta: float = 1.0, y: torch.Tensor | None = None,
+            stream: torch.cuda.Stream | None = None) -> torch.Tensor:
+    """GESUMMV (Table 1 / Table 2): ``y = alpha * (A x) + beta * (B x)``.
+
+    A and B are M x N float32/float64 CUDA tensors (unit column stride)."""
+    tag = {torch.float32: "f32", torch.float64: "f64"}.get(A.dtype)
+    if tag is None or not A.is_cuda:
+        raise TypeError("A must be a float32 or float64 CUDA tensor")
+    M, N, lda = _matrix(A, "A")
+    MB, NB, ldb = _matrix(B, "B")
+    if (MB, NB) != (M, N) or B.dtype != A.dtype or B.device != A.device:
+        raise ValueError("B must match A's shape, dtype and device")
+    _vector(x, N, A, "x")
+    if y is None:
+        y = torch.empty(M, dtype=A.dtype, device=A.device)
+    _vector(y, M, A, "y")
+    strm = stream if stream is not None else torch.cuda.current_stream(A.device)
+    with torch.cuda.device(A.device):
+        rc = getattr(B_, f"dualmv_gesummv_{tag}")(M, N, alpha, A.data_ptr(), lda, beta,
+                                                  B.data_ptr(), ldb, x.data_ptr(),
+                                                  y.data_ptr(), strm.cuda_stream)
+    if rc != B_.DUALMV_SUCCESS:
+        raise B_.DualmvError(rc, f"dualmv_gesummv_{tag}")
+    return y
+
+
+def atax(A: torch.Tensor, x: torch.Tensor, y: torch.Tensor | None = None,
+         stream: torch.cuda.Stream | None = None) -> torch.Tensor:
+    """ATAX (Table 1): ``y = A^T (A x)`` for an M x N float32/float64 A."""
+    tag = {torch.float32: "f32", torch.float64: "f64"}.get(A.dtype)
+    if tag is None or not A.is_cuda:
+        raise TypeError("A must be a float32 or float64 CUDA tensor")
+    M, N, lda = _matrix(A, "A")
+    _vector(x, N, A, "x")
+    if y is None:
+        y = torch.empty(N, dtype=A.dtype, device=A.device)
+    _vector(y, N, A, "y")
+    strm = stream if stream is not None else torch.cuda.current_stream(A.device)
+    with torch.cuda.device(A.device):
+        rc = getattr(B_, f"dualmv_atax_{tag}")(M, N, A.data_ptr(), lda, x.data_ptr(),
+                                               y.data_ptr(), strm.cuda_stream)
+    if rc != B_.DUALMV_SUCCESS:
+        raise B_.DualmvError(rc, f"dualmv_atax_{tag}")
+    return y

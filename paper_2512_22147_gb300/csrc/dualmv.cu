@@ -247,17 +247,20 @@ dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
 dualmv_status validate(int64_t M, int64_t N, const void *A, int64_t lda, int64_t strideA,
                        const void *p, int64_t strideP, const void *r, int64_t strideR,
                        const void *q, int64_t strideQ, const void *s, int64_t strideS,
-                       int64_t batch) {
+                       int64_t batch, uint32_t outputs = dmv::kOutBoth) {
+    const bool want_q = (outputs & dmv::kOutQ) != 0, want_s = (outputs & dmv::kOutS) != 0;
     if (M < 0 || N < 0 || batch < 0) return DUALMV_ERR_INVALID_VALUE;
     if (lda < (N > 1 ? N : 1)) return DUALMV_ERR_INVALID_VALUE;
     if (strideA < 0 || strideP < 0 || strideR < 0 || strideQ < 0 || strideS < 0)
         return DUALMV_ERR_INVALID_VALUE;
     if (batch == 0) return DUALMV_SUCCESS;
-    if (M > 0 && N > 0 && (A == nullptr || p == nullptr || r == nullptr))
+    if (M > 0 && N > 0 &&
+        (A == nullptr || (want_q && p == nullptr) || (want_s && r == nullptr)))
         return DUALMV_ERR_INVALID_VALUE;
-    if (M > 0 && q == nullptr) return DUALMV_ERR_INVALID_VALUE;
-    if (N > 0 && s == nullptr) return DUALMV_ERR_INVALID_VALUE;
-    if (batch > 1 && (strideQ < M || strideS < N)) return DUALMV_ERR_INVALID_VALUE;
+    if (want_q && M > 0 && q == nullptr) return DUALMV_ERR_INVALID_VALUE;
+    if (want_s && N > 0 && s == nullptr) return DUALMV_ERR_INVALID_VALUE;
+    if (batch > 1 && ((want_q && strideQ < M) || (want_s && strideS < N)))
+        return DUALMV_ERR_INVALID_VALUE;
     // Index arithmetic stays in int64: the last element of A must be addressable.
     if (M > 0 && N > 0) {
         const int64_t lim = INT64_MAX / 4;
@@ -275,11 +278,11 @@ bool fault_injected_alloc() {
 
 // ------------------------------------------------------------- launching --
 
-template <typename T, bool kTma, bool k3d>
+template <typename T, bool kTma, bool k3d, int kOut = dmv::kOutBoth>
 cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                           int dev, cudaStream_t stream) {
     constexpr int rpw = sizeof(T) == 4 ? kRpw4 : kRpw8;
-    auto kern = dmv::dualmv_stream_kernel<T, kWarps, rpw, kStages, kTma, k3d>;
+    auto kern = dmv::dualmv_stream_kernel<T, kWarps, rpw, kStages, kTma, k3d, kOut>;
     // The shared-memory opt-in is per device and per kernel; set it once.
     static std::atomic<uint64_t> opted_in{0};
     const uint64_t bit = 1ull << (dev & 63);
@@ -318,10 +321,11 @@ int combine_chunks(int64_t bands) {
     return c;
 }
 
-template <bool k3d>
+template <bool k3d, int kOut = dmv::kOutBoth>
 cudaError_t launch_f64e(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                         int dev, cudaStream_t stream) {
-    auto kern = dmv::dualmv_stream_f64e_kernel<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand, k3d>;
+    auto kern = dmv::dualmv_stream_f64e_kernel<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand,
+                                               k3d, kOut>;
     static std::atomic<uint64_t> opted_in{0};
     const uint64_t bit = 1ull << (dev & 63);
     if (!(opted_in.load(std::memory_order_acquire) & bit)) {
@@ -338,9 +342,12 @@ template <typename Acc>
 cudaError_t launch_combine(const Params &prm, cudaStream_t stream) {
     const int chunks = combine_chunks(prm.bands);
     const int64_t rows_per_block = 256 / chunks;
-    const int64_t q_blocks =
-        prm.bands > 1 ? (prm.batch * prm.M + rows_per_block - 1) / rows_per_block : 0;
-    const int64_t s_blocks = prm.grid > 1 ? prm.batch * prm.bands : 0;
+    const bool want_q = (prm.outputs & dmv::kOutQ) != 0;
+    const bool want_s = (prm.outputs & dmv::kOutS) != 0;
+    const int64_t q_blocks = (want_q && prm.bands > 1)
+                                 ? (prm.batch * prm.M + rows_per_block - 1) / rows_per_block
+                                 : 0;
+    const int64_t s_blocks = (want_s && prm.grid > 1) ? prm.batch * prm.bands : 0;
     const int64_t blocks = q_blocks + s_blocks;
     if (blocks == 0) return cudaSuccess;
     if (blocks > INT32_MAX) return cudaErrorInvalidConfiguration;
@@ -369,23 +376,30 @@ cudaError_t zero_fill(Acc *out, int64_t len, int64_t stride, int64_t batch,
     return cudaGetLastError();
 }
 
+// One dual (or single-sided) matrix-vector product.  `outputs` selects q,
+// s or both; single-sided calls (the building blocks of ATAX and GESUMMV)
+// are single problems of float or double.
 template <typename T, typename Out>
 dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA,
                   const T *p, int64_t strideP, const T *r, int64_t strideR, Out *q,
                   int64_t strideQ, Out *s, int64_t strideS, int64_t batch,
-                  cudaStream_t stream) {
+                  cudaStream_t stream, uint32_t outputs = dmv::kOutBoth) {
     using Acc = typename dmv::Traits<T>::Acc;
     static_assert(sizeof(Acc) == sizeof(Out), "accumulator and output widths differ");
+    constexpr bool kIntPath = std::is_same<T, int32_t>::value;
+    if (outputs != dmv::kOutBoth && (kIntPath || batch > 1)) return DUALMV_ERR_UNSUPPORTED;
+    const bool want_q = (outputs & dmv::kOutQ) != 0, want_s = (outputs & dmv::kOutS) != 0;
     dualmv_status st = validate(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ,
-                                s, strideS, batch);
+                                s, strideS, batch, outputs);
     if (st != DUALMV_SUCCESS || batch == 0) return st;
     if (batch == 1) {  // strides are irrelevant for one problem
         strideA = M * lda; strideP = N; strideR = M; strideQ = M; strideS = N;
     }
 
     if (M == 0 || N == 0) {
-        cudaError_t e = zero_fill(reinterpret_cast<Acc *>(q), M, strideQ, batch, stream);
-        if (e == cudaSuccess)
+        cudaError_t e = cudaSuccess;
+        if (want_q) e = zero_fill(reinterpret_cast<Acc *>(q), M, strideQ, batch, stream);
+        if (e == cudaSuccess && want_s)
             e = zero_fill(reinterpret_cast<Acc *>(s), N, strideS, batch, stream);
         return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
     }
@@ -441,6 +455,7 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     prm.q = q; prm.strideQ = strideQ;
     prm.s = s; prm.strideS = strideS;
     prm.M = M; prm.N = N; prm.batch = batch;
+    prm.outputs = outputs;
     prm.band_cols = pl.band_cols;
     prm.bands = pl.bands; prm.stripes = pl.stripes; prm.tiles = pl.tiles;
     prm.grid = pl.grid; prm.max_seg = pl.max_segments;
@@ -463,7 +478,23 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     g_kernel_ev_start = g_kernel_ev_stop = nullptr;
     e = ev_start ? cudaEventRecord(ev_start, stream) : cudaSuccess;
     if (e == cudaSuccess) {
-        if (kind == Kind::kF64e) {
+        if (outputs != dmv::kOutBoth) {
+            if constexpr (!kIntPath) {
+                // Single-sided products (one problem, float or double).
+                const bool only_q = outputs == dmv::kOutQ;
+                if (kind == Kind::kF64e) {
+                    if constexpr (std::is_same<T, double>::value)
+                        e = only_q ? launch_f64e<false, dmv::kOutQ>(map, prm, pl, dev, stream)
+                                   : launch_f64e<false, dmv::kOutS>(map, prm, pl, dev, stream);
+                } else if (kind == Kind::kTma) {
+                    e = only_q ? launch_stream<T, true, false, dmv::kOutQ>(map, prm, pl, dev, stream)
+                               : launch_stream<T, true, false, dmv::kOutS>(map, prm, pl, dev, stream);
+                } else {
+                    e = only_q ? launch_stream<T, false, false, dmv::kOutQ>(map, prm, pl, dev, stream)
+                               : launch_stream<T, false, false, dmv::kOutS>(map, prm, pl, dev, stream);
+                }
+            }
+        } else if (kind == Kind::kF64e) {
             e = three_d ? launch_f64e<true>(map, prm, pl, dev, stream)
                         : launch_f64e<false>(map, prm, pl, dev, stream);
         } else if (kind == Kind::kTma) {
@@ -479,6 +510,89 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     if (e != cudaSuccess) return cuda_fail(e);
     if (ef != cudaSuccess) return cuda_fail(ef);
     return DUALMV_SUCCESS;
+}
+
+// --------------------------------------------- operations built on dualmv --
+
+// Stream-ordered scratch of n elements from the device's pool.
+template <typename T>
+dualmv_status pool_alloc(T **out, int64_t n, cudaStream_t stream) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e);
+    DeviceState *ds = nullptr;
+    e = device_state(dev, &ds);
+    if (e != cudaSuccess) return cuda_fail(e);
+    void *p = nullptr;
+    e = cudaMallocFromPoolAsync(&p, (size_t)(n > 0 ? n : 1) * sizeof(T), ds->pool, stream);
+    if (e != cudaSuccess) {
+        g_last_cuda_error = static_cast<int>(e);
+        return DUALMV_ERR_ALLOC;
+    }
+    *out = static_cast<T *>(p);
+    return DUALMV_SUCCESS;
+}
+
+// GESUMMV (Table 1 / Table 2): tmp = A x, y = B x, y = alpha tmp + beta y.
+// Each matrix is streamed once by a rows-only pass; a small kernel forms y.
+template <typename T>
+dualmv_status gesummv_run(int64_t M, int64_t N, T alpha, const T *A, int64_t lda, T beta,
+                          const T *B, int64_t ldb, const T *x, T *y, cudaStream_t stream) {
+    if (M < 0 || N < 0 || lda < (N > 1 ? N : 1) || ldb < (N > 1 ? N : 1))
+        return DUALMV_ERR_INVALID_VALUE;
+    if (M == 0) return DUALMV_SUCCESS;
+    if (y == nullptr || (N > 0 && (A == nullptr || B == nullptr || x == nullptr)))
+        return DUALMV_ERR_INVALID_VALUE;
+    if (N == 0) {
+        cudaError_t e = zero_fill(y, M, M, 1, stream);
+        return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
+    }
+    if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
+    T *tmp = nullptr;
+    dualmv_status st = pool_alloc(&tmp, M, stream);
+    if (st != DUALMV_SUCCESS) return st;
+    st = run<T, T>(M, N, A, lda, 0, x, 0, nullptr, 0, tmp, 0, nullptr, 0, 1, stream,
+                   dmv::kOutQ);
+    if (st == DUALMV_SUCCESS)
+        st = run<T, T>(M, N, B, ldb, 0, x, 0, nullptr, 0, y, 0, nullptr, 0, 1, stream,
+                       dmv::kOutQ);
+    if (st == DUALMV_SUCCESS) {
+        int64_t blocks = (M + 255) / 256;
+        if (blocks > 4096) blocks = 4096;
+        dmv::axpby_kernel<T><<<(unsigned)blocks, 256, 0, stream>>>(tmp, y, M, alpha, beta);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) st = cuda_fail(e);
+    }
+    cudaError_t ef = cudaFreeAsync(tmp, stream);
+    if (st == DUALMV_SUCCESS && ef != cudaSuccess) st = cuda_fail(ef);
+    return st;
+}
+
+// ATAX (Table 1): tmp = A x, y = A^T tmp: a rows-only pass, then a
+// columns-only pass over the same A.
+template <typename T>
+dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x, T *y,
+                       cudaStream_t stream) {
+    if (M < 0 || N < 0 || lda < (N > 1 ? N : 1)) return DUALMV_ERR_INVALID_VALUE;
+    if (N == 0) return DUALMV_SUCCESS;
+    if (y == nullptr || (M > 0 && (A == nullptr || x == nullptr)))
+        return DUALMV_ERR_INVALID_VALUE;
+    if (M == 0) {
+        cudaError_t e = zero_fill(y, N, N, 1, stream);
+        return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
+    }
+    if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
+    T *tmp = nullptr;
+    dualmv_status st = pool_alloc(&tmp, M, stream);
+    if (st != DUALMV_SUCCESS) return st;
+    st = run<T, T>(M, N, A, lda, 0, x, 0, nullptr, 0, tmp, 0, nullptr, 0, 1, stream,
+                   dmv::kOutQ);
+    if (st == DUALMV_SUCCESS)
+        st = run<T, T>(M, N, A, lda, 0, nullptr, 0, tmp, 0, nullptr, 0, y, 0, 1, stream,
+                       dmv::kOutS);
+    cudaError_t ef = cudaFreeAsync(tmp, stream);
+    if (st == DUALMV_SUCCESS && ef != cudaSuccess) st = cuda_fail(ef);
+    return st;
 }
 
 // ------------------------------------------------- no-allocation variant --
@@ -562,6 +676,7 @@ dualmv_status run_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,
     prm.q = q; prm.strideQ = M;
     prm.s = s; prm.strideS = N;
     prm.M = M; prm.N = N; prm.batch = 1;
+    prm.outputs = dmv::kOutBoth;
     prm.band_cols = pl.band_cols;
     prm.bands = pl.bands; prm.stripes = pl.stripes; prm.tiles = pl.tiles;
     prm.grid = pl.grid; prm.max_seg = pl.max_segments;
@@ -627,6 +742,30 @@ dualmv_status dualmv_i32_strided_batched(int64_t M, int64_t N, const int32_t *A,
                                          dualmv_stream_t stream) {
     return run<int32_t, int64_t>(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ,
                                  s, strideS, batch, reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_gesummv_f32(int64_t M, int64_t N, float alpha, const float *A,
+                                 int64_t lda, float beta, const float *B, int64_t ldb,
+                                 const float *x, float *y, dualmv_stream_t stream) {
+    return gesummv_run<float>(M, N, alpha, A, lda, beta, B, ldb, x, y,
+                              reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_gesummv_f64(int64_t M, int64_t N, double alpha, const double *A,
+                                 int64_t lda, double beta, const double *B, int64_t ldb,
+                                 const double *x, double *y, dualmv_stream_t stream) {
+    return gesummv_run<double>(M, N, alpha, A, lda, beta, B, ldb, x, y,
+                               reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_atax_f32(int64_t M, int64_t N, const float *A, int64_t lda,
+                              const float *x, float *y, dualmv_stream_t stream) {
+    return atax_run<float>(M, N, A, lda, x, y, reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_atax_f64(int64_t M, int64_t N, const double *A, int64_t lda,
+                              const double *x, double *y, dualmv_stream_t stream) {
+    return atax_run<double>(M, N, A, lda, x, y, reinterpret_cast<cudaStream_t>(stream));
 }
 
 dualmv_status dualmv_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,

@@ -164,9 +164,11 @@ struct F64eLayout {
 //
 // W consumer warps x RPW rows per warp per tile; lane l holds columns
 // 2l, 2l+1 (+64, +128, +192) of the 256-column band (four double2 vectors).
-template <int W, int RPW, int STAGES, int BAND, bool kBatched3d>
+template <int W, int RPW, int STAGES, int BAND, bool kBatched3d, int kOut = kOutBoth>
 __global__ void __launch_bounds__((W + 1) * 32, 1)
 dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
+    constexpr bool kQ = (kOut & kOutQ) != 0;  // row sums q = A p
+    constexpr bool kS = (kOut & kOutS) != 0;  // column sums s = A^T r
     using T = double;
     using Acc = double;
     using Vec = double2;
@@ -294,7 +296,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     T r_next = T(0);
     {
         const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
-        if (lane < RPW && row < prm.M) r_next = rg[cur.b * prm.strideR + row];
+        if (kS && lane < RPW && row < prm.M) r_next = rg[cur.b * prm.strideR + row];
     }
     int stage = 0;
     uint32_t phase = 0;
@@ -308,13 +310,13 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         const int64_t row0 = stripe * BM + (int64_t)warp * RPW;
         const T rmine = r_next;
         cur.advance(S, prm.bands);
-        if (k + 1 < ntiles) {
+        if (kS && k + 1 < ntiles) {
             const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
             r_next = (lane < RPW && row < prm.M) ? rg[cur.b * prm.strideR + row] : T(0);
         }
 
-        if (k == 0 || stripe == 0) {  // new segment: split this band's p
-            seg_start_stripe = stripe;
+        if (k == 0 || stripe == 0) seg_start_stripe = stripe;
+        if (kQ && (k == 0 || stripe == 0)) {  // new segment: split this band's p
             const T *pb = pg + b * prm.strideP;
             p_bad = false;
 #pragma unroll
@@ -332,7 +334,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         float rh_mine, rl_mine;
         uint32_t r_habs;
         split_f64(rmine, rh_mine, rl_mine, r_habs);
-        const bool r_bad = !f64e_in_range(rmine);
+        const bool r_bad = kS && !f64e_in_range(rmine);
 
         const int slot = warp * STAGES + stage;
         if (ok) ok = mbar_wait_bounded(smem_u32(&full_bar[slot]), phase);
@@ -341,6 +343,8 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
 
         // Fast path: double-float arithmetic with a cheap range bound.
         DF q[RPW];
+#pragma unroll
+        for (int i = 0; i < RPW; ++i) q[i].s = q[i].c = 0.f;
         DF tacc[LANE_COLS];
         double tnat[kNativeCols > 0 ? kNativeCols : 1];
 #pragma unroll
@@ -366,7 +370,8 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                     uint32_t habs;
                     split_f64(vget(a[v], e), ah, al, habs);
                     span = max(span, habs - kF64eLoBits);
-                    if (ce < kFirstNative) {
+                    if (!kS) {
+                    } else if (ce < kFirstNative) {
                         float p0, p1;
                         df_prod(ah, al, rh, rl, p0, p1);
                         if (i == 0) {
@@ -379,9 +384,10 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                         tnat[ce - kFirstNative] =
                             fma(vget(a[v], e), rd, tnat[ce - kFirstNative]);
                     }
-                    df_prod(ah, al, ph[ce], pl[ce], qp[ce].s, qp[ce].c);
+                    if constexpr (kQ) df_prod(ah, al, ph[ce], pl[ce], qp[ce].s, qp[ce].c);
                 }
-            if constexpr (LANE_COLS == 8)
+            if constexpr (!kQ) {
+            } else if constexpr (LANE_COLS == 8)
                 q[i] = df_add(df_add(df_add(qp[0], qp[1]), df_add(qp[2], qp[3])),
                               df_add(df_add(qp[4], qp[5]), df_add(qp[6], qp[7])));
             else
@@ -389,7 +395,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         }
         // Anything suspicious in this warp's rows (zeros included)?
         const bool rows_r_bad = __any_sync(0xffffffffu, lane < RPW && r_bad);
-        bool need_fp64 = rows_r_bad || __any_sync(0xffffffffu, p_bad);
+        bool need_fp64 = rows_r_bad || __any_sync(0xffffffffu, kQ && p_bad);
         if (!need_fp64 && __any_sync(0xffffffffu, span >= kF64eSpanBits)) {
             // Exact re-check: zeros are fine, anything else out of range is not.
             bool bad = false;
@@ -408,8 +414,8 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         if (!need_fp64) {
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&empty_bar[slot]));
-            warp_rows_reduce_df<RPW>(q, lane);
-            if (butterfly_writer<RPW>(lane)) {
+            if constexpr (kQ) warp_rows_reduce_df<RPW>(q, lane);
+            if (kQ && butterfly_writer<RPW>(lane)) {
                 const int64_t row = row0 + butterfly_row<RPW>(lane);
                 if (row < prm.M) {
                     const double qv = df_to_double(q[0]);
@@ -432,7 +438,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
 #pragma unroll
                 for (int e = 0; e < VE; ++e) {
                     const int64_t col = col0 + lane_col<T>(v, lane, e);
-                    pd[v * VE + e] = col < prm.N ? pb[col] : 0.0;
+                    pd[v * VE + e] = (kQ && col < prm.N) ? pb[col] : 0.0;
                 }
             double qd[RPW];
             double td[LANE_COLS];
@@ -457,8 +463,8 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&empty_bar[slot]));
-            warp_rows_reduce<RPW>(qd, lane);
-            if (butterfly_writer<RPW>(lane)) {
+            if constexpr (kQ) warp_rows_reduce<RPW>(qd, lane);
+            if (kQ && butterfly_writer<RPW>(lane)) {
                 const int64_t row = row0 + butterfly_row<RPW>(lane);
                 if (row < prm.M) {
                     if (prm.bands == 1)
@@ -478,53 +484,55 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             phase ^= 1u;
         }
 
-        const bool seg_end = (stripe == S - 1 || k == ntiles - 1);
-        if (++ngrp == kGroupTiles || seg_end) {
-#pragma unroll
-            for (int v = 0; v < VPL; ++v)
-#pragma unroll
-                for (int e = 0; e < VE; ++e) {
-                    const int ce = v * VE + e;
-                    if (ce < kFirstNative) {
-                        segp[lane_col<T>(v, lane, e)] += df_to_double(grp[ce]);
-                        grp[ce].s = grp[ce].c = 0.f;
+        if constexpr (kS) {
+            const bool seg_end = (stripe == S - 1 || k == ntiles - 1);
+            if (++ngrp == kGroupTiles || seg_end) {
+    #pragma unroll
+                for (int v = 0; v < VPL; ++v)
+    #pragma unroll
+                    for (int e = 0; e < VE; ++e) {
+                        const int ce = v * VE + e;
+                        if (ce < kFirstNative) {
+                            segp[lane_col<T>(v, lane, e)] += df_to_double(grp[ce]);
+                            grp[ce].s = grp[ce].c = 0.f;
+                        }
                     }
-                }
-            ngrp = 0;
-        }
-        if (seg_end) {
-#pragma unroll
-            for (int v = 0; v < VPL; ++v)
-#pragma unroll
-                for (int e = 0; e < VE; ++e) {
-                    const int ce = v * VE + e;
-                    if (ce >= kFirstNative) {
-                        segp[lane_col<T>(v, lane, e)] += snat[ce - kFirstNative];
-                        snat[ce - kFirstNative] = 0.0;
-                    }
-                }
-        }
-
-        if (seg_end) {  // segment end: flush s
-            named_barrier(1, nthreads_c);
-            const bool whole_band = (seg_start_stripe == 0 && stripe == S - 1);
-            for (int col = threadIdx.x; col < BAND; col += nthreads_c) {
-                Acc acc = scratch[col];
-#pragma unroll
-                for (int w = 1; w < W; ++w) acc = acc + scratch[w * BAND + col];
-                if (whole_band) {
-                    if (col0 + col < prm.N)
-                        static_cast<Acc *>(prm.s)[b * prm.strideS + col0 + col] = acc;
-                } else {
-                    static_cast<Acc *>(prm.s_ws)[((c * prm.max_seg) + (g - g_first)) *
-                                                     BAND + col] = acc;
-                }
+                ngrp = 0;
             }
-            named_barrier(1, nthreads_c);
-#pragma unroll
-            for (int v = 0; v < VPL; ++v)
-#pragma unroll
-                for (int e = 0; e < VE; ++e) segp[lane_col<T>(v, lane, e)] = 0.0;
+            if (seg_end) {
+    #pragma unroll
+                for (int v = 0; v < VPL; ++v)
+    #pragma unroll
+                    for (int e = 0; e < VE; ++e) {
+                        const int ce = v * VE + e;
+                        if (ce >= kFirstNative) {
+                            segp[lane_col<T>(v, lane, e)] += snat[ce - kFirstNative];
+                            snat[ce - kFirstNative] = 0.0;
+                        }
+                    }
+            }
+
+            if (seg_end) {  // segment end: flush s
+                named_barrier(1, nthreads_c);
+                const bool whole_band = (seg_start_stripe == 0 && stripe == S - 1);
+                for (int col = threadIdx.x; col < BAND; col += nthreads_c) {
+                    Acc acc = scratch[col];
+    #pragma unroll
+                    for (int w = 1; w < W; ++w) acc = acc + scratch[w * BAND + col];
+                    if (whole_band) {
+                        if (col0 + col < prm.N)
+                            static_cast<Acc *>(prm.s)[b * prm.strideS + col0 + col] = acc;
+                    } else {
+                        static_cast<Acc *>(prm.s_ws)[((c * prm.max_seg) + (g - g_first)) *
+                                                         BAND + col] = acc;
+                    }
+                }
+                named_barrier(1, nthreads_c);
+    #pragma unroll
+                for (int v = 0; v < VPL; ++v)
+    #pragma unroll
+                    for (int e = 0; e < VE; ++e) segp[lane_col<T>(v, lane, e)] = 0.0;
+            }
         }
     }
 }

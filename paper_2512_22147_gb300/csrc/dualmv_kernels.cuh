@@ -47,6 +47,13 @@
 
 namespace dmv {
 
+// What a stream kernel computes: the row sums q = A p, the column sums
+// s = A^T r, or both (the dual product).  The single-sided modes serve the
+// operations built from one matrix-vector product (ATAX, GESUMMV).
+constexpr int kOutQ = 1;
+constexpr int kOutS = 2;
+constexpr int kOutBoth = kOutQ | kOutS;
+
 constexpr int kBandCols = 256;          // columns per band = TMA box width
 constexpr int kLaneCols = kBandCols / 32;  // columns per lane = 8
 constexpr int kGroupTiles = 16;         // tiles summed before the segment sum
@@ -268,6 +275,7 @@ struct Params {
     void *s;
     int64_t strideS;
     int64_t M, N, batch;
+    uint32_t outputs;   // kOutQ | kOutS: which of q and s this call computes
     int64_t band_cols;  // columns per band (the stream kernel's tile width)
     int64_t bands, stripes, tiles, grid, max_seg;
     void *q_ws;  // [batch][bands][M] band partials of q (bands > 1 only)
@@ -330,10 +338,13 @@ struct SmemLayout {
 // Template: element type T, W consumer warps, RPW rows per warp per tile,
 // STAGES ring depth, kTma = TMA producer (else plain loads), kBatched3d =
 // 3-D tensor map (batch as the outer coordinate).
-template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d>
+template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d,
+          int kOut = kOutBoth>
 __global__ void __launch_bounds__((W + (kTma ? 1 : 0)) * 32, 1)
 dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
     using Acc = typename Traits<T>::Acc;
+    constexpr bool kQ = (kOut & kOutQ) != 0;  // row sums q = A p
+    constexpr bool kS = (kOut & kOutS) != 0;  // column sums s = A^T r
     // Integer sums are exact modulo 2^64 in any order, so the int32 path adds
     // its band and segment partials straight into q and s with atomics (the
     // result is the same bits on every run) and needs no workspace and no
@@ -447,7 +458,7 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
     // r for this warp's RPW rows of the next tile (lane i < RPW holds row
     // row0 + i), loaded one tile ahead so its latency hides behind a tile.
     T r_next = T(0);
-    {
+    if constexpr (kS) {
         const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
         if (lane < RPW && row < prm.M) r_next = rg[cur.b * prm.strideR + row];
     }
@@ -464,13 +475,13 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
         const int64_t row0 = stripe * BM + (int64_t)warp * RPW;
         const T rmine = r_next;
         cur.advance(S, prm.bands);
-        if (k + 1 < ntiles) {
+        if (kS && k + 1 < ntiles) {
             const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
             r_next = (lane < RPW && row < prm.M) ? rg[cur.b * prm.strideR + row] : T(0);
         }
 
-        if (k == 0 || stripe == 0) {  // a new segment: this band's p
-            seg_start_stripe = stripe;
+        if (k == 0 || stripe == 0) seg_start_stripe = stripe;
+        if (kQ && (k == 0 || stripe == 0)) {  // a new segment: this band's p
             const T *pb = pg + b * prm.strideP;
 #pragma unroll
             for (int v = 0; v < VPL; ++v)
@@ -513,15 +524,15 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
                     else a[v] = Vec{tmp[0], tmp[1]};
                 }
             }
-            const T ri = __shfl_sync(0xffffffffu, rmine, i);
+            const T ri = kS ? __shfl_sync(0xffffffffu, rmine, i) : T(0);
             Acc dot = Acc(0);
 #pragma unroll
             for (int v = 0; v < VPL; ++v)
 #pragma unroll
                 for (int e = 0; e < VE; ++e) {
                     const T av = vget(a[v], e);
-                    dot = mul_acc(av, pv[v * VE + e], dot);
-                    tacc[v * VE + e] = mul_acc(av, ri, tacc[v * VE + e]);
+                    if constexpr (kQ) dot = mul_acc(av, pv[v * VE + e], dot);
+                    if constexpr (kS) tacc[v * VE + e] = mul_acc(av, ri, tacc[v * VE + e]);
                 }
             qp[i] = dot;
         }
@@ -535,8 +546,8 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
         }
 
         // q: complete band partial of each of this warp's rows.
-        warp_rows_reduce<RPW>(qp, lane);
-        if (butterfly_writer<RPW>(lane)) {
+        if constexpr (kQ) warp_rows_reduce<RPW>(qp, lane);
+        if (kQ && butterfly_writer<RPW>(lane)) {
             const int64_t row = row0 + butterfly_row<RPW>(lane);
             if (row < prm.M) {
                 if (prm.bands == 1) {
@@ -552,51 +563,53 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
         }
 
         // s: tile -> group -> segment accumulation.
-#pragma unroll
-        for (int e = 0; e < kLaneCols; ++e) grp[e] = grp[e] + tacc[e];
-        if (++ngrp == kGroupTiles) {
-#pragma unroll
-            for (int e = 0; e < kLaneCols; ++e) {
-                seg[e] = seg[e] + grp[e];
-                grp[e] = Acc(0);
-            }
-            ngrp = 0;
-        }
-
-        if (stripe == S - 1 || k == ntiles - 1) {  // segment end: flush s
-#pragma unroll
-            for (int e = 0; e < kLaneCols; ++e) seg[e] = seg[e] + grp[e];
-            Acc *sw = scratch + warp * kBandCols;
-#pragma unroll
-            for (int v = 0; v < VPL; ++v)
-#pragma unroll
-                for (int e = 0; e < VE; ++e) sw[lane_col<T>(v, lane, e)] = seg[v * VE + e];
-            named_barrier(1, nthreads_c);
-            const bool whole_band = (seg_start_stripe == 0 && stripe == S - 1);
-            for (int col = threadIdx.x; col < kBandCols; col += nthreads_c) {
-                Acc acc = scratch[col];
-#pragma unroll
-                for (int w = 1; w < W; ++w) acc = acc + scratch[w * kBandCols + col];
-                if (whole_band) {
-                    if (col0 + col < prm.N) {
-                        Acc *so = static_cast<Acc *>(prm.s);
-                        so[b * prm.strideS + col0 + col] = acc;
-                    }
-                } else if constexpr (kAtomicOut) {
-                    if (col0 + col < prm.N)
-                        atomicAdd(static_cast<Acc *>(prm.s) + b * prm.strideS + col0 + col, acc);
-                } else {
-                    Acc *sws = static_cast<Acc *>(prm.s_ws);
-                    sws[((c * prm.max_seg) + (g - g_first)) * kBandCols + col] = acc;
+        if constexpr (kS) {
+    #pragma unroll
+            for (int e = 0; e < kLaneCols; ++e) grp[e] = grp[e] + tacc[e];
+            if (++ngrp == kGroupTiles) {
+    #pragma unroll
+                for (int e = 0; e < kLaneCols; ++e) {
+                    seg[e] = seg[e] + grp[e];
+                    grp[e] = Acc(0);
                 }
+                ngrp = 0;
             }
-            named_barrier(1, nthreads_c);
-#pragma unroll
-            for (int e = 0; e < kLaneCols; ++e) {
-                grp[e] = Acc(0);
-                seg[e] = Acc(0);
+
+            if (stripe == S - 1 || k == ntiles - 1) {  // segment end: flush s
+    #pragma unroll
+                for (int e = 0; e < kLaneCols; ++e) seg[e] = seg[e] + grp[e];
+                Acc *sw = scratch + warp * kBandCols;
+    #pragma unroll
+                for (int v = 0; v < VPL; ++v)
+    #pragma unroll
+                    for (int e = 0; e < VE; ++e) sw[lane_col<T>(v, lane, e)] = seg[v * VE + e];
+                named_barrier(1, nthreads_c);
+                const bool whole_band = (seg_start_stripe == 0 && stripe == S - 1);
+                for (int col = threadIdx.x; col < kBandCols; col += nthreads_c) {
+                    Acc acc = scratch[col];
+    #pragma unroll
+                    for (int w = 1; w < W; ++w) acc = acc + scratch[w * kBandCols + col];
+                    if (whole_band) {
+                        if (col0 + col < prm.N) {
+                            Acc *so = static_cast<Acc *>(prm.s);
+                            so[b * prm.strideS + col0 + col] = acc;
+                        }
+                    } else if constexpr (kAtomicOut) {
+                        if (col0 + col < prm.N)
+                            atomicAdd(static_cast<Acc *>(prm.s) + b * prm.strideS + col0 + col, acc);
+                    } else {
+                        Acc *sws = static_cast<Acc *>(prm.s_ws);
+                        sws[((c * prm.max_seg) + (g - g_first)) * kBandCols + col] = acc;
+                    }
+                }
+                named_barrier(1, nthreads_c);
+    #pragma unroll
+                for (int e = 0; e < kLaneCols; ++e) {
+                    grp[e] = Acc(0);
+                    seg[e] = Acc(0);
+                }
+                ngrp = 0;
             }
-            ngrp = 0;
         }
     }
 }
@@ -622,7 +635,7 @@ dualmv_combine_kernel(const Params prm, int64_t q_blocks, int q_chunks) {
     __shared__ Acc part[256];
     const Acc *qw = static_cast<const Acc *>(prm.q_ws);
     const Acc *sw = static_cast<const Acc *>(prm.s_ws);
-    if ((int64_t)blockIdx.x < q_blocks) {
+    if ((int64_t)blockIdx.x < q_blocks) {  // (q_blocks is 0 unless q is computed)
         const int C = q_chunks, R = 256 / C;
         const int x = threadIdx.x % R, y = threadIdx.x / R;
         const int64_t idx = (int64_t)blockIdx.x * R + x;
@@ -688,6 +701,14 @@ __global__ void dualmv_zero_outputs_kernel(Acc *q, int64_t M, int64_t strideQ, A
             s[b * strideS + j] = Acc(0);
         }
     }
+}
+
+// y = alpha * t + beta * y (the GESUMMV epilogue).
+template <typename T>
+__global__ void axpby_kernel(const T *t, T *y, int64_t n, T alpha, T beta) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        y[i] = alpha * t[i] + beta * y[i];
 }
 
 // Zero-fill of strided outputs (empty problems).

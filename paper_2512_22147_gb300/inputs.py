@@ -36,6 +36,7 @@ class Workload:
     dist: str           # "uniform" | "normal" | "int8"
     seed: int
     batch: int = 0      # 0 = single problem; >= 1 = strided batch
+    op: str = "bicg"    # "bicg" (dual product) | "gesummv" | "atax"
 
     @property
     def batched(self) -> bool:
@@ -46,9 +47,15 @@ class Workload:
         return max(1, self.batch)
 
     def bytes_counted(self) -> int:
-        """Bytes of the logical A (padding excluded), of p and r read, and of
-        q and s written: the numerator of the effective-bandwidth metric."""
+        """Bytes of the logical matrices (padding excluded) read once, of the
+        input vectors and of the outputs: the numerator of the
+        effective-bandwidth metric.  Dual product: A, p, r, q, s.  GESUMMV:
+        A, B, x, y.  ATAX: A (once: the least any algorithm must move), x, y."""
         e, o = ELEM_BYTES[self.dtype], OUT_BYTES[self.dtype]
+        if self.op == "gesummv":
+            return 2 * self.M * self.N * e + self.N * e + self.M * o
+        if self.op == "atax":
+            return self.M * self.N * e + self.N * e + self.N * o
         per = (self.M * self.N * e + (self.M + self.N) * e
                + (self.M + self.N) * o)
         return per * self.nbatch
@@ -69,6 +76,20 @@ WORKLOADS = {
                  "int8", 3),
         Workload("f32_batch256_2048x2048", "f32", 2048, 2048, 2048, "uniform",
                  4, batch=256),
+    )
+}
+
+
+# Workloads of the two further PolyBench kernels built on the same products
+# (GESUMMV and ATAX, Table 1), sized like the dual product's square fp32
+# workload so that every matrix is far larger than L2.
+OP_WORKLOADS = {
+    w.name: w for w in (
+        Workload("gesummv_f32_16384x16384", "f32", 16384, 16384, 16384, "uniform", 5,
+                 op="gesummv"),
+        Workload("gesummv_f64_8192x8192", "f64", 8192, 8192, 8192, "normal", 6, op="gesummv"),
+        Workload("atax_f32_16384x16384", "f32", 16384, 16384, 16384, "uniform", 7, op="atax"),
+        Workload("atax_f64_16384x8192", "f64", 16384, 8192, 8192, "normal", 8, op="atax"),
     )
 }
 
@@ -130,3 +151,44 @@ def empty_outputs(w: Workload, device: str | torch.device = "cpu"):
     q = torch.empty(lead + (w.M,), dtype=t, device=device)
     s = torch.empty(lead + (w.N,), dtype=t, device=device)
     return q, s
+
+
+def _matrix(w: Workload, g: torch.Generator, dev) -> torch.Tensor:
+    A = torch.empty((w.M, w.lda), dtype=DTYPES[w.dtype], device=dev)
+    if w.lda > w.N:
+        A[:, w.N:] = _sentinel(w.dtype)
+    view = A[:, : w.N]
+    if view.numel():
+        if view.is_contiguous():
+            _fill(view, w.dist, g)
+        else:
+            tmp = torch.empty(view.shape, dtype=A.dtype, device=dev)
+            _fill(tmp, w.dist, g)
+            view.copy_(tmp)
+    return A
+
+
+def _vector(n: int, w: Workload, g: torch.Generator, dev) -> torch.Tensor:
+    v = torch.empty(n, dtype=DTYPES[w.dtype], device=dev)
+    if n:
+        _fill(v, w.dist, g)
+    return v
+
+
+def generate_gesummv(w: Workload, device: str | torch.device = "cpu"):
+    """``(A, B, x)`` for GESUMMV: one generator fills A, then B, then x."""
+    dev = torch.device(device)
+    g = torch.Generator(device=dev)
+    g.manual_seed(w.seed)
+    A = _matrix(w, g, dev)
+    B = _matrix(w, g, dev)
+    return A, B, _vector(w.N, w, g, dev)
+
+
+def generate_atax(w: Workload, device: str | torch.device = "cpu"):
+    """``(A, x)`` for ATAX: one generator fills A, then x."""
+    dev = torch.device(device)
+    g = torch.Generator(device=dev)
+    g.manual_seed(w.seed)
+    A = _matrix(w, g, dev)
+    return A, _vector(w.N, w, g, dev)

@@ -7,10 +7,10 @@ or a published error bound.  ``tests/test_oracle_pins.py`` runs them on the
 real oracle; ``tests/test_oracle_mutants.py`` runs them on copies of the
 oracle with a planted mistake and expects at least one to fail.
 
-The operation is the BICG kernel of the paper (Table 1 and Table 2):
-q = A p and s = A^T r.  The paper prints no worked example for it, so no
-printed values can serve as golden data; everything here is derived from
-the definition.
+The operations are the BICG kernel of the paper (Table 1 and Table 2):
+q = A p and s = A^T r, and the GESUMMV and ATAX kernels of the same tables.
+The paper prints no worked example for any of them, so no printed values
+can serve as golden data; everything here is derived from the definitions.
 """
 from __future__ import annotations
 
@@ -268,11 +268,110 @@ def pin_trimmed_mean(lib):
         raise AssertionError("R <= 2k accepted")
 
 
+# ------------------------------------------------------- GESUMMV, ATAX --
+
+def _exact_dot_rows(A, x, N):
+    M = A.shape[0]
+    F = [[Fraction(float(A[i, j])) for j in range(N)] for i in range(M)]
+    X = [Fraction(float(v)) for v in x]
+    dots = [sum((F[i][j] * X[j] for j in range(N)), Fraction(0)) for i in range(M)]
+    mags = [sum((abs(F[i][j] * X[j]) for j in range(N)), Fraction(0)) for i in range(M)]
+    return F, dots, mags
+
+
+def pin_gesummv_bruteforce(lib, seed=14, cases=30):
+    """y = alpha A x + beta B x against exact rationals, within
+    (gamma_(N+2) + 3u) (|alpha| sum|A||x| + |beta| sum|B||x|) (a
+    double-accumulated or Dot2 sum, then two products and one addition)."""
+    rng = np.random.default_rng(seed)
+    for case in range(cases):
+        dt = np.float32 if case % 2 == 0 else np.float64
+        M, N = (int(v) for v in rng.integers(0, 7, size=2))
+        ea, eb = (int(v) for v in rng.integers(0, 4, size=2))
+        A = _padded(rng, M, N, ea, dt, lambda g, sh: _rand_float(g, sh, dt))
+        B = _padded(rng, M, N, eb, dt, lambda g, sh: _rand_float(g, sh, dt))
+        x = _rand_float(rng, N, dt)
+        alpha, beta = 0.75, -1.5
+        y = oracle.gesummv(A, B, x, alpha, beta, N=N, lib=lib)
+        _, da, ma = _exact_dot_rows(A, x, N)
+        _, db, mb = _exact_dot_rows(B, x, N)
+        for i in range(M):
+            assert np.isfinite(y[i]), "padding read"
+            want = Fraction(alpha) * da[i] + Fraction(beta) * db[i]
+            mag = abs(Fraction(alpha)) * ma[i] + abs(Fraction(beta)) * mb[i]
+            assert abs(Fraction(float(y[i])) - want) <= (gamma(N + 2) + 3 * U53) * mag, (M, N, i)
+
+
+def pin_gesummv_closed_forms(lib):
+    """B = 0 gives alpha (A x) exactly (alpha a power of two); A = B with
+    alpha = beta = 1 gives exactly twice A x; an ill-conditioned row that
+    only compensated sums get right."""
+    rng = np.random.default_rng(15)
+    for dt in (np.float32, np.float64):
+        A = rng.uniform(-1, 1, (9, 13)).astype(dt)
+        x = rng.uniform(-1, 1, 13).astype(dt)
+        ax, _ = oracle.dualmv(A, x, np.zeros(9, dt), lib=lib)
+        y = oracle.gesummv(A, np.zeros_like(A), x, 4.0, 3.0, lib=lib)
+        assert (y == 4.0 * ax).all()
+        y = oracle.gesummv(A, A.copy(), x, 1.0, 1.0, lib=lib)
+        assert (y == 2.0 * ax).all()
+    big = 2.0 ** 60
+    A = np.array([[big, 1.0, -big]])
+    y = oracle.gesummv(A, -A, np.ones(3), 1.0, 0.5, lib=lib)
+    assert y[0] == 0.5, y
+
+
+def pin_atax_bruteforce(lib, seed=16, cases=30):
+    """y = A^T (A x) against exact rationals.  Bound per output j, with
+    D_j = sum_i |A_ij| sum_k |A_ik||x_k|: (gamma_N + gamma_M) D_j for the
+    double-accumulated float oracle, (4u + 2 gamma^2) D_j for Dot2 with tmp
+    rounded to double."""
+    rng = np.random.default_rng(seed)
+    for case in range(cases):
+        dt = np.float32 if case % 2 == 0 else np.float64
+        M, N, extra = (int(v) for v in rng.integers(0, 7, size=3))
+        A = _padded(rng, M, N, extra, dt, lambda g, sh: _rand_float(g, sh, dt))
+        x = _rand_float(rng, N, dt)
+        y = oracle.atax(A, x, N=N, lib=lib)
+        F, tmp, mags = _exact_dot_rows(A, x, N)
+        for j in range(N):
+            assert np.isfinite(y[j]), "padding read"
+            want = sum((F[i][j] * tmp[i] for i in range(M)), Fraction(0))
+            D = sum((abs(F[i][j]) * mags[i] for i in range(M)), Fraction(0))
+            g = max(M, N, 1)
+            bound = (2 * gamma(g)) * D if dt == np.float32 else (4 * U53 + 2 * gamma(g) ** 2) * D
+            assert abs(Fraction(float(y[j])) - want) <= bound, (M, N, j)
+
+
+def pin_atax_closed_forms(lib):
+    """A a permutation: y = x exactly; A = u v^T with small integers:
+    y = v (u.u)(v.x) exactly."""
+    rng = np.random.default_rng(17)
+    perm = rng.permutation(11)
+    for dt in (np.float32, np.float64):
+        P = np.zeros((11, 11), dt)
+        P[np.arange(11), perm] = 1.0
+        x = rng.uniform(-1, 1, 11).astype(dt)
+        assert (oracle.atax(P, x, lib=lib) == x.astype(np.float64)).all()
+        u = rng.integers(-8, 9, 7)
+        v = rng.integers(-8, 9, 5)
+        xi = rng.integers(-8, 9, 5)
+        A = np.outer(u, v).astype(dt)
+        want = v * int(u @ u) * int(v @ xi)
+        assert (oracle.atax(A, xi.astype(dt), lib=lib) == want).all()
+    # A row whose product with x cancels: tmp = 2^60 + 1 - 2^60 = 1 needs the
+    # compensated sum; then y = A^T tmp is that row itself.
+    big = 2.0 ** 60
+    A = np.array([[big, 1.0, -big]])
+    assert (oracle.atax(A, np.ones(3), lib=lib) == A[0]).all()
+
+
 ALL_PINS = [
     pin_bruteforce_f32, pin_bruteforce_f64, pin_bruteforce_i32,
     pin_wraparound_i32, pin_dot2_cancellation, pin_identity, pin_rank_one,
     pin_adjoint, pin_power_of_two_scaling, pin_shapes_and_empty, pin_absdot,
-    pin_trimmed_mean,
+    pin_trimmed_mean, pin_gesummv_bruteforce, pin_gesummv_closed_forms,
+    pin_atax_bruteforce, pin_atax_closed_forms,
 ]
 
 

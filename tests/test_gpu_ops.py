@@ -1,0 +1,132 @@
+"""GESUMMV and ATAX (Table 1 of the paper; GESUMMV also Table 2) on the GPU
+through the C ABI, against the CPU oracle.
+
+Tolerance, as for the dual product, relative to the magnitude of each
+output's terms: GESUMMV |y_i - y^_i| <= tol (|alpha| sum_j |A_ij||x_j| +
+|beta| sum_j |B_ij||x_j|); ATAX |y_j - y^_j| <= tol sum_i |A_ij| sum_k
+|A_ik||x_k| (the error of tmp = A x propagates through A^T).  tol = 1e-5
+(f32) and 1e-12 (f64)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2512_22147_gb300 as dm
+from paper_2512_22147_gb300 import inputs
+from parity import TOL, scaled_error
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+TAGS = {"f32": torch.float32, "f64": torch.float64}
+
+
+@pytest.fixture(params=[dm.DUALMV_PATH_TMA, dm.DUALMV_PATH_DIRECT], ids=["tma", "direct"])
+def path(request):
+    old = dm.dualmv_set_path(request.param)
+    yield request.param
+    dm.dualmv_set_path(old)
+
+
+def _w(op, dtype, M, N, lda, seed):
+    dist = "uniform" if dtype == "f32" else "normal"
+    return inputs.Workload(op, dtype, M, N, lda, dist, seed, op=op)
+
+
+def check_gesummv(A, B, x, N, alpha, beta, dtype):
+    y = dm.gesummv(A[:, :N], B[:, :N], x, alpha=alpha, beta=beta)
+    torch.cuda.synchronize()
+    An, Bn, xn = A.cpu().numpy(), B.cpu().numpy(), x.cpu().numpy()
+    want = oracle.gesummv(An, Bn, xn, alpha, beta, N=N)
+    qa, _ = oracle.absdot(An, xn, np.zeros(An.shape[0], An.dtype), N=N)
+    qb, _ = oracle.absdot(Bn, xn, np.zeros(Bn.shape[0], Bn.dtype), N=N)
+    den = abs(alpha) * qa + abs(beta) * qb
+    err = scaled_error(y.cpu().numpy(), want, den)
+    assert err <= TOL[dtype], err
+    return err
+
+
+def check_atax(A, x, N, dtype):
+    y = dm.atax(A[:, :N], x)
+    torch.cuda.synchronize()
+    An, xn = A.cpu().numpy(), x.cpu().numpy()
+    want = oracle.atax(An, xn, N=N)
+    qa, _ = oracle.absdot(An, xn, np.zeros(An.shape[0], An.dtype), N=N)
+    _, den = oracle.absdot(An.astype(np.float64), np.zeros(N), qa, N=N)
+    err = scaled_error(y.cpu().numpy(), want, den)
+    assert err <= TOL[dtype], err
+    return err
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+@pytest.mark.parametrize("M,N,pad", [(1000, 3000, 0), (3001, 257, 5), (1, 1, 0), (77, 1000, 3),
+                                     (2048, 64, 0)])
+def test_gesummv_matches_oracle(dtype, M, N, pad, path):
+    A, B, x = inputs.generate_gesummv(_w("gesummv", dtype, M, N, N + pad, M + N), DEV)
+    check_gesummv(A, B, x, N, 0.75, -1.25, dtype)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+@pytest.mark.parametrize("M,N,pad", [(1000, 3000, 0), (3001, 257, 5), (1, 1, 0), (77, 1000, 3),
+                                     (2048, 64, 0)])
+def test_atax_matches_oracle(dtype, M, N, pad, path):
+    A, x = inputs.generate_atax(_w("atax", dtype, M, N, N + pad, 3 * M + N), DEV)
+    check_atax(A, x, N, dtype)
+
+
+@pytest.mark.parametrize("name", list(inputs.OP_WORKLOADS))
+def test_op_workloads_full_size(name):
+    w = inputs.OP_WORKLOADS[name]
+    if w.op == "gesummv":
+        A, B, x = inputs.generate_gesummv(w, DEV)
+        err = check_gesummv(A, B, x, w.N, 1.5, 1.2, w.dtype)
+        del B
+    else:
+        A, x = inputs.generate_atax(w, DEV)
+        err = check_atax(A, x, w.N, w.dtype)
+    print(f"{name}: max scaled error {err:.3e}")
+    del A, x
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_gesummv_closed_forms(dtype, path):
+    """Both row passes are deterministic, so with B = A and alpha = beta = 1
+    the result is exactly twice the alpha = 1, B = 0 result, and alpha = 4
+    gives exactly four times it (powers of two scale exactly)."""
+    M, N = 513, 1300
+    A, _, x = inputs.generate_gesummv(_w("gesummv", dtype, M, N, N, 3), DEV)
+    Z = torch.zeros_like(A)
+    y_one = dm.gesummv(A, Z, x, alpha=1.0, beta=0.0)
+    y_two = dm.gesummv(A, A, x, alpha=1.0, beta=1.0)
+    y_four = dm.gesummv(A, Z, x, alpha=4.0, beta=3.0)
+    assert torch.equal(y_two, 2 * y_one) and torch.equal(y_four, 4 * y_one)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_atax_permutation_is_exact(dtype):
+    n = 900
+    g = torch.Generator(device="cpu").manual_seed(9)
+    perm = torch.randperm(n, generator=g)
+    P = torch.zeros(n, n, dtype=TAGS[dtype])
+    P[torch.arange(n), perm] = 1.0
+    x = torch.empty(n, dtype=TAGS[dtype]).uniform_(-1, 1, generator=g)
+    y = dm.atax(P.to(DEV), x.to(DEV))
+    if dtype == "f64":
+        assert float(((y.cpu() - x).abs() / x.abs()).max()) <= 2.0 ** -43
+    else:
+        assert torch.equal(y.cpu(), x)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_empty_shapes(dtype):
+    t = TAGS[dtype]
+    A = torch.empty(4, 0, dtype=t, device=DEV)
+    y = dm.gesummv(A, A, torch.empty(0, dtype=t, device=DEV))
+    assert (y.cpu() == 0).all() and y.shape == (4,)
+    A = torch.empty(0, 6, dtype=t, device=DEV)
+    y = dm.atax(A, torch.ones(6, dtype=t, device=DEV))
+    assert (y.cpu() == 0).all() and y.shape == (6,)
+
+
+def test_no_device_fault_recorded():
+    assert dm.device_fault() == dm.DUALMV_SUCCESS

@@ -36,6 +36,17 @@ MUTANTS = [
     ("trim_off_by_one", "for (int64_t i = k; i < R - k; ++i)",
      "for (int64_t i = k; i <= R - k; ++i)", 0),
     ("trim_wrong_count", "*out = sum / (double)(R - 2 * k);", "*out = sum / (double)(R - k);", 0),
+    ("gesummv_swapped_scalars", "y[i] = alpha * ta + beta * tb;",
+     "y[i] = beta * ta + alpha * tb;", 0),
+    ("gesummv_lda_for_ldb", "tb += (double)B[i * ldb + j] * (double)x[j];",
+     "tb += (double)B[i * lda + j] * (double)x[j];", 0),
+    ("gesummv_f64_lost_compensation", "y[i] = alpha * (a_hi + a_lo) + beta * (b_hi + b_lo);",
+     "y[i] = alpha * a_hi + beta * (b_hi + b_lo);", 0),
+    ("atax_second_pass_uses_x", "for (int64_t j = 0; j < N; ++j) y[j] += (double)A[i * lda + j] * tmp;",
+     "for (int64_t j = 0; j < N; ++j) y[j] += (double)A[i * lda + j] * (double)x[j];", 0),
+    ("atax_dropped_x", "for (int64_t j = 0; j < N; ++j) tmp += (double)A[i * lda + j] * (double)x[j];",
+     "for (int64_t j = 0; j < N; ++j) tmp += (double)A[i * lda + j];", 0),
+    ("atax_f64_tmp_uncompensated", "const double tmp = t_hi + t_lo;", "const double tmp = t_hi;", 0),
 ]
 
 

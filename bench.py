@@ -218,12 +218,17 @@ def run_native(args):
 
         def call():
             dm.gesummv(A[:, : w.N], Bm[:, : w.N], x, alpha=1.5, beta=1.2, y=y)
-    else:
+    elif w.op == "atax":
         A, x = inputs.generate_atax(w, dev)
         y = torch.empty(w.N, dtype=A.dtype, device=dev)
 
         def call():
             dm.atax(A[:, : w.N], x, y=y)
+    else:  # gemver: x and w accumulate in place from call to call
+        A, u1, v1, u2, v2, wv, x, y, z = inputs.generate_gemver(w, dev)
+
+        def call():
+            dm.gemver(A[:, : w.N], u1, v1, u2, v2, wv, x, y, z, alpha=1.5, beta=1.2)
 
     for _ in range(args.warmup):
         call()
@@ -294,6 +299,8 @@ def run_native(args):
         launches_per_call = 2 * launches_per_call + 1
     elif w.op == "atax":    # a row pass and a column pass
         launches_per_call = 2 * launches_per_call
+    elif w.op == "gemver":  # column pass, x update, row pass, w update
+        launches_per_call = 2 * launches_per_call + 2
     peak, peak_src = measured_peak()
     kern_avg_ms = sum(kern_ms) / len(kern_ms)
     achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9

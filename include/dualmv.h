@@ -133,6 +133,24 @@ dualmv_status dualmv_atax_f32(int64_t M, int64_t N, const float *A, int64_t lda,
 dualmv_status dualmv_atax_f64(int64_t M, int64_t N, const double *A, int64_t lda,
                               const double *x, double *y, dualmv_stream_t stream);
 
+/* GEMVER (Table 1 / Table 2, row "GEMVER"): with A M x N (lda >= max(1, N)),
+ * u1, u2, w, y of length M and v1, v2, x, z of length N:
+ *     A_hat = A + u1 v1^T + u2 v2^T
+ *     x     = x + beta * A_hat^T y + z        (x is read and written)
+ *     w     = w + alpha * A_hat x             (w is read and written)
+ * The rank-2 update is applied on the fly by each of the two passes over A
+ * (columns, then rows), so A_hat is never stored unless update_A is
+ * nonzero, in which case the second pass writes A_hat over A (as the
+ * PolyBench kernel does).  fp64 takes native fp64 arithmetic here. */
+dualmv_status dualmv_gemver_f32(int64_t M, int64_t N, float alpha, float beta, float *A,
+                                int64_t lda, int update_A, const float *u1, const float *v1,
+                                const float *u2, const float *v2, float *w, float *x,
+                                const float *y, const float *z, dualmv_stream_t stream);
+dualmv_status dualmv_gemver_f64(int64_t M, int64_t N, double alpha, double beta, double *A,
+                                int64_t lda, int update_A, const double *u1, const double *v1,
+                                const double *u2, const double *v2, double *w, double *x,
+                                const double *y, const double *z, dualmv_stream_t stream);
+
 /* ---- single problem without allocation --------------------------------
  * The paper has no counterpart to this entry point; it exists for callers
  * that cannot allocate device memory during the call: code inside a

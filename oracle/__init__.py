@@ -94,6 +94,10 @@ def _declare(lib):
         fn = getattr(lib, name)
         fn.argtypes = [i64, i64, vp, i64, vp, vp]
         fn.restype = ctypes.c_int
+    for name in ("oracle_gemver_f32", "oracle_gemver_f64"):
+        fn = getattr(lib, name)
+        fn.argtypes = [i64, i64, dbl, dbl, vp, i64] + [vp] * 11
+        fn.restype = ctypes.c_int
     return lib
 
 
@@ -246,3 +250,29 @@ def atax(A: np.ndarray, x: np.ndarray, N: int | None = None, lib=None) -> np.nda
     if rc != 0:
         raise RuntimeError(f"oracle_atax_{tag} returned {rc}")
     return y
+
+
+def gemver(A: np.ndarray, u1, v1, u2, v2, w, x, y, z, alpha: float, beta: float,
+           N: int | None = None, lib=None):
+    """GEMVER (Table 1 / Table 2): returns ``(A_hat, w_new, x_new)`` in
+    float64 for A_hat = A + u1 v1^T + u2 v2^T, x_new = x + beta A_hat^T y
+    + z, w_new = w + alpha A_hat x_new (A is M x lda storage)."""
+    lib = lib or load()
+    tag = _float_tag(A)
+    if A.ndim != 2 or not A.flags.c_contiguous:
+        raise ValueError("A must be a C-contiguous 2-D buffer")
+    M = A.shape[0]
+    N = A.shape[1] if N is None else int(N)
+    vecs = [np.ascontiguousarray(v, dtype=A.dtype) for v in (u1, v1, u2, v2, w, x, y, z)]
+    want = [M, N, M, N, M, N, M, N]
+    if any(v.shape != (n,) for v, n in zip(vecs, want)):
+        raise ValueError("vector lengths do not match A")
+    ahat = np.zeros((M, N), dtype=np.float64)
+    wo = np.zeros(M, dtype=np.float64)
+    xo = np.zeros(N, dtype=np.float64)
+    rc = getattr(lib, f"oracle_gemver_{tag}")(M, N, float(alpha), float(beta), _ptr(A),
+                                              max(A.shape[1], 1), *[_ptr(v) for v in vecs],
+                                              _ptr(ahat), _ptr(wo), _ptr(xo))
+    if rc != 0:
+        raise RuntimeError(f"oracle_gemver_{tag} returned {rc}")
+    return ahat, wo, xo

@@ -40,6 +40,8 @@
  * tables built from the same products, with the same precision rules:
  *     GESUMMV  y = alpha (A x) + beta (B x)       (Table 1, Table 2)
  *     ATAX     y = A^T (A x)                      (Table 1)
+ *     GEMVER   A_hat = A + u1 v1^T + u2 v2^T, x = x + beta A_hat^T y + z,
+ *              w = w + alpha A_hat x              (Table 1, Table 2)
  *
  * Build: plain C99, -O2 -fno-fast-math -ffp-contract=off, so the compiler
  * neither reassociates the sums nor fuses a multiply into an add.
@@ -338,5 +340,78 @@ int oracle_atax_f64(int64_t M, int64_t N, const double *A, int64_t lda, const do
     }
     for (int64_t j = 0; j < N; ++j) y[j] = y[j] + y_lo[j];
     free(y_lo);
+    return ORACLE_OK;
+}
+
+/* -------------------------------------------------------------- GEMVER --- */
+
+/* GEMVER (Table 1 / Table 2):  A_hat = A + u1 v1^T + u2 v2^T;
+ * x = x + beta A_hat^T y + z;  w = w + alpha A_hat x.
+ * Float inputs: everything in double (A_hat_ij = a + u1 v1 + u2 v2 summed
+ * left to right from exact products), A_hat returned in ahat (M x N, row
+ * stride N), x and w returned in xo and wo (double). */
+int oracle_gemver_f32(int64_t M, int64_t N, double alpha, double beta, const float *A,
+                      int64_t lda, const float *u1, const float *v1, const float *u2,
+                      const float *v2, const float *w, const float *x, const float *y,
+                      const float *z, double *ahat, double *wo, double *xo)
+{
+    if (M < 0 || N < 0 || lda < N || lda < 1) return ORACLE_EINVAL;
+    for (int64_t i = 0; i < M; ++i)
+        for (int64_t j = 0; j < N; ++j)
+            ahat[i * N + j] = (double)A[i * lda + j] + (double)u1[i] * (double)v1[j]
+                              + (double)u2[i] * (double)v2[j];
+    for (int64_t j = 0; j < N; ++j) {
+        double acc = 0.0;
+        for (int64_t i = 0; i < M; ++i) acc += ahat[i * N + j] * (double)y[i];
+        xo[j] = (double)x[j] + beta * acc + (double)z[j];
+    }
+    for (int64_t i = 0; i < M; ++i) {
+        double acc = 0.0;
+        for (int64_t j = 0; j < N; ++j) acc += ahat[i * N + j] * xo[j];
+        wo[i] = (double)w[i] + alpha * acc;
+    }
+    return ORACLE_OK;
+}
+
+/* Double inputs: each A_hat entry as a compensated sum of a, TwoProduct(u1,
+ * v1) and TwoProduct(u2, v2), rounded once; both products with Dot2 on the
+ * rounded A_hat (and on the rounded new x). */
+int oracle_gemver_f64(int64_t M, int64_t N, double alpha, double beta, const double *A,
+                      int64_t lda, const double *u1, const double *v1, const double *u2,
+                      const double *v2, const double *w, const double *x, const double *y,
+                      const double *z, double *ahat, double *wo, double *xo)
+{
+    if (M < 0 || N < 0 || lda < N || lda < 1) return ORACLE_EINVAL;
+    for (int64_t i = 0; i < M; ++i)
+        for (int64_t j = 0; j < N; ++j) {
+            double p1, e1, p2, e2, s1, t1, s2, t2;
+            two_prod(u1[i], v1[j], &p1, &e1);
+            two_prod(u2[i], v2[j], &p2, &e2);
+            two_sum(A[i * lda + j], p1, &s1, &t1);
+            two_sum(s1, p2, &s2, &t2);
+            ahat[i * N + j] = s2 + ((t1 + t2) + (e1 + e2));
+        }
+    for (int64_t j = 0; j < N; ++j) {
+        double hi = 0.0, lo = 0.0;
+        for (int64_t i = 0; i < M; ++i) {
+            double prod, perr, sum, serr;
+            two_prod(ahat[i * N + j], y[i], &prod, &perr);
+            two_sum(hi, prod, &sum, &serr);
+            hi = sum;
+            lo = lo + (perr + serr);
+        }
+        xo[j] = x[j] + beta * (hi + lo) + z[j];
+    }
+    for (int64_t i = 0; i < M; ++i) {
+        double hi = 0.0, lo = 0.0;
+        for (int64_t j = 0; j < N; ++j) {
+            double prod, perr, sum, serr;
+            two_prod(ahat[i * N + j], xo[j], &prod, &perr);
+            two_sum(hi, prod, &sum, &serr);
+            hi = sum;
+            lo = lo + (perr + serr);
+        }
+        wo[i] = w[i] + alpha * (hi + lo);
+    }
     return ORACLE_OK;
 }

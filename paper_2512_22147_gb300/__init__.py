@@ -22,9 +22,9 @@ _BINDING_NAMES = {
     "dualmv_plan", "dualmv_record_kernel_events", "dualmv_set_path",
     "dualmv_status_string", "library", "dualmv_f32_noalloc",
     "dualmv_f32_noalloc_scratch_bytes", "dualmv_gesummv_f32", "dualmv_gesummv_f64",
-    "dualmv_atax_f32", "dualmv_atax_f64",
+    "dualmv_atax_f32", "dualmv_atax_f64", "dualmv_gemver_f32", "dualmv_gemver_f64",
 }
-_API_NAMES = {"dualmv", "device_fault", "gesummv", "atax"}
+_API_NAMES = {"dualmv", "device_fault", "gesummv", "atax", "gemver"}
 
 
 def __getattr__(name):

@@ -40,6 +40,7 @@ EXPORTED = (
     "dualmv_set_path", "dualmv_plan", "dualmv_record_kernel_events",
     "dualmv_f32_noalloc", "dualmv_f32_noalloc_scratch_bytes",
     "dualmv_gesummv_f32", "dualmv_gesummv_f64", "dualmv_atax_f32", "dualmv_atax_f64",
+    "dualmv_gemver_f32", "dualmv_gemver_f64",
 )
 
 
@@ -83,6 +84,9 @@ def _load() -> ctypes.CDLL:
         f.restype = st
         f = getattr(lib, f"dualmv_atax_{tag}")
         f.argtypes = [i64, i64, vp, i64, vp, vp, vp]
+        f.restype = st
+        f = getattr(lib, f"dualmv_gemver_{tag}")
+        f.argtypes = [i64, i64, real, real, vp, i64, st, vp, vp, vp, vp, vp, vp, vp, vp, vp]
         f.restype = st
     lib.dualmv_status_string.argtypes = [st]
     lib.dualmv_status_string.restype = ctypes.c_char_p
@@ -160,6 +164,16 @@ def dualmv_atax_f32(M, N, A, lda, x, y, stream):
 
 def dualmv_atax_f64(M, N, A, lda, x, y, stream):
     return _lib.dualmv_atax_f64(M, N, A, lda, x, y, stream)
+
+
+def dualmv_gemver_f32(M, N, alpha, beta, A, lda, update_A, u1, v1, u2, v2, w, x, y, z, stream):
+    return _lib.dualmv_gemver_f32(M, N, alpha, beta, A, lda, update_A, u1, v1, u2, v2, w, x, y,
+                                  z, stream)
+
+
+def dualmv_gemver_f64(M, N, alpha, beta, A, lda, update_A, u1, v1, u2, v2, w, x, y, z, stream):
+    return _lib.dualmv_gemver_f64(M, N, alpha, beta, A, lda, update_A, u1, v1, u2, v2, w, x, y,
+                                  z, stream)
 
 
 def dualmv_status_string(status: int) -> str:

@@ -170,3 +170,30 @@ def atax(A: torch.Tensor, x: torch.Tensor, y: torch.Tensor | None = None,
     if rc != B_.DUALMV_SUCCESS:
         raise B_.DualmvError(rc, f"dualmv_atax_{tag}")
     return y
+
+
+def gemver(A: torch.Tensor, u1: torch.Tensor, v1: torch.Tensor, u2: torch.Tensor,
+           v2: torch.Tensor, w: torch.Tensor, x: torch.Tensor, y: torch.Tensor,
+           z: torch.Tensor, alpha: float = 1.0, beta: float = 1.0, update_A: bool = False,
+           stream: torch.cuda.Stream | None = None):
+    """GEMVER (Table 1 / Table 2): A_hat = A + u1 v1^T + u2 v2^T;
+    x = x + beta A_hat^T y + z;  w = w + alpha A_hat x.
+
+    x and w are updated in place (and A too when ``update_A``); returns
+    ``(w, x)``.  A is M x N; u1, u2, w, y have M elements; v1, v2, x, z N."""
+    tag = {torch.float32: "f32", torch.float64: "f64"}.get(A.dtype)
+    if tag is None or not A.is_cuda:
+        raise TypeError("A must be a float32 or float64 CUDA tensor")
+    M, N, lda = _matrix(A, "A")
+    for v, n, name in ((u1, M, "u1"), (u2, M, "u2"), (w, M, "w"), (y, M, "y"),
+                       (v1, N, "v1"), (v2, N, "v2"), (x, N, "x"), (z, N, "z")):
+        _vector(v, n, A, name)
+    strm = stream if stream is not None else torch.cuda.current_stream(A.device)
+    with torch.cuda.device(A.device):
+        rc = getattr(B_, f"dualmv_gemver_{tag}")(
+            M, N, alpha, beta, A.data_ptr(), lda, int(bool(update_A)), u1.data_ptr(),
+            v1.data_ptr(), u2.data_ptr(), v2.data_ptr(), w.data_ptr(), x.data_ptr(),
+            y.data_ptr(), z.data_ptr(), strm.cuda_stream)
+    if rc != B_.DUALMV_SUCCESS:
+        raise B_.DualmvError(rc, f"dualmv_gemver_{tag}")
+    return w, x

@@ -278,11 +278,11 @@ bool fault_injected_alloc() {
 
 // ------------------------------------------------------------- launching --
 
-template <typename T, bool kTma, bool k3d, int kOut = dmv::kOutBoth>
+template <typename T, bool kTma, bool k3d, int kOut = dmv::kOutBoth, bool kRank2 = false>
 cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                           int dev, cudaStream_t stream) {
     constexpr int rpw = sizeof(T) == 4 ? kRpw4 : kRpw8;
-    auto kern = dmv::dualmv_stream_kernel<T, kWarps, rpw, kStages, kTma, k3d, kOut>;
+    auto kern = dmv::dualmv_stream_kernel<T, kWarps, rpw, kStages, kTma, k3d, kOut, kRank2>;
     // The shared-memory opt-in is per device and per kernel; set it once.
     static std::atomic<uint64_t> opted_in{0};
     const uint64_t bit = 1ull << (dev & 63);
@@ -376,18 +376,28 @@ cudaError_t zero_fill(Acc *out, int64_t len, int64_t stride, int64_t batch,
     return cudaGetLastError();
 }
 
+// GEMVER's rank-2 update, applied on the fly by a single-sided pass.
+struct Rank2 {
+    const void *u1, *v1, *u2, *v2;
+    void *a_out;  // write A_hat here (may be A itself), or nullptr
+    int64_t lda_out;
+};
+
 // One dual (or single-sided) matrix-vector product.  `outputs` selects q,
-// s or both; single-sided calls (the building blocks of ATAX and GESUMMV)
-// are single problems of float or double.
+// s or both; single-sided calls (the building blocks of ATAX, GESUMMV and
+// GEMVER) are single problems of float or double; `rank2` adds GEMVER's
+// on-the-fly update to a single-sided call (native arithmetic for double).
 template <typename T, typename Out>
 dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA,
                   const T *p, int64_t strideP, const T *r, int64_t strideR, Out *q,
                   int64_t strideQ, Out *s, int64_t strideS, int64_t batch,
-                  cudaStream_t stream, uint32_t outputs = dmv::kOutBoth) {
+                  cudaStream_t stream, uint32_t outputs = dmv::kOutBoth,
+                  const Rank2 *rank2 = nullptr) {
     using Acc = typename dmv::Traits<T>::Acc;
     static_assert(sizeof(Acc) == sizeof(Out), "accumulator and output widths differ");
     constexpr bool kIntPath = std::is_same<T, int32_t>::value;
     if (outputs != dmv::kOutBoth && (kIntPath || batch > 1)) return DUALMV_ERR_UNSUPPORTED;
+    if (rank2 != nullptr && outputs == dmv::kOutBoth) return DUALMV_ERR_UNSUPPORTED;
     const bool want_q = (outputs & dmv::kOutQ) != 0, want_s = (outputs & dmv::kOutS) != 0;
     dualmv_status st = validate(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ,
                                 s, strideS, batch, outputs);
@@ -422,7 +432,10 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                (!three_d || (strideA > 0 && (strideA * es) % 16 == 0));
     // fp64 runs on the FP32 pipes unless native fp64 FMA is requested.
     Kind kind = Kind::kDirect;
-    if (tma) kind = (es == 8 && g_path != DUALMV_PATH_TMA_NATIVE_F64) ? Kind::kF64e : Kind::kTma;
+    if (tma)
+        kind = (es == 8 && g_path != DUALMV_PATH_TMA_NATIVE_F64 && rank2 == nullptr)
+                   ? Kind::kF64e
+                   : Kind::kTma;
     CUtensorMap map;
     std::memset(&map, 0, sizeof map);
     if (tma) {
@@ -456,6 +469,12 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     prm.s = s; prm.strideS = strideS;
     prm.M = M; prm.N = N; prm.batch = batch;
     prm.outputs = outputs;
+    prm.u1 = rank2 ? rank2->u1 : nullptr;
+    prm.v1 = rank2 ? rank2->v1 : nullptr;
+    prm.u2 = rank2 ? rank2->u2 : nullptr;
+    prm.v2 = rank2 ? rank2->v2 : nullptr;
+    prm.a_out = rank2 ? rank2->a_out : nullptr;
+    prm.lda_out = rank2 ? rank2->lda_out : 0;
     prm.band_cols = pl.band_cols;
     prm.bands = pl.bands; prm.stripes = pl.stripes; prm.tiles = pl.tiles;
     prm.grid = pl.grid; prm.max_seg = pl.max_segments;
@@ -478,7 +497,17 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     g_kernel_ev_start = g_kernel_ev_stop = nullptr;
     e = ev_start ? cudaEventRecord(ev_start, stream) : cudaSuccess;
     if (e == cudaSuccess) {
-        if (outputs != dmv::kOutBoth) {
+        if (rank2 != nullptr) {
+            if constexpr (!kIntPath) {
+                const bool only_q = outputs == dmv::kOutQ;
+                if (kind == Kind::kTma)
+                    e = only_q ? launch_stream<T, true, false, dmv::kOutQ, true>(map, prm, pl, dev, stream)
+                               : launch_stream<T, true, false, dmv::kOutS, true>(map, prm, pl, dev, stream);
+                else
+                    e = only_q ? launch_stream<T, false, false, dmv::kOutQ, true>(map, prm, pl, dev, stream)
+                               : launch_stream<T, false, false, dmv::kOutS, true>(map, prm, pl, dev, stream);
+            }
+        } else if (outputs != dmv::kOutBoth) {
             if constexpr (!kIntPath) {
                 // Single-sided products (one problem, float or double).
                 const bool only_q = outputs == dmv::kOutQ;
@@ -595,6 +624,59 @@ dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x
     return st;
 }
 
+// GEMVER (Table 1 / Table 2): A_hat = A + u1 v1^T + u2 v2^T;
+// x = x + beta A_hat^T y + z;  w = w + alpha A_hat x.  Two passes apply the
+// rank-2 update as they stream A: a columns-only pass (A_hat^T y) and, after
+// the x update, a rows-only pass (A_hat x) that also writes A_hat over A
+// when update_A is set.  A is read twice and written at most once.
+template <typename T>
+dualmv_status gemver_run(int64_t M, int64_t N, T alpha, T beta, T *A, int64_t lda,
+                         int update_A, const T *u1, const T *v1, const T *u2, const T *v2,
+                         T *w, T *x, const T *y, const T *z, cudaStream_t stream) {
+    if (M < 0 || N < 0 || lda < (N > 1 ? N : 1)) return DUALMV_ERR_INVALID_VALUE;
+    if (N > 0 && (x == nullptr || z == nullptr || v1 == nullptr || v2 == nullptr))
+        return DUALMV_ERR_INVALID_VALUE;
+    if (M > 0 && (w == nullptr || y == nullptr || u1 == nullptr || u2 == nullptr))
+        return DUALMV_ERR_INVALID_VALUE;
+    if (M > 0 && N > 0 && A == nullptr) return DUALMV_ERR_INVALID_VALUE;
+    if (M == 0 && N == 0) return DUALMV_SUCCESS;
+    if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
+    T *s = nullptr, *t = nullptr;
+    dualmv_status st = pool_alloc(&s, N, stream);
+    if (st != DUALMV_SUCCESS) return st;
+    st = pool_alloc(&t, M, stream);
+    if (st != DUALMV_SUCCESS) {
+        cudaFreeAsync(s, stream);
+        return st;
+    }
+    Rank2 upd{u1, v1, u2, v2, nullptr, lda};
+    if (N > 0)  // s = A_hat^T y (zero when M == 0)
+        st = run<T, T>(M, N, A, lda, 0, nullptr, 0, y, 0, nullptr, 0, s, 0, 1, stream,
+                       dmv::kOutS, &upd);
+    const int64_t bx = N > 0 ? (N + 255) / 256 : 0, bw = M > 0 ? (M + 255) / 256 : 0;
+    if (st == DUALMV_SUCCESS && N > 0) {
+        dmv::gemver_x_kernel<T><<<(unsigned)(bx > 4096 ? 4096 : bx), 256, 0, stream>>>(
+            x, s, z, N, beta);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) st = cuda_fail(e);
+    }
+    if (st == DUALMV_SUCCESS && M > 0) {  // t = A_hat x (zero when N == 0)
+        upd.a_out = update_A ? A : nullptr;
+        st = run<T, T>(M, N, A, lda, 0, x, 0, nullptr, 0, t, 0, nullptr, 0, 1, stream,
+                       dmv::kOutQ, &upd);
+    }
+    if (st == DUALMV_SUCCESS && M > 0) {
+        dmv::gemver_w_kernel<T><<<(unsigned)(bw > 4096 ? 4096 : bw), 256, 0, stream>>>(
+            w, t, M, alpha);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) st = cuda_fail(e);
+    }
+    cudaError_t e1 = cudaFreeAsync(s, stream), e2 = cudaFreeAsync(t, stream);
+    if (st == DUALMV_SUCCESS && (e1 != cudaSuccess || e2 != cudaSuccess))
+        st = cuda_fail(e1 != cudaSuccess ? e1 : e2);
+    return st;
+}
+
 // ------------------------------------------------- no-allocation variant --
 //
 // Some callers cannot allocate device memory while they run dualmv: code
@@ -677,6 +759,9 @@ dualmv_status run_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,
     prm.s = s; prm.strideS = N;
     prm.M = M; prm.N = N; prm.batch = 1;
     prm.outputs = dmv::kOutBoth;
+    prm.u1 = prm.v1 = prm.u2 = prm.v2 = nullptr;
+    prm.a_out = nullptr;
+    prm.lda_out = 0;
     prm.band_cols = pl.band_cols;
     prm.bands = pl.bands; prm.stripes = pl.stripes; prm.tiles = pl.tiles;
     prm.grid = pl.grid; prm.max_seg = pl.max_segments;
@@ -766,6 +851,22 @@ dualmv_status dualmv_atax_f32(int64_t M, int64_t N, const float *A, int64_t lda,
 dualmv_status dualmv_atax_f64(int64_t M, int64_t N, const double *A, int64_t lda,
                               const double *x, double *y, dualmv_stream_t stream) {
     return atax_run<double>(M, N, A, lda, x, y, reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_gemver_f32(int64_t M, int64_t N, float alpha, float beta, float *A,
+                                int64_t lda, int update_A, const float *u1, const float *v1,
+                                const float *u2, const float *v2, float *w, float *x,
+                                const float *y, const float *z, dualmv_stream_t stream) {
+    return gemver_run<float>(M, N, alpha, beta, A, lda, update_A, u1, v1, u2, v2, w, x, y, z,
+                             reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_gemver_f64(int64_t M, int64_t N, double alpha, double beta, double *A,
+                                int64_t lda, int update_A, const double *u1, const double *v1,
+                                const double *u2, const double *v2, double *w, double *x,
+                                const double *y, const double *z, dualmv_stream_t stream) {
+    return gemver_run<double>(M, N, alpha, beta, A, lda, update_A, u1, v1, u2, v2, w, x, y, z,
+                              reinterpret_cast<cudaStream_t>(stream));
 }
 
 dualmv_status dualmv_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,

@@ -275,6 +275,12 @@ struct Params {
     void *s;
     int64_t strideS;
     int64_t M, N, batch;
+    // GEMVER's rank-2 update, applied to every element as it is streamed:
+    // A_hat = A + u1 v1^T + u2 v2^T (u1, u2 of length M, v1, v2 of length
+    // N); with a_out set, A_hat is also written there (row stride lda_out).
+    const void *u1, *v1, *u2, *v2;
+    void *a_out;
+    int64_t lda_out;
     uint32_t outputs;   // kOutQ | kOutS: which of q and s this call computes
     int64_t band_cols;  // columns per band (the stream kernel's tile width)
     int64_t bands, stripes, tiles, grid, max_seg;
@@ -339,10 +345,11 @@ struct SmemLayout {
 // STAGES ring depth, kTma = TMA producer (else plain loads), kBatched3d =
 // 3-D tensor map (batch as the outer coordinate).
 template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d,
-          int kOut = kOutBoth>
+          int kOut = kOutBoth, bool kRank2 = false>
 __global__ void __launch_bounds__((W + (kTma ? 1 : 0)) * 32, 1)
 dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
     using Acc = typename Traits<T>::Acc;
+    static_assert(!kRank2 || !std::is_same<T, int32_t>::value, "rank-2 update: floats only");
     constexpr bool kQ = (kOut & kOutQ) != 0;  // row sums q = A p
     constexpr bool kS = (kOut & kOutS) != 0;  // column sums s = A^T r
     // Integer sums are exact modulo 2^64 in any order, so the int32 path adds
@@ -442,6 +449,7 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
     const int nthreads_c = W * 32;
 
     T pv[kLaneCols];
+    T v1v[kRank2 ? kLaneCols : 1], v2v[kRank2 ? kLaneCols : 1];  // GEMVER columns
     Acc grp[kLaneCols], seg[kLaneCols];
 #pragma unroll
     for (int e = 0; e < kLaneCols; ++e) {
@@ -457,10 +465,17 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
     cur.init(t0, S, prm.bands);
     // r for this warp's RPW rows of the next tile (lane i < RPW holds row
     // row0 + i), loaded one tile ahead so its latency hides behind a tile.
-    T r_next = T(0);
+    T r_next = T(0), u1_next = T(0), u2_next = T(0);
     if constexpr (kS) {
         const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
         if (lane < RPW && row < prm.M) r_next = rg[cur.b * prm.strideR + row];
+    }
+    if constexpr (kRank2) {
+        const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
+        if (lane < RPW && row < prm.M) {
+            u1_next = static_cast<const T *>(prm.u1)[row];
+            u2_next = static_cast<const T *>(prm.u2)[row];
+        }
     }
     int stage = 0;
     uint32_t phase = 0;
@@ -473,11 +488,27 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
         const int64_t b = cur.b;
         const int64_t col0 = band * kBandCols;
         const int64_t row0 = stripe * BM + (int64_t)warp * RPW;
-        const T rmine = r_next;
+        const T rmine = r_next, u1mine = u1_next, u2mine = u2_next;
         cur.advance(S, prm.bands);
         if (kS && k + 1 < ntiles) {
             const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
             r_next = (lane < RPW && row < prm.M) ? rg[cur.b * prm.strideR + row] : T(0);
+        }
+        if (kRank2 && k + 1 < ntiles) {
+            const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
+            const bool in = lane < RPW && row < prm.M;
+            u1_next = in ? static_cast<const T *>(prm.u1)[row] : T(0);
+            u2_next = in ? static_cast<const T *>(prm.u2)[row] : T(0);
+        }
+        if (kRank2 && (k == 0 || stripe == 0)) {  // a new segment: v1, v2 of this band
+#pragma unroll
+            for (int v = 0; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) {
+                    const int64_t col = col0 + lane_col<T>(v, lane, e);
+                    v1v[v * VE + e] = col < prm.N ? static_cast<const T *>(prm.v1)[col] : T(0);
+                    v2v[v * VE + e] = col < prm.N ? static_cast<const T *>(prm.v2)[col] : T(0);
+                }
         }
 
         if (k == 0 || stripe == 0) seg_start_stripe = stripe;
@@ -525,6 +556,32 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
                 }
             }
             const T ri = kS ? __shfl_sync(0xffffffffu, rmine, i) : T(0);
+            if constexpr (kRank2) {
+                // A_hat = A + u1 v1^T + u2 v2^T, element by element; written
+                // back when asked (in place is fine: each element is read
+                // before it is written, by the same thread).
+                const T u1i = __shfl_sync(0xffffffffu, u1mine, i);
+                const T u2i = __shfl_sync(0xffffffffu, u2mine, i);
+                const int64_t row = row0 + i;
+#pragma unroll
+                for (int v = 0; v < VPL; ++v) {
+                    T tmp[VE];
+#pragma unroll
+                    for (int e = 0; e < VE; ++e)
+                        tmp[e] = mul_acc(u2i, v2v[v * VE + e],
+                                         mul_acc(u1i, v1v[v * VE + e], vget(a[v], e)));
+                    if constexpr (VE == 4) a[v] = Vec{tmp[0], tmp[1], tmp[2], tmp[3]};
+                    else a[v] = Vec{tmp[0], tmp[1]};
+                    if (prm.a_out != nullptr && row < prm.M) {
+                        T *orow = static_cast<T *>(prm.a_out) + row * prm.lda_out;
+#pragma unroll
+                        for (int e = 0; e < VE; ++e) {
+                            const int64_t col = col0 + lane_col<T>(v, lane, e);
+                            if (col < prm.N) orow[col] = tmp[e];
+                        }
+                    }
+                }
+            }
             Acc dot = Acc(0);
 #pragma unroll
             for (int v = 0; v < VPL; ++v)
@@ -709,6 +766,20 @@ __global__ void axpby_kernel(const T *t, T *y, int64_t n, T alpha, T beta) {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x)
         y[i] = alpha * t[i] + beta * y[i];
+}
+
+// GEMVER vector steps: x = (x + beta * s) + z, then w = w + alpha * t.
+template <typename T>
+__global__ void gemver_x_kernel(T *x, const T *s, const T *z, int64_t n, T beta) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        x[i] = (x[i] + beta * s[i]) + z[i];
+}
+template <typename T>
+__global__ void gemver_w_kernel(T *w, const T *t, int64_t n, T alpha) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        w[i] = w[i] + alpha * t[i];
 }
 
 // Zero-fill of strided outputs (empty problems).

@@ -36,7 +36,7 @@ class Workload:
     dist: str           # "uniform" | "normal" | "int8"
     seed: int
     batch: int = 0      # 0 = single problem; >= 1 = strided batch
-    op: str = "bicg"    # "bicg" (dual product) | "gesummv" | "atax"
+    op: str = "bicg"    # "bicg" (dual product) | "gesummv" | "atax" | "gemver"
 
     @property
     def batched(self) -> bool:
@@ -56,6 +56,8 @@ class Workload:
             return 2 * self.M * self.N * e + self.N * e + self.M * o
         if self.op == "atax":
             return self.M * self.N * e + self.N * e + self.N * o
+        if self.op == "gemver":   # A once; u1 v1 u2 v2 y z read; x w read and written
+            return self.M * self.N * e + 3 * (self.M + self.N) * e + (self.M + self.N) * o
         per = (self.M * self.N * e + (self.M + self.N) * e
                + (self.M + self.N) * o)
         return per * self.nbatch
@@ -80,9 +82,9 @@ WORKLOADS = {
 }
 
 
-# Workloads of the two further PolyBench kernels built on the same products
-# (GESUMMV and ATAX, Table 1), sized like the dual product's square fp32
-# workload so that every matrix is far larger than L2.
+# Workloads of the further PolyBench kernels built on the same products
+# (GESUMMV, ATAX and GEMVER, Table 1), sized like the dual product's square
+# fp32 workload so that every matrix is far larger than L2.
 OP_WORKLOADS = {
     w.name: w for w in (
         Workload("gesummv_f32_16384x16384", "f32", 16384, 16384, 16384, "uniform", 5,
@@ -90,6 +92,9 @@ OP_WORKLOADS = {
         Workload("gesummv_f64_8192x8192", "f64", 8192, 8192, 8192, "normal", 6, op="gesummv"),
         Workload("atax_f32_16384x16384", "f32", 16384, 16384, 16384, "uniform", 7, op="atax"),
         Workload("atax_f64_16384x8192", "f64", 16384, 8192, 8192, "normal", 8, op="atax"),
+        Workload("gemver_f32_16384x16384", "f32", 16384, 16384, 16384, "uniform", 9,
+                 op="gemver"),
+        Workload("gemver_f64_8192x8192", "f64", 8192, 8192, 8192, "normal", 10, op="gemver"),
     )
 }
 
@@ -192,3 +197,22 @@ def generate_atax(w: Workload, device: str | torch.device = "cpu"):
     g.manual_seed(w.seed)
     A = _matrix(w, g, dev)
     return A, _vector(w.N, w, g, dev)
+
+
+def generate_gemver(w: Workload, device: str | torch.device = "cpu"):
+    """``(A, u1, v1, u2, v2, w, x, y, z)`` for GEMVER: one generator fills A,
+    then the vectors in that order (u's, w, y of length M; v's, x, z of
+    length N)."""
+    dev = torch.device(device)
+    g = torch.Generator(device=dev)
+    g.manual_seed(w.seed)
+    A = _matrix(w, g, dev)
+    u1 = _vector(w.M, w, g, dev)
+    v1 = _vector(w.N, w, g, dev)
+    u2 = _vector(w.M, w, g, dev)
+    v2 = _vector(w.N, w, g, dev)
+    wv = _vector(w.M, w, g, dev)
+    x = _vector(w.N, w, g, dev)
+    y = _vector(w.M, w, g, dev)
+    z = _vector(w.N, w, g, dev)
+    return A, u1, v1, u2, v2, wv, x, y, z

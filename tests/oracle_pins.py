@@ -8,7 +8,8 @@ real oracle; ``tests/test_oracle_mutants.py`` runs them on copies of the
 oracle with a planted mistake and expects at least one to fail.
 
 The operations are the BICG kernel of the paper (Table 1 and Table 2):
-q = A p and s = A^T r, and the GESUMMV and ATAX kernels of the same tables.
+q = A p and s = A^T r, and the GESUMMV, ATAX and GEMVER kernels of the same
+tables.
 The paper prints no worked example for any of them, so no printed values
 can serve as golden data; everything here is derived from the definitions.
 """
@@ -366,12 +367,83 @@ def pin_atax_closed_forms(lib):
     assert (oracle.atax(A, np.ones(3), lib=lib) == A[0]).all()
 
 
+# -------------------------------------------------------------- GEMVER --
+
+def pin_gemver_bruteforce(lib, seed=18, cases=24):
+    """GEMVER against exact rationals: A_hat, the new x and the new w, each
+    within a small multiple of the unit roundoff times the magnitude of its
+    terms (the new x's error carried into w)."""
+    rng = np.random.default_rng(seed)
+    for case in range(cases):
+        dt = np.float32 if case % 2 == 0 else np.float64
+        M, N, extra = (int(v) for v in rng.integers(1, 6, size=3))
+        A = _padded(rng, M, N, extra, dt, lambda g, sh: _rand_float(g, sh, dt))
+        u1, u2, w, y = (_rand_float(rng, M, dt) for _ in range(4))
+        v1, v2, x, z = (_rand_float(rng, N, dt) for _ in range(4))
+        alpha, beta = 1.5, -0.75
+        ah, wo, xo = oracle.gemver(A, u1, v1, u2, v2, w, x, y, z, alpha, beta, N=N, lib=lib)
+        F = lambda v: Fraction(float(v))  # noqa: E731
+        Ah = [[F(A[i, j]) + F(u1[i]) * F(v1[j]) + F(u2[i]) * F(v2[j]) for j in range(N)]
+              for i in range(M)]
+        Am = [[abs(F(A[i, j])) + abs(F(u1[i]) * F(v1[j])) + abs(F(u2[i]) * F(v2[j]))
+               for j in range(N)] for i in range(M)]
+        Xe = [F(x[j]) + Fraction(beta) * sum((Ah[i][j] * F(y[i]) for i in range(M)), Fraction(0))
+              + F(z[j]) for j in range(N)]
+        Xm = [abs(F(x[j])) + abs(Fraction(beta)) * sum((Am[i][j] * abs(F(y[i])) for i in range(M)),
+                                                       Fraction(0)) + abs(F(z[j])) for j in range(N)]
+        We = [F(w[i]) + Fraction(alpha) * sum((Ah[i][j] * Xe[j] for j in range(N)), Fraction(0))
+              for i in range(M)]
+        Wm = [abs(F(w[i])) + abs(Fraction(alpha)) * sum((Am[i][j] * Xm[j] for j in range(N)),
+                                                        Fraction(0)) for i in range(M)]
+        c = gamma(max(M, N) + 6) if dt == np.float32 else 16 * U53 + gamma(max(M, N)) ** 2
+        # A_hat: three exact products summed in double (f32 inputs), or a
+        # compensated sum rounded once (f64 inputs).
+        for i in range(M):
+            for j in range(N):
+                b = (2 * U53 * Am[i][j] if dt == np.float32
+                     else U53 * abs(Ah[i][j]) + 4 * U53 * U53 * Am[i][j])
+                assert abs(Fraction(float(ah[i, j])) - Ah[i][j]) <= b
+        for j in range(N):
+            assert abs(Fraction(float(xo[j])) - Xe[j]) <= c * Xm[j], (M, N, j)
+        for i in range(M):
+            assert abs(Fraction(float(wo[i])) - We[i]) <= 2 * c * Wm[i], (M, N, i)
+
+
+def pin_gemver_integers_exact(lib):
+    """Small integers keep every GEMVER quantity an exact integer; compare
+    with integer arithmetic, and check that u1 = u2 = 0 leaves A_hat = A."""
+    rng = np.random.default_rng(19)
+    M, N = 9, 13
+    A = rng.integers(-8, 9, (M, N))
+    u1, u2, w, y = (rng.integers(-4, 5, M) for _ in range(4))
+    v1, v2, x, z = (rng.integers(-4, 5, N) for _ in range(4))
+    Ah = A + np.outer(u1, v1) + np.outer(u2, v2)
+    X = x + 2 * (Ah.T @ y) + z
+    W = w + 3 * (Ah @ X)
+    for dt in (np.float32, np.float64):
+        ah, wo, xo = oracle.gemver(A.astype(dt), *(v.astype(dt) for v in (u1, v1, u2, v2, w, x, y, z)),
+                                   3.0, 2.0, lib=lib)
+        assert (ah == Ah).all() and (xo == X).all() and (wo == W).all()
+        zero = np.zeros(M, dt)
+        ah, _, _ = oracle.gemver(A.astype(dt), zero, v1.astype(dt), zero, v2.astype(dt),
+                                 w.astype(dt), x.astype(dt), y.astype(dt), z.astype(dt),
+                                 3.0, 2.0, lib=lib)
+        assert (ah == A).all()
+    # A cancelling update that only the compensated f64 sum gets right:
+    # 2^60 + 1*1 + (-2^60)*1 = 1.
+    one = np.ones(1)
+    ah, _, _ = oracle.gemver(np.array([[2.0 ** 60]]), one, one, -(2.0 ** 60) * one, one,
+                             one, one, one, one, 1.0, 1.0, lib=lib)
+    assert ah[0, 0] == 1.0, ah
+
+
 ALL_PINS = [
     pin_bruteforce_f32, pin_bruteforce_f64, pin_bruteforce_i32,
     pin_wraparound_i32, pin_dot2_cancellation, pin_identity, pin_rank_one,
     pin_adjoint, pin_power_of_two_scaling, pin_shapes_and_empty, pin_absdot,
     pin_trimmed_mean, pin_gesummv_bruteforce, pin_gesummv_closed_forms,
-    pin_atax_bruteforce, pin_atax_closed_forms,
+    pin_atax_bruteforce, pin_atax_closed_forms, pin_gemver_bruteforce,
+    pin_gemver_integers_exact,
 ]
 
 

@@ -1,5 +1,5 @@
-"""GESUMMV and ATAX (Table 1 of the paper; GESUMMV also Table 2) on the GPU
-through the C ABI, against the CPU oracle.
+"""GESUMMV, ATAX and GEMVER (Table 1 of the paper; GESUMMV and GEMVER also
+Table 2) on the GPU through the C ABI, against the CPU oracle.
 
 Tolerance, as for the dual product, relative to the magnitude of each
 output's terms: GESUMMV |y_i - y^_i| <= tol (|alpha| sum_j |A_ij||x_j| +
@@ -73,6 +73,43 @@ def test_atax_matches_oracle(dtype, M, N, pad, path):
     check_atax(A, x, N, dtype)
 
 
+def check_gemver(ops, N, alpha, beta, update_A, dtype):
+    """GEMVER on the GPU vs the oracle.  Denominators (terms' magnitudes):
+    A_hat: |A| + |u1 v1| + |u2 v2|;  x: |x| + |beta| sum_i Am_ij |y_i| + |z|;
+    w: |w| + |alpha| sum_j Am_ij Xm_j (the new x's error carried into w)."""
+    A, u1, v1, u2, v2, w, x, y, z = ops
+    host = [t.cpu().numpy() for t in (A, u1, v1, u2, v2, w, x, y, z)]
+    wg, xg = w.clone(), x.clone()
+    Ag = A.clone()
+    dm.gemver(Ag[:, :N], u1, v1, u2, v2, wg, xg, y, z, alpha=alpha, beta=beta,
+              update_A=update_A)
+    torch.cuda.synchronize()
+    ah, wo, xo = oracle.gemver(host[0], *host[1:], alpha, beta, N=N)
+    An = host[0].astype(np.float64)[:, :N]
+    au1, av1, au2, av2, aw, ax, ay, az = (np.abs(v.astype(np.float64)) for v in host[1:])
+    zeros_m = np.zeros(An.shape[0])
+    _, sa = oracle.absdot(np.ascontiguousarray(An), np.zeros(N), ay)
+    Xm = ax + abs(beta) * (sa + av1 * (au1 @ ay) + av2 * (au2 @ ay)) + az
+    qa, _ = oracle.absdot(np.ascontiguousarray(An), Xm, zeros_m)
+    Wm = aw + abs(alpha) * (qa + au1 * (av1 @ Xm) + au2 * (av2 @ Xm))
+    err = max(scaled_error(xg.cpu().numpy(), xo, Xm), scaled_error(wg.cpu().numpy(), wo, Wm))
+    if update_A:
+        Am = np.abs(An) + np.outer(au1, av1) + np.outer(au2, av2)
+        got = Ag[:, :N].cpu().numpy()
+        err = max(err, scaled_error(got.ravel(), ah.ravel(), Am.ravel()))
+        assert torch.equal(Ag[:, N:].cpu().isnan(), A[:, N:].cpu().isnan())  # padding untouched
+    assert err <= TOL[dtype], err
+    return err
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+@pytest.mark.parametrize("M,N,pad", [(1000, 3000, 0), (3001, 257, 5), (1, 1, 0), (77, 1000, 3)])
+@pytest.mark.parametrize("update_A", [False, True])
+def test_gemver_matches_oracle(dtype, M, N, pad, update_A, path):
+    w = _w("gemver", dtype, M, N, N + pad, 5 * M + N)
+    check_gemver(inputs.generate_gemver(w, DEV), N, 1.5, -0.75, update_A, dtype)
+
+
 @pytest.mark.parametrize("name", list(inputs.OP_WORKLOADS))
 def test_op_workloads_full_size(name):
     w = inputs.OP_WORKLOADS[name]
@@ -80,9 +117,13 @@ def test_op_workloads_full_size(name):
         A, B, x = inputs.generate_gesummv(w, DEV)
         err = check_gesummv(A, B, x, w.N, 1.5, 1.2, w.dtype)
         del B
-    else:
+    elif w.op == "atax":
         A, x = inputs.generate_atax(w, DEV)
         err = check_atax(A, x, w.N, w.dtype)
+    else:
+        ops = inputs.generate_gemver(w, DEV)
+        err = check_gemver(ops, w.N, 1.5, 1.2, False, w.dtype)
+        A = x = ops
     print(f"{name}: max scaled error {err:.3e}")
     del A, x
     torch.cuda.empty_cache()

@@ -47,6 +47,15 @@ MUTANTS = [
     ("atax_dropped_x", "for (int64_t j = 0; j < N; ++j) tmp += (double)A[i * lda + j] * (double)x[j];",
      "for (int64_t j = 0; j < N; ++j) tmp += (double)A[i * lda + j];", 0),
     ("atax_f64_tmp_uncompensated", "const double tmp = t_hi + t_lo;", "const double tmp = t_hi;", 0),
+    ("gemver_wrong_v", "+ (double)u1[i] * (double)v1[j]", "+ (double)u1[i] * (double)v2[j]", 0),
+    ("gemver_x_without_z", "xo[j] = (double)x[j] + beta * acc + (double)z[j];",
+     "xo[j] = (double)x[j] + beta * acc;", 0),
+    ("gemver_w_uses_old_x", "for (int64_t j = 0; j < N; ++j) acc += ahat[i * N + j] * xo[j];",
+     "for (int64_t j = 0; j < N; ++j) acc += ahat[i * N + j] * (double)x[j];", 0),
+    ("gemver_alpha_beta_swapped", "wo[i] = (double)w[i] + alpha * acc;",
+     "wo[i] = (double)w[i] + beta * acc;", 0),
+    ("gemver_f64_dropped_update_error", "ahat[i * N + j] = s2 + ((t1 + t2) + (e1 + e2));",
+     "ahat[i * N + j] = s2;", 0),
 ]
 
 

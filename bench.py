@@ -8,10 +8,14 @@ One step = one dualmv call over the whole workload (default: the 16384 x
   python bench.py --impl reference ...   (the CPU oracle, timed on the host)
 
 Metric: effective bandwidth = (bytes of the logical A, of p and r read and of
-q and s written) / device time, in GB/s (1e9 B/s).  The inputs (1 GiB) are
-larger than L2 (129 MB), so consecutive steps cannot hit in L2.  Device time
-comes from CUDA events on the launching stream, bracketed by a barrier and a
-device synchronisation; with several ranks the slowest rank's time counts.
+q and s written) / device time, in GB/s (1e9 B/s).  The default inputs (1 GiB)
+are larger than L2 (129 MB), so consecutive steps cannot hit in L2.  A
+workload that fits in twice the L2 is timed call by call instead, with a
+256 MiB buffer written between calls (outside the events) to evict it, and a
+hot-L2 figure is added from a CUDA graph of 100 back-to-back calls.  Device
+time comes from CUDA events on the launching stream, bracketed by a barrier
+and a device synchronisation; with several ranks the slowest rank's time
+counts.
 Per-step times are also summarised with the trimmed mean of Eq. 3
 (R timings sorted, k lowest and k highest dropped).
 
@@ -39,8 +43,11 @@ METRIC = "dualmv effective HBM GB/s (bytes of A+vectors / device time) and % of 
 DEFAULT_WORKLOAD = "f32_16384x16384"
 FALLBACK_HBM_GBS = 6800.0
 KERNEL_SOURCES = ("paper_2512_22147_gb300/csrc/dualmv_kernels.cuh",
+                  "paper_2512_22147_gb300/csrc/dualmv_f64e.cuh",
                   "paper_2512_22147_gb300/csrc/dualmv.cu")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+FLUSH_BYTES = 256 << 20      # written between timed calls of an L2-sized workload
+GRAPH_CALLS = 100            # calls captured in one CUDA graph (hot-L2 figure)
 
 
 # ------------------------------------------------------------- helpers ----
@@ -85,6 +92,80 @@ def recorded_traffic(workload: str):
     if not ent or ent.get("kernel_source_hash") != kernel_source_hash():
         return None
     return ent.get("dram_bytes_per_launch")
+
+
+_UNIT_SCALE = {"byte": 1.0, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "Tbyte": 1e12,
+               "B": 1.0, "KB": 1e3, "MB": 1e6, "GB": 1e9,
+               "nsecond": 1e-3, "usecond": 1.0, "msecond": 1e3, "second": 1e6,
+               "ns": 1e-3, "us": 1.0, "ms": 1e3, "s": 1e6}
+
+
+def parse_launch_list(path: str):
+    """Launches of an ncu ``--csv --log-file`` metrics capture:
+    ``[(id, kernel name, {metric: value in bytes or microseconds})]`` in
+    launch order."""
+    import csv
+    with open(path, newline="") as f:
+        lines = [ln for ln in f if ln.startswith('"')]
+    rows = list(csv.reader(lines))
+    hdr = rows[0]
+    ix = {h: i for i, h in enumerate(hdr)}
+    launches = {}
+    for row in rows[1:]:
+        lid = int(row[ix["ID"]])
+        name = row[ix["Kernel Name"]]
+        unit = row[ix["Metric Unit"]]
+        val = float(row[ix["Metric Value"]].replace(",", ""))
+        ent = launches.setdefault(lid, (name, {}))
+        ent[1][row[ix["Metric Name"]]] = val * _UNIT_SCALE.get(unit, 1.0)
+    return [(lid, n, m) for lid, (n, m) in sorted(launches.items())]
+
+
+def short_kernel_name(name: str) -> str:
+    name = name.split("(")[0]
+    return name[5:] if name.startswith("void ") else name
+
+
+def record_traffic(csv_path: str, workload: str, command: str) -> str:
+    """Write the streaming kernel's DRAM bytes per launch for ``workload``
+    into the traffic record (with the current kernel-source hash) and return
+    a markdown summary of the whole launch list: per kernel its launches,
+    total time, share and DRAM bytes per launch."""
+    launches = parse_launch_list(csv_path)
+    per = {}
+    for _, name, m in launches:
+        k = short_kernel_name(name)
+        e = per.setdefault(k, [0, 0.0, 0.0])
+        e[0] += 1
+        e[1] += m.get("gpu__time_duration.sum", 0.0)
+        e[2] += m.get("dram__bytes_read.sum", 0.0) + m.get("dram__bytes_write.sum", 0.0)
+    total = sum(e[1] for e in per.values()) or 1.0
+    stream = [k for k in per if k.startswith("dmv::dualmv_stream")]
+    if len(stream) != 1:
+        raise ValueError(f"expected one streaming kernel in the launch list, found {stream}")
+    n, _, dram = per[stream[0]]
+    rec = {}
+    if os.path.exists(TRAFFIC_FILE):
+        with open(TRAFFIC_FILE) as f:
+            rec = json.load(f)
+    rec[workload] = {
+        "kernel_source_hash": kernel_source_hash(),
+        "kernel": stream[0],
+        "dram_bytes_per_launch": int(round(dram / n)),
+        "how": "ncu launch list of bench.py on the full workload: dram__bytes_read.sum + "
+               "dram__bytes_write.sum of the streaming kernel, averaged over its launches",
+    }
+    with open(TRAFFIC_FILE, "w") as f:
+        json.dump(rec, f, indent=1)
+        f.write("\n")
+    out = [f"Command (from the repository root, on one GB300; the plain command exited 0 "
+           f"first):\n\n```\n{command}\n```\n",
+           "| kernel | launches | total us | share | us / launch | DRAM MB / launch |",
+           "|---|---|---|---|---|---|"]
+    for k, (cnt, us, b) in sorted(per.items(), key=lambda kv: -kv[1][1]):
+        out.append(f"| `{k[:120]}` | {cnt} | {us:.1f} | {100 * us / total:.1f} % | "
+                   f"{us / cnt:.2f} | {b / cnt / 1e6:.1f} |")
+    return "\n".join(out)
 
 
 class ClockSampler:
@@ -237,24 +318,42 @@ def run_native(args):
         raise RuntimeError("device fault during warm-up")
 
     K = args.steps
+    l2_bytes = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush = None
+    if nbytes <= 2 * l2_bytes:   # the operands could stay in L2 between calls
+        flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     region = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
 
-    # Timed region: K back-to-back calls, nothing recorded between them.
+    # Timed region: K back-to-back calls, nothing recorded between them; or,
+    # for an L2-sized workload, K calls each between its own events with an
+    # L2-evicting write before it, outside the events.
     sampler = ClockSampler(gpu_uuid(torch, dev))
     sampler.start()
     time.sleep(0.3)  # let the sampler start before the timed region
     barrier(world)
     torch.cuda.synchronize(dev)
-    region[0].record(stream)
-    for _ in range(K):
-        call()
-    region[1].record(stream)
+    if flush is None:
+        region[0].record(stream)
+        for _ in range(K):
+            call()
+        region[1].record(stream)
+    else:
+        flushed = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(K)]
+        for ev0, ev1 in flushed:
+            flush.zero_()
+            ev0.record(stream)
+            call()
+            ev1.record(stream)
     torch.cuda.synchronize(dev)
     barrier(world)
     clocks = sampler.stop()
     if dm.device_fault() != dm.DUALMV_SUCCESS:
         raise RuntimeError("device fault during the timed region")
-    region_ms = region[0].elapsed_time(region[1])
+    if flush is None:
+        region_ms = region[0].elapsed_time(region[1])
+    else:
+        region_ms = sum(a.elapsed_time(b) for a, b in flushed)
     region_ms = max_over_ranks(torch, region_ms, world, dev)
     ms_per_step = region_ms / K
     value = world * nbytes * K / (region_ms * 1e-3) / 1e9
@@ -276,6 +375,8 @@ def run_native(args):
     torch.cuda.synchronize(dev)
     for i in range(Ki):
         ks, ke = kern_ev[i]
+        if flush is not None:
+            flush.zero_()
         if w.op == "bicg":
             dm.dualmv_record_kernel_events(ks.cuda_event, ke.cuda_event)
         else:  # several streaming passes per call: time the whole call
@@ -306,6 +407,8 @@ def run_native(args):
     achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9
     traffic = recorded_traffic(args.workload)
 
+    hot = hot_l2_graph(torch, call, nbytes, dev) if flush is not None else None
+
     # End to end through the same public call with host buffers: pinned host
     # inputs copied in, the call, results copied out, every step.
     e2e = None
@@ -333,7 +436,9 @@ def run_native(args):
             "workload": w.name, "op": w.op, "M": w.M, "N": w.N, "lda": w.lda,
             "batch": w.batch, "dtype": w.dtype, "distribution": w.dist, "seed": w.seed,
             "bytes_per_step": nbytes,
-            "l2": "inputs larger than L2 (no flush needed)",
+            "l2": ("inputs larger than L2 (no flush needed)" if flush is None else
+                   f"L2 flushed: {FLUSH_BYTES >> 20} MiB written before each call, "
+                   "outside its events"),
             "parallelism": f"replicas x{world}",
         },
         "pct_of_peak": round(100.0 * value / (world * peak), 2),
@@ -358,11 +463,43 @@ def run_native(args):
         "instrumented_steps": Ki,
         "clocks": clocks,
     }
+    if hot is not None:
+        out["hot_l2_graph"] = hot
     if rank == 0:
         print(json.dumps(out), flush=True)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def hot_l2_graph(torch, call, nbytes, dev, reps=20):
+    """Per-call time of GRAPH_CALLS back-to-back calls captured in one CUDA
+    graph and replayed ``reps`` times: the operands stay in L2 and the host
+    launch cost is gone, which leaves the kernels' own latency."""
+    try:
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(torch.cuda.current_stream(dev))
+        with torch.cuda.stream(side):
+            call()
+        torch.cuda.current_stream(dev).wait_stream(side)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for _ in range(GRAPH_CALLS):
+                call()
+        g.replay()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            g.replay()
+        e1.record()
+        torch.cuda.synchronize(dev)
+    except Exception as ex:  # capture is a measurement extra; report why it failed
+        return {"error": f"{type(ex).__name__}: {ex}"[:300]}
+    per_call_ms = e0.elapsed_time(e1) / (reps * GRAPH_CALLS)
+    return {"calls_per_graph": GRAPH_CALLS, "replays": reps,
+            "per_call_us": round(per_call_ms * 1e3, 3),
+            "GBs": round(nbytes / (per_call_ms * 1e-3) / 1e9, 2)}
 
 
 def run_e2e(torch, dm, w, A, p, r, dev, stream, steps):
@@ -495,7 +632,14 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--record-traffic", metavar="CSV", default=None,
+                    help="record the streaming kernel's DRAM bytes per launch for --workload "
+                         "from an ncu launch-list CSV of this bench, then exit")
+    ap.add_argument("--record-command", default="", help="the command that made the CSV")
     args = ap.parse_args(argv)
+    if args.record_traffic:
+        print(record_traffic(args.record_traffic, args.workload, args.record_command))
+        return
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":

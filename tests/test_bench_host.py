@@ -114,3 +114,35 @@ def test_max_over_ranks_with_two_gloo_ranks():
         assert p.exitcode == 0
     res = sorted(q.get(timeout=10) for _ in range(2))
     assert res == [(0, 15.0), (1, 15.0)]
+
+
+def test_launch_list_parser_and_traffic_record(tmp_path, monkeypatch):
+    """The ncu CSV parser groups metric rows by launch, converts units, and
+    the traffic record keeps the streaming kernel's bytes per launch."""
+    hdr = ('"ID","Process ID","Process Name","Host Name","Kernel Name","Context","Stream",'
+           '"Block Size","Grid Size","Device","CC","Section Name","Metric Name","Metric Unit",'
+           '"Metric Value"\n')
+
+    def row(i, name, metric, unit, val):
+        return (f'"{i}","1","python3","h","{name}","1","7","(288, 1, 1)","(152, 1, 1)","0",'
+                f'"10.3","Command line profiler metrics","{metric}","{unit}","{val}"\n')
+
+    k = "void dmv::dualmv_stream_kernel<float, 8, 4, 6, 1, 0>(dmv::Params<float>)"
+    c = "void dmv::dualmv_combine_kernel<float>(dmv::Params<float>, int, int)"
+    lines = ["==PROF== Connected to process 1\n", hdr]
+    for i, (name, us, mb) in enumerate([(k, 160.0, 1000.0), (c, 8.0, 4.0), (k, 170.0, 1002.0)]):
+        lines += [row(i, name, "dram__bytes_read.sum", "Mbyte", f"{mb:.1f}"),
+                  row(i, name, "dram__bytes_write.sum", "Kbyte", "500"),
+                  row(i, name, "gpu__time_duration.sum", "ns", f"{us * 1e3:.0f}")]
+    csv_path = tmp_path / "launches.csv"
+    csv_path.write_text("".join(lines))
+    parsed = bench.parse_launch_list(str(csv_path))
+    assert [p[0] for p in parsed] == [0, 1, 2]
+    assert parsed[0][2]["dram__bytes_read.sum"] == 1000e6
+    assert parsed[0][2]["dram__bytes_write.sum"] == 500e3
+    rec = tmp_path / "traffic.json"
+    monkeypatch.setattr(bench, "TRAFFIC_FILE", str(rec))
+    md = bench.record_traffic(str(csv_path), "wl", "cmd")
+    assert "| `dmv::dualmv_stream_kernel<float, 8, 4, 6, 1, 0>` | 2 | 330.0 |" in md
+    assert bench.recorded_traffic("wl") == int(1001e6 + 500e3)
+    assert bench.recorded_traffic("other") is None

@@ -311,6 +311,22 @@ def run_native(args):
         def call():
             dm.gemver(A[:, : w.N], u1, v1, u2, v2, wv, x, y, z, alpha=1.5, beta=1.2)
 
+    tuned = None
+    if args.tune:
+        if w.op != "bicg" or w.batched:
+            raise SystemExit("--tune applies to one unbatched dual product")
+        t0 = time.time()
+        rep = dm.tune(Av, p, r, repeats=30, trim=3, max_rounds=4, candidates=8, min_gain=0.01,
+                      flush_l2=flush_needed(torch, nbytes, dev))
+        torch.cuda.synchronize(dev)
+        v = dm.dualmv_variant_info({"f32": 0, "f64": 1, "i32": 2}[w.dtype], rep["best"])
+        tuned = {k: (float(f"{val:.6g}") if isinstance(val, float) else val)
+                 for k, val in rep.items() if k not in ("q", "s", "trace")}
+        tuned["trace"] = [{k: (float(f"{val:.6g}") if isinstance(val, float) else val)
+                           for k, val in st.items()} for st in rep["trace"]]
+        tuned["variant"] = {f: getattr(v, f) for f, _ in v._fields_}
+        tuned["seconds"] = round(time.time() - t0, 2)
+
     for _ in range(args.warmup):
         call()
     torch.cuda.synchronize(dev)
@@ -318,9 +334,8 @@ def run_native(args):
         raise RuntimeError("device fault during warm-up")
 
     K = args.steps
-    l2_bytes = torch.cuda.get_device_properties(dev).L2_cache_size
     flush = None
-    if nbytes <= 2 * l2_bytes:   # the operands could stay in L2 between calls
+    if flush_needed(torch, nbytes, dev):   # the operands could stay in L2 between calls
         flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     region = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
 
@@ -465,11 +480,18 @@ def run_native(args):
     }
     if hot is not None:
         out["hot_l2_graph"] = hot
+    if tuned is not None:
+        out["tuned"] = tuned
     if rank == 0:
         print(json.dumps(out), flush=True)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def flush_needed(torch, nbytes: int, dev) -> bool:
+    """True when a workload's operands could stay in L2 between calls."""
+    return nbytes <= 2 * torch.cuda.get_device_properties(dev).L2_cache_size
 
 
 def hot_l2_graph(torch, call, nbytes, dev, reps=20):
@@ -632,6 +654,9 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--tune", action="store_true",
+                    help="run the variant tuner (Eq. 3-5) on the workload before warm-up; "
+                         "the timed calls then use the variant it chose")
     ap.add_argument("--record-traffic", metavar="CSV", default=None,
                     help="record the streaming kernel's DRAM bytes per launch for --workload "
                          "from an ncu launch-list CSV of this bench, then exit")

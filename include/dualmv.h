@@ -255,6 +255,136 @@ dualmv_status dualmv_plan(int64_t M, int64_t N, int64_t batch,
                           int64_t elem_bytes, int64_t acc_bytes,
                           int64_t num_sms, dualmv_plan_t *out);
 
+/* ---- kernel variants and the variant tuner (Section 3.2, Eq. 3-5) ------
+ * The dual product of one unbatched problem on the TMA path can run any of
+ * several compiled variants of its streaming kernel, which differ in tile
+ * shape (consumer warps x rows per warp), TMA ring depth and, for fp64,
+ * arithmetic (double-float on the FP32 pipes, or native fp64 FMA).  Entry 0
+ * of each element type's table is the default that untuned calls use.
+ * Batched calls, single-sided products (GESUMMV, ATAX, GEMVER) and the
+ * plain-load path always use their default kernel. */
+enum { DUALMV_DTYPE_F32 = 0, DUALMV_DTYPE_F64 = 1, DUALMV_DTYPE_I32 = 2 };
+enum {
+    DUALMV_KERNEL_STREAM = 0, /* TMA ring, native arithmetic of the dtype  */
+    DUALMV_KERNEL_F64E = 1    /* TMA ring per warp, double-float fp64      */
+};
+typedef struct dualmv_variant_t {
+    int32_t index;          /* position in its dtype's table              */
+    int32_t kernel;         /* DUALMV_KERNEL_*                            */
+    int32_t warps;          /* consumer warps per CTA                     */
+    int32_t rows_per_warp;  /* rows of a tile per consumer warp           */
+    int32_t stages;         /* TMA ring depth                             */
+    int32_t band_cols;      /* columns per band                           */
+    int32_t tile_rows;      /* warps * rows_per_warp                      */
+    int32_t threads;        /* threads per CTA (consumers + producer)     */
+    int64_t smem_bytes;     /* dynamic shared memory per CTA              */
+} dualmv_variant_t;
+
+/* Number of variants for `dtype` (DUALMV_DTYPE_*), or -1 for an unknown
+ * dtype.  Host only. */
+int32_t dualmv_variant_count(int32_t dtype);
+
+/* Description of variant `index` of `dtype`.  DUALMV_ERR_INVALID_VALUE for
+ * an unknown dtype, an index out of range or a NULL `out`.  Host only. */
+dualmv_status dualmv_variant_info(int32_t dtype, int32_t index, dualmv_variant_t *out);
+
+/* Forces variant `index` for every eligible call of `dtype` in this
+ * process (-1 restores the normal choice: a tuned variant for the shape if
+ * dualmv_tune_* recorded one, else entry 0).  Returns the previous setting,
+ * or -2 for an unknown dtype or an index out of range.  Meant for tests. */
+int32_t dualmv_set_variant(int32_t dtype, int32_t index);
+
+/* The variant recorded by dualmv_tune_* for this dtype and shape, or -1. */
+int32_t dualmv_tuned_variant(int32_t dtype, int64_t M, int64_t N, int64_t lda);
+
+/* Forgets every recorded tuning result. */
+void dualmv_tune_clear(void);
+
+/* The variant the calling thread's last dual-product call launched: its
+ * table index, or -1 if that call ran no TMA streaming kernel (an empty
+ * problem, the plain-load path, a batched or single-sided call, or an
+ * error).  Instrumentation for tests and benchmarks. */
+int32_t dualmv_last_variant(void);
+
+/* Trimmed mean of Eq. 3: the R values sorted, the k smallest and k largest
+ * dropped, the rest averaged.  DUALMV_ERR_INVALID_VALUE unless R > 2k,
+ * k >= 0 and both pointers are non-NULL.  Host only; `t` is not modified. */
+dualmv_status dualmv_trimmed_mean(const double *t, int64_t R, int64_t k, double *out);
+
+typedef struct dualmv_tune_config_t {
+    int32_t repeats;     /* R timed calls per candidate (R > 2 * trim)        */
+    int32_t trim;        /* k of Eq. 3                                        */
+    int32_t max_rounds;  /* D: rounds of candidate generation at most         */
+    int32_t candidates;  /* N: candidates per round at most (>= 1)            */
+    double min_gain;     /* stop once a round's best candidate is not faster  */
+                         /* than the baseline by at least this fraction       */
+    int32_t flush_l2;    /* nonzero: write a buffer of twice the L2 size      */
+                         /* before every timed call, outside its events       */
+} dualmv_tune_config_t;
+
+/* One evaluated candidate, in evaluation order. */
+typedef struct dualmv_tune_step_t {
+    int32_t index;       /* variant                                           */
+    int32_t round;       /* d (0-based)                                       */
+    int32_t feasible;    /* passed functional equivalence (Eq. 4)             */
+    int32_t pad_;
+    double ms;           /* trimmed mean (Eq. 3); 0 if not feasible           */
+    double fe;           /* largest per-element error against the baseline   */
+} dualmv_tune_step_t;
+
+#define DUALMV_TUNE_MAX_TRACE 64
+
+typedef struct dualmv_tune_result_t {
+    int32_t best;        /* index of the chosen variant (the final baseline)  */
+    int32_t rounds;      /* rounds run                                        */
+    int32_t evaluated;   /* candidates run, the initial baseline excluded     */
+    int32_t rejected;    /* candidates that failed functional equivalence     */
+    double baseline_ms;  /* trimmed mean of variant 0 (K^(0))                 */
+    double best_ms;      /* trimmed mean of the chosen variant                */
+    double worst_fe;     /* largest FE error among accepted candidates        */
+    int32_t trace_len;   /* entries of `trace` filled (min(evaluated, max))  */
+    int32_t pad_;
+    dualmv_tune_step_t trace[DUALMV_TUNE_MAX_TRACE];
+} dualmv_tune_result_t;
+
+/* Tunes the variant for this problem by the loop of Section 3.2:
+ *   K^(0) = variant 0.  In round d, up to `candidates` variants not tried
+ *   before that differ from K^(d) in one property (kernel, warps, rows per
+ *   warp or stages) are run once and checked for functional equivalence
+ *   with K^(d) (Eq. 4); each that passes is timed `repeats` times and
+ *   scored by the trimmed mean of Eq. 3.  The fastest feasible candidate
+ *   (Eq. 5) becomes K^(d+1) if it beats K^(d) by more than `min_gain`;
+ *   otherwise, or after `max_rounds` rounds, or when no untried neighbour is
+ *   left, the loop stops.
+ * Functional equivalence: int32 outputs equal bit for bit; floating-point
+ *   outputs within the parity bar |x - x_base| <= tol * sum|A||v| per
+ *   element (tol 1e-5 for f32, 1e-12 for f64), the sums |A||p| and |A|^T|r|
+ *   computed in double by separate simple kernels.
+ * The chosen variant is recorded for (dtype, M, N, lda) and used by later
+ *   calls of that shape (see dualmv_tuned_variant), and its outputs are
+ *   left in q and s.
+ * Synchronous: blocks the calling thread on `stream` while it measures.
+ *   Allocates its scratch from the library's pool on `stream`.
+ * Errors: DUALMV_ERR_INVALID_VALUE for the dualmv_* argument errors, NULL
+ *   `cfg` or `res`, repeats <= 2 * trim, trim < 0, max_rounds < 0,
+ *   candidates < 1 or a negative or NaN min_gain (nothing enqueued);
+ *   DUALMV_ERR_TIMEOUT if a candidate's kernel gave up a bounded wait;
+ *   otherwise as dualmv_*.  Problems off the TMA path (misaligned A,
+ *   DUALMV_PATH_DIRECT or DUALMV_PATH_TMA_NATIVE_F64 in force) and empty
+ *   problems run the default once and report evaluated = 0. */
+dualmv_status dualmv_tune_f32(int64_t M, int64_t N, const float *A, int64_t lda,
+                              const float *p, const float *r, float *q, float *s,
+                              const dualmv_tune_config_t *cfg,
+                              dualmv_tune_result_t *res, dualmv_stream_t stream);
+dualmv_status dualmv_tune_f64(int64_t M, int64_t N, const double *A, int64_t lda,
+                              const double *p, const double *r, double *q, double *s,
+                              const dualmv_tune_config_t *cfg,
+                              dualmv_tune_result_t *res, dualmv_stream_t stream);
+dualmv_status dualmv_tune_i32(int64_t M, int64_t N, const int32_t *A, int64_t lda,
+                              const int32_t *p, const int32_t *r, int64_t *q, int64_t *s,
+                              const dualmv_tune_config_t *cfg,
+                              dualmv_tune_result_t *res, dualmv_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -32,6 +32,12 @@ DUALMV_PATH_TMA = 1
 DUALMV_PATH_DIRECT = 2
 DUALMV_PATH_TMA_NATIVE_F64 = 3
 
+DUALMV_DTYPE_F32 = 0
+DUALMV_DTYPE_F64 = 1
+DUALMV_DTYPE_I32 = 2
+DUALMV_KERNEL_STREAM = 0
+DUALMV_KERNEL_F64E = 1
+
 EXPORTED = (
     "dualmv_f32", "dualmv_f64", "dualmv_i32",
     "dualmv_f32_strided_batched", "dualmv_f64_strided_batched",
@@ -41,6 +47,9 @@ EXPORTED = (
     "dualmv_f32_noalloc", "dualmv_f32_noalloc_scratch_bytes",
     "dualmv_gesummv_f32", "dualmv_gesummv_f64", "dualmv_atax_f32", "dualmv_atax_f64",
     "dualmv_gemver_f32", "dualmv_gemver_f64",
+    "dualmv_variant_count", "dualmv_variant_info", "dualmv_set_variant",
+    "dualmv_tuned_variant", "dualmv_tune_clear", "dualmv_trimmed_mean",
+    "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32", "dualmv_last_variant",
 )
 
 
@@ -57,6 +66,35 @@ class Plan(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in (
         "band_cols", "tile_rows", "bands", "stripes", "tiles", "grid",
         "max_segments", "workspace_bytes", "smem_bytes", "threads")]
+
+
+class Variant(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "index", "kernel", "warps", "rows_per_warp", "stages", "band_cols", "tile_rows",
+        "threads")] + [("smem_bytes", ctypes.c_int64)]
+
+
+class TuneConfig(ctypes.Structure):
+    _fields_ = [("repeats", ctypes.c_int32), ("trim", ctypes.c_int32),
+                ("max_rounds", ctypes.c_int32), ("candidates", ctypes.c_int32),
+                ("min_gain", ctypes.c_double), ("flush_l2", ctypes.c_int32)]
+
+
+TUNE_MAX_TRACE = 64
+
+
+class TuneStep(ctypes.Structure):
+    _fields_ = [("index", ctypes.c_int32), ("round", ctypes.c_int32),
+                ("feasible", ctypes.c_int32), ("pad_", ctypes.c_int32),
+                ("ms", ctypes.c_double), ("fe", ctypes.c_double)]
+
+
+class TuneResult(ctypes.Structure):
+    _fields_ = [("best", ctypes.c_int32), ("rounds", ctypes.c_int32),
+                ("evaluated", ctypes.c_int32), ("rejected", ctypes.c_int32),
+                ("baseline_ms", ctypes.c_double), ("best_ms", ctypes.c_double),
+                ("worst_fe", ctypes.c_double), ("trace_len", ctypes.c_int32),
+                ("pad_", ctypes.c_int32), ("trace", TuneStep * TUNE_MAX_TRACE)]
 
 
 def _load() -> ctypes.CDLL:
@@ -100,6 +138,21 @@ def _load() -> ctypes.CDLL:
     lib.dualmv_record_kernel_events.restype = None
     lib.dualmv_plan.argtypes = [i64, i64, i64, i64, i64, i64, ctypes.POINTER(Plan)]
     lib.dualmv_plan.restype = st
+    i32 = ctypes.c_int32
+    lib.dualmv_variant_count.argtypes, lib.dualmv_variant_count.restype = [i32], i32
+    lib.dualmv_variant_info.argtypes = [i32, i32, ctypes.POINTER(Variant)]
+    lib.dualmv_variant_info.restype = st
+    lib.dualmv_set_variant.argtypes, lib.dualmv_set_variant.restype = [i32, i32], i32
+    lib.dualmv_tuned_variant.argtypes, lib.dualmv_tuned_variant.restype = [i32, i64, i64, i64], i32
+    lib.dualmv_tune_clear.argtypes, lib.dualmv_tune_clear.restype = [], None
+    lib.dualmv_last_variant.argtypes, lib.dualmv_last_variant.restype = [], i32
+    lib.dualmv_trimmed_mean.argtypes = [ctypes.POINTER(ctypes.c_double), i64, i64,
+                                        ctypes.POINTER(ctypes.c_double)]
+    lib.dualmv_trimmed_mean.restype = st
+    for t in ("f32", "f64", "i32"):
+        f = getattr(lib, f"dualmv_tune_{t}")
+        f.argtypes = single[:-1] + [ctypes.POINTER(TuneConfig), ctypes.POINTER(TuneResult), vp]
+        f.restype = st
     return lib
 
 
@@ -209,3 +262,64 @@ def dualmv_plan(M, N, batch, elem_bytes, acc_bytes, num_sms) -> Plan:
     if rc != DUALMV_SUCCESS:
         raise DualmvError(rc, "dualmv_plan")
     return out
+
+
+# ---------------------------------------------------- variants and tuner ----
+
+def dualmv_variant_count(dtype: int) -> int:
+    return _lib.dualmv_variant_count(dtype)
+
+
+def dualmv_variant_info(dtype: int, index: int) -> Variant:
+    out = Variant()
+    rc = _lib.dualmv_variant_info(dtype, index, ctypes.byref(out))
+    if rc != DUALMV_SUCCESS:
+        raise DualmvError(rc, "dualmv_variant_info")
+    return out
+
+
+def dualmv_set_variant(dtype: int, index: int) -> int:
+    old = _lib.dualmv_set_variant(dtype, index)
+    if old == -2:
+        raise ValueError(f"unknown dtype {dtype} or variant {index}")
+    return old
+
+
+def dualmv_tuned_variant(dtype: int, M: int, N: int, lda: int) -> int:
+    return _lib.dualmv_tuned_variant(dtype, M, N, lda)
+
+
+def dualmv_tune_clear() -> None:
+    _lib.dualmv_tune_clear()
+
+
+def dualmv_last_variant() -> int:
+    return _lib.dualmv_last_variant()
+
+
+def dualmv_trimmed_mean(times, k: int) -> float:
+    arr = (ctypes.c_double * len(times))(*times)
+    out = ctypes.c_double()
+    rc = _lib.dualmv_trimmed_mean(arr, len(times), k, ctypes.byref(out))
+    if rc != DUALMV_SUCCESS:
+        raise DualmvError(rc, "dualmv_trimmed_mean")
+    return out.value
+
+
+def _tune(tag, M, N, A, lda, p, r, q, s, cfg, res, stream):
+    return getattr(_lib, f"dualmv_tune_{tag}")(M, N, A, lda, p, r, q, s,
+                                               ctypes.byref(cfg) if cfg is not None else None,
+                                               ctypes.byref(res) if res is not None else None,
+                                               stream)
+
+
+def dualmv_tune_f32(M, N, A, lda, p, r, q, s, cfg, res, stream):
+    return _tune("f32", M, N, A, lda, p, r, q, s, cfg, res, stream)
+
+
+def dualmv_tune_f64(M, N, A, lda, p, r, q, s, cfg, res, stream):
+    return _tune("f64", M, N, A, lda, p, r, q, s, cfg, res, stream)
+
+
+def dualmv_tune_i32(M, N, A, lda, p, r, q, s, cfg, res, stream):
+    return _tune("i32", M, N, A, lda, p, r, q, s, cfg, res, stream)

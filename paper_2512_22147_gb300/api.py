@@ -197,3 +197,55 @@ def gemver(A: torch.Tensor, u1: torch.Tensor, v1: torch.Tensor, u2: torch.Tensor
     if rc != B_.DUALMV_SUCCESS:
         raise B_.DualmvError(rc, f"dualmv_gemver_{tag}")
     return w, x
+
+
+_DTYPE_CODE = {torch.float32: B.DUALMV_DTYPE_F32, torch.float64: B.DUALMV_DTYPE_F64,
+               torch.int32: B.DUALMV_DTYPE_I32}
+
+
+def variants(dtype: torch.dtype) -> list[dict]:
+    """The compiled kernel variants for ``dtype`` (entry 0 is the default)."""
+    code = _DTYPE_CODE[dtype]
+    out = []
+    for i in range(B.dualmv_variant_count(code)):
+        v = B.dualmv_variant_info(code, i)
+        out.append({f: getattr(v, f) for f, _ in v._fields_})
+    return out
+
+
+def tune(A: torch.Tensor, p: torch.Tensor, r: torch.Tensor, q: torch.Tensor | None = None,
+         s: torch.Tensor | None = None, repeats: int = 30, trim: int = 3, max_rounds: int = 4,
+         candidates: int = 4, min_gain: float = 0.01, flush_l2: bool = True,
+         stream: torch.cuda.Stream | None = None) -> dict:
+    """Tune the kernel variant for this problem's shape (Section 3.2: Eq. 3
+    scores, the Eq. 4 equivalence gate, the Eq. 5 choice); later ``dualmv``
+    calls of the same shape use the result.  Blocks until done.  Returns the
+    tuner's report; q and s hold the chosen variant's outputs."""
+    if A.dtype not in _TAG or A.dim() != 2:
+        raise ValueError("tune takes one 2-D float32, float64 or int32 problem")
+    M, N = A.shape
+    if N > 1 and A.stride(1) != 1:
+        raise ValueError("A's last dimension must be contiguous")
+    lda = max(A.stride(0), N, 1) if M > 1 else max(N, 1)
+    out_t = _OUT[A.dtype]
+    if q is None:
+        q = torch.empty(M, dtype=out_t, device=A.device)
+    if s is None:
+        s = torch.empty(N, dtype=out_t, device=A.device)
+    for t_, n in ((p, "p"), (r, "r")):
+        if t_.dtype != A.dtype or t_.device != A.device or not t_.is_contiguous():
+            raise ValueError(f"{n} must be a contiguous vector of A's dtype on its device")
+    cfg = B.TuneConfig(repeats, trim, max_rounds, candidates, min_gain, int(flush_l2))
+    res = B.TuneResult()
+    strm = stream if stream is not None else torch.cuda.current_stream(A.device)
+    fn = getattr(B, f"dualmv_tune_{_TAG[A.dtype]}")
+    rc = fn(M, N, A.data_ptr(), lda, p.data_ptr(), r.data_ptr(), q.data_ptr(), s.data_ptr(),
+            cfg, res, strm.cuda_stream)
+    if rc != B.DUALMV_SUCCESS:
+        raise B.DualmvError(rc, "dualmv_tune")
+    rep = {f: getattr(res, f) for f, _ in res._fields_
+           if f not in ("trace", "trace_len", "pad_")}
+    rep["trace"] = [{"index": st.index, "round": st.round, "feasible": bool(st.feasible),
+                     "ms": st.ms, "fe": st.fe} for st in res.trace[:res.trace_len]]
+    rep["q"], rep["s"] = q, s
+    return rep

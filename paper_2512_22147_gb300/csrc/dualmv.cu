@@ -7,15 +7,20 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <atomic>
 #include <cstdint>
 #include <cstdlib>
 #include <cstring>
+#include <map>
 #include <mutex>
+#include <tuple>
 #include <type_traits>
+#include <vector>
 
 #include "dualmv_kernels.cuh"
 #include "dualmv_f64e.cuh"
+#include "dualmv_tune.cuh"
 
 namespace {
 
@@ -53,6 +58,7 @@ enum class Kind { kTma, kDirect, kF64e };
 thread_local int g_last_cuda_error = 0;
 thread_local cudaEvent_t g_kernel_ev_start = nullptr;
 thread_local cudaEvent_t g_kernel_ev_stop = nullptr;
+thread_local int32_t g_last_variant = -1;
 int g_path = DUALMV_PATH_AUTO;
 
 dualmv_status cuda_fail(cudaError_t e) {
@@ -175,42 +181,51 @@ struct Geometry {
 };
 
 template <typename T>
-Geometry generic_geometry(bool tma) {
-    constexpr int rpw = sizeof(T) == 4 ? kRpw4 : kRpw8;
+constexpr int default_rpw() { return sizeof(T) == 4 ? kRpw4 : kRpw8; }
+
+template <typename T, int W, int RPW, int S>
+Geometry stream_geometry(bool tma) {
     Geometry g;
     g.band_cols = kBandCols;
-    g.tile_rows = kWarps * rpw;
+    g.tile_rows = W * RPW;
     g.box_rows = g.tile_rows;
-    g.smem = tma ? dmv::SmemLayout<T, kWarps, rpw, kStages, true>::kTotal
-                 : dmv::SmemLayout<T, kWarps, rpw, kStages, false>::kTotal;
-    g.threads = (kWarps + (tma ? 1 : 0)) * 32;
+    g.smem = tma ? dmv::SmemLayout<T, W, RPW, S, true>::kTotal
+                 : dmv::SmemLayout<T, W, RPW, S, false>::kTotal;
+    g.threads = (W + (tma ? 1 : 0)) * 32;
     return g;
 }
 
+template <int W, int RPW, int S>
+Geometry f64e_geometry() {
+    Geometry g;
+    g.band_cols = kF64eBand;
+    g.tile_rows = W * RPW;
+    g.box_rows = RPW;  // one box per consumer warp
+    g.smem = dmv::F64eLayout<W, RPW, S, kF64eBand>::kTotal;
+    g.threads = (W + 1) * 32;
+    return g;
+}
+
+template <typename T>
+Geometry generic_geometry(bool tma) {
+    return stream_geometry<T, kWarps, default_rpw<T>(), kStages>(tma);
+}
+
 Geometry geometry(int64_t elem_bytes, int64_t acc_bytes, Kind kind) {
-    if (kind == Kind::kF64e) {
-        Geometry g;
-        g.band_cols = kF64eBand;
-        g.tile_rows = kF64eWarps * kF64eRpw;
-        g.box_rows = kF64eRpw;  // one box per consumer warp
-        g.smem = dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand>::kTotal;
-        g.threads = (kF64eWarps + 1) * 32;
-        return g;
-    }
+    if (kind == Kind::kF64e) return f64e_geometry<kF64eWarps, kF64eRpw, kF64eStages>();
     const bool tma = kind == Kind::kTma;
     if (elem_bytes == 8) return generic_geometry<double>(tma);
     return acc_bytes == 8 ? generic_geometry<int32_t>(tma) : generic_geometry<float>(tma);
 }
 
-dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
-                        int64_t acc_bytes, int64_t ctas, Kind kind, dualmv_plan_t *pl) {
+dualmv_status make_plan_geo(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
+                            int64_t acc_bytes, int64_t ctas, const Geometry &geo,
+                            dualmv_plan_t *pl) {
     if (M <= 0 || N <= 0 || batch <= 0 || ctas <= 0 || pl == nullptr)
         return DUALMV_ERR_INVALID_VALUE;
     if ((elem_bytes != 4 && elem_bytes != 8) || (acc_bytes != 4 && acc_bytes != 8) ||
         acc_bytes < elem_bytes)
         return DUALMV_ERR_INVALID_VALUE;
-    if (kind == Kind::kF64e && elem_bytes != 8) return DUALMV_ERR_INVALID_VALUE;
-    const Geometry geo = geometry(elem_bytes, acc_bytes, kind);
     const int64_t bm = geo.tile_rows;
     dualmv_plan_t p;
     std::memset(&p, 0, sizeof p);
@@ -242,6 +257,15 @@ dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
     return DUALMV_SUCCESS;
 }
 
+dualmv_status make_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
+                        int64_t acc_bytes, int64_t ctas, Kind kind, dualmv_plan_t *pl) {
+    if (kind == Kind::kF64e && elem_bytes != 8) return DUALMV_ERR_INVALID_VALUE;
+    if ((elem_bytes != 4 && elem_bytes != 8) || (acc_bytes != 4 && acc_bytes != 8))
+        return DUALMV_ERR_INVALID_VALUE;
+    return make_plan_geo(M, N, batch, elem_bytes, acc_bytes, ctas,
+                         geometry(elem_bytes, acc_bytes, kind), pl);
+}
+
 // ------------------------------------------------------------ validation --
 
 dualmv_status validate(int64_t M, int64_t N, const void *A, int64_t lda, int64_t strideA,
@@ -271,18 +295,20 @@ dualmv_status validate(int64_t M, int64_t N, const void *A, int64_t lda, int64_t
     return DUALMV_SUCCESS;
 }
 
-bool fault_injected_alloc() {
+bool fault_injected(const char *what) {
     const char *v = std::getenv("DUALMV_FAULT_INJECT");
-    return v != nullptr && std::strcmp(v, "alloc") == 0;
+    return v != nullptr && std::strcmp(v, what) == 0;
 }
+
+bool fault_injected_alloc() { return fault_injected("alloc"); }
 
 // ------------------------------------------------------------- launching --
 
-template <typename T, bool kTma, bool k3d, int kOut = dmv::kOutBoth, bool kRank2 = false>
+template <typename T, bool kTma, bool k3d, int kOut = dmv::kOutBoth, bool kRank2 = false,
+          int W = kWarps, int RPW = default_rpw<T>(), int S = kStages>
 cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                           int dev, cudaStream_t stream) {
-    constexpr int rpw = sizeof(T) == 4 ? kRpw4 : kRpw8;
-    auto kern = dmv::dualmv_stream_kernel<T, kWarps, rpw, kStages, kTma, k3d, kOut, kRank2>;
+    auto kern = dmv::dualmv_stream_kernel<T, W, RPW, S, kTma, k3d, kOut, kRank2>;
     // The shared-memory opt-in is per device and per kernel; set it once.
     static std::atomic<uint64_t> opted_in{0};
     const uint64_t bit = 1ull << (dev & 63);
@@ -321,11 +347,11 @@ int combine_chunks(int64_t bands) {
     return c;
 }
 
-template <bool k3d, int kOut = dmv::kOutBoth>
+template <bool k3d, int kOut = dmv::kOutBoth, int W = kF64eWarps, int RPW = kF64eRpw,
+          int S = kF64eStages>
 cudaError_t launch_f64e(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                         int dev, cudaStream_t stream) {
-    auto kern = dmv::dualmv_stream_f64e_kernel<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand,
-                                               k3d, kOut>;
+    auto kern = dmv::dualmv_stream_f64e_kernel<W, RPW, S, kF64eBand, k3d, kOut>;
     static std::atomic<uint64_t> opted_in{0};
     const uint64_t bit = 1ull << (dev & 63);
     if (!(opted_in.load(std::memory_order_acquire) & bit)) {
@@ -376,6 +402,135 @@ cudaError_t zero_fill(Acc *out, int64_t len, int64_t stride, int64_t batch,
     return cudaGetLastError();
 }
 
+// -------------------------------------------------------------- variants --
+//
+// Compiled variants of the streaming kernel for one unbatched dual product
+// on the TMA path: the search space of the tuner.  Entry 0 of each table is
+// the kernel untuned calls use, so selecting it changes nothing.
+
+using LaunchFn = cudaError_t (*)(const CUtensorMap &, const Params &, const dualmv_plan_t &,
+                                 int, cudaStream_t);
+
+struct Variant {
+    dualmv_variant_t info;
+    Kind kind;
+    Geometry geo;
+    LaunchFn launch;
+};
+
+template <typename T, int W, int RPW, int S>
+cudaError_t launch_stream_variant(const CUtensorMap &m, const Params &p,
+                                  const dualmv_plan_t &pl, int dev, cudaStream_t st) {
+    return launch_stream<T, true, false, dmv::kOutBoth, false, W, RPW, S>(m, p, pl, dev, st);
+}
+
+template <int W, int RPW, int S>
+cudaError_t launch_f64e_variant(const CUtensorMap &m, const Params &p, const dualmv_plan_t &pl,
+                                int dev, cudaStream_t st) {
+    return launch_f64e<false, dmv::kOutBoth, W, RPW, S>(m, p, pl, dev, st);
+}
+
+Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind kind,
+                     const Geometry &g, LaunchFn fn) {
+    Variant v;
+    v.info.index = index;
+    v.info.kernel = kernel;
+    v.info.warps = W;
+    v.info.rows_per_warp = RPW;
+    v.info.stages = S;
+    v.info.band_cols = (int32_t)g.band_cols;
+    v.info.tile_rows = (int32_t)g.tile_rows;
+    v.info.threads = (int32_t)g.threads;
+    v.info.smem_bytes = g.smem;
+    v.kind = kind;
+    v.geo = g;
+    v.launch = fn;
+    return v;
+}
+
+template <typename T, int W, int RPW, int S>
+Variant stream_variant(int32_t index) {
+    return make_variant(index, DUALMV_KERNEL_STREAM, W, RPW, S, Kind::kTma,
+                        stream_geometry<T, W, RPW, S>(true),
+                        &launch_stream_variant<T, W, RPW, S>);
+}
+
+template <int W, int RPW, int S>
+Variant f64e_variant(int32_t index) {
+    return make_variant(index, DUALMV_KERNEL_F64E, W, RPW, S, Kind::kF64e,
+                        f64e_geometry<W, RPW, S>(), &launch_f64e_variant<W, RPW, S>);
+}
+
+// Tile shapes of the 4-byte types: entry 0 is the default (8 x 4 rows, 6
+// stages); the others each differ from one of the earlier ones in one
+// property, so the neighbourhood graph the tuner walks is connected.
+template <typename T>
+const std::vector<Variant> &stream4_table() {
+    static const std::vector<Variant> tab = {
+        stream_variant<T, 8, 4, 6>(0), stream_variant<T, 8, 4, 4>(1),
+        stream_variant<T, 8, 4, 3>(2), stream_variant<T, 8, 2, 6>(3),
+        stream_variant<T, 4, 4, 6>(4), stream_variant<T, 8, 8, 3>(5),
+        stream_variant<T, 4, 8, 6>(6), stream_variant<T, 8, 2, 12>(7),
+    };
+    return tab;
+}
+
+const std::vector<Variant> &f64_table() {
+    static const std::vector<Variant> tab = {
+        f64e_variant<kF64eWarps, kF64eRpw, kF64eStages>(0),
+        f64e_variant<kF64eWarps, kF64eRpw, 2>(1),
+        f64e_variant<6, kF64eRpw, kF64eStages>(2),
+        f64e_variant<kF64eWarps, 2, kF64eStages>(3),
+        stream_variant<double, kF64eWarps, kF64eRpw, kF64eStages>(4),  // native fp64 FMA
+    };
+    return tab;
+}
+
+const std::vector<Variant> *variant_table(int32_t dtype) {
+    switch (dtype) {
+    case DUALMV_DTYPE_F32: return &stream4_table<float>();
+    case DUALMV_DTYPE_F64: return &f64_table();
+    case DUALMV_DTYPE_I32: return &stream4_table<int32_t>();
+    }
+    return nullptr;
+}
+
+template <typename T> constexpr int32_t dtype_code();
+template <> constexpr int32_t dtype_code<float>() { return DUALMV_DTYPE_F32; }
+template <> constexpr int32_t dtype_code<double>() { return DUALMV_DTYPE_F64; }
+template <> constexpr int32_t dtype_code<int32_t>() { return DUALMV_DTYPE_I32; }
+
+// Variants differ in one property: kernel, warps, rows per warp or stages.
+bool neighbours(const dualmv_variant_t &a, const dualmv_variant_t &b) {
+    const int diff = (a.kernel != b.kernel) + (a.warps != b.warps) +
+                     (a.rows_per_warp != b.rows_per_warp) + (a.stages != b.stages);
+    return diff == 1;
+}
+
+std::atomic<int32_t> g_forced_variant[3] = {{-1}, {-1}, {-1}};
+std::mutex g_tuned_mu;
+std::map<std::tuple<int32_t, int64_t, int64_t, int64_t>, int32_t> g_tuned;
+std::atomic<int> g_tuned_count{0};
+
+int32_t tuned_lookup(int32_t dtype, int64_t M, int64_t N, int64_t lda) {
+    if (g_tuned_count.load(std::memory_order_acquire) == 0) return -1;
+    std::lock_guard<std::mutex> lk(g_tuned_mu);
+    auto it = g_tuned.find(std::make_tuple(dtype, M, N, lda));
+    return it == g_tuned.end() ? -1 : it->second;
+}
+
+// The variant a call runs: `index` if the caller (the tuner) names one, else
+// the process-wide forced one, else the tuned one for this shape.  nullptr
+// means entry 0, which the ordinary launch code covers.
+const Variant *pick_variant(int32_t dtype, int64_t M, int64_t N, int64_t lda, int32_t index) {
+    const std::vector<Variant> *tab = variant_table(dtype);
+    if (tab == nullptr) return nullptr;
+    if (index < 0) index = g_forced_variant[dtype].load(std::memory_order_relaxed);
+    if (index < 0) index = tuned_lookup(dtype, M, N, lda);
+    if (index <= 0 || index >= (int32_t)tab->size()) return nullptr;
+    return &(*tab)[index];
+}
+
 // GEMVER's rank-2 update, applied on the fly by a single-sided pass.
 struct Rank2 {
     const void *u1, *v1, *u2, *v2;
@@ -392,13 +547,14 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                   const T *p, int64_t strideP, const T *r, int64_t strideR, Out *q,
                   int64_t strideQ, Out *s, int64_t strideS, int64_t batch,
                   cudaStream_t stream, uint32_t outputs = dmv::kOutBoth,
-                  const Rank2 *rank2 = nullptr) {
+                  const Rank2 *rank2 = nullptr, int32_t variant = -1) {
     using Acc = typename dmv::Traits<T>::Acc;
     static_assert(sizeof(Acc) == sizeof(Out), "accumulator and output widths differ");
     constexpr bool kIntPath = std::is_same<T, int32_t>::value;
     if (outputs != dmv::kOutBoth && (kIntPath || batch > 1)) return DUALMV_ERR_UNSUPPORTED;
     if (rank2 != nullptr && outputs == dmv::kOutBoth) return DUALMV_ERR_UNSUPPORTED;
     const bool want_q = (outputs & dmv::kOutQ) != 0, want_s = (outputs & dmv::kOutS) != 0;
+    g_last_variant = -1;
     dualmv_status st = validate(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ,
                                 s, strideS, batch, outputs);
     if (st != DUALMV_SUCCESS || batch == 0) return st;
@@ -436,18 +592,29 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
         kind = (es == 8 && g_path != DUALMV_PATH_TMA_NATIVE_F64 && rank2 == nullptr)
                    ? Kind::kF64e
                    : Kind::kTma;
+    // A compiled variant other than the default (forced, tuned or named by
+    // the tuner) for one unbatched dual product on the TMA path.
+    const Variant *var = nullptr;
+    if (tma && !three_d && outputs == dmv::kOutBoth && rank2 == nullptr &&
+        g_path != DUALMV_PATH_TMA_NATIVE_F64)
+        var = pick_variant(dtype_code<T>(), M, N, lda, variant);
+    if (var != nullptr) kind = var->kind;
     CUtensorMap map;
     std::memset(&map, 0, sizeof map);
     if (tma) {
-        const Geometry geo = geometry(es, sizeof(Acc), kind);
+        const Geometry geo = var ? var->geo : geometry(es, sizeof(Acc), kind);
         tma = encode_a<T>(&map, A, M, N, lda, strideA, batch, (int)geo.band_cols,
                           (int)geo.box_rows, three_d);
-        if (!tma) kind = Kind::kDirect;
+        if (!tma) {
+            kind = Kind::kDirect;
+            var = nullptr;
+        }
     }
 
     dualmv_plan_t pl;
-    st = make_plan(M, N, batch, es, sizeof(Acc),
-                   (int64_t)ds->sms * (tma ? 1 : kDirectCtasPerSm), kind, &pl);
+    st = var ? make_plan_geo(M, N, batch, es, sizeof(Acc), ds->sms, var->geo, &pl)
+             : make_plan(M, N, batch, es, sizeof(Acc),
+                         (int64_t)ds->sms * (tma ? 1 : kDirectCtasPerSm), kind, &pl);
     if (st != DUALMV_SUCCESS) return st;
 
     // The int32 path accumulates into q and s atomically (exact, so still
@@ -497,7 +664,10 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     g_kernel_ev_start = g_kernel_ev_stop = nullptr;
     e = ev_start ? cudaEventRecord(ev_start, stream) : cudaSuccess;
     if (e == cudaSuccess) {
-        if (rank2 != nullptr) {
+        if (var != nullptr) {
+            e = var->launch(map, prm, pl, dev, stream);
+            if (e == cudaSuccess) g_last_variant = var->info.index;
+        } else if (rank2 != nullptr) {
             if constexpr (!kIntPath) {
                 const bool only_q = outputs == dmv::kOutQ;
                 if (kind == Kind::kTma)
@@ -526,9 +696,14 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
         } else if (kind == Kind::kF64e) {
             e = three_d ? launch_f64e<true>(map, prm, pl, dev, stream)
                         : launch_f64e<false>(map, prm, pl, dev, stream);
+            if (e == cudaSuccess && !three_d) g_last_variant = 0;
         } else if (kind == Kind::kTma) {
             e = three_d ? launch_stream<T, true, true>(map, prm, pl, dev, stream)
                         : launch_stream<T, true, false>(map, prm, pl, dev, stream);
+            // Entry 0 of the f64 table is the double-float kernel: the
+            // native fp64 default kernel is no entry of it.
+            if (e == cudaSuccess && !three_d && !std::is_same<T, double>::value)
+                g_last_variant = 0;
         } else {
             e = launch_stream<T, false, false>(map, prm, pl, dev, stream);
         }
@@ -675,6 +850,267 @@ dualmv_status gemver_run(int64_t M, int64_t N, T alpha, T beta, T *A, int64_t ld
     if (st == DUALMV_SUCCESS && (e1 != cudaSuccess || e2 != cudaSuccess))
         st = cuda_fail(e1 != cudaSuccess ? e1 : e2);
     return st;
+}
+
+// ----------------------------------------------------------------- tuner --
+//
+// The performance-feedback loop of Section 3.2 over the compiled variants:
+// candidates near the current baseline, a functional-equivalence gate
+// (Eq. 4), the trimmed mean of repeated timings as the score (Eq. 3), and
+// the fastest feasible candidate as the next baseline (Eq. 5).
+
+bool trimmed_mean_of(std::vector<double> t, int64_t k, double *out) {
+    const int64_t R = (int64_t)t.size();
+    if (k < 0 || R <= 2 * k) return false;
+    std::sort(t.begin(), t.end());
+    double sum = 0.0;
+    for (int64_t i = k; i < R - k; ++i) sum += t[i];
+    *out = sum / (double)(R - 2 * k);
+    return true;
+}
+
+// Reads and clears the device fault word after synchronising `stream`.
+cudaError_t take_fault_word(cudaStream_t stream, unsigned int *word) {
+    cudaError_t e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return e;
+    e = cudaMemcpyFromSymbol(word, dmv::g_fault_word, sizeof *word);
+    if (e != cudaSuccess || *word == 0) return e;
+    const unsigned int zero = 0;
+    return cudaMemcpyToSymbol(dmv::g_fault_word, &zero, sizeof zero);
+}
+
+template <typename T> constexpr double fe_tolerance() {
+    return std::is_same<T, float>::value ? 1e-5 : std::is_same<T, double>::value ? 1e-12 : 0.0;
+}
+
+template <typename T, typename Out>
+class Tuner {
+  public:
+    Tuner(int64_t M, int64_t N, const T *A, int64_t lda, const T *p, const T *r, Out *q, Out *s,
+          const dualmv_tune_config_t &cfg, cudaStream_t stream)
+        : M_(M), N_(N), A_(A), lda_(lda), p_(p), r_(r), q_(q), s_(s), cfg_(cfg),
+          stream_(stream) {}
+
+    ~Tuner() {
+        for (cudaEvent_t ev : events_) cudaEventDestroy(ev);
+        void *bufs[] = {q_base_, s_base_, den_q_, den_s_, fe_word_, flush_};
+        for (void *b : bufs)
+            if (b) cudaFreeAsync(b, stream_);
+        cudaStreamSynchronize(stream_);
+    }
+
+    dualmv_status setup() {
+        dualmv_status st = pool_alloc(&q_base_, M_, stream_);
+        if (st == DUALMV_SUCCESS) st = pool_alloc(&s_base_, N_, stream_);
+        if (st == DUALMV_SUCCESS) st = pool_alloc(&fe_word_, 1, stream_);
+        constexpr bool kExact = std::is_same<T, int32_t>::value;
+        if (!kExact) {
+            if (st == DUALMV_SUCCESS) st = pool_alloc(&den_q_, M_, stream_);
+            if (st == DUALMV_SUCCESS) st = pool_alloc(&den_s_, N_, stream_);
+        }
+        if (st != DUALMV_SUCCESS) return st;
+        int dev = 0, l2 = 0, sms = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return cuda_fail(e);
+        if (cfg_.flush_l2) {
+            flush_bytes_ = 2 * (int64_t)l2;
+            st = pool_alloc(&flush_, flush_bytes_, stream_);
+            if (st != DUALMV_SUCCESS) return st;
+        }
+        events_.resize(2 * (size_t)cfg_.repeats, nullptr);
+        for (cudaEvent_t &ev : events_) {
+            e = cudaEventCreate(&ev);
+            if (e != cudaSuccess) return cuda_fail(e);
+        }
+        if (!kExact) {  // magnitude sums for the equivalence bar, once
+            dmv::abs_rows_kernel<T><<<4 * sms, 256, 0, stream_>>>(A_, M_, N_, lda_, p_, den_q_);
+            const int64_t bc = (N_ + 255) / 256;
+            dmv::abs_cols_kernel<T><<<(unsigned)(bc < 65535 ? bc : 65535), 256, 0, stream_>>>(
+                A_, M_, N_, lda_, r_, den_s_);
+            e = cudaGetLastError();
+            if (e != cudaSuccess) return cuda_fail(e);
+        }
+        return DUALMV_SUCCESS;
+    }
+
+    // One call of variant `v` into q, s (or the baseline buffers).
+    dualmv_status call(int32_t v, bool into_base) {
+        Out *q = into_base ? q_base_ : q_, *s = into_base ? s_base_ : s_;
+        return run<T, Out>(M_, N_, A_, lda_, 0, p_, 0, r_, 0, q, 0, s, 0, 1, stream_,
+                           dmv::kOutBoth, nullptr, v);
+    }
+
+    // Score of Eq. 3: `repeats` timed calls, trimmed mean of their times.
+    dualmv_status score(int32_t v, double *ms) {
+        const int R = cfg_.repeats;
+        for (int i = 0; i < R; ++i) {
+            cudaError_t e = cudaSuccess;
+            if (flush_) e = cudaMemsetAsync(flush_, i & 0xff, (size_t)flush_bytes_, stream_);
+            if (e == cudaSuccess) e = cudaEventRecord(events_[2 * i], stream_);
+            if (e != cudaSuccess) return cuda_fail(e);
+            dualmv_status st = call(v, false);
+            if (st != DUALMV_SUCCESS) return st;
+            e = cudaEventRecord(events_[2 * i + 1], stream_);
+            if (e != cudaSuccess) return cuda_fail(e);
+        }
+        dualmv_status st = check_fault();
+        if (st != DUALMV_SUCCESS) return st;
+        std::vector<double> t((size_t)R);
+        for (int i = 0; i < R; ++i) {
+            float f = 0.f;
+            cudaError_t e = cudaEventElapsedTime(&f, events_[2 * i], events_[2 * i + 1]);
+            if (e != cudaSuccess) return cuda_fail(e);
+            t[(size_t)i] = f;
+        }
+        trimmed_mean_of(t, cfg_.trim, ms);
+        return DUALMV_SUCCESS;
+    }
+
+    // Eq. 4: the largest per-element error of q, s against the baseline's.
+    dualmv_status equivalence(double *err) {
+        cudaError_t e = cudaMemsetAsync(fe_word_, 0, sizeof(unsigned long long), stream_);
+        const unsigned gq = (unsigned)std::min<int64_t>((M_ + 255) / 256, 1024);
+        const unsigned gs = (unsigned)std::min<int64_t>((N_ + 255) / 256, 1024);
+        if (e == cudaSuccess) {
+            dmv::fe_max_kernel<Out><<<gq, 256, 0, stream_>>>(q_, q_base_, den_q_, M_, fe_word_);
+            dmv::fe_max_kernel<Out><<<gs, 256, 0, stream_>>>(s_, s_base_, den_s_, N_, fe_word_);
+            e = cudaGetLastError();
+        }
+        unsigned long long bits = 0;
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(&bits, fe_word_, sizeof bits, cudaMemcpyDeviceToHost, stream_);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(stream_);
+        if (e != cudaSuccess) return cuda_fail(e);
+        std::memcpy(err, &bits, sizeof bits);
+        return DUALMV_SUCCESS;
+    }
+
+    dualmv_status check_fault() {
+        unsigned int word = 0;
+        cudaError_t e = take_fault_word(stream_, &word);
+        if (e != cudaSuccess) return cuda_fail(e);
+        return word ? DUALMV_ERR_TIMEOUT : DUALMV_SUCCESS;
+    }
+
+    // A planted mistake in a candidate's outputs, for testing the gate.
+    dualmv_status plant_mistake() {
+        cudaError_t e = cudaMemsetAsync(q_, 0x7f, sizeof(Out), stream_);
+        return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
+    }
+
+  private:
+    int64_t M_, N_;
+    const T *A_;
+    int64_t lda_;
+    const T *p_, *r_;
+    Out *q_, *s_;
+    dualmv_tune_config_t cfg_;
+    cudaStream_t stream_;
+    Out *q_base_ = nullptr, *s_base_ = nullptr;
+    double *den_q_ = nullptr, *den_s_ = nullptr;
+    unsigned long long *fe_word_ = nullptr;
+    unsigned char *flush_ = nullptr;
+    int64_t flush_bytes_ = 0;
+    std::vector<cudaEvent_t> events_;
+};
+
+template <typename T, typename Out>
+dualmv_status tune_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *p, const T *r,
+                       Out *q, Out *s, const dualmv_tune_config_t *cfg,
+                       dualmv_tune_result_t *res, cudaStream_t stream) {
+    if (cfg == nullptr || res == nullptr) return DUALMV_ERR_INVALID_VALUE;
+    if (cfg->trim < 0 || cfg->repeats <= 2 * cfg->trim || cfg->max_rounds < 0 ||
+        cfg->candidates < 1 || !(cfg->min_gain >= 0.0))
+        return DUALMV_ERR_INVALID_VALUE;
+    dualmv_status st = validate(M, N, A, lda, 0, p, 0, r, 0, q, 0, s, 0, 1);
+    if (st != DUALMV_SUCCESS) return st;
+    std::memset(res, 0, sizeof *res);
+    const int64_t es = sizeof(T);
+    const bool eligible = M > 0 && N > 0 && g_path != DUALMV_PATH_DIRECT &&
+                          g_path != DUALMV_PATH_TMA_NATIVE_F64 &&
+                          reinterpret_cast<uintptr_t>(A) % 16 == 0 && (lda * es) % 16 == 0 &&
+                          M < INT32_MAX && N < INT32_MAX;
+    if (!eligible) return run<T, Out>(M, N, A, lda, 0, p, 0, r, 0, q, 0, s, 0, 1, stream);
+    if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
+
+    const int32_t dtype = dtype_code<T>();
+    const std::vector<Variant> &tab = *variant_table(dtype);
+    constexpr double tol = fe_tolerance<T>();
+    const bool plant = fault_injected("fe");
+    Tuner<T, Out> tu(M, N, A, lda, p, r, q, s, *cfg, stream);
+    st = tu.setup();
+    if (st != DUALMV_SUCCESS) return st;
+
+    // K^(0): the default variant, its outputs kept as the reference.
+    int32_t base = 0;
+    st = tu.call(base, true);
+    if (st == DUALMV_SUCCESS) st = tu.score(base, &res->baseline_ms);
+    if (st != DUALMV_SUCCESS) return st;
+    double base_ms = res->baseline_ms;
+    std::vector<bool> tried(tab.size(), false);
+    tried[0] = true;
+
+    for (int32_t d = 0; d < cfg->max_rounds; ++d) {
+        std::vector<int32_t> cands;
+        for (const Variant &v : tab)
+            if (!tried[v.info.index] && neighbours(v.info, tab[base].info) &&
+                (int32_t)cands.size() < cfg->candidates)
+                cands.push_back(v.info.index);
+        if (cands.empty()) break;
+        res->rounds = d + 1;
+        int32_t best = -1;
+        double best_ms = 0.0;
+        for (int32_t c : cands) {
+            tried[c] = true;
+            ++res->evaluated;
+            dualmv_tune_step_t *step = nullptr;
+            if (res->trace_len < DUALMV_TUNE_MAX_TRACE) {
+                step = &res->trace[res->trace_len++];
+                step->index = c;
+                step->round = d;
+            }
+            st = tu.call(c, false);
+            if (st == DUALMV_SUCCESS && plant) st = tu.plant_mistake();
+            if (st == DUALMV_SUCCESS) st = tu.check_fault();
+            double err = 0.0;
+            if (st == DUALMV_SUCCESS) st = tu.equivalence(&err);
+            if (st != DUALMV_SUCCESS) return st;
+            if (step) step->fe = err;
+            if (!(err <= tol)) {  // Eq. 4: not in the feasible set
+                ++res->rejected;
+                continue;
+            }
+            if (err > res->worst_fe) res->worst_fe = err;
+            double ms = 0.0;
+            st = tu.score(c, &ms);
+            if (st != DUALMV_SUCCESS) return st;
+            if (step) {
+                step->feasible = 1;
+                step->ms = ms;
+            }
+            if (best < 0 || ms < best_ms) {  // Eq. 5
+                best = c;
+                best_ms = ms;
+            }
+        }
+        if (best < 0 || !(best_ms < base_ms * (1.0 - cfg->min_gain))) break;
+        base = best;
+        base_ms = best_ms;
+        st = tu.call(base, true);  // the new baseline's outputs, for Eq. 4
+        if (st != DUALMV_SUCCESS) return st;
+    }
+    res->best = base;
+    res->best_ms = base_ms;
+    {
+        std::lock_guard<std::mutex> lk(g_tuned_mu);
+        g_tuned[std::make_tuple(dtype, M, N, lda)] = base;
+        g_tuned_count.store((int)g_tuned.size(), std::memory_order_release);
+    }
+    st = tu.call(base, false);  // leave the chosen variant's outputs in q, s
+    if (st != DUALMV_SUCCESS) return st;
+    return tu.check_fault();
 }
 
 // ------------------------------------------------- no-allocation variant --
@@ -925,6 +1361,67 @@ dualmv_status dualmv_plan(int64_t M, int64_t N, int64_t batch, int64_t elem_byte
                           int64_t acc_bytes, int64_t num_sms, dualmv_plan_t *out) {
     return make_plan(M, N, batch, elem_bytes, acc_bytes, num_sms,
                      elem_bytes == 8 ? Kind::kF64e : Kind::kTma, out);
+}
+
+int32_t dualmv_variant_count(int32_t dtype) {
+    const std::vector<Variant> *tab = variant_table(dtype);
+    return tab ? (int32_t)tab->size() : -1;
+}
+
+dualmv_status dualmv_variant_info(int32_t dtype, int32_t index, dualmv_variant_t *out) {
+    const std::vector<Variant> *tab = variant_table(dtype);
+    if (tab == nullptr || out == nullptr || index < 0 || index >= (int32_t)tab->size())
+        return DUALMV_ERR_INVALID_VALUE;
+    *out = (*tab)[index].info;
+    return DUALMV_SUCCESS;
+}
+
+int32_t dualmv_set_variant(int32_t dtype, int32_t index) {
+    const std::vector<Variant> *tab = variant_table(dtype);
+    if (tab == nullptr || index < -1 || index >= (int32_t)tab->size()) return -2;
+    return g_forced_variant[dtype].exchange(index);
+}
+
+int32_t dualmv_tuned_variant(int32_t dtype, int64_t M, int64_t N, int64_t lda) {
+    return tuned_lookup(dtype, M, N, lda);
+}
+
+int32_t dualmv_last_variant(void) { return g_last_variant; }
+
+void dualmv_tune_clear(void) {
+    std::lock_guard<std::mutex> lk(g_tuned_mu);
+    g_tuned.clear();
+    g_tuned_count.store(0, std::memory_order_release);
+}
+
+dualmv_status dualmv_trimmed_mean(const double *t, int64_t R, int64_t k, double *out) {
+    if (t == nullptr || out == nullptr || R < 0) return DUALMV_ERR_INVALID_VALUE;
+    std::vector<double> v(t, t + R);
+    return trimmed_mean_of(std::move(v), k, out) ? DUALMV_SUCCESS : DUALMV_ERR_INVALID_VALUE;
+}
+
+dualmv_status dualmv_tune_f32(int64_t M, int64_t N, const float *A, int64_t lda, const float *p,
+                              const float *r, float *q, float *s,
+                              const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+                              dualmv_stream_t stream) {
+    return tune_run<float, float>(M, N, A, lda, p, r, q, s, cfg, res,
+                                  reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_tune_f64(int64_t M, int64_t N, const double *A, int64_t lda,
+                              const double *p, const double *r, double *q, double *s,
+                              const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+                              dualmv_stream_t stream) {
+    return tune_run<double, double>(M, N, A, lda, p, r, q, s, cfg, res,
+                                    reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_tune_i32(int64_t M, int64_t N, const int32_t *A, int64_t lda,
+                              const int32_t *p, const int32_t *r, int64_t *q, int64_t *s,
+                              const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+                              dualmv_stream_t stream) {
+    return tune_run<int32_t, int64_t>(M, N, A, lda, p, r, q, s, cfg, res,
+                                      reinterpret_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"

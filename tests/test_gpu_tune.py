@@ -1,0 +1,160 @@
+"""Kernel variants and the variant tuner on the GPU.  Every compiled variant
+of every dtype is held to the parity bar against the oracle on shapes that
+span several tiles with ragged tails; the tuner's loop (Section 3.2) is run
+on a mid-size problem per dtype and its report, its recorded choice and its
+outputs are checked; a mistake planted in every candidate's outputs must be
+caught by the equivalence gate (Eq. 4)."""
+import numpy as np
+import pytest
+import torch
+
+import paper_2512_22147_gb300 as dm
+from paper_2512_22147_gb300 import inputs
+from parity import TOL, compare_problem, run_and_compare
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+CODE = {"f32": dm.DUALMV_DTYPE_F32, "f64": dm.DUALMV_DTYPE_F64, "i32": dm.DUALMV_DTYPE_I32}
+DIST = {"f32": "uniform", "f64": "normal", "i32": "int8"}
+
+
+def _make(dtype, M, N, lda, seed):
+    return inputs.generate(inputs.Workload("t", dtype, M, N, lda, DIST[dtype], seed), DEV)
+
+
+def _all_variants():
+    out = []
+    for tag, code in CODE.items():
+        for i in range(dm.dualmv_variant_count(code)):
+            out.append((tag, i))
+    return out
+
+
+@pytest.fixture
+def forced():
+    olds = {}
+
+    def force(tag, index):
+        olds.setdefault(tag, dm.dualmv_set_variant(CODE[tag], index))
+        dm.dualmv_set_variant(CODE[tag], index)
+
+    yield force
+    for tag in olds:
+        dm.dualmv_set_variant(CODE[tag], -1)
+
+
+@pytest.mark.parametrize("tag,index", _all_variants())
+@pytest.mark.parametrize("M,N,pad", [(1000, 3000, 0), (3001, 257, 4), (77, 1000, 8),
+                                     (4096, 256, 0), (1, 1, 0)])
+def test_every_variant_matches_oracle(tag, index, M, N, pad, forced):
+    forced(tag, index)
+    A, p, r = _make(tag, M, N, N + pad, 100 + index + M)
+    run_and_compare(A, p, r, N)
+
+
+@pytest.mark.parametrize("tag,index", _all_variants())
+def test_every_variant_is_deterministic(tag, index, forced):
+    forced(tag, index)
+    A, p, r = _make(tag, 2000, 2000, 2000, 7)
+    q1, s1 = dm.dualmv(A, p, r)
+    q2, s2 = dm.dualmv(A, p, r)
+    torch.cuda.synchronize()
+    assert torch.equal(q1, q2) and torch.equal(s1, s2)
+
+
+@pytest.mark.parametrize("tag,index", _all_variants())
+def test_forced_variant_is_the_one_launched(tag, index, forced):
+    forced(tag, index)
+    A, p, r = _make(tag, 500, 700, 700, 5)
+    dm.dualmv(A, p, r)
+    torch.cuda.synchronize()
+    assert dm.dualmv_last_variant() == index
+
+
+@pytest.mark.parametrize("tag,index", [("f32", 3), ("f32", 4), ("f64", 4)])
+def test_other_summation_order_changes_bits(tag, index, forced):
+    """A variant with another tile shape (or fp64 arithmetic) rounds
+    differently: its outputs are not bit-identical to entry 0's on random
+    data, which shows the variant really ran."""
+    A, p, r = _make(tag, 4096, 4096, 4096, 21)
+    q0, s0 = dm.dualmv(A, p, r)
+    forced(tag, index)
+    q1, s1 = dm.dualmv(A, p, r)
+    torch.cuda.synchronize()
+    assert not (torch.equal(q0, q1) and torch.equal(s0, s1))
+
+
+def _tune(tag, M, N, **kw):
+    A, p, r = _make(tag, M, N, N, 11)
+    dm.dualmv_tune_clear()
+    rep = dm.tune(A, p, r, **kw)
+    torch.cuda.synchronize()
+    return A, p, r, rep
+
+
+@pytest.mark.parametrize("tag", ["f32", "f64", "i32"])
+def test_tuner_report_and_choice(tag):
+    M, N = 4096, 8192
+    A, p, r, rep = _tune(tag, M, N, repeats=12, trim=2, max_rounds=3, candidates=4,
+                         min_gain=0.0, flush_l2=True)
+    n = dm.dualmv_variant_count(CODE[tag])
+    assert 0 <= rep["best"] < n
+    assert 1 <= rep["rounds"] <= 3
+    assert rep["evaluated"] >= 1 and rep["rejected"] == 0
+    assert rep["baseline_ms"] > 0 and 0 < rep["best_ms"] <= rep["baseline_ms"]
+    assert rep["worst_fe"] <= TOL[tag]
+    tr = rep["trace"]
+    assert len(tr) == rep["evaluated"] and all(s["feasible"] for s in tr)
+    assert all(0 < s["ms"] and s["fe"] <= TOL[tag] for s in tr)
+    assert [s["round"] for s in tr] == sorted(s["round"] for s in tr)
+    if tag != "i32":   # round 0 holds variants with another summation order
+        assert max(s["fe"] for s in tr) > 0
+    best_seen = min([rep["baseline_ms"]] + [s["ms"] for s in tr])
+    assert rep["best_ms"] == best_seen or rep["best"] == 0
+    assert dm.dualmv_tuned_variant(CODE[tag], M, N, N) == rep["best"]
+    # The tuner's outputs are the chosen variant's, and they pass parity.
+    err = compare_problem(tag, rep["q"].cpu().numpy(), rep["s"].cpu().numpy(),
+                          A.cpu().numpy(), p.cpu().numpy(), r.cpu().numpy(), N)
+    assert err <= TOL[tag]
+    # Later calls of this shape run the recorded variant: same bits.
+    q, s = dm.dualmv(A, p, r)
+    torch.cuda.synchronize()
+    assert torch.equal(q, rep["q"]) and torch.equal(s, rep["s"])
+    dm.dualmv_tune_clear()
+    assert dm.dualmv_tuned_variant(CODE[tag], M, N, N) == -1
+
+
+@pytest.mark.parametrize("tag", ["f32", "i32"])
+def test_equivalence_gate_rejects_planted_mistake(tag, monkeypatch):
+    monkeypatch.setenv("DUALMV_FAULT_INJECT", "fe")
+    A, p, r, rep = _tune(tag, 2048, 2048, repeats=7, trim=1, max_rounds=2, candidates=3,
+                         min_gain=0.0, flush_l2=False)
+    assert rep["evaluated"] >= 1
+    assert rep["rejected"] == rep["evaluated"]
+    assert all(not s["feasible"] and s["fe"] > TOL[tag] for s in rep["trace"])
+    assert rep["best"] == 0 and rep["best_ms"] == rep["baseline_ms"]
+    # The outputs left behind are the default variant's, which are correct.
+    err = compare_problem(tag, rep["q"].cpu().numpy(), rep["s"].cpu().numpy(),
+                          A.cpu().numpy(), p.cpu().numpy(), r.cpu().numpy(), 2048)
+    assert err <= TOL[tag]
+    dm.dualmv_tune_clear()
+
+
+def test_tuner_off_the_tma_path_runs_default():
+    A, p, r = _make("f32", 300, 301, 301, 3)   # 301 * 4 bytes: not a multiple of 16
+    dm.dualmv_tune_clear()
+    rep = dm.tune(A, p, r, repeats=7, trim=1)
+    torch.cuda.synchronize()
+    assert rep["evaluated"] == 0 and rep["best"] == 0
+    err = compare_problem("f32", rep["q"].cpu().numpy(), rep["s"].cpu().numpy(),
+                          A.cpu().numpy(), p.cpu().numpy(), r.cpu().numpy(), 301)
+    assert err <= TOL["f32"]
+    assert dm.dualmv_tuned_variant(dm.DUALMV_DTYPE_F32, 300, 301, 301) == -1
+
+
+def test_batched_calls_ignore_forced_variant(forced):
+    forced("f32", 5)
+    w = inputs.Workload("t", "f32", 300, 700, 700, "uniform", 9, batch=3)
+    A, p, r = inputs.generate(w, DEV)
+    run_and_compare(A, p, r, 700)

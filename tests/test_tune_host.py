@@ -1,0 +1,148 @@
+"""The variant tables and the tuner's host-side parts, on the CPU: the
+tables describe compiled kernels that fit an SM, the neighbourhood the tuner
+walks (variants differing in one property) reaches every entry, the forced
+and tuned selections round-trip, the library's trimmed mean (Eq. 3) agrees
+with the oracle's, and bad tuner arguments are rejected before any CUDA
+call."""
+import math
+import random
+
+import pytest
+
+import oracle
+import paper_2512_22147_gb300 as dm
+
+DTYPES = [dm.DUALMV_DTYPE_F32, dm.DUALMV_DTYPE_F64, dm.DUALMV_DTYPE_I32]
+SMEM_LIMIT = 227 * 1024
+FAKE = 0x10000  # never dereferenced
+
+
+def table(dtype):
+    return [dm.dualmv_variant_info(dtype, i) for i in range(dm.dualmv_variant_count(dtype))]
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_variant_tables_are_well_formed(dtype):
+    tab = table(dtype)
+    assert len(tab) >= 4
+    keys = set()
+    for i, v in enumerate(tab):
+        assert v.index == i
+        assert v.kernel in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_F64E)
+        assert v.tile_rows == v.warps * v.rows_per_warp
+        assert v.threads == (v.warps + 1) * 32
+        assert 0 < v.smem_bytes <= SMEM_LIMIT
+        assert v.rows_per_warp in (1, 2, 4, 8, 16) and v.stages >= 2
+        assert v.band_cols == 256
+        keys.add((v.kernel, v.warps, v.rows_per_warp, v.stages))
+    assert len(keys) == len(tab), "two entries describe the same kernel"
+    if dtype != dm.DUALMV_DTYPE_F64:
+        assert all(v.kernel == dm.DUALMV_KERNEL_STREAM for v in tab)
+
+
+@pytest.mark.parametrize("dtype,elem,acc", [(dm.DUALMV_DTYPE_F32, 4, 4),
+                                            (dm.DUALMV_DTYPE_F64, 8, 8),
+                                            (dm.DUALMV_DTYPE_I32, 4, 8)])
+def test_entry_zero_is_the_default_plan(dtype, elem, acc):
+    v = dm.dualmv_variant_info(dtype, 0)
+    pl = dm.dualmv_plan(4096, 4096, 1, elem, acc, 152)
+    assert (v.tile_rows, v.band_cols, v.threads) == (pl.tile_rows, pl.band_cols, pl.threads)
+    assert v.smem_bytes == pl.smem_bytes
+
+
+def _neighbours(a, b):
+    return sum((a.kernel != b.kernel, a.warps != b.warps, a.rows_per_warp != b.rows_per_warp,
+                a.stages != b.stages)) == 1
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_neighbourhood_reaches_every_variant(dtype):
+    tab = table(dtype)
+    seen, todo = {0}, [0]
+    while todo:
+        i = todo.pop()
+        for j, v in enumerate(tab):
+            if j not in seen and _neighbours(tab[i], v):
+                seen.add(j)
+                todo.append(j)
+    assert seen == set(range(len(tab)))
+
+
+def test_unknown_dtype_and_index():
+    assert dm.dualmv_variant_count(7) == -1
+    with pytest.raises(dm.DualmvError):
+        dm.dualmv_variant_info(0, dm.dualmv_variant_count(0))
+    with pytest.raises(dm.DualmvError):
+        dm.dualmv_variant_info(5, 0)
+    with pytest.raises(ValueError):
+        dm.dualmv_set_variant(0, dm.dualmv_variant_count(0))
+    with pytest.raises(ValueError):
+        dm.dualmv_set_variant(3, 0)
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_forced_variant_round_trip(dtype):
+    old = dm.dualmv_set_variant(dtype, 2)
+    try:
+        assert old == -1
+        assert dm.dualmv_set_variant(dtype, 1) == 2
+    finally:
+        assert dm.dualmv_set_variant(dtype, -1) == 1
+
+
+def test_no_tuned_variant_recorded_by_default():
+    dm.dualmv_tune_clear()
+    assert dm.dualmv_tuned_variant(dm.DUALMV_DTYPE_F32, 16384, 16384, 16384) == -1
+
+
+def test_trimmed_mean_agrees_with_oracle():
+    rng = random.Random(5)
+    for _ in range(200):
+        R = rng.randint(1, 40)
+        k = rng.randint(0, (R - 1) // 2)
+        t = [rng.lognormvariate(0, 1) for _ in range(R)]
+        got = dm.dualmv_trimmed_mean(t, k)
+        want = oracle.trimmed_mean(t, k)
+        assert math.isclose(got, want, rel_tol=1e-15, abs_tol=0.0), (R, k, got, want)
+    assert dm.dualmv_trimmed_mean(list(range(1, 31)), 3) == 15.5
+
+
+def test_trimmed_mean_rejects_small_samples():
+    for R, k in ((0, 0), (2, 1), (6, 3), (5, -1)):
+        with pytest.raises(dm.DualmvError):
+            dm.dualmv_trimmed_mean([1.0] * R, k)
+
+
+def _cfg(**kw):
+    base = dict(repeats=10, trim=2, max_rounds=3, candidates=4, min_gain=0.0, flush_l2=0)
+    base.update(kw)
+    return dm.TuneConfig(base["repeats"], base["trim"], base["max_rounds"], base["candidates"],
+                         base["min_gain"], base["flush_l2"])
+
+
+@pytest.mark.parametrize("tag", ["f32", "f64", "i32"])
+@pytest.mark.parametrize("cfg", [
+    None, _cfg(repeats=4, trim=2), _cfg(trim=-1), _cfg(max_rounds=-1), _cfg(candidates=0),
+    _cfg(min_gain=-0.1), _cfg(min_gain=float("nan")),
+])
+def test_tune_rejects_bad_configuration(tag, cfg):
+    fn = getattr(dm, f"dualmv_tune_{tag}")
+    res = dm.TuneResult()
+    assert fn(64, 64, FAKE, 64, FAKE, FAKE, FAKE, FAKE, cfg, res, None) == \
+        dm.DUALMV_ERR_INVALID_VALUE
+
+
+@pytest.mark.parametrize("tag", ["f32", "f64", "i32"])
+def test_tune_rejects_bad_problem(tag):
+    fn = getattr(dm, f"dualmv_tune_{tag}")
+    res = dm.TuneResult()
+    assert fn(64, 64, FAKE, 63, FAKE, FAKE, FAKE, FAKE, _cfg(), res, None) == \
+        dm.DUALMV_ERR_INVALID_VALUE
+    assert fn(64, 64, None, 64, FAKE, FAKE, FAKE, FAKE, _cfg(), res, None) == \
+        dm.DUALMV_ERR_INVALID_VALUE
+    assert fn(64, 64, FAKE, 64, FAKE, FAKE, FAKE, FAKE, _cfg(), None, None) == \
+        dm.DUALMV_ERR_INVALID_VALUE
+
+
+def test_last_variant_before_any_call():
+    assert dm.dualmv_last_variant() == -1

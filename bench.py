@@ -44,6 +44,7 @@ DEFAULT_WORKLOAD = "f32_16384x16384"
 FALLBACK_HBM_GBS = 6800.0
 KERNEL_SOURCES = ("paper_2512_22147_gb300/csrc/dualmv_kernels.cuh",
                   "paper_2512_22147_gb300/csrc/dualmv_f64e.cuh",
+                  "paper_2512_22147_gb300/csrc/dualmv_wide.cuh",
                   "paper_2512_22147_gb300/csrc/dualmv.cu")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 FLUSH_BYTES = 256 << 20      # written between timed calls of an L2-sized workload
@@ -140,7 +141,7 @@ def record_traffic(csv_path: str, workload: str, command: str) -> str:
         e[1] += m.get("gpu__time_duration.sum", 0.0)
         e[2] += m.get("dram__bytes_read.sum", 0.0) + m.get("dram__bytes_write.sum", 0.0)
     total = sum(e[1] for e in per.values()) or 1.0
-    stream = [k for k in per if k.startswith("dmv::dualmv_stream")]
+    stream = [k for k in per if k.startswith(("dmv::dualmv_stream", "dmv::dualmv_wide"))]
     if len(stream) != 1:
         raise ValueError(f"expected one streaming kernel in the launch list, found {stream}")
     n, _, dram = per[stream[0]]
@@ -311,6 +312,8 @@ def run_native(args):
         def call():
             dm.gemver(A[:, : w.N], u1, v1, u2, v2, wv, x, y, z, alpha=1.5, beta=1.2)
 
+    if args.variant is not None:   # force one compiled kernel variant (profiling)
+        dm.dualmv_set_variant({"f32": 0, "f64": 1, "i32": 2}[w.dtype], args.variant)
     tuned = None
     if args.tune:
         if w.op != "bicg" or w.batched:
@@ -419,6 +422,16 @@ def run_native(args):
         launches_per_call = 2 * launches_per_call + 2
     peak, peak_src = measured_peak()
     kern_avg_ms = sum(kern_ms) / len(kern_ms)
+    kernel_name = f"whole {w.op} call"
+    if w.op == "bicg":   # the streaming kernel the last call launched
+        kernel_name = "dualmv_stream_kernel"
+        vi = dm.dualmv_last_variant()
+        if vi >= 0:
+            v = dm.dualmv_variant_info({"f32": 0, "f64": 1, "i32": 2}[w.dtype], vi)
+            kernel_name = {dm.DUALMV_KERNEL_STREAM: "dualmv_stream_kernel",
+                           dm.DUALMV_KERNEL_F64E: "dualmv_stream_f64e_kernel",
+                           dm.DUALMV_KERNEL_WIDE: "dualmv_wide_i32_kernel"}[v.kernel]
+            kernel_name += f"<warps {v.warps}, rows {v.rows_per_warp}, stages {v.stages}>"
     achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9
     traffic = recorded_traffic(args.workload)
 
@@ -455,13 +468,14 @@ def run_native(args):
                    f"L2 flushed: {FLUSH_BYTES >> 20} MiB written before each call, "
                    "outside its events"),
             "parallelism": f"replicas x{world}",
+            **({"variant": args.variant} if args.variant is not None else {}),
         },
         "pct_of_peak": round(100.0 * value / (world * peak), 2),
         "trimmed_mean_ms": round(trimmed_mean(step_ms, 3) if Ki > 6 else statistics.mean(step_ms), 5),
         "median_step_ms": round(statistics.median(step_ms), 5),
         "roofline": {
             "bound": "hbm",
-            "kernel": "dualmv_stream_kernel" if w.op == "bicg" else f"whole {w.op} call",
+            "kernel": kernel_name,
             "achieved": round(achieved, 2),
             "peak": peak,
             "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
@@ -654,6 +668,8 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--variant", type=int, default=None,
+                    help="force this entry of the dtype's kernel-variant table")
     ap.add_argument("--tune", action="store_true",
                     help="run the variant tuner (Eq. 3-5) on the workload before warm-up; "
                          "the timed calls then use the variant it chose")

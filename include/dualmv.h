@@ -262,11 +262,18 @@ dualmv_status dualmv_plan(int64_t M, int64_t N, int64_t batch,
  * arithmetic (double-float on the FP32 pipes, or native fp64 FMA).  Entry 0
  * of each element type's table is the default that untuned calls use.
  * Batched calls, single-sided products (GESUMMV, ATAX, GEMVER) and the
- * plain-load path always use their default kernel. */
+ * plain-load path always use their default kernel.  Untuned calls use
+ * entry 0, except int32 problems whose base or row stride is not a multiple
+ * of 128 bytes, which use the first DUALMV_KERNEL_WIDE entry: with such
+ * rows a 256-column box row straddles a 128-byte line that the next band
+ * fetches again, and the wide tiles read W KiB of each row at once. */
 enum { DUALMV_DTYPE_F32 = 0, DUALMV_DTYPE_F64 = 1, DUALMV_DTYPE_I32 = 2 };
 enum {
     DUALMV_KERNEL_STREAM = 0, /* TMA ring, native arithmetic of the dtype  */
-    DUALMV_KERNEL_F64E = 1    /* TMA ring per warp, double-float fp64      */
+    DUALMV_KERNEL_F64E = 1,   /* TMA ring per warp, double-float fp64      */
+    DUALMV_KERNEL_WIDE = 2    /* int32: tiles of rows_per_warp rows by     */
+                              /* warps * 256 columns, one 256-column       */
+                              /* sub-band per warp                         */
 };
 typedef struct dualmv_variant_t {
     int32_t index;          /* position in its dtype's table              */
@@ -339,16 +346,17 @@ typedef struct dualmv_tune_result_t {
     int32_t rounds;      /* rounds run                                        */
     int32_t evaluated;   /* candidates run, the initial baseline excluded     */
     int32_t rejected;    /* candidates that failed functional equivalence     */
-    double baseline_ms;  /* trimmed mean of variant 0 (K^(0))                 */
+    double baseline_ms;  /* trimmed mean of K^(0)                             */
     double best_ms;      /* trimmed mean of the chosen variant                */
     double worst_fe;     /* largest FE error among accepted candidates        */
     int32_t trace_len;   /* entries of `trace` filled (min(evaluated, max))  */
-    int32_t pad_;
+    int32_t initial;     /* index of K^(0), the shape's untuned variant       */
     dualmv_tune_step_t trace[DUALMV_TUNE_MAX_TRACE];
 } dualmv_tune_result_t;
 
 /* Tunes the variant for this problem by the loop of Section 3.2:
- *   K^(0) = variant 0.  In round d, up to `candidates` variants not tried
+ *   K^(0) = the variant an untuned call of this shape uses (see above).  In
+ *   round d, up to `candidates` variants not tried
  *   before that differ from K^(d) in one property (kernel, warps, rows per
  *   warp or stages) are run once and checked for functional equivalence
  *   with K^(d) (Eq. 4); each that passes is timed `repeats` times and

@@ -24,7 +24,7 @@ _BINDING_NAMES = {
     "dualmv_f32_noalloc_scratch_bytes", "dualmv_gesummv_f32", "dualmv_gesummv_f64",
     "dualmv_atax_f32", "dualmv_atax_f64", "dualmv_gemver_f32", "dualmv_gemver_f64",
     "DUALMV_DTYPE_F32", "DUALMV_DTYPE_F64", "DUALMV_DTYPE_I32", "DUALMV_KERNEL_STREAM",
-    "DUALMV_KERNEL_F64E", "Variant", "TuneConfig", "TuneResult", "dualmv_variant_count",
+    "DUALMV_KERNEL_F64E", "DUALMV_KERNEL_WIDE", "Variant", "TuneConfig", "TuneResult", "dualmv_variant_count",
     "dualmv_variant_info", "dualmv_set_variant", "dualmv_tuned_variant", "dualmv_tune_clear",
     "dualmv_trimmed_mean", "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32",
     "dualmv_last_variant", "TuneStep",

@@ -37,6 +37,7 @@ DUALMV_DTYPE_F64 = 1
 DUALMV_DTYPE_I32 = 2
 DUALMV_KERNEL_STREAM = 0
 DUALMV_KERNEL_F64E = 1
+DUALMV_KERNEL_WIDE = 2
 
 EXPORTED = (
     "dualmv_f32", "dualmv_f64", "dualmv_i32",
@@ -94,7 +95,7 @@ class TuneResult(ctypes.Structure):
                 ("evaluated", ctypes.c_int32), ("rejected", ctypes.c_int32),
                 ("baseline_ms", ctypes.c_double), ("best_ms", ctypes.c_double),
                 ("worst_fe", ctypes.c_double), ("trace_len", ctypes.c_int32),
-                ("pad_", ctypes.c_int32), ("trace", TuneStep * TUNE_MAX_TRACE)]
+                ("initial", ctypes.c_int32), ("trace", TuneStep * TUNE_MAX_TRACE)]
 
 
 def _load() -> ctypes.CDLL:

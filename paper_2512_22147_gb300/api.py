@@ -244,7 +244,7 @@ def tune(A: torch.Tensor, p: torch.Tensor, r: torch.Tensor, q: torch.Tensor | No
     if rc != B.DUALMV_SUCCESS:
         raise B.DualmvError(rc, "dualmv_tune")
     rep = {f: getattr(res, f) for f, _ in res._fields_
-           if f not in ("trace", "trace_len", "pad_")}
+           if f not in ("trace", "trace_len")}
     rep["trace"] = [{"index": st.index, "round": st.round, "feasible": bool(st.feasible),
                      "ms": st.ms, "fe": st.fe} for st in res.trace[:res.trace_len]]
     rep["q"], rep["s"] = q, s

@@ -18,8 +18,9 @@ INCLUDE = os.path.join(ROOT, "include")
 LIB_NAME = "libdualmv.so"
 LIB_PATH = os.path.join(PKG, LIB_NAME)
 SOURCES = [os.path.join(CSRC, "dualmv.cu")]
-DEPENDS = SOURCES + [os.path.join(CSRC, "dualmv_kernels.cuh"),
-                     os.path.join(INCLUDE, "dualmv.h")]
+DEPENDS = SOURCES + [os.path.join(CSRC, n) for n in (
+    "dualmv_kernels.cuh", "dualmv_f64e.cuh", "dualmv_tune.cuh", "dualmv_wide.cuh")] + [
+    os.path.join(INCLUDE, "dualmv.h")]
 
 NVCC_FLAGS = [
     "-gencode", "arch=compute_103a,code=sm_103a",

@@ -21,6 +21,7 @@
 #include "dualmv_kernels.cuh"
 #include "dualmv_f64e.cuh"
 #include "dualmv_tune.cuh"
+#include "dualmv_wide.cuh"
 
 namespace {
 
@@ -175,6 +176,7 @@ bool encode_a(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
 struct Geometry {
     int64_t band_cols;  // columns per band (tile width)
     int64_t tile_rows;  // rows per tile (stripe height)
+    int64_t box_cols;   // columns per TMA box
     int64_t box_rows;   // rows per TMA box
     int64_t smem;
     int64_t threads;
@@ -188,6 +190,7 @@ Geometry stream_geometry(bool tma) {
     Geometry g;
     g.band_cols = kBandCols;
     g.tile_rows = W * RPW;
+    g.box_cols = kBandCols;
     g.box_rows = g.tile_rows;
     g.smem = tma ? dmv::SmemLayout<T, W, RPW, S, true>::kTotal
                  : dmv::SmemLayout<T, W, RPW, S, false>::kTotal;
@@ -200,8 +203,23 @@ Geometry f64e_geometry() {
     Geometry g;
     g.band_cols = kF64eBand;
     g.tile_rows = W * RPW;
+    g.box_cols = kF64eBand;
     g.box_rows = RPW;  // one box per consumer warp
     g.smem = dmv::F64eLayout<W, RPW, S, kF64eBand>::kTotal;
+    g.threads = (W + 1) * 32;
+    return g;
+}
+
+// Wide int32 tiles: RPW rows by W * 256 columns, one 256-column box per
+// consumer warp.
+template <int W, int RPW, int S>
+Geometry wide_geometry() {
+    Geometry g;
+    g.band_cols = (int64_t)W * kBandCols;
+    g.tile_rows = RPW;
+    g.box_cols = kBandCols;
+    g.box_rows = RPW;
+    g.smem = dmv::WideLayout<W, RPW, S>::kTotal;
     g.threads = (W + 1) * 32;
     return g;
 }
@@ -339,6 +357,33 @@ cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualm
     }
 }
 
+template <int W, int RPW, int S>
+cudaError_t launch_wide(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
+                        int dev, cudaStream_t stream) {
+    auto kern = dmv::dualmv_wide_i32_kernel<W, RPW, S>;
+    static std::atomic<uint64_t> opted_in{0};
+    const uint64_t bit = 1ull << (dev & 63);
+    if (!(opted_in.load(std::memory_order_acquire) & bit)) {
+        cudaError_t e = cudaFuncSetAttribute(
+            kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem_bytes);
+        if (e != cudaSuccess) return e;
+        opted_in.fetch_or(bit, std::memory_order_acq_rel);
+    }
+    // Programmatic dependent of the zeroing kernel launched just before.
+    cudaLaunchConfig_t cfg;
+    std::memset(&cfg, 0, sizeof cfg);
+    cfg.gridDim = dim3((unsigned)pl.grid);
+    cfg.blockDim = dim3((unsigned)pl.threads);
+    cfg.dynamicSmemBytes = (size_t)pl.smem_bytes;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, map, prm);
+}
+
 // Chunks per q output in the combine kernel: the smallest power of two
 // giving at most about 8 band partials per thread, at most 32.
 int combine_chunks(int64_t bands) {
@@ -461,17 +506,44 @@ Variant f64e_variant(int32_t index) {
                         f64e_geometry<W, RPW, S>(), &launch_f64e_variant<W, RPW, S>);
 }
 
+template <int W, int RPW, int S>
+Variant wide_variant(int32_t index) {
+    return make_variant(index, DUALMV_KERNEL_WIDE, W, RPW, S, Kind::kTma,
+                        wide_geometry<W, RPW, S>(), &launch_wide<W, RPW, S>);
+}
+
 // Tile shapes of the 4-byte types: entry 0 is the default (8 x 4 rows, 6
 // stages); the others each differ from one of the earlier ones in one
 // property, so the neighbourhood graph the tuner walks is connected.
 template <typename T>
-const std::vector<Variant> &stream4_table() {
-    static const std::vector<Variant> tab = {
+std::vector<Variant> stream4_entries() {
+    return {
         stream_variant<T, 8, 4, 6>(0), stream_variant<T, 8, 4, 4>(1),
         stream_variant<T, 8, 4, 3>(2), stream_variant<T, 8, 2, 6>(3),
         stream_variant<T, 4, 4, 6>(4), stream_variant<T, 8, 8, 3>(5),
         stream_variant<T, 4, 8, 6>(6), stream_variant<T, 8, 2, 12>(7),
     };
+}
+
+const std::vector<Variant> &f32_table() {
+    static const std::vector<Variant> tab = stream4_entries<float>();
+    return tab;
+}
+
+// int32 adds the wide tiles (dualmv_wide.cuh); entry kI32Wide is the one
+// untuned calls use when rows are not 128-byte aligned.  Its boxes are 8
+// rows by 1 KiB: with 4-row (4 KiB) boxes the TMA unit, issuing eight boxes
+// per 32 KiB tile, held the kernel near 91% of HBM however few bytes it
+// moved.
+constexpr int32_t kI32Wide = 8;
+const std::vector<Variant> &i32_table() {
+    static const std::vector<Variant> tab = [] {
+        std::vector<Variant> v = stream4_entries<int32_t>();
+        v.push_back(wide_variant<8, 8, 3>(kI32Wide));  // 8 KiB boxes
+        v.push_back(wide_variant<8, 4, 6>(kI32Wide + 1));
+        v.push_back(wide_variant<4, 8, 6>(kI32Wide + 2));
+        return v;
+    }();
     return tab;
 }
 
@@ -488,9 +560,9 @@ const std::vector<Variant> &f64_table() {
 
 const std::vector<Variant> *variant_table(int32_t dtype) {
     switch (dtype) {
-    case DUALMV_DTYPE_F32: return &stream4_table<float>();
+    case DUALMV_DTYPE_F32: return &f32_table();
     case DUALMV_DTYPE_F64: return &f64_table();
-    case DUALMV_DTYPE_I32: return &stream4_table<int32_t>();
+    case DUALMV_DTYPE_I32: return &i32_table();
     }
     return nullptr;
 }
@@ -519,14 +591,27 @@ int32_t tuned_lookup(int32_t dtype, int64_t M, int64_t N, int64_t lda) {
     return it == g_tuned.end() ? -1 : it->second;
 }
 
+// The variant an untuned call of this shape uses: entry 0, except int32
+// rows that are not 128-byte aligned, which take the wide tiles (their 1 KiB
+// box rows would otherwise straddle a line shared with the next band).
+int32_t default_variant(int32_t dtype, const void *A, int64_t lda_bytes) {
+    if (dtype == DUALMV_DTYPE_I32 &&
+        (reinterpret_cast<uintptr_t>(A) % 128 != 0 || lda_bytes % 128 != 0))
+        return kI32Wide;
+    return 0;
+}
+
 // The variant a call runs: `index` if the caller (the tuner) names one, else
-// the process-wide forced one, else the tuned one for this shape.  nullptr
-// means entry 0, which the ordinary launch code covers.
-const Variant *pick_variant(int32_t dtype, int64_t M, int64_t N, int64_t lda, int32_t index) {
+// the process-wide forced one, else the tuned one for this shape, else the
+// default for the shape.  nullptr means entry 0, which the ordinary launch
+// code covers.
+const Variant *pick_variant(int32_t dtype, int64_t M, int64_t N, const void *A, int64_t lda,
+                            int64_t es, int32_t index) {
     const std::vector<Variant> *tab = variant_table(dtype);
     if (tab == nullptr) return nullptr;
     if (index < 0) index = g_forced_variant[dtype].load(std::memory_order_relaxed);
     if (index < 0) index = tuned_lookup(dtype, M, N, lda);
+    if (index < 0) index = default_variant(dtype, A, lda * es);
     if (index <= 0 || index >= (int32_t)tab->size()) return nullptr;
     return &(*tab)[index];
 }
@@ -597,13 +682,13 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     const Variant *var = nullptr;
     if (tma && !three_d && outputs == dmv::kOutBoth && rank2 == nullptr &&
         g_path != DUALMV_PATH_TMA_NATIVE_F64)
-        var = pick_variant(dtype_code<T>(), M, N, lda, variant);
+        var = pick_variant(dtype_code<T>(), M, N, A, lda, es, variant);
     if (var != nullptr) kind = var->kind;
     CUtensorMap map;
     std::memset(&map, 0, sizeof map);
     if (tma) {
         const Geometry geo = var ? var->geo : geometry(es, sizeof(Acc), kind);
-        tma = encode_a<T>(&map, A, M, N, lda, strideA, batch, (int)geo.band_cols,
+        tma = encode_a<T>(&map, A, M, N, lda, strideA, batch, (int)geo.box_cols,
                           (int)geo.box_rows, three_d);
         if (!tma) {
             kind = Kind::kDirect;
@@ -1043,14 +1128,16 @@ dualmv_status tune_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *p
     st = tu.setup();
     if (st != DUALMV_SUCCESS) return st;
 
-    // K^(0): the default variant, its outputs kept as the reference.
-    int32_t base = 0;
+    // K^(0): the variant an untuned call of this shape uses; its outputs are
+    // the reference for Eq. 4.
+    int32_t base = default_variant(dtype, A, lda * es);
+    res->initial = base;
     st = tu.call(base, true);
     if (st == DUALMV_SUCCESS) st = tu.score(base, &res->baseline_ms);
     if (st != DUALMV_SUCCESS) return st;
     double base_ms = res->baseline_ms;
     std::vector<bool> tried(tab.size(), false);
-    tried[0] = true;
+    tried[base] = true;
 
     for (int32_t d = 0; d < cfg->max_rounds; ++d) {
         std::vector<int32_t> cands;

@@ -46,7 +46,8 @@ def forced():
 
 @pytest.mark.parametrize("tag,index", _all_variants())
 @pytest.mark.parametrize("M,N,pad", [(1000, 3000, 0), (3001, 257, 4), (77, 1000, 8),
-                                     (4096, 256, 0), (1, 1, 0)])
+                                     (4096, 256, 0), (1, 1, 0), (513, 5000, 4),
+                                     (97, 2048, 0), (130, 4100, 8)])
 def test_every_variant_matches_oracle(tag, index, M, N, pad, forced):
     forced(tag, index)
     A, p, r = _make(tag, M, N, N + pad, 100 + index + M)
@@ -83,6 +84,39 @@ def test_other_summation_order_changes_bits(tag, index, forced):
     q1, s1 = dm.dualmv(A, p, r)
     torch.cuda.synchronize()
     assert not (torch.equal(q0, q1) and torch.equal(s0, s1))
+
+
+@pytest.mark.parametrize("N,lda,expect", [(8192, 8192, 0), (8190, 8196, 8), (1000, 1004, 8),
+                                          (4096, 4128, 0)])
+def test_int32_default_follows_row_alignment(N, lda, expect):
+    """Untuned int32 calls take the wide tiles when rows are not 128-byte
+    aligned (lda * 4 not a multiple of 128), entry 0 otherwise."""
+    dm.dualmv_tune_clear()
+    A, p, r = _make("i32", 300, N, lda, 4)
+    run_and_compare(A, p, r, N)
+    assert dm.dualmv_last_variant() == expect
+
+
+def test_int32_tuner_starts_from_the_shape_default():
+    M, N, lda = 1000, 8190, 8196
+    A, p, r = _make("i32", M, N, lda, 13)
+    dm.dualmv_tune_clear()
+    rep = dm.tune(A[:, :N], p, r, repeats=7, trim=1, max_rounds=2, candidates=4,
+                  min_gain=0.0, flush_l2=False)
+    torch.cuda.synchronize()
+    assert rep["initial"] == 8
+    assert all(s["index"] != 8 for s in rep["trace"])
+    w = dm.dualmv_variant_info(dm.DUALMV_DTYPE_I32, 8)
+    twin = [i for i in range(dm.dualmv_variant_count(dm.DUALMV_DTYPE_I32))
+            if (lambda v: v.kernel == dm.DUALMV_KERNEL_STREAM and
+                (v.warps, v.rows_per_warp, v.stages) == (w.warps, w.rows_per_warp, w.stages))(
+                dm.dualmv_variant_info(dm.DUALMV_DTYPE_I32, i))]
+    assert len(twin) == 1   # the same tile numbers on the other kernel kind
+    assert any(s["index"] == twin[0] for s in rep["trace"])
+    err = compare_problem("i32", rep["q"].cpu().numpy(), rep["s"].cpu().numpy(),
+                          A.cpu().numpy(), p.cpu().numpy(), r.cpu().numpy(), N)
+    assert err == 0.0
+    dm.dualmv_tune_clear()
 
 
 def _tune(tag, M, N, **kw):

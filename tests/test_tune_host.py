@@ -28,16 +28,23 @@ def test_variant_tables_are_well_formed(dtype):
     keys = set()
     for i, v in enumerate(tab):
         assert v.index == i
-        assert v.kernel in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_F64E)
-        assert v.tile_rows == v.warps * v.rows_per_warp
+        assert v.kernel in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_F64E, dm.DUALMV_KERNEL_WIDE)
+        if v.kernel == dm.DUALMV_KERNEL_WIDE:   # one 256-column sub-band per warp
+            assert v.tile_rows == v.rows_per_warp and v.band_cols == 256 * v.warps
+        else:
+            assert v.tile_rows == v.warps * v.rows_per_warp and v.band_cols == 256
         assert v.threads == (v.warps + 1) * 32
         assert 0 < v.smem_bytes <= SMEM_LIMIT
         assert v.rows_per_warp in (1, 2, 4, 8, 16) and v.stages >= 2
-        assert v.band_cols == 256
         keys.add((v.kernel, v.warps, v.rows_per_warp, v.stages))
     assert len(keys) == len(tab), "two entries describe the same kernel"
-    if dtype != dm.DUALMV_DTYPE_F64:
-        assert all(v.kernel == dm.DUALMV_KERNEL_STREAM for v in tab)
+    kinds = {v.kernel for v in tab}
+    if dtype == dm.DUALMV_DTYPE_F32:
+        assert kinds == {dm.DUALMV_KERNEL_STREAM}
+    elif dtype == dm.DUALMV_DTYPE_I32:
+        assert kinds == {dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_WIDE}
+    else:
+        assert kinds == {dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_F64E}
 
 
 @pytest.mark.parametrize("dtype,elem,acc", [(dm.DUALMV_DTYPE_F32, 4, 4),

@@ -42,10 +42,14 @@ if ROOT not in sys.path:
 METRIC = "dualmv effective HBM GB/s (bytes of A+vectors / device time) and % of GB300 peak"
 DEFAULT_WORKLOAD = "f32_16384x16384"
 FALLBACK_HBM_GBS = 6800.0
-KERNEL_SOURCES = ("paper_2512_22147_gb300/csrc/dualmv_kernels.cuh",
-                  "paper_2512_22147_gb300/csrc/dualmv_f64e.cuh",
-                  "paper_2512_22147_gb300/csrc/dualmv_wide.cuh",
-                  "paper_2512_22147_gb300/csrc/dualmv.cu")
+_CSRC = "paper_2512_22147_gb300/csrc/"
+# Device sources of each streaming-kernel family: a traffic record stays
+# valid while these are unchanged and the live call launches the same shape.
+KERNEL_FAMILIES = {
+    "dualmv_stream_kernel": (_CSRC + "dualmv_kernels.cuh",),
+    "dualmv_stream_f64e_kernel": (_CSRC + "dualmv_kernels.cuh", _CSRC + "dualmv_f64e.cuh"),
+    "dualmv_wide_i32_kernel": (_CSRC + "dualmv_kernels.cuh", _CSRC + "dualmv_wide.cuh"),
+}
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 FLUSH_BYTES = 256 << 20      # written between timed calls of an L2-sized workload
 GRAPH_CALLS = 100            # calls captured in one CUDA graph (hot-L2 figure)
@@ -62,9 +66,24 @@ def trimmed_mean(times, k: int) -> float:
     return sum(mid) / len(mid)
 
 
-def kernel_source_hash() -> str:
+def kernel_family(name: str) -> str:
+    """'dualmv_stream_f64e_kernel' from 'dmv::dualmv_stream_f64e_kernel<8, ...>'."""
+    base = name.split("<")[0]
+    return base.split("::")[-1]
+
+
+def kernel_shape(name: str):
+    """(warps, rows per warp, stages) from an ncu kernel name, by family."""
+    args = [a.strip() for a in name.split("<", 1)[1].rstrip(">").split(",")]
+    fam = kernel_family(name)
+    if fam == "dualmv_stream_kernel":   # <T, W, RPW, STAGES, ...>
+        return tuple(int(a) for a in args[1:4])
+    return tuple(int(a) for a in args[0:3])   # f64e and wide: <W, RPW, STAGES, ...>
+
+
+def kernel_source_hash(family: str) -> str:
     h = hashlib.sha256()
-    for rel in KERNEL_SOURCES:
+    for rel in KERNEL_FAMILIES[family]:
         with open(os.path.join(ROOT, rel), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
@@ -81,16 +100,22 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def recorded_traffic(workload: str):
+def recorded_traffic(workload: str, family: str | None = None, shape=None):
     """DRAM bytes per launch of the streaming kernel from a committed ncu
-    capture, if it was taken on the current kernel source; else None."""
+    capture, if it was taken on the current source of the kernel family the
+    live call launched, with the same shape; else None."""
     try:
         with open(TRAFFIC_FILE) as f:
             rec = json.load(f)
     except (OSError, ValueError):
         return None
     ent = rec.get(workload)
-    if not ent or ent.get("kernel_source_hash") != kernel_source_hash():
+    if not ent or "kernel" not in ent:
+        return None
+    fam = kernel_family(ent["kernel"])
+    if fam not in KERNEL_FAMILIES or ent.get("kernel_source_hash") != kernel_source_hash(fam):
+        return None
+    if family is not None and (fam != family or kernel_shape(ent["kernel"]) != tuple(shape)):
         return None
     return ent.get("dram_bytes_per_launch")
 
@@ -150,7 +175,7 @@ def record_traffic(csv_path: str, workload: str, command: str) -> str:
         with open(TRAFFIC_FILE) as f:
             rec = json.load(f)
     rec[workload] = {
-        "kernel_source_hash": kernel_source_hash(),
+        "kernel_source_hash": kernel_source_hash(kernel_family(stream[0])),
         "kernel": stream[0],
         "dram_bytes_per_launch": int(round(dram / n)),
         "how": "ncu launch list of bench.py on the full workload: dram__bytes_read.sum + "
@@ -423,17 +448,19 @@ def run_native(args):
     peak, peak_src = measured_peak()
     kern_avg_ms = sum(kern_ms) / len(kern_ms)
     kernel_name = f"whole {w.op} call"
+    family, shape = None, None
     if w.op == "bicg":   # the streaming kernel the last call launched
         kernel_name = "dualmv_stream_kernel"
         vi = dm.dualmv_last_variant()
         if vi >= 0:
             v = dm.dualmv_variant_info({"f32": 0, "f64": 1, "i32": 2}[w.dtype], vi)
-            kernel_name = {dm.DUALMV_KERNEL_STREAM: "dualmv_stream_kernel",
-                           dm.DUALMV_KERNEL_F64E: "dualmv_stream_f64e_kernel",
-                           dm.DUALMV_KERNEL_WIDE: "dualmv_wide_i32_kernel"}[v.kernel]
-            kernel_name += f"<warps {v.warps}, rows {v.rows_per_warp}, stages {v.stages}>"
+            family = {dm.DUALMV_KERNEL_STREAM: "dualmv_stream_kernel",
+                      dm.DUALMV_KERNEL_F64E: "dualmv_stream_f64e_kernel",
+                      dm.DUALMV_KERNEL_WIDE: "dualmv_wide_i32_kernel"}[v.kernel]
+            shape = (v.warps, v.rows_per_warp, v.stages)
+            kernel_name = family + f"<warps {v.warps}, rows {v.rows_per_warp}, stages {v.stages}>"
     achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9
-    traffic = recorded_traffic(args.workload)
+    traffic = recorded_traffic(args.workload, family, shape) if family else None
 
     hot = hot_l2_graph(torch, call, nbytes, dev) if flush is not None else None
 

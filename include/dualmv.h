@@ -284,6 +284,12 @@ typedef struct dualmv_variant_t {
     int32_t band_cols;      /* columns per band                           */
     int32_t tile_rows;      /* warps * rows_per_warp                      */
     int32_t threads;        /* threads per CTA (consumers + producer)     */
+    int32_t native_cols;    /* DUALMV_KERNEL_F64E: of each lane's 8       */
+                            /* columns, how many sum s with native fp64   */
+                            /* FMA (0 for the other kernels)              */
+    int32_t producer_warp;  /* 1: a dedicated TMA producer warp feeds the  */
+                            /* consumers; 0: each consumer warp issues its */
+                            /* own boxes (threads = warps * 32)            */
     int64_t smem_bytes;     /* dynamic shared memory per CTA              */
 } dualmv_variant_t;
 
@@ -358,7 +364,7 @@ typedef struct dualmv_tune_result_t {
  *   K^(0) = the variant an untuned call of this shape uses (see above).  In
  *   round d, up to `candidates` variants not tried
  *   before that differ from K^(d) in one property (kernel, warps, rows per
- *   warp or stages) are run once and checked for functional equivalence
+ *   warp, stages or native columns) are run once and checked for functional equivalence
  *   with K^(d) (Eq. 4); each that passes is timed `repeats` times and
  *   scored by the trimmed mean of Eq. 3.  The fastest feasible candidate
  *   (Eq. 5) becomes K^(d+1) if it beats K^(d) by more than `min_gain`;

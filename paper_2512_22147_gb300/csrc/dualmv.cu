@@ -37,7 +37,7 @@ constexpr int kStages = 6;
 constexpr int kDirectCtasPerSm = 4;
 // fp64 on the FP32 pipes (dualmv_f64e.cuh).
 #ifndef DUALMV_F64E_WARPS
-#define DUALMV_F64E_WARPS 7
+#define DUALMV_F64E_WARPS 8
 #endif
 #ifndef DUALMV_F64E_RPW
 #define DUALMV_F64E_RPW 4
@@ -52,6 +52,11 @@ constexpr int kF64eWarps = DUALMV_F64E_WARPS;
 constexpr int kF64eRpw = DUALMV_F64E_RPW;
 constexpr int kF64eStages = DUALMV_F64E_STAGES;
 constexpr int kF64eBand = DUALMV_F64E_BAND;
+// No producer warp: each consumer warp loads its own boxes.  That frees the
+// warp slot (and registers) for an eighth consumer warp, which this
+// latency-bound kernel turns into throughput; with a producer warp as well,
+// eight consumers would have to fit in 168 registers and spill.
+constexpr bool kF64eSelf = true;
 
 // Which stream kernel a call uses.
 enum class Kind { kTma, kDirect, kF64e };
@@ -198,7 +203,7 @@ Geometry stream_geometry(bool tma) {
     return g;
 }
 
-template <int W, int RPW, int S>
+template <int W, int RPW, int S, bool kSelf = kF64eSelf>
 Geometry f64e_geometry() {
     Geometry g;
     g.band_cols = kF64eBand;
@@ -206,7 +211,7 @@ Geometry f64e_geometry() {
     g.box_cols = kF64eBand;
     g.box_rows = RPW;  // one box per consumer warp
     g.smem = dmv::F64eLayout<W, RPW, S, kF64eBand>::kTotal;
-    g.threads = (W + 1) * 32;
+    g.threads = (W + (kSelf ? 0 : 1)) * 32;
     return g;
 }
 
@@ -393,10 +398,10 @@ int combine_chunks(int64_t bands) {
 }
 
 template <bool k3d, int kOut = dmv::kOutBoth, int W = kF64eWarps, int RPW = kF64eRpw,
-          int S = kF64eStages>
+          int S = kF64eStages, int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = kF64eSelf>
 cudaError_t launch_f64e(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                         int dev, cudaStream_t stream) {
-    auto kern = dmv::dualmv_stream_f64e_kernel<W, RPW, S, kF64eBand, k3d, kOut>;
+    auto kern = dmv::dualmv_stream_f64e_kernel<W, RPW, S, kF64eBand, k3d, kOut, NC, kSelf>;
     static std::atomic<uint64_t> opted_in{0};
     const uint64_t bit = 1ull << (dev & 63);
     if (!(opted_in.load(std::memory_order_acquire) & bit)) {
@@ -469,20 +474,22 @@ cudaError_t launch_stream_variant(const CUtensorMap &m, const Params &p,
     return launch_stream<T, true, false, dmv::kOutBoth, false, W, RPW, S>(m, p, pl, dev, st);
 }
 
-template <int W, int RPW, int S>
+template <int W, int RPW, int S, int NC, bool kSelf>
 cudaError_t launch_f64e_variant(const CUtensorMap &m, const Params &p, const dualmv_plan_t &pl,
                                 int dev, cudaStream_t st) {
-    return launch_f64e<false, dmv::kOutBoth, W, RPW, S>(m, p, pl, dev, st);
+    return launch_f64e<false, dmv::kOutBoth, W, RPW, S, NC, kSelf>(m, p, pl, dev, st);
 }
 
 Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind kind,
-                     const Geometry &g, LaunchFn fn) {
+                     const Geometry &g, LaunchFn fn, int NC = 0, bool self_load = false) {
     Variant v;
     v.info.index = index;
     v.info.kernel = kernel;
     v.info.warps = W;
     v.info.rows_per_warp = RPW;
     v.info.stages = S;
+    v.info.native_cols = NC;
+    v.info.producer_warp = self_load ? 0 : 1;
     v.info.band_cols = (int32_t)g.band_cols;
     v.info.tile_rows = (int32_t)g.tile_rows;
     v.info.threads = (int32_t)g.threads;
@@ -500,10 +507,11 @@ Variant stream_variant(int32_t index) {
                         &launch_stream_variant<T, W, RPW, S>);
 }
 
-template <int W, int RPW, int S>
+template <int W, int RPW, int S, int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = kF64eSelf>
 Variant f64e_variant(int32_t index) {
     return make_variant(index, DUALMV_KERNEL_F64E, W, RPW, S, Kind::kF64e,
-                        f64e_geometry<W, RPW, S>(), &launch_f64e_variant<W, RPW, S>);
+                        f64e_geometry<W, RPW, S, kSelf>(),
+                        &launch_f64e_variant<W, RPW, S, NC, kSelf>, NC, kSelf);
 }
 
 template <int W, int RPW, int S>
@@ -547,13 +555,21 @@ const std::vector<Variant> &i32_table() {
     return tab;
 }
 
+// fp64: the double-float kernel in several shapes (entry 0: 8 self-loading
+// warps x 4 rows, 3 stages, 2 native columns), the previous layout with a
+// producer warp and 7 consumers, and native fp64 FMA.
 const std::vector<Variant> &f64_table() {
     static const std::vector<Variant> tab = {
-        f64e_variant<kF64eWarps, kF64eRpw, kF64eStages>(0),
-        f64e_variant<kF64eWarps, kF64eRpw, 2>(1),
-        f64e_variant<6, kF64eRpw, kF64eStages>(2),
-        f64e_variant<kF64eWarps, 2, kF64eStages>(3),
-        stream_variant<double, kF64eWarps, kF64eRpw, kF64eStages>(4),  // native fp64 FMA
+        f64e_variant<8, 4, 3, 2, true>(0),
+        f64e_variant<8, 4, 2, 2, true>(1),
+        f64e_variant<8, 4, 3, 0, true>(2),
+        f64e_variant<8, 4, 3, 3, true>(3),
+        f64e_variant<7, 4, 3, 2, true>(4),
+        f64e_variant<7, 4, 3, 2, false>(5),   // a producer warp feeds 7 consumers
+        f64e_variant<7, 4, 3, 0, false>(6),
+        stream_variant<double, 7, 4, 3>(7),   // native fp64 FMA
+        f64e_variant<6, 4, 3, 2, false>(8),
+        f64e_variant<7, 4, 2, 2, false>(9),
     };
     return tab;
 }
@@ -572,10 +588,12 @@ template <> constexpr int32_t dtype_code<float>() { return DUALMV_DTYPE_F32; }
 template <> constexpr int32_t dtype_code<double>() { return DUALMV_DTYPE_F64; }
 template <> constexpr int32_t dtype_code<int32_t>() { return DUALMV_DTYPE_I32; }
 
-// Variants differ in one property: kernel, warps, rows per warp or stages.
+// Variants differ in one property: kernel, warps, rows per warp, stages,
+// (double-float kernel) native columns, or the loading scheme.
 bool neighbours(const dualmv_variant_t &a, const dualmv_variant_t &b) {
     const int diff = (a.kernel != b.kernel) + (a.warps != b.warps) +
-                     (a.rows_per_warp != b.rows_per_warp) + (a.stages != b.stages);
+                     (a.rows_per_warp != b.rows_per_warp) + (a.stages != b.stages) +
+                     (a.native_cols != b.native_cols) + (a.producer_warp != b.producer_warp);
     return diff == 1;
 }
 

@@ -14,10 +14,10 @@
 //   product a*x ~ a_hi x_hi + (err(a_hi x_hi) + a_hi x_lo + a_lo x_hi); the
 //           first term and its rounding error come from FMUL and FFMA
 //           exactly; the dropped a_lo x_lo is below 2^-44 |a x|.
-//   native  two of each lane's eight columns (kNativeCols) take their
-//           column sums from native fp64 FMA instead: GB300's FP64 pipe is
-//           otherwise idle here, and this moves a quarter of the s work off
-//           the FP32 pipes at about a third of the FP64 pipe's rate.
+//   native  NC of each lane's eight columns (default 2) take their column
+//           sums from native fp64 FMA instead: GB300's FP64 pipe is
+//           otherwise idle here, and this moves NC/8 of the s work off the
+//           FP32 pipes.
 //   sum     Knuth's TwoSum on the high parts, the low parts and the TwoSum
 //           errors summed in a second float ("sloppy" double-float
 //           accumulation), in three levels: the RPW rows of a tile (or the 8
@@ -164,8 +164,11 @@ struct F64eLayout {
 //
 // W consumer warps x RPW rows per warp per tile; lane l holds columns
 // 2l, 2l+1 (+64, +128, +192) of the 256-column band (four double2 vectors).
-template <int W, int RPW, int STAGES, int BAND, bool kBatched3d, int kOut = kOutBoth>
-__global__ void __launch_bounds__((W + 1) * 32, 1)
+// kSelf: no producer warp; lane 0 of each consumer warp issues its own
+// warp's boxes, refilling a stage as soon as the warp has consumed it.
+template <int W, int RPW, int STAGES, int BAND, bool kBatched3d, int kOut = kOutBoth,
+          int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = false>
+__global__ void __launch_bounds__((W + (kSelf ? 0 : 1)) * 32, 1)
 dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
     constexpr bool kQ = (kOut & kOutQ) != 0;  // row sums q = A p
     constexpr bool kS = (kOut & kOutS) != 0;  // column sums s = A^T r
@@ -209,7 +212,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     pdl_launch_dependents();
 
     // ------------------------------------------------------ producer ----
-    if (warp == W) {
+    if (!kSelf && warp == W) {
         if (lane == 0) {
             const uint64_t pol = policy_evict_first();
             bool ok = true;
@@ -265,8 +268,10 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     const T *__restrict__ rg = static_cast<const T *>(prm.r);
     const int nthreads_c = W * 32;
 
-    // Lane columns LANE_COLS - kNativeCols .. LANE_COLS - 1 sum s in fp64.
-    constexpr int kNativeCols = DUALMV_F64E_NATIVE_COLS * LANE_COLS / 8;
+    // Lane columns LANE_COLS - kNativeCols .. LANE_COLS - 1 sum s in fp64
+    // (NC of every 8).
+    static_assert(NC >= 0 && NC <= 8, "native columns: 0..8 of every 8");
+    constexpr int kNativeCols = NC * LANE_COLS / 8;
     constexpr int kFirstNative = LANE_COLS - kNativeCols;
     double snat[kNativeCols > 0 ? kNativeCols : 1];  // fp64 segment sums of s
 #pragma unroll
@@ -300,6 +305,48 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     }
     int stage = 0;
     uint32_t phase = 0;
+
+    // Self-loading: lane 0 keeps a second cursor STAGES tiles ahead and
+    // refills each stage of this warp's ring right after the warp read it.
+    TileCursor ld{0, 0, 0, 0};
+    int64_t issued = 0;           // boxes this warp issued (lane 0)
+    int64_t waited_to = ntiles;   // first tile whose wait was abandoned
+    uint64_t pol = 0;
+    auto issue = [&](int st) {
+        const int slot_i = warp * STAGES + st;
+        const uint32_t fb = smem_u32(&full_bar[slot_i]);
+        mbar_arrive_expect_tx(fb, BOX_BYTES);
+        const uint32_t dst = smem_u32(ring + (size_t)slot_i * BOX_BYTES);
+        const int x = (int)(ld.band * BAND), y = (int)(ld.stripe * BM) + warp * RPW;
+        if constexpr (kBatched3d)
+            tma_load_3d(dst, &tmap, x, y, (int)ld.b, fb, pol);
+        else
+            tma_load_2d(dst, &tmap, x, y, fb, pol);
+        ld.advance(S, prm.bands);
+        ++issued;
+    };
+    if constexpr (kSelf) {
+        if (lane == 0) {
+            pol = policy_evict_first();
+            ld.init(t0, S, prm.bands);
+            for (int st = 0; st < STAGES && st < ntiles; ++st) issue(st);
+        }
+    }
+    // Releases the stage just read: to the producer warp, or (self-loading)
+    // by refilling it with the tile STAGES ahead.
+    auto release = [&](int slot_r, int64_t k_r) {
+        __syncwarp();
+        if constexpr (kSelf) {
+            if (lane == 0 && ok && k_r + STAGES < ntiles) {
+                // The warp's reads of this stage (generic proxy) come before
+                // the copy that overwrites it (async proxy).
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                issue((int)(slot_r - warp * STAGES));
+            }
+        } else {
+            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[slot_r]));
+        }
+    };
 
     for (int64_t k = 0; k < ntiles; ++k) {
         const int64_t g = cur.g;
@@ -337,7 +384,10 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         const bool r_bad = kS && !f64e_in_range(rmine);
 
         const int slot = warp * STAGES + stage;
-        if (ok) ok = mbar_wait_bounded(smem_u32(&full_bar[slot]), phase);
+        if (ok) {
+            ok = mbar_wait_bounded(smem_u32(&full_bar[slot]), phase);
+            if (!ok) waited_to = k;
+        }
         // This warp's RPW rows of the tile.
         const Vec *tile = reinterpret_cast<const Vec *>(ring + (size_t)slot * BOX_BYTES);
 
@@ -412,8 +462,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         }
 
         if (!need_fp64) {
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[slot]));
+            release(slot, k);
             if constexpr (kQ) warp_rows_reduce_df<RPW>(q, lane);
             if (kQ && butterfly_writer<RPW>(lane)) {
                 const int64_t row = row0 + butterfly_row<RPW>(lane);
@@ -461,8 +510,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                 }
                 qd[i] = dot;
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[slot]));
+            release(slot, k);
             if constexpr (kQ) warp_rows_reduce<RPW>(qd, lane);
             if (kQ && butterfly_writer<RPW>(lane)) {
                 const int64_t row = row0 + butterfly_row<RPW>(lane);
@@ -534,6 +582,14 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                     for (int e = 0; e < VE; ++e) segp[lane_col<T>(v, lane, e)] = 0.0;
             }
         }
+    }
+    // Self-loading after an abandoned wait: boxes this warp issued for tiles
+    // it never waited for must land before the CTA exits (bounded).
+    if constexpr (kSelf) {
+        if (lane == 0)
+            for (int64_t kk = waited_to; kk < issued; ++kk)
+                mbar_wait_bounded(smem_u32(&full_bar[warp * STAGES + (int)(kk % STAGES)]),
+                                  (uint32_t)(kk / STAGES) & 1u);
     }
 }
 

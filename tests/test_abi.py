@@ -122,8 +122,8 @@ def _ref_first(c, T, G):
 ])
 def test_plan_covers_every_tile_once(M, N, batch, eb, ab, sms):
     pl = dm.dualmv_plan(M, N, batch, eb, ab, sms)
-    # fp64: 7 warps x 4 rows of 256-column bands (FP32-pipe kernel)
-    rows, width = (32, 256) if eb == 4 else (28, 256)
+    # fp64: 8 self-loading warps x 4 rows of 256-column bands (FP32-pipe kernel)
+    rows, width = (32, 256)
     assert pl.band_cols == width and pl.tile_rows == rows
     assert pl.bands == -(-N // width) and pl.stripes == -(-M // rows)
     assert pl.tiles == batch * pl.bands * pl.stripes

@@ -51,8 +51,9 @@ def test_bytes_counted():
 
 
 def test_traffic_record_goes_stale_with_the_kernel(tmp_path, monkeypatch):
-    rec = {"wl": {"kernel_source_hash": bench.kernel_source_hash(),
-                  "dram_bytes_per_launch": 123}}
+    name = "dmv::dualmv_stream_kernel<float, 8, 4, 6, 1, 0, 3, 0>"
+    rec = {"wl": {"kernel_source_hash": bench.kernel_source_hash("dualmv_stream_kernel"),
+                  "kernel": name, "dram_bytes_per_launch": 123}}
     f = tmp_path / "traffic.json"
     f.write_text(json.dumps(rec))
     monkeypatch.setattr(bench, "TRAFFIC_FILE", str(f))
@@ -145,4 +146,10 @@ def test_launch_list_parser_and_traffic_record(tmp_path, monkeypatch):
     md = bench.record_traffic(str(csv_path), "wl", "cmd")
     assert "| `dmv::dualmv_stream_kernel<float, 8, 4, 6, 1, 0>` | 2 | 330.0 |" in md
     assert bench.recorded_traffic("wl") == int(1001e6 + 500e3)
+    assert bench.recorded_traffic("wl", "dualmv_stream_kernel", (8, 4, 6)) == int(1001e6 + 500e3)
+    assert bench.recorded_traffic("wl", "dualmv_stream_kernel", (8, 4, 4)) is None
+    assert bench.recorded_traffic("wl", "dualmv_wide_i32_kernel", (8, 4, 6)) is None
     assert bench.recorded_traffic("other") is None
+    assert bench.kernel_shape("dmv::dualmv_stream_f64e_kernel<8, 4, 3, 256, 0, 3, 2, 1>") == \
+        (8, 4, 3)
+    assert bench.kernel_shape("dmv::dualmv_wide_i32_kernel<8, 8, 3>") == (8, 8, 3)

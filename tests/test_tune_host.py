@@ -33,10 +33,16 @@ def test_variant_tables_are_well_formed(dtype):
             assert v.tile_rows == v.rows_per_warp and v.band_cols == 256 * v.warps
         else:
             assert v.tile_rows == v.warps * v.rows_per_warp and v.band_cols == 256
-        assert v.threads == (v.warps + 1) * 32
+        assert v.threads == (v.warps + v.producer_warp) * 32
+        assert v.producer_warp in (0, 1)
+        if v.kernel != dm.DUALMV_KERNEL_F64E:
+            assert v.producer_warp == 1
         assert 0 < v.smem_bytes <= SMEM_LIMIT
         assert v.rows_per_warp in (1, 2, 4, 8, 16) and v.stages >= 2
-        keys.add((v.kernel, v.warps, v.rows_per_warp, v.stages))
+        if v.kernel != dm.DUALMV_KERNEL_F64E:
+            assert v.native_cols == 0
+        keys.add((v.kernel, v.warps, v.rows_per_warp, v.stages, v.native_cols,
+                  v.producer_warp))
     assert len(keys) == len(tab), "two entries describe the same kernel"
     kinds = {v.kernel for v in tab}
     if dtype == dm.DUALMV_DTYPE_F32:
@@ -59,7 +65,8 @@ def test_entry_zero_is_the_default_plan(dtype, elem, acc):
 
 def _neighbours(a, b):
     return sum((a.kernel != b.kernel, a.warps != b.warps, a.rows_per_warp != b.rows_per_warp,
-                a.stages != b.stages)) == 1
+                a.stages != b.stages, a.native_cols != b.native_cols,
+                a.producer_warp != b.producer_warp)) == 1
 
 
 @pytest.mark.parametrize("dtype", DTYPES)

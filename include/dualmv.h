@@ -290,6 +290,10 @@ typedef struct dualmv_variant_t {
     int32_t producer_warp;  /* 1: a dedicated TMA producer warp feeds the  */
                             /* consumers; 0: each consumer warp issues its */
                             /* own boxes (threads = warps * 32)            */
+    int32_t packed;         /* DUALMV_KERNEL_F64E: 1 if the double-float   */
+                            /* arithmetic of column pairs runs as packed   */
+                            /* FP32x2 instructions                         */
+    int32_t pad_;
     int64_t smem_bytes;     /* dynamic shared memory per CTA              */
 } dualmv_variant_t;
 

@@ -72,7 +72,8 @@ class Plan(ctypes.Structure):
 class Variant(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "index", "kernel", "warps", "rows_per_warp", "stages", "band_cols", "tile_rows",
-        "threads", "native_cols", "producer_warp")] + [("smem_bytes", ctypes.c_int64)]
+        "threads", "native_cols", "producer_warp", "packed", "pad_")] + [
+        ("smem_bytes", ctypes.c_int64)]
 
 
 class TuneConfig(ctypes.Structure):

@@ -57,6 +57,11 @@ constexpr int kF64eBand = DUALMV_F64E_BAND;
 // latency-bound kernel turns into throughput; with a producer warp as well,
 // eight consumers would have to fit in 168 registers and spill.
 constexpr bool kF64eSelf = true;
+// The double-float arithmetic of each lane's column pairs runs as packed
+// FP32x2 instructions, with no native fp64 columns: the kernel is bound by
+// instruction issue, and the pairs halve the FP32 instructions.
+constexpr bool kF64ePack = true;
+constexpr int kF64eNativeCols = 0;
 
 // Which stream kernel a call uses.
 enum class Kind { kTma, kDirect, kF64e };
@@ -398,10 +403,12 @@ int combine_chunks(int64_t bands) {
 }
 
 template <bool k3d, int kOut = dmv::kOutBoth, int W = kF64eWarps, int RPW = kF64eRpw,
-          int S = kF64eStages, int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = kF64eSelf>
+          int S = kF64eStages, int NC = kF64eNativeCols, bool kSelf = kF64eSelf,
+          bool kPack = kF64ePack>
 cudaError_t launch_f64e(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                         int dev, cudaStream_t stream) {
-    auto kern = dmv::dualmv_stream_f64e_kernel<W, RPW, S, kF64eBand, k3d, kOut, NC, kSelf>;
+    auto kern =
+        dmv::dualmv_stream_f64e_kernel<W, RPW, S, kF64eBand, k3d, kOut, NC, kSelf, kPack>;
     static std::atomic<uint64_t> opted_in{0};
     const uint64_t bit = 1ull << (dev & 63);
     if (!(opted_in.load(std::memory_order_acquire) & bit)) {
@@ -474,10 +481,10 @@ cudaError_t launch_stream_variant(const CUtensorMap &m, const Params &p,
     return launch_stream<T, true, false, dmv::kOutBoth, false, W, RPW, S>(m, p, pl, dev, st);
 }
 
-template <int W, int RPW, int S, int NC, bool kSelf>
+template <int W, int RPW, int S, int NC, bool kSelf, bool kPack>
 cudaError_t launch_f64e_variant(const CUtensorMap &m, const Params &p, const dualmv_plan_t &pl,
                                 int dev, cudaStream_t st) {
-    return launch_f64e<false, dmv::kOutBoth, W, RPW, S, NC, kSelf>(m, p, pl, dev, st);
+    return launch_f64e<false, dmv::kOutBoth, W, RPW, S, NC, kSelf, kPack>(m, p, pl, dev, st);
 }
 
 Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind kind,
@@ -490,6 +497,7 @@ Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind 
     v.info.stages = S;
     v.info.native_cols = NC;
     v.info.producer_warp = self_load ? 0 : 1;
+    v.info.packed = 0;
     v.info.band_cols = (int32_t)g.band_cols;
     v.info.tile_rows = (int32_t)g.tile_rows;
     v.info.threads = (int32_t)g.threads;
@@ -507,11 +515,14 @@ Variant stream_variant(int32_t index) {
                         &launch_stream_variant<T, W, RPW, S>);
 }
 
-template <int W, int RPW, int S, int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = kF64eSelf>
+template <int W, int RPW, int S, int NC = kF64eNativeCols, bool kSelf = kF64eSelf,
+          bool kPack = kF64ePack>
 Variant f64e_variant(int32_t index) {
-    return make_variant(index, DUALMV_KERNEL_F64E, W, RPW, S, Kind::kF64e,
-                        f64e_geometry<W, RPW, S, kSelf>(),
-                        &launch_f64e_variant<W, RPW, S, NC, kSelf>, NC, kSelf);
+    Variant v = make_variant(index, DUALMV_KERNEL_F64E, W, RPW, S, Kind::kF64e,
+                             f64e_geometry<W, RPW, S, kSelf>(),
+                             &launch_f64e_variant<W, RPW, S, NC, kSelf, kPack>, NC, kSelf);
+    v.info.packed = kPack ? 1 : 0;
+    return v;
 }
 
 template <int W, int RPW, int S>
@@ -556,20 +567,22 @@ const std::vector<Variant> &i32_table() {
 }
 
 // fp64: the double-float kernel in several shapes (entry 0: 8 self-loading
-// warps x 4 rows, 3 stages, 2 native columns), the previous layout with a
-// producer warp and 7 consumers, and native fp64 FMA.
+// warps x 4 rows, 3 stages, packed pairs), the scalar forms with and without
+// native fp64 columns, the earlier layout with a producer warp and 7
+// consumers, and native fp64 FMA.
 const std::vector<Variant> &f64_table() {
     static const std::vector<Variant> tab = {
-        f64e_variant<8, 4, 3, 2, true>(0),
-        f64e_variant<8, 4, 2, 2, true>(1),
-        f64e_variant<8, 4, 3, 0, true>(2),
-        f64e_variant<8, 4, 3, 3, true>(3),
-        f64e_variant<7, 4, 3, 2, true>(4),
-        f64e_variant<7, 4, 3, 2, false>(5),   // a producer warp feeds 7 consumers
-        f64e_variant<7, 4, 3, 0, false>(6),
-        stream_variant<double, 7, 4, 3>(7),   // native fp64 FMA
-        f64e_variant<6, 4, 3, 2, false>(8),
-        f64e_variant<7, 4, 2, 2, false>(9),
+        f64e_variant<8, 4, 3, 0, true, true>(0),
+        f64e_variant<8, 4, 2, 0, true, true>(1),
+        f64e_variant<8, 4, 3, 0, true, false>(2),    // scalar FP32 instructions
+        f64e_variant<8, 4, 3, 2, true, false>(3),
+        f64e_variant<8, 4, 3, 3, true, false>(4),
+        f64e_variant<7, 4, 3, 2, true, false>(5),
+        f64e_variant<7, 4, 3, 2, false, false>(6),   // a producer warp feeds 7 consumers
+        f64e_variant<7, 4, 3, 0, false, false>(7),
+        stream_variant<double, 7, 4, 3>(8),          // native fp64 FMA
+        f64e_variant<6, 4, 3, 2, false, false>(9),
+        f64e_variant<7, 4, 2, 2, false, false>(10),
     };
     return tab;
 }
@@ -593,7 +606,8 @@ template <> constexpr int32_t dtype_code<int32_t>() { return DUALMV_DTYPE_I32; }
 bool neighbours(const dualmv_variant_t &a, const dualmv_variant_t &b) {
     const int diff = (a.kernel != b.kernel) + (a.warps != b.warps) +
                      (a.rows_per_warp != b.rows_per_warp) + (a.stages != b.stages) +
-                     (a.native_cols != b.native_cols) + (a.producer_warp != b.producer_warp);
+                     (a.native_cols != b.native_cols) + (a.producer_warp != b.producer_warp) +
+                     (a.packed != b.packed);
     return diff == 1;
 }
 

@@ -145,6 +145,55 @@ __device__ __forceinline__ void warp_rows_reduce_df(DF (&v)[RPW], int lane) {
     }
 }
 
+// ---- packed pairs --------------------------------------------------------
+// GB300 issues a packed FP32 add, multiply or FMA on two floats per lane as
+// one instruction (the FMA pipe takes two cycles for it).  This kernel is
+// bound by instruction issue, not by the FMA pipe, so the double-float
+// arithmetic of a lane's two adjacent columns runs as pairs: same
+// operations, same roundings, half the instructions.
+
+struct DF2 {
+    float2 s;  // high parts of two values
+    float2 c;  // low parts
+};
+
+__device__ __forceinline__ float2 add2(float2 a, float2 b) { return __fadd2_rn(a, b); }
+// a - b, exactly as a scalar subtraction rounds it: b * -1 is exact, the FMA
+// rounds once.
+__device__ __forceinline__ float2 sub2(float2 a, float2 b) {
+    return __ffma2_rn(b, make_float2(-1.f, -1.f), a);
+}
+
+__device__ __forceinline__ void two_sum2(float2 a, float2 b, float2 &s, float2 &e) {
+    s = add2(a, b);
+    const float2 bb = sub2(s, a);
+    e = add2(sub2(a, sub2(s, bb)), sub2(b, bb));
+}
+
+// a * x for two pairs, as df_prod.
+__device__ __forceinline__ void df_prod2(float2 ah, float2 al, float2 xh, float2 xl, float2 &p,
+                                         float2 &q) {
+    p = __fmul2_rn(ah, xh);
+    q = __ffma2_rn(ah, xh, make_float2(-p.x, -p.y));  // exact rounding errors of p
+    q = __ffma2_rn(ah, xl, q);
+    q = __ffma2_rn(al, xh, q);
+}
+
+__device__ __forceinline__ void df_acc2(DF2 &acc, float2 p, float2 q) {
+    float2 s, e;
+    two_sum2(acc.s, p, s, e);
+    acc.s = s;
+    acc.c = add2(acc.c, add2(e, q));
+}
+
+__device__ __forceinline__ DF2 df_add2(DF2 x, DF2 y) {
+    DF2 r;
+    float2 e;
+    two_sum2(x.s, y.s, r.s, e);
+    r.c = add2(add2(x.c, y.c), e);
+    return r;
+}
+
 // Dynamic shared memory of the fp64 kernel: every consumer warp has its own
 // ring of STAGES boxes (its RPW rows of a tile), so warps wait only for
 // their own rows and drift apart instead of finishing every tile together;
@@ -166,8 +215,10 @@ struct F64eLayout {
 // 2l, 2l+1 (+64, +128, +192) of the 256-column band (four double2 vectors).
 // kSelf: no producer warp; lane 0 of each consumer warp issues its own
 // warp's boxes, refilling a stage as soon as the warp has consumed it.
+// kPack: the double-float arithmetic of each lane's two adjacent columns
+// runs as packed pairs (no native columns).
 template <int W, int RPW, int STAGES, int BAND, bool kBatched3d, int kOut = kOutBoth,
-          int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = false>
+          int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = false, bool kPack = false>
 __global__ void __launch_bounds__((W + (kSelf ? 0 : 1)) * 32, 1)
 dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
     constexpr bool kQ = (kOut & kOutQ) != 0;  // row sums q = A p
@@ -271,12 +322,15 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     // Lane columns LANE_COLS - kNativeCols .. LANE_COLS - 1 sum s in fp64
     // (NC of every 8).
     static_assert(NC >= 0 && NC <= 8, "native columns: 0..8 of every 8");
+    static_assert(!kPack || (NC == 0 && VE == 2), "packed pairs: no native columns");
     constexpr int kNativeCols = NC * LANE_COLS / 8;
     constexpr int kFirstNative = LANE_COLS - kNativeCols;
     double snat[kNativeCols > 0 ? kNativeCols : 1];  // fp64 segment sums of s
 #pragma unroll
     for (int j = 0; j < kNativeCols; ++j) snat[j] = 0.0;
     float ph[LANE_COLS], pl[LANE_COLS];  // split p of this lane's columns
+    float2 ph2[VPL], pl2[VPL];           // the same, as pairs (kPack)
+    DF2 grp2[VPL];                       // group sums of s as pairs (kPack)
     bool p_bad = false;                  // some p of this lane out of range
     DF grp[LANE_COLS];                   // group sums of s (double-float)
     // Segment sums of s (fp64) live in this warp's row of the flush scratch;
@@ -287,6 +341,11 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     for (int e = 0; e < LANE_COLS; ++e) {
         ph[e] = pl[e] = 0.f;
         grp[e].s = grp[e].c = 0.f;
+    }
+#pragma unroll
+    for (int v = 0; v < VPL; ++v) {
+        ph2[v] = pl2[v] = make_float2(0.f, 0.f);
+        grp2[v].s = grp2[v].c = make_float2(0.f, 0.f);
     }
 #pragma unroll
     for (int v = 0; v < VPL; ++v)
@@ -376,6 +435,13 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                     split_f64(pv, ph[v * VE + e], pl[v * VE + e], habs);
                     p_bad |= !f64e_in_range(pv);
                 }
+            if constexpr (kPack) {
+#pragma unroll
+                for (int v = 0; v < VPL; ++v) {
+                    ph2[v] = make_float2(ph[v * VE], ph[v * VE + 1]);
+                    pl2[v] = make_float2(pl[v * VE], pl[v * VE + 1]);
+                }
+            }
         }
         // r of this warp's rows, split by its owner lane.
         float rh_mine, rl_mine;
@@ -396,10 +462,55 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
 #pragma unroll
         for (int i = 0; i < RPW; ++i) q[i].s = q[i].c = 0.f;
         DF tacc[LANE_COLS];
+        DF2 tacc2[VPL];
         double tnat[kNativeCols > 0 ? kNativeCols : 1];
 #pragma unroll
         for (int j = 0; j < kNativeCols; ++j) tnat[j] = 0.0;
         uint32_t span = 0;  // max over elements of (|a| bits - 2^-40 bits)
+        if constexpr (kPack) {
+#pragma unroll
+            for (int i = 0; i < RPW; ++i) {
+                const Vec *rowp = tile + (size_t)i * (ROW_BYTES / 16);
+                Vec a[VPL];
+#pragma unroll
+                for (int v = 0; v < VPL; ++v) a[v] = rowp[v * 32 + lane];
+                const float rh = __shfl_sync(0xffffffffu, rh_mine, i);
+                const float rl = __shfl_sync(0xffffffffu, rl_mine, i);
+                const float2 rh2 = make_float2(rh, rh), rl2 = make_float2(rl, rl);
+                DF2 qp[VPL];
+#pragma unroll
+                for (int v = 0; v < VPL; ++v) {
+                    float ah0, al0, ah1, al1;
+                    uint32_t habs0, habs1;
+                    split_f64(a[v].x, ah0, al0, habs0);
+                    split_f64(a[v].y, ah1, al1, habs1);
+                    span = max(span, max(habs0 - kF64eLoBits, habs1 - kF64eLoBits));
+                    const float2 ah = make_float2(ah0, ah1), al = make_float2(al0, al1);
+                    if constexpr (kS) {
+                        float2 p0, p1;
+                        df_prod2(ah, al, rh2, rl2, p0, p1);
+                        if (i == 0) {
+                            tacc2[v].s = p0;
+                            tacc2[v].c = p1;
+                        } else {
+                            df_acc2(tacc2[v], p0, p1);
+                        }
+                    }
+                    if constexpr (kQ) df_prod2(ah, al, ph2[v], pl2[v], qp[v].s, qp[v].c);
+                }
+                if constexpr (kQ) {
+                    // Pairwise over the lane's 8 columns: the two halves of
+                    // each pair separately, then the halves together.
+                    const DF2 h = df_add2(df_add2(qp[0], qp[1]), df_add2(qp[2], qp[3]));
+                    DF lo, hi;
+                    lo.s = h.s.x;
+                    lo.c = h.c.x;
+                    hi.s = h.s.y;
+                    hi.c = h.c.y;
+                    q[i] = df_add(lo, hi);
+                }
+            }
+        } else {
 #pragma unroll
         for (int i = 0; i < RPW; ++i) {
             const Vec *rowp = tile + (size_t)i * (ROW_BYTES / 16);
@@ -443,6 +554,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             else
                 q[i] = df_add(df_add(qp[0], qp[1]), df_add(qp[2], qp[3]));
         }
+        }
         // Anything suspicious in this warp's rows (zeros included)?
         const bool rows_r_bad = __any_sync(0xffffffffu, lane < RPW && r_bad);
         bool need_fp64 = rows_r_bad || __any_sync(0xffffffffu, kQ && p_bad);
@@ -474,10 +586,15 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                         static_cast<Acc *>(prm.q_ws)[(b * prm.bands + band) * prm.M + row] = qv;
                 }
             }
+            if constexpr (kPack) {
 #pragma unroll
-            for (int e = 0; e < kFirstNative; ++e) grp[e] = df_add(grp[e], tacc[e]);
+                for (int v = 0; v < VPL; ++v) grp2[v] = df_add2(grp2[v], tacc2[v]);
+            } else {
 #pragma unroll
-            for (int j = 0; j < kNativeCols; ++j) snat[j] += tnat[j];
+                for (int e = 0; e < kFirstNative; ++e) grp[e] = df_add(grp[e], tacc[e]);
+#pragma unroll
+                for (int j = 0; j < kNativeCols; ++j) snat[j] += tnat[j];
+            }
         } else {
             // Out-of-range values in these rows: native fp64 for them.
             double pd[LANE_COLS];
@@ -540,11 +657,20 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     #pragma unroll
                     for (int e = 0; e < VE; ++e) {
                         const int ce = v * VE + e;
-                        if (ce < kFirstNative) {
+                        if constexpr (kPack) {
+                            DF x;
+                            x.s = e == 0 ? grp2[v].s.x : grp2[v].s.y;
+                            x.c = e == 0 ? grp2[v].c.x : grp2[v].c.y;
+                            segp[lane_col<T>(v, lane, e)] += df_to_double(x);
+                        } else if (ce < kFirstNative) {
                             segp[lane_col<T>(v, lane, e)] += df_to_double(grp[ce]);
                             grp[ce].s = grp[ce].c = 0.f;
                         }
                     }
+                if constexpr (kPack) {
+    #pragma unroll
+                    for (int v = 0; v < VPL; ++v) grp2[v].s = grp2[v].c = make_float2(0.f, 0.f);
+                }
                 ngrp = 0;
             }
             if (seg_end) {

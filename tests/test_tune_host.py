@@ -41,8 +41,10 @@ def test_variant_tables_are_well_formed(dtype):
         assert v.rows_per_warp in (1, 2, 4, 8, 16) and v.stages >= 2
         if v.kernel != dm.DUALMV_KERNEL_F64E:
             assert v.native_cols == 0
+        if v.packed:
+            assert v.kernel == dm.DUALMV_KERNEL_F64E and v.native_cols == 0
         keys.add((v.kernel, v.warps, v.rows_per_warp, v.stages, v.native_cols,
-                  v.producer_warp))
+                  v.producer_warp, v.packed))
     assert len(keys) == len(tab), "two entries describe the same kernel"
     kinds = {v.kernel for v in tab}
     if dtype == dm.DUALMV_DTYPE_F32:
@@ -66,7 +68,7 @@ def test_entry_zero_is_the_default_plan(dtype, elem, acc):
 def _neighbours(a, b):
     return sum((a.kernel != b.kernel, a.warps != b.warps, a.rows_per_warp != b.rows_per_warp,
                 a.stages != b.stages, a.native_cols != b.native_cols,
-                a.producer_warp != b.producer_warp)) == 1
+                a.producer_warp != b.producer_warp, a.packed != b.packed)) == 1
 
 
 @pytest.mark.parametrize("dtype", DTYPES)

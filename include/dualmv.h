@@ -133,6 +133,16 @@ dualmv_status dualmv_atax_f32(int64_t M, int64_t N, const float *A, int64_t lda,
 dualmv_status dualmv_atax_f64(int64_t M, int64_t N, const double *A, int64_t lda,
                               const double *x, double *y, dualmv_stream_t stream);
 
+/* ATAX with one read of A: fp32 problems whose base and row stride meet the
+ * TMA rules and whose width fits a cluster of at most 16 CTAs (N <= 32768)
+ * stream A once: the CTAs of a thread-block cluster share each 8-row stripe,
+ * exchange the stripe's partial row sums through distributed shared memory
+ * and form A^T t from the copy still on chip.  Other problems, and fp64,
+ * read A twice (a rows-only pass, then a columns-only pass).
+ * dualmv_atax_set_two_pass(1) forces the two-pass path for every problem
+ * (tests, benchmarks); 0 restores the choice.  Returns the previous setting. */
+int dualmv_atax_set_two_pass(int two_pass);
+
 /* GEMVER (Table 1 / Table 2, row "GEMVER"): with A M x N (lda >= max(1, N)),
  * u1, u2, w, y of length M and v1, v2, x, z of length N:
  *     A_hat = A + u1 v1^T + u2 v2^T

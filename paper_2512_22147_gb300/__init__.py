@@ -27,7 +27,7 @@ _BINDING_NAMES = {
     "DUALMV_KERNEL_F64E", "DUALMV_KERNEL_WIDE", "Variant", "TuneConfig", "TuneResult", "dualmv_variant_count",
     "dualmv_variant_info", "dualmv_set_variant", "dualmv_tuned_variant", "dualmv_tune_clear",
     "dualmv_trimmed_mean", "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32",
-    "dualmv_last_variant", "TuneStep",
+    "dualmv_last_variant", "TuneStep", "dualmv_atax_set_two_pass",
 }
 _API_NAMES = {"dualmv", "device_fault", "gesummv", "atax", "gemver", "tune", "variants"}
 

@@ -51,6 +51,7 @@ EXPORTED = (
     "dualmv_variant_count", "dualmv_variant_info", "dualmv_set_variant",
     "dualmv_tuned_variant", "dualmv_tune_clear", "dualmv_trimmed_mean",
     "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32", "dualmv_last_variant",
+    "dualmv_atax_set_two_pass",
 )
 
 
@@ -136,6 +137,8 @@ def _load() -> ctypes.CDLL:
     lib.dualmv_device_fault.restype = st
     lib.dualmv_set_path.argtypes = [st]
     lib.dualmv_set_path.restype = st
+    lib.dualmv_atax_set_two_pass.argtypes = [st]
+    lib.dualmv_atax_set_two_pass.restype = st
     lib.dualmv_record_kernel_events.argtypes = [vp, vp]
     lib.dualmv_record_kernel_events.restype = None
     lib.dualmv_plan.argtypes = [i64, i64, i64, i64, i64, i64, ctypes.POINTER(Plan)]
@@ -244,6 +247,11 @@ def dualmv_last_cuda_error() -> int:
 
 def dualmv_device_fault(stream=None) -> int:
     return _lib.dualmv_device_fault(stream)
+
+
+def dualmv_atax_set_two_pass(two_pass: int) -> int:
+    """1: ATAX always reads A twice; 0: single-read cluster path where it fits."""
+    return _lib.dualmv_atax_set_two_pass(two_pass)
 
 
 def dualmv_set_path(path: int) -> int:

@@ -22,6 +22,7 @@
 #include "dualmv_f64e.cuh"
 #include "dualmv_tune.cuh"
 #include "dualmv_wide.cuh"
+#include "dualmv_atax.cuh"
 
 namespace {
 
@@ -71,6 +72,7 @@ thread_local cudaEvent_t g_kernel_ev_start = nullptr;
 thread_local cudaEvent_t g_kernel_ev_stop = nullptr;
 thread_local int32_t g_last_variant = -1;
 int g_path = DUALMV_PATH_AUTO;
+int g_atax_two_pass = 0;  // 1: ATAX always takes the two-pass path
 
 dualmv_status cuda_fail(cudaError_t e) {
     g_last_cuda_error = static_cast<int>(e);
@@ -889,8 +891,110 @@ dualmv_status gesummv_run(int64_t M, int64_t N, T alpha, const T *A, int64_t lda
     return st;
 }
 
-// ATAX (Table 1): tmp = A x, y = A^T tmp: a rows-only pass, then a
-// columns-only pass over the same A.
+// ATAX with one read of A (dualmv_atax.cuh): fp32, clusters of C CTAs of
+// kAtaxWarps warps, each warp a 256-column sub-band of kAtaxRows-row
+// stripes.  Returns with *used = false, having enqueued nothing, when the
+// problem does not fit the cluster path (alignment, width, no cluster of
+// that size can be placed), so that the caller takes the two-pass path.
+#ifndef DUALMV_ATAX_ROWS
+#define DUALMV_ATAX_ROWS 8
+#endif
+#ifndef DUALMV_ATAX_STAGES
+#define DUALMV_ATAX_STAGES 3
+#endif
+constexpr int kAtaxWarps = 8, kAtaxRows = DUALMV_ATAX_ROWS, kAtaxStages = DUALMV_ATAX_STAGES;
+
+struct AtaxClusterCache {
+    std::mutex mu;
+    int max_clusters[kMaxDevices][dmv::kAtaxMaxCluster + 1] = {};
+    bool known[kMaxDevices][dmv::kAtaxMaxCluster + 1] = {};
+};
+AtaxClusterCache g_atax_cache;
+
+dualmv_status atax_cluster_run(int64_t M, int64_t N, const float *A, int64_t lda,
+                               const float *x, float *y, cudaStream_t stream, bool *used) {
+    *used = false;
+    using L = dmv::AtaxLayout<kAtaxWarps, kAtaxRows, kAtaxStages>;
+    const int64_t bands = (N + kBandCols - 1) / kBandCols;
+    const int64_t C = (bands + kAtaxWarps - 1) / kAtaxWarps;
+    if (g_path == DUALMV_PATH_DIRECT || C > dmv::kAtaxMaxCluster ||
+        reinterpret_cast<uintptr_t>(A) % 16 != 0 || (lda * 4) % 16 != 0 || M >= INT32_MAX ||
+        N >= INT32_MAX)
+        return DUALMV_SUCCESS;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (dev < 0 || dev >= kMaxDevices) return DUALMV_SUCCESS;
+    auto kern = dmv::atax_cluster_kernel<kAtaxWarps, kAtaxRows, kAtaxStages>;
+    cudaLaunchConfig_t cfg;
+    std::memset(&cfg, 0, sizeof cfg);
+    cfg.blockDim = dim3(kAtaxWarps * 32);
+    cfg.dynamicSmemBytes = (size_t)L::kTotal;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int max_clusters = 0;
+    {
+        std::lock_guard<std::mutex> lk(g_atax_cache.mu);
+        if (!g_atax_cache.known[dev][C]) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)L::kTotal);
+            if (e == cudaSuccess && C > 8)
+                e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+            if (e == cudaSuccess) {
+                cfg.gridDim = dim3((unsigned)C);
+                e = cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg);
+            }
+            if (e != cudaSuccess) {  // no such cluster here: use two passes
+                (void)cudaGetLastError();
+                max_clusters = 0;
+            }
+            g_atax_cache.max_clusters[dev][C] = max_clusters;
+            g_atax_cache.known[dev][C] = true;
+        }
+        max_clusters = g_atax_cache.max_clusters[dev][C];
+    }
+    if (max_clusters <= 0) return DUALMV_SUCCESS;
+    CUtensorMap map;
+    std::memset(&map, 0, sizeof map);
+    if (!encode_a<float>(&map, A, M, N, lda, M * lda, 1, kBandCols, kAtaxRows, false))
+        return DUALMV_SUCCESS;
+    const int64_t stripes = (M + kAtaxRows - 1) / kAtaxRows;
+    const int64_t clusters = stripes < max_clusters ? stripes : max_clusters;
+    float *ws = nullptr;
+    dualmv_status st = pool_alloc(&ws, clusters * N, stream);
+    if (st != DUALMV_SUCCESS) return st;
+    *used = true;
+    dmv::AtaxParams prm;
+    prm.x = x;
+    prm.y_ws = ws;
+    prm.M = M;
+    prm.N = N;
+    prm.stripes = stripes;
+    prm.clusters = clusters;
+    prm.bands = bands;
+    cfg.gridDim = dim3((unsigned)(clusters * C));
+    e = cudaLaunchKernelEx(&cfg, kern, map, prm);
+    if (e == cudaSuccess) {
+        int64_t blocks = (N + 255) / 256;
+        if (blocks > 4096) blocks = 4096;
+        dmv::atax_sum_kernel<<<(unsigned)blocks, 256, 0, stream>>>(ws, y, N, clusters);
+        e = cudaGetLastError();
+    }
+    cudaError_t ef = cudaFreeAsync(ws, stream);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (ef != cudaSuccess) return cuda_fail(ef);
+    return DUALMV_SUCCESS;
+}
+
+// ATAX (Table 1): y = A^T (A x).  fp32 takes the single-read cluster path
+// when it fits; otherwise (and for fp64) tmp = A x by a rows-only pass and
+// y = A^T tmp by a columns-only pass over the same A.
 template <typename T>
 dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x, T *y,
                        cudaStream_t stream) {
@@ -903,6 +1007,13 @@ dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x
         return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
     }
     if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
+    if constexpr (std::is_same<T, float>::value) {
+        if (g_atax_two_pass == 0) {
+            bool used = false;
+            dualmv_status sc = atax_cluster_run(M, N, A, lda, x, y, stream, &used);
+            if (sc != DUALMV_SUCCESS || used) return sc;
+        }
+    }
     T *tmp = nullptr;
     dualmv_status st = pool_alloc(&tmp, M, stream);
     if (st != DUALMV_SUCCESS) return st;
@@ -1465,6 +1576,12 @@ dualmv_status dualmv_device_fault(dualmv_stream_t stream) {
 void dualmv_record_kernel_events(void *start, void *stop) {
     g_kernel_ev_start = static_cast<cudaEvent_t>(start);
     g_kernel_ev_stop = static_cast<cudaEvent_t>(stop);
+}
+
+int dualmv_atax_set_two_pass(int two_pass) {
+    const int old = g_atax_two_pass;
+    g_atax_two_pass = two_pass ? 1 : 0;
+    return old;
 }
 
 int dualmv_set_path(int path) {

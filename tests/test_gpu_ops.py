@@ -27,6 +27,13 @@ def path(request):
     dm.dualmv_set_path(old)
 
 
+@pytest.fixture(params=[0, 1], ids=["one_read", "two_pass"])
+def atax_mode(request):
+    old = dm.dualmv_atax_set_two_pass(request.param)
+    yield request.param
+    dm.dualmv_atax_set_two_pass(old)
+
+
 def _w(op, dtype, M, N, lda, seed):
     dist = "uniform" if dtype == "f32" else "normal"
     return inputs.Workload(op, dtype, M, N, lda, dist, seed, op=op)
@@ -67,10 +74,45 @@ def test_gesummv_matches_oracle(dtype, M, N, pad, path):
 
 @pytest.mark.parametrize("dtype", ["f32", "f64"])
 @pytest.mark.parametrize("M,N,pad", [(1000, 3000, 0), (3001, 257, 5), (1, 1, 0), (77, 1000, 3),
-                                     (2048, 64, 0)])
-def test_atax_matches_oracle(dtype, M, N, pad, path):
+                                     (2048, 64, 0), (513, 5000, 4), (1030, 2048, 0)])
+def test_atax_matches_oracle(dtype, M, N, pad, path, atax_mode):
     A, x = inputs.generate_atax(_w("atax", dtype, M, N, N + pad, 3 * M + N), DEV)
     check_atax(A, x, N, dtype)
+
+
+# fp32 widths for the single-read path: clusters of 1, 2, 3, 8 and 10 CTAs
+# (8 sub-bands of 256 columns per CTA), and one too wide for a cluster of 16
+# (two passes).
+@pytest.mark.parametrize("M,N", [(4096, 16384), (300, 20000), (1000, 700), (1999, 4100),
+                                 (33, 6144), (256, 40000), (9, 16384)])
+def test_atax_one_read_widths(M, N, atax_mode):
+    A, x = inputs.generate_atax(_w("atax", "f32", M, N, N, 7 * M + N), DEV)
+    check_atax(A, x, N, "f32")
+
+
+def test_atax_one_read_path_runs():
+    """The single-read path adds the row sums in another order than the
+    two-pass path, so on random data their bits differ: the cluster kernel
+    really ran.  Both are checked against the oracle elsewhere."""
+    A, x = inputs.generate_atax(_w("atax", "f32", 4096, 4096, 4096, 5), DEV)
+    old = dm.dualmv_atax_set_two_pass(0)
+    try:
+        y1 = dm.atax(A, x)
+        dm.dualmv_atax_set_two_pass(1)
+        y2 = dm.atax(A, x)
+        torch.cuda.synchronize()
+    finally:
+        dm.dualmv_atax_set_two_pass(old)
+    assert not torch.equal(y1, y2)
+    assert dm.device_fault() == dm.DUALMV_SUCCESS
+
+
+def test_atax_one_read_is_deterministic():
+    A, x = inputs.generate_atax(_w("atax", "f32", 3000, 9000, 9000, 6), DEV)
+    y1 = dm.atax(A, x)
+    y2 = dm.atax(A, x)
+    torch.cuda.synchronize()
+    assert torch.equal(y1, y2)
 
 
 def check_gemver(ops, N, alpha, beta, update_A, dtype):
@@ -144,7 +186,7 @@ def test_gesummv_closed_forms(dtype, path):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "f64"])
-def test_atax_permutation_is_exact(dtype):
+def test_atax_permutation_is_exact(dtype, atax_mode):
     n = 900
     g = torch.Generator(device="cpu").manual_seed(9)
     perm = torch.randperm(n, generator=g)

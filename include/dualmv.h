@@ -161,6 +161,16 @@ dualmv_status dualmv_gemver_f64(int64_t M, int64_t N, double alpha, double beta,
                                 const double *u2, const double *v2, double *w, double *x,
                                 const double *y, const double *z, dualmv_stream_t stream);
 
+/* How GEMVER applies the rank-2 update when A is not to be overwritten
+ * (update_A == 0).  By default it uses the factorisation
+ * A_hat^T y = A^T y + v1 (u1 . y) + v2 (u2 . y) and
+ * A_hat x = A x + u1 (v1 . x) + u2 (v2 . x): a columns-only and a rows-only
+ * pass of the plain kernels plus four dot products (compensated, fixed
+ * order), with no per-element update.  dualmv_gemver_set_onthefly(1) makes
+ * it form A_hat element by element as it streams A, as it always does with
+ * update_A (tests, benchmarks).  Returns the previous setting. */
+int dualmv_gemver_set_onthefly(int onthefly);
+
 /* ---- single problem without allocation --------------------------------
  * The paper has no counterpart to this entry point; it exists for callers
  * that cannot allocate device memory during the call: code inside a

@@ -28,6 +28,7 @@ _BINDING_NAMES = {
     "dualmv_variant_info", "dualmv_set_variant", "dualmv_tuned_variant", "dualmv_tune_clear",
     "dualmv_trimmed_mean", "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32",
     "dualmv_last_variant", "TuneStep", "dualmv_atax_set_two_pass",
+    "dualmv_gemver_set_onthefly",
 }
 _API_NAMES = {"dualmv", "device_fault", "gesummv", "atax", "gemver", "tune", "variants"}
 

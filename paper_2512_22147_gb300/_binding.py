@@ -51,7 +51,7 @@ EXPORTED = (
     "dualmv_variant_count", "dualmv_variant_info", "dualmv_set_variant",
     "dualmv_tuned_variant", "dualmv_tune_clear", "dualmv_trimmed_mean",
     "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32", "dualmv_last_variant",
-    "dualmv_atax_set_two_pass",
+    "dualmv_atax_set_two_pass", "dualmv_gemver_set_onthefly",
 )
 
 
@@ -139,6 +139,8 @@ def _load() -> ctypes.CDLL:
     lib.dualmv_set_path.restype = st
     lib.dualmv_atax_set_two_pass.argtypes = [st]
     lib.dualmv_atax_set_two_pass.restype = st
+    lib.dualmv_gemver_set_onthefly.argtypes = [st]
+    lib.dualmv_gemver_set_onthefly.restype = st
     lib.dualmv_record_kernel_events.argtypes = [vp, vp]
     lib.dualmv_record_kernel_events.restype = None
     lib.dualmv_plan.argtypes = [i64, i64, i64, i64, i64, i64, ctypes.POINTER(Plan)]
@@ -252,6 +254,11 @@ def dualmv_device_fault(stream=None) -> int:
 def dualmv_atax_set_two_pass(two_pass: int) -> int:
     """1: ATAX always reads A twice; 0: single-read cluster path where it fits."""
     return _lib.dualmv_atax_set_two_pass(two_pass)
+
+
+def dualmv_gemver_set_onthefly(onthefly: int) -> int:
+    """1: GEMVER forms A_hat element by element even without update_A."""
+    return _lib.dualmv_gemver_set_onthefly(onthefly)
 
 
 def dualmv_set_path(path: int) -> int:

@@ -73,6 +73,7 @@ thread_local cudaEvent_t g_kernel_ev_stop = nullptr;
 thread_local int32_t g_last_variant = -1;
 int g_path = DUALMV_PATH_AUTO;
 int g_atax_two_pass = 0;  // 1: ATAX always takes the two-pass path
+int g_gemver_onthefly = 0;  // 1: GEMVER applies the update element by element
 
 dualmv_status cuda_fail(cudaError_t e) {
     g_last_cuda_error = static_cast<int>(e);
@@ -1027,11 +1028,66 @@ dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x
     return st;
 }
 
+// GEMVER without writing A_hat: the rank-2 update factorises,
+//   A_hat^T y = A^T y + v1 (u1 . y) + v2 (u2 . y),
+//   A_hat x   = A x   + u1 (v1 . x) + u2 (v2 . x),
+// so a columns-only and a rows-only pass of the plain kernels (double-float
+// for fp64) and four dot products give x and w without any per-element
+// update.  Each term's error stays within the bar of A_hat's magnitudes.
+template <typename T>
+dualmv_status gemver_factored(int64_t M, int64_t N, T alpha, T beta, const T *A, int64_t lda,
+                              const T *u1, const T *v1, const T *u2, const T *v2, T *w, T *x,
+                              const T *y, const T *z, cudaStream_t stream) {
+    T *s = nullptr, *t = nullptr;
+    double *part = nullptr;  // [2 products][kDotChunks][sum, error], one side at a time
+    dualmv_status st = pool_alloc(&s, N, stream);
+    if (st == DUALMV_SUCCESS) st = pool_alloc(&t, M, stream);
+    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * dmv::kDotChunks, stream);
+    cudaError_t e = cudaSuccess;
+    if (st == DUALMV_SUCCESS && N > 0) {  // s = A^T y (zero when M == 0)
+        dmv::dots2_partial_kernel<T><<<2 * dmv::kDotChunks, 256, 0, stream>>>(u1, u2, y, M,
+                                                                               part);
+        e = cudaGetLastError();
+        if (e == cudaSuccess)
+            st = run<T, T>(M, N, A, lda, 0, nullptr, 0, y, 0, nullptr, 0, s, 0, 1, stream,
+                           dmv::kOutS);
+        if (e == cudaSuccess && st == DUALMV_SUCCESS) {
+            const int64_t bx = (N + 255) / 256;
+            dmv::gemver_x2_kernel<T><<<(unsigned)(bx > 4096 ? 4096 : bx), 256, 0, stream>>>(
+                x, s, v1, v2, part, z, N, beta);
+            e = cudaGetLastError();
+        }
+    }
+    if (st == DUALMV_SUCCESS && e == cudaSuccess && M > 0) {  // t = A x (zero when N == 0)
+        dmv::dots2_partial_kernel<T><<<2 * dmv::kDotChunks, 256, 0, stream>>>(v1, v2, x, N,
+                                                                               part);
+        e = cudaGetLastError();
+        if (e == cudaSuccess)
+            st = run<T, T>(M, N, A, lda, 0, x, 0, nullptr, 0, t, 0, nullptr, 0, 1, stream,
+                           dmv::kOutQ);
+        if (e == cudaSuccess && st == DUALMV_SUCCESS) {
+            const int64_t bw = (M + 255) / 256;
+            dmv::gemver_w2_kernel<T><<<(unsigned)(bw > 4096 ? 4096 : bw), 256, 0, stream>>>(
+                w, t, u1, u2, part, M, alpha);
+            e = cudaGetLastError();
+        }
+    }
+    if (st == DUALMV_SUCCESS && e != cudaSuccess) st = cuda_fail(e);
+    void *bufs[3] = {s, t, part};
+    for (void *bp : bufs) {
+        if (bp == nullptr) continue;
+        cudaError_t ef = cudaFreeAsync(bp, stream);
+        if (st == DUALMV_SUCCESS && ef != cudaSuccess) st = cuda_fail(ef);
+    }
+    return st;
+}
+
 // GEMVER (Table 1 / Table 2): A_hat = A + u1 v1^T + u2 v2^T;
-// x = x + beta A_hat^T y + z;  w = w + alpha A_hat x.  Two passes apply the
-// rank-2 update as they stream A: a columns-only pass (A_hat^T y) and, after
-// the x update, a rows-only pass (A_hat x) that also writes A_hat over A
-// when update_A is set.  A is read twice and written at most once.
+// x = x + beta A_hat^T y + z;  w = w + alpha A_hat x.  Without update_A the
+// factorised form above runs.  With it, two passes apply the rank-2 update
+// as they stream A: a columns-only pass (A_hat^T y) and, after the x
+// update, a rows-only pass (A_hat x) that also writes A_hat over A.  A is
+// read twice and written once.
 template <typename T>
 dualmv_status gemver_run(int64_t M, int64_t N, T alpha, T beta, T *A, int64_t lda,
                          int update_A, const T *u1, const T *v1, const T *u2, const T *v2,
@@ -1044,6 +1100,9 @@ dualmv_status gemver_run(int64_t M, int64_t N, T alpha, T beta, T *A, int64_t ld
     if (M > 0 && N > 0 && A == nullptr) return DUALMV_ERR_INVALID_VALUE;
     if (M == 0 && N == 0) return DUALMV_SUCCESS;
     if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
+    if (!update_A && g_gemver_onthefly == 0)
+        return gemver_factored<T>(M, N, alpha, beta, A, lda, u1, v1, u2, v2, w, x, y, z,
+                                  stream);
     T *s = nullptr, *t = nullptr;
     dualmv_status st = pool_alloc(&s, N, stream);
     if (st != DUALMV_SUCCESS) return st;
@@ -1576,6 +1635,12 @@ dualmv_status dualmv_device_fault(dualmv_stream_t stream) {
 void dualmv_record_kernel_events(void *start, void *stop) {
     g_kernel_ev_start = static_cast<cudaEvent_t>(start);
     g_kernel_ev_stop = static_cast<cudaEvent_t>(stop);
+}
+
+int dualmv_gemver_set_onthefly(int onthefly) {
+    const int old = g_gemver_onthefly;
+    g_gemver_onthefly = onthefly ? 1 : 0;
+    return old;
 }
 
 int dualmv_atax_set_two_pass(int two_pass) {

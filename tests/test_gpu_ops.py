@@ -144,10 +144,18 @@ def check_gemver(ops, N, alpha, beta, update_A, dtype):
     return err
 
 
+@pytest.fixture(params=[0, 1], ids=["factored", "onthefly"])
+def gemver_mode(request):
+    old = dm.dualmv_gemver_set_onthefly(request.param)
+    yield request.param
+    dm.dualmv_gemver_set_onthefly(old)
+
+
 @pytest.mark.parametrize("dtype", ["f32", "f64"])
-@pytest.mark.parametrize("M,N,pad", [(1000, 3000, 0), (3001, 257, 5), (1, 1, 0), (77, 1000, 3)])
+@pytest.mark.parametrize("M,N,pad", [(1000, 3000, 0), (3001, 257, 5), (1, 1, 0), (77, 1000, 3),
+                                     (1, 5000, 0), (5000, 1, 0)])
 @pytest.mark.parametrize("update_A", [False, True])
-def test_gemver_matches_oracle(dtype, M, N, pad, update_A, path):
+def test_gemver_matches_oracle(dtype, M, N, pad, update_A, path, gemver_mode):
     w = _w("gemver", dtype, M, N, N + pad, 5 * M + N)
     check_gemver(inputs.generate_gemver(w, DEV), N, 1.5, -0.75, update_A, dtype)
 

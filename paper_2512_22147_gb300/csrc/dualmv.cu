@@ -23,6 +23,7 @@
 #include "dualmv_tune.cuh"
 #include "dualmv_wide.cuh"
 #include "dualmv_atax.cuh"
+#include "dualmv_ops.cuh"
 
 namespace {
 

@@ -470,9 +470,24 @@ def run_native(args):
     if not args.no_e2e and w.op == "bicg":
         e2e = run_e2e(torch, dm, w, A, p, r, dev, stream, args.e2e_steps)
 
+    # Bitwise determinism: two more calls, compared bit for bit.
+    deterministic = None
+    if w.op == "bicg":
+        call()
+        q1, s1 = q.clone(), s.clone()
+        call()
+        torch.cuda.synchronize(dev)
+        deterministic = bool(torch.equal(q1, q) and torch.equal(s1, s))
+    elif w.op in ("gesummv", "atax"):
+        call()
+        y1 = y.clone()
+        call()
+        torch.cuda.synchronize(dev)
+        deterministic = bool(torch.equal(y1, y))
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline and w.op == "bicg":
-        cpu = cpu_baseline(w, A, p, r, args.cpu_seconds)
+        cpu = cpu_baseline(w, A, p, r, args.cpu_seconds, q, s)
 
     out = {
         "metric": METRIC,
@@ -516,6 +531,7 @@ def run_native(args):
         "cpu_baseline": cpu,
         "e2e": e2e,
         "gpu_launches": launches_per_call * K,
+        "deterministic": deterministic,
         "instrumented_steps": Ki,
         "clocks": clocks,
     }
@@ -605,7 +621,7 @@ def oracle_sample(w, A_np, p_np, r_np, budget_s: float):
     """Times the oracle on leading rows of the workload (of each problem,
     batched: leading problems), growing the sample until it takes about
     ``budget_s`` seconds or covers the whole workload.  Returns
-    (bytes per second, seconds, description)."""
+    (bytes per second, seconds, description, n, oracle outputs)."""
     import oracle
     from paper_2512_22147_gb300 import inputs
 
@@ -618,10 +634,10 @@ def oracle_sample(w, A_np, p_np, r_np, budget_s: float):
     while True:
         t0 = time.perf_counter()
         if w.batched:
-            oracle.dualmv_batched(A_np[:n], p_np[:n], r_np[:n], N=w.N)
+            outs = oracle.dualmv_batched(A_np[:n], p_np[:n], r_np[:n], N=w.N)
             nbytes = n * (w.M * w.N * e + (w.M + w.N) * (e + o))
         else:
-            oracle.dualmv(A_np[:n], p_np, r_np[:n], N=w.N)
+            outs = oracle.dualmv(A_np[:n], p_np, r_np[:n], N=w.N)
             nbytes = n * w.N * e + (n + w.N) * (e + o)
         dt = time.perf_counter() - t0
         if dt >= budget_s or n >= units:
@@ -630,15 +646,61 @@ def oracle_sample(w, A_np, p_np, r_np, budget_s: float):
         n = min(units, int(math.ceil(n * grow)))
     what = (f"first {n} of {units} {'problems' if w.batched else 'rows'} of {w.name}, "
             f"single-threaded C oracle (double/Dot2/int64 sums)")
-    return nbytes / dt / 1e9, dt, what
+    return nbytes / dt / 1e9, dt, what, n, outs
 
 
-def cpu_baseline(w, A, p, r, budget_s):
+PARITY_TOL = {"f32": 1e-5, "f64": 1e-12, "i32": 0.0}
+
+
+def sample_parity(w, A_np, p_np, r_np, n, outs, q_gpu, s_gpu):
+    """Scaled error of the benchmark's own GPU outputs against the oracle's
+    outputs on the sampled part: q of the sampled rows (problems), and s too
+    when the sample is the whole workload.  Integer outputs must be equal."""
+    import numpy as np
+    import oracle
+
+    q_o, s_o = outs
+    whole = n >= (w.batch if w.batched else w.M)
+    qg = q_gpu[:n]
+    sg = s_gpu[:n] if w.batched else s_gpu
+    if w.dtype == "i32":
+        ok_q = np.array_equal(qg, q_o)
+        ok_s = (not whole) or np.array_equal(sg, s_o)
+        err = 0.0 if (ok_q and ok_s) else float("inf")
+    else:
+        def scaled(got, want, den):
+            diff = np.abs(got.astype(np.float64) - want)
+            z = den == 0
+            if z.any() and (diff[z] != 0).any():
+                return float("inf")
+            return float((diff[~z] / den[~z]).max()) if (~z).any() else 0.0
+        if w.batched:
+            errs = []
+            for b in range(n):
+                qa, sa = oracle.absdot(A_np[b], p_np[b], r_np[b], N=w.N)
+                errs += [scaled(qg[b], q_o[b], qa), scaled(sg[b], s_o[b], sa)]
+            err = max(errs)
+        else:
+            qa, sa = oracle.absdot(A_np[:n], p_np, r_np[:n], N=w.N)
+            err = scaled(qg, q_o, qa)
+            if whole:
+                err = max(err, scaled(sg, s_o, sa))
+    checked = (f"q and s of the first {n} problems" if w.batched else
+               ("q and s, every element" if whole else f"q of the first {n} rows"))
+    return {"max_scaled_error": err, "tolerance": PARITY_TOL[w.dtype],
+            "checked": checked, "pass": bool(err <= PARITY_TOL[w.dtype])}
+
+
+def cpu_baseline(w, A, p, r, budget_s, q=None, s=None):
     A_np = A.cpu().numpy()
     p_np, r_np = p.cpu().numpy(), r.cpu().numpy()
-    gbs, dt, what = oracle_sample(w, A_np, p_np, r_np, budget_s)
-    return {"value": round(gbs, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
-            "sample": what, "seconds": round(dt, 3), "host_cpus": os.cpu_count()}
+    gbs, dt, what, n, outs = oracle_sample(w, A_np, p_np, r_np, budget_s)
+    out = {"value": round(gbs, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+           "sample": what, "seconds": round(dt, 3), "host_cpus": os.cpu_count()}
+    if q is not None:
+        out["parity"] = sample_parity(w, A_np, p_np, r_np, n, outs, q.cpu().numpy(),
+                                      s.cpu().numpy())
+    return out
 
 
 def run_reference(args):
@@ -656,7 +718,7 @@ def run_reference(args):
     vals, secs = [], []
     what = ""
     for i in range(args.warmup + args.steps):
-        gbs, dt, what = oracle_sample(w, A_np, p_np, r_np, budget)
+        gbs, dt, what, _, _ = oracle_sample(w, A_np, p_np, r_np, budget)
         if i >= args.warmup:
             vals.append(gbs)
             secs.append(dt)

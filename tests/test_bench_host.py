@@ -153,3 +153,27 @@ def test_launch_list_parser_and_traffic_record(tmp_path, monkeypatch):
     assert bench.kernel_shape("dmv::dualmv_stream_f64e_kernel<8, 4, 3, 256, 0, 3, 2, 1>") == \
         (8, 4, 3)
     assert bench.kernel_shape("dmv::dualmv_wide_i32_kernel<8, 8, 3>") == (8, 8, 3)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64", "i32"])
+def test_sample_parity_accepts_oracle_and_rejects_a_perturbation(dtype):
+    """The bench's parity block: the oracle's own outputs pass; one output
+    moved by far more than the bar fails."""
+    import oracle
+    from paper_2512_22147_gb300 import inputs
+    w = inputs.Workload("t", dtype, 40, 70, 72, {"f32": "uniform", "f64": "normal",
+                                                 "i32": "int8"}[dtype], 3)
+    A, p, r = inputs.generate(w)
+    A_np, p_np, r_np = A.numpy(), p.numpy(), r.numpy()
+    q_o, s_o = oracle.dualmv(A_np, p_np, r_np, N=w.N)
+    cast = {"f32": np.float32, "f64": np.float64, "i32": np.int64}[dtype]
+    qg, sg = q_o.astype(cast), s_o.astype(cast)
+    ok = bench.sample_parity(w, A_np, p_np, r_np, w.M, (q_o, s_o), qg, sg)
+    assert ok["pass"] and ok["checked"] == "q and s, every element"
+    part = bench.sample_parity(w, A_np, p_np, r_np, 10, oracle.dualmv(A_np[:10], p_np,
+                                                                        r_np[:10], N=w.N),
+                               qg, sg)
+    assert part["pass"] and part["checked"] == "q of the first 10 rows"
+    bad = sg.copy()
+    bad[5] = bad[5] + (7 if dtype == "i32" else 1.0)
+    assert not bench.sample_parity(w, A_np, p_np, r_np, w.M, (q_o, s_o), qg, bad)["pass"]

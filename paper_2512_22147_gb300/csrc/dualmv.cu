@@ -212,14 +212,14 @@ Geometry stream_geometry(bool tma) {
     return g;
 }
 
-template <int W, int RPW, int S, bool kSelf = kF64eSelf>
+template <int W, int RPW, int S, bool kSelf = kF64eSelf, int BAND = kF64eBand>
 Geometry f64e_geometry() {
     Geometry g;
-    g.band_cols = kF64eBand;
+    g.band_cols = BAND;
     g.tile_rows = W * RPW;
-    g.box_cols = kF64eBand;
+    g.box_cols = BAND;
     g.box_rows = RPW;  // one box per consumer warp
-    g.smem = dmv::F64eLayout<W, RPW, S, kF64eBand>::kTotal;
+    g.smem = dmv::F64eLayout<W, RPW, S, BAND>::kTotal;
     g.threads = (W + (kSelf ? 0 : 1)) * 32;
     return g;
 }
@@ -408,11 +408,10 @@ int combine_chunks(int64_t bands) {
 
 template <bool k3d, int kOut = dmv::kOutBoth, int W = kF64eWarps, int RPW = kF64eRpw,
           int S = kF64eStages, int NC = kF64eNativeCols, bool kSelf = kF64eSelf,
-          bool kPack = kF64ePack>
+          bool kPack = kF64ePack, int BAND = kF64eBand>
 cudaError_t launch_f64e(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                         int dev, cudaStream_t stream) {
-    auto kern =
-        dmv::dualmv_stream_f64e_kernel<W, RPW, S, kF64eBand, k3d, kOut, NC, kSelf, kPack>;
+    auto kern = dmv::dualmv_stream_f64e_kernel<W, RPW, S, BAND, k3d, kOut, NC, kSelf, kPack>;
     static std::atomic<uint64_t> opted_in{0};
     const uint64_t bit = 1ull << (dev & 63);
     if (!(opted_in.load(std::memory_order_acquire) & bit)) {
@@ -485,10 +484,11 @@ cudaError_t launch_stream_variant(const CUtensorMap &m, const Params &p,
     return launch_stream<T, true, false, dmv::kOutBoth, false, W, RPW, S>(m, p, pl, dev, st);
 }
 
-template <int W, int RPW, int S, int NC, bool kSelf, bool kPack>
+template <int W, int RPW, int S, int NC, bool kSelf, bool kPack, int BAND>
 cudaError_t launch_f64e_variant(const CUtensorMap &m, const Params &p, const dualmv_plan_t &pl,
                                 int dev, cudaStream_t st) {
-    return launch_f64e<false, dmv::kOutBoth, W, RPW, S, NC, kSelf, kPack>(m, p, pl, dev, st);
+    return launch_f64e<false, dmv::kOutBoth, W, RPW, S, NC, kSelf, kPack, BAND>(m, p, pl, dev,
+                                                                               st);
 }
 
 Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind kind,
@@ -520,11 +520,11 @@ Variant stream_variant(int32_t index) {
 }
 
 template <int W, int RPW, int S, int NC = kF64eNativeCols, bool kSelf = kF64eSelf,
-          bool kPack = kF64ePack>
+          bool kPack = kF64ePack, int BAND = kF64eBand>
 Variant f64e_variant(int32_t index) {
     Variant v = make_variant(index, DUALMV_KERNEL_F64E, W, RPW, S, Kind::kF64e,
-                             f64e_geometry<W, RPW, S, kSelf>(),
-                             &launch_f64e_variant<W, RPW, S, NC, kSelf, kPack>, NC, kSelf);
+                             f64e_geometry<W, RPW, S, kSelf, BAND>(),
+                             &launch_f64e_variant<W, RPW, S, NC, kSelf, kPack, BAND>, NC, kSelf);
     v.info.packed = kPack ? 1 : 0;
     return v;
 }
@@ -587,6 +587,12 @@ const std::vector<Variant> &f64_table() {
         stream_variant<double, 7, 4, 3>(8),          // native fp64 FMA
         f64e_variant<6, 4, 3, 2, false, false>(9),
         f64e_variant<7, 4, 2, 2, false, false>(10),
+        // 128-column bands: 4 columns per lane, so 12 warps (3 per SM
+        // sub-partition) fit in 168 registers.
+        f64e_variant<8, 4, 3, 0, true, true, 128>(11),
+        f64e_variant<12, 4, 3, 0, true, true, 128>(12),
+        f64e_variant<12, 4, 2, 0, true, true, 128>(13),
+        f64e_variant<8, 8, 3, 0, true, true, 128>(14),
     };
     return tab;
 }
@@ -606,12 +612,15 @@ template <> constexpr int32_t dtype_code<double>() { return DUALMV_DTYPE_F64; }
 template <> constexpr int32_t dtype_code<int32_t>() { return DUALMV_DTYPE_I32; }
 
 // Variants differ in one property: kernel, warps, rows per warp, stages,
-// (double-float kernel) native columns, or the loading scheme.
+// band width, or (double-float kernel) native columns, loading scheme or
+// packing.
 bool neighbours(const dualmv_variant_t &a, const dualmv_variant_t &b) {
     const int diff = (a.kernel != b.kernel) + (a.warps != b.warps) +
                      (a.rows_per_warp != b.rows_per_warp) + (a.stages != b.stages) +
                      (a.native_cols != b.native_cols) + (a.producer_warp != b.producer_warp) +
-                     (a.packed != b.packed);
+                     (a.packed != b.packed) +
+                     // the wide kernel's band width follows from its kind
+                     (a.kernel == b.kernel && a.band_cols != b.band_cols);
     return diff == 1;
 }
 

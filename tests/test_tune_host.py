@@ -31,6 +31,8 @@ def test_variant_tables_are_well_formed(dtype):
         assert v.kernel in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_F64E, dm.DUALMV_KERNEL_WIDE)
         if v.kernel == dm.DUALMV_KERNEL_WIDE:   # one 256-column sub-band per warp
             assert v.tile_rows == v.rows_per_warp and v.band_cols == 256 * v.warps
+        elif v.kernel == dm.DUALMV_KERNEL_F64E:
+            assert v.tile_rows == v.warps * v.rows_per_warp and v.band_cols in (128, 256)
         else:
             assert v.tile_rows == v.warps * v.rows_per_warp and v.band_cols == 256
         assert v.threads == (v.warps + v.producer_warp) * 32
@@ -44,7 +46,7 @@ def test_variant_tables_are_well_formed(dtype):
         if v.packed:
             assert v.kernel == dm.DUALMV_KERNEL_F64E and v.native_cols == 0
         keys.add((v.kernel, v.warps, v.rows_per_warp, v.stages, v.native_cols,
-                  v.producer_warp, v.packed))
+                  v.producer_warp, v.packed, v.band_cols))
     assert len(keys) == len(tab), "two entries describe the same kernel"
     kinds = {v.kernel for v in tab}
     if dtype == dm.DUALMV_DTYPE_F32:
@@ -68,7 +70,8 @@ def test_entry_zero_is_the_default_plan(dtype, elem, acc):
 def _neighbours(a, b):
     return sum((a.kernel != b.kernel, a.warps != b.warps, a.rows_per_warp != b.rows_per_warp,
                 a.stages != b.stages, a.native_cols != b.native_cols,
-                a.producer_warp != b.producer_warp, a.packed != b.packed)) == 1
+                a.producer_warp != b.producer_warp, a.packed != b.packed,
+                a.kernel == b.kernel and a.band_cols != b.band_cols)) == 1
 
 
 @pytest.mark.parametrize("dtype", DTYPES)

@@ -344,9 +344,14 @@ struct SmemLayout {
 // Template: element type T, W consumer warps, RPW rows per warp per tile,
 // STAGES ring depth, kTma = TMA producer (else plain loads), kBatched3d =
 // 3-D tensor map (batch as the outer coordinate).
+// The plain-load path keeps its loads in registers and hides their latency
+// with warps.  Its int32 form (64-bit sums) would otherwise take 168
+// registers and one CTA per SM; it asks for two (128 registers), as the
+// float forms get by themselves.
 template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d,
           int kOut = kOutBoth, bool kRank2 = false>
-__global__ void __launch_bounds__((W + (kTma ? 1 : 0)) * 32, 1)
+__global__ void __launch_bounds__((W + (kTma ? 1 : 0)) * 32,
+                                  (!kTma && std::is_same<T, int32_t>::value) ? 2 : 1)
 dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
     using Acc = typename Traits<T>::Acc;
     static_assert(!kRank2 || !std::is_same<T, int32_t>::value, "rank-2 update: floats only");

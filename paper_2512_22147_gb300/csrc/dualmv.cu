@@ -336,66 +336,61 @@ bool fault_injected_alloc() { return fault_injected("alloc"); }
 
 // ------------------------------------------------------------- launching --
 
-template <typename T, bool kTma, bool k3d, int kOut = dmv::kOutBoth, bool kRank2 = false,
-          int W = kWarps, int RPW = default_rpw<T>(), int S = kStages>
-cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
-                          int dev, cudaStream_t stream) {
-    auto kern = dmv::dualmv_stream_kernel<T, W, RPW, S, kTma, k3d, kOut, kRank2>;
-    // The shared-memory opt-in is per device and per kernel; set it once.
-    static std::atomic<uint64_t> opted_in{0};
+// Raises kernel K's dynamic shared-memory limit to `bytes` the first time K
+// is launched on device `dev` (the attribute is per device and per kernel).
+template <auto K>
+cudaError_t smem_opt_in(int64_t bytes, int dev) {
+    static std::atomic<uint64_t> done{0};
     const uint64_t bit = 1ull << (dev & 63);
-    if (!(opted_in.load(std::memory_order_acquire) & bit)) {
-        cudaError_t e = cudaFuncSetAttribute(
-            kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem_bytes);
-        if (e != cudaSuccess) return e;
-        opted_in.fetch_or(bit, std::memory_order_acq_rel);
-    }
-    if constexpr (std::is_same<T, int32_t>::value) {
-        // Programmatic dependent of the zeroing kernel launched just before.
-        cudaLaunchConfig_t cfg;
-        std::memset(&cfg, 0, sizeof cfg);
-        cfg.gridDim = dim3((unsigned)pl.grid);
-        cfg.blockDim = dim3((unsigned)pl.threads);
-        cfg.dynamicSmemBytes = (size_t)pl.smem_bytes;
-        cfg.stream = stream;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr[0].val.programmaticStreamSerializationAllowed = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        return cudaLaunchKernelEx(&cfg, kern, map, prm);
-    } else {
-        kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(map,
-                                                                                       prm);
-        return cudaGetLastError();
-    }
+    if (done.load(std::memory_order_acquire) & bit) return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(K, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)bytes);
+    if (e == cudaSuccess) done.fetch_or(bit, std::memory_order_acq_rel);
+    return e;
 }
 
-template <int W, int RPW, int S>
-cudaError_t launch_wide(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
-                        int dev, cudaStream_t stream) {
-    auto kern = dmv::dualmv_wide_i32_kernel<W, RPW, S>;
-    static std::atomic<uint64_t> opted_in{0};
-    const uint64_t bit = 1ull << (dev & 63);
-    if (!(opted_in.load(std::memory_order_acquire) & bit)) {
-        cudaError_t e = cudaFuncSetAttribute(
-            kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem_bytes);
-        if (e != cudaSuccess) return e;
-        opted_in.fetch_or(bit, std::memory_order_acq_rel);
-    }
-    // Programmatic dependent of the zeroing kernel launched just before.
+// Launches `kern` as a programmatic dependent of the kernel enqueued just
+// before it on `stream`: it may start early and waits (griddepcontrol.wait)
+// before using that kernel's results.
+template <typename Kern, typename... Args>
+cudaError_t launch_dependent(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                             Args... args) {
     cudaLaunchConfig_t cfg;
     std::memset(&cfg, 0, sizeof cfg);
-    cfg.gridDim = dim3((unsigned)pl.grid);
-    cfg.blockDim = dim3((unsigned)pl.threads);
-    cfg.dynamicSmemBytes = (size_t)pl.smem_bytes;
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, map, prm);
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
+template <typename T, bool kTma, bool k3d, int kOut = dmv::kOutBoth, bool kRank2 = false,
+          int W = kWarps, int RPW = default_rpw<T>(), int S = kStages>
+cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
+                          int dev, cudaStream_t stream) {
+    constexpr auto kern = dmv::dualmv_stream_kernel<T, W, RPW, S, kTma, k3d, kOut, kRank2>;
+    cudaError_t e = smem_opt_in<kern>(pl.smem_bytes, dev);
+    if (e != cudaSuccess) return e;
+    if constexpr (std::is_same<T, int32_t>::value)  // after the zeroing kernel
+        return launch_dependent(kern, dim3((unsigned)pl.grid), dim3((unsigned)pl.threads),
+                                (size_t)pl.smem_bytes, stream, map, prm);
+    kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(map, prm);
+    return cudaGetLastError();
+}
+
+template <int W, int RPW, int S>
+cudaError_t launch_wide(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
+                        int dev, cudaStream_t stream) {
+    constexpr auto kern = dmv::dualmv_wide_i32_kernel<W, RPW, S>;
+    cudaError_t e = smem_opt_in<kern>(pl.smem_bytes, dev);
+    if (e != cudaSuccess) return e;
+    return launch_dependent(kern, dim3((unsigned)pl.grid), dim3((unsigned)pl.threads),
+                            (size_t)pl.smem_bytes, stream, map, prm);  // after the zeroing
 }
 
 // Chunks per q output in the combine kernel: the smallest power of two
@@ -411,15 +406,10 @@ template <bool k3d, int kOut = dmv::kOutBoth, int W = kF64eWarps, int RPW = kF64
           bool kPack = kF64ePack, int BAND = kF64eBand>
 cudaError_t launch_f64e(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                         int dev, cudaStream_t stream) {
-    auto kern = dmv::dualmv_stream_f64e_kernel<W, RPW, S, BAND, k3d, kOut, NC, kSelf, kPack>;
-    static std::atomic<uint64_t> opted_in{0};
-    const uint64_t bit = 1ull << (dev & 63);
-    if (!(opted_in.load(std::memory_order_acquire) & bit)) {
-        cudaError_t e = cudaFuncSetAttribute(
-            kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem_bytes);
-        if (e != cudaSuccess) return e;
-        opted_in.fetch_or(bit, std::memory_order_acq_rel);
-    }
+    constexpr auto kern =
+        dmv::dualmv_stream_f64e_kernel<W, RPW, S, BAND, k3d, kOut, NC, kSelf, kPack>;
+    cudaError_t e = smem_opt_in<kern>(pl.smem_bytes, dev);
+    if (e != cudaSuccess) return e;
     kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(map, prm);
     return cudaGetLastError();
 }
@@ -437,18 +427,9 @@ cudaError_t launch_combine(const Params &prm, cudaStream_t stream) {
     const int64_t blocks = q_blocks + s_blocks;
     if (blocks == 0) return cudaSuccess;
     if (blocks > INT32_MAX) return cudaErrorInvalidConfiguration;
-    cudaLaunchConfig_t cfg;
-    std::memset(&cfg, 0, sizeof cfg);
-    cfg.gridDim = dim3((unsigned)blocks);
-    cfg.blockDim = dim3(256);
-    cfg.dynamicSmemBytes = 0;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, dmv::dualmv_combine_kernel<Acc>, prm, q_blocks, chunks);
+    // After the streaming kernel, whose workspace it reads.
+    return launch_dependent(dmv::dualmv_combine_kernel<Acc>, dim3((unsigned)blocks), dim3(256),
+                            0, stream, prm, q_blocks, chunks);
 }
 
 template <typename Acc>

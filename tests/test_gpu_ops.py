@@ -221,3 +221,50 @@ def test_empty_shapes(dtype):
 
 def test_no_device_fault_recorded():
     assert dm.device_fault() == dm.DUALMV_SUCCESS
+
+
+# ---------------------------------------------------------- golden fixtures ---
+
+import glob as _glob
+import json as _json
+import os as _os
+
+_GOLDEN = sorted(_glob.glob(_os.path.join(_os.path.dirname(_os.path.abspath(__file__)),
+                                          "golden", "*.json")))
+_T = {"f32": torch.float32, "f64": torch.float64, "i32": torch.int32}
+
+
+@pytest.mark.parametrize("fixture", _GOLDEN, ids=_os.path.basename)
+def test_golden_fixture_exact(fixture, path):
+    """Every stored value is exact in its type, so any summation order gives
+    it: the CUDA path must reproduce the fixture exactly, on both paths."""
+    with open(fixture) as f:
+        fx = _json.load(f)
+    t = _T[fx["dtype"]]
+
+    def dev(key):
+        return torch.tensor(fx[key], dtype=t, device=DEV)
+
+    if fx["op"] == "bicg":
+        q, s = dm.dualmv(dev("A")[:, : fx["N"]], dev("p"), dev("r"))
+        got = {"q": q, "s": s}
+    elif fx["op"] == "gesummv":
+        got = {"y": dm.gesummv(dev("A"), dev("B"), dev("x"), alpha=fx["alpha"],
+                               beta=fx["beta"])}
+    elif fx["op"] == "atax":
+        got = {"y": dm.atax(dev("A"), dev("x"))}
+    else:  # with write-back (on the fly), then without (factorised)
+        A, w, x = dev("A"), dev("w"), dev("x")
+        dm.gemver(A, dev("u1"), dev("v1"), dev("u2"), dev("v2"), w, x, dev("y"), dev("z"),
+                  alpha=fx["alpha"], beta=fx["beta"], update_A=True)
+        w2, x2 = dev("w"), dev("x")
+        dm.gemver(dev("A"), dev("u1"), dev("v1"), dev("u2"), dev("v2"), w2, x2, dev("y"),
+                  dev("z"), alpha=fx["alpha"], beta=fx["beta"], update_A=False)
+        got = {"A_hat": A, "w_out": w, "x_out": x}
+        torch.cuda.synchronize()
+        assert torch.equal(w2.cpu(), torch.tensor(fx["w_out"], dtype=t))
+        assert torch.equal(x2.cpu(), torch.tensor(fx["x_out"], dtype=t))
+    torch.cuda.synchronize()
+    for key, val in got.items():
+        want = torch.tensor(fx[key], dtype=val.dtype)
+        assert torch.equal(val.cpu(), want), key

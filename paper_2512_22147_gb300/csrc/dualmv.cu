@@ -165,9 +165,42 @@ CUtensorMapL2promotion l2_promotion(uintptr_t base, int64_t row_bytes, int64_t b
 
 // Encodes A as a 2-D (N, M) or 3-D (N, M, batch) tiled tensor with a box of
 // kBandCols x tile_rows (x 1).  Columns >= N and rows >= M read as zero.
+// The last tensor map this thread encoded, reused when a call repeats the
+// matrix (same address, shape, strides, box and element type).
+struct MapMemo {
+    bool valid = false;
+    int64_t key[10];
+    CUtensorMap map;
+};
+thread_local MapMemo g_map_memo;
+
+template <typename T>
+bool encode_a_uncached(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
+                       int64_t strideA, int64_t batch, int box_cols, int tile_rows,
+                       bool three_d);
+
 template <typename T>
 bool encode_a(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
               int64_t strideA, int64_t batch, int box_cols, int tile_rows, bool three_d) {
+    const int64_t key[10] = {(int64_t)reinterpret_cast<uintptr_t>(A), M, N, lda,
+                             three_d ? strideA : 0, three_d ? batch : 1, box_cols, tile_rows,
+                             three_d ? 1 : 0, (int64_t)tma_dtype<T>()};
+    if (g_map_memo.valid && std::memcmp(key, g_map_memo.key, sizeof key) == 0) {
+        *map = g_map_memo.map;
+        return true;
+    }
+    if (!encode_a_uncached<T>(map, A, M, N, lda, strideA, batch, box_cols, tile_rows, three_d))
+        return false;
+    std::memcpy(g_map_memo.key, key, sizeof key);
+    g_map_memo.map = *map;
+    g_map_memo.valid = true;
+    return true;
+}
+
+template <typename T>
+bool encode_a_uncached(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64_t lda,
+                       int64_t strideA, int64_t batch, int box_cols, int tile_rows,
+                       bool three_d) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     const int64_t es = sizeof(T);
@@ -250,6 +283,15 @@ Geometry geometry(int64_t elem_bytes, int64_t acc_bytes, Kind kind) {
     return acc_bytes == 8 ? generic_geometry<int32_t>(tma) : generic_geometry<float>(tma);
 }
 
+// The last plan this thread made, reused when a call repeats the shape (the
+// segment count below loops over every CTA, a few microseconds per call).
+struct PlanMemo {
+    bool valid = false;
+    int64_t key[9];
+    dualmv_plan_t plan;
+};
+thread_local PlanMemo g_plan_memo;
+
 dualmv_status make_plan_geo(int64_t M, int64_t N, int64_t batch, int64_t elem_bytes,
                             int64_t acc_bytes, int64_t ctas, const Geometry &geo,
                             dualmv_plan_t *pl) {
@@ -258,6 +300,12 @@ dualmv_status make_plan_geo(int64_t M, int64_t N, int64_t batch, int64_t elem_by
     if ((elem_bytes != 4 && elem_bytes != 8) || (acc_bytes != 4 && acc_bytes != 8) ||
         acc_bytes < elem_bytes)
         return DUALMV_ERR_INVALID_VALUE;
+    const int64_t key[9] = {M, N, batch, elem_bytes, acc_bytes, ctas, geo.band_cols,
+                            geo.tile_rows, geo.smem * 4096 + geo.threads};
+    if (g_plan_memo.valid && std::memcmp(key, g_plan_memo.key, sizeof key) == 0) {
+        *pl = g_plan_memo.plan;
+        return DUALMV_SUCCESS;
+    }
     const int64_t bm = geo.tile_rows;
     dualmv_plan_t p;
     std::memset(&p, 0, sizeof p);
@@ -286,6 +334,9 @@ dualmv_status make_plan_geo(int64_t M, int64_t N, int64_t batch, int64_t elem_by
     p.smem_bytes = geo.smem;
     p.threads = geo.threads;
     *pl = p;
+    std::memcpy(g_plan_memo.key, key, sizeof key);
+    g_plan_memo.plan = p;
+    g_plan_memo.valid = true;
     return DUALMV_SUCCESS;
 }
 

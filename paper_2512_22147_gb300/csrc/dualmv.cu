@@ -39,13 +39,13 @@ constexpr int kStages = 6;
 constexpr int kDirectCtasPerSm = 4;
 // fp64 on the FP32 pipes (dualmv_f64e.cuh).
 #ifndef DUALMV_F64E_WARPS
-#define DUALMV_F64E_WARPS 8
+#define DUALMV_F64E_WARPS 12
 #endif
 #ifndef DUALMV_F64E_RPW
 #define DUALMV_F64E_RPW 4
 #endif
 #ifndef DUALMV_F64E_STAGES
-#define DUALMV_F64E_STAGES 3
+#define DUALMV_F64E_STAGES 2
 #endif
 #ifndef DUALMV_F64E_BAND
 #define DUALMV_F64E_BAND 256
@@ -54,10 +54,11 @@ constexpr int kF64eWarps = DUALMV_F64E_WARPS;
 constexpr int kF64eRpw = DUALMV_F64E_RPW;
 constexpr int kF64eStages = DUALMV_F64E_STAGES;
 constexpr int kF64eBand = DUALMV_F64E_BAND;
-// No producer warp: each consumer warp loads its own boxes.  That frees the
-// warp slot (and registers) for an eighth consumer warp, which this
-// latency-bound kernel turns into throughput; with a producer warp as well,
-// eight consumers would have to fit in 168 registers and spill.
+// No producer warp: each consumer warp loads its own boxes.  The kernel is
+// latency-bound (dependent chains of error-free FP32 transformations), so it
+// turns warps into throughput: 12 warps (three per SM sub-partition, 163
+// registers each) with two 8 KiB stages apiece, as many as shared memory
+// holds.  A producer warp would take a warp slot and registers from them.
 constexpr bool kF64eSelf = true;
 // The double-float arithmetic of each lane's column pairs runs as packed
 // FP32x2 instructions, with no native fp64 columns: the kernel is bound by
@@ -602,13 +603,13 @@ const std::vector<Variant> &i32_table() {
     return tab;
 }
 
-// fp64: the double-float kernel in several shapes (entry 0: 8 self-loading
-// warps x 4 rows, 3 stages, packed pairs), the scalar forms with and without
+// fp64: the double-float kernel in several shapes (entry 0: 12 self-loading
+// warps x 4 rows, 2 stages, packed pairs), the scalar forms with and without
 // native fp64 columns, the earlier layout with a producer warp and 7
 // consumers, and native fp64 FMA.
 const std::vector<Variant> &f64_table() {
     static const std::vector<Variant> tab = {
-        f64e_variant<8, 4, 3, 0, true, true>(0),
+        f64e_variant<12, 4, 2, 0, true, true>(0),
         f64e_variant<8, 4, 2, 0, true, true>(1),
         f64e_variant<8, 4, 3, 0, true, false>(2),    // scalar FP32 instructions
         f64e_variant<8, 4, 3, 2, true, false>(3),
@@ -619,12 +620,18 @@ const std::vector<Variant> &f64_table() {
         stream_variant<double, 7, 4, 3>(8),          // native fp64 FMA
         f64e_variant<6, 4, 3, 2, false, false>(9),
         f64e_variant<7, 4, 2, 2, false, false>(10),
-        // 128-column bands: 4 columns per lane, so 12 warps (3 per SM
-        // sub-partition) fit in 168 registers.
+        // 128-column bands: 4 columns per lane (fewer registers, twice the
+        // share of the row reduction per element).
         f64e_variant<8, 4, 3, 0, true, true, 128>(11),
         f64e_variant<12, 4, 3, 0, true, true, 128>(12),
         f64e_variant<12, 4, 2, 0, true, true, 128>(13),
         f64e_variant<8, 8, 3, 0, true, true, 128>(14),
+        f64e_variant<8, 4, 3, 0, true, true>(15),    // two warps per sub-partition
+        // Fewer warps or rows than entry 0.
+        f64e_variant<10, 4, 2, 0, true, true>(16),
+        f64e_variant<12, 2, 2, 0, true, true>(17),
+        // Four warps per sub-partition on 128-column bands (128 registers).
+        f64e_variant<16, 4, 3, 0, true, true, 128>(18),
     };
     return tab;
 }
@@ -761,6 +768,17 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
         g_path != DUALMV_PATH_TMA_NATIVE_F64)
         var = pick_variant(dtype_code<T>(), M, N, A, lda, es, variant);
     if (var != nullptr) kind = var->kind;
+    if (kind == Kind::kF64e) {
+        // The double-float kernel counts tiles in 32 bits; a launch of 2^31
+        // tiles or more (a huge batch of tiny problems) takes native fp64.
+        const Geometry g = var ? var->geo : geometry(es, sizeof(Acc), kind);
+        const int64_t per_problem = ((N + g.band_cols - 1) / g.band_cols) *
+                                    ((M + g.tile_rows - 1) / g.tile_rows);
+        if (per_problem > (INT32_MAX - 1) / batch) {
+            kind = Kind::kTma;
+            var = nullptr;
+        }
+    }
     CUtensorMap map;
     std::memset(&map, 0, sizeof map);
     if (tma) {

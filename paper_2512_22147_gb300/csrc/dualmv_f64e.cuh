@@ -194,6 +194,57 @@ __device__ __forceinline__ DF2 df_add2(DF2 x, DF2 y) {
     return r;
 }
 
+// Reduce-scatter butterfly without selects, for values a lane computed in a
+// permuted row order: slot j of lane l holds row j ^ butterfly_row(l), so at
+// every halving level each lane sends slot k + h and keeps slot k (its
+// partner, which differs in that level's lane bit, holds the same row in
+// slot k + h).  Slot 0 ends with the full sum of row butterfly_row(l), as in
+// warp_rows_reduce_df.  The first level adds its pairs of slots as packed
+// pairs.
+template <int RPW>
+__device__ __forceinline__ void warp_rows_reduce_df_perm(DF (&v)[RPW]) {
+    int off = 16;
+    int h = RPW / 2;
+    if constexpr (RPW >= 4) {
+        // First level: RPW / 2 sums, as packed pairs.
+#pragma unroll
+        for (int k = 0; k < RPW / 2; k += 2) {
+            DF2 keep, recv;
+            keep.s = make_float2(v[k].s, v[k + 1].s);
+            keep.c = make_float2(v[k].c, v[k + 1].c);
+            recv.s = make_float2(__shfl_xor_sync(0xffffffffu, v[k + RPW / 2].s, off),
+                                 __shfl_xor_sync(0xffffffffu, v[k + RPW / 2 + 1].s, off));
+            recv.c = make_float2(__shfl_xor_sync(0xffffffffu, v[k + RPW / 2].c, off),
+                                 __shfl_xor_sync(0xffffffffu, v[k + RPW / 2 + 1].c, off));
+            const DF2 sum = df_add2(keep, recv);
+            v[k].s = sum.s.x;
+            v[k].c = sum.c.x;
+            v[k + 1].s = sum.s.y;
+            v[k + 1].c = sum.c.y;
+        }
+        off >>= 1;
+        h /= 2;
+    }
+#pragma unroll
+    for (; h >= 1; h /= 2) {
+#pragma unroll
+        for (int k = 0; k < h; ++k) {
+            DF recv;
+            recv.s = __shfl_xor_sync(0xffffffffu, v[k + h].s, off);
+            recv.c = __shfl_xor_sync(0xffffffffu, v[k + h].c, off);
+            v[k] = df_add(v[k], recv);
+        }
+        off >>= 1;
+    }
+#pragma unroll
+    for (; off >= 1; off >>= 1) {
+        DF recv;
+        recv.s = __shfl_xor_sync(0xffffffffu, v[0].s, off);
+        recv.c = __shfl_xor_sync(0xffffffffu, v[0].c, off);
+        v[0] = df_add(v[0], recv);
+    }
+}
+
 // Dynamic shared memory of the fp64 kernel: every consumer warp has its own
 // ring of STAGES boxes (its RPW rows of a tile), so warps wait only for
 // their own rows and drift apart instead of finishing every tile together;
@@ -245,12 +296,13 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int64_t T_ = prm.tiles, G = prm.grid, S = prm.stripes;
+    // Tile indices fit 32 bits (the host sends larger launches elsewhere).
+    const int S = (int)prm.stripes, NB = (int)prm.bands;
     const int64_t c = blockIdx.x;
-    const int64_t t0 = cta_first_tile(c, T_, G);
-    const int64_t t1 = cta_first_tile(c + 1, T_, G);
-    const int64_t ntiles = t1 - t0;
-    const int64_t g_first = t0 / S;
+    const int t0 = (int)cta_first_tile(c, prm.tiles, prm.grid);
+    const int t1 = (int)cta_first_tile(c + 1, prm.tiles, prm.grid);
+    const int ntiles = t1 - t0;
+    const int g_first = t0 / S;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < W * STAGES; ++i) {
@@ -267,13 +319,13 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         if (lane == 0) {
             const uint64_t pol = policy_evict_first();
             bool ok = true;
-            int64_t issued = 0;
+            int issued = 0;
             int partial_w = 0;
-            TileCursor cur;
-            cur.init(t0, S, prm.bands);
+            TileCursor32 cur;
+            cur.init(t0, S, NB);
             int stage = 0;
             uint32_t phase = 0;
-            for (int64_t k = 0; k < ntiles; ++k) {
+            for (int k = 0; k < ntiles; ++k) {
                 const int x = (int)(cur.band * BAND), y = (int)(cur.stripe * BM);
                 // One box of RPW rows per consumer warp, into that warp's ring.
                 for (int w = 0; w < W && ok; ++w) {
@@ -294,7 +346,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                 }
                 if (!ok) break;
                 issued = k + 1;
-                cur.advance(S, prm.bands);
+                cur.advance(S, NB);
                 if (++stage == STAGES) {
                     stage = 0;
                     phase ^= 1u;
@@ -303,7 +355,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             // Every box issued must land before the CTA exits (bounded): the
             // last STAGES whole tiles, and the first partial_w boxes of a
             // tile abandoned half way by a timeout.
-            for (int64_t k = issued > STAGES ? issued - STAGES : 0; k <= issued; ++k) {
+            for (int k = issued > STAGES ? issued - STAGES : 0; k <= issued; ++k) {
                 const int st = (int)(k % STAGES);
                 const int nw = k < issued ? W : partial_w;
                 for (int w = 0; w < nw; ++w)
@@ -352,11 +404,11 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
 #pragma unroll
         for (int e = 0; e < VE; ++e) segp[lane_col<T>(v, lane, e)] = 0.0;
     int ngrp = 0;
-    int64_t seg_start_stripe = 0;
+    int seg_start_stripe = 0;
     bool ok = true;
 
-    TileCursor cur;
-    cur.init(t0, S, prm.bands);
+    TileCursor32 cur;
+    cur.init(t0, S, NB);
     T r_next = T(0);
     {
         const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
@@ -367,9 +419,9 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
 
     // Self-loading: lane 0 keeps a second cursor STAGES tiles ahead and
     // refills each stage of this warp's ring right after the warp read it.
-    TileCursor ld{0, 0, 0, 0};
-    int64_t issued = 0;           // boxes this warp issued (lane 0)
-    int64_t waited_to = ntiles;   // first tile whose wait was abandoned
+    TileCursor32 ld{0, 0, 0, 0};
+    int issued = 0;           // boxes this warp issued (lane 0)
+    int waited_to = ntiles;   // first tile whose wait was abandoned
     uint64_t pol = 0;
     auto issue = [&](int st) {
         const int slot_i = warp * STAGES + st;
@@ -381,19 +433,19 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             tma_load_3d(dst, &tmap, x, y, (int)ld.b, fb, pol);
         else
             tma_load_2d(dst, &tmap, x, y, fb, pol);
-        ld.advance(S, prm.bands);
+        ld.advance(S, NB);
         ++issued;
     };
     if constexpr (kSelf) {
         if (lane == 0) {
             pol = policy_evict_first();
-            ld.init(t0, S, prm.bands);
+            ld.init(t0, S, NB);
             for (int st = 0; st < STAGES && st < ntiles; ++st) issue(st);
         }
     }
     // Releases the stage just read: to the producer warp, or (self-loading)
     // by refilling it with the tile STAGES ahead.
-    auto release = [&](int slot_r, int64_t k_r) {
+    auto release = [&](int slot_r, int k_r) {
         __syncwarp();
         if constexpr (kSelf) {
             if (lane == 0 && ok && k_r + STAGES < ntiles) {
@@ -407,15 +459,15 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         }
     };
 
-    for (int64_t k = 0; k < ntiles; ++k) {
-        const int64_t g = cur.g;
-        const int64_t stripe = cur.stripe;
-        const int64_t band = cur.band;
+    for (int k = 0; k < ntiles; ++k) {
+        const int g = cur.g;
+        const int stripe = cur.stripe;
+        const int band = cur.band;
         const int64_t b = cur.b;
         const int64_t col0 = band * BAND;
         const int64_t row0 = stripe * BM + (int64_t)warp * RPW;
         const T rmine = r_next;
-        cur.advance(S, prm.bands);
+        cur.advance(S, NB);
         if (kS && k + 1 < ntiles) {
             const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
             r_next = (lane < RPW && row < prm.M) ? rg[cur.b * prm.strideR + row] : T(0);
@@ -468,14 +520,17 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         for (int j = 0; j < kNativeCols; ++j) tnat[j] = 0.0;
         uint32_t span = 0;  // max over elements of (|a| bits - 2^-40 bits)
         if constexpr (kPack) {
+            // Slot i of this lane is row i ^ perm (see warp_rows_reduce_df_perm).
+            const int perm = butterfly_row<RPW>(lane);
 #pragma unroll
             for (int i = 0; i < RPW; ++i) {
-                const Vec *rowp = tile + (size_t)i * (ROW_BYTES / 16);
+                const int ri = i ^ perm;
+                const Vec *rowp = tile + (size_t)ri * (ROW_BYTES / 16);
                 Vec a[VPL];
 #pragma unroll
                 for (int v = 0; v < VPL; ++v) a[v] = rowp[v * 32 + lane];
-                const float rh = __shfl_sync(0xffffffffu, rh_mine, i);
-                const float rl = __shfl_sync(0xffffffffu, rl_mine, i);
+                const float rh = __shfl_sync(0xffffffffu, rh_mine, ri);
+                const float rl = __shfl_sync(0xffffffffu, rl_mine, ri);
                 const float2 rh2 = make_float2(rh, rh), rl2 = make_float2(rl, rl);
                 DF2 qp[VPL];
 #pragma unroll
@@ -575,7 +630,12 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
 
         if (!need_fp64) {
             release(slot, k);
-            if constexpr (kQ) warp_rows_reduce_df<RPW>(q, lane);
+            if constexpr (kQ) {
+                if constexpr (kPack)
+                    warp_rows_reduce_df_perm<RPW>(q);
+                else
+                    warp_rows_reduce_df<RPW>(q, lane);
+            }
             if (kQ && butterfly_writer<RPW>(lane)) {
                 const int64_t row = row0 + butterfly_row<RPW>(lane);
                 if (row < prm.M) {
@@ -713,7 +773,7 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     // it never waited for must land before the CTA exits (bounded).
     if constexpr (kSelf) {
         if (lane == 0)
-            for (int64_t kk = waited_to; kk < issued; ++kk)
+            for (int kk = waited_to; kk < issued; ++kk)
                 mbar_wait_bounded(smem_u32(&full_bar[warp * STAGES + (int)(kk % STAGES)]),
                                   (uint32_t)(kk / STAGES) & 1u);
     }

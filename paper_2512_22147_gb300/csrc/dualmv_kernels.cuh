@@ -327,6 +327,28 @@ struct TileCursor {
     }
 };
 
+// The same in 32 bits, for kernels whose launch guarantees fewer than 2^31
+// tiles (the double-float fp64 kernel, where the registers it saves pay).
+struct TileCursor32 {
+    int g, b, band, stripe;
+    __device__ __forceinline__ void init(int t, int S, int bands) {
+        g = t / S;
+        stripe = t - g * S;
+        b = g / bands;
+        band = g - b * bands;
+    }
+    __device__ __forceinline__ void advance(int S, int bands) {
+        if (++stripe == S) {
+            stripe = 0;
+            ++g;
+            if (++band == bands) {
+                band = 0;
+                ++b;
+            }
+        }
+    }
+};
+
 template <typename T, int W, int RPW, int STAGES, bool kTma>
 struct SmemLayout {
     using Acc = typename Traits<T>::Acc;

@@ -122,8 +122,9 @@ def _ref_first(c, T, G):
 ])
 def test_plan_covers_every_tile_once(M, N, batch, eb, ab, sms):
     pl = dm.dualmv_plan(M, N, batch, eb, ab, sms)
-    # fp64: 8 self-loading warps x 4 rows of 256-column bands (FP32-pipe kernel)
-    rows, width = (32, 256)
+    # 4-byte types: 8 warps x 4 rows; fp64: 12 self-loading warps x 4 rows
+    # (FP32-pipe kernel); all on 256-column bands
+    rows, width = (48 if eb == 8 else 32, 256)
     assert pl.band_cols == width and pl.tile_rows == rows
     assert pl.bands == -(-N // width) and pl.stripes == -(-M // rows)
     assert pl.tiles == batch * pl.bands * pl.stripes
@@ -141,7 +142,7 @@ def test_plan_covers_every_tile_once(M, N, batch, eb, ab, sms):
         assert pl.workspace_bytes == 0
     else:
         assert pl.workspace_bytes == -(-q_ws // 256) * 256 + s_ws
-    assert pl.smem_bytes <= 227 * 1024 and pl.threads == (288 if eb == 4 else 256)
+    assert pl.smem_bytes <= 227 * 1024 and pl.threads == (288 if eb == 4 else 384)
 
 
 def test_plan_rejects_bad_shapes():

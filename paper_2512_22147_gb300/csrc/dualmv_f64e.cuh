@@ -313,6 +313,9 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     }
     __syncthreads();
     pdl_launch_dependents();
+    // Launched as a dependent of whatever precedes it on the stream: nothing
+    // is read or written before that grid has completed.
+    pdl_wait();
 
     // ------------------------------------------------------ producer ----
     if (!kSelf && warp == W) {

@@ -715,6 +715,10 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
 template <typename Acc>
 __global__ void __launch_bounds__(256)
 dualmv_combine_kernel(const Params prm, int64_t q_blocks, int q_chunks) {
+    // The next call's fp64 streaming kernel may launch once every block of
+    // this grid has started (it waits for this grid's completion before it
+    // reads or writes anything).
+    pdl_launch_dependents();
     pdl_wait();
     __shared__ Acc part[256];
     const Acc *qw = static_cast<const Acc *>(prm.q_ws);

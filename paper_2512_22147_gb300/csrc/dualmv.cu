@@ -23,6 +23,7 @@
 #include "dualmv_tune.cuh"
 #include "dualmv_wide.cuh"
 #include "dualmv_atax.cuh"
+#include "dualmv_atax_f64.cuh"
 #include "dualmv_ops.cuh"
 
 namespace {
@@ -957,11 +958,12 @@ dualmv_status gesummv_run(int64_t M, int64_t N, T alpha, const T *A, int64_t lda
     return st;
 }
 
-// ATAX with one read of A (dualmv_atax.cuh): fp32, clusters of C CTAs of
-// kAtaxWarps warps, each warp a 256-column sub-band of kAtaxRows-row
-// stripes.  Returns with *used = false, having enqueued nothing, when the
-// problem does not fit the cluster path (alignment, width, no cluster of
-// that size can be placed), so that the caller takes the two-pass path.
+// ATAX with one read of A: clusters of C CTAs, each warp a 256-column
+// sub-band of R-row stripes (fp32: dualmv_atax.cuh, 8 warps x 8 rows; fp64:
+// dualmv_atax_f64.cuh, 8 warps x 4 rows in double-float arithmetic).
+// Returns with *used = false, having enqueued nothing, when the problem does
+// not fit the cluster path (alignment, width, no cluster of that size can be
+// placed), so that the caller takes the two-pass path.
 #ifndef DUALMV_ATAX_ROWS
 #define DUALMV_ATAX_ROWS 8
 #endif
@@ -970,31 +972,61 @@ dualmv_status gesummv_run(int64_t M, int64_t N, T alpha, const T *A, int64_t lda
 #endif
 constexpr int kAtaxWarps = 8, kAtaxRows = DUALMV_ATAX_ROWS, kAtaxStages = DUALMV_ATAX_STAGES;
 
+template <typename T>
+struct AtaxCfg;
+template <>
+struct AtaxCfg<float> {
+    static constexpr int W = kAtaxWarps, R = kAtaxRows, S = kAtaxStages;
+    static constexpr int kThreads = W * 32;
+    using L = dmv::AtaxLayout<W, R, S>;
+    using Params = dmv::AtaxParams;
+    static constexpr auto kern = dmv::atax_cluster_kernel<W, R, S>;
+    static void fill(Params &p, const float *, int64_t) {}
+};
+template <>
+struct AtaxCfg<double> {
+    // Three 8 KiB stages per warp (the column phase of a stripe runs one
+    // stripe later) leave room for 8 warps.
+    static constexpr int W = 8, R = 4, S = 3;
+    static constexpr int kThreads = (W + 1) * 32;  // and a control warp
+    using L = dmv::AtaxLayout64<W, R, S>;
+    using Params = dmv::AtaxParams64;
+    static constexpr auto kern = dmv::atax_cluster_f64_kernel<W, R, S>;
+    static void fill(Params &p, const double *A, int64_t lda) {
+        p.A = A;
+        p.lda = lda;
+    }
+};
+
 struct AtaxClusterCache {
     std::mutex mu;
-    int max_clusters[kMaxDevices][dmv::kAtaxMaxCluster + 1] = {};
-    bool known[kMaxDevices][dmv::kAtaxMaxCluster + 1] = {};
+    int max_clusters[2][kMaxDevices][dmv::kAtaxMaxCluster + 1] = {};
+    bool known[2][kMaxDevices][dmv::kAtaxMaxCluster + 1] = {};
 };
 AtaxClusterCache g_atax_cache;
 
-dualmv_status atax_cluster_run(int64_t M, int64_t N, const float *A, int64_t lda,
-                               const float *x, float *y, cudaStream_t stream, bool *used) {
+template <typename T>
+dualmv_status atax_cluster_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x, T *y,
+                               cudaStream_t stream, bool *used) {
     *used = false;
-    using L = dmv::AtaxLayout<kAtaxWarps, kAtaxRows, kAtaxStages>;
+    using Cfg = AtaxCfg<T>;
+    using L = typename Cfg::L;
+    constexpr int kT = sizeof(T) == 8 ? 1 : 0;
+    const int64_t es = sizeof(T);
     const int64_t bands = (N + kBandCols - 1) / kBandCols;
-    const int64_t C = (bands + kAtaxWarps - 1) / kAtaxWarps;
+    const int64_t C = (bands + Cfg::W - 1) / Cfg::W;
     if (g_path == DUALMV_PATH_DIRECT || C > dmv::kAtaxMaxCluster ||
-        reinterpret_cast<uintptr_t>(A) % 16 != 0 || (lda * 4) % 16 != 0 || M >= INT32_MAX ||
+        reinterpret_cast<uintptr_t>(A) % 16 != 0 || (lda * es) % 16 != 0 || M >= INT32_MAX ||
         N >= INT32_MAX)
         return DUALMV_SUCCESS;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return cuda_fail(e);
     if (dev < 0 || dev >= kMaxDevices) return DUALMV_SUCCESS;
-    auto kern = dmv::atax_cluster_kernel<kAtaxWarps, kAtaxRows, kAtaxStages>;
+    auto kern = Cfg::kern;
     cudaLaunchConfig_t cfg;
     std::memset(&cfg, 0, sizeof cfg);
-    cfg.blockDim = dim3(kAtaxWarps * 32);
+    cfg.blockDim = dim3(Cfg::kThreads);
     cfg.dynamicSmemBytes = (size_t)L::kTotal;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
@@ -1007,7 +1039,7 @@ dualmv_status atax_cluster_run(int64_t M, int64_t N, const float *A, int64_t lda
     int max_clusters = 0;
     {
         std::lock_guard<std::mutex> lk(g_atax_cache.mu);
-        if (!g_atax_cache.known[dev][C]) {
+        if (!g_atax_cache.known[kT][dev][C]) {
             e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)L::kTotal);
             if (e == cudaSuccess && C > 8)
@@ -1020,23 +1052,25 @@ dualmv_status atax_cluster_run(int64_t M, int64_t N, const float *A, int64_t lda
                 (void)cudaGetLastError();
                 max_clusters = 0;
             }
-            g_atax_cache.max_clusters[dev][C] = max_clusters;
-            g_atax_cache.known[dev][C] = true;
+            g_atax_cache.max_clusters[kT][dev][C] = max_clusters;
+            g_atax_cache.known[kT][dev][C] = true;
         }
-        max_clusters = g_atax_cache.max_clusters[dev][C];
+        max_clusters = g_atax_cache.max_clusters[kT][dev][C];
     }
     if (max_clusters <= 0) return DUALMV_SUCCESS;
     CUtensorMap map;
     std::memset(&map, 0, sizeof map);
-    if (!encode_a<float>(&map, A, M, N, lda, M * lda, 1, kBandCols, kAtaxRows, false))
+    if (!encode_a<T>(&map, A, M, N, lda, M * lda, 1, kBandCols, Cfg::R, false))
         return DUALMV_SUCCESS;
-    const int64_t stripes = (M + kAtaxRows - 1) / kAtaxRows;
+    const int64_t stripes = (M + Cfg::R - 1) / Cfg::R;
     const int64_t clusters = stripes < max_clusters ? stripes : max_clusters;
-    float *ws = nullptr;
+    T *ws = nullptr;
     dualmv_status st = pool_alloc(&ws, clusters * N, stream);
     if (st != DUALMV_SUCCESS) return st;
     *used = true;
-    dmv::AtaxParams prm;
+    typename Cfg::Params prm;
+    std::memset(&prm, 0, sizeof prm);
+    Cfg::fill(prm, A, lda);
     prm.x = x;
     prm.y_ws = ws;
     prm.M = M;
@@ -1049,7 +1083,7 @@ dualmv_status atax_cluster_run(int64_t M, int64_t N, const float *A, int64_t lda
     if (e == cudaSuccess) {
         int64_t blocks = (N + 255) / 256;
         if (blocks > 4096) blocks = 4096;
-        dmv::atax_sum_kernel<<<(unsigned)blocks, 256, 0, stream>>>(ws, y, N, clusters);
+        dmv::atax_sum_kernel<T><<<(unsigned)blocks, 256, 0, stream>>>(ws, y, N, clusters);
         e = cudaGetLastError();
     }
     cudaError_t ef = cudaFreeAsync(ws, stream);
@@ -1058,9 +1092,9 @@ dualmv_status atax_cluster_run(int64_t M, int64_t N, const float *A, int64_t lda
     return DUALMV_SUCCESS;
 }
 
-// ATAX (Table 1): y = A^T (A x).  fp32 takes the single-read cluster path
-// when it fits; otherwise (and for fp64) tmp = A x by a rows-only pass and
-// y = A^T tmp by a columns-only pass over the same A.
+// ATAX (Table 1): y = A^T (A x).  The single-read cluster path when it fits;
+// otherwise tmp = A x by a rows-only pass and y = A^T tmp by a columns-only
+// pass over the same A.
 template <typename T>
 dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x, T *y,
                        cudaStream_t stream) {
@@ -1073,12 +1107,10 @@ dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x
         return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
     }
     if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
-    if constexpr (std::is_same<T, float>::value) {
-        if (g_atax_two_pass == 0) {
-            bool used = false;
-            dualmv_status sc = atax_cluster_run(M, N, A, lda, x, y, stream, &used);
-            if (sc != DUALMV_SUCCESS || used) return sc;
-        }
+    if (g_atax_two_pass == 0) {
+        bool used = false;
+        dualmv_status sc = atax_cluster_run<T>(M, N, A, lda, x, y, stream, &used);
+        if (sc != DUALMV_SUCCESS || used) return sc;
     }
     T *tmp = nullptr;
     dualmv_status st = pool_alloc(&tmp, M, stream);

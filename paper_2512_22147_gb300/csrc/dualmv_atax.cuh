@@ -308,11 +308,12 @@ atax_cluster_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxParams p
 }
 
 // y = sum over clusters of their column sums, in cluster order.
-__global__ void __launch_bounds__(256) atax_sum_kernel(const float *y_ws, float *y, int64_t N,
+template <typename T>
+__global__ void __launch_bounds__(256) atax_sum_kernel(const T *y_ws, T *y, int64_t N,
                                                        int64_t clusters) {
     const int64_t threads = (int64_t)gridDim.x * blockDim.x;
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N; j += threads) {
-        float acc = 0.f;
+        T acc = T(0);
         for (int64_t c = 0; c < clusters; ++c) acc += y_ws[c * N + j];
         y[j] = acc;
     }

@@ -115,6 +115,74 @@ def test_atax_one_read_is_deterministic():
     assert torch.equal(y1, y2)
 
 
+# fp64 widths for the single-read path (8 sub-bands of 256 columns per CTA):
+# clusters of 1, 2, 3, 4, 8 and 10 CTAs, and one too wide for a cluster of
+# 16 (two passes).
+@pytest.mark.parametrize("M,N", [(1000, 700), (2049, 3000), (301, 5000), (4096, 8192),
+                                 (517, 16384), (64, 20000), (40, 40000)])
+def test_atax_f64_one_read_widths(M, N, atax_mode):
+    A, x = inputs.generate_atax(_w("atax", "f64", M, N, N, 11 * M + N), DEV)
+    check_atax(A, x, N, "f64")
+
+
+def test_atax_f64_one_read_path_runs():
+    """As for fp32: the cluster kernel's summation order differs from the
+    two-pass path's, so its bits differ on random data."""
+    A, x = inputs.generate_atax(_w("atax", "f64", 2048, 4096, 4096, 15), DEV)
+    old = dm.dualmv_atax_set_two_pass(0)
+    try:
+        y1 = dm.atax(A, x)
+        dm.dualmv_atax_set_two_pass(1)
+        y2 = dm.atax(A, x)
+        torch.cuda.synchronize()
+    finally:
+        dm.dualmv_atax_set_two_pass(old)
+    assert not torch.equal(y1, y2)
+    assert dm.device_fault() == dm.DUALMV_SUCCESS
+
+
+def test_atax_f64_one_read_is_deterministic():
+    A, x = inputs.generate_atax(_w("atax", "f64", 3000, 5000, 5000, 16), DEV)
+    y1 = dm.atax(A, x)
+    y2 = dm.atax(A, x)
+    torch.cuda.synchronize()
+    assert torch.equal(y1, y2)
+
+
+@pytest.mark.parametrize("case", ["zeros", "a_huge_tiny", "x_zero_huge", "t_out_of_range",
+                                  "zero_rows"])
+def test_atax_f64_one_read_range(case, atax_mode):
+    """The double-float cluster kernel is exact only for |a|, |x|, |t| in
+    [2^-40, 2^40) or zero: zeros stay on the fast path, anything else sends
+    the stripe (or the warp) to native fp64.  Every case matches the
+    oracle."""
+    M, N = 1500, 3000
+    A, x = inputs.generate_atax(_w("atax", "f64", M, N, N + 2, 17), DEV)
+    if case == "zeros":
+        A[:, ::3] = 0.0
+        A[::5, :] = 0.0
+        x[::7] = 0.0
+    elif case == "a_huge_tiny":
+        A[13, 100] = 3.0e20
+        A[700, 2500] = -2.5e-20
+        A[1499, 2999] = 1.0e100     # t of row 1499 ~ 1e100; y stays finite
+    elif case == "x_zero_huge":
+        x[::11] = 0.0
+        x[1024] = 7.0e15
+    elif case == "t_out_of_range":
+        # a stays in range; t does not.  Rows 40-43: |a| ~ 1e11, so t is near
+        # 1e11 * sqrt(N) > 2^40.  Row 900: two entries whose products cancel
+        # to a rounding residue, t ~ 1e-16 < 2^-40.
+        A[40:44, :] *= 1.0e11
+        A[900, :] = 0.0
+        A[900, 0] = 1.0
+        A[900, 1] = -(x[0] / x[1])
+    elif case == "zero_rows":
+        A[200:208, :] = 0.0         # t exactly zero
+    check_atax(A, x, N, "f64")
+    assert dm.device_fault() == dm.DUALMV_SUCCESS
+
+
 def check_gemver(ops, N, alpha, beta, update_A, dtype):
     """GEMVER on the GPU vs the oracle.  Denominators (terms' magnitudes):
     A_hat: |A| + |u1 v1| + |u2 v2|;  x: |x| + |beta| sum_i Am_ij |y_i| + |z|;

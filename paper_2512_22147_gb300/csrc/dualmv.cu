@@ -983,11 +983,21 @@ struct AtaxCfg<float> {
     static constexpr auto kern = dmv::atax_cluster_kernel<W, R, S>;
     static void fill(Params &p, const float *, int64_t) {}
 };
+#ifndef DUALMV_ATAX64_WARPS
+#define DUALMV_ATAX64_WARPS 8
+#endif
+#ifndef DUALMV_ATAX64_ROWS
+#define DUALMV_ATAX64_ROWS 4
+#endif
+#ifndef DUALMV_ATAX64_STAGES
+#define DUALMV_ATAX64_STAGES 3
+#endif
 template <>
 struct AtaxCfg<double> {
     // Three 8 KiB stages per warp (the column phase of a stripe runs one
     // stripe later) leave room for 8 warps.
-    static constexpr int W = 8, R = 4, S = 3;
+    static constexpr int W = DUALMV_ATAX64_WARPS, R = DUALMV_ATAX64_ROWS,
+                         S = DUALMV_ATAX64_STAGES;
     static constexpr int kThreads = (W + 1) * 32;  // and a control warp
     using L = dmv::AtaxLayout64<W, R, S>;
     using Params = dmv::AtaxParams64;

@@ -1146,37 +1146,38 @@ dualmv_status gemver_factored(int64_t M, int64_t N, T alpha, T beta, const T *A,
                               const T *u1, const T *v1, const T *u2, const T *v2, T *w, T *x,
                               const T *y, const T *z, cudaStream_t stream) {
     T *s = nullptr, *t = nullptr;
-    double *part = nullptr;  // [2 products][kDotChunks][sum, error], one side at a time
+    // [side][2 products][kDotChunks][sum, error]: u . y, then v . x
+    double *part = nullptr;
     dualmv_status st = pool_alloc(&s, N, stream);
     if (st == DUALMV_SUCCESS) st = pool_alloc(&t, M, stream);
-    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * dmv::kDotChunks, stream);
+    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * 2 * dmv::kDotChunks, stream);
+    double *part_u = part, *part_v = part ? part + 2 * 2 * dmv::kDotChunks : nullptr;
     cudaError_t e = cudaSuccess;
+    // The vector kernels are programmatic dependents of the kernel before
+    // them (each waits for it before reading): their launches overlap it.
     if (st == DUALMV_SUCCESS && N > 0) {  // s = A^T y (zero when M == 0)
-        dmv::dots2_partial_kernel<T><<<2 * dmv::kDotChunks, 256, 0, stream>>>(u1, u2, y, M,
-                                                                               part);
-        e = cudaGetLastError();
+        e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks), dim3(256),
+                             0, stream, u1, u2, y, M, part_u);
         if (e == cudaSuccess)
             st = run<T, T>(M, N, A, lda, 0, nullptr, 0, y, 0, nullptr, 0, s, 0, 1, stream,
                            dmv::kOutS);
-        if (e == cudaSuccess && st == DUALMV_SUCCESS) {
-            const int64_t bx = (N + 255) / 256;
-            dmv::gemver_x2_kernel<T><<<(unsigned)(bx > 4096 ? 4096 : bx), 256, 0, stream>>>(
-                x, s, v1, v2, part, z, N, beta);
-            e = cudaGetLastError();
-        }
+        // x, and the chunk sums of v1 . x and v2 . x for the new x.
+        if (e == cudaSuccess && st == DUALMV_SUCCESS)
+            e = launch_dependent(dmv::gemver_x2_kernel<T>, dim3(dmv::kDotChunks), dim3(256), 0,
+                                 stream, x, (const T *)s, v1, v2, (const double *)part_u, z, N,
+                                 beta, part_v);
+    } else if (st == DUALMV_SUCCESS && M > 0) {  // N == 0: v . x is zero
+        e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks), dim3(256),
+                             0, stream, v1, v2, x, N, part_v);
     }
     if (st == DUALMV_SUCCESS && e == cudaSuccess && M > 0) {  // t = A x (zero when N == 0)
-        dmv::dots2_partial_kernel<T><<<2 * dmv::kDotChunks, 256, 0, stream>>>(v1, v2, x, N,
-                                                                               part);
-        e = cudaGetLastError();
-        if (e == cudaSuccess)
-            st = run<T, T>(M, N, A, lda, 0, x, 0, nullptr, 0, t, 0, nullptr, 0, 1, stream,
-                           dmv::kOutQ);
-        if (e == cudaSuccess && st == DUALMV_SUCCESS) {
+        st = run<T, T>(M, N, A, lda, 0, x, 0, nullptr, 0, t, 0, nullptr, 0, 1, stream,
+                       dmv::kOutQ);
+        if (st == DUALMV_SUCCESS) {
             const int64_t bw = (M + 255) / 256;
-            dmv::gemver_w2_kernel<T><<<(unsigned)(bw > 4096 ? 4096 : bw), 256, 0, stream>>>(
-                w, t, u1, u2, part, M, alpha);
-            e = cudaGetLastError();
+            e = launch_dependent(dmv::gemver_w2_kernel<T>, dim3((unsigned)(bw > 4096 ? 4096 : bw)),
+                                 dim3(256), 0, stream, w, (const T *)t, u1, u2,
+                                 (const double *)part_v, M, alpha);
         }
     }
     if (st == DUALMV_SUCCESS && e != cudaSuccess) st = cuda_fail(e);

@@ -6,6 +6,8 @@
 
 #include <cstdint>
 
+#include "dualmv_kernels.cuh"
+
 namespace dmv {
 
 template <typename T>
@@ -46,23 +48,20 @@ __device__ __forceinline__ void two_sum_d(double a, double b, double &s, double 
     e = (a - (s - bb)) + (b - bb);
 }
 
-template <typename T>
-__global__ void __launch_bounds__(256) dots2_partial_kernel(const T *a, const T *b, const T *c,
-                                                            int64_t n, double *part) {
-    __shared__ double hs[256], hc[256];
-    const int dot = blockIdx.x / kDotChunks, chunk = blockIdx.x % kDotChunks;
-    const T *u = dot == 0 ? a : b;
-    const int64_t k0 = chunk * n / kDotChunks, k1 = (chunk + 1) * n / kDotChunks;
-    double s = 0.0, cc = 0.0;
-    for (int64_t k = k0 + threadIdx.x; k < k1; k += 256) {
-        const double x = (double)u[k], y = (double)c[k];
-        const double p = x * y;
-        const double pe = fma(x, y, -p);  // exact rounding error of the product
-        double t, e;
-        two_sum_d(s, p, t, e);
-        s = t;
-        cc += e + pe;
-    }
+// s + cc += x y, compensated (TwoProduct, TwoSum).
+__device__ __forceinline__ void dot2_step(double x, double y, double &s, double &cc) {
+    const double p = x * y;
+    const double pe = fma(x, y, -p);  // exact rounding error of the product
+    double t, e;
+    two_sum_d(s, p, t, e);
+    s = t;
+    cc += e + pe;
+}
+
+// The block's 256 compensated sums in a fixed pairwise tree; thread 0
+// writes the block's (sum, error) to part[2 * slot].
+__device__ __forceinline__ void dot2_block_store(double s, double cc, double *hs, double *hc,
+                                                 double *part, int slot) {
     hs[threadIdx.x] = s;
     hc[threadIdx.x] = cc;
     __syncthreads();
@@ -76,49 +75,131 @@ __global__ void __launch_bounds__(256) dots2_partial_kernel(const T *a, const T 
         __syncthreads();
     }
     if (threadIdx.x == 0) {
-        part[2 * blockIdx.x] = hs[0];
-        part[2 * blockIdx.x + 1] = hc[0];
+        part[2 * slot] = hs[0];
+        part[2 * slot + 1] = hc[0];
+    }
+    __syncthreads();
+}
+
+// dot2_block_store for two sums at once (one tree, both in each step):
+// (s1, c1) to part[2 * slot1], (s2, c2) to part[2 * slot2].
+__device__ __forceinline__ void dot2_block_store2(double s1, double c1, double s2, double c2,
+                                                  double *hs, double *hc, double *part,
+                                                  int slot1, int slot2) {
+    const int t = threadIdx.x;
+    hs[t] = s1;
+    hc[t] = c1;
+    hs[256 + t] = s2;
+    hc[256 + t] = c2;
+    __syncthreads();
+    for (int h = 128; h >= 1; h >>= 1) {
+        if (t < h) {
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                const int i = q * 256 + t;
+                double s, e;
+                two_sum_d(hs[i], hs[i + h], s, e);
+                hc[i] += hc[i + h] + e;
+                hs[i] = s;
+            }
+        }
+        __syncthreads();
+    }
+    if (t == 0) {
+        part[2 * slot1] = hs[0];
+        part[2 * slot1 + 1] = hc[0];
+        part[2 * slot2] = hs[256];
+        part[2 * slot2 + 1] = hc[256];
     }
 }
 
-// Dot product `dot` (0 or 1) from its chunk sums, in chunk order.
+// Launched as a programmatic dependent of the kernel before it: waits for
+// that grid before reading its inputs.
 template <typename T>
-__device__ __forceinline__ T dots2_final(const double *part, int dot) {
+__global__ void __launch_bounds__(256) dots2_partial_kernel(const T *a, const T *b, const T *c,
+                                                            int64_t n, double *part) {
+    pdl_launch_dependents();
+    pdl_wait();
+    __shared__ double hs[256], hc[256];
+    const int dot = blockIdx.x / kDotChunks, chunk = blockIdx.x % kDotChunks;
+    const T *u = dot == 0 ? a : b;
+    const int64_t k0 = chunk * n / kDotChunks, k1 = (chunk + 1) * n / kDotChunks;
     double s = 0.0, cc = 0.0;
-    for (int i = 0; i < kDotChunks; ++i) {
-        const int blk = dot * kDotChunks + i;
-        double t, e;
-        two_sum_d(s, part[2 * blk], t, e);
-        s = t;
-        cc += part[2 * blk + 1] + e;
+    for (int64_t k = k0 + threadIdx.x; k < k1; k += 256)
+        dot2_step((double)u[k], (double)c[k], s, cc);
+    dot2_block_store(s, cc, hs, hc, part, blockIdx.x);
+}
+
+// Both dot products from their chunk sums, by every thread of a 256-thread
+// block: threads 0-63 take dot 0's chunks, 64-127 dot 1's, and add them in
+// a fixed pairwise tree (TwoSum on the sums, the errors carried).  GB300's
+// FP64 pipe is narrow, so a tree of 6 levels replaces a chain of 64 steps.
+// dd[0], dd[1] hold the results on return.
+template <typename T>
+__device__ __forceinline__ void dots2_final_block(const double *part, double *hs, double *hc,
+                                                  T *dd) {
+    static_assert(2 * kDotChunks <= 256, "one thread per chunk sum");
+    const int t = threadIdx.x;
+    if (t < 2 * kDotChunks) {
+        hs[t] = part[2 * t];
+        hc[t] = part[2 * t + 1];
     }
-    return (T)(s + cc);
+    __syncthreads();
+    for (int h = kDotChunks / 2; h >= 1; h >>= 1) {
+        const int k = t % kDotChunks;  // position within its dot's chunks
+        if (t < 2 * kDotChunks && k < h) {
+            double s, e;
+            two_sum_d(hs[t], hs[t + h], s, e);
+            hc[t] += hc[t + h] + e;
+            hs[t] = s;
+        }
+        __syncthreads();
+    }
+    if (t == 0) dd[0] = (T)(hs[0] + hc[0]);
+    if (t == kDotChunks) dd[1] = (T)(hs[kDotChunks] + hc[kDotChunks]);
+    __syncthreads();
 }
 
 // x = x + beta (s + v1 d0 + v2 d1) + z, d0 = u1 . y and d1 = u2 . y from
-// their chunk sums (every block forms them the same way).
+// their chunk sums (every block forms them the same way); and, in the same
+// pass, the chunk sums of v1 . x and v2 . x for the new x (part_v, laid out
+// as dots2_partial_kernel's).  kDotChunks blocks, block k on chunk k, each
+// thread on the elements k0 + thread, k0 + thread + 256, ... in order.
+// Launched as a programmatic dependent: waits for the grid before it.
 template <typename T>
-__global__ void gemver_x2_kernel(T *x, const T *s, const T *v1, const T *v2,
-                                 const double *part, const T *z, int64_t n, T beta) {
+__global__ void __launch_bounds__(256) gemver_x2_kernel(T *x, const T *s, const T *v1,
+                                                        const T *v2, const double *part_u,
+                                                        const T *z, int64_t n, T beta,
+                                                        double *part_v) {
+    pdl_launch_dependents();
+    pdl_wait();
     __shared__ T dd[2];
-    if (threadIdx.x < 2) dd[threadIdx.x] = dots2_final<T>(part, threadIdx.x);
-    __syncthreads();
+    __shared__ double hs[512], hc[512];
+    dots2_final_block<T>(part_u, hs, hc, dd);
     const T d0 = dd[0], d1 = dd[1];
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
-         i += (int64_t)gridDim.x * blockDim.x) {
+    const int chunk = blockIdx.x;
+    const int64_t k0 = chunk * n / kDotChunks, k1 = (chunk + 1) * n / kDotChunks;
+    double s1 = 0.0, c1 = 0.0, s2 = 0.0, c2 = 0.0;
+    for (int64_t i = k0 + threadIdx.x; i < k1; i += 256) {
         const T inner = fma(v2[i], d1, fma(v1[i], d0, s[i]));
-        x[i] = fma(beta, inner, x[i]) + z[i];
+        const T xn = fma(beta, inner, x[i]) + z[i];
+        x[i] = xn;
+        dot2_step((double)v1[i], (double)xn, s1, c1);
+        dot2_step((double)v2[i], (double)xn, s2, c2);
     }
+    dot2_block_store2(s1, c1, s2, c2, hs, hc, part_v, chunk, kDotChunks + chunk);
 }
 
 // w = w + alpha (t + u1 e0 + u2 e1), e0 = v1 . x and e1 = v2 . x from
 // their chunk sums.
 template <typename T>
-__global__ void gemver_w2_kernel(T *w, const T *t, const T *u1, const T *u2,
+__global__ void __launch_bounds__(256) gemver_w2_kernel(T *w, const T *t, const T *u1, const T *u2,
                                  const double *part, int64_t n, T alpha) {
+    pdl_launch_dependents();
+    pdl_wait();
     __shared__ T dd[2];
-    if (threadIdx.x < 2) dd[threadIdx.x] = dots2_final<T>(part, threadIdx.x);
-    __syncthreads();
+    __shared__ double hs[2 * kDotChunks], hc[2 * kDotChunks];
+    dots2_final_block<T>(part, hs, hc, dd);
     const T d0 = dd[0], d1 = dd[1];
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {

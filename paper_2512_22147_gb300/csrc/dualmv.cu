@@ -959,18 +959,25 @@ dualmv_status gesummv_run(int64_t M, int64_t N, T alpha, const T *A, int64_t lda
 }
 
 // ATAX with one read of A: clusters of C CTAs, each warp a 256-column
-// sub-band of R-row stripes (fp32: dualmv_atax.cuh, 8 warps x 8 rows; fp64:
-// dualmv_atax_f64.cuh, 8 warps x 4 rows in double-float arithmetic).
+// sub-band of R-row stripes (fp32: dualmv_atax.cuh, 16 warps x 4 rows;
+// fp64: dualmv_atax_f64.cuh, 8 warps x 4 rows in double-float arithmetic).
 // Returns with *used = false, having enqueued nothing, when the problem does
 // not fit the cluster path (alignment, width, no cluster of that size can be
 // placed), so that the caller takes the two-pass path.
 #ifndef DUALMV_ATAX_ROWS
-#define DUALMV_ATAX_ROWS 8
+#define DUALMV_ATAX_ROWS 4
 #endif
 #ifndef DUALMV_ATAX_STAGES
 #define DUALMV_ATAX_STAGES 3
 #endif
-constexpr int kAtaxWarps = 8, kAtaxRows = DUALMV_ATAX_ROWS, kAtaxStages = DUALMV_ATAX_STAGES;
+// fp32: 16 warps x 4-row stripes, so that a CTA covers 4096 columns and
+// 16384 columns take clusters of 4 (36 fit at once: 144 SMs) instead of 8
+// (15: 120 SMs).  89.2% -> 96.9% of HBM on 16384 x 16384.
+#ifndef DUALMV_ATAX_WARPS
+#define DUALMV_ATAX_WARPS 16
+#endif
+constexpr int kAtaxWarps = DUALMV_ATAX_WARPS, kAtaxRows = DUALMV_ATAX_ROWS,
+              kAtaxStages = DUALMV_ATAX_STAGES;
 
 template <typename T>
 struct AtaxCfg;

@@ -80,11 +80,12 @@ def test_atax_matches_oracle(dtype, M, N, pad, path, atax_mode):
     check_atax(A, x, N, dtype)
 
 
-# fp32 widths for the single-read path: clusters of 1, 2, 3, 8 and 10 CTAs
-# (8 sub-bands of 256 columns per CTA), and one too wide for a cluster of 16
-# (two passes).
+# fp32 widths for the single-read path: clusters of 1, 2, 4, 5, 10 and 16
+# CTAs (16 sub-bands of 256 columns per CTA), and one too wide for a cluster
+# of 16 (two passes).
 @pytest.mark.parametrize("M,N", [(4096, 16384), (300, 20000), (1000, 700), (1999, 4100),
-                                 (33, 6144), (256, 40000), (9, 16384)])
+                                 (33, 6144), (256, 40000), (9, 16384), (17, 65536),
+                                 (40, 70000)])
 def test_atax_one_read_widths(M, N, atax_mode):
     A, x = inputs.generate_atax(_w("atax", "f32", M, N, N, 7 * M + N), DEV)
     check_atax(A, x, N, "f32")

@@ -39,63 +39,103 @@ def _vec_stride(v: torch.Tensor, length: int, batch: int, name: str) -> int:
     return v.stride(0)
 
 
+# Per input dtype: (output dtype, single-problem entry, batched entry, tag).
+_ENTRY: dict = {}
+
+# The current device and the raw handle of its current stream, as plain
+# integers when torch has these bindings (building a torch.cuda.Stream
+# object costs microseconds a call); else through the public API.
+_get_device = getattr(torch._C, "_cuda_getDevice", None) or torch.cuda.current_device
+_raw_stream = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+
+
+def _current_stream_handle(dev_idx: int) -> int:
+    if _raw_stream is not None:
+        return _raw_stream(dev_idx)
+    return torch.cuda.current_stream(dev_idx).cuda_stream
+
+
+def _call_on(dev_idx: int, stream, fn, *args):
+    """fn(*args, stream handle) with device dev_idx current (switched to only
+    when it is not); stream None means that device's current stream."""
+    ctx = torch.cuda.device(dev_idx) if dev_idx != _get_device() else None
+    if ctx is not None:
+        ctx.__enter__()
+    try:
+        h = _current_stream_handle(dev_idx) if stream is None else stream.cuda_stream
+        return fn(*args, h)
+    finally:
+        if ctx is not None:
+            ctx.__exit__(None, None, None)
+
+
+def _entry(dtype):
+    e = _ENTRY.get(dtype)
+    if e is None:
+        tag = _TAG.get(dtype)
+        if tag is None:
+            raise TypeError(f"unsupported dtype {dtype}; use float32, float64 or int32")
+        e = (_OUT[dtype], getattr(B, f"dualmv_{tag}"),
+             getattr(B, f"dualmv_{tag}_strided_batched"), tag)
+        _ENTRY[dtype] = e
+    return e
+
+
 def dualmv(A: torch.Tensor, p: torch.Tensor, r: torch.Tensor,
            q: torch.Tensor | None = None, s: torch.Tensor | None = None,
            stream: torch.cuda.Stream | None = None):
     """Compute ``q = A p`` and ``s = A^T r`` (per problem when batched).
 
     Returns ``(q, s)``; pass ``q``/``s`` to write into existing buffers.
-    Runs asynchronously on ``stream`` (default: the current stream).
+    Runs asynchronously on ``stream`` (default: the current stream of A's
+    device).
     """
-    if A.dtype not in _TAG:
-        raise TypeError(f"unsupported dtype {A.dtype}; use float32, float64 or int32")
+    dt = A.dtype
+    out_t, fn_single, fn_batched, tag = _entry(dt)
     if not A.is_cuda:
         raise ValueError("A must be a CUDA tensor (the library has no CPU path)")
+    dev_idx = A.get_device()
     for t, n in ((p, "p"), (r, "r")):
-        if t.dtype != A.dtype or t.device != A.device:
+        if t.dtype != dt or t.get_device() != dev_idx:
             raise ValueError(f"{n} must match A's dtype and device")
-    batched = A.dim() == 3
-    if A.dim() not in (2, 3):
+    nd = A.dim()
+    if nd not in (2, 3):
         raise ValueError("A must be 2-D (M, N) or 3-D (B, M, N)")
-    Bn = A.shape[0] if batched else 1
-    M, N = A.shape[-2], A.shape[-1]
-    if N > 1 and A.stride(-1) != 1:
+    batched = nd == 3
+    shape, strides = A.shape, A.stride()
+    Bn = shape[0] if batched else 1
+    M, N = shape[-2], shape[-1]
+    if N > 1 and strides[-1] != 1:
         raise ValueError("A's last dimension must be contiguous")
-    if M > 1 and A.stride(-2) < N:
+    if M > 1 and strides[-2] < N:
         raise ValueError("A's rows overlap (row stride smaller than N)")
-    lda = max(A.stride(-2), N, 1) if M > 1 else max(N, 1)
-    strideA = A.stride(0) if batched else 0
-    out_t = _OUT[A.dtype]
+    lda = max(strides[-2], N, 1) if M > 1 else max(N, 1)
     shape_q = (Bn, M) if batched else (M,)
     shape_s = (Bn, N) if batched else (N,)
     if q is None:
         q = torch.empty(shape_q, dtype=out_t, device=A.device)
+    elif q.dtype != out_t or tuple(q.shape) != shape_q:
+        raise ValueError(f"q must be {out_t} of shape {shape_q}")
     if s is None:
         s = torch.empty(shape_s, dtype=out_t, device=A.device)
-    if q.dtype != out_t or s.dtype != out_t:
-        raise ValueError(f"outputs must be {out_t}")
-    if tuple(q.shape) != shape_q or tuple(s.shape) != shape_s:
-        raise ValueError("output shapes do not match")
-    strm = stream if stream is not None else torch.cuda.current_stream(A.device)
-    h = strm.cuda_stream
-    tag = _TAG[A.dtype]
-    with torch.cuda.device(A.device):
-        if batched:
-            sP = _vec_stride(p, N, Bn, "p")
-            sR = _vec_stride(r, M, Bn, "r")
-            sQ = _vec_stride(q, M, Bn, "q") if q.dim() == 2 else M
-            sS = _vec_stride(s, N, Bn, "s") if s.dim() == 2 else N
-            fn = getattr(B, f"dualmv_{tag}_strided_batched")
-            rc = fn(M, N, A.data_ptr(), lda, strideA, p.data_ptr(), sP, r.data_ptr(), sR,
-                    q.data_ptr(), sQ, s.data_ptr(), sS, Bn, h)
-        else:
-            _vec_stride(p, N, 1, "p")
-            _vec_stride(r, M, 1, "r")
-            if not (q.is_contiguous() and s.is_contiguous()):
-                raise ValueError("q and s must be contiguous")
-            fn = getattr(B, f"dualmv_{tag}")
-            rc = fn(M, N, A.data_ptr(), lda, p.data_ptr(), r.data_ptr(), q.data_ptr(),
-                    s.data_ptr(), h)
+    elif s.dtype != out_t or tuple(s.shape) != shape_s:
+        raise ValueError(f"s must be {out_t} of shape {shape_s}")
+    if batched:
+        sP = _vec_stride(p, N, Bn, "p")
+        sR = _vec_stride(r, M, Bn, "r")
+        sQ = _vec_stride(q, M, Bn, "q") if q.dim() == 2 else M
+        sS = _vec_stride(s, N, Bn, "s") if s.dim() == 2 else N
+        rc = _call_on(dev_idx, stream, fn_batched, M, N, A.data_ptr(), lda, strides[0],
+                      p.data_ptr(), sP, r.data_ptr(), sR, q.data_ptr(), sQ, s.data_ptr(), sS,
+                      Bn)
+    else:
+        if p.dim() != 1 or r.dim() != 1 or p.shape[0] != N or r.shape[0] != M or \
+                not (p.is_contiguous() and r.is_contiguous()):
+            raise ValueError(f"p and r must be contiguous vectors of lengths {N} and {M}")
+        if not (q.is_contiguous() and s.is_contiguous()):
+            raise ValueError("q and s must be contiguous")
+        rc = _call_on(dev_idx, stream, fn_single, M, N, A.data_ptr(), lda, p.data_ptr(),
+                      r.data_ptr(), q.data_ptr(), s.data_ptr())
     if rc != B.DUALMV_SUCCESS:
         raise B.DualmvError(rc, f"dualmv_{tag}")
     return q, s
@@ -103,8 +143,8 @@ def dualmv(A: torch.Tensor, p: torch.Tensor, r: torch.Tensor,
 
 def device_fault(stream: torch.cuda.Stream | None = None) -> int:
     """Synchronise ``stream`` and return (and clear) the device fault status."""
-    strm = stream if stream is not None else torch.cuda.current_stream()
-    return B.dualmv_device_fault(strm.cuda_stream)
+    h = _current_stream_handle(_get_device()) if stream is None else stream.cuda_stream
+    return B.dualmv_device_fault(h)
 
 
 def _matrix(A: torch.Tensor, name: str):
@@ -142,11 +182,8 @@ def gesummv(A: torch.Tensor, B: torch.Tensor, x: torch.Tensor, alpha: float = 1.
     if y is None:
         y = torch.empty(M, dtype=A.dtype, device=A.device)
     _vector(y, M, A, "y")
-    strm = stream if stream is not None else torch.cuda.current_stream(A.device)
-    with torch.cuda.device(A.device):
-        rc = getattr(B_, f"dualmv_gesummv_{tag}")(M, N, alpha, A.data_ptr(), lda, beta,
-                                                  B.data_ptr(), ldb, x.data_ptr(),
-                                                  y.data_ptr(), strm.cuda_stream)
+    rc = _call_on(A.get_device(), stream, getattr(B_, f"dualmv_gesummv_{tag}"), M, N, alpha,
+                  A.data_ptr(), lda, beta, B.data_ptr(), ldb, x.data_ptr(), y.data_ptr())
     if rc != B_.DUALMV_SUCCESS:
         raise B_.DualmvError(rc, f"dualmv_gesummv_{tag}")
     return y
@@ -163,10 +200,8 @@ def atax(A: torch.Tensor, x: torch.Tensor, y: torch.Tensor | None = None,
     if y is None:
         y = torch.empty(N, dtype=A.dtype, device=A.device)
     _vector(y, N, A, "y")
-    strm = stream if stream is not None else torch.cuda.current_stream(A.device)
-    with torch.cuda.device(A.device):
-        rc = getattr(B_, f"dualmv_atax_{tag}")(M, N, A.data_ptr(), lda, x.data_ptr(),
-                                               y.data_ptr(), strm.cuda_stream)
+    rc = _call_on(A.get_device(), stream, getattr(B_, f"dualmv_atax_{tag}"), M, N,
+                  A.data_ptr(), lda, x.data_ptr(), y.data_ptr())
     if rc != B_.DUALMV_SUCCESS:
         raise B_.DualmvError(rc, f"dualmv_atax_{tag}")
     return y
@@ -188,12 +223,10 @@ def gemver(A: torch.Tensor, u1: torch.Tensor, v1: torch.Tensor, u2: torch.Tensor
     for v, n, name in ((u1, M, "u1"), (u2, M, "u2"), (w, M, "w"), (y, M, "y"),
                        (v1, N, "v1"), (v2, N, "v2"), (x, N, "x"), (z, N, "z")):
         _vector(v, n, A, name)
-    strm = stream if stream is not None else torch.cuda.current_stream(A.device)
-    with torch.cuda.device(A.device):
-        rc = getattr(B_, f"dualmv_gemver_{tag}")(
-            M, N, alpha, beta, A.data_ptr(), lda, int(bool(update_A)), u1.data_ptr(),
-            v1.data_ptr(), u2.data_ptr(), v2.data_ptr(), w.data_ptr(), x.data_ptr(),
-            y.data_ptr(), z.data_ptr(), strm.cuda_stream)
+    rc = _call_on(A.get_device(), stream, getattr(B_, f"dualmv_gemver_{tag}"), M, N, alpha,
+                  beta, A.data_ptr(), lda, int(bool(update_A)), u1.data_ptr(), v1.data_ptr(),
+                  u2.data_ptr(), v2.data_ptr(), w.data_ptr(), x.data_ptr(), y.data_ptr(),
+                  z.data_ptr())
     if rc != B_.DUALMV_SUCCESS:
         raise B_.DualmvError(rc, f"dualmv_gemver_{tag}")
     return w, x

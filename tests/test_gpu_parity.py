@@ -249,3 +249,31 @@ def test_tma_and_direct_paths_agree_within_tolerance():
 
 def test_no_device_fault_recorded():
     assert dm.device_fault() == dm.DUALMV_SUCCESS
+
+
+def test_tensor_api_checks_its_arguments():
+    """The tensor entry point rejects what the C ABI cannot take, before
+    any launch, and accepts caller-provided outputs."""
+    A = torch.randn(64, 96, device="cuda:0")
+    p = torch.randn(96, device="cuda:0")
+    r = torch.randn(64, device="cuda:0")
+    with pytest.raises(ValueError):
+        dm.dualmv(A.cpu(), p.cpu(), r.cpu())                   # no CPU path
+    with pytest.raises(ValueError):
+        dm.dualmv(A, p.double(), r)                            # dtype mismatch
+    with pytest.raises(ValueError):
+        dm.dualmv(A, p, r, q=torch.empty(63, device="cuda:0"))  # q shape
+    with pytest.raises(ValueError):
+        dm.dualmv(A, p, r, q=torch.empty(64, device="cuda:0", dtype=torch.float64))
+    with pytest.raises(ValueError):
+        dm.dualmv(A.t(), r, p)                                 # not row-major
+    with pytest.raises(TypeError):
+        dm.dualmv(A.long(), p.long(), r.long())                # no int64 entry point
+    q = torch.empty(64, device="cuda:0")
+    s = torch.empty(96, device="cuda:0")
+    q2, s2 = dm.dualmv(A, p, r, q=q, s=s)
+    torch.cuda.synchronize()
+    assert q2 is q and s2 is s
+    An = A.double().cpu()
+    assert torch.allclose(q.double().cpu(), An @ p.double().cpu(), rtol=1e-4, atol=1e-4)
+    assert torch.allclose(s.double().cpu(), An.t() @ r.double().cpu(), rtol=1e-4, atol=1e-4)

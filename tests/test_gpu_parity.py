@@ -152,6 +152,23 @@ def test_rank_one_is_bit_exact(dtype, path):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "f64", "i32"])
+@pytest.mark.parametrize("M,N,pad", [(1000, 3000, 5), (4096, 2048, 0)])
+def test_power_of_two_scaling_is_bit_exact(dtype, M, N, pad, path):
+    """q(A, 2p, r) = 2 q and s(A, p, 4r) = 4 s bit for bit: binary scaling
+    commutes with every rounding (and with the double-float split) while
+    nothing overflows, and integer sums are exact.  Pins the GPU path
+    without the oracle."""
+    A, p, r = _make(dtype, M, N, N + pad, 21)
+    A = A[:, :N]
+    q, s = dm.dualmv(A, p, r)
+    q2, s1 = dm.dualmv(A, p * 2, r)
+    q1, s4 = dm.dualmv(A, p, r * 4)
+    torch.cuda.synchronize()
+    assert torch.equal(q2, q * 2) and torch.equal(s1, s)
+    assert torch.equal(s4, s * 4) and torch.equal(q1, q)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64", "i32"])
 def test_transpose_swaps_outputs(dtype):
     """dualmv(A^T, r, p) gives (s, q): the row and column paths agree."""
     M, N = 513, 1200

@@ -291,9 +291,13 @@ enum { DUALMV_DTYPE_F32 = 0, DUALMV_DTYPE_F64 = 1, DUALMV_DTYPE_I32 = 2 };
 enum {
     DUALMV_KERNEL_STREAM = 0, /* TMA ring, native arithmetic of the dtype  */
     DUALMV_KERNEL_F64E = 1,   /* TMA ring per warp, double-float fp64      */
-    DUALMV_KERNEL_WIDE = 2    /* int32: tiles of rows_per_warp rows by     */
+    DUALMV_KERNEL_WIDE = 2,   /* int32: tiles of rows_per_warp rows by     */
                               /* warps * 256 columns, one 256-column       */
                               /* sub-band per warp                         */
+    DUALMV_KERNEL_PHASED = 3, /* 4-byte rows whose stride or base is not   */
+                              /* 16-byte aligned: TMA through one pair of  */
+                              /* tensor maps per row phase (no variants)   */
+    DUALMV_KERNEL_PLAIN = 4   /* plain global loads (no variants)          */
 };
 typedef struct dualmv_variant_t {
     int32_t index;          /* position in its dtype's table              */
@@ -342,6 +346,14 @@ void dualmv_tune_clear(void);
  * problem, the plain-load path, a batched or single-sided call, or an
  * error).  Instrumentation for tests and benchmarks. */
 int32_t dualmv_last_variant(void);
+
+/* The kind of streaming kernel (DUALMV_KERNEL_*) that the calling thread's
+ * last dual product ran (dualmv_f32/f64/i32 and their strided-batched forms,
+ * and the passes inside GESUMMV, ATAX and GEMVER), or -1 if it ran none (an
+ * empty problem or an error).  PHASED: rows whose stride or base the TMA
+ * unit cannot take as one tensor, for one 4-byte dual product; PLAIN: the
+ * remaining unaligned cases.  Instrumentation for tests and benchmarks. */
+int32_t dualmv_last_kernel(void);
 
 /* Trimmed mean of Eq. 3: the R values sorted, the k smallest and k largest
  * dropped, the rest averaged.  DUALMV_ERR_INVALID_VALUE unless R > 2k,

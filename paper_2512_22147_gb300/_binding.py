@@ -38,6 +38,8 @@ DUALMV_DTYPE_I32 = 2
 DUALMV_KERNEL_STREAM = 0
 DUALMV_KERNEL_F64E = 1
 DUALMV_KERNEL_WIDE = 2
+DUALMV_KERNEL_PHASED = 3
+DUALMV_KERNEL_PLAIN = 4
 
 EXPORTED = (
     "dualmv_f32", "dualmv_f64", "dualmv_i32",
@@ -51,7 +53,7 @@ EXPORTED = (
     "dualmv_variant_count", "dualmv_variant_info", "dualmv_set_variant",
     "dualmv_tuned_variant", "dualmv_tune_clear", "dualmv_trimmed_mean",
     "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32", "dualmv_last_variant",
-    "dualmv_atax_set_two_pass", "dualmv_gemver_set_onthefly",
+    "dualmv_atax_set_two_pass", "dualmv_gemver_set_onthefly", "dualmv_last_kernel",
 )
 
 
@@ -153,6 +155,7 @@ def _load() -> ctypes.CDLL:
     lib.dualmv_tuned_variant.argtypes, lib.dualmv_tuned_variant.restype = [i32, i64, i64, i64], i32
     lib.dualmv_tune_clear.argtypes, lib.dualmv_tune_clear.restype = [], None
     lib.dualmv_last_variant.argtypes, lib.dualmv_last_variant.restype = [], i32
+    lib.dualmv_last_kernel.argtypes, lib.dualmv_last_kernel.restype = [], i32
     lib.dualmv_trimmed_mean.argtypes = [ctypes.POINTER(ctypes.c_double), i64, i64,
                                         ctypes.POINTER(ctypes.c_double)]
     lib.dualmv_trimmed_mean.restype = st
@@ -312,6 +315,11 @@ def dualmv_tune_clear() -> None:
 
 def dualmv_last_variant() -> int:
     return _lib.dualmv_last_variant()
+
+
+def dualmv_last_kernel() -> int:
+    """DUALMV_KERNEL_* of this thread's last dual product, or -1."""
+    return _lib.dualmv_last_kernel()
 
 
 def dualmv_trimmed_mean(times, k: int) -> float:

@@ -74,6 +74,7 @@ thread_local int g_last_cuda_error = 0;
 thread_local cudaEvent_t g_kernel_ev_start = nullptr;
 thread_local cudaEvent_t g_kernel_ev_stop = nullptr;
 thread_local int32_t g_last_variant = -1;
+thread_local int32_t g_last_kernel = -1;
 int g_path = DUALMV_PATH_AUTO;
 int g_atax_two_pass = 0;  // 1: ATAX always takes the two-pass path
 int g_gemver_onthefly = 0;  // 1: GEMVER applies the update element by element
@@ -217,6 +218,50 @@ bool encode_a_uncached(CUtensorMap *map, const T *A, int64_t M, int64_t N, int64
                      CU_TENSOR_MAP_SWIZZLE_NONE, promo,
                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return rc == CUDA_SUCCESS;
+}
+
+// Phased tensor maps for one problem whose row stride or base TMA cannot
+// take: NPH = 16 / gcd(lda * size, 16) phases (rows ph, ph + NPH, ...), each
+// a 2-D tensor of N + ph_off columns from its first row's start rounded down
+// to 16 bytes (ph_off elements before it), with row stride NPH * lda * size.
+// A band's box starts at the band's column (16-byte aligned in the tensor)
+// and so holds the row's columns shifted by ph_off; the small box after it
+// holds the ph_off columns pushed past it.  Columns past N + ph_off are out
+// of the tensor: no copy reads past a row's last element.  Returns the phase
+// count, or 0 when the shape does not fit this path.
+template <typename T>
+int encode_phased(dmv::TmapSet *maps, Params *prm, const T *A, int64_t M, int64_t N,
+                  int64_t lda, int tile_rows) {
+    constexpr int64_t es = sizeof(T);
+    const int64_t row_bytes = lda * es;
+    const int nph = row_bytes % 16 == 0 ? 1 : row_bytes % 8 == 0 ? 2 : 4;
+    if (reinterpret_cast<uintptr_t>(A) % es != 0 || (int64_t)nph * row_bytes % 16 != 0 ||
+        M < nph || N < 1 || M >= INT32_MAX || N >= INT32_MAX - 16 || tile_rows % nph != 0)
+        return 0;
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return 0;
+    for (int ph = 0; ph < nph; ++ph) {
+        const uintptr_t addr = reinterpret_cast<uintptr_t>(A + ph * lda);
+        const uintptr_t base = addr & ~(uintptr_t)15;
+        const int64_t off = (int64_t)(addr - base) / es;
+        const int64_t rows = (M - ph + nph - 1) / nph;
+        cuuint64_t dims[2] = {(cuuint64_t)(N + off), (cuuint64_t)rows};
+        cuuint64_t strides[1] = {(cuuint64_t)(nph * row_bytes)};
+        cuuint32_t estr[2] = {1u, 1u};
+        for (int k = 0; k < 2; ++k) {
+            cuuint32_t box[2] = {(cuuint32_t)(k == 0 ? kBandCols : 16 / es),
+                                 (cuuint32_t)(tile_rows / nph)};
+            CUresult rc = fn(&maps->m[2 * ph + k], tma_dtype<T>(), 2u,
+                             reinterpret_cast<void *>(base), dims, strides, box, estr,
+                             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+            if (rc != CUDA_SUCCESS) return 0;
+        }
+        prm->ph_off[ph] = (int32_t)off;
+    }
+    prm->ph_n = nph;
+    return nph;
 }
 
 // ------------------------------------------------------------------ plan --
@@ -434,6 +479,44 @@ cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualm
                                 (size_t)pl.smem_bytes, stream, map, prm);
     kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(map, prm);
     return cudaGetLastError();
+}
+
+template <typename T, int NPH>
+Geometry phased_geometry_n() {
+    Geometry g = stream_geometry<T, kWarps, default_rpw<T>(), kStages>(true);
+    g.smem = dmv::SmemLayout<T, kWarps, default_rpw<T>(), kStages, true, NPH>::kTotal;
+    return g;
+}
+template <typename T>
+Geometry phased_geometry(int nph) {
+    return nph == 1 ? phased_geometry_n<T, 1>()
+                    : nph == 2 ? phased_geometry_n<T, 2>() : phased_geometry_n<T, 4>();
+}
+
+template <typename T, int NPH>
+cudaError_t launch_phased_n(const dmv::TmapSet &maps, const Params &prm, const dualmv_plan_t &pl,
+                            int dev, cudaStream_t stream) {
+    constexpr auto kern =
+        dmv::dualmv_stream_phased_kernel<T, kWarps, default_rpw<T>(), kStages, NPH>;
+    cudaError_t e = smem_opt_in<kern>(pl.smem_bytes, dev);
+    if (e != cudaSuccess) return e;
+    if constexpr (std::is_same<T, int32_t>::value)  // after the zeroing kernel
+        return launch_dependent(kern, dim3((unsigned)pl.grid), dim3((unsigned)pl.threads),
+                                (size_t)pl.smem_bytes, stream, maps, prm);
+    kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(maps, prm);
+    return cudaGetLastError();
+}
+template <typename T>
+cudaError_t launch_phased(int nph, const dmv::TmapSet &maps, const Params &prm,
+                          const dualmv_plan_t &pl, int dev, cudaStream_t stream) {
+    if constexpr (sizeof(T) == 4) {  // 4-byte elements: 4 rows a warp, up to 4 phases
+        switch (nph) {
+        case 1: return launch_phased_n<T, 1>(maps, prm, pl, dev, stream);
+        case 2: return launch_phased_n<T, 2>(maps, prm, pl, dev, stream);
+        case 4: return launch_phased_n<T, 4>(maps, prm, pl, dev, stream);
+        }
+    }
+    return cudaErrorInvalidValue;
 }
 
 template <int W, int RPW, int S>
@@ -730,6 +813,7 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     if (rank2 != nullptr && outputs == dmv::kOutBoth) return DUALMV_ERR_UNSUPPORTED;
     const bool want_q = (outputs & dmv::kOutQ) != 0, want_s = (outputs & dmv::kOutS) != 0;
     g_last_variant = -1;
+    g_last_kernel = -1;
     dualmv_status st = validate(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ,
                                 s, strideS, batch, outputs);
     if (st != DUALMV_SUCCESS || batch == 0) return st;
@@ -797,8 +881,25 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
         }
     }
 
+    // Rows the TMA unit cannot take as one tensor (row stride or base not
+    // 16-byte aligned): phased tensor maps, for one 4-byte dual product.
+    dmv::TmapSet pmaps;
+    Params pinfo;
+    std::memset(&pinfo, 0, sizeof pinfo);
+    pinfo.ph_n = 1;
+    int nph = 0;
+    if (kind == Kind::kDirect && g_path != DUALMV_PATH_DIRECT && es == 4 && !three_d &&
+        rank2 == nullptr && outputs == dmv::kOutBoth) {
+        std::memset(&pmaps, 0, sizeof pmaps);
+        nph = encode_phased<T>(&pmaps, &pinfo, A, M, N, lda,
+                               (int)stream_geometry<T, kWarps, default_rpw<T>(), kStages>(true)
+                                   .tile_rows);
+    }
+
     dualmv_plan_t pl;
     st = var ? make_plan_geo(M, N, batch, es, sizeof(Acc), ds->sms, var->geo, &pl)
+         : nph > 0
+             ? make_plan_geo(M, N, batch, es, sizeof(Acc), ds->sms, phased_geometry<T>(nph), &pl)
              : make_plan(M, N, batch, es, sizeof(Acc),
                          (int64_t)ds->sms * (tma ? 1 : kDirectCtasPerSm), kind, &pl);
     if (st != DUALMV_SUCCESS) return st;
@@ -815,6 +916,9 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
         }
     }
     Params prm;
+    std::memset(&prm, 0, sizeof prm);
+    prm.ph_n = pinfo.ph_n;
+    for (int ph = 0; ph < dmv::kMaxPhases; ++ph) prm.ph_off[ph] = pinfo.ph_off[ph];
     prm.A = A; prm.lda = lda; prm.strideA = strideA;
     prm.p = p; prm.strideP = strideP;
     prm.r = r; prm.strideR = strideR;
@@ -849,6 +953,12 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     cudaEvent_t ev_start = g_kernel_ev_start, ev_stop = g_kernel_ev_stop;
     g_kernel_ev_start = g_kernel_ev_stop = nullptr;
     e = ev_start ? cudaEventRecord(ev_start, stream) : cudaSuccess;
+    // The kind of streaming kernel this call launches (dualmv_last_kernel).
+    const int32_t kernel_kind = var != nullptr         ? var->info.kernel
+                                : nph > 0              ? (int32_t)DUALMV_KERNEL_PHASED
+                                : kind == Kind::kF64e  ? (int32_t)DUALMV_KERNEL_F64E
+                                : kind == Kind::kTma   ? (int32_t)DUALMV_KERNEL_STREAM
+                                                       : (int32_t)DUALMV_KERNEL_PLAIN;
     if (e == cudaSuccess) {
         if (var != nullptr) {
             e = var->launch(map, prm, pl, dev, stream);
@@ -890,10 +1000,13 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
             // native fp64 default kernel is no entry of it.
             if (e == cudaSuccess && !three_d && !std::is_same<T, double>::value)
                 g_last_variant = 0;
+        } else if (nph > 0) {
+            e = launch_phased<T>(nph, pmaps, prm, pl, dev, stream);
         } else {
             e = launch_stream<T, false, false>(map, prm, pl, dev, stream);
         }
     }
+    if (e == cudaSuccess) g_last_kernel = kernel_kind;
     if (e == cudaSuccess && ev_stop) e = cudaEventRecord(ev_stop, stream);
     if (e == cudaSuccess && !kAtomicOut) e = launch_combine<Acc>(prm, stream);
     cudaError_t ef = ws ? cudaFreeAsync(ws, stream) : cudaSuccess;
@@ -1592,6 +1705,8 @@ dualmv_status run_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,
     // Every scratch word the combine kernel reads is written earlier in the
     // same call, so nothing needs clearing between calls.
     Params prm;
+    std::memset(&prm, 0, sizeof prm);
+    prm.ph_n = 1;
     prm.A = A; prm.lda = lda; prm.strideA = M * lda;
     prm.p = p; prm.strideP = N;
     prm.r = r; prm.strideR = M;
@@ -1803,6 +1918,8 @@ int32_t dualmv_tuned_variant(int32_t dtype, int64_t M, int64_t N, int64_t lda) {
 }
 
 int32_t dualmv_last_variant(void) { return g_last_variant; }
+
+int32_t dualmv_last_kernel(void) { return g_last_kernel; }
 
 void dualmv_tune_clear(void) {
     std::lock_guard<std::mutex> lk(g_tuned_mu);

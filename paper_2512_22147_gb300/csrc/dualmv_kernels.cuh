@@ -286,6 +286,20 @@ struct Params {
     int64_t bands, stripes, tiles, grid, max_seg;
     void *q_ws;  // [batch][bands][M] band partials of q (bands > 1 only)
     void *s_ws;  // [grid][max_seg][kBandCols] segment partials of s
+    // Rows whose stride (or base) is not 16-byte aligned, read through tensor
+    // maps per row phase (dualmv_stream_phased_kernel): row r is in phase
+    // r % ph_n, and its columns start at element ph_off[phase] of its box
+    // row.  ph_n = 1 and zeros otherwise.
+    int32_t ph_n;
+    int32_t ph_off[4];
+};
+
+// Phased tensor maps: two per phase, over the same rows: m[2 ph] with
+// 256-column boxes, m[2 ph + 1] with 16-byte boxes (the columns that the
+// phase's offset pushes past the band's box).
+constexpr int kMaxPhases = 4;
+struct TmapSet {
+    CUtensorMap m[2 * kMaxPhases];
 };
 
 // First tile of CTA c, and the CTA that owns tile t (inverse of the split).
@@ -349,10 +363,13 @@ struct TileCursor32 {
     }
 };
 
-template <typename T, int W, int RPW, int STAGES, bool kTma>
+template <typename T, int W, int RPW, int STAGES, bool kTma, int NPH = 0>
 struct SmemLayout {
     using Acc = typename Traits<T>::Acc;
-    static constexpr int kTileBytes = W * RPW * kBandCols * (int)sizeof(T);
+    // NPH > 0 (phased maps): a tile row is the band's box row (1 KiB for
+    // 4-byte elements) plus 16 bytes from the small box.
+    static constexpr int kRowBytes = kBandCols * (int)sizeof(T);
+    static constexpr int kTileBytes = W * RPW * (kRowBytes + (NPH > 0 ? 16 : 0));
     static constexpr int kAlign = kTma ? 1024 : 16;
     static constexpr int kRing = kTma ? STAGES * kTileBytes : 0;
     static constexpr int kScratch = W * kBandCols * (int)sizeof(Acc);
@@ -370,11 +387,11 @@ struct SmemLayout {
 // with warps.  Its int32 form (64-bit sums) would otherwise take 168
 // registers and one CTA per SM; it asks for two (128 registers), as the
 // float forms get by themselves.
-template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d,
-          int kOut = kOutBoth, bool kRank2 = false>
-__global__ void __launch_bounds__((W + (kTma ? 1 : 0)) * 32,
-                                  (!kTma && std::is_same<T, int32_t>::value) ? 2 : 1)
-dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
+// The kernel body, shared by dualmv_stream_kernel (one tensor map, NPH = 0)
+// and dualmv_stream_phased_kernel (NPH phase maps, tmaps[0 .. NPH - 1]).
+template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d, int kOut,
+          bool kRank2, int NPH>
+__device__ __forceinline__ void stream_body(const CUtensorMap *tmaps, const Params &prm) {
     using Acc = typename Traits<T>::Acc;
     static_assert(!kRank2 || !std::is_same<T, int32_t>::value, "rank-2 update: floats only");
     constexpr bool kQ = (kOut & kOutQ) != 0;  // row sums q = A p
@@ -390,10 +407,17 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
     constexpr int VE = Traits<T>::kVecElems;
     constexpr int VPL = kLaneCols / VE;  // 16-byte vectors per lane per row
     constexpr int BM = W * RPW;
-    constexpr int ROW_BYTES = kBandCols * (int)sizeof(T);
-    constexpr int TILE_BYTES = BM * ROW_BYTES;
-    using L = SmemLayout<T, W, RPW, STAGES, kTma>;
-    static_assert(L::kTileBytes == TILE_BYTES, "tile size mismatch");
+    using L = SmemLayout<T, W, RPW, STAGES, kTma, NPH>;
+    constexpr int ROW_BYTES = L::kRowBytes;  // smem pitch of a tile row (the band's box)
+    constexpr int TILE_BYTES = L::kTileBytes;
+    static_assert(NPH == 0 || (kTma && !kBatched3d && !kRank2 && RPW % NPH == 0 &&
+                               BM % NPH == 0 && NPH <= kMaxPhases),
+                  "phased maps: one unbatched problem, each warp's rows in whole phase groups");
+    // Phased maps: per phase, the band's box (BM / NPH rows of ROW_BYTES) and
+    // then the small box (BM / NPH rows of 16 bytes).
+    constexpr int PH = NPH > 0 ? NPH : 1;
+    constexpr int PHASE_ROWS = BM / PH;
+    constexpr int PHASE_BYTES = PHASE_ROWS * (ROW_BYTES + 16);
 
     extern __shared__ unsigned char smem_raw[];
     unsigned char *smem = smem_raw + shared_align_pad<L::kAlign>(smem_raw);
@@ -446,10 +470,21 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
                     mbar_arrive_expect_tx(fb, TILE_BYTES);
                     const uint32_t dst = smem_u32(ring + (size_t)stage * TILE_BYTES);
                     const int x = (int)(cur.band * kBandCols), y = (int)(cur.stripe * BM);
-                    if constexpr (kBatched3d)
-                        tma_load_3d(dst, &tmap, x, y, (int)cur.b, fb, pol);
-                    else
-                        tma_load_2d(dst, &tmap, x, y, fb, pol);
+                    if constexpr (NPH > 0) {
+                        // Per phase: the band's columns of its BM / NPH rows
+                        // (shifted by the phase's offset) and the 16 bytes after.
+#pragma unroll
+                        for (int ph = 0; ph < NPH; ++ph) {
+                            const uint32_t d = dst + (uint32_t)(ph * PHASE_BYTES);
+                            tma_load_2d(d, &tmaps[2 * ph], x, y / NPH, fb, pol);
+                            tma_load_2d(d + (uint32_t)(PHASE_ROWS * ROW_BYTES), &tmaps[2 * ph + 1],
+                                        x + kBandCols, y / NPH, fb, pol);
+                        }
+                    } else if constexpr (kBatched3d) {
+                        tma_load_3d(dst, &tmaps[0], x, y, (int)cur.b, fb, pol);
+                    } else {
+                        tma_load_2d(dst, &tmaps[0], x, y, fb, pol);
+                    }
                     issued = k + 1;
                     cur.advance(S, prm.bands);
                     if (++stage == STAGES) {
@@ -561,7 +596,43 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
 #pragma unroll
         for (int i = 0; i < RPW; ++i) {
             Vec a[VPL];
-            if constexpr (kTma) {
+            if constexpr (NPH > 0) {
+                // Tile row warp * RPW + i: phase i % NPH (RPW is a multiple of
+                // NPH), row (warp * RPW + i) / NPH of that phase's box, its
+                // columns from element ph_off of the box row.
+                const int ph = i % PH;
+                const int off = prm.ph_off[ph];
+                // The box row (16-byte aligned); the row's element j is at box
+                // position j + off, off < VE.
+                const int prow = (warp * RPW + i) / PH;
+                const unsigned char *phb = ring + (size_t)stage * TILE_BYTES + (size_t)ph * PHASE_BYTES;
+                const Vec *boxrow = reinterpret_cast<const Vec *>(phb + (size_t)prow * ROW_BYTES);
+                if (off == 0) {
+#pragma unroll
+                    for (int v = 0; v < VPL; ++v) a[v] = boxrow[v * 32 + lane];
+                } else {
+                    // Lane l's vector v is the tail of aligned vector v * 32 + l
+                    // and the head of the next one (lane 31's last: the row's 16
+                    // bytes of the small box).  Both are read as aligned 16-byte
+                    // vectors (consecutive lanes, consecutive vectors: no bank
+                    // conflicts), and the row's elements picked from them.
+                    const Vec *tailrow = reinterpret_cast<const Vec *>(
+                        phb + (size_t)PHASE_ROWS * ROW_BYTES + (size_t)prow * 16);
+#pragma unroll
+                    for (int v = 0; v < VPL; ++v) {
+                        const Vec cur = boxrow[v * 32 + lane];
+                        const Vec nxt = (v == VPL - 1 && lane == 31) ? *tailrow
+                                                                     : boxrow[v * 32 + lane + 1];
+                        if constexpr (VE == 4) {
+                            if (off == 1) a[v] = Vec{cur.y, cur.z, cur.w, nxt.x};
+                            else if (off == 2) a[v] = Vec{cur.z, cur.w, nxt.x, nxt.y};
+                            else a[v] = Vec{cur.w, nxt.x, nxt.y, nxt.z};
+                        } else {
+                            a[v] = Vec{cur.y, nxt.x};
+                        }
+                    }
+                }
+            } else if constexpr (kTma) {
                 const Vec *rowp = reinterpret_cast<const Vec *>(
                     ring + (size_t)stage * TILE_BYTES +
                     (size_t)(warp * RPW + i) * ROW_BYTES);
@@ -696,6 +767,25 @@ dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm)
             }
         }
     }
+}
+
+template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d,
+          int kOut = kOutBoth, bool kRank2 = false>
+__global__ void __launch_bounds__((W + (kTma ? 1 : 0)) * 32,
+                                  (!kTma && std::is_same<T, int32_t>::value) ? 2 : 1)
+dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
+    stream_body<T, W, RPW, STAGES, kTma, kBatched3d, kOut, kRank2, 0>(&tmap, prm);
+}
+
+// The same kernel for one problem whose row stride or base is not 16-byte
+// aligned (the TMA unit cannot take it as one 2-D tensor): row phase ph (rows
+// r = ph mod NPH) is its own 2-D tensor with the base rounded down to 16
+// bytes, so that its row stride NPH * lda * size is a multiple of 16 bytes.
+// NPH = 1 covers an unaligned base alone.
+template <typename T, int W, int RPW, int STAGES, int NPH>
+__global__ void __launch_bounds__((W + 1) * 32, 1)
+dualmv_stream_phased_kernel(const __grid_constant__ TmapSet maps, const Params prm) {
+    stream_body<T, W, RPW, STAGES, true, false, kOutBoth, false, NPH>(maps.m, prm);
 }
 
 // --------------------------------------------------------- combine kernel --

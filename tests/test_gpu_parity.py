@@ -294,3 +294,45 @@ def test_tensor_api_checks_its_arguments():
     An = A.double().cpu()
     assert torch.allclose(q.double().cpu(), An @ p.double().cpu(), rtol=1e-4, atol=1e-4)
     assert torch.allclose(s.double().cpu(), An.t() @ r.double().cpu(), rtol=1e-4, atol=1e-4)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "i32"])
+@pytest.mark.parametrize("lda_mod4", [1, 2, 3, 0])
+@pytest.mark.parametrize("base", [0, 1, 2, 3])
+def test_unaligned_rows_take_phased_maps(dtype, lda_mod4, base):
+    """Rows whose stride or base is not 16-byte aligned go through one pair
+    of tensor maps per row phase (lda odd: 4 phases, lda = 2 mod 4: 2,
+    base alone: 1).  Ragged M and N, N below one band, and fewer rows than
+    phases (which fall back to plain loads) all match the oracle."""
+    for M, N in ((67, 517), (130, 250), (5, 1030), (33, 256), (3, 300)):
+        lda = N + (lda_mod4 - N) % 4
+        A, p, r = _make(dtype, M, N, lda, 91 + 7 * lda_mod4 + base)
+        store = torch.empty(M * lda + base + 8, dtype=A.dtype, device=DEV)
+        view = store[base:base + M * lda].view(M, lda)
+        view.copy_(A)
+        run_and_compare(view, p, r, N)
+        nph = 1 if lda % 4 == 0 else 2 if lda % 2 == 0 else 4
+        kind = dm.dualmv_last_kernel()
+        if lda % 4 == 0 and base == 0:
+            assert kind in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_WIDE)
+        elif M >= nph:
+            assert kind == dm.DUALMV_KERNEL_PHASED, (M, N, lda, base, kind)
+        else:
+            assert kind == dm.DUALMV_KERNEL_PLAIN
+
+
+def test_last_kernel_reports_each_path():
+    A, p, r = _make("f64", 96, 512, 512, 92)
+    dm.dualmv(A, p, r)
+    assert dm.dualmv_last_kernel() == dm.DUALMV_KERNEL_F64E
+    old = dm.dualmv_set_path(dm.DUALMV_PATH_DIRECT)
+    try:
+        dm.dualmv(A, p, r)
+        assert dm.dualmv_last_kernel() == dm.DUALMV_KERNEL_PLAIN
+    finally:
+        dm.dualmv_set_path(old)
+    A, p, r = _make("f32", 96, 512, 512, 93)
+    dm.dualmv(A, p, r)
+    assert dm.dualmv_last_kernel() == dm.DUALMV_KERNEL_STREAM
+    dm.dualmv(A[:0], p, r[:0])
+    assert dm.dualmv_last_kernel() == -1

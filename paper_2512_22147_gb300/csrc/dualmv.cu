@@ -481,6 +481,24 @@ cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualm
     return cudaGetLastError();
 }
 
+template <int NPH>
+Geometry f64e_phased_geometry_n() {
+    Geometry g = f64e_geometry<kF64eWarps, kF64eRpw, kF64eStages>();
+    g.smem = dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand, NPH>::kTotal;
+    return g;
+}
+
+template <int NPH>
+cudaError_t launch_f64e_phased_n(const dmv::TmapSet &maps, const Params &prm,
+                                 const dualmv_plan_t &pl, int dev, cudaStream_t stream) {
+    constexpr auto kern =
+        dmv::dualmv_stream_f64e_phased_kernel<kF64eWarps, kF64eRpw, kF64eStages, NPH>;
+    cudaError_t e = smem_opt_in<kern>(pl.smem_bytes, dev);
+    if (e != cudaSuccess) return e;
+    return launch_dependent(kern, dim3((unsigned)pl.grid), dim3((unsigned)pl.threads),
+                            (size_t)pl.smem_bytes, stream, maps, prm);
+}
+
 template <typename T, int NPH>
 Geometry phased_geometry_n() {
     Geometry g = stream_geometry<T, kWarps, default_rpw<T>(), kStages>(true);
@@ -489,6 +507,8 @@ Geometry phased_geometry_n() {
 }
 template <typename T>
 Geometry phased_geometry(int nph) {
+    if constexpr (sizeof(T) == 8)  // the double-float kernel's layout
+        return nph == 1 ? f64e_phased_geometry_n<1>() : f64e_phased_geometry_n<2>();
     return nph == 1 ? phased_geometry_n<T, 1>()
                     : nph == 2 ? phased_geometry_n<T, 2>() : phased_geometry_n<T, 4>();
 }
@@ -514,6 +534,11 @@ cudaError_t launch_phased(int nph, const dmv::TmapSet &maps, const Params &prm,
         case 1: return launch_phased_n<T, 1>(maps, prm, pl, dev, stream);
         case 2: return launch_phased_n<T, 2>(maps, prm, pl, dev, stream);
         case 4: return launch_phased_n<T, 4>(maps, prm, pl, dev, stream);
+        }
+    } else {  // fp64: the double-float kernel, up to 2 phases
+        switch (nph) {
+        case 1: return launch_f64e_phased_n<1>(maps, prm, pl, dev, stream);
+        case 2: return launch_f64e_phased_n<2>(maps, prm, pl, dev, stream);
         }
     }
     return cudaErrorInvalidValue;
@@ -888,12 +913,16 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     std::memset(&pinfo, 0, sizeof pinfo);
     pinfo.ph_n = 1;
     int nph = 0;
-    if (kind == Kind::kDirect && g_path != DUALMV_PATH_DIRECT && es == 4 && !three_d &&
-        rank2 == nullptr && outputs == dmv::kOutBoth) {
+    if (kind == Kind::kDirect && g_path != DUALMV_PATH_DIRECT && !three_d &&
+        rank2 == nullptr && outputs == dmv::kOutBoth &&
+        (es == 4 || g_path != DUALMV_PATH_TMA_NATIVE_F64)) {
         std::memset(&pmaps, 0, sizeof pmaps);
-        nph = encode_phased<T>(&pmaps, &pinfo, A, M, N, lda,
-                               (int)stream_geometry<T, kWarps, default_rpw<T>(), kStages>(true)
-                                   .tile_rows);
+        // Box rows: a tile's rows of one phase (4-byte kernel), or a warp's
+        // (the self-loading fp64 kernel).
+        const int box_rows = es == 8 ? kF64eRpw
+                                     : (int)stream_geometry<T, kWarps, default_rpw<T>(), kStages>(
+                                           true).tile_rows;
+        nph = encode_phased<T>(&pmaps, &pinfo, A, M, N, lda, box_rows);
     }
 
     dualmv_plan_t pl;

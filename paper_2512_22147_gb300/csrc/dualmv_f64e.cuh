@@ -250,9 +250,17 @@ __device__ __forceinline__ void warp_rows_reduce_df_perm(DF (&v)[RPW]) {
 // their own rows and drift apart instead of finishing every tile together;
 // then the warp scratch for the s flush and one full/empty mbarrier pair
 // per (warp, stage).
-template <int W, int RPW, int STAGES, int BAND>
+template <int W, int RPW, int STAGES, int BAND, int NPH = 0>
 struct F64eLayout {
-    static constexpr int kBoxBytes = RPW * BAND * (int)sizeof(double);
+    // NPH > 0 (phased maps): per phase, its RPW / NPH rows of the band's box
+    // and then their 16 bytes each from the small box, padded to 128 bytes
+    // so that every copy's destination stays 128-byte aligned.  kBoxTx is
+    // what a warp's copies deliver, kBoxBytes the slot they land in.
+    static constexpr int kPhRows = NPH > 0 ? RPW / NPH : RPW;
+    static_assert(kPhRows * 16 <= 128, "small boxes of a phase exceed their pad");
+    static constexpr int kPhBytes = kPhRows * BAND * (int)sizeof(double) + (NPH > 0 ? 128 : 0);
+    static constexpr int kBoxBytes = (NPH > 0 ? NPH : 1) * kPhBytes;
+    static constexpr int kBoxTx = RPW * (BAND * (int)sizeof(double) + (NPH > 0 ? 16 : 0));
     static constexpr int kAlign = 1024;
     static constexpr int kRing = W * STAGES * kBoxBytes;
     static constexpr int kScratch = W * BAND * (int)sizeof(double);
@@ -268,10 +276,12 @@ struct F64eLayout {
 // warp's boxes, refilling a stage as soon as the warp has consumed it.
 // kPack: the double-float arithmetic of each lane's two adjacent columns
 // runs as packed pairs (no native columns).
-template <int W, int RPW, int STAGES, int BAND, bool kBatched3d, int kOut = kOutBoth,
-          int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = false, bool kPack = false>
-__global__ void __launch_bounds__((W + (kSelf ? 0 : 1)) * 32, 1)
-dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
+// The kernel body, shared by dualmv_stream_f64e_kernel (one tensor map,
+// NPH = 0) and dualmv_stream_f64e_phased_kernel (a pair of maps per row
+// phase, tmaps[0 .. 2 NPH - 1]; see dualmv_stream_phased_kernel).
+template <int W, int RPW, int STAGES, int BAND, bool kBatched3d, int kOut, int NC, bool kSelf,
+          bool kPack, int NPH>
+__device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params &prm) {
     constexpr bool kQ = (kOut & kOutQ) != 0;  // row sums q = A p
     constexpr bool kS = (kOut & kOutS) != 0;  // column sums s = A^T r
     using T = double;
@@ -282,10 +292,15 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     constexpr int VPL = LANE_COLS / VE;   // 16-byte vectors per lane per row
     constexpr int BM = W * RPW;
     constexpr int ROW_BYTES = BAND * (int)sizeof(T);
-    using L = F64eLayout<W, RPW, STAGES, BAND>;
+    using L = F64eLayout<W, RPW, STAGES, BAND, NPH>;
     static_assert(LANE_COLS == 4 || LANE_COLS == 8, "band of 128 or 256 columns");
     constexpr int BOX_BYTES = L::kBoxBytes;
-    static_assert(BOX_BYTES == RPW * ROW_BYTES, "box size mismatch");
+    static_assert(NPH == 0 || (kSelf && !kBatched3d && RPW % NPH == 0 && NPH <= 2),
+                  "phased maps: self-loading warps, one problem, whole phase groups");
+    // Phased maps: per phase, the band's box (PROWS rows) then the small box.
+    constexpr int PH = NPH > 0 ? NPH : 1;
+    constexpr int PROWS = RPW / PH;
+    constexpr int PH_BYTES = L::kPhBytes;
 
     extern __shared__ unsigned char smem_raw[];
     unsigned char *smem = smem_raw + shared_align_pad<L::kAlign>(smem_raw);
@@ -340,12 +355,12 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                         break;
                     }
                     const uint32_t fb = smem_u32(&full_bar[slot]);
-                    mbar_arrive_expect_tx(fb, BOX_BYTES);
+                    mbar_arrive_expect_tx(fb, L::kBoxTx);
                     const uint32_t dst = smem_u32(ring + (size_t)slot * BOX_BYTES);
                     if constexpr (kBatched3d)
-                        tma_load_3d(dst, &tmap, x, y + w * RPW, (int)cur.b, fb, pol);
+                        tma_load_3d(dst, &tmaps[0], x, y + w * RPW, (int)cur.b, fb, pol);
                     else
-                        tma_load_2d(dst, &tmap, x, y + w * RPW, fb, pol);
+                        tma_load_2d(dst, &tmaps[0], x, y + w * RPW, fb, pol);
                 }
                 if (!ok) break;
                 issued = k + 1;
@@ -429,13 +444,22 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
     auto issue = [&](int st) {
         const int slot_i = warp * STAGES + st;
         const uint32_t fb = smem_u32(&full_bar[slot_i]);
-        mbar_arrive_expect_tx(fb, BOX_BYTES);
+        mbar_arrive_expect_tx(fb, L::kBoxTx);
         const uint32_t dst = smem_u32(ring + (size_t)slot_i * BOX_BYTES);
         const int x = (int)(ld.band * BAND), y = (int)(ld.stripe * BM) + warp * RPW;
-        if constexpr (kBatched3d)
-            tma_load_3d(dst, &tmap, x, y, (int)ld.b, fb, pol);
-        else
-            tma_load_2d(dst, &tmap, x, y, fb, pol);
+        if constexpr (NPH > 0) {
+#pragma unroll
+            for (int ph = 0; ph < NPH; ++ph) {
+                const uint32_t d = dst + (uint32_t)(ph * PH_BYTES);
+                tma_load_2d(d, &tmaps[2 * ph], x, y / NPH, fb, pol);
+                tma_load_2d(d + (uint32_t)(PROWS * ROW_BYTES), &tmaps[2 * ph + 1], x + BAND,
+                            y / NPH, fb, pol);
+            }
+        } else if constexpr (kBatched3d) {
+            tma_load_3d(dst, &tmaps[0], x, y, (int)ld.b, fb, pol);
+        } else {
+            tma_load_2d(dst, &tmaps[0], x, y, fb, pol);
+        }
         ld.advance(S, NB);
         ++issued;
     };
@@ -510,7 +534,28 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             if (!ok) waited_to = k;
         }
         // This warp's RPW rows of the tile.
-        const Vec *tile = reinterpret_cast<const Vec *>(ring + (size_t)slot * BOX_BYTES);
+        const unsigned char *tileb = ring + (size_t)slot * BOX_BYTES;
+        // Vector v of row r of the box.  Phased maps: row r is row r / NPH of
+        // phase r % NPH, its columns start ph_off doubles into its box row; an
+        // offset row is read as aligned vectors, its own and the next (the
+        // last lane's last: the small box), and realigned.
+        auto rowvec = [&](int r, int v) -> Vec {
+            if constexpr (NPH == 0) {
+                return reinterpret_cast<const Vec *>(tileb + (size_t)r * ROW_BYTES)[v * 32 + lane];
+            } else {
+                const int ph = r % NPH, pr = r / NPH;
+                const unsigned char *phb = tileb + (size_t)ph * PH_BYTES;
+                const Vec *row = reinterpret_cast<const Vec *>(phb + (size_t)pr * ROW_BYTES);
+                const Vec cur = row[v * 32 + lane];
+                if ((ph == 0 ? prm.ph_off[0] : prm.ph_off[NPH - 1]) == 0) return cur;
+                const Vec nxt =
+                    (v == VPL - 1 && lane == 31)
+                        ? *reinterpret_cast<const Vec *>(phb + (size_t)PROWS * ROW_BYTES +
+                                                         (size_t)pr * 16)
+                        : row[v * 32 + lane + 1];
+                return Vec{cur.y, nxt.x};
+            }
+        };
 
         // Fast path: double-float arithmetic with a cheap range bound.
         DF q[RPW];
@@ -528,10 +573,9 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
 #pragma unroll
             for (int i = 0; i < RPW; ++i) {
                 const int ri = i ^ perm;
-                const Vec *rowp = tile + (size_t)ri * (ROW_BYTES / 16);
                 Vec a[VPL];
 #pragma unroll
-                for (int v = 0; v < VPL; ++v) a[v] = rowp[v * 32 + lane];
+                for (int v = 0; v < VPL; ++v) a[v] = rowvec(ri, v);
                 const float rh = __shfl_sync(0xffffffffu, rh_mine, ri);
                 const float rl = __shfl_sync(0xffffffffu, rl_mine, ri);
                 const float2 rh2 = make_float2(rh, rh), rl2 = make_float2(rl, rl);
@@ -571,10 +615,9 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
         } else {
 #pragma unroll
         for (int i = 0; i < RPW; ++i) {
-            const Vec *rowp = tile + (size_t)i * (ROW_BYTES / 16);
             Vec a[VPL];
 #pragma unroll
-            for (int v = 0; v < VPL; ++v) a[v] = rowp[v * 32 + lane];
+            for (int v = 0; v < VPL; ++v) a[v] = rowvec(i, v);
             const float rh = __shfl_sync(0xffffffffu, rh_mine, i);
             const float rl = __shfl_sync(0xffffffffu, rl_mine, i);
             const double rd = __shfl_sync(0xffffffffu, rmine, i);
@@ -621,10 +664,9 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             bool bad = false;
 #pragma unroll
             for (int i = 0; i < RPW; ++i) {
-                const Vec *rowp = tile + (size_t)i * (ROW_BYTES / 16);
 #pragma unroll
                 for (int v = 0; v < VPL; ++v) {
-                    const Vec av = rowp[v * 32 + lane];
+                    const Vec av = rowvec(i, v);
                     bad |= !f64e_in_range(av.x) || !f64e_in_range(av.y);
                 }
             }
@@ -675,12 +717,11 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
             for (int e = 0; e < LANE_COLS; ++e) td[e] = 0.0;
 #pragma unroll
             for (int i = 0; i < RPW; ++i) {
-                const Vec *rowp = tile + (size_t)i * (ROW_BYTES / 16);
                 const double ri = __shfl_sync(0xffffffffu, rmine, i);
                 double dot = 0.0;
 #pragma unroll
                 for (int v = 0; v < VPL; ++v) {
-                    const Vec av = rowp[v * 32 + lane];
+                    const Vec av = rowvec(i, v);
 #pragma unroll
                     for (int e = 0; e < VE; ++e) {
                         const double x = vget(av, e);
@@ -780,6 +821,21 @@ dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params
                 mbar_wait_bounded(smem_u32(&full_bar[warp * STAGES + (int)(kk % STAGES)]),
                                   (uint32_t)(kk / STAGES) & 1u);
     }
+}
+
+template <int W, int RPW, int STAGES, int BAND, bool kBatched3d, int kOut = kOutBoth,
+          int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = false, bool kPack = false>
+__global__ void __launch_bounds__((W + (kSelf ? 0 : 1)) * 32, 1)
+dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
+    f64e_body<W, RPW, STAGES, BAND, kBatched3d, kOut, NC, kSelf, kPack, 0>(&tmap, prm);
+}
+
+// fp64 rows whose stride or base is not 16-byte aligned (odd lda): the same
+// kernel reading through a pair of tensor maps per row phase.
+template <int W, int RPW, int STAGES, int NPH>
+__global__ void __launch_bounds__(W * 32, 1)
+dualmv_stream_f64e_phased_kernel(const __grid_constant__ TmapSet maps, const Params prm) {
+    f64e_body<W, RPW, STAGES, 256, false, kOutBoth, 0, true, true, NPH>(maps.m, prm);
 }
 
 }  // namespace dmv

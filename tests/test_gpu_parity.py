@@ -4,6 +4,8 @@ Every test here needs a GB300 and the built library.  Sizes span several
 tiles (256-column bands, 32- or 16-row stripes) with ragged tails; the five
 named workloads run at full size, in the launch configuration the benchmark
 times, and every output element is compared."""
+import math
+
 import numpy as np
 import pytest
 import torch
@@ -296,29 +298,59 @@ def test_tensor_api_checks_its_arguments():
     assert torch.allclose(s.double().cpu(), An.t() @ r.double().cpu(), rtol=1e-4, atol=1e-4)
 
 
-@pytest.mark.parametrize("dtype", ["f32", "i32"])
+@pytest.mark.parametrize("dtype", ["f32", "i32", "f64"])
 @pytest.mark.parametrize("lda_mod4", [1, 2, 3, 0])
 @pytest.mark.parametrize("base", [0, 1, 2, 3])
 def test_unaligned_rows_take_phased_maps(dtype, lda_mod4, base):
     """Rows whose stride or base is not 16-byte aligned go through one pair
-    of tensor maps per row phase (lda odd: 4 phases, lda = 2 mod 4: 2,
-    base alone: 1).  Ragged M and N, N below one band, and fewer rows than
+    of tensor maps per row phase (4-byte elements: lda odd gives 4 phases,
+    lda = 2 mod 4 gives 2, a base alone 1; 8-byte elements: lda odd gives 2,
+    a base alone 1).  Ragged M and N, N below one band, and fewer rows than
     phases (which fall back to plain loads) all match the oracle."""
-    for M, N in ((67, 517), (130, 250), (5, 1030), (33, 256), (3, 300)):
+    per16 = 2 if dtype == "f64" else 4          # elements per 16 bytes
+    for M, N in ((67, 517), (130, 250), (5, 1030), (33, 256), (3, 300), (1, 70)):
         lda = N + (lda_mod4 - N) % 4
         A, p, r = _make(dtype, M, N, lda, 91 + 7 * lda_mod4 + base)
         store = torch.empty(M * lda + base + 8, dtype=A.dtype, device=DEV)
         view = store[base:base + M * lda].view(M, lda)
         view.copy_(A)
         run_and_compare(view, p, r, N)
-        nph = 1 if lda % 4 == 0 else 2 if lda % 2 == 0 else 4
+        eff = lda if M > 1 else N                 # one row: the API passes lda = N
+        nph = per16 // math.gcd(eff, per16)
         kind = dm.dualmv_last_kernel()
-        if lda % 4 == 0 and base == 0:
-            assert kind in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_WIDE)
+        if eff % per16 == 0 and base % per16 == 0:
+            assert kind in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_WIDE,
+                            dm.DUALMV_KERNEL_F64E), (M, N, lda, base, kind)
         elif M >= nph:
             assert kind == dm.DUALMV_KERNEL_PHASED, (M, N, lda, base, kind)
         else:
             assert kind == dm.DUALMV_KERNEL_PLAIN
+
+
+def test_unaligned_f64_rows_keep_the_double_float_range_check():
+    """fp64 rows at an odd stride take the phased double-float kernel, whose
+    per-tile range check still sends tiles with huge, tiny or non-finite
+    entries to native fp64: the results match the oracle and every
+    non-finite value lands where it should."""
+    M, N = 150, 777
+    lda = N + 2                                   # odd: two row phases
+    A, p, r = _make("f64", M, N, lda, 95)
+    A[3, 5] = 1e60
+    A[70, 600] = 3e-200
+    A[100, 260] = 0.0
+    store = torch.empty(M * lda + 8, dtype=A.dtype, device=DEV)
+    view = store[1:1 + M * lda].view(M, lda)
+    view.copy_(A)
+    run_and_compare(view, p, r, N)
+    assert dm.dualmv_last_kernel() == dm.DUALMV_KERNEL_PHASED
+    view[40, 300] = float("inf")
+    q, s = dm.dualmv(view[:, :N], p, r)
+    torch.cuda.synchronize()
+    qc, sc = q.cpu(), s.cpu()
+    assert math.isinf(qc[40].item()) or math.isnan(qc[40].item())
+    assert torch.isfinite(torch.cat([qc[:40], qc[41:]])).all()
+    assert not math.isfinite(sc[300].item())
+    assert torch.isfinite(torch.cat([sc[:300], sc[301:]])).all()
 
 
 def test_last_kernel_reports_each_path():

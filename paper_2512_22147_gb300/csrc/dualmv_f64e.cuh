@@ -536,24 +536,26 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
         // This warp's RPW rows of the tile.
         const unsigned char *tileb = ring + (size_t)slot * BOX_BYTES;
         // Vector v of row r of the box.  Phased maps: row r is row r / NPH of
-        // phase r % NPH, its columns start ph_off doubles into its box row; an
-        // offset row is read as aligned vectors, its own and the next (the
-        // last lane's last: the small box), and realigned.
+        // phase r % NPH, its columns start ph_off doubles into its box row.
+        // An offset row is read as two 8-byte halves (the last lane's last
+        // upper half: the small box), which costs the shared-memory
+        // wavefronts of one aligned 16-byte vector.
         auto rowvec = [&](int r, int v) -> Vec {
             if constexpr (NPH == 0) {
                 return reinterpret_cast<const Vec *>(tileb + (size_t)r * ROW_BYTES)[v * 32 + lane];
             } else {
                 const int ph = r % NPH, pr = r / NPH;
                 const unsigned char *phb = tileb + (size_t)ph * PH_BYTES;
-                const Vec *row = reinterpret_cast<const Vec *>(phb + (size_t)pr * ROW_BYTES);
-                const Vec cur = row[v * 32 + lane];
-                if ((ph == 0 ? prm.ph_off[0] : prm.ph_off[NPH - 1]) == 0) return cur;
-                const Vec nxt =
+                const unsigned char *rowb = phb + (size_t)pr * ROW_BYTES;
+                if ((ph == 0 ? prm.ph_off[0] : prm.ph_off[NPH - 1]) == 0)
+                    return reinterpret_cast<const Vec *>(rowb)[v * 32 + lane];
+                const double *lo = reinterpret_cast<const double *>(rowb) + 2 * (v * 32 + lane) + 1;
+                const double *hi =
                     (v == VPL - 1 && lane == 31)
-                        ? *reinterpret_cast<const Vec *>(phb + (size_t)PROWS * ROW_BYTES +
-                                                         (size_t)pr * 16)
-                        : row[v * 32 + lane + 1];
-                return Vec{cur.y, nxt.x};
+                        ? reinterpret_cast<const double *>(phb + (size_t)PROWS * ROW_BYTES +
+                                                           (size_t)pr * 16)
+                        : lo + 1;
+                return Vec{*lo, *hi};
             }
         };
 

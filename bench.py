@@ -459,6 +459,12 @@ def run_native(args):
                       dm.DUALMV_KERNEL_WIDE: "dualmv_wide_i32_kernel"}[v.kernel]
             shape = (v.warps, v.rows_per_warp, v.stages)
             kernel_name = family + f"<warps {v.warps}, rows {v.rows_per_warp}, stages {v.stages}>"
+        else:  # rows TMA cannot take as one tensor, or a forced plain-load path
+            kernel_name = {
+                dm.DUALMV_KERNEL_PHASED: ("dualmv_stream_f64e_phased_kernel" if w.dtype == "f64"
+                                          else "dualmv_stream_phased_kernel"),
+                dm.DUALMV_KERNEL_PLAIN: "dualmv_stream_kernel (plain loads)",
+            }.get(dm.dualmv_last_kernel(), kernel_name)
     achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9
     traffic = recorded_traffic(args.workload, family, shape) if family else None
 

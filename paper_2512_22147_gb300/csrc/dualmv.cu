@@ -1125,7 +1125,7 @@ template <typename T>
 struct AtaxCfg;
 template <>
 struct AtaxCfg<float> {
-    static constexpr int W = kAtaxWarps, R = kAtaxRows, S = kAtaxStages;
+    static constexpr int W = kAtaxWarps, R = kAtaxRows, S = kAtaxStages, kBand = kBandCols;
     static constexpr int kThreads = W * 32;
     using L = dmv::AtaxLayout<W, R, S>;
     using Params = dmv::AtaxParams;
@@ -1141,16 +1141,19 @@ struct AtaxCfg<float> {
 #ifndef DUALMV_ATAX64_STAGES
 #define DUALMV_ATAX64_STAGES 3
 #endif
+#ifndef DUALMV_ATAX64_BAND
+#define DUALMV_ATAX64_BAND 256
+#endif
 template <>
 struct AtaxCfg<double> {
     // Three 8 KiB stages per warp (the column phase of a stripe runs one
     // stripe later) leave room for 8 warps.
     static constexpr int W = DUALMV_ATAX64_WARPS, R = DUALMV_ATAX64_ROWS,
-                         S = DUALMV_ATAX64_STAGES;
+                         S = DUALMV_ATAX64_STAGES, kBand = DUALMV_ATAX64_BAND;
     static constexpr int kThreads = (W + 1) * 32;  // and a control warp
-    using L = dmv::AtaxLayout64<W, R, S>;
+    using L = dmv::AtaxLayout64<W, R, S, kBand>;
     using Params = dmv::AtaxParams64;
-    static constexpr auto kern = dmv::atax_cluster_f64_kernel<W, R, S>;
+    static constexpr auto kern = dmv::atax_cluster_f64_kernel<W, R, S, kBand>;
     static void fill(Params &p, const double *A, int64_t lda) {
         p.A = A;
         p.lda = lda;
@@ -1172,7 +1175,7 @@ dualmv_status atax_cluster_run(int64_t M, int64_t N, const T *A, int64_t lda, co
     using L = typename Cfg::L;
     constexpr int kT = sizeof(T) == 8 ? 1 : 0;
     const int64_t es = sizeof(T);
-    const int64_t bands = (N + kBandCols - 1) / kBandCols;
+    const int64_t bands = (N + Cfg::kBand - 1) / Cfg::kBand;
     const int64_t C = (bands + Cfg::W - 1) / Cfg::W;
     if (g_path == DUALMV_PATH_DIRECT || C > dmv::kAtaxMaxCluster ||
         reinterpret_cast<uintptr_t>(A) % 16 != 0 || (lda * es) % 16 != 0 || M >= INT32_MAX ||
@@ -1219,7 +1222,7 @@ dualmv_status atax_cluster_run(int64_t M, int64_t N, const T *A, int64_t lda, co
     if (max_clusters <= 0) return DUALMV_SUCCESS;
     CUtensorMap map;
     std::memset(&map, 0, sizeof map);
-    if (!encode_a<T>(&map, A, M, N, lda, M * lda, 1, kBandCols, Cfg::R, false))
+    if (!encode_a<T>(&map, A, M, N, lda, M * lda, 1, Cfg::kBand, Cfg::R, false))
         return DUALMV_SUCCESS;
     const int64_t stripes = (M + Cfg::R - 1) / Cfg::R;
     const int64_t clusters = stripes < max_clusters ? stripes : max_clusters;

@@ -54,19 +54,19 @@ struct AtaxParams64 {
     int64_t M, N;
     int64_t stripes;   // ceil(M / R)
     int64_t clusters;  // clusters launched
-    int64_t bands;     // ceil(N / 256) sub-bands
+    int64_t bands;     // ceil(N / BAND) sub-bands
 };
 
-template <int W, int R, int STAGES>
+template <int W, int R, int STAGES, int BAND = kBandCols>
 struct AtaxLayout64 {
-    static constexpr int kBoxBytes = R * kBandCols * 8;  // one warp's sub-band, R rows
+    static constexpr int kBoxBytes = R * BAND * 8;  // one warp's sub-band, R rows
     static constexpr int kAlign = 1024;
     static constexpr int kRing = W * STAGES * kBoxBytes;
     static constexpr int kWarpPart = kAtaxSlots * W * R * 8;               // [slot][W][R] fp64
     static constexpr int kPart = kAtaxSlots * kAtaxMaxCluster * R * 8;     // [slot][C][R] fp64
     // [slot][R] t (fp64), [slot][R] its split (float2), [slot] out-of-range flag
     static constexpr int kT = kAtaxSlots * (R * 8 + R * 8 + 8);
-    static constexpr int kSeg = W * kBandCols * 8;                         // [W][256] fp64
+    static constexpr int kSeg = W * BAND * 8;                              // [W][BAND] fp64
     // full[W][STAGES], part[slot], wfull[slot], tready[slot]
     static constexpr int kBars = (W * STAGES + 3 * kAtaxSlots) * 8;
     static constexpr int kTotal = kAlign + kRing + kWarpPart + kPart + kT + kSeg + kBars;
@@ -78,15 +78,15 @@ __device__ __forceinline__ void st_async_f64(uint32_t raddr, double v, uint32_t 
                  ::"r"(raddr), "l"(__double_as_longlong(v)), "r"(rbar) : "memory");
 }
 
-template <int W, int R, int STAGES>
+template <int W, int R, int STAGES, int BAND = kBandCols>
 __global__ void __launch_bounds__((W + 1) * 32, 1)
 atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxParams64 prm) {
-    using L = AtaxLayout64<W, R, STAGES>;
+    using L = AtaxLayout64<W, R, STAGES, BAND>;
     using Vec = double2;
-    constexpr int VE = 2, LANE_COLS = kBandCols / 32, VPL = LANE_COLS / VE;
-    constexpr int ROW_BYTES = kBandCols * 8;
+    constexpr int VE = 2, LANE_COLS = BAND / 32, VPL = LANE_COLS / VE;
+    constexpr int ROW_BYTES = BAND * 8;
     static_assert(L::kBoxBytes == R * ROW_BYTES, "box size mismatch");
-    static_assert(VPL == 4, "the packed row tree sums four pairs");
+    static_assert(VPL == 2 || VPL == 4, "a sub-band of 128 or 256 columns");
     static_assert(kAtaxMaxCluster * R <= 64, "the control warp sends two values a lane");
 
     extern __shared__ unsigned char smem_raw[];
@@ -186,8 +186,8 @@ atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxPara
     // --------------------------------------------------- compute warps ----
     const int64_t sb = (int64_t)crank * W + warp;  // this warp's sub-band
     const bool live = sb < prm.bands;
-    const int64_t col0 = sb * kBandCols;
-    double *segp = segs + warp * kBandCols;  // this warp's fp64 column sums
+    const int64_t col0 = sb * BAND;
+    double *segp = segs + warp * BAND;  // this warp's fp64 column sums
 
     // x of this warp's columns, split once; its range checked once.
     float2 xh2[VPL], xl2[VPL];
@@ -278,7 +278,11 @@ atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxPara
                         reinterpret_cast<float4 *>(rowp)[v * 32 + lane] =
                             make_float4(ah0, ah1, al0, al1);
                     }
-                    const DF2 h = df_add2(df_add2(qp[0], qp[1]), df_add2(qp[2], qp[3]));
+                    DF2 h;
+                    if constexpr (VPL == 4)
+                        h = df_add2(df_add2(qp[0], qp[1]), df_add2(qp[2], qp[3]));
+                    else
+                        h = df_add2(qp[0], qp[1]);
                     DF lo, hi;
                     lo.s = h.s.x;
                     lo.c = h.c.x;

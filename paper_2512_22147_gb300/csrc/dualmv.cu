@@ -505,10 +505,23 @@ cudaError_t launch_f64e_phased_n(const dmv::TmapSet &maps, const Params &prm,
                             (size_t)pl.smem_bytes, stream, maps, prm);
 }
 
+// The 4-byte phased kernel's tile: W consumer warps x 4 rows, ring depth.
+// Its realignment makes it latency bound where the aligned kernel is not, so
+// it takes more warps: 12 x 4 rows, 4 stages (13 warps keep 128 registers).
+// Against 8 warps x 6 stages: f32 16384 x 16383 83.5% -> 87.9% of HBM,
+// int32 4001 x 100003 (lda 100003) 66.7% -> 85.7%.
+#ifndef DUALMV_PHASED_WARPS
+#define DUALMV_PHASED_WARPS 12
+#endif
+#ifndef DUALMV_PHASED_STAGES
+#define DUALMV_PHASED_STAGES 4
+#endif
+constexpr int kPhasedWarps = DUALMV_PHASED_WARPS, kPhasedStages = DUALMV_PHASED_STAGES;
+
 template <typename T, int NPH>
 Geometry phased_geometry_n() {
-    Geometry g = stream_geometry<T, kWarps, default_rpw<T>(), kStages>(true);
-    g.smem = dmv::SmemLayout<T, kWarps, default_rpw<T>(), kStages, true, NPH>::kTotal;
+    Geometry g = stream_geometry<T, kPhasedWarps, default_rpw<T>(), kPhasedStages>(true);
+    g.smem = dmv::SmemLayout<T, kPhasedWarps, default_rpw<T>(), kPhasedStages, true, NPH>::kTotal;
     return g;
 }
 template <typename T>
@@ -523,7 +536,7 @@ template <typename T, int NPH>
 cudaError_t launch_phased_n(const dmv::TmapSet &maps, const Params &prm, const dualmv_plan_t &pl,
                             int dev, cudaStream_t stream) {
     constexpr auto kern =
-        dmv::dualmv_stream_phased_kernel<T, kWarps, default_rpw<T>(), kStages, NPH>;
+        dmv::dualmv_stream_phased_kernel<T, kPhasedWarps, default_rpw<T>(), kPhasedStages, NPH>;
     cudaError_t e = smem_opt_in<kern>(pl.smem_bytes, dev);
     if (e != cudaSuccess) return e;
     if constexpr (std::is_same<T, int32_t>::value)  // after the zeroing kernel
@@ -925,9 +938,7 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
         std::memset(&pmaps, 0, sizeof pmaps);
         // Box rows: a tile's rows of one phase (4-byte kernel), or a warp's
         // (the self-loading fp64 kernel).
-        const int box_rows = es == 8 ? kF64eRpw
-                                     : (int)stream_geometry<T, kWarps, default_rpw<T>(), kStages>(
-                                           true).tile_rows;
+        const int box_rows = es == 8 ? kF64eRpw : kPhasedWarps * default_rpw<T>();
         nph = encode_phased<T>(&pmaps, &pinfo, A, M, N, lda, box_rows);
     }
 

@@ -366,10 +366,16 @@ struct TileCursor32 {
 template <typename T, int W, int RPW, int STAGES, bool kTma, int NPH = 0>
 struct SmemLayout {
     using Acc = typename Traits<T>::Acc;
-    // NPH > 0 (phased maps): a tile row is the band's box row (1 KiB for
-    // 4-byte elements) plus 16 bytes from the small box.
+    // NPH > 0 (phased maps): per phase, its W * RPW / NPH rows of the band's
+    // box (1 KiB a row for 4-byte elements), then their 16 bytes each from
+    // the small box, padded to 128 bytes so that every copy lands 128-byte
+    // aligned.  kTileTx is what a tile's copies deliver, kTileBytes its slot.
     static constexpr int kRowBytes = kBandCols * (int)sizeof(T);
-    static constexpr int kTileBytes = W * RPW * (kRowBytes + (NPH > 0 ? 16 : 0));
+    static constexpr int kPhaseRows = NPH > 0 ? W * RPW / NPH : W * RPW;
+    static constexpr int kPhaseBytes =
+        kPhaseRows * kRowBytes + (NPH > 0 ? (kPhaseRows * 16 + 127) / 128 * 128 : 0);
+    static constexpr int kTileBytes = (NPH > 0 ? NPH : 1) * kPhaseBytes;
+    static constexpr int kTileTx = W * RPW * (kRowBytes + (NPH > 0 ? 16 : 0));
     static constexpr int kAlign = kTma ? 1024 : 16;
     static constexpr int kRing = kTma ? STAGES * kTileBytes : 0;
     static constexpr int kScratch = W * kBandCols * (int)sizeof(Acc);
@@ -417,7 +423,9 @@ __device__ __forceinline__ void stream_body(const CUtensorMap *tmaps, const Para
     // then the small box (BM / NPH rows of 16 bytes).
     constexpr int PH = NPH > 0 ? NPH : 1;
     constexpr int PHASE_ROWS = BM / PH;
-    constexpr int PHASE_BYTES = PHASE_ROWS * (ROW_BYTES + 16);
+    constexpr int PHASE_BYTES = L::kPhaseBytes;
+    static_assert(PHASE_ROWS == L::kPhaseRows && PHASE_BYTES % 128 == 0,
+                  "phased maps: every copy must land 128-byte aligned");
 
     extern __shared__ unsigned char smem_raw[];
     unsigned char *smem = smem_raw + shared_align_pad<L::kAlign>(smem_raw);
@@ -467,7 +475,7 @@ __device__ __forceinline__ void stream_body(const CUtensorMap *tmaps, const Para
                         ok = mbar_wait_bounded(smem_u32(&empty_bar[stage]), phase ^ 1u);
                     if (!ok) break;
                     const uint32_t fb = smem_u32(&full_bar[stage]);
-                    mbar_arrive_expect_tx(fb, TILE_BYTES);
+                    mbar_arrive_expect_tx(fb, L::kTileTx);
                     const uint32_t dst = smem_u32(ring + (size_t)stage * TILE_BYTES);
                     const int x = (int)(cur.band * kBandCols), y = (int)(cur.stripe * BM);
                     if constexpr (NPH > 0) {

@@ -506,22 +506,40 @@ cudaError_t launch_f64e_phased_n(const dmv::TmapSet &maps, const Params &prm,
 }
 
 // The 4-byte phased kernel's tile: W consumer warps x 4 rows, ring depth.
-// Its realignment makes it latency bound where the aligned kernel is not, so
-// it takes more warps: 12 x 4 rows, 4 stages (13 warps keep 128 registers).
-// Against 8 warps x 6 stages: f32 16384 x 16383 83.5% -> 87.9% of HBM,
-// int32 4001 x 100003 (lda 100003) 66.7% -> 85.7%.
-#ifndef DUALMV_PHASED_WARPS
-#define DUALMV_PHASED_WARPS 12
+// Its realignment makes it latency bound where the aligned kernel is not.
+// Measured (% of HBM, whole call; f32 16384 x 16383 / int32 4001 x 100003,
+// both at lda = N):
+//   warps x stages   8 x 6   10 x 5   12 x 4   15 x 3
+//   f32              83.5    90.6     88.5     87.2
+//   int32            66.7    72.8     85.7     94.4
+// f32 wants ring depth, int32 (64-bit sums) warps.  16 x 3 leaves f32 at
+// 96 registers and does not fit int32's 8-byte scratch.
+#ifndef DUALMV_PHASED_WARPS_F32
+#define DUALMV_PHASED_WARPS_F32 10
 #endif
-#ifndef DUALMV_PHASED_STAGES
-#define DUALMV_PHASED_STAGES 4
+#ifndef DUALMV_PHASED_STAGES_F32
+#define DUALMV_PHASED_STAGES_F32 5
 #endif
-constexpr int kPhasedWarps = DUALMV_PHASED_WARPS, kPhasedStages = DUALMV_PHASED_STAGES;
+#ifndef DUALMV_PHASED_WARPS_I32
+#define DUALMV_PHASED_WARPS_I32 15
+#endif
+#ifndef DUALMV_PHASED_STAGES_I32
+#define DUALMV_PHASED_STAGES_I32 3
+#endif
+template <typename T>
+constexpr int phased_warps() {
+    return std::is_same<T, int32_t>::value ? DUALMV_PHASED_WARPS_I32 : DUALMV_PHASED_WARPS_F32;
+}
+template <typename T>
+constexpr int phased_stages() {
+    return std::is_same<T, int32_t>::value ? DUALMV_PHASED_STAGES_I32 : DUALMV_PHASED_STAGES_F32;
+}
 
 template <typename T, int NPH>
 Geometry phased_geometry_n() {
-    Geometry g = stream_geometry<T, kPhasedWarps, default_rpw<T>(), kPhasedStages>(true);
-    g.smem = dmv::SmemLayout<T, kPhasedWarps, default_rpw<T>(), kPhasedStages, true, NPH>::kTotal;
+    constexpr int W = phased_warps<T>(), S = phased_stages<T>();
+    Geometry g = stream_geometry<T, W, default_rpw<T>(), S>(true);
+    g.smem = dmv::SmemLayout<T, W, default_rpw<T>(), S, true, NPH>::kTotal;
     return g;
 }
 template <typename T>
@@ -536,7 +554,8 @@ template <typename T, int NPH>
 cudaError_t launch_phased_n(const dmv::TmapSet &maps, const Params &prm, const dualmv_plan_t &pl,
                             int dev, cudaStream_t stream) {
     constexpr auto kern =
-        dmv::dualmv_stream_phased_kernel<T, kPhasedWarps, default_rpw<T>(), kPhasedStages, NPH>;
+        dmv::dualmv_stream_phased_kernel<T, phased_warps<T>(), default_rpw<T>(), phased_stages<T>(),
+                                         NPH>;
     cudaError_t e = smem_opt_in<kern>(pl.smem_bytes, dev);
     if (e != cudaSuccess) return e;
     if constexpr (std::is_same<T, int32_t>::value)  // after the zeroing kernel
@@ -938,7 +957,7 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
         std::memset(&pmaps, 0, sizeof pmaps);
         // Box rows: a tile's rows of one phase (4-byte kernel), or a warp's
         // (the self-loading fp64 kernel).
-        const int box_rows = es == 8 ? kF64eRpw : kPhasedWarps * default_rpw<T>();
+        const int box_rows = es == 8 ? kF64eRpw : phased_warps<T>() * default_rpw<T>();
         nph = encode_phased<T>(&pmaps, &pinfo, A, M, N, lda, box_rows);
     }
 

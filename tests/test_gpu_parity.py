@@ -353,6 +353,26 @@ def test_unaligned_f64_rows_keep_the_double_float_range_check():
     assert torch.isfinite(torch.cat([sc[:300], sc[301:]])).all()
 
 
+@pytest.mark.parametrize("dtype,M,N,lda", [
+    ("f32", 3000, 5000, 5001),      # 4 phases; many CTAs per band
+    ("f32", 2500, 4098, 4098),      # 2 phases
+    ("i32", 777, 20001, 20003),     # 4 phases, exact
+    ("f64", 2000, 3000, 3001),      # 2 phases, double-float
+])
+def test_phased_many_tiles_match_oracle_and_repeat_bitwise(dtype, M, N, lda):
+    """The phased kernels over many stripes and bands, where several CTAs
+    share a band and their column partials meet in the combine: every
+    output matches the oracle, and repeated calls give the same bits."""
+    A, p, r = _make(dtype, M, N, lda, 97)
+    run_and_compare(A, p, r, N)
+    assert dm.dualmv_last_kernel() == dm.DUALMV_KERNEL_PHASED
+    view = A[:, :N]
+    outs = [dm.dualmv(view, p, r) for _ in range(3)]
+    torch.cuda.synchronize()
+    for q, s in outs[1:]:
+        assert torch.equal(q, outs[0][0]) and torch.equal(s, outs[0][1])
+
+
 def test_last_kernel_reports_each_path():
     A, p, r = _make("f64", 96, 512, 512, 92)
     dm.dualmv(A, p, r)

@@ -294,9 +294,10 @@ enum {
     DUALMV_KERNEL_WIDE = 2,   /* int32: tiles of rows_per_warp rows by     */
                               /* warps * 256 columns, one 256-column       */
                               /* sub-band per warp                         */
-    DUALMV_KERNEL_PHASED = 3, /* 4-byte rows whose stride or base is not   */
-                              /* 16-byte aligned: TMA through one pair of  */
-                              /* tensor maps per row phase (no variants)   */
+    DUALMV_KERNEL_PHASED = 3, /* rows whose stride or base is not 16-byte  */
+                              /* aligned: TMA through one pair of tensor   */
+                              /* maps per row phase (no variants; fp64 in  */
+                              /* double-float arithmetic)                  */
     DUALMV_KERNEL_PLAIN = 4   /* plain global loads (no variants)          */
 };
 typedef struct dualmv_variant_t {
@@ -351,8 +352,8 @@ int32_t dualmv_last_variant(void);
  * last dual product ran (dualmv_f32/f64/i32 and their strided-batched forms,
  * and the passes inside GESUMMV, ATAX and GEMVER), or -1 if it ran none (an
  * empty problem or an error).  PHASED: rows whose stride or base the TMA
- * unit cannot take as one tensor, for one 4-byte dual product; PLAIN: the
- * remaining unaligned cases.  Instrumentation for tests and benchmarks. */
+ * unit cannot take as one tensor, for one dual product (fp64 unless
+ * DUALMV_PATH_TMA_NATIVE_F64 is set); PLAIN: the remaining unaligned cases.  Instrumentation for tests and benchmarks. */
 int32_t dualmv_last_kernel(void);
 
 /* Trimmed mean of Eq. 3: the R values sorted, the k smallest and k largest

@@ -945,7 +945,8 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     }
 
     // Rows the TMA unit cannot take as one tensor (row stride or base not
-    // 16-byte aligned): phased tensor maps, for one 4-byte dual product.
+    // 16-byte aligned): phased tensor maps, for one dual product (fp64 in the
+    // double-float kernel).
     dmv::TmapSet pmaps;
     Params pinfo;
     std::memset(&pinfo, 0, sizeof pinfo);

@@ -1,7 +1,7 @@
 // Device kernels of the variant tuner: the functional-equivalence check of
 // Eq. 4 (a candidate's outputs against the current baseline's) and the
 // magnitude sums that scale it.  They are deliberately simple and share no
-// code with the streaming kernels whose outputs they judge.
+// code with the streaming kernels whose outputs they check.
 #pragma once
 
 #include <cstdint>

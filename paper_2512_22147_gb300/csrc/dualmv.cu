@@ -535,6 +535,23 @@ constexpr int phased_stages() {
     return std::is_same<T, int32_t>::value ? DUALMV_PHASED_STAGES_I32 : DUALMV_PHASED_STAGES_F32;
 }
 
+// Dynamic shared memory a CTA may opt into on sm_100-class parts.
+constexpr int kMaxDynSmem = 227 * 1024;
+template <typename T>
+constexpr bool phased_layouts_fit() {
+    constexpr int W = phased_warps<T>(), R = default_rpw<T>(), S = phased_stages<T>();
+    return dmv::SmemLayout<T, W, R, S, true, 1>::kTotal <= kMaxDynSmem &&
+           dmv::SmemLayout<T, W, R, S, true, 2>::kTotal <= kMaxDynSmem &&
+           dmv::SmemLayout<T, W, R, S, true, 4>::kTotal <= kMaxDynSmem;
+}
+static_assert(phased_layouts_fit<float>() && phased_layouts_fit<int32_t>(),
+              "a phased tile shape exceeds the shared memory of a CTA");
+static_assert(dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand, 1>::kTotal <=
+                      kMaxDynSmem &&
+                  dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand, 2>::kTotal <=
+                      kMaxDynSmem,
+              "a phased fp64 layout exceeds the shared memory of a CTA");
+
 template <typename T, int NPH>
 Geometry phased_geometry_n() {
     constexpr int W = phased_warps<T>(), S = phased_stages<T>();

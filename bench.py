@@ -115,7 +115,8 @@ def recorded_traffic(workload: str, family: str | None = None, shape=None):
     fam = kernel_family(ent["kernel"])
     if fam not in KERNEL_FAMILIES or ent.get("kernel_source_hash") != kernel_source_hash(fam):
         return None
-    if family is not None and (fam != family or kernel_shape(ent["kernel"]) != tuple(shape)):
+    if family is not None and (fam != family or (
+            shape is not None and kernel_shape(ent["kernel"]) != tuple(shape))):
         return None
     return ent.get("dram_bytes_per_launch")
 
@@ -459,12 +460,16 @@ def run_native(args):
                       dm.DUALMV_KERNEL_WIDE: "dualmv_wide_i32_kernel"}[v.kernel]
             shape = (v.warps, v.rows_per_warp, v.stages)
             kernel_name = family + f"<warps {v.warps}, rows {v.rows_per_warp}, stages {v.stages}>"
-        else:  # rows TMA cannot take as one tensor, or a forced plain-load path
+        else:  # batched (the default kernel), unaligned rows, or plain loads
+            kind = dm.dualmv_last_kernel()
             kernel_name = {
                 dm.DUALMV_KERNEL_PHASED: ("dualmv_stream_f64e_phased_kernel" if w.dtype == "f64"
                                           else "dualmv_stream_phased_kernel"),
                 dm.DUALMV_KERNEL_PLAIN: "dualmv_stream_kernel (plain loads)",
-            }.get(dm.dualmv_last_kernel(), kernel_name)
+            }.get(kind, kernel_name)
+            if w.batched and kind in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_F64E):
+                family = {dm.DUALMV_KERNEL_STREAM: "dualmv_stream_kernel",
+                          dm.DUALMV_KERNEL_F64E: "dualmv_stream_f64e_kernel"}[kind]
     achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9
     traffic = recorded_traffic(args.workload, family, shape) if family else None
 

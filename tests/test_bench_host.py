@@ -149,6 +149,9 @@ def test_launch_list_parser_and_traffic_record(tmp_path, monkeypatch):
     assert bench.recorded_traffic("wl", "dualmv_stream_kernel", (8, 4, 6)) == int(1001e6 + 500e3)
     assert bench.recorded_traffic("wl", "dualmv_stream_kernel", (8, 4, 4)) is None
     assert bench.recorded_traffic("wl", "dualmv_wide_i32_kernel", (8, 4, 6)) is None
+    # Batched calls name the family only (their default kernel has no variant).
+    assert bench.recorded_traffic("wl", "dualmv_stream_kernel", None) == int(1001e6 + 500e3)
+    assert bench.recorded_traffic("wl", "dualmv_wide_i32_kernel", None) is None
     assert bench.recorded_traffic("other") is None
     assert bench.kernel_shape("dmv::dualmv_stream_f64e_kernel<8, 4, 3, 256, 0, 3, 2, 1>") == \
         (8, 4, 3)

@@ -489,8 +489,9 @@ cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualm
 
 template <int NPH>
 Geometry f64e_phased_geometry_n() {
-    Geometry g = f64e_geometry<kF64eWarps, kF64eRpw, kF64eStages>();
-    g.smem = dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand, NPH>::kTotal;
+    // The phased fp64 kernel: self-loading warps on 256-column bands.
+    Geometry g = f64e_geometry<kF64eWarps, kF64eRpw, kF64eStages, true, kBandCols>();
+    g.smem = dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kBandCols, NPH>::kTotal;
     return g;
 }
 
@@ -546,9 +547,9 @@ constexpr bool phased_layouts_fit() {
 }
 static_assert(phased_layouts_fit<float>() && phased_layouts_fit<int32_t>(),
               "a phased tile shape exceeds the shared memory of a CTA");
-static_assert(dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand, 1>::kTotal <=
+static_assert(dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kBandCols, 1>::kTotal <=
                       kMaxDynSmem &&
-                  dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kF64eBand, 2>::kTotal <=
+                  dmv::F64eLayout<kF64eWarps, kF64eRpw, kF64eStages, kBandCols, 2>::kTotal <=
                       kMaxDynSmem,
               "a phased fp64 layout exceeds the shared memory of a CTA");
 

@@ -142,8 +142,7 @@ atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxPara
                     for (uint32_t k = 1; k < csize; ++k)
                         tt += part[(bp * kAtaxMaxCluster + k) * R + lane];
                     float th, tl;
-                    uint32_t habs;
-                    split_f64(tt, th, tl, habs);
+                    split_f64(tt, th, tl);
                     bad = !f64e_in_range(tt);
                     tvec[bp * R + lane] = tt;
                     tsplit[bp * R + lane] = make_float2(th, tl);
@@ -199,8 +198,7 @@ atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxPara
         for (int e = 0; e < VE; ++e) {
             const int64_t col = col0 + lane_col<double>(v, lane, e);
             const double xv = (live && col < prm.N) ? prm.x[col] : 0.0;
-            uint32_t habs;
-            split_f64(xv, h[e], l[e], habs);
+            split_f64(xv, h[e], l[e]);
             x_bad |= !f64e_in_range(xv);
             segp[lane_col<double>(v, lane, e)] = 0.0;
         }
@@ -268,10 +266,10 @@ atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxPara
 #pragma unroll
                     for (int v = 0; v < VPL; ++v) {
                         float ah0, al0, ah1, al1;
-                        uint32_t habs0, habs1;
-                        split_f64(a[v].x, ah0, al0, habs0);
-                        split_f64(a[v].y, ah1, al1, habs1);
-                        span = max(span, max(habs0 - kF64eLoBits, habs1 - kF64eLoBits));
+                        split_f64(a[v].x, ah0, al0);
+                        split_f64(a[v].y, ah1, al1);
+                        span = __vimax3_u32(span, f64e_range_key(a[v].x),
+                                            f64e_range_key(a[v].y));
                         const float2 ah = make_float2(ah0, ah1), al = make_float2(al0, al1);
                         df_prod2(ah, al, xh2[v], xl2[v], qp[v].s, qp[v].c);
                         // The column phase reads the split, not the double.
@@ -291,7 +289,7 @@ atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxPara
                     q[i] = df_add(lo, hi);
                 }
                 bool native = warp_x_bad;
-                if (!native && __any_sync(0xffffffffu, span >= kF64eSpanBits)) {
+                if (!native && __any_sync(0xffffffffu, span >= kF64eRangeSpan)) {
                     // Exact re-check from global memory: zeros pass.
                     bool bad = false;
 #pragma unroll

@@ -9,27 +9,36 @@
 // operations only, into an unevaluated sum of two floats, and products and
 // sums use error-free FP32 transformations.
 //
-//   split   a = a_hi + a_lo + d, a_hi the top 21 significant bits of a, a_lo
-//           the remaining 32 rounded to 24, |d| <= 2^-45 |a|.
-//   product a*x ~ a_hi x_hi + (err(a_hi x_hi) + a_hi x_lo + a_lo x_hi); the
-//           first term and its rounding error come from FMUL and FFMA
-//           exactly; the dropped a_lo x_lo is below 2^-44 |a x|.
-//   native  NC of each lane's eight columns (default 2) take their column
-//           sums from native fp64 FMA instead: GB300's FP64 pipe is
-//           otherwise idle here, and this moves NC/8 of the s work off the
-//           FP32 pipes.
-//   sum     Knuth's TwoSum on the high parts, the low parts and the TwoSum
-//           errors summed in a second float ("sloppy" double-float
-//           accumulation), in three levels: the RPW rows of a tile (or the 8
-//           columns of a lane), groups of kGroupTiles tiles, then fp64 for
-//           the segment.  Every level sums few terms, so the bound stays
-//           near (terms per level) * 2^-47 * sum |a x|, far below 1e-12.
+// Error bound (u = 2^-24, every |a|, |p_j|, |r_i| in [2^-40, 2^40) or 0):
+//   split   a = a_hi + a_lo + d: a_hi is a truncated to 24 significant bits,
+//           so |a - a_hi| < 2^-23 |a|; a_lo is that remainder rounded to a
+//           float, |d| <= u |a - a_hi| < 2^-47 |a|.
+//   product a*x ~ p + q, p = fl(a_hi x_hi), q = err(p) + a_hi x_lo +
+//           a_lo x_hi (two FMA roundings).  Dropped: a_lo x_lo < 2^-46 |ax|
+//           and the split residues d x, a d_x < 2^-46 |ax|; the roundings of
+//           q (|q| < 1.25 2^-22 |ax|) add at most 2^-45 |ax|.  In all,
+//           |ax - p - q| < 2^-44 |ax|.
+//   sum     Knuth's TwoSum on the high parts (exact); the low parts, which
+//           hold the products' q and the TwoSum errors (|low| < 1.5 2^-22
+//           of the sum of |terms| beneath it), take two roundings per
+//           addition: at most 3 2^-46 of those terms' sum |ax| per addition
+//           node.  A term of q passes 8 nodes (the lane's 8 columns in a
+//           tree, the 32 lanes in a butterfly); a term of s at most 19 (the
+//           4 rows of a tile in a chain, then kGroupTiles = 16 tiles in a
+//           chain); then fp64 for segments and band partials.
+//   So |q_i - q^_i| < (2^-44 + 24 2^-46 + fp64 sums) sum_j |A_ij p_j|
+//   ~ 4.1e-13 and |s_j - s^_j| < (2^-44 + 57 2^-46 + fp64 sums)
+//   sum_i |A_ij r_i| ~ 8.8e-13 of the sums of magnitudes, inside the 1e-12
+//   bar; random data sits near 1e-14.
+//   native  NC of each lane's eight columns (default 2; 0 in the packed
+//           kernel) take their column sums from native fp64 FMA instead.
 //
 // Range.  The split and the FP32 arithmetic are exact only while every
 // |a|, |p_j|, |r_i| lies in [2^-40, 2^40) or is zero (products then stay
-// inside FP32's normal range).  Each element costs two integer ops of range
-// bookkeeping; a warp whose rows of a tile hold anything else re-checks
-// them exactly (zeros are fine) and, if a value really is out of range,
+// inside FP32's normal range).  Each element costs about one and a half
+// integer ops of range bookkeeping (a key per element, a three-way max per
+// pair); a warp whose rows of a tile hold anything else re-checks them
+// exactly (zeros are fine) and, if a value really is out of range,
 // recomputes those rows with native fp64 FMA.  Results are the same
 // arithmetic on every call, so they are deterministic.
 #pragma once
@@ -42,10 +51,17 @@ namespace dmv {
 #define DUALMV_F64E_NATIVE_COLS 2
 #endif
 
-// Bits of |a| as the high word of a double: 2^-40 has biased exponent 983,
-// 2^40 has 1063.
-constexpr uint32_t kF64eLoBits = 983u << 20;
-constexpr uint32_t kF64eSpanBits = (1063u - 983u) << 20;
+// Range key of a double: its high word shifted left by one (the sign bit
+// dropped), less the key of 2^-40 (biased exponent 983).  |a| lies in
+// [2^-40, 2^40) exactly when the key is below kF64eRangeSpan (2^40 has
+// biased exponent 1063); zero and everything out of range give a key at or
+// above it.
+constexpr uint32_t kF64eRangeLo = 983u << 21;
+constexpr uint32_t kF64eRangeSpan = (1063u - 983u) << 21;
+
+__device__ __forceinline__ uint32_t f64e_range_key(double a) {
+    return ((uint32_t)__double2hiint(a) << 1) - kF64eRangeLo;
+}
 
 struct DF {
     float s;  // high part
@@ -53,29 +69,30 @@ struct DF {
 };
 
 // Split a double into hi + lo floats without touching the FP64 pipe.
-// a_hi keeps the sign, exponent and top 20 mantissa bits (the double's high
-// word, rebiased); a_lo is the low word converted to float (rounded to 24 of
-// its 32 bits) and scaled by 2^(e-52).  |a - a_hi - a_lo| <= 2^-45 |a|.
-// Zero (either sign) gives two zeros; values outside [2^-40, 2^40) give
-// garbage and must be caught by the range check.
-__device__ __forceinline__ void split_f64(double a, float &hi, float &lo, uint32_t &habs) {
+// hi is a truncated to 24 significant bits: sign, exponent and the top 23
+// stored mantissa bits.  A float's biased exponent is the double's less
+// 896; for double exponents 897..1150 that is the double's low seven
+// exponent bits under its top exponent bit (bit 30 of the high word), so
+// hi is the two words funnel-shifted left by three places with bits 31 and
+// 30 taken from the high word.  lo is the 29 stored bits left over, as an
+// integer (shifted up by three) converted to float, so rounded to 24
+// significant bits, times 2^(e - 55) with the sign of a (e the exponent of
+// a).  |a - hi| < 2^-23 |a| and |a - hi - lo| < 2^-47 |a|.  Zero (either
+// sign) gives two zeros; values outside [2^-40, 2^40) give garbage and
+// must be caught by the range check.
+__device__ __forceinline__ void split_f64(double a, float &hi, float &lo) {
     const uint32_t h = (uint32_t)__double2hiint(a);
     const uint32_t l = (uint32_t)__double2loint(a);
-    habs = h & 0x7FFFFFFFu;
-    // Rebias the exponent from 1023 to 127 (896 << 20); zero keeps zero.
-    const uint32_t t = h - min(habs, 896u << 20);
-    const uint32_t hi_bits = ((t << 3) & 0x7FFFFFFFu) | (h & 0x80000000u);
+    const uint32_t hi_bits = (h & 0xC0000000u) | (__funnelshift_l(l, h, 3) & 0x3FFFFFFFu);
     hi = __uint_as_float(hi_bits);
-    // 2^(e-52) with the sign of a.
-    const float scale = __uint_as_float((hi_bits & 0xFF800000u) - (52u << 23));
-    lo = __fmul_rn(__uint2float_rn(l), scale);
+    const float scale = __uint_as_float((hi_bits & 0xFF800000u) - (55u << 23));
+    lo = __fmul_rn(__uint2float_rn(l << 3), scale);
 }
 
 // Exact range test: |a| in [2^-40, 2^40) or a == 0.
 __device__ __forceinline__ bool f64e_in_range(double a) {
     const uint32_t h = (uint32_t)__double2hiint(a), l = (uint32_t)__double2loint(a);
-    const uint32_t habs = h & 0x7FFFFFFFu;
-    return (habs - kF64eLoBits) < kF64eSpanBits || (habs | l) == 0u;
+    return f64e_range_key(a) < kF64eRangeSpan || ((h << 1) | l) == 0u;
 }
 
 __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
@@ -84,7 +101,8 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
     e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
 }
 
-// a * x as (p, q) with p + q within 2^-46 |a x| of the exact product.
+// a * x as (p, q), from the splits of a and x (a_lo x_lo dropped): p + q
+// is within 2^-44 |a x| of the exact product.
 __device__ __forceinline__ void df_prod(float ah, float al, float xh, float xl, float &p,
                                         float &q) {
     p = __fmul_rn(ah, xh);
@@ -510,8 +528,7 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
                 for (int e = 0; e < VE; ++e) {
                     const int64_t col = col0 + lane_col<T>(v, lane, e);
                     const T pv = col < prm.N ? pb[col] : T(0);
-                    uint32_t habs;
-                    split_f64(pv, ph[v * VE + e], pl[v * VE + e], habs);
+                    split_f64(pv, ph[v * VE + e], pl[v * VE + e]);
                     p_bad |= !f64e_in_range(pv);
                 }
             if constexpr (kPack) {
@@ -524,8 +541,7 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
         }
         // r of this warp's rows, split by its owner lane.
         float rh_mine, rl_mine;
-        uint32_t r_habs;
-        split_f64(rmine, rh_mine, rl_mine, r_habs);
+        split_f64(rmine, rh_mine, rl_mine);
         const bool r_bad = kS && !f64e_in_range(rmine);
 
         const int slot = warp * STAGES + stage;
@@ -568,7 +584,7 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
         double tnat[kNativeCols > 0 ? kNativeCols : 1];
 #pragma unroll
         for (int j = 0; j < kNativeCols; ++j) tnat[j] = 0.0;
-        uint32_t span = 0;  // max over elements of (|a| bits - 2^-40 bits)
+        uint32_t span = 0;  // max over elements of their range keys
         if constexpr (kPack) {
             // Slot i of this lane is row i ^ perm (see warp_rows_reduce_df_perm).
             const int perm = butterfly_row<RPW>(lane);
@@ -585,10 +601,9 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
 #pragma unroll
                 for (int v = 0; v < VPL; ++v) {
                     float ah0, al0, ah1, al1;
-                    uint32_t habs0, habs1;
-                    split_f64(a[v].x, ah0, al0, habs0);
-                    split_f64(a[v].y, ah1, al1, habs1);
-                    span = max(span, max(habs0 - kF64eLoBits, habs1 - kF64eLoBits));
+                    split_f64(a[v].x, ah0, al0);
+                    split_f64(a[v].y, ah1, al1);
+                    span = __vimax3_u32(span, f64e_range_key(a[v].x), f64e_range_key(a[v].y));
                     const float2 ah = make_float2(ah0, ah1), al = make_float2(al0, al1);
                     if constexpr (kS) {
                         float2 p0, p1;
@@ -631,9 +646,8 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
                 for (int e = 0; e < VE; ++e) {
                     const int ce = v * VE + e;
                     float ah, al;
-                    uint32_t habs;
-                    split_f64(vget(a[v], e), ah, al, habs);
-                    span = max(span, habs - kF64eLoBits);
+                    split_f64(vget(a[v], e), ah, al);
+                    span = max(span, f64e_range_key(vget(a[v], e)));
                     if (!kS) {
                     } else if (ce < kFirstNative) {
                         float p0, p1;
@@ -661,7 +675,7 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
         // Anything suspicious in this warp's rows (zeros included)?
         const bool rows_r_bad = __any_sync(0xffffffffu, lane < RPW && r_bad);
         bool need_fp64 = rows_r_bad || __any_sync(0xffffffffu, kQ && p_bad);
-        if (!need_fp64 && __any_sync(0xffffffffu, span >= kF64eSpanBits)) {
+        if (!need_fp64 && __any_sync(0xffffffffu, span >= kF64eRangeSpan)) {
             // Exact re-check: zeros are fine, anything else out of range is not.
             bool bad = false;
 #pragma unroll

@@ -116,14 +116,15 @@ def _identity_case(dtype, n=700):
 @pytest.mark.parametrize("dtype", ["f32", "f64", "i32"])
 def test_identity_is_bit_exact(dtype, path):
     """A = I: q = p and s = r bit for bit (each sum has one nonzero term),
-    except fp64 on the FP32-pipe path, whose double-float split keeps 45 of
-    the 53 significant bits: there the result is within 2^-44 relative."""
+    except fp64 on the FP32-pipe path, whose double-float split rounds the
+    29 low mantissa bits to a float's 24: there the result is within 2^-47
+    relative (tested against 2^-46)."""
     A, p, r = _identity_case(dtype)
     q, s = dm.dualmv(A, p, r)
     if dtype == "f64" and path == dm.DUALMV_PATH_TMA:
         for got, want in ((q, p), (s, r)):
             rel = ((got - want).abs() / want.abs()).max()
-            assert float(rel) <= 2.0 ** -44
+            assert float(rel) <= 2.0 ** -46
     else:
         assert torch.equal(q.cpu(), p.cpu().to(q.dtype)) and torch.equal(s.cpu(), r.cpu().to(s.dtype))
 

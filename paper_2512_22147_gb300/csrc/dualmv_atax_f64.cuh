@@ -253,7 +253,10 @@ atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxPara
                 unsigned char *box = ring + (size_t)slot * L::kBoxBytes;
                 const int64_t row0 = (s0 + j) * R;
                 DF q[R];
+                // Range keys: one running max per column vector (independent
+                // chains; one chain through the stripe serialises the warp).
                 uint32_t span = 0;
+                uint32_t spanv[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
                 for (int i = 0; i < R; ++i) {
                     // Slot i of this lane is row i ^ perm (warp_rows_reduce_df_perm).
@@ -268,8 +271,8 @@ atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxPara
                         float ah0, al0, ah1, al1;
                         split_f64(a[v].x, ah0, al0);
                         split_f64(a[v].y, ah1, al1);
-                        span = __vimax3_u32(span, f64e_range_key(a[v].x),
-                                            f64e_range_key(a[v].y));
+                        spanv[v] = __vimax3_u32(spanv[v], f64e_range_key(a[v].x),
+                                                f64e_range_key(a[v].y));
                         const float2 ah = make_float2(ah0, ah1), al = make_float2(al0, al1);
                         df_prod2(ah, al, xh2[v], xl2[v], qp[v].s, qp[v].c);
                         // The column phase reads the split, not the double.
@@ -288,6 +291,10 @@ atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxPara
                     hi.c = h.c.y;
                     q[i] = df_add(lo, hi);
                 }
+                if constexpr (VPL == 4)
+                    span = max(max(spanv[0], spanv[1]), max(spanv[2], spanv[3]));
+                else
+                    span = max(spanv[0], spanv[1]);
                 bool native = warp_x_bad;
                 if (!native && __any_sync(0xffffffffu, span >= kF64eRangeSpan)) {
                     // Exact re-check from global memory: zeros pass.

@@ -105,9 +105,10 @@ dualmv_status dualmv_i32_strided_batched(
     dualmv_stream_t stream);
 
 /* ---- operations built on the same streaming kernels --------------------
- * Two more kernels the paper tunes (Table 1 and Table 2), each a short
- * sequence of single-sided passes of the dual product's streaming kernel
- * (rows only or columns only), so every pass reads its matrix once.
+ * Three more kernels the paper tunes (Table 1 and Table 2), built from the
+ * dual product's streaming kernels run single-sided (rows only or columns
+ * only, every pass reading its matrix once), and for ATAX from a cluster
+ * form of them that reads A once.
  * Conventions as above (row-major, caller-owned device memory, asynchronous
  * on `stream`, stream-ordered scratch from the library's pool).
  *
@@ -126,32 +127,48 @@ dualmv_status dualmv_gesummv_f64(int64_t M, int64_t N, double alpha, const doubl
 
 /* ATAX (Table 1, row "ATAX"): with A M x N (lda >= max(1, N)), x of length
  * N and y of length N:  tmp = A x (length M);  y = A^T tmp.  The second
- * product needs all of tmp, so A is streamed twice (rows, then columns).
- * M == 0 sets y to zero. */
+ * product needs all of tmp; see dualmv_atax_set_two_pass below for when A
+ * is read once and when twice.  Floating-point sums have a fixed order
+ * (deterministic).  M == 0 sets y to zero. */
 dualmv_status dualmv_atax_f32(int64_t M, int64_t N, const float *A, int64_t lda,
                               const float *x, float *y, dualmv_stream_t stream);
 dualmv_status dualmv_atax_f64(int64_t M, int64_t N, const double *A, int64_t lda,
                               const double *x, double *y, dualmv_stream_t stream);
 
-/* ATAX with one read of A: fp32 problems whose base and row stride meet the
- * TMA rules and whose width fits a cluster of at most 16 CTAs (N <= 32768)
- * stream A once: the CTAs of a thread-block cluster share each 8-row stripe,
- * exchange the stripe's partial row sums through distributed shared memory
- * and form A^T t from the copy still on chip.  Other problems, and fp64,
- * read A twice (a rows-only pass, then a columns-only pass).
+/* ATAX with one read of A.  A problem whose base is 16-byte aligned, whose
+ * row stride lda * sizeof(element) is a multiple of 16 bytes and whose
+ * width fits a thread-block cluster of at most 16 CTAs streams A once: the
+ * CTAs of a cluster share each 4-row stripe (each CTA a slice of the
+ * columns: 16 warps x 256 columns = 4096 for fp32, 8 warps x 256 = 2048 for
+ * fp64), exchange the stripe's partial row sums through distributed shared
+ * memory, and form A^T tmp from the copy still on chip.  So fp32 takes this
+ * path for N <= 65536 and fp64 (in double-float arithmetic on the FP32
+ * pipes, native fp64 for stripes with values outside [2^-40, 2^40)) for
+ * N <= 32768, when the GPU can place such a cluster.  Other problems read A
+ * twice: a rows-only pass (tmp = A x), then a columns-only pass.
  * dualmv_atax_set_two_pass(1) forces the two-pass path for every problem
  * (tests, benchmarks); 0 restores the choice.  Returns the previous setting. */
 int dualmv_atax_set_two_pass(int two_pass);
+
+/* Which path the calling thread's last ATAX call with M > 0 and N > 0 took:
+ * DUALMV_ATAX_ONE_READ (the cluster kernel) or DUALMV_ATAX_TWO_PASS; -1
+ * after an empty problem or an error.  Instrumentation for tests. */
+enum { DUALMV_ATAX_TWO_PASS = 0, DUALMV_ATAX_ONE_READ = 1 };
+int32_t dualmv_atax_last_path(void);
 
 /* GEMVER (Table 1 / Table 2, row "GEMVER"): with A M x N (lda >= max(1, N)),
  * u1, u2, w, y of length M and v1, v2, x, z of length N:
  *     A_hat = A + u1 v1^T + u2 v2^T
  *     x     = x + beta * A_hat^T y + z        (x is read and written)
  *     w     = w + alpha * A_hat x             (w is read and written)
- * The rank-2 update is applied on the fly by each of the two passes over A
- * (columns, then rows), so A_hat is never stored unless update_A is
- * nonzero, in which case the second pass writes A_hat over A (as the
- * PolyBench kernel does).  fp64 takes native fp64 arithmetic here. */
+ * w depends on all of the new x, so A is streamed twice: a columns-only
+ * pass (A_hat^T y), then a rows-only pass (A_hat x).  Without update_A
+ * (the default use) the rank-2 update is factorised (see
+ * dualmv_gemver_set_onthefly): the passes are the plain streaming kernels,
+ * in double-float arithmetic on the FP32 pipes for fp64.  With update_A
+ * nonzero both passes form A_hat element by element as they stream A, and
+ * the rows-only pass writes A_hat over A (as the PolyBench kernel does);
+ * that form runs fp64 in native fp64 arithmetic. */
 dualmv_status dualmv_gemver_f32(int64_t M, int64_t N, float alpha, float beta, float *A,
                                 int64_t lda, int update_A, const float *u1, const float *v1,
                                 const float *u2, const float *v2, float *w, float *x,

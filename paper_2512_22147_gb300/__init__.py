@@ -29,7 +29,8 @@ _BINDING_NAMES = {
     "dualmv_trimmed_mean", "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32",
     "dualmv_last_variant", "TuneStep", "dualmv_atax_set_two_pass",
     "dualmv_gemver_set_onthefly", "dualmv_last_kernel", "DUALMV_KERNEL_PHASED",
-    "DUALMV_KERNEL_PLAIN",
+    "DUALMV_KERNEL_PLAIN", "dualmv_atax_last_path", "DUALMV_ATAX_ONE_READ",
+    "DUALMV_ATAX_TWO_PASS",
 }
 _API_NAMES = {"dualmv", "device_fault", "gesummv", "atax", "gemver", "tune", "variants"}
 

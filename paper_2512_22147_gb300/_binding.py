@@ -40,6 +40,8 @@ DUALMV_KERNEL_F64E = 1
 DUALMV_KERNEL_WIDE = 2
 DUALMV_KERNEL_PHASED = 3
 DUALMV_KERNEL_PLAIN = 4
+DUALMV_ATAX_TWO_PASS = 0
+DUALMV_ATAX_ONE_READ = 1
 
 EXPORTED = (
     "dualmv_f32", "dualmv_f64", "dualmv_i32",
@@ -54,6 +56,7 @@ EXPORTED = (
     "dualmv_tuned_variant", "dualmv_tune_clear", "dualmv_trimmed_mean",
     "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32", "dualmv_last_variant",
     "dualmv_atax_set_two_pass", "dualmv_gemver_set_onthefly", "dualmv_last_kernel",
+    "dualmv_atax_last_path",
 )
 
 
@@ -156,6 +159,7 @@ def _load() -> ctypes.CDLL:
     lib.dualmv_tune_clear.argtypes, lib.dualmv_tune_clear.restype = [], None
     lib.dualmv_last_variant.argtypes, lib.dualmv_last_variant.restype = [], i32
     lib.dualmv_last_kernel.argtypes, lib.dualmv_last_kernel.restype = [], i32
+    lib.dualmv_atax_last_path.argtypes, lib.dualmv_atax_last_path.restype = [], i32
     lib.dualmv_trimmed_mean.argtypes = [ctypes.POINTER(ctypes.c_double), i64, i64,
                                         ctypes.POINTER(ctypes.c_double)]
     lib.dualmv_trimmed_mean.restype = st
@@ -320,6 +324,12 @@ def dualmv_last_variant() -> int:
 def dualmv_last_kernel() -> int:
     """DUALMV_KERNEL_* of this thread's last dual product, or -1."""
     return _lib.dualmv_last_kernel()
+
+
+def dualmv_atax_last_path() -> int:
+    """DUALMV_ATAX_ONE_READ or DUALMV_ATAX_TWO_PASS for this thread's last
+    ATAX call, or -1."""
+    return _lib.dualmv_atax_last_path()
 
 
 def dualmv_trimmed_mean(times, k: int) -> float:

@@ -75,6 +75,7 @@ thread_local cudaEvent_t g_kernel_ev_start = nullptr;
 thread_local cudaEvent_t g_kernel_ev_stop = nullptr;
 thread_local int32_t g_last_variant = -1;
 thread_local int32_t g_last_kernel = -1;
+thread_local int32_t g_last_atax_path = -1;
 int g_path = DUALMV_PATH_AUTO;
 int g_atax_two_pass = 0;  // 1: ATAX always takes the two-pass path
 int g_gemver_onthefly = 0;  // 1: GEMVER applies the update element by element
@@ -1317,6 +1318,7 @@ dualmv_status atax_cluster_run(int64_t M, int64_t N, const T *A, int64_t lda, co
 template <typename T>
 dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x, T *y,
                        cudaStream_t stream) {
+    g_last_atax_path = -1;
     if (M < 0 || N < 0 || lda < (N > 1 ? N : 1)) return DUALMV_ERR_INVALID_VALUE;
     if (N == 0) return DUALMV_SUCCESS;
     if (y == nullptr || (M > 0 && (A == nullptr || x == nullptr)))
@@ -1329,6 +1331,7 @@ dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x
     if (g_atax_two_pass == 0) {
         bool used = false;
         dualmv_status sc = atax_cluster_run<T>(M, N, A, lda, x, y, stream, &used);
+        if (sc == DUALMV_SUCCESS && used) g_last_atax_path = DUALMV_ATAX_ONE_READ;
         if (sc != DUALMV_SUCCESS || used) return sc;
     }
     T *tmp = nullptr;
@@ -1341,6 +1344,7 @@ dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x
                        dmv::kOutS);
     cudaError_t ef = cudaFreeAsync(tmp, stream);
     if (st == DUALMV_SUCCESS && ef != cudaSuccess) st = cuda_fail(ef);
+    if (st == DUALMV_SUCCESS) g_last_atax_path = DUALMV_ATAX_TWO_PASS;
     return st;
 }
 
@@ -2009,6 +2013,8 @@ int32_t dualmv_tuned_variant(int32_t dtype, int64_t M, int64_t N, int64_t lda) {
 int32_t dualmv_last_variant(void) { return g_last_variant; }
 
 int32_t dualmv_last_kernel(void) { return g_last_kernel; }
+
+int32_t dualmv_atax_last_path(void) { return g_last_atax_path; }
 
 void dualmv_tune_clear(void) {
     std::lock_guard<std::mutex> lk(g_tuned_mu);

@@ -108,6 +108,44 @@ def test_atax_one_read_path_runs():
     assert dm.device_fault() == dm.DUALMV_SUCCESS
 
 
+# The one-read path's stated limits (include/dualmv.h): a cluster of at most
+# 16 CTAs, each 4096 (fp32) or 2048 (fp64) columns wide, and TMA-aligned rows.
+@pytest.mark.parametrize("dtype,limit", [("f32", 65536), ("f64", 32768)])
+def test_atax_width_limit_chooses_the_path(dtype, limit):
+    """Just inside the width limit the cluster kernel reads A once; one
+    column past it (rows still 16-byte aligned), A is read twice."""
+    per16 = 4 if dtype == "f32" else 2
+    for N, want in ((limit, dm.DUALMV_ATAX_ONE_READ),
+                    (limit + 1, dm.DUALMV_ATAX_TWO_PASS)):
+        lda = (N + per16 - 1) // per16 * per16
+        A, x = inputs.generate_atax(_w("atax", dtype, 9, N, lda, N), DEV)
+        check_atax(A, x, N, dtype)
+        assert dm.dualmv_atax_last_path() == want, (N, dm.dualmv_atax_last_path())
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_atax_alignment_and_override_choose_two_passes(dtype):
+    """Rows whose stride or base is not 16-byte aligned, and the two-pass
+    override, take two passes; the aligned problem takes one read."""
+    M, N = 300, 1000
+    A, x = inputs.generate_atax(_w("atax", dtype, M, N + 8, N + 8, 17), DEV)
+    check_atax(A, x[:N].contiguous(), N, dtype)
+    assert dm.dualmv_atax_last_path() == dm.DUALMV_ATAX_ONE_READ
+    A1, x1 = inputs.generate_atax(_w("atax", dtype, M, N, N + 1, 18), DEV)
+    check_atax(A1, x1, N, dtype)                      # odd row stride
+    assert dm.dualmv_atax_last_path() == dm.DUALMV_ATAX_TWO_PASS
+    y = dm.atax(A[:, 1:N + 1], x[:N].contiguous())    # base one element in
+    torch.cuda.synchronize()
+    assert dm.dualmv_atax_last_path() == dm.DUALMV_ATAX_TWO_PASS
+    old = dm.dualmv_atax_set_two_pass(1)
+    try:
+        check_atax(A, x[:N].contiguous(), N, dtype)
+        assert dm.dualmv_atax_last_path() == dm.DUALMV_ATAX_TWO_PASS
+    finally:
+        dm.dualmv_atax_set_two_pass(old)
+    assert y.shape == (N,)
+
+
 def test_atax_one_read_is_deterministic():
     A, x = inputs.generate_atax(_w("atax", "f32", 3000, 9000, 9000, 6), DEV)
     y1 = dm.atax(A, x)

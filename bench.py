@@ -300,6 +300,181 @@ def barrier(world: int):
 
 # --------------------------------------------------------------- native ---
 
+def make_call(torch, dm, inputs, w, dev):
+    """The closure that runs one step of workload ``w`` and the tensors it
+    uses: ``(call, state)``; state holds A, p, r, q, s for the dual product."""
+    if w.op == "bicg":
+        A, p, r = inputs.generate(w, dev)
+        Av = A[..., : w.N]
+        q, s = inputs.empty_outputs(w, dev)
+
+        def call():
+            dm.dualmv(Av, p, r, q=q, s=s)
+        return call, {"A": A, "p": p, "r": r, "q": q, "s": s}
+    if w.op == "gesummv":
+        A, Bm, x = inputs.generate_gesummv(w, dev)
+        y = torch.empty(w.M, dtype=A.dtype, device=dev)
+
+        def call():
+            dm.gesummv(A[:, : w.N], Bm[:, : w.N], x, alpha=1.5, beta=1.2, y=y)
+        return call, {"A": A, "B": Bm, "x": x, "y": y}
+    if w.op == "atax":
+        A, x = inputs.generate_atax(w, dev)
+        y = torch.empty(w.N, dtype=A.dtype, device=dev)
+
+        def call():
+            dm.atax(A[:, : w.N], x, y=y)
+        return call, {"A": A, "x": x, "y": y}
+    # gemver: x and w accumulate in place from call to call
+    A, u1, v1, u2, v2, wv, x, y, z = inputs.generate_gemver(w, dev)
+
+    def call():
+        dm.gemver(A[:, : w.N], u1, v1, u2, v2, wv, x, y, z, alpha=1.5, beta=1.2)
+    return call, {"A": A, "x": x, "w": wv}
+
+
+def timed_region(torch, call, K, W, flush, stream, dev, world, uuid):
+    """The contract's timed region.  The clock sampler starts, then the W
+    warm-up calls run right before the region (so the GPU is at speed when
+    it opens, not idle after the sampler's start-up pause); a barrier and a
+    device synchronisation on both sides; K calls back to back between two
+    events, or, with ``flush`` (an L2-sized workload), each call between its
+    own events after an L2-evicting write outside them.  Returns (region
+    milliseconds, clock record)."""
+    sampler = ClockSampler(uuid)
+    sampler.start()
+    time.sleep(0.3)  # let the sampler start before the GPU work
+    for _ in range(W):
+        call()
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    if flush is None:
+        ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+        ev[0].record(stream)
+        for _ in range(K):
+            call()
+        ev[1].record(stream)
+    else:
+        flushed = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(K)]
+        for ev0, ev1 in flushed:
+            flush.zero_()
+            ev0.record(stream)
+            call()
+            ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clocks = sampler.stop()
+    if flush is None:
+        return ev[0].elapsed_time(ev[1]), clocks
+    return sum(a.elapsed_time(b) for a, b in flushed), clocks
+
+
+def instrumented_calls(torch, dm, call, n, flush, stream, dev, per_kernel: bool):
+    """``n`` more calls, each between its own events; with ``per_kernel`` the
+    library also records events around its streaming kernel on the stream it
+    runs on (dualmv_record_kernel_events).  Returns (per-call ms, kernel ms);
+    without ``per_kernel`` the kernel times are the whole calls."""
+    call_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(n)]
+    kern_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(n)]
+    # torch creates a CUDA event lazily on its first record; the library
+    # records the kernel events itself, so make them exist first.
+    for ks, ke in kern_ev:
+        ks.record(stream)
+        ke.record(stream)
+    torch.cuda.synchronize(dev)
+    for i in range(n):
+        ks, ke = kern_ev[i]
+        if flush is not None:
+            flush.zero_()
+        if per_kernel:
+            dm.dualmv_record_kernel_events(ks.cuda_event, ke.cuda_event)
+        else:
+            ks.record(stream)
+        call_ev[i][0].record(stream)
+        call()
+        call_ev[i][1].record(stream)
+        if not per_kernel:
+            ke.record(stream)
+    torch.cuda.synchronize(dev)
+    return ([a.elapsed_time(b) for a, b in call_ev], [a.elapsed_time(b) for a, b in kern_ev])
+
+
+def streaming_kernel_name(dm, w):
+    """(name, family, shape) of the streaming kernel the last dual product
+    launched, for the roofline record."""
+    kernel_name = f"whole {w.op} call"
+    family, shape = None, None
+    if w.op != "bicg":
+        return kernel_name, family, shape
+    kernel_name = "dualmv_stream_kernel"
+    vi = dm.dualmv_last_variant()
+    if vi >= 0:
+        v = dm.dualmv_variant_info({"f32": 0, "f64": 1, "i32": 2}[w.dtype], vi)
+        family = {dm.DUALMV_KERNEL_STREAM: "dualmv_stream_kernel",
+                  dm.DUALMV_KERNEL_F64E: "dualmv_stream_f64e_kernel",
+                  dm.DUALMV_KERNEL_WIDE: "dualmv_wide_i32_kernel"}[v.kernel]
+        shape = (v.warps, v.rows_per_warp, v.stages)
+        kernel_name = family + f"<warps {v.warps}, rows {v.rows_per_warp}, stages {v.stages}>"
+    else:  # batched (the default kernel), unaligned rows, or plain loads
+        kind = dm.dualmv_last_kernel()
+        kernel_name = {
+            dm.DUALMV_KERNEL_PHASED: ("dualmv_stream_f64e_phased_kernel" if w.dtype == "f64"
+                                      else "dualmv_stream_phased_kernel"),
+            dm.DUALMV_KERNEL_PLAIN: "dualmv_stream_kernel (plain loads)",
+        }.get(kind, kernel_name)
+        if w.batched and kind in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_F64E):
+            family = {dm.DUALMV_KERNEL_STREAM: "dualmv_stream_kernel",
+                      dm.DUALMV_KERNEL_F64E: "dualmv_stream_f64e_kernel"}[kind]
+    return kernel_name, family, shape
+
+
+def launches_per_call(torch, dm, inputs, w, dev) -> int:
+    """Kernels of this library one call launches."""
+    plan = dm.dualmv_plan(w.M, w.N, w.nbatch, inputs.ELEM_BYTES[w.dtype],
+                          inputs.OUT_BYTES[w.dtype],
+                          torch.cuda.get_device_properties(dev).multi_processor_count)
+    n = 1 + (1 if (plan.bands > 1 or plan.grid > 1) else 0)
+    if w.op == "gesummv":   # two row passes (stream + combine each) + epilogue
+        return 2 * n + 1
+    if w.op == "atax":      # a row pass and a column pass
+        return 2 * n
+    if w.op == "gemver":    # column pass, x update, row pass, w update
+        return 2 * n + 2
+    return n
+
+
+def read_ceiling(torch, dm, dev, stream, reps=10, nbytes=2 << 30):
+    """Read-only bandwidth of this GPU: the library's read probe (16-byte
+    loads over every SM) on a 2 GiB buffer, larger than L2, timed with
+    events on the launching stream after three warm-up passes."""
+    buf = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    out = torch.zeros(1, dtype=torch.int32, device=dev)
+    sp = stream.cuda_stream
+
+    def one():
+        rc = dm.dualmv_read_probe(buf.data_ptr(), nbytes, out.data_ptr(), sp)
+        if rc != dm.DUALMV_SUCCESS:
+            raise RuntimeError(f"dualmv_read_probe: status {rc}")
+    for _ in range(3):
+        one()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    gbs = nbytes * reps / (e0.elapsed_time(e1) * 1e-3) / 1e9
+    del buf, out
+    return {"gbs": round(gbs, 1), "bytes": nbytes, "reps": reps,
+            "how": "dualmv_read_probe: 16-byte loads, 8 in flight per thread, 2048 threads per "
+                   "SM, over a 2 GiB buffer; CUDA events on the launching stream"}
+
+
 def run_native(args):
     import torch
 
@@ -313,30 +488,7 @@ def run_native(args):
     w = workload_from_args(inputs, args)
     stream = torch.cuda.current_stream(dev)
     nbytes = w.bytes_counted()
-    if w.op == "bicg":
-        A, p, r = inputs.generate(w, dev)
-        Av = A[..., : w.N]
-        q, s = inputs.empty_outputs(w, dev)
-
-        def call():
-            dm.dualmv(Av, p, r, q=q, s=s)
-    elif w.op == "gesummv":
-        A, Bm, x = inputs.generate_gesummv(w, dev)
-        y = torch.empty(w.M, dtype=A.dtype, device=dev)
-
-        def call():
-            dm.gesummv(A[:, : w.N], Bm[:, : w.N], x, alpha=1.5, beta=1.2, y=y)
-    elif w.op == "atax":
-        A, x = inputs.generate_atax(w, dev)
-        y = torch.empty(w.N, dtype=A.dtype, device=dev)
-
-        def call():
-            dm.atax(A[:, : w.N], x, y=y)
-    else:  # gemver: x and w accumulate in place from call to call
-        A, u1, v1, u2, v2, wv, x, y, z = inputs.generate_gemver(w, dev)
-
-        def call():
-            dm.gemver(A[:, : w.N], u1, v1, u2, v2, wv, x, y, z, alpha=1.5, beta=1.2)
+    call, st = make_call(torch, dm, inputs, w, dev)
 
     if args.variant is not None:   # force one compiled kernel variant (profiling)
         dm.dualmv_set_variant({"f32": 0, "f64": 1, "i32": 2}[w.dtype], args.variant)
@@ -345,133 +497,45 @@ def run_native(args):
         if w.op != "bicg" or w.batched:
             raise SystemExit("--tune applies to one unbatched dual product")
         t0 = time.time()
-        rep = dm.tune(Av, p, r, repeats=30, trim=3, max_rounds=4, candidates=8, min_gain=0.01,
-                      flush_l2=flush_needed(torch, nbytes, dev))
+        Av = st["A"][..., : w.N]
+        rep = dm.tune(Av, st["p"], st["r"], repeats=30, trim=3, max_rounds=4, candidates=8,
+                      min_gain=0.01, flush_l2=flush_needed(torch, nbytes, dev))
         torch.cuda.synchronize(dev)
         v = dm.dualmv_variant_info({"f32": 0, "f64": 1, "i32": 2}[w.dtype], rep["best"])
         tuned = {k: (float(f"{val:.6g}") if isinstance(val, float) else val)
                  for k, val in rep.items() if k not in ("q", "s", "trace")}
         tuned["trace"] = [{k: (float(f"{val:.6g}") if isinstance(val, float) else val)
-                           for k, val in st.items()} for st in rep["trace"]]
+                           for k, val in stp.items()} for stp in rep["trace"]]
         tuned["variant"] = {f: getattr(v, f) for f, _ in v._fields_}
         tuned["seconds"] = round(time.time() - t0, 2)
-
-    for _ in range(args.warmup):
-        call()
-    torch.cuda.synchronize(dev)
-    if dm.device_fault() != dm.DUALMV_SUCCESS:
-        raise RuntimeError("device fault during warm-up")
 
     K = args.steps
     flush = None
     if flush_needed(torch, nbytes, dev):   # the operands could stay in L2 between calls
         flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
-    region = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    uuid = gpu_uuid(torch, dev)
 
-    # Timed region: K back-to-back calls, nothing recorded between them; or,
-    # for an L2-sized workload, K calls each between its own events with an
-    # L2-evicting write before it, outside the events.
-    sampler = ClockSampler(gpu_uuid(torch, dev))
-    sampler.start()
-    time.sleep(0.3)  # let the sampler start before the timed region
-    barrier(world)
-    torch.cuda.synchronize(dev)
-    if flush is None:
-        region[0].record(stream)
-        for _ in range(K):
-            call()
-        region[1].record(stream)
-    else:
-        flushed = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                   for _ in range(K)]
-        for ev0, ev1 in flushed:
-            flush.zero_()
-            ev0.record(stream)
-            call()
-            ev1.record(stream)
-    torch.cuda.synchronize(dev)
-    barrier(world)
-    clocks = sampler.stop()
+    region_ms, clocks = timed_region(torch, call, K, args.warmup, flush, stream, dev, world,
+                                     uuid)
     if dm.device_fault() != dm.DUALMV_SUCCESS:
         raise RuntimeError("device fault during the timed region")
-    if flush is None:
-        region_ms = region[0].elapsed_time(region[1])
-    else:
-        region_ms = sum(a.elapsed_time(b) for a, b in flushed)
     region_ms = max_over_ranks(torch, region_ms, world, dev)
     ms_per_step = region_ms / K
     value = world * nbytes * K / (region_ms * 1e-3) / 1e9
 
-    # Instrumented region: the same calls, each bracketed by events, and the
-    # streaming kernel bracketed by events the library records on its own
-    # stream (dualmv_record_kernel_events).  Gives the per-call times for the
-    # trimmed mean of Eq. 3 and the kernel time for the roofline.
+    # Instrumented region: per-call events for the trimmed mean of Eq. 3 and
+    # the streaming kernel's own time for the roofline.
     Ki = min(K, args.instrumented_steps)
-    call_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(Ki)]
-    kern_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(Ki)]
-    # torch creates the CUDA event lazily on its first record; the library
-    # records the kernel events itself, so make them exist first.
-    for ks, ke in kern_ev:
-        ks.record(stream)
-        ke.record(stream)
-    torch.cuda.synchronize(dev)
-    for i in range(Ki):
-        ks, ke = kern_ev[i]
-        if flush is not None:
-            flush.zero_()
-        if w.op == "bicg":
-            dm.dualmv_record_kernel_events(ks.cuda_event, ke.cuda_event)
-        else:  # several streaming passes per call: time the whole call
-            ks.record(stream)
-        call_ev[i][0].record(stream)
-        call()
-        call_ev[i][1].record(stream)
-        if w.op != "bicg":
-            ke.record(stream)
-    torch.cuda.synchronize(dev)
+    step_ms, kern_ms = instrumented_calls(torch, dm, call, Ki, flush, stream, dev,
+                                          per_kernel=w.op == "bicg")
     if dm.device_fault() != dm.DUALMV_SUCCESS:
         raise RuntimeError("device fault during the instrumented region")
-    step_ms = [a.elapsed_time(b) for a, b in call_ev]
-    kern_ms = [a.elapsed_time(b) for a, b in kern_ev]
-
-    plan = dm.dualmv_plan(w.M, w.N, w.nbatch, inputs.ELEM_BYTES[w.dtype],
-                          inputs.OUT_BYTES[w.dtype],
-                          torch.cuda.get_device_properties(dev).multi_processor_count)
-    launches_per_call = 1 + (1 if (plan.bands > 1 or plan.grid > 1) else 0)
-    if w.op == "gesummv":   # two row passes (stream + combine each) + epilogue
-        launches_per_call = 2 * launches_per_call + 1
-    elif w.op == "atax":    # a row pass and a column pass
-        launches_per_call = 2 * launches_per_call
-    elif w.op == "gemver":  # column pass, x update, row pass, w update
-        launches_per_call = 2 * launches_per_call + 2
     peak, peak_src = measured_peak()
     kern_avg_ms = sum(kern_ms) / len(kern_ms)
-    kernel_name = f"whole {w.op} call"
-    family, shape = None, None
-    if w.op == "bicg":   # the streaming kernel the last call launched
-        kernel_name = "dualmv_stream_kernel"
-        vi = dm.dualmv_last_variant()
-        if vi >= 0:
-            v = dm.dualmv_variant_info({"f32": 0, "f64": 1, "i32": 2}[w.dtype], vi)
-            family = {dm.DUALMV_KERNEL_STREAM: "dualmv_stream_kernel",
-                      dm.DUALMV_KERNEL_F64E: "dualmv_stream_f64e_kernel",
-                      dm.DUALMV_KERNEL_WIDE: "dualmv_wide_i32_kernel"}[v.kernel]
-            shape = (v.warps, v.rows_per_warp, v.stages)
-            kernel_name = family + f"<warps {v.warps}, rows {v.rows_per_warp}, stages {v.stages}>"
-        else:  # batched (the default kernel), unaligned rows, or plain loads
-            kind = dm.dualmv_last_kernel()
-            kernel_name = {
-                dm.DUALMV_KERNEL_PHASED: ("dualmv_stream_f64e_phased_kernel" if w.dtype == "f64"
-                                          else "dualmv_stream_phased_kernel"),
-                dm.DUALMV_KERNEL_PLAIN: "dualmv_stream_kernel (plain loads)",
-            }.get(kind, kernel_name)
-            if w.batched and kind in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_F64E):
-                family = {dm.DUALMV_KERNEL_STREAM: "dualmv_stream_kernel",
-                          dm.DUALMV_KERNEL_F64E: "dualmv_stream_f64e_kernel"}[kind]
+    kernel_name, family, shape = streaming_kernel_name(dm, w)
     achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9
     traffic = recorded_traffic(args.workload, family, shape) if family else None
+    ceiling = None if args.no_read_ceiling else read_ceiling(torch, dm, dev, stream)
 
     hot = hot_l2_graph(torch, call, nbytes, dev) if flush is not None else None
 
@@ -479,26 +543,28 @@ def run_native(args):
     # inputs copied in, the call, results copied out, every step.
     e2e = None
     if not args.no_e2e and w.op == "bicg":
-        e2e = run_e2e(torch, dm, w, A, p, r, dev, stream, args.e2e_steps)
+        e2e = run_e2e(torch, dm, w, st["A"], st["p"], st["r"], dev, stream, args.e2e_steps,
+                      uuid)
 
-    # Bitwise determinism: two more calls, compared bit for bit.
-    deterministic = None
-    if w.op == "bicg":
-        call()
-        q1, s1 = q.clone(), s.clone()
-        call()
-        torch.cuda.synchronize(dev)
-        deterministic = bool(torch.equal(q1, q) and torch.equal(s1, s))
-    elif w.op in ("gesummv", "atax"):
-        call()
-        y1 = y.clone()
-        call()
-        torch.cuda.synchronize(dev)
-        deterministic = bool(torch.equal(y1, y))
+    deterministic = bitwise_repeat(torch, call, st, w, dev)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline and w.op == "bicg":
-        cpu = cpu_baseline(w, A, p, r, args.cpu_seconds, q, s)
+        cpu = cpu_baseline(w, st["A"], st["p"], st["r"], args.cpu_seconds, st["q"], st["s"],
+                           parallel_s=args.cpu_parallel_seconds)
+
+    configs = None
+    if (world == 1 and not args.no_configs and w.op == "bicg" and args.variant is None
+            and not args.tune and w.name in inputs.WORKLOADS):
+        del st, call
+        torch.cuda.empty_cache()
+        configs = {}
+        for name, wc in inputs.WORKLOADS.items():
+            if name == w.name:
+                continue
+            configs[name] = measure_config(torch, dm, inputs, wc, dev, stream, args.warmup,
+                                           uuid, peak, ceiling, args.config_seconds)
+            torch.cuda.empty_cache()
 
     out = {
         "metric": METRIC,
@@ -538,10 +604,12 @@ def run_native(args):
             "traffic": traffic,
             "algorithmic_bytes_per_launch": nbytes,
             "kernel_avg_ms": round(kern_avg_ms, 5),
+            **({"read_ceiling": ceiling,
+                "frac_of_read_ceiling": round(achieved / ceiling["gbs"], 4)} if ceiling else {}),
         },
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": launches_per_call * K,
+        "gpu_launches": launches_per_call(torch, dm, inputs, w, dev) * K,
         "deterministic": deterministic,
         "instrumented_steps": Ki,
         "clocks": clocks,
@@ -550,11 +618,101 @@ def run_native(args):
         out["hot_l2_graph"] = hot
     if tuned is not None:
         out["tuned"] = tuned
+    if configs is not None:
+        out["configs"] = configs
     if rank == 0:
         print(json.dumps(out), flush=True)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def bitwise_repeat(torch, call, st, w, dev):
+    """Two more calls compared bit for bit (None for GEMVER, whose x and w
+    change from call to call)."""
+    if w.op == "bicg":
+        call()
+        q1, s1 = st["q"].clone(), st["s"].clone()
+        call()
+        torch.cuda.synchronize(dev)
+        return bool(torch.equal(q1, st["q"]) and torch.equal(s1, st["s"]))
+    if w.op in ("gesummv", "atax"):
+        call()
+        y1 = st["y"].clone()
+        call()
+        torch.cuda.synchronize(dev)
+        return bool(torch.equal(y1, st["y"]))
+    return None
+
+
+def measure_config(torch, dm, inputs, w, dev, stream, W, uuid, peak, ceiling, target_s):
+    """One more of the benchmark's dual-product workloads, measured in the
+    same process as the headline: W warm-up calls, then K calls timed as the
+    headline is (K sized for about ``target_s`` seconds of GPU time), the
+    streaming kernel timed on its own stream over 30 further calls, the
+    clocks sampled during the timed region, the outputs compared with the
+    oracle (every element; the first 8 problems of a batch) and two further
+    calls compared bit for bit."""
+    nbytes = w.bytes_counted()
+    call, st = make_call(torch, dm, inputs, w, dev)
+    flush = None
+    if flush_needed(torch, nbytes, dev):
+        flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    for _ in range(max(W, 3)):   # size K from the warm-up calls' time
+        call()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(5):
+        call()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    est_ms = max(e0.elapsed_time(e1) / 5, 1e-3)
+    K = int(min(3000, max(20, math.ceil(target_s * 1e3 / est_ms))))
+    region_ms, clocks = timed_region(torch, call, K, W, flush, stream, dev, 1, uuid)
+    step_ms, kern_ms = instrumented_calls(torch, dm, call, 30, flush, stream, dev, True)
+    kernel_name, _, _ = streaming_kernel_name(dm, w)
+    fault = dm.device_fault()
+    value = nbytes * K / (region_ms * 1e-3) / 1e9
+    kern_avg_ms = sum(kern_ms) / len(kern_ms)
+    achieved = nbytes / (kern_avg_ms * 1e-3) / 1e9
+    hot = hot_l2_graph(torch, call, nbytes, dev) if flush is not None else None
+    deterministic = bitwise_repeat(torch, call, st, w, dev)
+    n = min(w.batch, 8) if w.batched else w.M
+    A_np = st["A"][:n].cpu().numpy() if w.batched else st["A"].cpu().numpy()
+    p_np = st["p"][:n].cpu().numpy() if w.batched else st["p"].cpu().numpy()
+    r_np = st["r"][:n].cpu().numpy() if w.batched else st["r"].cpu().numpy()
+    import oracle
+    outs = (oracle.dualmv_batched(A_np, p_np, r_np, N=w.N) if w.batched
+            else oracle.dualmv(A_np, p_np, r_np, N=w.N))
+    parity = sample_parity(w, A_np, p_np, r_np, n, outs, st["q"].cpu().numpy(),
+                           st["s"].cpu().numpy())
+    out = {
+        "value": round(value, 2), "unit": "GB/s",
+        "pct_of_peak": round(100.0 * value / peak, 2),
+        "ms_per_step": round(region_ms / K, 5), "steps": K, "warmup": W,
+        "bytes_per_step": nbytes,
+        "config": {"M": w.M, "N": w.N, "lda": w.lda, "batch": w.batch, "dtype": w.dtype,
+                   "distribution": w.dist, "seed": w.seed},
+        "l2": ("inputs larger than L2 (no flush needed)" if flush is None else
+               f"L2 flushed: {FLUSH_BYTES >> 20} MiB written before each call, outside its "
+               "events"),
+        "trimmed_mean_ms": round(trimmed_mean(step_ms, 3), 5),
+        "kernel": kernel_name,
+        "kernel_avg_ms": round(kern_avg_ms, 5),
+        "kernel_frac": round(achieved / peak, 4),
+        **({"kernel_frac_of_read_ceiling": round(achieved / ceiling["gbs"], 4)} if ceiling
+           else {}),
+        "gpu_launches": launches_per_call(torch, dm, inputs, w, dev) * K,
+        "parity": parity,
+        "deterministic": deterministic,
+        "device_fault": fault != dm.DUALMV_SUCCESS,
+        "clocks": clocks,
+    }
+    if hot is not None:
+        out["hot_l2_graph"] = hot
+    del st, call, flush
+    return out
 
 
 def flush_needed(torch, nbytes: int, dev) -> bool:
@@ -592,7 +750,7 @@ def hot_l2_graph(torch, call, nbytes, dev, reps=20):
             "GBs": round(nbytes / (per_call_ms * 1e-3) / 1e9, 2)}
 
 
-def run_e2e(torch, dm, w, A, p, r, dev, stream, steps):
+def run_e2e(torch, dm, w, A, p, r, dev, stream, steps, uuid=None):
     Ah = A.cpu().pin_memory()
     ph = p.cpu().pin_memory()
     rh = r.cpu().pin_memory()
@@ -623,7 +781,65 @@ def run_e2e(torch, dm, w, A, p, r, dev, stream, steps):
             "ms_per_step": round(ms, 4), "steps": steps,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "how": "pinned host A, p, r copied to the GPU, dualmv through the C ABI, q and s "
-                   "copied back, all on one stream inside CUDA events"}
+                   "copied back, all on one stream inside CUDA events",
+            "host_placement": host_placement(Ah.data_ptr(), h2d, uuid)}
+
+
+def _cpulist(text: str) -> set:
+    cpus = set()
+    for part in text.strip().split(","):
+        if part:
+            a, _, b = part.partition("-")
+            cpus |= set(range(int(a), int(b or a) + 1))
+    return cpus
+
+
+def host_placement(ptr: int, nbytes: int, uuid=None, samples: int = 64):
+    """Where the pinned input buffer lives: the NUMA nodes of a sample of its
+    pages (move_pages with no target node reports each page's node), the
+    nodes of the CPUs this process may run on, and the NUMA node sysfs gives
+    for the GPU's PCI function.  Linux only; fields it cannot read are null."""
+    import ctypes
+    import platform
+    out = {"buffer_page_nodes": None, "process_cpu_nodes": None, "gpu_numa_node": None}
+    try:
+        nr = {"aarch64": 239, "x86_64": 279}[platform.machine()]
+        libc = ctypes.CDLL(None, use_errno=True)
+        ps = os.sysconf("SC_PAGE_SIZE")
+        addrs = [(ptr + k * (nbytes // samples)) & ~(ps - 1) for k in range(samples)]
+        arr = (ctypes.c_void_p * samples)(*addrs)
+        status = (ctypes.c_int * samples)()
+        if libc.syscall(nr, 0, ctypes.c_ulong(samples), arr, None, status, 0) == 0:
+            counts = {}
+            for v in status:
+                counts[str(v)] = counts.get(str(v), 0) + 1
+            out["buffer_page_nodes"] = counts
+    except (KeyError, OSError, AttributeError):
+        pass
+    try:
+        allowed = os.sched_getaffinity(0)
+        nodes = []
+        base = "/sys/devices/system/node"
+        for n in sorted(os.listdir(base)):
+            if n.startswith("node"):
+                with open(os.path.join(base, n, "cpulist")) as f:
+                    if _cpulist(f.read()) & allowed:
+                        nodes.append(int(n[4:]))
+        out["process_cpu_nodes"] = nodes
+    except OSError:
+        pass
+    try:
+        cmd = ["nvidia-smi", "--query-gpu=pci.bus_id", "--format=csv,noheader"]
+        if uuid:
+            cmd += ["-i", uuid]
+        bus = subprocess.run(cmd, capture_output=True, text=True,
+                             timeout=20).stdout.strip().splitlines()[0]
+        dom, rest = bus.split(":", 1)
+        with open(f"/sys/bus/pci/devices/{(dom[-4:] + ':' + rest).lower()}/numa_node") as f:
+            out["gpu_numa_node"] = int(f.read().strip())
+    except (OSError, ValueError, IndexError, subprocess.SubprocessError):
+        pass
+    return out
 
 
 # ------------------------------------------------------- CPU (oracle) ----
@@ -712,7 +928,7 @@ def sample_parity(w, A_np, p_np, r_np, n, outs, q_gpu, s_gpu):
             "checked": checked, "pass": bool(err <= PARITY_TOL[w.dtype])}
 
 
-def cpu_baseline(w, A, p, r, budget_s, q=None, s=None):
+def cpu_baseline(w, A, p, r, budget_s, q=None, s=None, parallel_s=0.0):
     A_np = A.cpu().numpy()
     p_np, r_np = p.cpu().numpy(), r.cpu().numpy()
     gbs, dt, what, n, outs = oracle_sample(w, A_np, p_np, r_np, budget_s)
@@ -721,7 +937,41 @@ def cpu_baseline(w, A, p, r, budget_s, q=None, s=None):
     if q is not None:
         out["parity"] = sample_parity(w, A_np, p_np, r_np, n, outs, q.cpu().numpy(),
                                       s.cpu().numpy())
+    if parallel_s > 0 and not w.batched:
+        out["parallel"] = parallel_baseline(w, A_np, p_np, r_np, n, outs, parallel_s)
     return out
+
+
+def parallel_baseline(w, A_np, p_np, r_np, n, outs, budget_s):
+    """The oracle's loops on every host core (oracle/oracle_omp.c, OpenMP):
+    the same rows as the single-core sample, repeated for about ``budget_s``
+    seconds.  Each output is summed in the oracle's order, so the outputs
+    must equal the oracle's bit for bit; that is checked too."""
+    import numpy as np
+    import oracle
+
+    e, o = inputs_sizes(w)
+    nbytes = n * w.N * e + (n + w.N) * (e + o)
+    A_s, r_s = A_np[:n], r_np[:n]
+    t0 = time.perf_counter()
+    q_p, s_p = oracle.dualmv_omp(A_s, p_np, r_s, N=w.N)
+    dt = time.perf_counter() - t0
+    passes = max(1, min(1000, int(budget_s / max(dt, 1e-6))))
+    t0 = time.perf_counter()
+    for _ in range(passes):
+        oracle.dualmv_omp(A_s, p_np, r_s, N=w.N)
+    dt = time.perf_counter() - t0
+    same = bool(np.array_equal(q_p, outs[0]) and np.array_equal(s_p, outs[1]))
+    return {"value": round(nbytes * passes / dt / 1e9, 4), "unit": "GB/s",
+            "cores": oracle.omp_threads(), "kind": "oracle loops on every host core (OpenMP)",
+            "sample": f"first {n} of {w.M} rows of {w.name}, {passes} passes; A read twice "
+                      "(rows for q, column blocks for s)",
+            "seconds": round(dt, 3), "bitwise_equal_to_oracle": same}
+
+
+def inputs_sizes(w):
+    from paper_2512_22147_gb300 import inputs
+    return inputs.ELEM_BYTES[w.dtype], inputs.OUT_BYTES[w.dtype]
 
 
 def run_reference(args):
@@ -778,6 +1028,14 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-parallel-seconds", type=float, default=3.0,
+                    help="time budget of the all-core (OpenMP) oracle baseline; 0 skips it")
+    ap.add_argument("--no-read-ceiling", action="store_true",
+                    help="skip the read-only bandwidth probe")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the other dual-product workloads (the 'configs' block)")
+    ap.add_argument("--config-seconds", type=float, default=0.25,
+                    help="GPU time of each other workload's timed region")
     ap.add_argument("--variant", type=int, default=None,
                     help="force this entry of the dtype's kernel-variant table")
     ap.add_argument("--tune", action="store_true",

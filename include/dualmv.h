@@ -264,6 +264,17 @@ int dualmv_set_path(int path);
  * problems, invalid arguments) leave the request pending. */
 void dualmv_record_kernel_events(void *start, void *stop);
 
+/* Instrumentation for benchmarks, not part of the method: reads `bytes`
+ * bytes of device memory at `buf` once with 16-byte loads spread over every
+ * SM, and xor-folds them into the device word *out (its value means
+ * nothing; it keeps the loads alive).  `buf` must be 16-byte aligned and
+ * `bytes` a multiple of 16 (else DUALMV_ERR_INVALID_VALUE, nothing
+ * enqueued).  Asynchronous on `stream`.  Timed over a buffer larger than
+ * L2, it gives the read-only bandwidth ceiling that the streaming kernels
+ * are compared with beside the measured copy bandwidth. */
+dualmv_status dualmv_read_probe(const void *buf, int64_t bytes, uint32_t *out,
+                                dualmv_stream_t stream);
+
 /* ---- planner (pure host code, no CUDA call) ----------------------------
  * The work decomposition a call would use.  A is cut into column bands of
  * `band_cols` columns and row stripes of `tile_rows` rows; a tile is one

@@ -43,6 +43,10 @@ _CFLAGS = ["-std=c99", "-O2", "-fno-fast-math", "-ffp-contract=off", "-fPIC",
            "-shared"]
 _lock = threading.Lock()
 _lib = None
+# The all-core baseline (oracle_omp.c): the same loops on every host core.
+_OMP_SRC = os.path.join(_HERE, "oracle_omp.c")
+_OMP_LIB_PATH = os.path.join(_HERE, "liboracle_omp.so")
+_omp_lib = None
 
 
 def build(src: str = _SRC, out: str = _LIB_PATH) -> str:
@@ -50,6 +54,52 @@ def build(src: str = _SRC, out: str = _LIB_PATH) -> str:
     cmd = ["gcc", *_CFLAGS, "-o", out, src, "-lm"]
     subprocess.run(cmd, check=True)
     return out
+
+
+def build_omp(src: str = _OMP_SRC, out: str = _OMP_LIB_PATH) -> str:
+    """Compile the OpenMP all-core baseline ``oracle_omp.c`` with gcc."""
+    cmd = ["gcc", *_CFLAGS, "-fopenmp", "-o", out, src, "-lm"]
+    subprocess.run(cmd, check=True)
+    return out
+
+
+def load_omp():
+    """Load (building first if needed) the all-core baseline library."""
+    global _omp_lib
+    with _lock:
+        if _omp_lib is None:
+            if (not os.path.exists(_OMP_LIB_PATH)
+                    or os.path.getmtime(_OMP_LIB_PATH) < os.path.getmtime(_OMP_SRC)):
+                build_omp()
+            lib = ctypes.CDLL(_OMP_LIB_PATH)
+            i64, vp = ctypes.c_int64, ctypes.c_void_p
+            for t in ("f32", "f64", "i32"):
+                fn = getattr(lib, f"oracle_omp_dualmv_{t}")
+                fn.argtypes = [i64, i64, vp, i64, vp, vp, vp, vp]
+                fn.restype = ctypes.c_int
+            lib.oracle_omp_threads.argtypes, lib.oracle_omp_threads.restype = [], ctypes.c_int
+            _omp_lib = lib
+    return _omp_lib
+
+
+def omp_threads() -> int:
+    """Threads the all-core baseline runs on (OpenMP's default team size)."""
+    return int(load_omp().oracle_omp_threads())
+
+
+def dualmv_omp(A: np.ndarray, p: np.ndarray, r: np.ndarray, N: int | None = None):
+    """``dualmv`` on every host core (OpenMP): the same outputs as
+    :func:`dualmv`, bit for bit (each output summed in the same order)."""
+    lib = load_omp()
+    M, N, lda, p, r = _prep(A, p, r, N)
+    tag, out_t = _IN[A.dtype]
+    q = np.zeros(M, dtype=out_t)
+    s = np.zeros(N, dtype=out_t)
+    rc = getattr(lib, f"oracle_omp_dualmv_{tag}")(M, N, _ptr(A), lda, _ptr(p), _ptr(r),
+                                                 _ptr(q), _ptr(s))
+    if rc != 0:
+        raise RuntimeError(f"oracle_omp_dualmv_{tag} returned {rc}")
+    return q, s
 
 
 def _stale() -> bool:

@@ -56,7 +56,7 @@ EXPORTED = (
     "dualmv_tuned_variant", "dualmv_tune_clear", "dualmv_trimmed_mean",
     "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32", "dualmv_last_variant",
     "dualmv_atax_set_two_pass", "dualmv_gemver_set_onthefly", "dualmv_last_kernel",
-    "dualmv_atax_last_path",
+    "dualmv_atax_last_path", "dualmv_read_probe",
 )
 
 
@@ -160,6 +160,8 @@ def _load() -> ctypes.CDLL:
     lib.dualmv_last_variant.argtypes, lib.dualmv_last_variant.restype = [], i32
     lib.dualmv_last_kernel.argtypes, lib.dualmv_last_kernel.restype = [], i32
     lib.dualmv_atax_last_path.argtypes, lib.dualmv_atax_last_path.restype = [], i32
+    lib.dualmv_read_probe.argtypes = [vp, i64, vp, vp]
+    lib.dualmv_read_probe.restype = st
     lib.dualmv_trimmed_mean.argtypes = [ctypes.POINTER(ctypes.c_double), i64, i64,
                                         ctypes.POINTER(ctypes.c_double)]
     lib.dualmv_trimmed_mean.restype = st
@@ -324,6 +326,12 @@ def dualmv_last_variant() -> int:
 def dualmv_last_kernel() -> int:
     """DUALMV_KERNEL_* of this thread's last dual product, or -1."""
     return _lib.dualmv_last_kernel()
+
+
+def dualmv_read_probe(buf, nbytes: int, out, stream) -> int:
+    """Benchmark instrumentation: one 16-byte-load pass over ``nbytes`` of
+    device memory at ``buf`` (xor-folded into the device word ``out``)."""
+    return _lib.dualmv_read_probe(buf, nbytes, out, stream)
 
 
 def dualmv_atax_last_path() -> int:

@@ -25,6 +25,7 @@
 #include "dualmv_atax.cuh"
 #include "dualmv_atax_f64.cuh"
 #include "dualmv_ops.cuh"
+#include "dualmv_probe.cuh"
 
 namespace {
 
@@ -1953,6 +1954,26 @@ dualmv_status dualmv_device_fault(dualmv_stream_t stream) {
         return DUALMV_ERR_TIMEOUT;
     }
     return DUALMV_SUCCESS;
+}
+
+dualmv_status dualmv_read_probe(const void *buf, int64_t bytes, uint32_t *out,
+                                dualmv_stream_t stream) {
+    if (bytes < 0 || bytes % 16 != 0 || reinterpret_cast<uintptr_t>(buf) % 16 != 0 ||
+        out == nullptr || (bytes > 0 && buf == nullptr))
+        return DUALMV_ERR_INVALID_VALUE;
+    if (bytes == 0) return DUALMV_SUCCESS;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e);
+    DeviceState *ds = nullptr;
+    e = device_state(dev, &ds);
+    if (e != cudaSuccess) return cuda_fail(e);
+    // Four blocks of 512 threads fill an SM's 2048 thread slots.
+    dmv::read_probe_kernel<<<(unsigned)(4 * ds->sms), dmv::kProbeThreads, 0,
+                             reinterpret_cast<cudaStream_t>(stream)>>>(
+        static_cast<const uint4 *>(buf), bytes / 16, out);
+    e = cudaGetLastError();
+    return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
 }
 
 void dualmv_record_kernel_events(void *start, void *stop) {

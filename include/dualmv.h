@@ -202,10 +202,13 @@ int dualmv_gemver_set_onthefly(int onthefly);
  * exits.  The call makes no cudaMalloc, cudaFree or pool allocation.
  * The caller still passes A, p, r, q and s.
  *
- * Limit: the partial sums need about ceil(N / 256) * M * 4 bytes (none
- * when N <= 256) plus under 1 MiB; a 16384 x 16384 matrix fits, a
- * 32768 x 16384 one does not.  Larger problems return DUALMV_ERR_TOO_LARGE
- * and enqueue nothing.
+ * Limit: the row partials need ceil(N / 256) * M * 4 bytes (none when
+ * N <= 256), and the column partials 1 KiB for every CTA and band it
+ * touches (usually two): about 0.3 MiB on the TMA path (one CTA per SM,
+ * 152 on GB300) and 1.2 MiB on the plain-load path (four per SM), more for
+ * very short matrices.  A 16384 x 16384 matrix fits, a 32768 x 16384 one
+ * does not.  Larger problems return DUALMV_ERR_TOO_LARGE and enqueue
+ * nothing.
  * Set-up: the first call on each device looks up the SM count and the
  * device address of the array (cudaGetSymbolAddress) with that device
  * current; make that first call before any stream capture.
@@ -237,6 +240,16 @@ int dualmv_last_cuda_error(void);
  * DUALMV_SUCCESS otherwise.  A kernel that gives up writes no output it has
  * not finished; the outputs of that call are then unspecified. */
 dualmv_status dualmv_device_fault(dualmv_stream_t stream);
+
+/* The library's stream-ordered workspace pool on `device` (created by the
+ * first call that needs it on that device, or by this call): bytes it holds
+ * now, and the high-water mark of bytes in use since the last reset.  With
+ * reset_high nonzero the mark is reset to the current use after it is read.
+ * Returns DUALMV_ERR_INVALID_VALUE for a bad device or NULL outputs.
+ * Diagnostics for tests: a call that takes no workspace leaves the mark at
+ * the use it had before the call. */
+dualmv_status dualmv_pool_usage(int device, int64_t *reserved_bytes, int64_t *used_high_bytes,
+                                int reset_high);
 
 /* Which kernel streams A.  DUALMV_PATH_AUTO (default) uses the TMA pipeline
  * when the alignment rules above hold and the plain-load kernel otherwise;

@@ -56,7 +56,7 @@ EXPORTED = (
     "dualmv_tuned_variant", "dualmv_tune_clear", "dualmv_trimmed_mean",
     "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32", "dualmv_last_variant",
     "dualmv_atax_set_two_pass", "dualmv_gemver_set_onthefly", "dualmv_last_kernel",
-    "dualmv_atax_last_path", "dualmv_read_probe",
+    "dualmv_atax_last_path", "dualmv_read_probe", "dualmv_pool_usage",
 )
 
 
@@ -162,6 +162,9 @@ def _load() -> ctypes.CDLL:
     lib.dualmv_atax_last_path.argtypes, lib.dualmv_atax_last_path.restype = [], i32
     lib.dualmv_read_probe.argtypes = [vp, i64, vp, vp]
     lib.dualmv_read_probe.restype = st
+    lib.dualmv_pool_usage.argtypes = [ctypes.c_int, ctypes.POINTER(i64), ctypes.POINTER(i64),
+                                      ctypes.c_int]
+    lib.dualmv_pool_usage.restype = st
     lib.dualmv_trimmed_mean.argtypes = [ctypes.POINTER(ctypes.c_double), i64, i64,
                                         ctypes.POINTER(ctypes.c_double)]
     lib.dualmv_trimmed_mean.restype = st
@@ -332,6 +335,18 @@ def dualmv_read_probe(buf, nbytes: int, out, stream) -> int:
     """Benchmark instrumentation: one 16-byte-load pass over ``nbytes`` of
     device memory at ``buf`` (xor-folded into the device word ``out``)."""
     return _lib.dualmv_read_probe(buf, nbytes, out, stream)
+
+
+def dualmv_pool_usage(device: int, reset_high: bool = False):
+    """(bytes held, high-water mark of bytes in use) of the library's
+    workspace pool on ``device``; ``reset_high`` resets the mark after
+    reading it."""
+    reserved, high = ctypes.c_int64(0), ctypes.c_int64(0)
+    rc = _lib.dualmv_pool_usage(device, ctypes.byref(reserved), ctypes.byref(high),
+                                1 if reset_high else 0)
+    if rc != DUALMV_SUCCESS:
+        raise DualmvError(rc, "dualmv_pool_usage")
+    return reserved.value, high.value
 
 
 def dualmv_atax_last_path() -> int:

@@ -1976,6 +1976,30 @@ dualmv_status dualmv_read_probe(const void *buf, int64_t bytes, uint32_t *out,
     return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
 }
 
+dualmv_status dualmv_pool_usage(int device, int64_t *reserved_bytes, int64_t *used_high_bytes,
+                                int reset_high) {
+    if (device < 0 || device >= kMaxDevices || reserved_bytes == nullptr ||
+        used_high_bytes == nullptr)
+        return DUALMV_ERR_INVALID_VALUE;
+    *reserved_bytes = 0;
+    *used_high_bytes = 0;
+    DeviceState *ds = nullptr;
+    cudaError_t e = device_state(device, &ds);
+    if (e != cudaSuccess) return cuda_fail(e);
+    uint64_t reserved = 0, high = 0;
+    e = cudaMemPoolGetAttribute(ds->pool, cudaMemPoolAttrReservedMemCurrent, &reserved);
+    if (e == cudaSuccess)
+        e = cudaMemPoolGetAttribute(ds->pool, cudaMemPoolAttrUsedMemHigh, &high);
+    if (e == cudaSuccess && reset_high) {
+        uint64_t zero = 0;  // resets the high-water mark to the current use
+        e = cudaMemPoolSetAttribute(ds->pool, cudaMemPoolAttrUsedMemHigh, &zero);
+    }
+    if (e != cudaSuccess) return cuda_fail(e);
+    *reserved_bytes = (int64_t)reserved;
+    *used_high_bytes = (int64_t)high;
+    return DUALMV_SUCCESS;
+}
+
 void dualmv_record_kernel_events(void *start, void *stop) {
     g_kernel_ev_start = static_cast<cudaEvent_t>(start);
     g_kernel_ev_stop = static_cast<cudaEvent_t>(stop);

@@ -153,12 +153,8 @@ def short_kernel_name(name: str) -> str:
     return name[5:] if name.startswith("void ") else name
 
 
-def record_traffic(csv_path: str, workload: str, command: str) -> str:
-    """Write the streaming kernel's DRAM bytes per launch for ``workload``
-    into the traffic record (with the current kernel-source hash) and return
-    a markdown summary of the whole launch list: per kernel its launches,
-    total time, share and DRAM bytes per launch."""
-    launches = parse_launch_list(csv_path)
+def launch_table(launches):
+    """Per kernel of a parsed launch list: [launches, total us, DRAM bytes]."""
     per = {}
     for _, name, m in launches:
         k = short_kernel_name(name)
@@ -166,11 +162,42 @@ def record_traffic(csv_path: str, workload: str, command: str) -> str:
         e[0] += 1
         e[1] += m.get("gpu__time_duration.sum", 0.0)
         e[2] += m.get("dram__bytes_read.sum", 0.0) + m.get("dram__bytes_write.sum", 0.0)
+    return per
+
+
+def summarize_launches(csv_path: str, command: str) -> str:
+    """Markdown summary of an ncu launch list taken with
+    ``--metrics gpu__time_duration.sum`` alone (one pass per launch, so it is
+    safe on the full workload): per kernel its launches, total time and
+    share.  ncu serialises launches and runs them cold: compare shares."""
+    per = launch_table(parse_launch_list(csv_path))
     total = sum(e[1] for e in per.values()) or 1.0
-    stream = [k for k in per if k.startswith(("dmv::dualmv_stream", "dmv::dualmv_wide"))]
+    out = [f"Command (from the repository root, on one GB300; the plain command exited 0 "
+           f"first):\n\n```\n{command}\n```\n",
+           "| kernel | launches | total us | share | us / launch |",
+           "|---|---|---|---|---|"]
+    for k, (cnt, us, _) in sorted(per.items(), key=lambda kv: -kv[1][1]):
+        out.append(f"| `{k[:120]}` | {cnt} | {us:.1f} | {100 * us / total:.1f} % | "
+                   f"{us / cnt:.2f} |")
+    return "\n".join(out)
+
+
+def record_traffic(csv_path: str, workload: str, command: str, full_bytes: int,
+                   case_bytes: int, case: str) -> str:
+    """From a capture of the streaming kernel alone on a small case of
+    ``workload`` (ncu ``-k`` one kernel, ``-c`` a few launches, DRAM and L2
+    counters): its DRAM bytes (read + write) per launch, scaled to a full
+    launch by the algorithmic bytes (``full_bytes / case_bytes``; A's bytes
+    dominate and its traffic grows in proportion), written into the traffic
+    record with the current kernel-source hash.  Returns a markdown summary
+    of the captured counters."""
+    launches = parse_launch_list(csv_path)
+    per = launch_table(launches)
+    stream = [k for k in per if kernel_family(k).startswith(("dualmv_stream", "dualmv_wide"))]
     if len(stream) != 1:
-        raise ValueError(f"expected one streaming kernel in the launch list, found {stream}")
-    n, _, dram = per[stream[0]]
+        raise ValueError(f"expected one streaming kernel in the capture, found {stream}")
+    n, us, dram = per[stream[0]]
+    scale = full_bytes / case_bytes
     rec = {}
     if os.path.exists(TRAFFIC_FILE):
         with open(TRAFFIC_FILE) as f:
@@ -178,20 +205,28 @@ def record_traffic(csv_path: str, workload: str, command: str) -> str:
     rec[workload] = {
         "kernel_source_hash": kernel_source_hash(kernel_family(stream[0])),
         "kernel": stream[0],
-        "dram_bytes_per_launch": int(round(dram / n)),
-        "how": "ncu launch list of bench.py on the full workload: dram__bytes_read.sum + "
-               "dram__bytes_write.sum of the streaming kernel, averaged over its launches",
+        "dram_bytes_per_launch": int(round(dram / n * scale)),
+        "how": (f"ncu capture of the streaming kernel alone (-k, {n} launch(es)) on {case}: "
+                f"dram__bytes_read.sum + dram__bytes_write.sum per launch = "
+                f"{dram / n:.0f} B for {case_bytes} algorithmic bytes, scaled by "
+                f"{scale:.4f} to the full workload's {full_bytes} algorithmic bytes"),
     }
     with open(TRAFFIC_FILE, "w") as f:
         json.dump(rec, f, indent=1)
         f.write("\n")
+    metrics = {}
+    for _, name, m in launches:
+        if short_kernel_name(name) == stream[0]:
+            for key, val in m.items():
+                metrics.setdefault(key, []).append(val)
     out = [f"Command (from the repository root, on one GB300; the plain command exited 0 "
            f"first):\n\n```\n{command}\n```\n",
-           "| kernel | launches | total us | share | us / launch | DRAM MB / launch |",
-           "|---|---|---|---|---|---|"]
-    for k, (cnt, us, b) in sorted(per.items(), key=lambda kv: -kv[1][1]):
-        out.append(f"| `{k[:120]}` | {cnt} | {us:.1f} | {100 * us / total:.1f} % | "
-                   f"{us / cnt:.2f} | {b / cnt / 1e6:.1f} |")
+           f"Kernel `{stream[0]}`, {n} launch(es) on {case} ({case_bytes} algorithmic bytes).\n",
+           "| metric | per launch |", "|---|---|"]
+    for key in sorted(metrics):
+        out.append(f"| {key} | {sum(metrics[key]) / len(metrics[key]):.6g} |")
+    out.append(f"\nDRAM read + write per launch: {dram / n / case_bytes:.4f} x the algorithmic "
+               f"bytes; scaled to the full workload: {int(round(dram / n * scale))} B.")
     return "\n".join(out)
 
 
@@ -1042,12 +1077,24 @@ def main(argv=None):
                     help="run the variant tuner (Eq. 3-5) on the workload before warm-up; "
                          "the timed calls then use the variant it chose")
     ap.add_argument("--record-traffic", metavar="CSV", default=None,
-                    help="record the streaming kernel's DRAM bytes per launch for --workload "
-                         "from an ncu launch-list CSV of this bench, then exit")
+                    help="from an ncu capture of the streaming kernel alone on the case that "
+                         "--workload with --M/--N/--lda/--batch names, record its DRAM bytes "
+                         "per launch scaled to the full --workload, then exit")
+    ap.add_argument("--summarize-launches", metavar="CSV", default=None,
+                    help="print a markdown summary of an ncu launch list (time only), then exit")
     ap.add_argument("--record-command", default="", help="the command that made the CSV")
     args = ap.parse_args(argv)
+    if args.summarize_launches:
+        print(summarize_launches(args.summarize_launches, args.record_command))
+        return
     if args.record_traffic:
-        print(record_traffic(args.record_traffic, args.workload, args.record_command))
+        from paper_2512_22147_gb300 import inputs
+        case = workload_from_args(inputs, args)
+        full = inputs.WORKLOADS.get(args.workload) or inputs.OP_WORKLOADS[args.workload]
+        desc = (f"{case.M} x {case.N}, lda {case.lda}" + (f", batch {case.batch}" if case.batch
+                                                           else "") + f", {case.dtype}")
+        print(record_traffic(args.record_traffic, args.workload, args.record_command,
+                             full.bytes_counted(), case.bytes_counted(), desc))
         return
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")

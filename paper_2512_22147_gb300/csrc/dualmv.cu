@@ -972,11 +972,12 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     std::memset(&pinfo, 0, sizeof pinfo);
     pinfo.ph_n = 1;
     int nph = 0;
-    // The fp64 phased kernel streams 256-column bands, as its maps' boxes are.
-    constexpr bool kF64ePhased = kF64eBand == kBandCols;
+    // The fp64 phased kernel streams 256-column bands of self-loading warps
+    // whatever band width the aligned fp64 kernel is built with
+    // (f64e_phased_geometry_n), so every fp64 band width may take it.
     if (kind == Kind::kDirect && g_path != DUALMV_PATH_DIRECT && !three_d &&
         rank2 == nullptr && outputs == dmv::kOutBoth &&
-        (es == 4 || (kF64ePhased && g_path != DUALMV_PATH_TMA_NATIVE_F64))) {
+        (es == 4 || g_path != DUALMV_PATH_TMA_NATIVE_F64)) {
         std::memset(&pmaps, 0, sizeof pmaps);
         // Box rows: a tile's rows of one phase (4-byte kernel), or a warp's
         // (the self-loading fp64 kernel).

@@ -141,16 +141,21 @@ def test_launch_list_parser_and_traffic_record(tmp_path, monkeypatch):
     assert [p[0] for p in parsed] == [0, 1, 2]
     assert parsed[0][2]["dram__bytes_read.sum"] == 1000e6
     assert parsed[0][2]["dram__bytes_write.sum"] == 500e3
+    md = bench.summarize_launches(str(csv_path), "cmd")
+    assert "| `dmv::dualmv_stream_kernel<float, 8, 4, 6, 1, 0>` | 2 | 330.0 | 97.6 % |" in md
     rec = tmp_path / "traffic.json"
     monkeypatch.setattr(bench, "TRAFFIC_FILE", str(rec))
-    md = bench.record_traffic(str(csv_path), "wl", "cmd")
-    assert "| `dmv::dualmv_stream_kernel<float, 8, 4, 6, 1, 0>` | 2 | 330.0 |" in md
-    assert bench.recorded_traffic("wl") == int(1001e6 + 500e3)
-    assert bench.recorded_traffic("wl", "dualmv_stream_kernel", (8, 4, 6)) == int(1001e6 + 500e3)
+    # A small-case capture scaled to the full workload (here 4x its bytes).
+    md = bench.record_traffic(str(csv_path), "wl", "cmd", full_bytes=4000, case_bytes=1000,
+                              case="a small case")
+    full = int(round(4 * (1001e6 + 500e3)))
+    assert "scaled to the full workload" in md
+    assert bench.recorded_traffic("wl") == full
+    assert bench.recorded_traffic("wl", "dualmv_stream_kernel", (8, 4, 6)) == full
     assert bench.recorded_traffic("wl", "dualmv_stream_kernel", (8, 4, 4)) is None
     assert bench.recorded_traffic("wl", "dualmv_wide_i32_kernel", (8, 4, 6)) is None
     # Batched calls name the family only (their default kernel has no variant).
-    assert bench.recorded_traffic("wl", "dualmv_stream_kernel", None) == int(1001e6 + 500e3)
+    assert bench.recorded_traffic("wl", "dualmv_stream_kernel", None) == full
     assert bench.recorded_traffic("wl", "dualmv_wide_i32_kernel", None) is None
     assert bench.recorded_traffic("other") is None
     assert bench.kernel_shape("dmv::dualmv_stream_f64e_kernel<8, 4, 3, 256, 0, 3, 2, 1>") == \

@@ -882,31 +882,17 @@ dualmv_combine_kernel(const Params prm, int64_t q_blocks, int q_chunks) {
     if (col >= prm.band_cols) return;
     const int64_t j = band * prm.band_cols + col;
     if (j >= prm.N) return;
-    // CTA cc's segment of band g is g minus the band of its first tile,
-    // floor(cc T / G) / S.  Both quotients advance from one CTA to the next
-    // by additions (two 64-bit divisions per segment made this kernel take
-    // longer than the stream kernel on small, many-segment problems).
-    const int64_t step_q = T_ / G, step_r = T_ % G;
-    int64_t rem = (c_lo * T_) % G;
-    const int64_t first = (c_lo * T_) / G;
-    int64_t fband = first / S, foff = first - fband * S;
-    Acc acc = Acc(0);
-#pragma unroll 4
-    for (int64_t cc = c_lo; cc <= c_hi; ++cc) {
-        const Acc v = sw[(cc * prm.max_seg + (g - fband)) * prm.band_cols + col];
-        acc = (cc == c_lo) ? v : acc + v;
-        int64_t step = step_q;
-        rem += step_r;
-        if (rem >= G) {
-            rem -= G;
-            ++step;
-        }
-        foff += step;
-        while (foff >= S) {
-            foff -= S;
-            ++fband;
-        }
-    }
+    // CTA cc's segment of band g is g minus the band of its first tile.  For
+    // every CTA after c_lo, band g is its first band (its range starts inside
+    // band g): segment 0.  So only c_lo's segment needs a division, and the
+    // loads do not wait on one another (a running segment count between
+    // them had made the small workload's combine take 5 of its 8 us).
+    const int64_t seg0 = g - ((c_lo * T_) / G) / S;
+    const Acc *src = sw + col;
+    const int64_t pitch = prm.max_seg * prm.band_cols;
+    Acc acc = src[c_lo * pitch + seg0 * prm.band_cols];
+#pragma unroll 8
+    for (int64_t cc = c_lo + 1; cc <= c_hi; ++cc) acc = acc + src[cc * pitch];
     static_cast<Acc *>(prm.s)[b * prm.strideS + j] = acc;
 }
 

@@ -479,10 +479,11 @@ cudaError_t launch_dependent(Kern kern, dim3 grid, dim3 block, size_t smem, cuda
 }
 
 template <typename T, bool kTma, bool k3d, int kOut = dmv::kOutBoth, bool kRank2 = false,
-          int W = kWarps, int RPW = default_rpw<T>(), int S = kStages>
+          int W = kWarps, int RPW = default_rpw<T>(), int S = kStages, bool kRev = false>
 cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                           int dev, cudaStream_t stream) {
-    constexpr auto kern = dmv::dualmv_stream_kernel<T, W, RPW, S, kTma, k3d, kOut, kRank2>;
+    constexpr auto kern =
+        dmv::dualmv_stream_kernel<T, W, RPW, S, kTma, k3d, kOut, kRank2, kRev>;
     cudaError_t e = smem_opt_in<kern>(pl.smem_bytes, dev);
     if (e != cudaSuccess) return e;
     if constexpr (std::is_same<T, int32_t>::value)  // after the zeroing kernel
@@ -625,11 +626,11 @@ int combine_chunks(int64_t bands) {
 
 template <bool k3d, int kOut = dmv::kOutBoth, int W = kF64eWarps, int RPW = kF64eRpw,
           int S = kF64eStages, int NC = kF64eNativeCols, bool kSelf = kF64eSelf,
-          bool kPack = kF64ePack, int BAND = kF64eBand>
+          bool kPack = kF64ePack, int BAND = kF64eBand, bool kRev = false>
 cudaError_t launch_f64e(const CUtensorMap &map, const Params &prm, const dualmv_plan_t &pl,
                         int dev, cudaStream_t stream) {
     constexpr auto kern =
-        dmv::dualmv_stream_f64e_kernel<W, RPW, S, BAND, k3d, kOut, NC, kSelf, kPack>;
+        dmv::dualmv_stream_f64e_kernel<W, RPW, S, BAND, k3d, kOut, NC, kSelf, kPack, kRev>;
     cudaError_t e = smem_opt_in<kern>(pl.smem_bytes, dev);
     if (e != cudaSuccess) return e;
     // A programmatic dependent of the kernel before it (on repeated calls, the
@@ -876,6 +877,18 @@ const Variant *pick_variant(int32_t dtype, int64_t M, int64_t N, const void *A, 
 }
 
 // GEMVER's rank-2 update, applied on the fly by a single-sided pass.
+// A pass whose combine a later kernel takes over: run() leaves its partial
+// sums in the workspace, launches no combine kernel and does not free the
+// workspace; the caller launches the kernel that adds them and then frees
+// `ws` on the same stream.  used = false: the pass took no workspace (an
+// empty problem, its outputs zero-filled).
+struct Deferred {
+    bool used = false;
+    Params prm;
+    void *ws = nullptr;
+    int chunks = 1;
+};
+
 struct Rank2 {
     const void *u1, *v1, *u2, *v2;
     void *a_out;  // write A_hat here (may be A itself), or nullptr
@@ -891,7 +904,8 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                   const T *p, int64_t strideP, const T *r, int64_t strideR, Out *q,
                   int64_t strideQ, Out *s, int64_t strideS, int64_t batch,
                   cudaStream_t stream, uint32_t outputs = dmv::kOutBoth,
-                  const Rank2 *rank2 = nullptr, int32_t variant = -1) {
+                  const Rank2 *rank2 = nullptr, int32_t variant = -1,
+                  Deferred *defer = nullptr, bool reverse = false) {
     using Acc = typename dmv::Traits<T>::Acc;
     static_assert(sizeof(Acc) == sizeof(Out), "accumulator and output widths differ");
     constexpr bool kIntPath = std::is_same<T, int32_t>::value;
@@ -900,6 +914,7 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     const bool want_q = (outputs & dmv::kOutQ) != 0, want_s = (outputs & dmv::kOutS) != 0;
     g_last_variant = -1;
     g_last_kernel = -1;
+    if (defer != nullptr) defer->used = false;
     dualmv_status st = validate(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ,
                                 s, strideS, batch, outputs);
     if (st != DUALMV_SUCCESS || batch == 0) return st;
@@ -1069,13 +1084,22 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
             if constexpr (!kIntPath) {
                 // Single-sided products (one problem, float or double).
                 const bool only_q = outputs == dmv::kOutQ;
+                // reverse: a rows-only pass that follows a pass over the same
+                // A walks each CTA's tiles backwards (see Deferred).
+                const bool rev = reverse && only_q;
                 if (kind == Kind::kF64e) {
                     if constexpr (std::is_same<T, double>::value)
-                        e = only_q ? launch_f64e<false, dmv::kOutQ>(map, prm, pl, dev, stream)
-                                   : launch_f64e<false, dmv::kOutS>(map, prm, pl, dev, stream);
+                        e = rev ? launch_f64e<false, dmv::kOutQ, kF64eWarps, kF64eRpw, kF64eStages,
+                                              kF64eNativeCols, kF64eSelf, kF64ePack, kF64eBand,
+                                              true>(map, prm, pl, dev, stream)
+                            : only_q ? launch_f64e<false, dmv::kOutQ>(map, prm, pl, dev, stream)
+                                     : launch_f64e<false, dmv::kOutS>(map, prm, pl, dev, stream);
                 } else if (kind == Kind::kTma) {
-                    e = only_q ? launch_stream<T, true, false, dmv::kOutQ>(map, prm, pl, dev, stream)
-                               : launch_stream<T, true, false, dmv::kOutS>(map, prm, pl, dev, stream);
+                    e = rev ? launch_stream<T, true, false, dmv::kOutQ, false, kWarps,
+                                            default_rpw<T>(), kStages, true>(map, prm, pl, dev,
+                                                                              stream)
+                        : only_q ? launch_stream<T, true, false, dmv::kOutQ>(map, prm, pl, dev, stream)
+                                 : launch_stream<T, true, false, dmv::kOutS>(map, prm, pl, dev, stream);
                 } else {
                     e = only_q ? launch_stream<T, false, false, dmv::kOutQ>(map, prm, pl, dev, stream)
                                : launch_stream<T, false, false, dmv::kOutS>(map, prm, pl, dev, stream);
@@ -1100,6 +1124,13 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     }
     if (e == cudaSuccess) g_last_kernel = kernel_kind;
     if (e == cudaSuccess && ev_stop) e = cudaEventRecord(ev_stop, stream);
+    if (e == cudaSuccess && defer != nullptr && !kAtomicOut) {
+        defer->used = true;
+        defer->prm = prm;
+        defer->ws = ws;
+        defer->chunks = combine_chunks(prm.bands);
+        return DUALMV_SUCCESS;
+    }
     if (e == cudaSuccess && !kAtomicOut) e = launch_combine<Acc>(prm, stream);
     cudaError_t ef = ws ? cudaFreeAsync(ws, stream) : cudaSuccess;
     if (e != cudaSuccess) return cuda_fail(e);
@@ -1359,10 +1390,81 @@ dualmv_status atax_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *x
 // so a columns-only and a rows-only pass of the plain kernels (double-float
 // for fp64) and four dot products give x and w without any per-element
 // update.  Each term's error stays within the bar of A_hat's magnitudes.
+// The general shape (M, N > 0): five kernels.  The u . y dot products; the
+// columns-only pass, which leaves its partials for gemver_x3_kernel, which
+// adds them and updates x; the rows-only pass, which leaves its partials for
+// gemver_w3_kernel, which adds them and updates w.  (Seven before: each pass
+// had its own combine kernel.  Forming u . y inside the x kernel, every
+// block for itself, put 130 thousand fp64 operations on each SM's narrow
+// FP64 pipe and doubled the call.)
+template <typename T>
+dualmv_status gemver_factored_fused(int64_t M, int64_t N, T alpha, T beta, const T *A,
+                                    int64_t lda, const T *u1, const T *v1, const T *u2,
+                                    const T *v2, T *w, T *x, const T *y, const T *z,
+                                    cudaStream_t stream) {
+    T *s = nullptr, *t = nullptr;
+    // [side][2 products][kDotChunks][sum, error]: u . y, then v . x
+    double *part = nullptr;
+    dualmv_status st = pool_alloc(&s, N, stream);
+    if (st == DUALMV_SUCCESS) st = pool_alloc(&t, M, stream);
+    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * 2 * dmv::kDotChunks, stream);
+    double *part_u = part, *part_v = part ? part + 2 * 2 * dmv::kDotChunks : nullptr;
+    cudaError_t e = cudaSuccess;
+    Deferred ds, dq;
+    if (st == DUALMV_SUCCESS)
+        e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks), dim3(256),
+                             0, stream, u1, u2, y, M, part_u);
+    if (st == DUALMV_SUCCESS && e == cudaSuccess)  // s = A^T y, left as partials
+        st = run<T, T>(M, N, A, lda, 0, nullptr, 0, y, 0, nullptr, 0, s, 0, 1, stream,
+                       dmv::kOutS, nullptr, -1, &ds);
+    if (st == DUALMV_SUCCESS && e == cudaSuccess) {
+        if (!ds.used) ds.prm.s = s;
+        e = launch_dependent(dmv::gemver_x3_kernel<T>, dim3(dmv::kDotChunks), dim3(256), 0,
+                             stream, ds.prm, ds.used ? 0 : 1, (const double *)part_u, x, v1,
+                             v2, z, N, beta, part_v);
+    }
+    if (ds.ws != nullptr) {
+        cudaError_t ef = cudaFreeAsync(ds.ws, stream);
+        if (e == cudaSuccess) e = ef;
+    }
+    // t = A x, left as partials; each CTA walks its tiles backwards, so it
+    // starts on those the columns-only pass read last (still in L2).
+    if (st == DUALMV_SUCCESS && e == cudaSuccess)
+        st = run<T, T>(M, N, A, lda, 0, x, 0, nullptr, 0, t, 0, nullptr, 0, 1, stream,
+                       dmv::kOutQ, nullptr, -1, &dq, true);
+    if (st == DUALMV_SUCCESS && e == cudaSuccess) {
+        if (!dq.used) dq.prm.q = t;
+        const int direct = (!dq.used || dq.prm.bands == 1) ? 1 : 0;
+        const int64_t rows = 256 / dq.chunks;
+        const int64_t bw = (M + rows - 1) / rows;
+        if (bw > INT32_MAX) e = cudaErrorInvalidConfiguration;
+        else
+            e = launch_dependent(dmv::gemver_w3_kernel<T>, dim3((unsigned)bw), dim3(256), 0,
+                                 stream, dq.prm, direct, dq.chunks, w, u1, u2,
+                                 (const double *)part_v, M, alpha);
+    }
+    if (dq.ws != nullptr) {
+        cudaError_t ef = cudaFreeAsync(dq.ws, stream);
+        if (e == cudaSuccess) e = ef;
+    }
+    if (st == DUALMV_SUCCESS && e != cudaSuccess) st = cuda_fail(e);
+    void *bufs[3] = {s, t, part};
+    for (void *bp : bufs) {
+        if (bp == nullptr) continue;
+        cudaError_t ef = cudaFreeAsync(bp, stream);
+        if (st == DUALMV_SUCCESS && ef != cudaSuccess) st = cuda_fail(ef);
+    }
+    return st;
+}
+
 template <typename T>
 dualmv_status gemver_factored(int64_t M, int64_t N, T alpha, T beta, const T *A, int64_t lda,
                               const T *u1, const T *v1, const T *u2, const T *v2, T *w, T *x,
                               const T *y, const T *z, cudaStream_t stream) {
+    if (M > 0 && N > 0)
+        return gemver_factored_fused<T>(M, N, alpha, beta, A, lda, u1, v1, u2, v2, w, x, y, z,
+                                        stream);
+    // An empty dimension: the vector kernels alone (each pass zero-fills).
     T *s = nullptr, *t = nullptr;
     // [side][2 products][kDotChunks][sum, error]: u . y, then v . x
     double *part = nullptr;

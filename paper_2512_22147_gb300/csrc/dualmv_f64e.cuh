@@ -298,10 +298,12 @@ struct F64eLayout {
 // NPH = 0) and dualmv_stream_f64e_phased_kernel (a pair of maps per row
 // phase, tmaps[0 .. 2 NPH - 1]; see dualmv_stream_phased_kernel).
 template <int W, int RPW, int STAGES, int BAND, bool kBatched3d, int kOut, int NC, bool kSelf,
-          bool kPack, int NPH>
+          bool kPack, int NPH, bool kRev = false>
 __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params &prm) {
     constexpr bool kQ = (kOut & kOutQ) != 0;  // row sums q = A p
     constexpr bool kS = (kOut & kOutS) != 0;  // column sums s = A^T r
+    // kRev: each CTA walks its tile range backwards (as stream_body's).
+    static_assert(!kRev || kOut == kOutQ, "backward walk: rows-only passes");
     using T = double;
     using Acc = double;
     using Vec = double2;
@@ -358,7 +360,7 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
             int issued = 0;
             int partial_w = 0;
             TileCursor32 cur;
-            cur.init(t0, S, NB);
+            cur.init(kRev ? t1 - 1 : t0, S, NB);
             int stage = 0;
             uint32_t phase = 0;
             for (int k = 0; k < ntiles; ++k) {
@@ -382,7 +384,10 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
                 }
                 if (!ok) break;
                 issued = k + 1;
-                cur.advance(S, NB);
+                if constexpr (kRev)
+                    cur.retreat(S, NB);
+                else
+                    cur.advance(S, NB);
                 if (++stage == STAGES) {
                     stage = 0;
                     phase ^= 1u;
@@ -444,7 +449,7 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
     bool ok = true;
 
     TileCursor32 cur;
-    cur.init(t0, S, NB);
+    cur.init(kRev ? t1 - 1 : t0, S, NB);
     T r_next = T(0);
     {
         const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
@@ -478,13 +483,16 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
         } else {
             tma_load_2d(dst, &tmaps[0], x, y, fb, pol);
         }
-        ld.advance(S, NB);
+        if constexpr (kRev)
+            ld.retreat(S, NB);
+        else
+            ld.advance(S, NB);
         ++issued;
     };
     if constexpr (kSelf) {
         if (lane == 0) {
             pol = policy_evict_first();
-            ld.init(t0, S, NB);
+            ld.init(kRev ? t1 - 1 : t0, S, NB);
             for (int st = 0; st < STAGES && st < ntiles; ++st) issue(st);
         }
     }
@@ -512,14 +520,18 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
         const int64_t col0 = band * BAND;
         const int64_t row0 = stripe * BM + (int64_t)warp * RPW;
         const T rmine = r_next;
-        cur.advance(S, NB);
+        if constexpr (kRev)
+            cur.retreat(S, NB);
+        else
+            cur.advance(S, NB);
         if (kS && k + 1 < ntiles) {
             const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
             r_next = (lane < RPW && row < prm.M) ? rg[cur.b * prm.strideR + row] : T(0);
         }
 
-        if (k == 0 || stripe == 0) seg_start_stripe = stripe;
-        if (kQ && (k == 0 || stripe == 0)) {  // new segment: split this band's p
+        const bool seg_start = k == 0 || stripe == (kRev ? S - 1 : 0);
+        if (seg_start) seg_start_stripe = stripe;
+        if (kQ && seg_start) {  // new segment: split this band's p
             const T *pb = pg + b * prm.strideP;
             p_bad = false;
 #pragma unroll
@@ -852,10 +864,11 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
 }
 
 template <int W, int RPW, int STAGES, int BAND, bool kBatched3d, int kOut = kOutBoth,
-          int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = false, bool kPack = false>
+          int NC = DUALMV_F64E_NATIVE_COLS, bool kSelf = false, bool kPack = false,
+          bool kRev = false>
 __global__ void __launch_bounds__((W + (kSelf ? 0 : 1)) * 32, 1)
 dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
-    f64e_body<W, RPW, STAGES, BAND, kBatched3d, kOut, NC, kSelf, kPack, 0>(&tmap, prm);
+    f64e_body<W, RPW, STAGES, BAND, kBatched3d, kOut, NC, kSelf, kPack, 0, kRev>(&tmap, prm);
 }
 
 // fp64 rows whose stride or base is not 16-byte aligned (odd lda): the same

@@ -339,6 +339,17 @@ struct TileCursor {
             }
         }
     }
+    // The tile before (for a CTA that walks its range backwards).
+    __device__ __forceinline__ void retreat(int64_t S, int64_t bands) {
+        if (stripe-- == 0) {
+            stripe = S - 1;
+            --g;
+            if (band-- == 0) {
+                band = bands - 1;
+                --b;
+            }
+        }
+    }
 };
 
 // The same in 32 bits, for kernels whose launch guarantees fewer than 2^31
@@ -358,6 +369,16 @@ struct TileCursor32 {
             if (++band == bands) {
                 band = 0;
                 ++b;
+            }
+        }
+    }
+    __device__ __forceinline__ void retreat(int S, int bands) {
+        if (stripe-- == 0) {
+            stripe = S - 1;
+            --g;
+            if (band-- == 0) {
+                band = bands - 1;
+                --b;
             }
         }
     }
@@ -396,10 +417,14 @@ struct SmemLayout {
 // The kernel body, shared by dualmv_stream_kernel (one tensor map, NPH = 0)
 // and dualmv_stream_phased_kernel (NPH phase maps, tmaps[0 .. NPH - 1]).
 template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d, int kOut,
-          bool kRank2, int NPH>
+          bool kRank2, int NPH, bool kRev = false>
 __device__ __forceinline__ void stream_body(const CUtensorMap *tmaps, const Params &prm) {
     using Acc = typename Traits<T>::Acc;
     static_assert(!kRank2 || !std::is_same<T, int32_t>::value, "rank-2 update: floats only");
+    // kRev: each CTA walks its tile range backwards (last tile first), so a
+    // pass that follows another over the same A starts on the tiles that
+    // pass read last, which may still be in L2.  Rows-only passes only.
+    static_assert(!kRev || kOut == kOutQ, "backward walk: rows-only passes");
     constexpr bool kQ = (kOut & kOutQ) != 0;  // row sums q = A p
     constexpr bool kS = (kOut & kOutS) != 0;  // column sums s = A^T r
     // Integer sums are exact modulo 2^64 in any order, so the int32 path adds
@@ -465,7 +490,7 @@ __device__ __forceinline__ void stream_body(const CUtensorMap *tmaps, const Para
                 bool ok = true;
                 int64_t issued = 0;
                 TileCursor cur;
-                cur.init(t0, S, prm.bands);
+                cur.init(kRev ? t1 - 1 : t0, S, prm.bands);
                 int stage = 0;
                 uint32_t phase = 0;  // parity of the ring pass, flips each pass
                 for (int64_t k = 0; k < ntiles; ++k) {
@@ -494,7 +519,10 @@ __device__ __forceinline__ void stream_body(const CUtensorMap *tmaps, const Para
                         tma_load_2d(dst, &tmaps[0], x, y, fb, pol);
                     }
                     issued = k + 1;
-                    cur.advance(S, prm.bands);
+                    if constexpr (kRev)
+                        cur.retreat(S, prm.bands);
+                    else
+                        cur.advance(S, prm.bands);
                     if (++stage == STAGES) {
                         stage = 0;
                         phase ^= 1u;
@@ -532,7 +560,7 @@ __device__ __forceinline__ void stream_body(const CUtensorMap *tmaps, const Para
     bool ok = true;
 
     TileCursor cur;
-    cur.init(t0, S, prm.bands);
+    cur.init(kRev ? t1 - 1 : t0, S, prm.bands);
     // r for this warp's RPW rows of the next tile (lane i < RPW holds row
     // row0 + i), loaded one tile ahead so its latency hides behind a tile.
     T r_next = T(0), u1_next = T(0), u2_next = T(0);
@@ -559,7 +587,10 @@ __device__ __forceinline__ void stream_body(const CUtensorMap *tmaps, const Para
         const int64_t col0 = band * kBandCols;
         const int64_t row0 = stripe * BM + (int64_t)warp * RPW;
         const T rmine = r_next, u1mine = u1_next, u2mine = u2_next;
-        cur.advance(S, prm.bands);
+        if constexpr (kRev)
+            cur.retreat(S, prm.bands);
+        else
+            cur.advance(S, prm.bands);
         if (kS && k + 1 < ntiles) {
             const int64_t row = cur.stripe * BM + (int64_t)warp * RPW + lane;
             r_next = (lane < RPW && row < prm.M) ? rg[cur.b * prm.strideR + row] : T(0);
@@ -581,8 +612,11 @@ __device__ __forceinline__ void stream_body(const CUtensorMap *tmaps, const Para
                 }
         }
 
-        if (k == 0 || stripe == 0) seg_start_stripe = stripe;
-        if (kQ && (k == 0 || stripe == 0)) {  // a new segment: this band's p
+        // A new segment: the CTA's first tile, or a band entered (at its
+        // first stripe walking forwards, its last walking backwards).
+        const bool seg_start = k == 0 || stripe == (kRev ? S - 1 : 0);
+        if (seg_start) seg_start_stripe = stripe;
+        if (kQ && seg_start) {  // a new segment: this band's p
             const T *pb = pg + b * prm.strideP;
 #pragma unroll
             for (int v = 0; v < VPL; ++v)
@@ -801,11 +835,11 @@ __device__ __forceinline__ void stream_body(const CUtensorMap *tmaps, const Para
 }
 
 template <typename T, int W, int RPW, int STAGES, bool kTma, bool kBatched3d,
-          int kOut = kOutBoth, bool kRank2 = false>
+          int kOut = kOutBoth, bool kRank2 = false, bool kRev = false>
 __global__ void __launch_bounds__((W + (kTma ? 1 : 0)) * 32,
                                   (!kTma && std::is_same<T, int32_t>::value) ? 2 : 1)
 dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
-    stream_body<T, W, RPW, STAGES, kTma, kBatched3d, kOut, kRank2, 0>(&tmap, prm);
+    stream_body<T, W, RPW, STAGES, kTma, kBatched3d, kOut, kRank2, 0, kRev>(&tmap, prm);
 }
 
 // The same kernel for one problem whose row stride or base is not 16-byte
@@ -817,6 +851,57 @@ template <typename T, int W, int RPW, int STAGES, int NPH>
 __global__ void __launch_bounds__((W + 1) * 32, 1)
 dualmv_stream_phased_kernel(const __grid_constant__ TmapSet maps, const Params prm) {
     stream_body<T, W, RPW, STAGES, true, false, kOutBoth, false, NPH>(maps.m, prm);
+}
+
+// ------------------------------------------------------- combine arithmetic --
+// The two sums the combine kernel forms, as device functions, so that a kernel
+// that takes over a pass's combine (GEMVER's vector updates) adds the
+// partials in the same order and gets the same bits.
+
+// Output i of problem b from its band partials: C interleaved chunks (chunk y
+// adds bands y, y + C, ... in ascending order), then the chunks in order.
+template <typename Acc>
+__device__ __forceinline__ Acc q_band_sum(const Params &prm, int64_t b, int64_t i, int C) {
+    const Acc *base = static_cast<const Acc *>(prm.q_ws) + (b * prm.bands) * prm.M + i;
+    Acc tot = Acc(0);
+    for (int y = 0; y < C; ++y) {
+        Acc acc = Acc(0);
+        int64_t k = y;
+        if (k < prm.bands) {
+            acc = base[k * prm.M];
+            k += C;
+        }
+        for (; k < prm.bands; k += C) acc = acc + base[k * prm.M];
+        tot = y == 0 ? acc : tot + acc;
+    }
+    return tot;
+}
+
+// The CTAs holding stripes of global band g (b * bands + band): c_lo .. c_hi.
+// When they are one CTA, that CTA wrote the band's s directly.
+__device__ __forceinline__ void band_ctas_of(const Params &prm, int64_t g, int64_t &c_lo,
+                                             int64_t &c_hi) {
+    const int64_t S = prm.stripes;
+    c_lo = cta_of_tile(g * S, prm.tiles, prm.grid);
+    c_hi = cta_of_tile(g * S + S - 1, prm.tiles, prm.grid);
+}
+
+// Column col of global band g (split between CTAs c_lo < c_hi): its segment
+// partials added in CTA order.  CTA cc's segment of band g is g minus the
+// band of its first tile; every CTA after c_lo starts inside band g, so the
+// band is its segment 0, and only c_lo's segment needs a division: the loads
+// do not wait on one another (a running segment count between them had made
+// the combine of the 1024^2 workload take 5 of its 8 us).
+template <typename Acc>
+__device__ __forceinline__ Acc s_segment_sum(const Params &prm, int64_t g, int col, int64_t c_lo,
+                                             int64_t c_hi) {
+    const Acc *src = static_cast<const Acc *>(prm.s_ws) + col;
+    const int64_t seg0 = g - ((c_lo * prm.tiles) / prm.grid) / prm.stripes;
+    const int64_t pitch = prm.max_seg * prm.band_cols;
+    Acc acc = src[c_lo * pitch + seg0 * prm.band_cols];
+#pragma unroll 8
+    for (int64_t cc = c_lo + 1; cc <= c_hi; ++cc) acc = acc + src[cc * pitch];
+    return acc;
 }
 
 // --------------------------------------------------------- combine kernel --
@@ -843,7 +928,6 @@ dualmv_combine_kernel(const Params prm, int64_t q_blocks, int q_chunks) {
     pdl_wait();
     __shared__ Acc part[256];
     const Acc *qw = static_cast<const Acc *>(prm.q_ws);
-    const Acc *sw = static_cast<const Acc *>(prm.s_ws);
     if ((int64_t)blockIdx.x < q_blocks) {  // (q_blocks is 0 unless q is computed)
         const int C = q_chunks, R = 256 / C;
         const int x = threadIdx.x % R, y = threadIdx.x / R;
@@ -872,28 +956,16 @@ dualmv_combine_kernel(const Params prm, int64_t q_blocks, int q_chunks) {
         }
         return;
     }
-    const int64_t T_ = prm.tiles, G = prm.grid, S = prm.stripes;
     const int64_t g = (int64_t)blockIdx.x - q_blocks;  // b * bands + band
     const int64_t b = g / prm.bands, band = g - b * prm.bands;
-    const int64_t c_lo = cta_of_tile(g * S, T_, G);
-    const int64_t c_hi = cta_of_tile(g * S + S - 1, T_, G);
+    int64_t c_lo, c_hi;
+    band_ctas_of(prm, g, c_lo, c_hi);
     if (c_lo == c_hi) return;  // written directly by the stream kernel
     const int col = threadIdx.x;
     if (col >= prm.band_cols) return;
     const int64_t j = band * prm.band_cols + col;
     if (j >= prm.N) return;
-    // CTA cc's segment of band g is g minus the band of its first tile.  For
-    // every CTA after c_lo, band g is its first band (its range starts inside
-    // band g): segment 0.  So only c_lo's segment needs a division, and the
-    // loads do not wait on one another (a running segment count between
-    // them had made the small workload's combine take 5 of its 8 us).
-    const int64_t seg0 = g - ((c_lo * T_) / G) / S;
-    const Acc *src = sw + col;
-    const int64_t pitch = prm.max_seg * prm.band_cols;
-    Acc acc = src[c_lo * pitch + seg0 * prm.band_cols];
-#pragma unroll 8
-    for (int64_t cc = c_lo + 1; cc <= c_hi; ++cc) acc = acc + src[cc * pitch];
-    static_cast<Acc *>(prm.s)[b * prm.strideS + j] = acc;
+    static_cast<Acc *>(prm.s)[b * prm.strideS + j] = s_segment_sum<Acc>(prm, g, col, c_lo, c_hi);
 }
 
 // Zeroes q and s (strided batches) ahead of a stream kernel that adds into

@@ -208,4 +208,91 @@ __global__ void __launch_bounds__(256) gemver_w2_kernel(T *w, const T *t, const 
     }
 }
 
+// ---- GEMVER's vector steps with the passes' combine folded in -----------
+// The columns-only and rows-only passes leave their partial sums in their
+// workspace, and these kernels add them (in the combine kernel's order, so
+// with its bits) where they are used: GEMVER then runs five kernels instead
+// of seven.
+
+// gemver_x2_kernel with s = A^T y from the columns-only pass's partials
+// (ps: that pass's parameters; s_direct: the pass wrote s itself).
+template <typename T>
+__global__ void __launch_bounds__(256) gemver_x3_kernel(const Params ps, int s_direct,
+                                                        const double *part_u, T *x, const T *v1,
+                                                        const T *v2, const T *z, int64_t n,
+                                                        T beta, double *part_v) {
+    pdl_launch_dependents();
+    pdl_wait();
+    __shared__ T dd[2];
+    __shared__ double hs[512], hc[512];
+    dots2_final_block<T>(part_u, hs, hc, dd);
+    const T d0 = dd[0], d1 = dd[1];
+    const T *sv = static_cast<const T *>(ps.s);
+    const int chunk = blockIdx.x;
+    const int64_t k0 = chunk * n / kDotChunks, k1 = (chunk + 1) * n / kDotChunks;
+    double s1 = 0.0, c1 = 0.0, s2 = 0.0, c2 = 0.0;
+    for (int64_t i = k0 + threadIdx.x; i < k1; i += 256) {
+        T si;
+        int64_t c_lo = 0, c_hi = 0;
+        const int64_t band = i / ps.band_cols;
+        if (!s_direct) band_ctas_of(ps, band, c_lo, c_hi);
+        if (s_direct || c_lo == c_hi)
+            si = sv[i];
+        else
+            si = s_segment_sum<T>(ps, band, (int)(i - band * ps.band_cols), c_lo, c_hi);
+        const T inner = fma(v2[i], d1, fma(v1[i], d0, si));
+        const T xn = fma(beta, inner, x[i]) + z[i];
+        x[i] = xn;
+        dot2_step((double)v1[i], (double)xn, s1, c1);
+        dot2_step((double)v2[i], (double)xn, s2, c2);
+    }
+    dot2_block_store2(s1, c1, s2, c2, hs, hc, part_v, chunk, kDotChunks + chunk);
+}
+
+// w = w + alpha (t + u1 e0 + u2 e1) with t = A x from the rows-only pass's
+// band partials, added as the combine kernel adds them: C threads per row,
+// thread y adding bands y, y + C, ..., then the C chunk sums in order (pq:
+// that pass's parameters; q_direct: the pass wrote t itself).  e0 = v1 . x
+// and e1 = v2 . x from their chunk sums.  Blocks of 256 threads over
+// 256 / C rows each.  Launched as a programmatic dependent of the pass.
+template <typename T>
+__global__ void __launch_bounds__(256) gemver_w3_kernel(const Params pq, int q_direct, int C,
+                                                        T *w, const T *u1, const T *u2,
+                                                        const double *part, int64_t m, T alpha) {
+    pdl_launch_dependents();
+    pdl_wait();
+    __shared__ T dd[2];
+    __shared__ double hs[2 * kDotChunks], hc[2 * kDotChunks];
+    __shared__ T chunk_sum[256];
+    dots2_final_block<T>(part, hs, hc, dd);
+    const T d0 = dd[0], d1 = dd[1];
+    const int R = 256 / C, xr = threadIdx.x % R, y = threadIdx.x / R;
+    const int64_t i = (int64_t)blockIdx.x * R + xr;
+    const bool valid = i < m;
+    T acc = T(0);
+    if (valid && !q_direct) {
+        const T *base = static_cast<const T *>(pq.q_ws) + i;
+        int64_t k = y;
+        if (k < pq.bands) {
+            acc = base[k * pq.M];
+            k += C;
+        }
+#pragma unroll 4
+        for (; k < pq.bands; k += C) acc = acc + base[k * pq.M];
+    }
+    chunk_sum[threadIdx.x] = acc;
+    __syncthreads();
+    if (y == 0 && valid) {
+        T ti;
+        if (q_direct) {
+            ti = static_cast<const T *>(pq.q)[i];
+        } else {
+            ti = chunk_sum[xr];
+            for (int yy = 1; yy < C; ++yy) ti = ti + chunk_sum[yy * R + xr];
+        }
+        const T inner = fma(u2[i], d1, fma(u1[i], d0, ti));
+        w[i] = fma(alpha, inner, w[i]);
+    }
+}
+
 }  // namespace dmv

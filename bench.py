@@ -460,6 +460,7 @@ def streaming_kernel_name(dm, w):
             dm.DUALMV_KERNEL_PHASED: ("dualmv_stream_f64e_phased_kernel" if w.dtype == "f64"
                                       else "dualmv_stream_phased_kernel"),
             dm.DUALMV_KERNEL_PLAIN: "dualmv_stream_kernel (plain loads)",
+            dm.DUALMV_KERNEL_CLUSTER: "dualmv_small_cluster_kernel (one cluster of 16 CTAs)",
         }.get(kind, kernel_name)
         if w.batched and kind in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_F64E):
             family = {dm.DUALMV_KERNEL_STREAM: "dualmv_stream_kernel",
@@ -473,6 +474,8 @@ def launches_per_call(torch, dm, inputs, w, dev) -> int:
                           inputs.OUT_BYTES[w.dtype],
                           torch.cuda.get_device_properties(dev).multi_processor_count)
     n = 1 + (1 if (plan.bands > 1 or plan.grid > 1) else 0)
+    if w.op == "bicg" and dm.dualmv_last_kernel() == dm.DUALMV_KERNEL_CLUSTER:
+        n = 1   # one cluster computes both outputs, no combine kernel
     if w.op == "gesummv":   # two row passes (stream + combine each) + epilogue
         return 2 * n + 1
     if w.op == "atax":      # a row pass and a column pass

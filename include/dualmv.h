@@ -339,7 +339,9 @@ enum {
                               /* aligned: TMA through one pair of tensor   */
                               /* maps per row phase (no variants; fp64 in  */
                               /* double-float arithmetic)                  */
-    DUALMV_KERNEL_PLAIN = 4   /* plain global loads (no variants)          */
+    DUALMV_KERNEL_PLAIN = 4,  /* plain global loads (no variants)          */
+    DUALMV_KERNEL_CLUSTER = 5 /* small fp32 problems: one cluster of 16    */
+                              /* CTAs does the whole call (no variants)   */
 };
 typedef struct dualmv_variant_t {
     int32_t index;          /* position in its dtype's table              */
@@ -394,7 +396,12 @@ int32_t dualmv_last_variant(void);
  * and the passes inside GESUMMV, ATAX and GEMVER), or -1 if it ran none (an
  * empty problem or an error).  PHASED: rows whose stride or base the TMA
  * unit cannot take as one tensor, for one dual product (fp64 unless
- * DUALMV_PATH_TMA_NATIVE_F64 is set); PLAIN: the remaining unaligned cases.  Instrumentation for tests and benchmarks. */
+ * DUALMV_PATH_TMA_NATIVE_F64 is set); PLAIN: the remaining unaligned cases;
+ * CLUSTER: one fp32 dual product of at most 8 MiB with 256 <= N <= 2048
+ * (N and lda multiples of 4, A and p 16-byte aligned), under
+ * DUALMV_PATH_AUTO and with no variant forced or tuned for it, which one
+ * cluster of 16 CTAs computes without workspace or combine kernel.
+ * Instrumentation for tests and benchmarks. */
 int32_t dualmv_last_kernel(void);
 
 /* Trimmed mean of Eq. 3: the R values sorted, the k smallest and k largest

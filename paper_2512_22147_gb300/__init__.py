@@ -30,7 +30,7 @@ _BINDING_NAMES = {
     "dualmv_last_variant", "TuneStep", "dualmv_atax_set_two_pass",
     "dualmv_gemver_set_onthefly", "dualmv_last_kernel", "DUALMV_KERNEL_PHASED",
     "DUALMV_KERNEL_PLAIN", "dualmv_atax_last_path", "DUALMV_ATAX_ONE_READ",
-    "DUALMV_ATAX_TWO_PASS", "dualmv_read_probe", "dualmv_pool_usage",
+    "DUALMV_ATAX_TWO_PASS", "dualmv_read_probe", "dualmv_pool_usage", "DUALMV_KERNEL_CLUSTER",
 }
 _API_NAMES = {"dualmv", "device_fault", "gesummv", "atax", "gemver", "tune", "variants"}
 

@@ -40,6 +40,7 @@ DUALMV_KERNEL_F64E = 1
 DUALMV_KERNEL_WIDE = 2
 DUALMV_KERNEL_PHASED = 3
 DUALMV_KERNEL_PLAIN = 4
+DUALMV_KERNEL_CLUSTER = 5
 DUALMV_ATAX_TWO_PASS = 0
 DUALMV_ATAX_ONE_READ = 1
 

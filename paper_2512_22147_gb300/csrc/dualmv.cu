@@ -26,6 +26,7 @@
 #include "dualmv_atax_f64.cuh"
 #include "dualmv_ops.cuh"
 #include "dualmv_probe.cuh"
+#include "dualmv_small.cuh"
 
 namespace {
 
@@ -876,6 +877,67 @@ const Variant *pick_variant(int32_t dtype, int64_t M, int64_t N, const void *A, 
     return &(*tab)[index];
 }
 
+// True when the call names a variant, or one is forced or tuned for this
+// shape (even entry 0): such calls run the streaming kernels as chosen.
+bool explicit_variant(int32_t dtype, int64_t M, int64_t N, int64_t lda, int32_t index) {
+    if (index >= 0) return true;
+    if (variant_table(dtype) == nullptr) return false;
+    if (g_forced_variant[dtype].load(std::memory_order_relaxed) >= 0) return true;
+    return tuned_lookup(dtype, M, N, lda) >= 0;
+}
+
+// ---- small fp32 problems: one thread-block cluster (dualmv_small.cuh) ----
+// A call of at most kSmallMaxBytes of A, 256 <= N <= 2048, runs as one
+// cluster of 16 CTAs with no workspace and no combine kernel: on the 1024^2
+// workload the streaming kernel and its combine take 6.7 us hot in a graph.
+constexpr int64_t kSmallMaxBytes = 8ll << 20;
+
+struct SmallClusterCache {
+    std::mutex mu;
+    int ok[2][kMaxDevices] = {};  // 0 unknown, 1 placeable, -1 not
+};
+SmallClusterCache g_small_cache;
+
+template <int VPL>
+cudaError_t launch_small_cluster(const Params &prm, int dev, cudaStream_t stream, bool *done) {
+    *done = false;
+    constexpr auto kern = dmv::dualmv_small_cluster_kernel<VPL>;
+    constexpr int smem = dmv::SmallLayout<VPL>::kTotal;
+    cudaLaunchConfig_t cfg;
+    std::memset(&cfg, 0, sizeof cfg);
+    cfg.gridDim = dim3(dmv::kSmallCluster);
+    cfg.blockDim = dim3(dmv::kSmallWarps * 32);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = dmv::kSmallCluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const int slot = VPL == 8 ? 0 : 1;
+    {
+        std::lock_guard<std::mutex> lk(g_small_cache.mu);
+        if (g_small_cache.ok[slot][dev] == 0) {
+            int clusters = 0;
+            cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 smem);
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+            if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg);
+            if (e != cudaSuccess) {  // no such cluster here: the streaming kernels
+                (void)cudaGetLastError();
+                clusters = 0;
+            }
+            g_small_cache.ok[slot][dev] = clusters > 0 ? 1 : -1;
+        }
+        if (g_small_cache.ok[slot][dev] < 0) return cudaSuccess;
+    }
+    *done = true;
+    return cudaLaunchKernelEx(&cfg, kern, prm);
+}
+
 // GEMVER's rank-2 update, applied on the fly by a single-sided pass.
 // A pass whose combine a later kernel takes over: run() leaves its partial
 // sums in the workspace, launches no combine kernel and does not free the
@@ -937,6 +999,34 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     DeviceState *ds = nullptr;
     e = device_state(dev, &ds);
     if (e != cudaSuccess) return cuda_fail(e);
+
+    // Small fp32 dual products: one thread-block cluster, no workspace.
+    if constexpr (std::is_same<T, float>::value) {
+        if (batch == 1 && outputs == dmv::kOutBoth && rank2 == nullptr &&
+            g_path == DUALMV_PATH_AUTO && N >= 256 && N <= 2048 && N % 4 == 0 &&
+            lda % 4 == 0 && M * N * (int64_t)sizeof(T) <= kSmallMaxBytes &&
+            reinterpret_cast<uintptr_t>(A) % 16 == 0 && reinterpret_cast<uintptr_t>(p) % 16 == 0 &&
+            !explicit_variant(DUALMV_DTYPE_F32, M, N, lda, variant)) {
+            Params sp;
+            std::memset(&sp, 0, sizeof sp);
+            sp.A = A; sp.lda = lda; sp.p = p; sp.r = r; sp.q = q; sp.s = s;
+            sp.M = M; sp.N = N; sp.batch = 1; sp.outputs = dmv::kOutBoth; sp.ph_n = 1;
+            cudaEvent_t ev0 = g_kernel_ev_start, ev1 = g_kernel_ev_stop;
+            bool done = false;
+            e = ev0 ? cudaEventRecord(ev0, stream) : cudaSuccess;
+            if (e == cudaSuccess)
+                e = N <= 1024 ? launch_small_cluster<8>(sp, dev, stream, &done)
+                              : launch_small_cluster<16>(sp, dev, stream, &done);
+            if (e != cudaSuccess) return cuda_fail(e);
+            if (done) {
+                g_kernel_ev_start = g_kernel_ev_stop = nullptr;
+                if (ev1) e = cudaEventRecord(ev1, stream);
+                if (e != cudaSuccess) return cuda_fail(e);
+                g_last_kernel = DUALMV_KERNEL_CLUSTER;
+                return DUALMV_SUCCESS;
+            }
+        }
+    }
 
     // Path choice: TMA needs a 16-byte aligned base, 16-byte multiple
     // strides and 32-bit coordinates.

@@ -321,7 +321,8 @@ def test_unaligned_rows_take_phased_maps(dtype, lda_mod4, base):
         kind = dm.dualmv_last_kernel()
         if eff % per16 == 0 and base % per16 == 0:
             assert kind in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_WIDE,
-                            dm.DUALMV_KERNEL_F64E), (M, N, lda, base, kind)
+                            dm.DUALMV_KERNEL_F64E, dm.DUALMV_KERNEL_CLUSTER), (M, N, lda, base,
+                                                                               kind)
         elif M >= nph:
             assert kind == dm.DUALMV_KERNEL_PHASED, (M, N, lda, base, kind)
         else:
@@ -386,6 +387,12 @@ def test_last_kernel_reports_each_path():
         dm.dualmv_set_path(old)
     A, p, r = _make("f32", 96, 512, 512, 93)
     dm.dualmv(A, p, r)
-    assert dm.dualmv_last_kernel() == dm.DUALMV_KERNEL_STREAM
+    assert dm.dualmv_last_kernel() == dm.DUALMV_KERNEL_CLUSTER
+    old = dm.dualmv_set_path(dm.DUALMV_PATH_TMA)
+    try:
+        dm.dualmv(A, p, r)
+        assert dm.dualmv_last_kernel() == dm.DUALMV_KERNEL_STREAM
+    finally:
+        dm.dualmv_set_path(old)
     dm.dualmv(A[:0], p, r[:0])
     assert dm.dualmv_last_kernel() == -1

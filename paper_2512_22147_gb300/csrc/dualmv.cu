@@ -898,10 +898,10 @@ struct SmallClusterCache {
 };
 SmallClusterCache g_small_cache;
 
-template <int VPL>
+template <int VPL, int D>
 cudaError_t launch_small_cluster(const Params &prm, int dev, cudaStream_t stream, bool *done) {
     *done = false;
-    constexpr auto kern = dmv::dualmv_small_cluster_kernel<VPL>;
+    constexpr auto kern = dmv::dualmv_small_cluster_kernel<VPL, D>;
     constexpr int smem = dmv::SmallLayout<VPL>::kTotal;
     cudaLaunchConfig_t cfg;
     std::memset(&cfg, 0, sizeof cfg);
@@ -1005,6 +1005,7 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
         if (batch == 1 && outputs == dmv::kOutBoth && rank2 == nullptr &&
             g_path == DUALMV_PATH_AUTO && N >= 256 && N <= 2048 && N % 4 == 0 &&
             lda % 4 == 0 && M * N * (int64_t)sizeof(T) <= kSmallMaxBytes &&
+            (M + dmv::kSmallCluster - 1) / dmv::kSmallCluster <= dmv::kSmallMaxRows &&
             reinterpret_cast<uintptr_t>(A) % 16 == 0 && reinterpret_cast<uintptr_t>(p) % 16 == 0 &&
             !explicit_variant(DUALMV_DTYPE_F32, M, N, lda, variant)) {
             Params sp;
@@ -1015,8 +1016,8 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
             bool done = false;
             e = ev0 ? cudaEventRecord(ev0, stream) : cudaSuccess;
             if (e == cudaSuccess)
-                e = N <= 1024 ? launch_small_cluster<8>(sp, dev, stream, &done)
-                              : launch_small_cluster<16>(sp, dev, stream, &done);
+                e = N <= 1024 ? launch_small_cluster<8, 3>(sp, dev, stream, &done)
+                              : launch_small_cluster<16, 1>(sp, dev, stream, &done);
             if (e != cudaSuccess) return cuda_fail(e);
             if (done) {
                 g_kernel_ev_start = g_kernel_ev_stop = nullptr;

@@ -364,7 +364,8 @@ def make_call(torch, dm, inputs, w, dev):
     A, u1, v1, u2, v2, wv, x, y, z = inputs.generate_gemver(w, dev)
 
     def call():
-        dm.gemver(A[:, : w.N], u1, v1, u2, v2, wv, x, y, z, alpha=1.5, beta=1.2)
+        dm.gemver(A[:, : w.N], u1, v1, u2, v2, wv, x, y, z, alpha=1.5, beta=1.2,
+                  update_A=w.update_a)
     return call, {"A": A, "x": x, "w": wv}
 
 
@@ -480,8 +481,8 @@ def launches_per_call(torch, dm, inputs, w, dev) -> int:
         return 2 * n + 1
     if w.op == "atax":      # a row pass and a column pass
         return 2 * n
-    if w.op == "gemver":    # column pass, x update, row pass, w update
-        return 2 * n + 2
+    if w.op == "gemver":    # u.y dots, column pass, x update, row pass, w update
+        return 5
     return n
 
 

@@ -166,9 +166,17 @@ int32_t dualmv_atax_last_path(void);
  * (the default use) the rank-2 update is factorised (see
  * dualmv_gemver_set_onthefly): the passes are the plain streaming kernels,
  * in double-float arithmetic on the FP32 pipes for fp64.  With update_A
- * nonzero both passes form A_hat element by element as they stream A, and
- * the rows-only pass writes A_hat over A (as the PolyBench kernel does);
- * that form runs fp64 in native fp64 arithmetic. */
+ * nonzero the rows-only pass also writes A_hat over A (as the PolyBench
+ * kernel does), each element read before it is written by the same thread:
+ *   - fp64 with A 16-byte aligned and lda even: the columns-only pass and
+ *     the x update are those of the factorised form; the rows pass writes
+ *     A_hat = fma(u2_i, v2_j, fma(u1_i, v1_j, a)) in native fp64 and forms
+ *     A x + u1 (v1 . x) + u2 (v2 . x) from the original A in double-float
+ *     (native fp64 for rows or bands with values outside [2^-40, 2^40),
+ *     zeros excepted);
+ *   - otherwise both passes form A_hat element by element as they stream
+ *     A (native fp64 arithmetic for fp64).
+ * The written A_hat is the same fused form on every path. */
 dualmv_status dualmv_gemver_f32(int64_t M, int64_t N, float alpha, float beta, float *A,
                                 int64_t lda, int update_A, const float *u1, const float *v1,
                                 const float *u2, const float *v2, float *w, float *x,
@@ -187,6 +195,14 @@ dualmv_status dualmv_gemver_f64(int64_t M, int64_t N, double alpha, double beta,
  * it form A_hat element by element as it streams A, as it always does with
  * update_A (tests, benchmarks).  Returns the previous setting. */
 int dualmv_gemver_set_onthefly(int onthefly);
+
+/* Which form the calling thread's last GEMVER call took:
+ * DUALMV_GEMVER_FACTORED (update_A == 0 without the on-the-fly setting),
+ * DUALMV_GEMVER_UPDATE_SPLIT (update_A, fp64, the double-float rows pass
+ * above) or DUALMV_GEMVER_ONTHEFLY (A_hat formed element by element); -1
+ * after an empty problem or an argument error.  Instrumentation for tests. */
+enum { DUALMV_GEMVER_FACTORED = 0, DUALMV_GEMVER_ONTHEFLY = 1, DUALMV_GEMVER_UPDATE_SPLIT = 2 };
+int32_t dualmv_gemver_last_path(void);
 
 /* ---- single problem without allocation --------------------------------
  * The paper has no counterpart to this entry point; it exists for callers

@@ -31,6 +31,8 @@ _BINDING_NAMES = {
     "dualmv_gemver_set_onthefly", "dualmv_last_kernel", "DUALMV_KERNEL_PHASED",
     "DUALMV_KERNEL_PLAIN", "dualmv_atax_last_path", "DUALMV_ATAX_ONE_READ",
     "DUALMV_ATAX_TWO_PASS", "dualmv_read_probe", "dualmv_pool_usage", "DUALMV_KERNEL_CLUSTER",
+    "dualmv_gemver_last_path", "DUALMV_GEMVER_FACTORED", "DUALMV_GEMVER_ONTHEFLY",
+    "DUALMV_GEMVER_UPDATE_SPLIT",
 }
 _API_NAMES = {"dualmv", "device_fault", "gesummv", "atax", "gemver", "tune", "variants"}
 

@@ -43,6 +43,9 @@ DUALMV_KERNEL_PLAIN = 4
 DUALMV_KERNEL_CLUSTER = 5
 DUALMV_ATAX_TWO_PASS = 0
 DUALMV_ATAX_ONE_READ = 1
+DUALMV_GEMVER_FACTORED = 0
+DUALMV_GEMVER_ONTHEFLY = 1
+DUALMV_GEMVER_UPDATE_SPLIT = 2
 
 EXPORTED = (
     "dualmv_f32", "dualmv_f64", "dualmv_i32",
@@ -58,6 +61,7 @@ EXPORTED = (
     "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32", "dualmv_last_variant",
     "dualmv_atax_set_two_pass", "dualmv_gemver_set_onthefly", "dualmv_last_kernel",
     "dualmv_atax_last_path", "dualmv_read_probe", "dualmv_pool_usage",
+    "dualmv_gemver_last_path",
 )
 
 
@@ -161,6 +165,7 @@ def _load() -> ctypes.CDLL:
     lib.dualmv_last_variant.argtypes, lib.dualmv_last_variant.restype = [], i32
     lib.dualmv_last_kernel.argtypes, lib.dualmv_last_kernel.restype = [], i32
     lib.dualmv_atax_last_path.argtypes, lib.dualmv_atax_last_path.restype = [], i32
+    lib.dualmv_gemver_last_path.argtypes, lib.dualmv_gemver_last_path.restype = [], i32
     lib.dualmv_read_probe.argtypes = [vp, i64, vp, vp]
     lib.dualmv_read_probe.restype = st
     lib.dualmv_pool_usage.argtypes = [ctypes.c_int, ctypes.POINTER(i64), ctypes.POINTER(i64),
@@ -354,6 +359,12 @@ def dualmv_atax_last_path() -> int:
     """DUALMV_ATAX_ONE_READ or DUALMV_ATAX_TWO_PASS for this thread's last
     ATAX call, or -1."""
     return _lib.dualmv_atax_last_path()
+
+
+def dualmv_gemver_last_path() -> int:
+    """DUALMV_GEMVER_FACTORED, DUALMV_GEMVER_ONTHEFLY or
+    DUALMV_GEMVER_UPDATE_SPLIT for this thread's last GEMVER call, or -1."""
+    return _lib.dualmv_gemver_last_path()
 
 
 def dualmv_trimmed_mean(times, k: int) -> float:

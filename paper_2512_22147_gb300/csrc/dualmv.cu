@@ -27,6 +27,7 @@
 #include "dualmv_ops.cuh"
 #include "dualmv_probe.cuh"
 #include "dualmv_small.cuh"
+#include "dualmv_gemver64.cuh"
 
 namespace {
 
@@ -84,6 +85,7 @@ thread_local int32_t g_last_atax_path = -1;
 int g_path = DUALMV_PATH_AUTO;
 int g_atax_two_pass = 0;  // 1: ATAX always takes the two-pass path
 int g_gemver_onthefly = 0;  // 1: GEMVER applies the update element by element
+thread_local int32_t g_last_gemver_path = -1;
 
 dualmv_status cuda_fail(cudaError_t e) {
     g_last_cuda_error = static_cast<int>(e);
@@ -1602,6 +1604,94 @@ dualmv_status gemver_factored(int64_t M, int64_t N, T alpha, T beta, const T *A,
 }
 
 // GEMVER (Table 1 / Table 2): A_hat = A + u1 v1^T + u2 v2^T;
+// GEMVER with update_A in fp64: the factorised columns pass and x update of
+// gemver_factored_fused, then gemver_rows_update_f64_kernel, which writes
+// A_hat over A and leaves the band partials of A x (original A, in
+// double-float), and the w update, which adds them.  A read twice and
+// written once; two DFMAs per element (A_hat) where the on-the-fly kernel
+// takes three.  Needs A 16-byte aligned and lda even.
+dualmv_status gemver_update_f64(int64_t M, int64_t N, double alpha, double beta, double *A,
+                                int64_t lda, const double *u1, const double *v1,
+                                const double *u2, const double *v2, double *w, double *x,
+                                const double *y, const double *z, cudaStream_t stream) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e);
+    DeviceState *dst = nullptr;
+    e = device_state(dev, &dst);
+    if (e != cudaSuccess) return cuda_fail(e);
+    const int64_t bands = (N + dmv::kGvBand - 1) / dmv::kGvBand;
+    int64_t row_chunks = (2 * (int64_t)dst->sms + bands - 1) / bands;
+    if (row_chunks > M) row_chunks = M;
+    if (row_chunks < 1) row_chunks = 1;
+    if (bands > 65535 || row_chunks > INT32_MAX) return DUALMV_ERR_UNSUPPORTED;
+    double *s = nullptr, *part = nullptr, *qws = nullptr;
+    dualmv_status st = pool_alloc(&s, N, stream);
+    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * 2 * dmv::kDotChunks, stream);
+    if (st == DUALMV_SUCCESS) st = pool_alloc(&qws, bands * M, stream);
+    double *part_u = part, *part_v = part ? part + 2 * 2 * dmv::kDotChunks : nullptr;
+    Deferred ds;
+    if (st == DUALMV_SUCCESS)
+        e = launch_dependent(dmv::dots2_partial_kernel<double>, dim3(2 * dmv::kDotChunks),
+                             dim3(256), 0, stream, u1, u2, y, M, part_u);
+    if (st == DUALMV_SUCCESS && e == cudaSuccess)  // s = A^T y, left as partials
+        st = run<double, double>(M, N, A, lda, 0, nullptr, 0, y, 0, nullptr, 0, s, 0, 1, stream,
+                                 dmv::kOutS, nullptr, -1, &ds);
+    if (st == DUALMV_SUCCESS && e == cudaSuccess) {
+        if (!ds.used) ds.prm.s = s;
+        e = launch_dependent(dmv::gemver_x3_kernel<double>, dim3(dmv::kDotChunks), dim3(256), 0,
+                             stream, ds.prm, ds.used ? 0 : 1, (const double *)part_u, x, v1,
+                             v2, z, N, beta, part_v);
+    }
+    if (ds.ws != nullptr) {
+        cudaError_t ef = cudaFreeAsync(ds.ws, stream);
+        if (e == cudaSuccess) e = ef;
+    }
+    if (st == DUALMV_SUCCESS && e == cudaSuccess) {
+        dmv::GvParams gp;
+        std::memset(&gp, 0, sizeof gp);
+        gp.A = A;
+        gp.lda = lda;
+        gp.u1 = u1;
+        gp.u2 = u2;
+        gp.v1 = v1;
+        gp.v2 = v2;
+        gp.x = x;
+        gp.q_ws = qws;
+        gp.M = M;
+        gp.N = N;
+        gp.bands = bands;
+        gp.row_chunks = row_chunks;
+        e = launch_dependent(dmv::gemver_rows_update_f64_kernel,
+                             dim3((unsigned)row_chunks, (unsigned)bands), dim3(dmv::kGvWarps * 32),
+                             0, stream, gp);
+    }
+    if (st == DUALMV_SUCCESS && e == cudaSuccess) {
+        Params pq;
+        std::memset(&pq, 0, sizeof pq);
+        pq.q_ws = qws;
+        pq.bands = bands;
+        pq.M = M;
+        pq.batch = 1;
+        const int chunks = combine_chunks(bands);
+        const int64_t rows = 256 / chunks;
+        const int64_t bw = (M + rows - 1) / rows;
+        if (bw > INT32_MAX) e = cudaErrorInvalidConfiguration;
+        else
+            e = launch_dependent(dmv::gemver_w3_kernel<double>, dim3((unsigned)bw), dim3(256), 0,
+                                 stream, pq, 0, chunks, w, u1, u2, (const double *)part_v, M,
+                                 alpha);
+    }
+    if (st == DUALMV_SUCCESS && e != cudaSuccess) st = cuda_fail(e);
+    void *bufs[3] = {s, part, qws};
+    for (void *bp : bufs) {
+        if (bp == nullptr) continue;
+        cudaError_t ef = cudaFreeAsync(bp, stream);
+        if (st == DUALMV_SUCCESS && ef != cudaSuccess) st = cuda_fail(ef);
+    }
+    return st;
+}
+
 // x = x + beta A_hat^T y + z;  w = w + alpha A_hat x.  Without update_A the
 // factorised form above runs.  With it, two passes apply the rank-2 update
 // as they stream A: a columns-only pass (A_hat^T y) and, after the x
@@ -1611,6 +1701,7 @@ template <typename T>
 dualmv_status gemver_run(int64_t M, int64_t N, T alpha, T beta, T *A, int64_t lda,
                          int update_A, const T *u1, const T *v1, const T *u2, const T *v2,
                          T *w, T *x, const T *y, const T *z, cudaStream_t stream) {
+    g_last_gemver_path = -1;
     if (M < 0 || N < 0 || lda < (N > 1 ? N : 1)) return DUALMV_ERR_INVALID_VALUE;
     if (N > 0 && (x == nullptr || z == nullptr || v1 == nullptr || v2 == nullptr))
         return DUALMV_ERR_INVALID_VALUE;
@@ -1619,9 +1710,20 @@ dualmv_status gemver_run(int64_t M, int64_t N, T alpha, T beta, T *A, int64_t ld
     if (M > 0 && N > 0 && A == nullptr) return DUALMV_ERR_INVALID_VALUE;
     if (M == 0 && N == 0) return DUALMV_SUCCESS;
     if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
-    if (!update_A && g_gemver_onthefly == 0)
+    if (!update_A && g_gemver_onthefly == 0) {
+        g_last_gemver_path = DUALMV_GEMVER_FACTORED;
         return gemver_factored<T>(M, N, alpha, beta, A, lda, u1, v1, u2, v2, w, x, y, z,
                                   stream);
+    }
+    if constexpr (std::is_same<T, double>::value) {
+        if (g_gemver_onthefly == 0 && M > 0 && N > 0 && lda % 2 == 0 &&
+            reinterpret_cast<uintptr_t>(A) % 16 == 0) {
+            g_last_gemver_path = DUALMV_GEMVER_UPDATE_SPLIT;
+            return gemver_update_f64(M, N, alpha, beta, A, lda, u1, v1, u2, v2, w, x, y, z,
+                                     stream);
+        }
+    }
+    g_last_gemver_path = DUALMV_GEMVER_ONTHEFLY;
     T *s = nullptr, *t = nullptr;
     dualmv_status st = pool_alloc(&s, N, stream);
     if (st != DUALMV_SUCCESS) return st;
@@ -2257,6 +2359,8 @@ int32_t dualmv_last_variant(void) { return g_last_variant; }
 int32_t dualmv_last_kernel(void) { return g_last_kernel; }
 
 int32_t dualmv_atax_last_path(void) { return g_last_atax_path; }
+
+int32_t dualmv_gemver_last_path(void) { return g_last_gemver_path; }
 
 void dualmv_tune_clear(void) {
     std::lock_guard<std::mutex> lk(g_tuned_mu);

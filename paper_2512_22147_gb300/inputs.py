@@ -37,6 +37,7 @@ class Workload:
     seed: int
     batch: int = 0      # 0 = single problem; >= 1 = strided batch
     op: str = "bicg"    # "bicg" (dual product) | "gesummv" | "atax" | "gemver"
+    update_a: bool = False  # gemver: A_hat written over A
 
     @property
     def batched(self) -> bool:
@@ -50,14 +51,17 @@ class Workload:
         """Bytes of the logical matrices (padding excluded) read once, of the
         input vectors and of the outputs: the numerator of the
         effective-bandwidth metric.  Dual product: A, p, r, q, s.  GESUMMV:
-        A, B, x, y.  ATAX: A (once: the least any algorithm must move), x, y."""
+        A, B, x, y.  ATAX: A (once: the least any algorithm must move), x, y.
+        GEMVER: A (and, with update_a, A_hat written), the six input vectors,
+        x and w read and written."""
         e, o = ELEM_BYTES[self.dtype], OUT_BYTES[self.dtype]
         if self.op == "gesummv":
             return 2 * self.M * self.N * e + self.N * e + self.M * o
         if self.op == "atax":
             return self.M * self.N * e + self.N * e + self.N * o
-        if self.op == "gemver":   # A once; u1 v1 u2 v2 y z read; x w read and written
-            return self.M * self.N * e + 3 * (self.M + self.N) * e + (self.M + self.N) * o
+        if self.op == "gemver":   # A once (and A_hat written); u1 v1 u2 v2 y z read; x w in and out
+            mat = (2 if self.update_a else 1) * self.M * self.N * e
+            return mat + 3 * (self.M + self.N) * e + (self.M + self.N) * o
         per = (self.M * self.N * e + (self.M + self.N) * e
                + (self.M + self.N) * o)
         return per * self.nbatch
@@ -95,6 +99,8 @@ OP_WORKLOADS = {
         Workload("gemver_f32_16384x16384", "f32", 16384, 16384, 16384, "uniform", 9,
                  op="gemver"),
         Workload("gemver_f64_8192x8192", "f64", 8192, 8192, 8192, "normal", 10, op="gemver"),
+        Workload("gemver_update_f64_8192x8192", "f64", 8192, 8192, 8192, "normal", 11,
+                 op="gemver", update_a=True),
     )
 }
 

@@ -1,0 +1,135 @@
+"""GEMVER with update_A in fp64: the double-float rows pass
+(dualmv_gemver64.cuh) against the oracle.
+
+With A 16-byte aligned and lda even, an fp64 call with update_A runs the
+factorised columns pass and x update, then one kernel that writes
+A_hat = fma(u2_i, v2_j, fma(u1_i, v1_j, a)) over A and forms A x from the
+original A in double-float arithmetic.  These tests check, element by
+element against the oracle within the fp64 bar (A_hat, x and w):
+
+  * the path taken (and the fallbacks: odd lda, a base off the 16-byte
+    grid, fp32, the on-the-fly setting);
+  * widths around the kernel's 512-column bands (ragged last band, one
+    column, a band and one);
+  * values outside [2^-40, 2^40) in rows of A and in the new x (native fp64
+    for those rows or that band), and zero rows;
+  * repeated calls giving the same bits, and the padding columns untouched;
+  * the adversarial all-positive inputs of the fp64 error-bound tests.
+The full-size workload (gemver_update_f64_8192x8192) runs in
+test_gpu_ops.py with the other operation workloads."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2512_22147_gb300 as dm
+from paper_2512_22147_gb300 import inputs
+from parity import TOL, scaled_error
+from test_gpu_f64_adversarial import adversarial
+from test_gpu_ops import _w, check_gemver
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+
+
+def _ops(M, N, lda, seed):
+    return inputs.generate_gemver(_w("gemver", "f64", M, N, lda, seed), DEV)
+
+
+@pytest.mark.parametrize("M,N,pad", [(300, 512, 0), (300, 511, 1), (300, 513, 1), (64, 1, 1),
+                                     (200, 1025, 1), (2, 4096, 0), (4097, 300, 2)])
+def test_update_split_matches_oracle(M, N, pad):
+    err = check_gemver(_ops(M, N, N + pad, M * 7 + N), N, 1.5, -0.75, True, "f64")
+    assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_UPDATE_SPLIT
+    print(f"gemver update_A {M}x{N}+{pad}: {err:.3e}")
+
+
+def test_path_taken_and_fallbacks():
+    A, u1, v1, u2, v2, w, x, y, z = _ops(100, 300, 301, 3)
+    args = (u1, v1, u2, v2, w.clone(), x.clone(), y, z)
+    dm.gemver(A.clone()[:, :300], *args, update_A=True)          # lda 301: odd
+    assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_ONTHEFLY
+    B = torch.empty(100, 303, dtype=torch.float64, device=DEV)
+    B[:, 1:301] = A[:, :300]
+    dm.gemver(B[:, 1:301], *args, update_A=True)                  # base 8 bytes off the grid
+    assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_ONTHEFLY
+    C = torch.empty(100, 302, dtype=torch.float64, device=DEV)
+    C[:, :300] = A[:, :300]
+    dm.gemver(C[:, :300], *args, update_A=True)                   # lda 302: even
+    assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_UPDATE_SPLIT
+    dm.gemver(C[:, :300], *args, update_A=False)
+    assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_FACTORED
+    old = dm.dualmv_gemver_set_onthefly(1)
+    try:
+        dm.gemver(C[:, :300], *args, update_A=True)
+        assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_ONTHEFLY
+    finally:
+        dm.dualmv_gemver_set_onthefly(old)
+    f = [t.float() for t in (C[:, :300],) + args]
+    dm.gemver(f[0], *f[1:], update_A=True)
+    assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_ONTHEFLY
+    dm.gemver(C[:0, :0], u1[:0], v1[:0], u2[:0], v2[:0], w[:0], x[:0], y[:0], z[:0],
+              update_A=True)
+    assert dm.dualmv_gemver_last_path() == -1
+
+
+@pytest.mark.parametrize("case", ["huge_rows", "tiny_rows", "zero_rows", "x_out_of_range"])
+def test_out_of_range_values(case):
+    M, N = 700, 1100
+    A, u1, v1, u2, v2, w, x, y, z = _ops(M, N, N, 11)
+    if case == "huge_rows":
+        A[10:13, :] *= 1.0e13          # |a| beyond 2^40
+    elif case == "tiny_rows":
+        A[500:504, 600:] *= 1.0e-14    # |a| below 2^-40 in the second and third bands
+    elif case == "zero_rows":
+        A[20:40, :] = 0.0              # zeros stay on the double-float path
+    else:
+        z[520:530] = 1.0e14            # the new x beyond 2^40 in the second band
+    check_gemver((A, u1, v1, u2, v2, w, x, y, z), N, 1.5, -0.75, True, "f64")
+    assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_UPDATE_SPLIT
+    assert dm.device_fault() == dm.DUALMV_SUCCESS
+
+
+def test_repeated_calls_are_bit_identical():
+    M, N = 1500, 2000
+    ops = _ops(M, N, N + 2, 5)
+    outs = []
+    for _ in range(2):
+        A, u1, v1, u2, v2, w, x, y, z = (t.clone() for t in ops)
+        dm.gemver(A[:, :N], u1, v1, u2, v2, w, x, y, z, alpha=0.5, beta=2.0, update_A=True)
+        outs.append((A, w, x))
+    torch.cuda.synchronize()
+    A0, A1 = outs[0][0], outs[1][0]
+    assert torch.equal(A0[:, :N], A1[:, :N])
+    for a, b in zip(outs[0][1:], outs[1][1:]):
+        assert torch.equal(a, b)
+    # The padding columns (NaN in the generated storage) are untouched.
+    assert torch.equal(A0[:, N:].isnan(), ops[0][:, N:].isnan())
+    assert bool(A0[:, N:].isnan().all())
+
+
+@pytest.mark.parametrize("family", ["low32_set", "low29_set"])
+def test_adversarial_inputs(family):
+    """All inputs positive with the low mantissa bits set: the double-float
+    errors all of one sign."""
+    M, N = 2048, 4096
+    A = adversarial((M, N), 21, family)
+    vecs = [adversarial((n,), 22 + i, family) for i, n in enumerate((M, N, M, N, M, N, M, N))]
+    u1, v1, u2, v2, w, x, y, z = vecs
+    host = [t.cpu().numpy() for t in (A, u1, v1, u2, v2, w, x, y, z)]
+    alpha, beta = 1.5, 0.75
+    dm.gemver(A, u1, v1, u2, v2, w, x, y, z, alpha=alpha, beta=beta, update_A=True)
+    torch.cuda.synchronize()
+    assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_UPDATE_SPLIT
+    An, hu1, hv1, hu2, hv2, hw, hx, hy, hz = host
+    ah, wo, xo = oracle.gemver(An.copy(), hu1, hv1, hu2, hv2, hw.copy(), hx.copy(), hy, hz,
+                               alpha, beta, N=N)
+    _, sa = oracle.absdot(An, np.zeros(N), hy)
+    Xm = hx + beta * (sa + hv1 * (hu1 @ hy) + hv2 * (hu2 @ hy)) + hz
+    qa, _ = oracle.absdot(An, Xm, np.zeros(M))
+    Wm = hw + alpha * (qa + hu1 * (hv1 @ Xm) + hu2 * (hv2 @ Xm))
+    Am = An + np.outer(hu1, hv1) + np.outer(hu2, hv2)
+    err = max(scaled_error(x.cpu().numpy(), xo, Xm), scaled_error(w.cpu().numpy(), wo, Wm),
+              scaled_error(A.cpu().numpy().ravel(), ah.ravel(), Am.ravel()))
+    print(f"adversarial gemver update_A {family}: {err:.3e}")
+    assert err <= TOL["f64"], err

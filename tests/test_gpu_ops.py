@@ -279,7 +279,7 @@ def test_op_workloads_full_size(name):
         err = check_atax(A, x, w.N, w.dtype)
     else:
         ops = inputs.generate_gemver(w, DEV)
-        err = check_gemver(ops, w.N, 1.5, 1.2, False, w.dtype)
+        err = check_gemver(ops, w.N, 1.5, 1.2, w.update_a, w.dtype)
         A = x = ops
     print(f"{name}: max scaled error {err:.3e}")
     del A, x

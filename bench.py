@@ -49,6 +49,8 @@ KERNEL_FAMILIES = {
     "dualmv_stream_kernel": (_CSRC + "dualmv_kernels.cuh",),
     "dualmv_stream_f64e_kernel": (_CSRC + "dualmv_kernels.cuh", _CSRC + "dualmv_f64e.cuh"),
     "dualmv_wide_i32_kernel": (_CSRC + "dualmv_kernels.cuh", _CSRC + "dualmv_wide.cuh"),
+    "dualmv_small_cluster_kernel": (_CSRC + "dualmv_kernels.cuh", _CSRC + "dualmv_atax.cuh",
+                                    _CSRC + "dualmv_small.cuh"),
 }
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 FLUSH_BYTES = 256 << 20      # written between timed calls of an L2-sized workload
@@ -78,6 +80,8 @@ def kernel_shape(name: str):
     fam = kernel_family(name)
     if fam == "dualmv_stream_kernel":   # <T, W, RPW, STAGES, ...>
         return tuple(int(a) for a in args[1:4])
+    if fam == "dualmv_small_cluster_kernel":   # <VPL, D>
+        return tuple(int(a) for a in args[0:2])
     return tuple(int(a) for a in args[0:3])   # f64e and wide: <W, RPW, STAGES, ...>
 
 
@@ -193,7 +197,8 @@ def record_traffic(csv_path: str, workload: str, command: str, full_bytes: int,
     of the captured counters."""
     launches = parse_launch_list(csv_path)
     per = launch_table(launches)
-    stream = [k for k in per if kernel_family(k).startswith(("dualmv_stream", "dualmv_wide"))]
+    stream = [k for k in per if kernel_family(k).startswith(("dualmv_stream", "dualmv_wide",
+                                                             "dualmv_small_cluster"))]
     if len(stream) != 1:
         raise ValueError(f"expected one streaming kernel in the capture, found {stream}")
     n, us, dram = per[stream[0]]
@@ -466,6 +471,8 @@ def streaming_kernel_name(dm, w):
         if w.batched and kind in (dm.DUALMV_KERNEL_STREAM, dm.DUALMV_KERNEL_F64E):
             family = {dm.DUALMV_KERNEL_STREAM: "dualmv_stream_kernel",
                       dm.DUALMV_KERNEL_F64E: "dualmv_stream_f64e_kernel"}[kind]
+        if kind == dm.DUALMV_KERNEL_CLUSTER:
+            family = "dualmv_small_cluster_kernel"
     return kernel_name, family, shape
 
 

@@ -161,6 +161,9 @@ def test_launch_list_parser_and_traffic_record(tmp_path, monkeypatch):
     assert bench.kernel_shape("dmv::dualmv_stream_f64e_kernel<8, 4, 3, 256, 0, 3, 2, 1>") == \
         (8, 4, 3)
     assert bench.kernel_shape("dmv::dualmv_wide_i32_kernel<8, 8, 3>") == (8, 8, 3)
+    assert bench.kernel_shape("dmv::dualmv_small_cluster_kernel<8, 3>") == (8, 3)
+    assert bench.kernel_family("void dmv::dualmv_small_cluster_kernel<8, 3>") in \
+        bench.KERNEL_FAMILIES
 
 
 @pytest.mark.parametrize("dtype", ["f32", "f64", "i32"])

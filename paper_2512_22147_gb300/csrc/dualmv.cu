@@ -1331,16 +1331,26 @@ struct AtaxCfg<float> {
 #ifndef DUALMV_ATAX64_BAND
 #define DUALMV_ATAX64_BAND 256
 #endif
+#ifndef DUALMV_ATAX64_SPLIT_WARPS
+#define DUALMV_ATAX64_SPLIT_WARPS 1
+#endif
 template <>
 struct AtaxCfg<double> {
-    // Three 8 KiB stages per warp (the column phase of a stripe runs one
-    // stripe later) leave room for 8 warps.
+    // Three 8 KiB stages per sub-band (the column phase of a stripe runs
+    // after its row phase) leave room for 8 sub-bands.  With split warps
+    // each sub-band has a row warp and a column warp.
     static constexpr int W = DUALMV_ATAX64_WARPS, R = DUALMV_ATAX64_ROWS,
                          S = DUALMV_ATAX64_STAGES, kBand = DUALMV_ATAX64_BAND;
+#if DUALMV_ATAX64_SPLIT_WARPS
+    static constexpr int kThreads = (2 * W + 1) * 32;  // and a control warp
+    using L = dmv::AtaxLayout64WS<W, R, S, kBand>;
+    static constexpr auto kern = dmv::atax_cluster_f64_ws_kernel<W, R, S, kBand>;
+#else
     static constexpr int kThreads = (W + 1) * 32;  // and a control warp
     using L = dmv::AtaxLayout64<W, R, S, kBand>;
-    using Params = dmv::AtaxParams64;
     static constexpr auto kern = dmv::atax_cluster_f64_kernel<W, R, S, kBand>;
+#endif
+    using Params = dmv::AtaxParams64;
     static void fill(Params &p, const double *A, int64_t lda) {
         p.A = A;
         p.lda = lda;

@@ -55,6 +55,7 @@ KERNEL_FAMILIES = {
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 FLUSH_BYTES = 256 << 20      # written between timed calls of an L2-sized workload
 GRAPH_CALLS = 100            # calls captured in one CUDA graph (hot-L2 figure)
+GB300_L2_BYTES = 126 << 20   # L2 size used when no GPU can be asked (reference arm on a CPU)
 
 
 # ------------------------------------------------------------- helpers ----
@@ -625,16 +626,7 @@ def run_native(args):
         "vs_baseline": None,
         "dtype": w.dtype,
         "data": "synthetic",
-        "config": {
-            "workload": w.name, "op": w.op, "M": w.M, "N": w.N, "lda": w.lda,
-            "batch": w.batch, "dtype": w.dtype, "distribution": w.dist, "seed": w.seed,
-            "bytes_per_step": nbytes,
-            "l2": ("inputs larger than L2 (no flush needed)" if flush is None else
-                   f"L2 flushed: {FLUSH_BYTES >> 20} MiB written before each call, "
-                   "outside its events"),
-            "parallelism": f"replicas x{world}",
-            **({"variant": args.variant} if args.variant is not None else {}),
-        },
+        "config": workload_config(w, nbytes, flush is not None, world, args.variant),
         "pct_of_peak": round(100.0 * value / (world * peak), 2),
         "trimmed_mean_ms": round(trimmed_mean(step_ms, 3) if Ki > 6 else statistics.mean(step_ms), 5),
         "median_step_ms": round(statistics.median(step_ms), 5),
@@ -759,6 +751,21 @@ def measure_config(torch, dm, inputs, w, dev, stream, W, uuid, peak, ceiling, ta
         out["hot_l2_graph"] = hot
     del st, call, flush
     return out
+
+
+def workload_config(w, nbytes: int, flushed: bool, world: int, variant=None) -> dict:
+    """The JSON line's ``config``: the workload and how it is timed.  Both
+    arms print the same dict for the same workload."""
+    return {
+        "workload": w.name, "op": w.op, "M": w.M, "N": w.N, "lda": w.lda,
+        "batch": w.batch, "dtype": w.dtype, "distribution": w.dist, "seed": w.seed,
+        "bytes_per_step": nbytes,
+        "l2": (f"L2 flushed: {FLUSH_BYTES >> 20} MiB written before each call, "
+               "outside its events" if flushed else
+               "inputs larger than L2 (no flush needed)"),
+        "parallelism": f"replicas x{world}",
+        **({"variant": variant} if variant is not None else {}),
+    }
 
 
 def flush_needed(torch, nbytes: int, dev) -> bool:
@@ -1040,6 +1047,11 @@ def run_reference(args):
             vals.append(gbs)
             secs.append(dt)
     value = statistics.mean(vals)
+    nbytes = w.bytes_counted()
+    if torch.cuda.is_available():   # the native arm's rule for this GPU's L2
+        flushed = flush_needed(torch, nbytes, 0)
+    else:
+        flushed = nbytes <= 2 * GB300_L2_BYTES
     del torch
     out = {
         "impl": "reference",
@@ -1048,8 +1060,7 @@ def run_reference(args):
         "ms_per_step": round(1e3 * statistics.mean(secs), 4), "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-        "config": {"workload": w.name, "M": w.M, "N": w.N, "lda": w.lda, "batch": w.batch,
-                   "dtype": w.dtype, "distribution": w.dist, "seed": w.seed},
+        "config": workload_config(w, nbytes, flushed, world, args.variant),
         "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1,
                          "kind": "oracle", "sample": what},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,

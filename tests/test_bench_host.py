@@ -75,6 +75,15 @@ def test_reference_arm_prints_one_json_line():
     assert d["impl"] == "reference" and d["unit"] == "GB/s" and d["value"] > 0
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] == 1
     assert d["e2e"]["h2d_bytes_per_step"] == 0
+    # The native arm's config for the same workload: the same dict (its L2
+    # line as the native arm decides it, a flush for this 4 MiB workload).
+    from paper_2512_22147_gb300 import inputs
+    w = inputs.WORKLOADS["f32_1024x1024"]
+    assert d["config"] == bench.workload_config(w, w.bytes_counted(), True, 1)
+    big = inputs.WORKLOADS["f32_16384x16384"]
+    cfg = bench.workload_config(big, big.bytes_counted(), False, 1)
+    assert cfg["op"] == "bicg" and cfg["bytes_per_step"] == big.bytes_counted()
+    assert "larger than L2" in cfg["l2"]
 
 
 def test_reference_arm_other_ranks_stay_silent():

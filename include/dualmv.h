@@ -377,7 +377,9 @@ typedef struct dualmv_variant_t {
     int32_t packed;         /* DUALMV_KERNEL_F64E: 1 if the double-float   */
                             /* arithmetic of column pairs runs as packed   */
                             /* FP32x2 instructions                         */
-    int32_t pad_;
+    int32_t batched;        /* 1 if the variant also runs strided batches  */
+                            /* (a 3-D tensor-map instance), so that        */
+                            /* dualmv_tune_*_strided_batched may choose it */
     int64_t smem_bytes;     /* dynamic shared memory per CTA              */
 } dualmv_variant_t;
 
@@ -391,19 +393,28 @@ dualmv_status dualmv_variant_info(int32_t dtype, int32_t index, dualmv_variant_t
 
 /* Forces variant `index` for every eligible call of `dtype` in this
  * process (-1 restores the normal choice: a tuned variant for the shape if
- * dualmv_tune_* recorded one, else entry 0).  Returns the previous setting,
- * or -2 for an unknown dtype or an index out of range.  Meant for tests. */
+ * dualmv_tune_* recorded one, else entry 0).  A strided-batched call runs
+ * the forced variant if it has a batched instance, else entry 0.  Returns
+ * the previous setting, or -2 for an unknown dtype or an index out of
+ * range.  Meant for tests. */
 int32_t dualmv_set_variant(int32_t dtype, int32_t index);
 
-/* The variant recorded by dualmv_tune_* for this dtype and shape, or -1. */
+/* The variant recorded by dualmv_tune_* for this dtype and shape (one
+ * problem), or -1. */
 int32_t dualmv_tuned_variant(int32_t dtype, int64_t M, int64_t N, int64_t lda);
+
+/* The variant recorded by dualmv_tune_*_strided_batched for this dtype,
+ * shape and batch count (batch 1: as dualmv_tuned_variant), or -1. */
+int32_t dualmv_tuned_variant_batched(int32_t dtype, int64_t M, int64_t N, int64_t lda,
+                                     int64_t batch);
 
 /* Forgets every recorded tuning result. */
 void dualmv_tune_clear(void);
 
-/* The variant the calling thread's last dual-product call launched: its
- * table index, or -1 if that call ran no TMA streaming kernel (an empty
- * problem, the plain-load path, a batched or single-sided call, or an
+/* The variant the calling thread's last dual-product call launched (one
+ * problem or a strided batch): its table index, or -1 if that call ran no
+ * variant of the table (an empty problem, the phased, plain-load or
+ * single-cluster path, a single-sided call, native fp64 by default, or an
  * error).  Instrumentation for tests and benchmarks. */
 int32_t dualmv_last_variant(void);
 
@@ -499,6 +510,29 @@ dualmv_status dualmv_tune_i32(int64_t M, int64_t N, const int32_t *A, int64_t ld
                               const int32_t *p, const int32_t *r, int64_t *q, int64_t *s,
                               const dualmv_tune_config_t *cfg,
                               dualmv_tune_result_t *res, dualmv_stream_t stream);
+
+/* The same loop for a strided batch (arguments as
+ * dualmv_*_strided_batched, then cfg, res, stream).  Candidates are the
+ * variants with a batched instance (dualmv_variant_t.batched); K^(0) is
+ * entry 0; Eq. 4 compares every problem's outputs; the choice is recorded
+ * for (dtype, M, N, lda, batch) and used by later strided-batched calls of
+ * that shape (dualmv_tuned_variant_batched).  batch == 1 tunes one problem
+ * as dualmv_tune_*.  Blocks until done. */
+dualmv_status dualmv_tune_f32_strided_batched(
+    int64_t M, int64_t N, const float *A, int64_t lda, int64_t strideA, const float *p,
+    int64_t strideP, const float *r, int64_t strideR, float *q, int64_t strideQ, float *s,
+    int64_t strideS, int64_t batch, const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+    dualmv_stream_t stream);
+dualmv_status dualmv_tune_f64_strided_batched(
+    int64_t M, int64_t N, const double *A, int64_t lda, int64_t strideA, const double *p,
+    int64_t strideP, const double *r, int64_t strideR, double *q, int64_t strideQ, double *s,
+    int64_t strideS, int64_t batch, const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+    dualmv_stream_t stream);
+dualmv_status dualmv_tune_i32_strided_batched(
+    int64_t M, int64_t N, const int32_t *A, int64_t lda, int64_t strideA, const int32_t *p,
+    int64_t strideP, const int32_t *r, int64_t strideR, int64_t *q, int64_t strideQ, int64_t *s,
+    int64_t strideS, int64_t batch, const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+    dualmv_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -32,7 +32,9 @@ _BINDING_NAMES = {
     "DUALMV_KERNEL_PLAIN", "dualmv_atax_last_path", "DUALMV_ATAX_ONE_READ",
     "DUALMV_ATAX_TWO_PASS", "dualmv_read_probe", "dualmv_pool_usage", "DUALMV_KERNEL_CLUSTER",
     "dualmv_gemver_last_path", "DUALMV_GEMVER_FACTORED", "DUALMV_GEMVER_ONTHEFLY",
-    "DUALMV_GEMVER_UPDATE_SPLIT",
+    "DUALMV_GEMVER_UPDATE_SPLIT", "dualmv_tune_f32_strided_batched",
+    "dualmv_tune_f64_strided_batched", "dualmv_tune_i32_strided_batched",
+    "dualmv_tuned_variant_batched",
 }
 _API_NAMES = {"dualmv", "device_fault", "gesummv", "atax", "gemver", "tune", "variants"}
 

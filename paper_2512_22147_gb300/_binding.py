@@ -59,6 +59,8 @@ EXPORTED = (
     "dualmv_variant_count", "dualmv_variant_info", "dualmv_set_variant",
     "dualmv_tuned_variant", "dualmv_tune_clear", "dualmv_trimmed_mean",
     "dualmv_tune_f32", "dualmv_tune_f64", "dualmv_tune_i32", "dualmv_last_variant",
+    "dualmv_tune_f32_strided_batched", "dualmv_tune_f64_strided_batched",
+    "dualmv_tune_i32_strided_batched", "dualmv_tuned_variant_batched",
     "dualmv_atax_set_two_pass", "dualmv_gemver_set_onthefly", "dualmv_last_kernel",
     "dualmv_atax_last_path", "dualmv_read_probe", "dualmv_pool_usage",
     "dualmv_gemver_last_path",
@@ -83,7 +85,7 @@ class Plan(ctypes.Structure):
 class Variant(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "index", "kernel", "warps", "rows_per_warp", "stages", "band_cols", "tile_rows",
-        "threads", "native_cols", "producer_warp", "packed", "pad_")] + [
+        "threads", "native_cols", "producer_warp", "packed", "batched")] + [
         ("smem_bytes", ctypes.c_int64)]
 
 
@@ -178,6 +180,11 @@ def _load() -> ctypes.CDLL:
         f = getattr(lib, f"dualmv_tune_{t}")
         f.argtypes = single[:-1] + [ctypes.POINTER(TuneConfig), ctypes.POINTER(TuneResult), vp]
         f.restype = st
+        f = getattr(lib, f"dualmv_tune_{t}_strided_batched")
+        f.argtypes = batched[:-1] + [ctypes.POINTER(TuneConfig), ctypes.POINTER(TuneResult), vp]
+        f.restype = st
+    lib.dualmv_tuned_variant_batched.argtypes = [i32, i64, i64, i64, i64]
+    lib.dualmv_tuned_variant_batched.restype = i32
     return lib
 
 
@@ -324,6 +331,10 @@ def dualmv_tuned_variant(dtype: int, M: int, N: int, lda: int) -> int:
     return _lib.dualmv_tuned_variant(dtype, M, N, lda)
 
 
+def dualmv_tuned_variant_batched(dtype: int, M: int, N: int, lda: int, batch: int) -> int:
+    return _lib.dualmv_tuned_variant_batched(dtype, M, N, lda, batch)
+
+
 def dualmv_tune_clear() -> None:
     _lib.dualmv_tune_clear()
 
@@ -393,3 +404,22 @@ def dualmv_tune_f64(M, N, A, lda, p, r, q, s, cfg, res, stream):
 
 def dualmv_tune_i32(M, N, A, lda, p, r, q, s, cfg, res, stream):
     return _tune("i32", M, N, A, lda, p, r, q, s, cfg, res, stream)
+
+
+def _tune_batched(tag, M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS, batch, cfg, res, stream):
+    return getattr(_lib, f"dualmv_tune_{tag}_strided_batched")(
+        M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS, batch,
+        ctypes.byref(cfg) if cfg is not None else None,
+        ctypes.byref(res) if res is not None else None, stream)
+
+
+def dualmv_tune_f32_strided_batched(*args):
+    return _tune_batched("f32", *args)
+
+
+def dualmv_tune_f64_strided_batched(*args):
+    return _tune_batched("f64", *args)
+
+
+def dualmv_tune_i32_strided_batched(*args):
+    return _tune_batched("i32", *args)

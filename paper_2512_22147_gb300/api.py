@@ -252,28 +252,45 @@ def tune(A: torch.Tensor, p: torch.Tensor, r: torch.Tensor, q: torch.Tensor | No
          stream: torch.cuda.Stream | None = None) -> dict:
     """Tune the kernel variant for this problem's shape (Section 3.2: Eq. 3
     scores, the Eq. 4 equivalence gate, the Eq. 5 choice); later ``dualmv``
-    calls of the same shape use the result.  Blocks until done.  Returns the
-    tuner's report; q and s hold the chosen variant's outputs."""
-    if A.dtype not in _TAG or A.dim() != 2:
-        raise ValueError("tune takes one 2-D float32, float64 or int32 problem")
-    M, N = A.shape
-    if N > 1 and A.stride(1) != 1:
+    calls of the same shape use the result.  A is one (M, N) problem or a
+    strided batch (B, M, N) with p (B, N) and r (B, M), as ``dualmv`` takes
+    them.  Blocks until done.  Returns the tuner's report; q and s hold the
+    chosen variant's outputs."""
+    if A.dtype not in _TAG or A.dim() not in (2, 3):
+        raise ValueError("tune takes a 2-D (or 3-D batched) float32, float64 or int32 A")
+    batched = A.dim() == 3
+    Bn = A.shape[0] if batched else 1
+    M, N = A.shape[-2], A.shape[-1]
+    if N > 1 and A.stride(-1) != 1:
         raise ValueError("A's last dimension must be contiguous")
-    lda = max(A.stride(0), N, 1) if M > 1 else max(N, 1)
+    lda = max(A.stride(-2), N, 1) if M > 1 else max(N, 1)
     out_t = _OUT[A.dtype]
     if q is None:
-        q = torch.empty(M, dtype=out_t, device=A.device)
+        q = torch.empty((Bn, M) if batched else M, dtype=out_t, device=A.device)
     if s is None:
-        s = torch.empty(N, dtype=out_t, device=A.device)
-    for t_, n in ((p, "p"), (r, "r")):
-        if t_.dtype != A.dtype or t_.device != A.device or not t_.is_contiguous():
-            raise ValueError(f"{n} must be a contiguous vector of A's dtype on its device")
+        s = torch.empty((Bn, N) if batched else N, dtype=out_t, device=A.device)
+    for t_, n in ((p, "p"), (r, "r"), (q, "q"), (s, "s")):
+        dt = A.dtype if n in ("p", "r") else out_t
+        if t_.dtype != dt or t_.device != A.device:
+            raise ValueError(f"{n} must be of dtype {dt} on A's device")
+    if batched:   # per-problem vectors (B, n), or p, r shared by every problem
+        sP, sR = _vec_stride(p, N, Bn, "p"), _vec_stride(r, M, Bn, "r")
+        if q.dim() != 2 or s.dim() != 2:
+            raise ValueError(f"q and s must have shapes ({Bn}, {M}) and ({Bn}, {N})")
+        sQ, sS = _vec_stride(q, M, Bn, "q"), _vec_stride(s, N, Bn, "s")
+    elif not all(t_.dim() == 1 and t_.is_contiguous() for t_ in (p, r, q, s)):
+        raise ValueError("p, r, q and s must be contiguous vectors")
     cfg = B.TuneConfig(repeats, trim, max_rounds, candidates, min_gain, int(flush_l2))
     res = B.TuneResult()
     strm = stream if stream is not None else torch.cuda.current_stream(A.device)
-    fn = getattr(B, f"dualmv_tune_{_TAG[A.dtype]}")
-    rc = fn(M, N, A.data_ptr(), lda, p.data_ptr(), r.data_ptr(), q.data_ptr(), s.data_ptr(),
-            cfg, res, strm.cuda_stream)
+    if batched:
+        fn = getattr(B, f"dualmv_tune_{_TAG[A.dtype]}_strided_batched")
+        rc = fn(M, N, A.data_ptr(), lda, A.stride(0), p.data_ptr(), sP, r.data_ptr(), sR,
+                q.data_ptr(), sQ, s.data_ptr(), sS, Bn, cfg, res, strm.cuda_stream)
+    else:
+        fn = getattr(B, f"dualmv_tune_{_TAG[A.dtype]}")
+        rc = fn(M, N, A.data_ptr(), lda, p.data_ptr(), r.data_ptr(), q.data_ptr(),
+                s.data_ptr(), cfg, res, strm.cuda_stream)
     if rc != B.DUALMV_SUCCESS:
         raise B.DualmvError(rc, "dualmv_tune")
     rep = {f: getattr(res, f) for f, _ in res._fields_

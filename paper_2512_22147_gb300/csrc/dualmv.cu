@@ -688,23 +688,25 @@ struct Variant {
     Kind kind;
     Geometry geo;
     LaunchFn launch;
+    LaunchFn launch3d;  // strided batches (3-D tensor map), or nullptr
 };
 
-template <typename T, int W, int RPW, int S>
+template <typename T, int W, int RPW, int S, bool k3d = false>
 cudaError_t launch_stream_variant(const CUtensorMap &m, const Params &p,
                                   const dualmv_plan_t &pl, int dev, cudaStream_t st) {
-    return launch_stream<T, true, false, dmv::kOutBoth, false, W, RPW, S>(m, p, pl, dev, st);
+    return launch_stream<T, true, k3d, dmv::kOutBoth, false, W, RPW, S>(m, p, pl, dev, st);
 }
 
-template <int W, int RPW, int S, int NC, bool kSelf, bool kPack, int BAND>
+template <int W, int RPW, int S, int NC, bool kSelf, bool kPack, int BAND, bool k3d = false>
 cudaError_t launch_f64e_variant(const CUtensorMap &m, const Params &p, const dualmv_plan_t &pl,
                                 int dev, cudaStream_t st) {
-    return launch_f64e<false, dmv::kOutBoth, W, RPW, S, NC, kSelf, kPack, BAND>(m, p, pl, dev,
-                                                                               st);
+    return launch_f64e<k3d, dmv::kOutBoth, W, RPW, S, NC, kSelf, kPack, BAND>(m, p, pl, dev,
+                                                                             st);
 }
 
 Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind kind,
-                     const Geometry &g, LaunchFn fn, int NC = 0, bool self_load = false) {
+                     const Geometry &g, LaunchFn fn, int NC = 0, bool self_load = false,
+                     LaunchFn fn3d = nullptr) {
     Variant v;
     v.info.index = index;
     v.info.kernel = kernel;
@@ -714,6 +716,7 @@ Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind 
     v.info.native_cols = NC;
     v.info.producer_warp = self_load ? 0 : 1;
     v.info.packed = 0;
+    v.info.batched = fn3d != nullptr ? 1 : 0;
     v.info.band_cols = (int32_t)g.band_cols;
     v.info.tile_rows = (int32_t)g.tile_rows;
     v.info.threads = (int32_t)g.threads;
@@ -721,22 +724,32 @@ Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind 
     v.kind = kind;
     v.geo = g;
     v.launch = fn;
+    v.launch3d = fn3d;
     return v;
 }
 
-template <typename T, int W, int RPW, int S>
+// kBatched: the variant also has a strided-batched instance (every shape of
+// the 4-byte tables; not the native fp64 entry, which no batched entry
+// neighbours).
+template <typename T, int W, int RPW, int S, bool kBatched = true>
 Variant stream_variant(int32_t index) {
+    LaunchFn fn3d = nullptr;
+    if constexpr (kBatched) fn3d = &launch_stream_variant<T, W, RPW, S, true>;
     return make_variant(index, DUALMV_KERNEL_STREAM, W, RPW, S, Kind::kTma,
                         stream_geometry<T, W, RPW, S>(true),
-                        &launch_stream_variant<T, W, RPW, S>);
+                        &launch_stream_variant<T, W, RPW, S>, 0, false, fn3d);
 }
 
+// kBatched: the variant also has a strided-batched instance.
 template <int W, int RPW, int S, int NC = kF64eNativeCols, bool kSelf = kF64eSelf,
-          bool kPack = kF64ePack, int BAND = kF64eBand>
+          bool kPack = kF64ePack, int BAND = kF64eBand, bool kBatched = false>
 Variant f64e_variant(int32_t index) {
+    LaunchFn fn3d = nullptr;
+    if constexpr (kBatched) fn3d = &launch_f64e_variant<W, RPW, S, NC, kSelf, kPack, BAND, true>;
     Variant v = make_variant(index, DUALMV_KERNEL_F64E, W, RPW, S, Kind::kF64e,
                              f64e_geometry<W, RPW, S, kSelf, BAND>(),
-                             &launch_f64e_variant<W, RPW, S, NC, kSelf, kPack, BAND>, NC, kSelf);
+                             &launch_f64e_variant<W, RPW, S, NC, kSelf, kPack, BAND>, NC, kSelf,
+                             fn3d);
     v.info.packed = kPack ? 1 : 0;
     return v;
 }
@@ -788,15 +801,15 @@ const std::vector<Variant> &i32_table() {
 // consumers, and native fp64 FMA.
 const std::vector<Variant> &f64_table() {
     static const std::vector<Variant> tab = {
-        f64e_variant<12, 4, 2, 0, true, true>(0),
-        f64e_variant<8, 4, 2, 0, true, true>(1),
+        f64e_variant<12, 4, 2, 0, true, true, kF64eBand, true>(0),
+        f64e_variant<8, 4, 2, 0, true, true, kF64eBand, true>(1),
         f64e_variant<8, 4, 3, 0, true, false>(2),    // scalar FP32 instructions
         f64e_variant<8, 4, 3, 2, true, false>(3),
         f64e_variant<8, 4, 3, 3, true, false>(4),
         f64e_variant<7, 4, 3, 2, true, false>(5),
         f64e_variant<7, 4, 3, 2, false, false>(6),   // a producer warp feeds 7 consumers
         f64e_variant<7, 4, 3, 0, false, false>(7),
-        stream_variant<double, 7, 4, 3>(8),          // native fp64 FMA
+        stream_variant<double, 7, 4, 3, false>(8),   // native fp64 FMA
         f64e_variant<6, 4, 3, 2, false, false>(9),
         f64e_variant<7, 4, 2, 2, false, false>(10),
         // 128-column bands: 4 columns per lane (fewer registers, twice the
@@ -805,10 +818,10 @@ const std::vector<Variant> &f64_table() {
         f64e_variant<12, 4, 3, 0, true, true, 128>(12),
         f64e_variant<12, 4, 2, 0, true, true, 128>(13),
         f64e_variant<8, 8, 3, 0, true, true, 128>(14),
-        f64e_variant<8, 4, 3, 0, true, true>(15),    // two warps per sub-partition
+        f64e_variant<8, 4, 3, 0, true, true, kF64eBand, true>(15),  // two warps per sub-partition
         // Fewer warps or rows than entry 0.
-        f64e_variant<10, 4, 2, 0, true, true>(16),
-        f64e_variant<12, 2, 2, 0, true, true>(17),
+        f64e_variant<10, 4, 2, 0, true, true, kF64eBand, true>(16),
+        f64e_variant<12, 2, 2, 0, true, true, kF64eBand, true>(17),
         // Four warps per sub-partition on 128-column bands (128 registers).
         f64e_variant<16, 4, 3, 0, true, true, 128>(18),
     };
@@ -844,13 +857,14 @@ bool neighbours(const dualmv_variant_t &a, const dualmv_variant_t &b) {
 
 std::atomic<int32_t> g_forced_variant[3] = {{-1}, {-1}, {-1}};
 std::mutex g_tuned_mu;
-std::map<std::tuple<int32_t, int64_t, int64_t, int64_t>, int32_t> g_tuned;
+// Tuned choices by (dtype, M, N, lda, batch); batch 1 for single problems.
+std::map<std::tuple<int32_t, int64_t, int64_t, int64_t, int64_t>, int32_t> g_tuned;
 std::atomic<int> g_tuned_count{0};
 
-int32_t tuned_lookup(int32_t dtype, int64_t M, int64_t N, int64_t lda) {
+int32_t tuned_lookup(int32_t dtype, int64_t M, int64_t N, int64_t lda, int64_t batch = 1) {
     if (g_tuned_count.load(std::memory_order_acquire) == 0) return -1;
     std::lock_guard<std::mutex> lk(g_tuned_mu);
-    auto it = g_tuned.find(std::make_tuple(dtype, M, N, lda));
+    auto it = g_tuned.find(std::make_tuple(dtype, M, N, lda, batch));
     return it == g_tuned.end() ? -1 : it->second;
 }
 
@@ -867,15 +881,17 @@ int32_t default_variant(int32_t dtype, const void *A, int64_t lda_bytes) {
 // The variant a call runs: `index` if the caller (the tuner) names one, else
 // the process-wide forced one, else the tuned one for this shape, else the
 // default for the shape.  nullptr means entry 0, which the ordinary launch
-// code covers.
+// code covers.  A strided batch (batch > 1) runs a variant only if it has a
+// batched instance; otherwise entry 0.
 const Variant *pick_variant(int32_t dtype, int64_t M, int64_t N, const void *A, int64_t lda,
-                            int64_t es, int32_t index) {
+                            int64_t es, int32_t index, int64_t batch = 1) {
     const std::vector<Variant> *tab = variant_table(dtype);
     if (tab == nullptr) return nullptr;
     if (index < 0) index = g_forced_variant[dtype].load(std::memory_order_relaxed);
-    if (index < 0) index = tuned_lookup(dtype, M, N, lda);
-    if (index < 0) index = default_variant(dtype, A, lda * es);
+    if (index < 0) index = tuned_lookup(dtype, M, N, lda, batch);
+    if (index < 0) index = batch > 1 ? 0 : default_variant(dtype, A, lda * es);
     if (index <= 0 || index >= (int32_t)tab->size()) return nullptr;
+    if (batch > 1 && (*tab)[index].launch3d == nullptr) return nullptr;
     return &(*tab)[index];
 }
 
@@ -1046,11 +1062,12 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                    ? Kind::kF64e
                    : Kind::kTma;
     // A compiled variant other than the default (forced, tuned or named by
-    // the tuner) for one unbatched dual product on the TMA path.
+    // the tuner) for a dual product (one problem or a strided batch) on the
+    // TMA path.
     const Variant *var = nullptr;
-    if (tma && !three_d && outputs == dmv::kOutBoth && rank2 == nullptr &&
+    if (tma && outputs == dmv::kOutBoth && rank2 == nullptr &&
         g_path != DUALMV_PATH_TMA_NATIVE_F64)
-        var = pick_variant(dtype_code<T>(), M, N, A, lda, es, variant);
+        var = pick_variant(dtype_code<T>(), M, N, A, lda, es, variant, batch);
     if (var != nullptr) kind = var->kind;
     if (kind == Kind::kF64e) {
         // The double-float kernel counts tiles in 32 bits; a launch of 2^31
@@ -1161,7 +1178,8 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                                                        : (int32_t)DUALMV_KERNEL_PLAIN;
     if (e == cudaSuccess) {
         if (var != nullptr) {
-            e = var->launch(map, prm, pl, dev, stream);
+            e = three_d ? var->launch3d(map, prm, pl, dev, stream)
+                        : var->launch(map, prm, pl, dev, stream);
             if (e == cudaSuccess) g_last_variant = var->info.index;
         } else if (rank2 != nullptr) {
             if constexpr (!kIntPath) {
@@ -1201,14 +1219,13 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
         } else if (kind == Kind::kF64e) {
             e = three_d ? launch_f64e<true>(map, prm, pl, dev, stream)
                         : launch_f64e<false>(map, prm, pl, dev, stream);
-            if (e == cudaSuccess && !three_d) g_last_variant = 0;
+            if (e == cudaSuccess) g_last_variant = 0;
         } else if (kind == Kind::kTma) {
             e = three_d ? launch_stream<T, true, true>(map, prm, pl, dev, stream)
                         : launch_stream<T, true, false>(map, prm, pl, dev, stream);
             // Entry 0 of the f64 table is the double-float kernel: the
             // native fp64 default kernel is no entry of it.
-            if (e == cudaSuccess && !three_d && !std::is_same<T, double>::value)
-                g_last_variant = 0;
+            if (e == cudaSuccess && !std::is_same<T, double>::value) g_last_variant = 0;
         } else if (nph > 0) {
             e = launch_phased<T>(nph, pmaps, prm, pl, dev, stream);
         } else {
@@ -1804,10 +1821,13 @@ template <typename T> constexpr double fe_tolerance() {
 template <typename T, typename Out>
 class Tuner {
   public:
-    Tuner(int64_t M, int64_t N, const T *A, int64_t lda, const T *p, const T *r, Out *q, Out *s,
-          const dualmv_tune_config_t &cfg, cudaStream_t stream)
-        : M_(M), N_(N), A_(A), lda_(lda), p_(p), r_(r), q_(q), s_(s), cfg_(cfg),
-          stream_(stream) {}
+    // One problem (batch 1) or a strided batch; strides in elements.
+    Tuner(int64_t M, int64_t N, int64_t batch, const T *A, int64_t lda, int64_t strideA,
+          const T *p, int64_t strideP, const T *r, int64_t strideR, Out *q, int64_t strideQ,
+          Out *s, int64_t strideS, const dualmv_tune_config_t &cfg, cudaStream_t stream)
+        : M_(M), N_(N), batch_(batch), A_(A), lda_(lda), strideA_(strideA), p_(p),
+          strideP_(strideP), r_(r), strideR_(strideR), q_(q), strideQ_(strideQ), s_(s),
+          strideS_(strideS), cfg_(cfg), stream_(stream) {}
 
     ~Tuner() {
         for (cudaEvent_t ev : events_) cudaEventDestroy(ev);
@@ -1818,13 +1838,13 @@ class Tuner {
     }
 
     dualmv_status setup() {
-        dualmv_status st = pool_alloc(&q_base_, M_, stream_);
-        if (st == DUALMV_SUCCESS) st = pool_alloc(&s_base_, N_, stream_);
+        dualmv_status st = pool_alloc(&q_base_, batch_ * M_, stream_);
+        if (st == DUALMV_SUCCESS) st = pool_alloc(&s_base_, batch_ * N_, stream_);
         if (st == DUALMV_SUCCESS) st = pool_alloc(&fe_word_, 1, stream_);
         constexpr bool kExact = std::is_same<T, int32_t>::value;
         if (!kExact) {
-            if (st == DUALMV_SUCCESS) st = pool_alloc(&den_q_, M_, stream_);
-            if (st == DUALMV_SUCCESS) st = pool_alloc(&den_s_, N_, stream_);
+            if (st == DUALMV_SUCCESS) st = pool_alloc(&den_q_, batch_ * M_, stream_);
+            if (st == DUALMV_SUCCESS) st = pool_alloc(&den_s_, batch_ * N_, stream_);
         }
         if (st != DUALMV_SUCCESS) return st;
         int dev = 0, l2 = 0, sms = 0;
@@ -1842,22 +1862,26 @@ class Tuner {
             e = cudaEventCreate(&ev);
             if (e != cudaSuccess) return cuda_fail(e);
         }
-        if (!kExact) {  // magnitude sums for the equivalence bar, once
-            dmv::abs_rows_kernel<T><<<4 * sms, 256, 0, stream_>>>(A_, M_, N_, lda_, p_, den_q_);
+        if (!kExact) {  // magnitude sums for the equivalence bar, once per problem
             const int64_t bc = (N_ + 255) / 256;
-            dmv::abs_cols_kernel<T><<<(unsigned)(bc < 65535 ? bc : 65535), 256, 0, stream_>>>(
-                A_, M_, N_, lda_, r_, den_s_);
-            e = cudaGetLastError();
-            if (e != cudaSuccess) return cuda_fail(e);
+            for (int64_t b = 0; b < batch_; ++b) {
+                dmv::abs_rows_kernel<T><<<4 * sms, 256, 0, stream_>>>(
+                    A_ + b * strideA_, M_, N_, lda_, p_ + b * strideP_, den_q_ + b * M_);
+                dmv::abs_cols_kernel<T><<<(unsigned)(bc < 65535 ? bc : 65535), 256, 0, stream_>>>(
+                    A_ + b * strideA_, M_, N_, lda_, r_ + b * strideR_, den_s_ + b * N_);
+                e = cudaGetLastError();
+                if (e != cudaSuccess) return cuda_fail(e);
+            }
         }
         return DUALMV_SUCCESS;
     }
 
-    // One call of variant `v` into q, s (or the baseline buffers).
+    // One call of variant `v` into q, s (or the baseline buffers, packed).
     dualmv_status call(int32_t v, bool into_base) {
         Out *q = into_base ? q_base_ : q_, *s = into_base ? s_base_ : s_;
-        return run<T, Out>(M_, N_, A_, lda_, 0, p_, 0, r_, 0, q, 0, s, 0, 1, stream_,
-                           dmv::kOutBoth, nullptr, v);
+        const int64_t sq = into_base ? M_ : strideQ_, ss = into_base ? N_ : strideS_;
+        return run<T, Out>(M_, N_, A_, lda_, strideA_, p_, strideP_, r_, strideR_, q, sq, s, ss,
+                           batch_, stream_, dmv::kOutBoth, nullptr, v);
     }
 
     // Score of Eq. 3: `repeats` timed calls, trimmed mean of their times.
@@ -1891,9 +1915,13 @@ class Tuner {
         cudaError_t e = cudaMemsetAsync(fe_word_, 0, sizeof(unsigned long long), stream_);
         const unsigned gq = (unsigned)std::min<int64_t>((M_ + 255) / 256, 1024);
         const unsigned gs = (unsigned)std::min<int64_t>((N_ + 255) / 256, 1024);
-        if (e == cudaSuccess) {
-            dmv::fe_max_kernel<Out><<<gq, 256, 0, stream_>>>(q_, q_base_, den_q_, M_, fe_word_);
-            dmv::fe_max_kernel<Out><<<gs, 256, 0, stream_>>>(s_, s_base_, den_s_, N_, fe_word_);
+        for (int64_t b = 0; b < batch_ && e == cudaSuccess; ++b) {
+            dmv::fe_max_kernel<Out><<<gq, 256, 0, stream_>>>(q_ + b * strideQ_, q_base_ + b * M_,
+                                                             den_q_ ? den_q_ + b * M_ : nullptr,
+                                                             M_, fe_word_);
+            dmv::fe_max_kernel<Out><<<gs, 256, 0, stream_>>>(s_ + b * strideS_, s_base_ + b * N_,
+                                                             den_s_ ? den_s_ + b * N_ : nullptr,
+                                                             N_, fe_word_);
             e = cudaGetLastError();
         }
         unsigned long long bits = 0;
@@ -1919,11 +1947,17 @@ class Tuner {
     }
 
   private:
-    int64_t M_, N_;
+    int64_t M_, N_, batch_;
     const T *A_;
-    int64_t lda_;
-    const T *p_, *r_;
-    Out *q_, *s_;
+    int64_t lda_, strideA_;
+    const T *p_;
+    int64_t strideP_;
+    const T *r_;
+    int64_t strideR_;
+    Out *q_;
+    int64_t strideQ_;
+    Out *s_;
+    int64_t strideS_;
     dualmv_tune_config_t cfg_;
     cudaStream_t stream_;
     Out *q_base_ = nullptr, *s_base_ = nullptr;
@@ -1934,36 +1968,46 @@ class Tuner {
     std::vector<cudaEvent_t> events_;
 };
 
+// The loop of Section 3.2 for one problem (batch 1) or a strided batch (the
+// candidates then are the variants with a batched instance).
 template <typename T, typename Out>
-dualmv_status tune_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *p, const T *r,
-                       Out *q, Out *s, const dualmv_tune_config_t *cfg,
-                       dualmv_tune_result_t *res, cudaStream_t stream) {
+dualmv_status tune_run(int64_t M, int64_t N, int64_t batch, const T *A, int64_t lda,
+                       int64_t strideA, const T *p, int64_t strideP, const T *r,
+                       int64_t strideR, Out *q, int64_t strideQ, Out *s, int64_t strideS,
+                       const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+                       cudaStream_t stream) {
     if (cfg == nullptr || res == nullptr) return DUALMV_ERR_INVALID_VALUE;
     if (cfg->trim < 0 || cfg->repeats <= 2 * cfg->trim || cfg->max_rounds < 0 ||
         cfg->candidates < 1 || !(cfg->min_gain >= 0.0))
         return DUALMV_ERR_INVALID_VALUE;
-    dualmv_status st = validate(M, N, A, lda, 0, p, 0, r, 0, q, 0, s, 0, 1);
+    dualmv_status st = validate(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ, s,
+                                strideS, batch);
     if (st != DUALMV_SUCCESS) return st;
     std::memset(res, 0, sizeof *res);
     const int64_t es = sizeof(T);
-    const bool eligible = M > 0 && N > 0 && g_path != DUALMV_PATH_DIRECT &&
+    const bool batched = batch > 1;
+    const bool eligible = M > 0 && N > 0 && batch > 0 && g_path != DUALMV_PATH_DIRECT &&
                           g_path != DUALMV_PATH_TMA_NATIVE_F64 &&
                           reinterpret_cast<uintptr_t>(A) % 16 == 0 && (lda * es) % 16 == 0 &&
-                          M < INT32_MAX && N < INT32_MAX;
-    if (!eligible) return run<T, Out>(M, N, A, lda, 0, p, 0, r, 0, q, 0, s, 0, 1, stream);
+                          (!batched || (strideA * es) % 16 == 0) && M < INT32_MAX &&
+                          N < INT32_MAX && batch < INT32_MAX;
+    if (!eligible)
+        return run<T, Out>(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ, s, strideS,
+                           batch, stream);
     if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
 
     const int32_t dtype = dtype_code<T>();
     const std::vector<Variant> &tab = *variant_table(dtype);
     constexpr double tol = fe_tolerance<T>();
     const bool plant = fault_injected("fe");
-    Tuner<T, Out> tu(M, N, A, lda, p, r, q, s, *cfg, stream);
+    Tuner<T, Out> tu(M, N, batch, A, lda, strideA, p, strideP, r, strideR, q, strideQ, s,
+                     strideS, *cfg, stream);
     st = tu.setup();
     if (st != DUALMV_SUCCESS) return st;
 
     // K^(0): the variant an untuned call of this shape uses; its outputs are
     // the reference for Eq. 4.
-    int32_t base = default_variant(dtype, A, lda * es);
+    int32_t base = batched ? 0 : default_variant(dtype, A, lda * es);
     res->initial = base;
     st = tu.call(base, true);
     if (st == DUALMV_SUCCESS) st = tu.score(base, &res->baseline_ms);
@@ -1975,8 +2019,8 @@ dualmv_status tune_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *p
     for (int32_t d = 0; d < cfg->max_rounds; ++d) {
         std::vector<int32_t> cands;
         for (const Variant &v : tab)
-            if (!tried[v.info.index] && neighbours(v.info, tab[base].info) &&
-                (int32_t)cands.size() < cfg->candidates)
+            if (!tried[v.info.index] && (!batched || v.launch3d != nullptr) &&
+                neighbours(v.info, tab[base].info) && (int32_t)cands.size() < cfg->candidates)
                 cands.push_back(v.info.index);
         if (cands.empty()) break;
         res->rounds = d + 1;
@@ -2025,7 +2069,7 @@ dualmv_status tune_run(int64_t M, int64_t N, const T *A, int64_t lda, const T *p
     res->best_ms = base_ms;
     {
         std::lock_guard<std::mutex> lk(g_tuned_mu);
-        g_tuned[std::make_tuple(dtype, M, N, lda)] = base;
+        g_tuned[std::make_tuple(dtype, M, N, lda, batched ? batch : (int64_t)1)] = base;
         g_tuned_count.store((int)g_tuned.size(), std::memory_order_release);
     }
     st = tu.call(base, false);  // leave the chosen variant's outputs in q, s
@@ -2364,6 +2408,11 @@ int32_t dualmv_tuned_variant(int32_t dtype, int64_t M, int64_t N, int64_t lda) {
     return tuned_lookup(dtype, M, N, lda);
 }
 
+int32_t dualmv_tuned_variant_batched(int32_t dtype, int64_t M, int64_t N, int64_t lda,
+                                     int64_t batch) {
+    return tuned_lookup(dtype, M, N, lda, batch > 1 ? batch : 1);
+}
+
 int32_t dualmv_last_variant(void) { return g_last_variant; }
 
 int32_t dualmv_last_kernel(void) { return g_last_kernel; }
@@ -2388,7 +2437,7 @@ dualmv_status dualmv_tune_f32(int64_t M, int64_t N, const float *A, int64_t lda,
                               const float *r, float *q, float *s,
                               const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
                               dualmv_stream_t stream) {
-    return tune_run<float, float>(M, N, A, lda, p, r, q, s, cfg, res,
+    return tune_run<float, float>(M, N, 1, A, lda, 0, p, 0, r, 0, q, 0, s, 0, cfg, res,
                                   reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -2396,7 +2445,7 @@ dualmv_status dualmv_tune_f64(int64_t M, int64_t N, const double *A, int64_t lda
                               const double *p, const double *r, double *q, double *s,
                               const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
                               dualmv_stream_t stream) {
-    return tune_run<double, double>(M, N, A, lda, p, r, q, s, cfg, res,
+    return tune_run<double, double>(M, N, 1, A, lda, 0, p, 0, r, 0, q, 0, s, 0, cfg, res,
                                     reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -2404,7 +2453,37 @@ dualmv_status dualmv_tune_i32(int64_t M, int64_t N, const int32_t *A, int64_t ld
                               const int32_t *p, const int32_t *r, int64_t *q, int64_t *s,
                               const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
                               dualmv_stream_t stream) {
-    return tune_run<int32_t, int64_t>(M, N, A, lda, p, r, q, s, cfg, res,
+    return tune_run<int32_t, int64_t>(M, N, 1, A, lda, 0, p, 0, r, 0, q, 0, s, 0, cfg, res,
+                                      reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_tune_f32_strided_batched(
+    int64_t M, int64_t N, const float *A, int64_t lda, int64_t strideA, const float *p,
+    int64_t strideP, const float *r, int64_t strideR, float *q, int64_t strideQ, float *s,
+    int64_t strideS, int64_t batch, const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+    dualmv_stream_t stream) {
+    return tune_run<float, float>(M, N, batch, A, lda, strideA, p, strideP, r, strideR, q,
+                                  strideQ, s, strideS, cfg, res,
+                                  reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_tune_f64_strided_batched(
+    int64_t M, int64_t N, const double *A, int64_t lda, int64_t strideA, const double *p,
+    int64_t strideP, const double *r, int64_t strideR, double *q, int64_t strideQ, double *s,
+    int64_t strideS, int64_t batch, const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+    dualmv_stream_t stream) {
+    return tune_run<double, double>(M, N, batch, A, lda, strideA, p, strideP, r, strideR, q,
+                                    strideQ, s, strideS, cfg, res,
+                                    reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_tune_i32_strided_batched(
+    int64_t M, int64_t N, const int32_t *A, int64_t lda, int64_t strideA, const int32_t *p,
+    int64_t strideP, const int32_t *r, int64_t strideR, int64_t *q, int64_t strideQ, int64_t *s,
+    int64_t strideS, int64_t batch, const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+    dualmv_stream_t stream) {
+    return tune_run<int32_t, int64_t>(M, N, batch, A, lda, strideA, p, strideP, r, strideR, q,
+                                      strideQ, s, strideS, cfg, res,
                                       reinterpret_cast<cudaStream_t>(stream));
 }
 

@@ -187,8 +187,82 @@ def test_tuner_off_the_tma_path_runs_default():
     assert dm.dualmv_tuned_variant(dm.DUALMV_DTYPE_F32, 300, 301, 301) == -1
 
 
-def test_batched_calls_ignore_forced_variant(forced):
-    forced("f32", 5)
-    w = inputs.Workload("t", "f32", 300, 700, 700, "uniform", 9, batch=3)
-    A, p, r = inputs.generate(w, DEV)
-    run_and_compare(A, p, r, 700)
+# ---- strided batches --------------------------------------------------------
+
+def _batched_variants():
+    return [(tag, i) for tag, code in CODE.items() for i in range(dm.dualmv_variant_count(code))
+            if dm.dualmv_variant_info(code, i).batched]
+
+
+def _make_batched(dtype, B, M, N, lda, seed):
+    w = inputs.Workload("tb", dtype, M, N, lda, DIST[dtype], seed, batch=B)
+    return inputs.generate(w, DEV)
+
+
+# Row strides and problem strides are multiples of 16 bytes (the 3-D tensor
+# map); ragged M and N, one band, many bands.
+BATCHED_SHAPES = [(3, 513, 1000, 4), (5, 64, 3000, 4), (2, 1000, 257, 7), (4, 1, 300, 4)]
+
+
+@pytest.mark.parametrize("tag,index", _batched_variants())
+@pytest.mark.parametrize("B,M,N,pad", BATCHED_SHAPES)
+def test_every_batched_variant_matches_oracle(tag, index, B, M, N, pad, forced):
+    forced(tag, index)
+    A, p, r = _make_batched(tag, B, M, N, N + pad, 300 + index + M)
+    run_and_compare(A, p, r, N)
+    assert dm.dualmv_last_variant() == index
+
+
+def test_batched_calls_run_entry_zero_for_a_variant_without_batched_instance(forced):
+    for tag, code in CODE.items():
+        plain = [i for i in range(dm.dualmv_variant_count(code))
+                 if not dm.dualmv_variant_info(code, i).batched]
+        if not plain:
+            continue
+        forced(tag, plain[0])
+        A, p, r = _make_batched(tag, 3, 300, 700, 704, 9)
+        run_and_compare(A, p, r, 700)
+        assert dm.dualmv_last_variant() == 0, (tag, plain[0])
+
+
+@pytest.mark.parametrize("tag", ["f32", "f64", "i32"])
+def test_batched_tuner_report_and_choice(tag):
+    B, M, N = 16, 1024, 2048
+    A, p, r = _make_batched(tag, B, M, N, N, 17)
+    code = CODE[tag]
+    dm.dualmv_tune_clear()
+    rep = dm.tune(A, p, r, repeats=9, trim=2, max_rounds=2, candidates=3, min_gain=0.0,
+                  flush_l2=True)
+    torch.cuda.synchronize()
+    assert rep["initial"] == 0
+    assert dm.dualmv_variant_info(code, rep["best"]).batched == 1
+    assert rep["evaluated"] >= 1 and rep["rejected"] == 0
+    assert all(dm.dualmv_variant_info(code, st["index"]).batched for st in rep["trace"])
+    assert 0 < rep["best_ms"] <= rep["baseline_ms"]
+    assert rep["worst_fe"] <= TOL[tag]
+    # The outputs the tuner left are the chosen variant's: against the oracle.
+    An, pn, rn = A.cpu().numpy(), p.cpu().numpy(), r.cpu().numpy()
+    qg, sg = rep["q"].cpu().numpy(), rep["s"].cpu().numpy()
+    for b in range(B):
+        assert compare_problem(tag, qg[b], sg[b], An[b], pn[b], rn[b], N) <= TOL[tag]
+    # Recorded for (dtype, M, N, lda, batch) and used by later batched calls;
+    # the single-problem record and other batch counts are untouched.
+    assert dm.dualmv_tuned_variant_batched(code, M, N, N, B) == rep["best"]
+    assert dm.dualmv_tuned_variant(code, M, N, N) == -1
+    assert dm.dualmv_tuned_variant_batched(code, M, N, N, B + 1) == -1
+    dm.dualmv(A, p, r)
+    torch.cuda.synchronize()
+    assert dm.dualmv_last_variant() == rep["best"]
+    dm.dualmv_tune_clear()
+
+
+def test_batched_tuner_catches_a_planted_mistake(monkeypatch):
+    monkeypatch.setenv("DUALMV_FAULT_INJECT", "fe")
+    A, p, r = _make_batched("f32", 8, 512, 1024, 1024, 23)
+    dm.dualmv_tune_clear()
+    rep = dm.tune(A, p, r, repeats=7, trim=1, max_rounds=2, candidates=3, min_gain=0.0,
+                  flush_l2=False)
+    torch.cuda.synchronize()
+    assert rep["evaluated"] >= 1 and rep["rejected"] == rep["evaluated"]
+    assert rep["best"] == 0
+    dm.dualmv_tune_clear()

@@ -165,3 +165,61 @@ def test_tune_rejects_bad_problem(tag):
 
 def test_last_variant_before_any_call():
     assert dm.dualmv_last_variant() == -1
+
+
+# ---- strided batches ------------------------------------------------------
+
+def _batched_ids(tab):
+    return {i for i, v in enumerate(tab) if v.batched}
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_batched_instances(dtype):
+    """Entry 0 (what untuned batched calls run) and every streaming-kernel
+    shape have a batched instance; the wide int32 tiles do not; the tuner's
+    walk over the batched entries reaches each of them from entry 0."""
+    tab = table(dtype)
+    ids = _batched_ids(tab)
+    assert 0 in ids
+    for i, v in enumerate(tab):
+        if v.kernel == dm.DUALMV_KERNEL_STREAM and dtype != dm.DUALMV_DTYPE_F64:
+            assert v.batched == 1, i
+        if v.kernel == dm.DUALMV_KERNEL_WIDE:
+            assert v.batched == 0, i
+        assert v.batched in (0, 1)
+    assert len(ids) >= 4
+    seen, todo = {0}, [0]
+    while todo:
+        i = todo.pop()
+        for j in ids:
+            if j not in seen and _neighbours(tab[i], tab[j]):
+                seen.add(j)
+                todo.append(j)
+    assert seen == ids
+
+
+def test_no_batched_tuned_variant_recorded_by_default():
+    dm.dualmv_tune_clear()
+    assert dm.dualmv_tuned_variant_batched(dm.DUALMV_DTYPE_F32, 2048, 2048, 2048, 256) == -1
+    assert dm.dualmv_tuned_variant_batched(dm.DUALMV_DTYPE_F64, 64, 64, 64, 1) == -1
+
+
+@pytest.mark.parametrize("tag", ["f32", "f64", "i32"])
+def test_batched_tune_rejects_bad_arguments(tag):
+    fn = getattr(dm, f"dualmv_tune_{tag}_strided_batched")
+    res = dm.TuneResult()
+    good = (64, 64, FAKE, 64, 4096, FAKE, 64, FAKE, 64, FAKE, 64, FAKE, 64, 3)
+
+    def call(args, cfg=_cfg(), r=res):
+        return fn(*args, cfg, r, None)
+    assert call(good, cfg=_cfg(repeats=4, trim=2)) == dm.DUALMV_ERR_INVALID_VALUE
+    assert call(good, cfg=None) == dm.DUALMV_ERR_INVALID_VALUE
+    assert call(good, r=None) == dm.DUALMV_ERR_INVALID_VALUE
+    bad_lda = good[:3] + (63,) + good[4:]
+    assert call(bad_lda) == dm.DUALMV_ERR_INVALID_VALUE
+    bad_stride_q = good[:10] + (63,) + good[11:]          # q rows overlap
+    assert call(bad_stride_q) == dm.DUALMV_ERR_INVALID_VALUE
+    neg_batch = good[:13] + (-1,)
+    assert call(neg_batch) == dm.DUALMV_ERR_INVALID_VALUE
+    null_a = good[:2] + (None,) + good[3:]
+    assert call(null_a) == dm.DUALMV_ERR_INVALID_VALUE

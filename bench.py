@@ -541,8 +541,8 @@ def run_native(args):
         dm.dualmv_set_variant({"f32": 0, "f64": 1, "i32": 2}[w.dtype], args.variant)
     tuned = None
     if args.tune:
-        if w.op != "bicg" or w.batched:
-            raise SystemExit("--tune applies to one unbatched dual product")
+        if w.op != "bicg":
+            raise SystemExit("--tune applies to the dual product (one problem or a batch)")
         t0 = time.time()
         Av = st["A"][..., : w.N]
         rep = dm.tune(Av, st["p"], st["r"], repeats=30, trim=3, max_rounds=4, candidates=8,

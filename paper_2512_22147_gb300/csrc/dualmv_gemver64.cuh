@@ -97,7 +97,7 @@ gemver_rows_update_f64_kernel(const GvParams prm) {
         const double u1i = prm.u1[i], u2i = prm.u2[i];
 
         // t's partial from the original a: products as double-float pairs,
-        // summed in a pairwise tree over the lane's 16 column pairs.
+        // summed in a pairwise tree over the lane's kGvVec column pairs.
         DF2 stk[5];
         uint32_t spanv[2] = {0u, 0u};
 #pragma unroll

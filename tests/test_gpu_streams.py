@@ -1,0 +1,137 @@
+"""Calls in flight together, and calls captured in a CUDA graph.
+
+Every call takes its scratch from the library's stream-ordered pool, so
+calls on different streams may run at once, and calls captured in a graph
+replay with scratch of their own.  These tests check, for each path (the
+single-cluster kernel, the fp32 and int32 streaming kernels, the
+double-float fp64 kernel, a strided batch, GEMVER):
+
+  * the same problems launched on several streams without waiting for one
+    another give the bits of the same problems run one after another;
+  * a graph of such calls, replayed several times, gives the bits of the
+    eager calls, and those bits match the oracle."""
+import pytest
+import torch
+
+import paper_2512_22147_gb300 as dm
+from paper_2512_22147_gb300 import inputs
+from parity import TOL, compare_problem
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+
+PROBLEMS = [
+    inputs.Workload("cluster", "f32", 1024, 1024, 1024, "uniform", 41),
+    inputs.Workload("stream32", "f32", 3000, 5000, 5000, "uniform", 42),
+    inputs.Workload("f64e", "f64", 2000, 3000, 3000, "normal", 43),
+    inputs.Workload("int32", "i32", 1000, 4100, 4104, "int8", 44),
+    inputs.Workload("batch", "f32", 500, 700, 704, "uniform", 45, batch=3),
+]
+
+
+def _problems():
+    out = []
+    for w in PROBLEMS:
+        A, p, r = inputs.generate(w, DEV)
+        q, s = inputs.empty_outputs(w, DEV)
+        out.append((w, A[..., :w.N], p, r, q, s))
+    return out
+
+
+def _check_oracle(w, A, p, r, q, s):
+    An, pn, rn = A.cpu().numpy(), p.cpu().numpy(), r.cpu().numpy()
+    qg, sg = q.cpu().numpy(), s.cpu().numpy()
+    if w.batched:
+        for b in range(w.batch):
+            assert compare_problem(w.dtype, qg[b], sg[b], An[b], pn[b], rn[b], w.N) <= TOL[w.dtype]
+    else:
+        assert compare_problem(w.dtype, qg, sg, An, pn, rn, w.N) <= TOL[w.dtype]
+
+
+def test_concurrent_streams_give_the_serial_bits():
+    probs = _problems()
+    serial = []
+    for w, A, p, r, q, s in probs:
+        dm.dualmv(A, p, r, q=q, s=s)
+        torch.cuda.synchronize()
+        serial.append((q.clone(), s.clone()))
+        _check_oracle(w, A, p, r, q, s)
+    streams = [torch.cuda.Stream(DEV) for _ in probs]
+    for rep in range(3):
+        for (w, A, p, r, q, s) in probs:
+            q.zero_()
+            s.zero_()
+        torch.cuda.synchronize()
+        # Each problem on its own stream, twice in a row, nothing in between.
+        for st, (w, A, p, r, q, s) in zip(streams, probs):
+            with torch.cuda.stream(st):
+                dm.dualmv(A, p, r, q=q, s=s)
+                dm.dualmv(A, p, r, q=q, s=s)
+        torch.cuda.synchronize()
+        assert dm.device_fault() == dm.DUALMV_SUCCESS
+        for (w, A, p, r, q, s), (q0, s0) in zip(probs, serial):
+            assert torch.equal(q, q0) and torch.equal(s, s0), (w.name, rep)
+
+
+def test_graph_replays_give_the_eager_bits():
+    probs = _problems()
+    eager = []
+    for w, A, p, r, q, s in probs:
+        dm.dualmv(A, p, r, q=q, s=s)
+        torch.cuda.synchronize()
+        eager.append((q.clone(), s.clone()))
+    side = torch.cuda.Stream(DEV)
+    side.wait_stream(torch.cuda.current_stream(DEV))
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side):
+        for w, A, p, r, q, s in probs:   # warm the pool on this stream first
+            dm.dualmv(A, p, r, q=q, s=s)
+        side.synchronize()
+        with torch.cuda.graph(graph, stream=side):
+            for w, A, p, r, q, s in probs:
+                dm.dualmv(A, p, r, q=q, s=s)
+    torch.cuda.current_stream(DEV).wait_stream(side)
+    for rep in range(3):
+        for (w, A, p, r, q, s) in probs:
+            q.zero_()
+            s.zero_()
+        graph.replay()
+        torch.cuda.synchronize()
+        for (w, A, p, r, q, s), (q0, s0) in zip(probs, eager):
+            assert torch.equal(q, q0) and torch.equal(s, s0), (w.name, rep)
+    for w, A, p, r, q, s in probs:
+        _check_oracle(w, A, p, r, q, s)
+    del graph
+
+
+def test_gemver_on_two_streams_at_once():
+    """Two GEMVER problems (fp64 factorised and with update_A) on two
+    streams at once give the bits of the same calls run one after another."""
+    ops = [inputs.generate_gemver(inputs.Workload("g", "f64", 1500, 2000, 2000, "normal",
+                                                  50 + k, op="gemver"), DEV) for k in range(2)]
+    upd = [False, True]
+
+    def run_all(concurrent):
+        outs = []
+        streams = [torch.cuda.Stream(DEV) for _ in ops]
+        copies = [[t.clone() for t in o] for o in ops]
+        torch.cuda.synchronize()
+        for k, (st, c) in enumerate(zip(streams, copies)):
+            A, u1, v1, u2, v2, w, x, y, z = c
+            if concurrent:
+                with torch.cuda.stream(st):
+                    dm.gemver(A, u1, v1, u2, v2, w, x, y, z, alpha=1.5, beta=0.5,
+                              update_A=upd[k])
+            else:
+                dm.gemver(A, u1, v1, u2, v2, w, x, y, z, alpha=1.5, beta=0.5, update_A=upd[k])
+                torch.cuda.synchronize()
+            outs.append((A, w, x))
+        torch.cuda.synchronize()
+        return outs
+
+    serial = run_all(False)
+    for _ in range(2):
+        conc = run_all(True)
+        for a, b in zip(serial, conc):
+            for t0, t1 in zip(a, b):
+                assert torch.equal(t0, t1)

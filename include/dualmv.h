@@ -139,9 +139,10 @@ dualmv_status dualmv_atax_f64(int64_t M, int64_t N, const double *A, int64_t lda
  * row stride lda * sizeof(element) is a multiple of 16 bytes and whose
  * width fits a thread-block cluster of at most 16 CTAs streams A once: the
  * CTAs of a cluster share each 4-row stripe (each CTA a slice of the
- * columns: 16 warps x 256 columns = 4096 for fp32, 8 warps x 256 = 2048 for
- * fp64), exchange the stripe's partial row sums through distributed shared
- * memory, and form A^T tmp from the copy still on chip.  So fp32 takes this
+ * columns: 16 warps x 256 columns = 4096 for fp32; 8 sub-bands x 256 = 2048
+ * for fp64, each sub-band with a warp for its row sums and one for its
+ * column sums), exchange the stripe's partial row sums through distributed
+ * shared memory, and form A^T tmp from the copy still on chip.  So fp32 takes this
  * path for N <= 65536 and fp64 (in double-float arithmetic on the FP32
  * pipes, native fp64 for stripes with values outside [2^-40, 2^40)) for
  * N <= 32768, when the GPU can place such a cluster.  Other problems read A

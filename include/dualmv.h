@@ -169,12 +169,12 @@ int32_t dualmv_atax_last_path(void);
  * in double-float arithmetic on the FP32 pipes for fp64.  With update_A
  * nonzero the rows-only pass also writes A_hat over A (as the PolyBench
  * kernel does), each element read before it is written by the same thread:
- *   - fp64 with A 16-byte aligned and lda even: the columns-only pass and
- *     the x update are those of the factorised form; the rows pass writes
- *     A_hat = fma(u2_i, v2_j, fma(u1_i, v1_j, a)) in native fp64 and forms
- *     A x + u1 (v1 . x) + u2 (v2 . x) from the original A in double-float
- *     (native fp64 for rows or bands with values outside [2^-40, 2^40),
- *     zeros excepted);
+ *   - A 16-byte aligned and lda * sizeof(element) a multiple of 16: the
+ *     columns-only pass and the x update are those of the factorised form;
+ *     one rows pass writes A_hat = fma(u2_i, v2_j, fma(u1_i, v1_j, a)) and
+ *     forms A x + u1 (v1 . x) + u2 (v2 . x) from the original A (fp64:
+ *     A_hat in native fp64, A x in double-float, native fp64 for rows or
+ *     bands with values outside [2^-40, 2^40), zeros excepted);
  *   - otherwise both passes form A_hat element by element as they stream
  *     A (native fp64 arithmetic for fp64).
  * The written A_hat is the same fused form on every path. */
@@ -199,8 +199,9 @@ int dualmv_gemver_set_onthefly(int onthefly);
 
 /* Which form the calling thread's last GEMVER call took:
  * DUALMV_GEMVER_FACTORED (update_A == 0 without the on-the-fly setting),
- * DUALMV_GEMVER_UPDATE_SPLIT (update_A, fp64, the double-float rows pass
- * above) or DUALMV_GEMVER_ONTHEFLY (A_hat formed element by element); -1
+ * DUALMV_GEMVER_UPDATE_SPLIT (update_A, aligned rows: the factorised
+ * columns pass and the rows pass that writes A_hat, above) or
+ * DUALMV_GEMVER_ONTHEFLY (A_hat formed element by element); -1
  * after an empty problem or an argument error.  Instrumentation for tests. */
 enum { DUALMV_GEMVER_FACTORED = 0, DUALMV_GEMVER_ONTHEFLY = 1, DUALMV_GEMVER_UPDATE_SPLIT = 2 };
 int32_t dualmv_gemver_last_path(void);

@@ -21,7 +21,7 @@ SOURCES = [os.path.join(CSRC, "dualmv.cu")]
 DEPENDS = SOURCES + [os.path.join(CSRC, n) for n in (
     "dualmv_kernels.cuh", "dualmv_f64e.cuh", "dualmv_tune.cuh", "dualmv_wide.cuh",
     "dualmv_atax.cuh", "dualmv_atax_f64.cuh", "dualmv_ops.cuh", "dualmv_probe.cuh", "dualmv_small.cuh",
-    "dualmv_gemver64.cuh")] + [
+    "dualmv_gemver_update.cuh")] + [
     os.path.join(INCLUDE, "dualmv.h")]
 
 NVCC_FLAGS = [

@@ -27,7 +27,7 @@
 #include "dualmv_ops.cuh"
 #include "dualmv_probe.cuh"
 #include "dualmv_small.cuh"
-#include "dualmv_gemver64.cuh"
+#include "dualmv_gemver_update.cuh"
 
 namespace {
 
@@ -1631,42 +1631,45 @@ dualmv_status gemver_factored(int64_t M, int64_t N, T alpha, T beta, const T *A,
 }
 
 // GEMVER (Table 1 / Table 2): A_hat = A + u1 v1^T + u2 v2^T;
-// GEMVER with update_A in fp64: the factorised columns pass and x update of
-// gemver_factored_fused, then gemver_rows_update_f64_kernel, which writes
-// A_hat over A and leaves the band partials of A x (original A, in
-// double-float), and the w update, which adds them.  A read twice and
-// written once; two DFMAs per element (A_hat) where the on-the-fly kernel
-// takes three.  Needs A 16-byte aligned and lda even.
-dualmv_status gemver_update_f64(int64_t M, int64_t N, double alpha, double beta, double *A,
-                                int64_t lda, const double *u1, const double *v1,
-                                const double *u2, const double *v2, double *w, double *x,
-                                const double *y, const double *z, cudaStream_t stream) {
+// GEMVER with update_A: the factorised columns pass and x update of
+// gemver_factored_fused, then gemver_rows_update_{f64,f32}_kernel, which
+// writes A_hat over A and leaves the band partials of A x (original A), and
+// the w update, which adds them.  A read twice and written once.  fp64: two
+// DFMAs per element (A_hat) where the on-the-fly kernel takes three.
+// Needs A 16-byte aligned and a row stride that is a multiple of 16 bytes.
+template <typename T>
+dualmv_status gemver_update(int64_t M, int64_t N, T alpha, T beta, T *A, int64_t lda,
+                            const T *u1, const T *v1, const T *u2, const T *v2, T *w, T *x,
+                            const T *y, const T *z, cudaStream_t stream) {
+    constexpr bool kF64 = std::is_same<T, double>::value;
+    constexpr int64_t kBand = kF64 ? dmv::kGvBand : dmv::kGvBand32;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return cuda_fail(e);
     DeviceState *dst = nullptr;
     e = device_state(dev, &dst);
     if (e != cudaSuccess) return cuda_fail(e);
-    const int64_t bands = (N + dmv::kGvBand - 1) / dmv::kGvBand;
+    const int64_t bands = (N + kBand - 1) / kBand;
     int64_t row_chunks = (2 * (int64_t)dst->sms + bands - 1) / bands;
     if (row_chunks > M) row_chunks = M;
     if (row_chunks < 1) row_chunks = 1;
     if (bands > 65535 || row_chunks > INT32_MAX) return DUALMV_ERR_UNSUPPORTED;
-    double *s = nullptr, *part = nullptr, *qws = nullptr;
+    T *s = nullptr, *qws = nullptr;
+    double *part = nullptr;  // [side][2 products][kDotChunks][sum, error]
     dualmv_status st = pool_alloc(&s, N, stream);
     if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * 2 * dmv::kDotChunks, stream);
     if (st == DUALMV_SUCCESS) st = pool_alloc(&qws, bands * M, stream);
     double *part_u = part, *part_v = part ? part + 2 * 2 * dmv::kDotChunks : nullptr;
     Deferred ds;
     if (st == DUALMV_SUCCESS)
-        e = launch_dependent(dmv::dots2_partial_kernel<double>, dim3(2 * dmv::kDotChunks),
+        e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks),
                              dim3(256), 0, stream, u1, u2, y, M, part_u);
     if (st == DUALMV_SUCCESS && e == cudaSuccess)  // s = A^T y, left as partials
-        st = run<double, double>(M, N, A, lda, 0, nullptr, 0, y, 0, nullptr, 0, s, 0, 1, stream,
-                                 dmv::kOutS, nullptr, -1, &ds);
+        st = run<T, T>(M, N, A, lda, 0, nullptr, 0, y, 0, nullptr, 0, s, 0, 1, stream,
+                       dmv::kOutS, nullptr, -1, &ds);
     if (st == DUALMV_SUCCESS && e == cudaSuccess) {
         if (!ds.used) ds.prm.s = s;
-        e = launch_dependent(dmv::gemver_x3_kernel<double>, dim3(dmv::kDotChunks), dim3(256), 0,
+        e = launch_dependent(dmv::gemver_x3_kernel<T>, dim3(dmv::kDotChunks), dim3(256), 0,
                              stream, ds.prm, ds.used ? 0 : 1, (const double *)part_u, x, v1,
                              v2, z, N, beta, part_v);
     }
@@ -1675,7 +1678,7 @@ dualmv_status gemver_update_f64(int64_t M, int64_t N, double alpha, double beta,
         if (e == cudaSuccess) e = ef;
     }
     if (st == DUALMV_SUCCESS && e == cudaSuccess) {
-        dmv::GvParams gp;
+        dmv::GvParams<T> gp;
         std::memset(&gp, 0, sizeof gp);
         gp.A = A;
         gp.lda = lda;
@@ -1689,9 +1692,13 @@ dualmv_status gemver_update_f64(int64_t M, int64_t N, double alpha, double beta,
         gp.N = N;
         gp.bands = bands;
         gp.row_chunks = row_chunks;
-        e = launch_dependent(dmv::gemver_rows_update_f64_kernel,
-                             dim3((unsigned)row_chunks, (unsigned)bands), dim3(dmv::kGvWarps * 32),
-                             0, stream, gp);
+        const dim3 grid((unsigned)row_chunks, (unsigned)bands);
+        if constexpr (kF64)
+            e = launch_dependent(dmv::gemver_rows_update_f64_kernel, grid,
+                                 dim3(dmv::kGvWarps * 32), 0, stream, gp);
+        else
+            e = launch_dependent(dmv::gemver_rows_update_f32_kernel, grid,
+                                 dim3(dmv::kGvWarps * 32), 0, stream, gp);
     }
     if (st == DUALMV_SUCCESS && e == cudaSuccess) {
         Params pq;
@@ -1705,7 +1712,7 @@ dualmv_status gemver_update_f64(int64_t M, int64_t N, double alpha, double beta,
         const int64_t bw = (M + rows - 1) / rows;
         if (bw > INT32_MAX) e = cudaErrorInvalidConfiguration;
         else
-            e = launch_dependent(dmv::gemver_w3_kernel<double>, dim3((unsigned)bw), dim3(256), 0,
+            e = launch_dependent(dmv::gemver_w3_kernel<T>, dim3((unsigned)bw), dim3(256), 0,
                                  stream, pq, 0, chunks, w, u1, u2, (const double *)part_v, M,
                                  alpha);
     }
@@ -1742,13 +1749,10 @@ dualmv_status gemver_run(int64_t M, int64_t N, T alpha, T beta, T *A, int64_t ld
         return gemver_factored<T>(M, N, alpha, beta, A, lda, u1, v1, u2, v2, w, x, y, z,
                                   stream);
     }
-    if constexpr (std::is_same<T, double>::value) {
-        if (g_gemver_onthefly == 0 && M > 0 && N > 0 && lda % 2 == 0 &&
-            reinterpret_cast<uintptr_t>(A) % 16 == 0) {
-            g_last_gemver_path = DUALMV_GEMVER_UPDATE_SPLIT;
-            return gemver_update_f64(M, N, alpha, beta, A, lda, u1, v1, u2, v2, w, x, y, z,
-                                     stream);
-        }
+    if (g_gemver_onthefly == 0 && M > 0 && N > 0 && (lda * (int64_t)sizeof(T)) % 16 == 0 &&
+        reinterpret_cast<uintptr_t>(A) % 16 == 0) {
+        g_last_gemver_path = DUALMV_GEMVER_UPDATE_SPLIT;
+        return gemver_update<T>(M, N, alpha, beta, A, lda, u1, v1, u2, v2, w, x, y, z, stream);
     }
     g_last_gemver_path = DUALMV_GEMVER_ONTHEFLY;
     T *s = nullptr, *t = nullptr;

@@ -101,6 +101,8 @@ OP_WORKLOADS = {
         Workload("gemver_f64_8192x8192", "f64", 8192, 8192, 8192, "normal", 10, op="gemver"),
         Workload("gemver_update_f64_8192x8192", "f64", 8192, 8192, 8192, "normal", 11,
                  op="gemver", update_a=True),
+        Workload("gemver_update_f32_16384x16384", "f32", 16384, 16384, 16384, "uniform", 12,
+                 op="gemver", update_a=True),
     )
 }
 

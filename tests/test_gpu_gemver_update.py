@@ -1,16 +1,17 @@
-"""GEMVER with update_A in fp64: the double-float rows pass
-(dualmv_gemver64.cuh) against the oracle.
+"""GEMVER with update_A: the rows pass that writes A_hat
+(dualmv_gemver_update.cuh) against the oracle.
 
-With A 16-byte aligned and lda even, an fp64 call with update_A runs the
-factorised columns pass and x update, then one kernel that writes
-A_hat = fma(u2_i, v2_j, fma(u1_i, v1_j, a)) over A and forms A x from the
-original A in double-float arithmetic.  These tests check, element by
-element against the oracle within the fp64 bar (A_hat, x and w):
+With A 16-byte aligned and a row stride that is a multiple of 16 bytes, a
+call with update_A runs the factorised columns pass and x update, then one
+kernel that writes A_hat = fma(u2_i, v2_j, fma(u1_i, v1_j, a)) over A and
+forms A x from the original A (fp64: in double-float arithmetic).  These
+tests check, element by element against the oracle within the dtype's bar
+(A_hat, x and w):
 
-  * the path taken (and the fallbacks: odd lda, a base off the 16-byte
-    grid, fp32, the on-the-fly setting);
-  * widths around the kernel's 512-column bands (ragged last band, one
-    column, a band and one);
+  * the path taken (and the fallbacks: a row stride off the 16-byte grid, a
+    base off it, the on-the-fly setting);
+  * widths around the kernels' bands (fp64: 512 columns, fp32: 1024; ragged
+    last band, one column, a band and one);
   * values outside [2^-40, 2^40) in rows of A and in the new x (native fp64
     for those rows or that band), and zero rows;
   * repeated calls giving the same bits, and the padding columns untouched;
@@ -32,8 +33,8 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
 
 
-def _ops(M, N, lda, seed):
-    return inputs.generate_gemver(_w("gemver", "f64", M, N, lda, seed), DEV)
+def _ops(M, N, lda, seed, dtype="f64"):
+    return inputs.generate_gemver(_w("gemver", dtype, M, N, lda, seed), DEV)
 
 
 @pytest.mark.parametrize("M,N,pad", [(300, 512, 0), (300, 511, 1), (300, 513, 1), (64, 1, 1),
@@ -42,6 +43,14 @@ def test_update_split_matches_oracle(M, N, pad):
     err = check_gemver(_ops(M, N, N + pad, M * 7 + N), N, 1.5, -0.75, True, "f64")
     assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_UPDATE_SPLIT
     print(f"gemver update_A {M}x{N}+{pad}: {err:.3e}")
+
+
+@pytest.mark.parametrize("M,N,pad", [(300, 1024, 0), (300, 1023, 1), (300, 1025, 3), (64, 1, 3),
+                                     (200, 2049, 3), (2, 8192, 0), (4097, 300, 0)])
+def test_update_f32_matches_oracle(M, N, pad):
+    err = check_gemver(_ops(M, N, N + pad, M * 5 + N, "f32"), N, 1.5, -0.75, True, "f32")
+    assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_UPDATE_SPLIT
+    print(f"gemver f32 update_A {M}x{N}+{pad}: {err:.3e}")
 
 
 def test_path_taken_and_fallbacks():
@@ -66,7 +75,11 @@ def test_path_taken_and_fallbacks():
     finally:
         dm.dualmv_gemver_set_onthefly(old)
     f = [t.float() for t in (C[:, :300],) + args]
-    dm.gemver(f[0], *f[1:], update_A=True)
+    dm.gemver(f[0], *f[1:], update_A=True)                       # fp32, 1200-byte rows
+    assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_UPDATE_SPLIT
+    F = torch.empty(100, 302, dtype=torch.float32, device=DEV)   # 1208-byte rows
+    F[:, :300] = f[0]
+    dm.gemver(F[:, :300], *f[1:], update_A=True)
     assert dm.dualmv_gemver_last_path() == dm.DUALMV_GEMVER_ONTHEFLY
     dm.gemver(C[:0, :0], u1[:0], v1[:0], u2[:0], v2[:0], w[:0], x[:0], y[:0], z[:0],
               update_A=True)
@@ -90,9 +103,10 @@ def test_out_of_range_values(case):
     assert dm.device_fault() == dm.DUALMV_SUCCESS
 
 
-def test_repeated_calls_are_bit_identical():
+@pytest.mark.parametrize("dtype", ["f64", "f32"])
+def test_repeated_calls_are_bit_identical(dtype):
     M, N = 1500, 2000
-    ops = _ops(M, N, N + 2, 5)
+    ops = _ops(M, N, N + 4, 5, dtype)
     outs = []
     for _ in range(2):
         A, u1, v1, u2, v2, w, x, y, z = (t.clone() for t in ops)

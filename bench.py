@@ -485,8 +485,8 @@ def launches_per_call(torch, dm, inputs, w, dev) -> int:
     n = 1 + (1 if (plan.bands > 1 or plan.grid > 1) else 0)
     if w.op == "bicg" and dm.dualmv_last_kernel() == dm.DUALMV_KERNEL_CLUSTER:
         n = 1   # one cluster computes both outputs, no combine kernel
-    if w.op == "gesummv":   # two row passes (stream + combine each) + epilogue
-        return 2 * n + 1
+    if w.op == "gesummv":   # two row passes, then one kernel adds their partials into y
+        return 3
     if w.op == "atax":      # a row pass and a column pass
         return 2 * n
     if w.op == "gemver":    # u.y dots, column pass, x update, row pass, w update

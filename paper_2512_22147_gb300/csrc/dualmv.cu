@@ -1284,23 +1284,41 @@ dualmv_status gesummv_run(int64_t M, int64_t N, T alpha, const T *A, int64_t lda
         return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
     }
     if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
+    // Both rows-only passes leave their band partials (no combine kernels);
+    // gesummv_final_kernel adds them in the combine's order and forms y.
     T *tmp = nullptr;
     dualmv_status st = pool_alloc(&tmp, M, stream);
     if (st != DUALMV_SUCCESS) return st;
+    Deferred da, db;
     st = run<T, T>(M, N, A, lda, 0, x, 0, nullptr, 0, tmp, 0, nullptr, 0, 1, stream,
-                   dmv::kOutQ);
+                   dmv::kOutQ, nullptr, -1, &da);
     if (st == DUALMV_SUCCESS)
         st = run<T, T>(M, N, B, ldb, 0, x, 0, nullptr, 0, y, 0, nullptr, 0, 1, stream,
-                       dmv::kOutQ);
+                       dmv::kOutQ, nullptr, -1, &db);
+    cudaError_t e = cudaSuccess;
     if (st == DUALMV_SUCCESS) {
-        int64_t blocks = (M + 255) / 256;
-        if (blocks > 4096) blocks = 4096;
-        dmv::axpby_kernel<T><<<(unsigned)blocks, 256, 0, stream>>>(tmp, y, M, alpha, beta);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) st = cuda_fail(e);
+        if (!da.used) da.prm.q = tmp;
+        if (!db.used) db.prm.q = y;
+        const int a_direct = (!da.used || da.prm.bands == 1) ? 1 : 0;
+        const int b_direct = (!db.used || db.prm.bands == 1) ? 1 : 0;
+        const int chunks = da.used ? da.chunks : db.used ? db.chunks : 1;
+        const int64_t rows = 256 / chunks;
+        const int64_t blocks = (M + rows - 1) / rows;
+        if (blocks > INT32_MAX) {
+            st = DUALMV_ERR_UNSUPPORTED;
+        } else {
+            e = launch_dependent(dmv::gesummv_final_kernel<T>, dim3((unsigned)blocks), dim3(256),
+                                 0, stream, da.prm, a_direct, db.prm, b_direct, chunks, y, M,
+                                 alpha, beta);
+            if (e != cudaSuccess) st = cuda_fail(e);
+        }
     }
-    cudaError_t ef = cudaFreeAsync(tmp, stream);
-    if (st == DUALMV_SUCCESS && ef != cudaSuccess) st = cuda_fail(ef);
+    void *bufs[3] = {da.ws, db.ws, tmp};
+    for (void *bp : bufs) {
+        if (bp == nullptr) continue;
+        cudaError_t ef = cudaFreeAsync(bp, stream);
+        if (st == DUALMV_SUCCESS && ef != cudaSuccess) st = cuda_fail(ef);
+    }
     return st;
 }
 

@@ -17,6 +17,57 @@ __global__ void axpby_kernel(const T *t, T *y, int64_t n, T alpha, T beta) {
         y[i] = alpha * t[i] + beta * y[i];
 }
 
+// GESUMMV's last step with both passes' combines folded in: row i of each
+// pass from its band partials, added as the combine kernel adds them (C
+// threads per row, thread y adding bands y, y + C, ..., then the C chunk
+// sums in order: the combine's bits), or read from the pass's output when
+// it wrote q itself; then y = alpha * t_A + beta * t_B, as axpby_kernel
+// forms it.  Both passes have the same bands, so one C.  Blocks of 256
+// threads over 256 / C rows; launched as a programmatic dependent of the
+// second pass.
+template <typename T>
+__global__ void __launch_bounds__(256)
+gesummv_final_kernel(const Params pa, int a_direct, const Params pb, int b_direct, int C, T *y,
+                     int64_t m, T alpha, T beta) {
+    pdl_launch_dependents();
+    pdl_wait();
+    __shared__ T chunk_a[256], chunk_b[256];
+    const int R = 256 / C, xr = threadIdx.x % R, yc = threadIdx.x / R;
+    const int64_t i = (int64_t)blockIdx.x * R + xr;
+    const bool valid = i < m;
+    auto chunk = [&](const Params &pp) -> T {
+        const T *base = static_cast<const T *>(pp.q_ws) + i;
+        T acc = T(0);
+        int64_t k = yc;
+        if (k < pp.bands) {
+            acc = base[k * pp.M];
+            k += C;
+        }
+#pragma unroll 4
+        for (; k < pp.bands; k += C) acc = acc + base[k * pp.M];
+        return acc;
+    };
+    chunk_a[threadIdx.x] = (valid && !a_direct) ? chunk(pa) : T(0);
+    chunk_b[threadIdx.x] = (valid && !b_direct) ? chunk(pb) : T(0);
+    __syncthreads();
+    if (yc == 0 && valid) {
+        T ta, tb;
+        if (a_direct) {
+            ta = static_cast<const T *>(pa.q)[i];
+        } else {
+            ta = chunk_a[xr];
+            for (int c = 1; c < C; ++c) ta = ta + chunk_a[c * R + xr];
+        }
+        if (b_direct) {
+            tb = static_cast<const T *>(pb.q)[i];
+        } else {
+            tb = chunk_b[xr];
+            for (int c = 1; c < C; ++c) tb = tb + chunk_b[c * R + xr];
+        }
+        y[i] = alpha * ta + beta * tb;
+    }
+}
+
 // GEMVER vector steps: x = (x + beta * s) + z, then w = w + alpha * t.
 template <typename T>
 __global__ void gemver_x_kernel(T *x, const T *s, const T *z, int64_t n, T beta) {

@@ -1423,13 +1423,16 @@ dualmv_status atax_cluster_run(int64_t M, int64_t N, const T *A, int64_t lda, co
     cfg.blockDim = dim3(Cfg::kThreads);
     cfg.dynamicSmemBytes = (size_t)L::kTotal;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
+    // Clusters of C CTAs; a programmatic dependent of the kernel before it.
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = (unsigned)C;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 1;  // the occupancy query takes the cluster shape alone
     int max_clusters = 0;
     {
         std::lock_guard<std::mutex> lk(g_atax_cache.mu);
@@ -1473,12 +1476,13 @@ dualmv_status atax_cluster_run(int64_t M, int64_t N, const T *A, int64_t lda, co
     prm.clusters = clusters;
     prm.bands = bands;
     cfg.gridDim = dim3((unsigned)(clusters * C));
+    cfg.numAttrs = 2;
     e = cudaLaunchKernelEx(&cfg, kern, map, prm);
     if (e == cudaSuccess) {
         int64_t blocks = (N + 255) / 256;
         if (blocks > 4096) blocks = 4096;
-        dmv::atax_sum_kernel<T><<<(unsigned)blocks, 256, 0, stream>>>(ws, y, N, clusters);
-        e = cudaGetLastError();
+        e = launch_dependent(dmv::atax_sum_kernel<T>, dim3((unsigned)blocks), dim3(256), 0,
+                             stream, (const T *)ws, y, N, clusters);
     }
     cudaError_t ef = cudaFreeAsync(ws, stream);
     if (e != cudaSuccess) return cuda_fail(e);

@@ -150,6 +150,11 @@ atax_cluster_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxParams p
     }
     // Every CTA's barriers exist before any peer sends to them.
     cluster_sync();
+    // A programmatic dependent of the kernel before it: its launch and the
+    // set-up above overlap that kernel; nothing in global memory is touched
+    // before that grid has completed.  The sum kernel after it may launch.
+    pdl_wait();
+    pdl_launch_dependents();
 
     float xv[kLaneCols];
 #pragma unroll
@@ -311,6 +316,9 @@ atax_cluster_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxParams p
 template <typename T>
 __global__ void __launch_bounds__(256) atax_sum_kernel(const T *y_ws, T *y, int64_t N,
                                                        int64_t clusters) {
+    // A programmatic dependent of the cluster kernel: waits for its grid.
+    pdl_launch_dependents();
+    pdl_wait();
     const int64_t threads = (int64_t)gridDim.x * blockDim.x;
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < N; j += threads) {
         T acc = T(0);

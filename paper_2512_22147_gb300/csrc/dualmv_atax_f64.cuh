@@ -122,6 +122,9 @@ atax_cluster_f64_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxPara
     }
     // Every CTA's barriers exist before any peer sends to them.
     cluster_sync();
+    // A programmatic dependent of the kernel before it (see atax_cluster_kernel).
+    pdl_wait();
+    pdl_launch_dependents();
 
     // ---------------------------------------------------- control warp ----
     if (warp == W) {
@@ -531,6 +534,9 @@ atax_cluster_f64_ws_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxP
     for (int i = threadIdx.x; i < kAtaxSlots * W * R; i += blockDim.x) wpart[i] = 0.0;
     // Every CTA's barriers exist before any peer sends to them.
     cluster_sync();
+    // A programmatic dependent of the kernel before it (see atax_cluster_kernel).
+    pdl_wait();
+    pdl_launch_dependents();
 
     // ---------------------------------------------------- control warp ----
     if (warp == 2 * W) {

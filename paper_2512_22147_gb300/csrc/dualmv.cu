@@ -927,13 +927,15 @@ cudaError_t launch_small_cluster(const Params &prm, int dev, cudaStream_t stream
     cfg.blockDim = dim3(dmv::kSmallWarps * 32);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = dmv::kSmallCluster;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 1;  // the occupancy query takes the cluster shape alone
     const int slot = VPL == 8 ? 0 : 1;
     {
         std::lock_guard<std::mutex> lk(g_small_cache.mu);
@@ -953,6 +955,7 @@ cudaError_t launch_small_cluster(const Params &prm, int dev, cudaStream_t stream
         if (g_small_cache.ok[slot][dev] < 0) return cudaSuccess;
     }
     *done = true;
+    cfg.numAttrs = 2;  // and a programmatic dependent of the kernel before it
     return cudaLaunchKernelEx(&cfg, kern, prm);
 }
 

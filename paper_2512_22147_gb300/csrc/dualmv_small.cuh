@@ -69,6 +69,11 @@ dualmv_small_cluster_kernel(const Params prm) {
     float *q = static_cast<float *>(prm.q);
     float *s = static_cast<float *>(prm.s);
 
+    // A programmatic dependent of the kernel before it: launched while that
+    // kernel runs, it touches global memory only once that grid is done.
+    pdl_wait();
+    pdl_launch_dependents();
+
     float4 p4[VPL], s4[VPL];
 #pragma unroll
     for (int v = 0; v < VPL; ++v) {

@@ -10,19 +10,12 @@
 
 namespace dmv {
 
-template <typename T>
-__global__ void axpby_kernel(const T *t, T *y, int64_t n, T alpha, T beta) {
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
-         i += (int64_t)gridDim.x * blockDim.x)
-        y[i] = alpha * t[i] + beta * y[i];
-}
-
 // GESUMMV's last step with both passes' combines folded in: row i of each
 // pass from its band partials, added as the combine kernel adds them (C
 // threads per row, thread y adding bands y, y + C, ..., then the C chunk
 // sums in order: the combine's bits), or read from the pass's output when
-// it wrote q itself; then y = alpha * t_A + beta * t_B, as axpby_kernel
-// forms it.  Both passes have the same bands, so one C.  Blocks of 256
+// it wrote q itself; then y = alpha * t_A + beta * t_B.  Both passes have
+// the same bands, so one C.  Blocks of 256
 // threads over 256 / C rows; launched as a programmatic dependent of the
 // second pass.
 template <typename T>

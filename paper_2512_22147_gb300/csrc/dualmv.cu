@@ -1549,12 +1549,12 @@ dualmv_status gemver_factored_fused(int64_t M, int64_t N, T alpha, T beta, const
                                     const T *v2, T *w, T *x, const T *y, const T *z,
                                     cudaStream_t stream) {
     T *s = nullptr, *t = nullptr;
-    // [side][2 products][kDotChunks][sum, error]: u . y, then v . x
+    // [side][2 products][kDotChunks] chunk sums: u . y, then v . x
     double *part = nullptr;
     dualmv_status st = pool_alloc(&s, N, stream);
     if (st == DUALMV_SUCCESS) st = pool_alloc(&t, M, stream);
-    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * 2 * dmv::kDotChunks, stream);
-    double *part_u = part, *part_v = part ? part + 2 * 2 * dmv::kDotChunks : nullptr;
+    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * dmv::kDotChunks, stream);
+    double *part_u = part, *part_v = part ? part + 2 * dmv::kDotChunks : nullptr;
     cudaError_t e = cudaSuccess;
     Deferred ds, dq;
     if (st == DUALMV_SUCCESS)
@@ -1612,12 +1612,12 @@ dualmv_status gemver_factored(int64_t M, int64_t N, T alpha, T beta, const T *A,
                                         stream);
     // An empty dimension: the vector kernels alone (each pass zero-fills).
     T *s = nullptr, *t = nullptr;
-    // [side][2 products][kDotChunks][sum, error]: u . y, then v . x
+    // [side][2 products][kDotChunks] chunk sums: u . y, then v . x
     double *part = nullptr;
     dualmv_status st = pool_alloc(&s, N, stream);
     if (st == DUALMV_SUCCESS) st = pool_alloc(&t, M, stream);
-    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * 2 * dmv::kDotChunks, stream);
-    double *part_u = part, *part_v = part ? part + 2 * 2 * dmv::kDotChunks : nullptr;
+    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * dmv::kDotChunks, stream);
+    double *part_u = part, *part_v = part ? part + 2 * dmv::kDotChunks : nullptr;
     cudaError_t e = cudaSuccess;
     // The vector kernels are programmatic dependents of the kernel before
     // them (each waits for it before reading): their launches overlap it.
@@ -1681,11 +1681,11 @@ dualmv_status gemver_update(int64_t M, int64_t N, T alpha, T beta, T *A, int64_t
     if (row_chunks < 1) row_chunks = 1;
     if (bands > 65535 || row_chunks > INT32_MAX) return DUALMV_ERR_UNSUPPORTED;
     T *s = nullptr, *qws = nullptr;
-    double *part = nullptr;  // [side][2 products][kDotChunks][sum, error]
+    double *part = nullptr;  // [side][2 products][kDotChunks] chunk sums
     dualmv_status st = pool_alloc(&s, N, stream);
-    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * 2 * dmv::kDotChunks, stream);
+    if (st == DUALMV_SUCCESS) st = pool_alloc(&part, 2 * 2 * dmv::kDotChunks, stream);
     if (st == DUALMV_SUCCESS) st = pool_alloc(&qws, bands * M, stream);
-    double *part_u = part, *part_v = part ? part + 2 * 2 * dmv::kDotChunks : nullptr;
+    double *part_u = part, *part_v = part ? part + 2 * dmv::kDotChunks : nullptr;
     Deferred ds;
     if (st == DUALMV_SUCCESS)
         e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks),

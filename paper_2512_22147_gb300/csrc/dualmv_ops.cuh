@@ -78,12 +78,18 @@ __global__ void gemver_w_kernel(T *w, const T *t, int64_t n, T alpha) {
 // ---- GEMVER with the rank-2 update factorised ----------------------------
 //   A_hat^T y = A^T y + v1 (u1 . y) + v2 (u2 . y)
 //   A_hat x   = A x   + u1 (v1 . x) + u2 (v2 . x)
-// Two dot products per side (a . c and b . c), deterministic and
-// compensated: kDotChunks blocks per product each take one contiguous chunk
-// (thread k: elements k, k + 256, ... of the chunk, in order), sum it with
-// TwoProduct/TwoSum in double, and add their threads' sums in a fixed
-// pairwise tree; a second kernel adds the chunks in order.  GB300's FP64
-// pipe is narrow, so the work is spread over many SMs.
+// Two dot products per side (a . c and b . c), deterministic: kDotChunks
+// blocks per product each take one contiguous chunk (thread k: elements
+// k, k + 256, ... of the chunk, in order), sum it with TwoProduct/TwoSum in
+// double, round that compensated sum once, and add the threads' sums in a
+// fixed tree of plain fp64 adds; the kernel that uses the products adds the
+// chunk sums in a fixed tree too.  Along any path there are at most 16
+// roundings after the compensated thread sums, so the error stays within
+// about 16 u sum |a_k c_k|: each term's error is inside the bar, whose
+// denominator holds |u1| (|u1| . |y|) and the like.  GB300's FP64 pipe is
+// narrow, so the work is spread over many SMs and the trees take one add
+// per level (TwoSum trees, eight operations per level, cost the x update
+// 11 us of its call at 8192^2).
 constexpr int kDotChunks = 64;
 
 __device__ __forceinline__ void two_sum_d(double a, double b, double &s, double &e) {
@@ -102,58 +108,54 @@ __device__ __forceinline__ void dot2_step(double x, double y, double &s, double 
     cc += e + pe;
 }
 
-// The block's 256 compensated sums in a fixed pairwise tree; thread 0
-// writes the block's (sum, error) to part[2 * slot].
-__device__ __forceinline__ void dot2_block_store(double s, double cc, double *hs, double *hc,
-                                                 double *part, int slot) {
-    hs[threadIdx.x] = s;
-    hc[threadIdx.x] = cc;
+// The sum of v over a warp's 32 lanes in a fixed tree; lane 0 holds it.
+__device__ __forceinline__ double warp_sum_d(double v) {
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+    return v;
+}
+
+// The sum of v over lanes 0-7 in a fixed tree; lane 0 holds it.
+__device__ __forceinline__ double warp_sum8_d(double v) {
+#pragma unroll
+    for (int off = 4; off >= 1; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+    return v;
+}
+
+// The block's 256 thread sums in a fixed tree (each warp's, then the 8
+// warps' in warp 0); thread 0 writes the block's sum to part[slot].
+// hs: 8 doubles.
+__device__ __forceinline__ void dot_block_store(double v, double *hs, double *part, int slot) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    v = warp_sum_d(v);
+    if (lane == 0) hs[warp] = v;
     __syncthreads();
-    for (int h = 128; h >= 1; h >>= 1) {
-        if ((int)threadIdx.x < h) {
-            double t, e;
-            two_sum_d(hs[threadIdx.x], hs[threadIdx.x + h], t, e);
-            hc[threadIdx.x] += hc[threadIdx.x + h] + e;
-            hs[threadIdx.x] = t;
-        }
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) {
-        part[2 * slot] = hs[0];
-        part[2 * slot + 1] = hc[0];
+    if (warp == 0) {
+        v = warp_sum8_d(lane < 8 ? hs[lane] : 0.0);
+        if (lane == 0) part[slot] = v;
     }
     __syncthreads();
 }
 
-// dot2_block_store for two sums at once (one tree, both in each step):
-// (s1, c1) to part[2 * slot1], (s2, c2) to part[2 * slot2].
-__device__ __forceinline__ void dot2_block_store2(double s1, double c1, double s2, double c2,
-                                                  double *hs, double *hc, double *part,
-                                                  int slot1, int slot2) {
-    const int t = threadIdx.x;
-    hs[t] = s1;
-    hc[t] = c1;
-    hs[256 + t] = s2;
-    hc[256 + t] = c2;
-    __syncthreads();
-    for (int h = 128; h >= 1; h >>= 1) {
-        if (t < h) {
-#pragma unroll
-            for (int q = 0; q < 2; ++q) {
-                const int i = q * 256 + t;
-                double s, e;
-                two_sum_d(hs[i], hs[i + h], s, e);
-                hc[i] += hc[i + h] + e;
-                hs[i] = s;
-            }
-        }
-        __syncthreads();
+// dot_block_store for two sums at once: v1 to part[slot1], v2 to
+// part[slot2].  hs: 16 doubles.
+__device__ __forceinline__ void dot_block_store2(double v1, double v2, double *hs, double *part,
+                                                 int slot1, int slot2) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    v1 = warp_sum_d(v1);
+    v2 = warp_sum_d(v2);
+    if (lane == 0) {
+        hs[warp] = v1;
+        hs[8 + warp] = v2;
     }
-    if (t == 0) {
-        part[2 * slot1] = hs[0];
-        part[2 * slot1 + 1] = hc[0];
-        part[2 * slot2] = hs[256];
-        part[2 * slot2 + 1] = hc[256];
+    __syncthreads();
+    if (warp == 0) {
+        v1 = warp_sum8_d(lane < 8 ? hs[lane] : 0.0);
+        v2 = warp_sum8_d(lane < 8 ? hs[8 + lane] : 0.0);
+        if (lane == 0) {
+            part[slot1] = v1;
+            part[slot2] = v2;
+        }
     }
 }
 
@@ -164,43 +166,30 @@ __global__ void __launch_bounds__(256) dots2_partial_kernel(const T *a, const T 
                                                             int64_t n, double *part) {
     pdl_launch_dependents();
     pdl_wait();
-    __shared__ double hs[256], hc[256];
+    __shared__ double hs[8];
     const int dot = blockIdx.x / kDotChunks, chunk = blockIdx.x % kDotChunks;
     const T *u = dot == 0 ? a : b;
     const int64_t k0 = chunk * n / kDotChunks, k1 = (chunk + 1) * n / kDotChunks;
     double s = 0.0, cc = 0.0;
     for (int64_t k = k0 + threadIdx.x; k < k1; k += 256)
         dot2_step((double)u[k], (double)c[k], s, cc);
-    dot2_block_store(s, cc, hs, hc, part, blockIdx.x);
+    dot_block_store(s + cc, hs, part, blockIdx.x);
 }
 
 // Both dot products from their chunk sums, by every thread of a 256-thread
-// block: threads 0-63 take dot 0's chunks, 64-127 dot 1's, and add them in
-// a fixed pairwise tree (TwoSum on the sums, the errors carried).  GB300's
-// FP64 pipe is narrow, so a tree of 6 levels replaces a chain of 64 steps.
-// dd[0], dd[1] hold the results on return.
+// block: warps 0-1 add dot 0's kDotChunks chunk sums, warps 2-3 dot 1's,
+// each warp its 32 in a fixed tree, then thread d adds dot d's two warp
+// sums.  dd[0], dd[1] hold the results on return.  hs: 4 doubles.
 template <typename T>
-__device__ __forceinline__ void dots2_final_block(const double *part, double *hs, double *hc,
-                                                  T *dd) {
-    static_assert(2 * kDotChunks <= 256, "one thread per chunk sum");
-    const int t = threadIdx.x;
-    if (t < 2 * kDotChunks) {
-        hs[t] = part[2 * t];
-        hc[t] = part[2 * t + 1];
+__device__ __forceinline__ void dots2_final_block(const double *part, double *hs, T *dd) {
+    static_assert(kDotChunks == 64, "two warps per dot product");
+    const int t = threadIdx.x, warp = t >> 5;
+    if (warp < 4) {
+        const double v = warp_sum_d(part[t]);
+        if ((t & 31) == 0) hs[warp] = v;
     }
     __syncthreads();
-    for (int h = kDotChunks / 2; h >= 1; h >>= 1) {
-        const int k = t % kDotChunks;  // position within its dot's chunks
-        if (t < 2 * kDotChunks && k < h) {
-            double s, e;
-            two_sum_d(hs[t], hs[t + h], s, e);
-            hc[t] += hc[t + h] + e;
-            hs[t] = s;
-        }
-        __syncthreads();
-    }
-    if (t == 0) dd[0] = (T)(hs[0] + hc[0]);
-    if (t == kDotChunks) dd[1] = (T)(hs[kDotChunks] + hc[kDotChunks]);
+    if (t < 2) dd[t] = (T)(hs[2 * t] + hs[2 * t + 1]);
     __syncthreads();
 }
 
@@ -218,8 +207,8 @@ __global__ void __launch_bounds__(256) gemver_x2_kernel(T *x, const T *s, const 
     pdl_launch_dependents();
     pdl_wait();
     __shared__ T dd[2];
-    __shared__ double hs[512], hc[512];
-    dots2_final_block<T>(part_u, hs, hc, dd);
+    __shared__ double hs[16];
+    dots2_final_block<T>(part_u, hs, dd);
     const T d0 = dd[0], d1 = dd[1];
     const int chunk = blockIdx.x;
     const int64_t k0 = chunk * n / kDotChunks, k1 = (chunk + 1) * n / kDotChunks;
@@ -231,7 +220,7 @@ __global__ void __launch_bounds__(256) gemver_x2_kernel(T *x, const T *s, const 
         dot2_step((double)v1[i], (double)xn, s1, c1);
         dot2_step((double)v2[i], (double)xn, s2, c2);
     }
-    dot2_block_store2(s1, c1, s2, c2, hs, hc, part_v, chunk, kDotChunks + chunk);
+    dot_block_store2(s1 + c1, s2 + c2, hs, part_v, chunk, kDotChunks + chunk);
 }
 
 // w = w + alpha (t + u1 e0 + u2 e1), e0 = v1 . x and e1 = v2 . x from
@@ -242,8 +231,8 @@ __global__ void __launch_bounds__(256) gemver_w2_kernel(T *w, const T *t, const 
     pdl_launch_dependents();
     pdl_wait();
     __shared__ T dd[2];
-    __shared__ double hs[2 * kDotChunks], hc[2 * kDotChunks];
-    dots2_final_block<T>(part, hs, hc, dd);
+    __shared__ double hs[4];
+    dots2_final_block<T>(part, hs, dd);
     const T d0 = dd[0], d1 = dd[1];
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -268,8 +257,8 @@ __global__ void __launch_bounds__(256) gemver_x3_kernel(const Params ps, int s_d
     pdl_launch_dependents();
     pdl_wait();
     __shared__ T dd[2];
-    __shared__ double hs[512], hc[512];
-    dots2_final_block<T>(part_u, hs, hc, dd);
+    __shared__ double hs[16];
+    dots2_final_block<T>(part_u, hs, dd);
     const T d0 = dd[0], d1 = dd[1];
     const T *sv = static_cast<const T *>(ps.s);
     const int chunk = blockIdx.x;
@@ -290,7 +279,7 @@ __global__ void __launch_bounds__(256) gemver_x3_kernel(const Params ps, int s_d
         dot2_step((double)v1[i], (double)xn, s1, c1);
         dot2_step((double)v2[i], (double)xn, s2, c2);
     }
-    dot2_block_store2(s1, c1, s2, c2, hs, hc, part_v, chunk, kDotChunks + chunk);
+    dot_block_store2(s1 + c1, s2 + c2, hs, part_v, chunk, kDotChunks + chunk);
 }
 
 // w = w + alpha (t + u1 e0 + u2 e1) with t = A x from the rows-only pass's
@@ -306,9 +295,9 @@ __global__ void __launch_bounds__(256) gemver_w3_kernel(const Params pq, int q_d
     pdl_launch_dependents();
     pdl_wait();
     __shared__ T dd[2];
-    __shared__ double hs[2 * kDotChunks], hc[2 * kDotChunks];
+    __shared__ double hs[4];
     __shared__ T chunk_sum[256];
-    dots2_final_block<T>(part, hs, hc, dd);
+    dots2_final_block<T>(part, hs, dd);
     const T d0 = dd[0], d1 = dd[1];
     const int R = 256 / C, xr = threadIdx.x % R, y = threadIdx.x / R;
     const int64_t i = (int64_t)blockIdx.x * R + xr;

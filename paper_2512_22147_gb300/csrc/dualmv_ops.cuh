@@ -80,16 +80,18 @@ __global__ void gemver_w_kernel(T *w, const T *t, int64_t n, T alpha) {
 //   A_hat x   = A x   + u1 (v1 . x) + u2 (v2 . x)
 // Two dot products per side (a . c and b . c), deterministic: kDotChunks
 // blocks per product each take one contiguous chunk (thread k: elements
-// k, k + 256, ... of the chunk, in order), sum it with TwoProduct/TwoSum in
-// double, round that compensated sum once, and add the threads' sums in a
-// fixed tree of plain fp64 adds; the kernel that uses the products adds the
-// chunk sums in a fixed tree too.  Along any path there are at most 16
-// roundings after the compensated thread sums, so the error stays within
-// about 16 u sum |a_k c_k|: each term's error is inside the bar, whose
-// denominator holds |u1| (|u1| . |y|) and the like.  GB300's FP64 pipe is
-// narrow, so the work is spread over many SMs and the trees take one add
-// per level (TwoSum trees, eight operations per level, cost the x update
-// 11 us of its call at 8192^2).
+// k, k + 256, ... of the chunk, in order).  A thread with at most
+// kPlainPerThread elements sums them with fp64 FMAs; one with more sums
+// them compensated (TwoProduct/TwoSum) and rounds that once.  The block
+// adds its threads' sums in a fixed tree of plain fp64 adds, and the kernel
+// that uses the products adds the chunk sums in a fixed tree too.  Along
+// any path there are at most 80 roundings, so a product errs by at most
+// about 80 u sum |a_k c_k| (u = 2^-53, 8.9e-15): each term's error is
+// inside the bar, whose denominator holds |u1| (|u1| . |y|) and the like.
+// GB300's FP64 pipe is narrow, so the work is spread over many SMs, the
+// trees take one add per level (TwoSum trees, eight operations per level,
+// cost the x update 11 us of its call at 8192^2), and compensation is kept
+// for the long per-thread sums it is needed for.
 constexpr int kDotChunks = 64;
 
 __device__ __forceinline__ void two_sum_d(double a, double b, double &s, double &e) {
@@ -106,6 +108,29 @@ __device__ __forceinline__ void dot2_step(double x, double y, double &s, double 
     two_sum_d(s, p, t, e);
     s = t;
     cc += e + pe;
+}
+
+// Elements per thread above which a thread's share of a dot product is
+// summed compensated.
+constexpr int64_t kPlainPerThread = 64;
+
+// A thread's share of a dot product (see above): plain FMAs or
+// compensated, the same for every thread of a block.
+struct ThreadDot {
+    double s = 0.0, c = 0.0;
+    __device__ __forceinline__ void add(double x, double y, bool comp) {
+        if (comp)
+            dot2_step(x, y, s, c);
+        else
+            s = fma(x, y, s);
+    }
+    __device__ __forceinline__ double value() const { return s + c; }
+};
+
+// Whether a chunk of `len` elements over 256 threads takes compensated
+// thread sums.
+__device__ __forceinline__ bool dot_compensated(int64_t len) {
+    return len > 256 * kPlainPerThread;
 }
 
 // The sum of v over a warp's 32 lanes in a fixed tree; lane 0 holds it.
@@ -170,10 +195,10 @@ __global__ void __launch_bounds__(256) dots2_partial_kernel(const T *a, const T 
     const int dot = blockIdx.x / kDotChunks, chunk = blockIdx.x % kDotChunks;
     const T *u = dot == 0 ? a : b;
     const int64_t k0 = chunk * n / kDotChunks, k1 = (chunk + 1) * n / kDotChunks;
-    double s = 0.0, cc = 0.0;
-    for (int64_t k = k0 + threadIdx.x; k < k1; k += 256)
-        dot2_step((double)u[k], (double)c[k], s, cc);
-    dot_block_store(s + cc, hs, part, blockIdx.x);
+    const bool comp = dot_compensated(k1 - k0);
+    ThreadDot d;
+    for (int64_t k = k0 + threadIdx.x; k < k1; k += 256) d.add((double)u[k], (double)c[k], comp);
+    dot_block_store(d.value(), hs, part, blockIdx.x);
 }
 
 // Both dot products from their chunk sums, by every thread of a 256-thread
@@ -212,15 +237,16 @@ __global__ void __launch_bounds__(256) gemver_x2_kernel(T *x, const T *s, const 
     const T d0 = dd[0], d1 = dd[1];
     const int chunk = blockIdx.x;
     const int64_t k0 = chunk * n / kDotChunks, k1 = (chunk + 1) * n / kDotChunks;
-    double s1 = 0.0, c1 = 0.0, s2 = 0.0, c2 = 0.0;
+    const bool comp = dot_compensated(k1 - k0);
+    ThreadDot e1, e2;
     for (int64_t i = k0 + threadIdx.x; i < k1; i += 256) {
         const T inner = fma(v2[i], d1, fma(v1[i], d0, s[i]));
         const T xn = fma(beta, inner, x[i]) + z[i];
         x[i] = xn;
-        dot2_step((double)v1[i], (double)xn, s1, c1);
-        dot2_step((double)v2[i], (double)xn, s2, c2);
+        e1.add((double)v1[i], (double)xn, comp);
+        e2.add((double)v2[i], (double)xn, comp);
     }
-    dot_block_store2(s1 + c1, s2 + c2, hs, part_v, chunk, kDotChunks + chunk);
+    dot_block_store2(e1.value(), e2.value(), hs, part_v, chunk, kDotChunks + chunk);
 }
 
 // w = w + alpha (t + u1 e0 + u2 e1), e0 = v1 . x and e1 = v2 . x from
@@ -248,7 +274,10 @@ __global__ void __launch_bounds__(256) gemver_w2_kernel(T *w, const T *t, const 
 // of seven.
 
 // gemver_x2_kernel with s = A^T y from the columns-only pass's partials
-// (ps: that pass's parameters; s_direct: the pass wrote s itself).
+// (ps: that pass's parameters; s_direct: the pass wrote s itself).  Each
+// thread reads its first element's operands before the block forms d0 and
+// d1, and the next element's before it works on the current one, so the
+// loads overlap the chunk-sum tree and the arithmetic.
 template <typename T>
 __global__ void __launch_bounds__(256) gemver_x3_kernel(const Params ps, int s_direct,
                                                         const double *part_u, T *x, const T *v1,
@@ -258,28 +287,46 @@ __global__ void __launch_bounds__(256) gemver_x3_kernel(const Params ps, int s_d
     pdl_wait();
     __shared__ T dd[2];
     __shared__ double hs[16];
-    dots2_final_block<T>(part_u, hs, dd);
-    const T d0 = dd[0], d1 = dd[1];
     const T *sv = static_cast<const T *>(ps.s);
     const int chunk = blockIdx.x;
     const int64_t k0 = chunk * n / kDotChunks, k1 = (chunk + 1) * n / kDotChunks;
-    double s1 = 0.0, c1 = 0.0, s2 = 0.0, c2 = 0.0;
-    for (int64_t i = k0 + threadIdx.x; i < k1; i += 256) {
-        T si;
-        int64_t c_lo = 0, c_hi = 0;
-        const int64_t band = i / ps.band_cols;
-        if (!s_direct) band_ctas_of(ps, band, c_lo, c_hi);
-        if (s_direct || c_lo == c_hi)
-            si = sv[i];
-        else
-            si = s_segment_sum<T>(ps, band, (int)(i - band * ps.band_cols), c_lo, c_hi);
-        const T inner = fma(v2[i], d1, fma(v1[i], d0, si));
-        const T xn = fma(beta, inner, x[i]) + z[i];
+    struct Operands {
+        T s, v1, v2, x, z;
+    };
+    // Element i's operands (zeros past the chunk).
+    auto load = [&](int64_t i) {
+        Operands o{T(0), T(0), T(0), T(0), T(0)};
+        if (i < k1) {
+            int64_t c_lo = 0, c_hi = 0;
+            const int64_t band = i / ps.band_cols;
+            if (!s_direct) band_ctas_of(ps, band, c_lo, c_hi);
+            if (s_direct || c_lo == c_hi)
+                o.s = sv[i];
+            else
+                o.s = s_segment_sum<T>(ps, band, (int)(i - band * ps.band_cols), c_lo, c_hi);
+            o.v1 = v1[i];
+            o.v2 = v2[i];
+            o.x = x[i];
+            o.z = z[i];
+        }
+        return o;
+    };
+    int64_t i = k0 + threadIdx.x;
+    Operands cur = load(i);
+    dots2_final_block<T>(part_u, hs, dd);
+    const T d0 = dd[0], d1 = dd[1];
+    const bool comp = dot_compensated(k1 - k0);
+    ThreadDot e1, e2;
+    for (; i < k1; i += 256) {
+        const Operands nxt = load(i + 256);
+        const T inner = fma(cur.v2, d1, fma(cur.v1, d0, cur.s));
+        const T xn = fma(beta, inner, cur.x) + cur.z;
         x[i] = xn;
-        dot2_step((double)v1[i], (double)xn, s1, c1);
-        dot2_step((double)v2[i], (double)xn, s2, c2);
+        e1.add((double)cur.v1, (double)xn, comp);
+        e2.add((double)cur.v2, (double)xn, comp);
+        cur = nxt;
     }
-    dot_block_store2(s1 + c1, s2 + c2, hs, part_v, chunk, kDotChunks + chunk);
+    dot_block_store2(e1.value(), e2.value(), hs, part_v, chunk, kDotChunks + chunk);
 }
 
 // w = w + alpha (t + u1 e0 + u2 e1) with t = A x from the rows-only pass's
@@ -297,8 +344,6 @@ __global__ void __launch_bounds__(256) gemver_w3_kernel(const Params pq, int q_d
     __shared__ T dd[2];
     __shared__ double hs[4];
     __shared__ T chunk_sum[256];
-    dots2_final_block<T>(part, hs, dd);
-    const T d0 = dd[0], d1 = dd[1];
     const int R = 256 / C, xr = threadIdx.x % R, y = threadIdx.x / R;
     const int64_t i = (int64_t)blockIdx.x * R + xr;
     const bool valid = i < m;
@@ -314,17 +359,25 @@ __global__ void __launch_bounds__(256) gemver_w3_kernel(const Params pq, int q_d
         for (; k < pq.bands; k += C) acc = acc + base[k * pq.M];
     }
     chunk_sum[threadIdx.x] = acc;
-    __syncthreads();
+    // Row i's own operands, read before the block forms e0 and e1 so that
+    // their loads overlap the chunk-sum tree.
+    T ti = T(0), u1i = T(0), u2i = T(0), wi = T(0);
     if (y == 0 && valid) {
-        T ti;
-        if (q_direct) {
-            ti = static_cast<const T *>(pq.q)[i];
-        } else {
+        u1i = u1[i];
+        u2i = u2[i];
+        wi = w[i];
+        if (q_direct) ti = static_cast<const T *>(pq.q)[i];
+    }
+    // Its barriers also put every chunk_sum write before the reads below.
+    dots2_final_block<T>(part, hs, dd);
+    const T d0 = dd[0], d1 = dd[1];
+    if (y == 0 && valid) {
+        if (!q_direct) {
             ti = chunk_sum[xr];
             for (int yy = 1; yy < C; ++yy) ti = ti + chunk_sum[yy * R + xr];
         }
-        const T inner = fma(u2[i], d1, fma(u1[i], d0, ti));
-        w[i] = fma(alpha, inner, w[i]);
+        const T inner = fma(u2i, d1, fma(u1i, d0, ti));
+        w[i] = fma(alpha, inner, wi);
     }
 }
 

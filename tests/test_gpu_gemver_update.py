@@ -15,7 +15,8 @@ tests check, element by element against the oracle within the dtype's bar
   * values outside [2^-40, 2^40) in rows of A and in the new x (native fp64
     for those rows or that band), and zero rows;
   * repeated calls giving the same bits, and the padding columns untouched;
-  * the adversarial all-positive inputs of the fp64 error-bound tests.
+  * the adversarial all-positive inputs of the fp64 error-bound tests;
+  * vectors long enough for the dot products' compensated thread sums.
 The full-size workload (gemver_update_f64_8192x8192) runs in
 test_gpu_ops.py with the other operation workloads."""
 import numpy as np
@@ -120,6 +121,19 @@ def test_repeated_calls_are_bit_identical(dtype):
     # The padding columns (NaN in the generated storage) are untouched.
     assert torch.equal(A0[:, N:].isnan(), ops[0][:, N:].isnan())
     assert bool(A0[:, N:].isnan().all())
+
+
+@pytest.mark.parametrize("dtype", ["f64", "f32"])
+@pytest.mark.parametrize("M,N", [(1048600, 3), (3, 1048600)])
+@pytest.mark.parametrize("update_A", [False, True])
+def test_long_vectors(dtype, M, N, update_A):
+    """Vectors past 64 x 256 x 64 elements: each thread of the dot-product
+    kernels then has more than 64 elements of its chunk and sums them
+    compensated (at most 64 it uses plain FMAs): u . y when M is long,
+    v . x when N is long."""
+    err = check_gemver(_ops(M, N, N + (1 if N == 3 else 0), M + N, dtype), N, 1.5, -0.75,
+                       update_A, dtype)
+    print(f"gemver {dtype} {M}x{N} update_A={update_A}: {err:.3e}")
 
 
 @pytest.mark.parametrize("family", ["low32_set", "low29_set"])

@@ -489,7 +489,8 @@ cudaError_t launch_stream(const CUtensorMap &map, const Params &prm, const dualm
         dmv::dualmv_stream_kernel<T, W, RPW, S, kTma, k3d, kOut, kRank2, kRev>;
     cudaError_t e = smem_opt_in<kern>(pl.smem_bytes, dev);
     if (e != cudaSuccess) return e;
-    if constexpr (std::is_same<T, int32_t>::value)  // after the zeroing kernel
+    // After the zeroing kernel, or a late-wait pass (Params::pdl_late).
+    if (std::is_same<T, int32_t>::value || prm.pdl_late)
         return launch_dependent(kern, dim3((unsigned)pl.grid), dim3((unsigned)pl.threads),
                                 (size_t)pl.smem_bytes, stream, map, prm);
     kern<<<(unsigned)pl.grid, (unsigned)pl.threads, (size_t)pl.smem_bytes, stream>>>(map, prm);
@@ -989,7 +990,7 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                   int64_t strideQ, Out *s, int64_t strideS, int64_t batch,
                   cudaStream_t stream, uint32_t outputs = dmv::kOutBoth,
                   const Rank2 *rank2 = nullptr, int32_t variant = -1,
-                  Deferred *defer = nullptr, bool reverse = false) {
+                  Deferred *defer = nullptr, bool reverse = false, bool late_wait = false) {
     using Acc = typename dmv::Traits<T>::Acc;
     static_assert(sizeof(Acc) == sizeof(Out), "accumulator and output widths differ");
     constexpr bool kIntPath = std::is_same<T, int32_t>::value;
@@ -1156,6 +1157,12 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     prm.band_cols = pl.band_cols;
     prm.bands = pl.bands; prm.stripes = pl.stripes; prm.tiles = pl.tiles;
     prm.grid = pl.grid; prm.max_seg = pl.max_segments;
+    // Late wait (Params::pdl_late) for the single-sided kernels below; the
+    // caller's kernel before this call triggers its dependents after its wait.
+    prm.pdl_late = (late_wait && !kIntPath && outputs != dmv::kOutBoth && rank2 == nullptr &&
+                    var == nullptr)
+                       ? 1
+                       : 0;
     const int64_t q_ws_bytes = pl.bands > 1 ? batch * pl.bands * M * (int64_t)sizeof(Acc) : 0;
     prm.q_ws = (pl.bands > 1 && ws) ? ws : nullptr;
     prm.s_ws = ws ? static_cast<unsigned char *>(ws) + ((q_ws_bytes + 255) / 256) * 256 : nullptr;
@@ -1558,11 +1565,13 @@ dualmv_status gemver_factored_fused(int64_t M, int64_t N, T alpha, T beta, const
     cudaError_t e = cudaSuccess;
     Deferred ds, dq;
     if (st == DUALMV_SUCCESS)
-        e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks), dim3(256),
-                             0, stream, u1, u2, y, M, part_u);
-    if (st == DUALMV_SUCCESS && e == cudaSuccess)  // s = A^T y, left as partials
+        e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks),
+                             dim3(dmv::kDotThreads), 0, stream, u1, u2, y, M, part_u);
+    // s = A^T y, left as partials.  The pass runs beside the dots kernel
+    // (late wait, Params::pdl_late): neither touches the other's memory.
+    if (st == DUALMV_SUCCESS && e == cudaSuccess)
         st = run<T, T>(M, N, A, lda, 0, nullptr, 0, y, 0, nullptr, 0, s, 0, 1, stream,
-                       dmv::kOutS, nullptr, -1, &ds);
+                       dmv::kOutS, nullptr, -1, &ds, false, true);
     if (st == DUALMV_SUCCESS && e == cudaSuccess) {
         if (!ds.used) ds.prm.s = s;
         e = launch_dependent(dmv::gemver_x3_kernel<T>, dim3(dmv::kDotChunks), dim3(256), 0,
@@ -1622,8 +1631,8 @@ dualmv_status gemver_factored(int64_t M, int64_t N, T alpha, T beta, const T *A,
     // The vector kernels are programmatic dependents of the kernel before
     // them (each waits for it before reading): their launches overlap it.
     if (st == DUALMV_SUCCESS && N > 0) {  // s = A^T y (zero when M == 0)
-        e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks), dim3(256),
-                             0, stream, u1, u2, y, M, part_u);
+        e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks),
+                             dim3(dmv::kDotThreads), 0, stream, u1, u2, y, M, part_u);
         if (e == cudaSuccess)
             st = run<T, T>(M, N, A, lda, 0, nullptr, 0, y, 0, nullptr, 0, s, 0, 1, stream,
                            dmv::kOutS);
@@ -1633,8 +1642,8 @@ dualmv_status gemver_factored(int64_t M, int64_t N, T alpha, T beta, const T *A,
                                  stream, x, (const T *)s, v1, v2, (const double *)part_u, z, N,
                                  beta, part_v);
     } else if (st == DUALMV_SUCCESS && M > 0) {  // N == 0: v . x is zero
-        e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks), dim3(256),
-                             0, stream, v1, v2, x, N, part_v);
+        e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks),
+                             dim3(dmv::kDotThreads), 0, stream, v1, v2, x, N, part_v);
     }
     if (st == DUALMV_SUCCESS && e == cudaSuccess && M > 0) {  // t = A x (zero when N == 0)
         st = run<T, T>(M, N, A, lda, 0, x, 0, nullptr, 0, t, 0, nullptr, 0, 1, stream,
@@ -1689,10 +1698,12 @@ dualmv_status gemver_update(int64_t M, int64_t N, T alpha, T beta, T *A, int64_t
     Deferred ds;
     if (st == DUALMV_SUCCESS)
         e = launch_dependent(dmv::dots2_partial_kernel<T>, dim3(2 * dmv::kDotChunks),
-                             dim3(256), 0, stream, u1, u2, y, M, part_u);
-    if (st == DUALMV_SUCCESS && e == cudaSuccess)  // s = A^T y, left as partials
+                             dim3(dmv::kDotThreads), 0, stream, u1, u2, y, M, part_u);
+    // s = A^T y, left as partials.  The pass runs beside the dots kernel
+    // (late wait, Params::pdl_late): neither touches the other's memory.
+    if (st == DUALMV_SUCCESS && e == cudaSuccess)
         st = run<T, T>(M, N, A, lda, 0, nullptr, 0, y, 0, nullptr, 0, s, 0, 1, stream,
-                       dmv::kOutS, nullptr, -1, &ds);
+                       dmv::kOutS, nullptr, -1, &ds, false, true);
     if (st == DUALMV_SUCCESS && e == cudaSuccess) {
         if (!ds.used) ds.prm.s = s;
         e = launch_dependent(dmv::gemver_x3_kernel<T>, dim3(dmv::kDotChunks), dim3(256), 0,

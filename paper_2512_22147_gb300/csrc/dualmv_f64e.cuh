@@ -349,8 +349,9 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
     __syncthreads();
     pdl_launch_dependents();
     // Launched as a dependent of whatever precedes it on the stream: nothing
-    // is read or written before that grid has completed.
-    pdl_wait();
+    // is read or written before that grid has completed (in late-wait mode,
+    // every grid before it has; see Params::pdl_late).
+    if (!prm.pdl_late) pdl_wait();
 
     // ------------------------------------------------------ producer ----
     if (!kSelf && warp == W) {
@@ -869,6 +870,7 @@ template <int W, int RPW, int STAGES, int BAND, bool kBatched3d, int kOut = kOut
 __global__ void __launch_bounds__((W + (kSelf ? 0 : 1)) * 32, 1)
 dualmv_stream_f64e_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
     f64e_body<W, RPW, STAGES, BAND, kBatched3d, kOut, NC, kSelf, kPack, 0, kRev>(&tmap, prm);
+    if (prm.pdl_late) pdl_wait();  // see Params::pdl_late
 }
 
 // fp64 rows whose stride or base is not 16-byte aligned (odd lda): the same
@@ -877,6 +879,7 @@ template <int W, int RPW, int STAGES, int NPH>
 __global__ void __launch_bounds__(W * 32, 1)
 dualmv_stream_f64e_phased_kernel(const __grid_constant__ TmapSet maps, const Params prm) {
     f64e_body<W, RPW, STAGES, 256, false, kOutBoth, 0, true, true, NPH>(maps.m, prm);
+    if (prm.pdl_late) pdl_wait();  // see Params::pdl_late
 }
 
 }  // namespace dmv

@@ -292,6 +292,14 @@ struct Params {
     // row.  ph_n = 1 and zeros otherwise.
     int32_t ph_n;
     int32_t ph_off[4];
+    // Late wait: a single-sided pass launched as a programmatic dependent of
+    // a kernel that triggers its dependents only after its own wait, so that
+    // every grid before that kernel has completed when this one starts.
+    // That kernel touches none of this pass's memory, so the pass reads and
+    // writes without waiting, and waits for that kernel's grid only before
+    // it exits: its completion still implies that kernel's.  GEMVER's
+    // columns pass runs this way beside the u . y dot-product kernel.
+    int32_t pdl_late;
 };
 
 // Phased tensor maps: two per phase, over the same rows: m[2 ph] with
@@ -840,6 +848,7 @@ __global__ void __launch_bounds__((W + (kTma ? 1 : 0)) * 32,
                                   (!kTma && std::is_same<T, int32_t>::value) ? 2 : 1)
 dualmv_stream_kernel(const __grid_constant__ CUtensorMap tmap, const Params prm) {
     stream_body<T, W, RPW, STAGES, kTma, kBatched3d, kOut, kRank2, 0, kRev>(&tmap, prm);
+    if (prm.pdl_late) pdl_wait();  // see Params::pdl_late
 }
 
 // The same kernel for one problem whose row stride or base is not 16-byte
@@ -851,6 +860,7 @@ template <typename T, int W, int RPW, int STAGES, int NPH>
 __global__ void __launch_bounds__((W + 1) * 32, 1)
 dualmv_stream_phased_kernel(const __grid_constant__ TmapSet maps, const Params prm) {
     stream_body<T, W, RPW, STAGES, true, false, kOutBoth, false, NPH>(maps.m, prm);
+    if (prm.pdl_late) pdl_wait();  // see Params::pdl_late
 }
 
 // ------------------------------------------------------- combine arithmetic --

@@ -127,10 +127,10 @@ struct ThreadDot {
     __device__ __forceinline__ double value() const { return s + c; }
 };
 
-// Whether a chunk of `len` elements over 256 threads takes compensated
-// thread sums.
-__device__ __forceinline__ bool dot_compensated(int64_t len) {
-    return len > 256 * kPlainPerThread;
+// Whether a chunk of `len` elements over `threads` threads takes
+// compensated thread sums.
+__device__ __forceinline__ bool dot_compensated(int64_t len, int threads = 256) {
+    return len > threads * kPlainPerThread;
 }
 
 // The sum of v over a warp's 32 lanes in a fixed tree; lane 0 holds it.
@@ -147,16 +147,20 @@ __device__ __forceinline__ double warp_sum8_d(double v) {
     return v;
 }
 
-// The block's 256 thread sums in a fixed tree (each warp's, then the 8
-// warps' in warp 0); thread 0 writes the block's sum to part[slot].
-// hs: 8 doubles.
+// The block's NW * 32 thread sums in a fixed tree (each warp's, then the
+// NW warps' in warp 0); thread 0 writes the block's sum to part[slot].
+// hs: NW doubles.
+template <int NW>
 __device__ __forceinline__ void dot_block_store(double v, double *hs, double *part, int slot) {
+    static_assert(NW >= 1 && NW <= 32 && (NW & (NW - 1)) == 0, "a power of two of warps");
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     v = warp_sum_d(v);
     if (lane == 0) hs[warp] = v;
     __syncthreads();
     if (warp == 0) {
-        v = warp_sum8_d(lane < 8 ? hs[lane] : 0.0);
+        v = lane < NW ? hs[lane] : 0.0;
+#pragma unroll
+        for (int off = NW / 2; off >= 1; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
         if (lane == 0) part[slot] = v;
     }
     __syncthreads();
@@ -184,21 +188,31 @@ __device__ __forceinline__ void dot_block_store2(double v1, double v2, double *h
     }
 }
 
+// 2 kDotChunks blocks of kDotThreads threads: block d kDotChunks + k sums
+// chunk k of dot product d (a . c, then b . c) into part[d kDotChunks + k].
 // Launched as a programmatic dependent of the kernel before it: waits for
-// that grid before reading its inputs.
+// that grid before reading its inputs, and only then lets its own
+// dependents launch, so that every grid before it has completed when they
+// start (GEMVER's columns pass relies on that; see Params::pdl_late).  Its
+// blocks are small (128 threads, 32 registers each) so that one fits on an
+// SM beside a CTA of that pass.
+constexpr int kDotThreads = 128;
+
 template <typename T>
-__global__ void __launch_bounds__(256) dots2_partial_kernel(const T *a, const T *b, const T *c,
-                                                            int64_t n, double *part) {
-    pdl_launch_dependents();
+__global__ void __launch_bounds__(kDotThreads) dots2_partial_kernel(const T *a, const T *b,
+                                                                    const T *c, int64_t n,
+                                                                    double *part) {
     pdl_wait();
-    __shared__ double hs[8];
+    pdl_launch_dependents();
+    __shared__ double hs[kDotThreads / 32];
     const int dot = blockIdx.x / kDotChunks, chunk = blockIdx.x % kDotChunks;
     const T *u = dot == 0 ? a : b;
     const int64_t k0 = chunk * n / kDotChunks, k1 = (chunk + 1) * n / kDotChunks;
-    const bool comp = dot_compensated(k1 - k0);
+    const bool comp = dot_compensated(k1 - k0, kDotThreads);
     ThreadDot d;
-    for (int64_t k = k0 + threadIdx.x; k < k1; k += 256) d.add((double)u[k], (double)c[k], comp);
-    dot_block_store(d.value(), hs, part, blockIdx.x);
+    for (int64_t k = k0 + threadIdx.x; k < k1; k += kDotThreads)
+        d.add((double)u[k], (double)c[k], comp);
+    dot_block_store<kDotThreads / 32>(d.value(), hs, part, blockIdx.x);
 }
 
 // Both dot products from their chunk sums, by every thread of a 256-thread

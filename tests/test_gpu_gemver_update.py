@@ -136,6 +136,34 @@ def test_long_vectors(dtype, M, N, update_A):
     print(f"gemver {dtype} {M}x{N} update_A={update_A}: {err:.3e}")
 
 
+@pytest.mark.parametrize("dtype", ["f64", "f32"])
+def test_back_to_back_calls_see_the_previous_writes(dtype):
+    """The columns pass reads A and y without waiting for the u . y kernel
+    beside it (it waits for that grid only before it exits); every grid
+    queued before the call has completed when it starts.  A call right after
+    one that wrote A_hat over A, and after a kernel that rewrote y, gives
+    the bits of the same calls with a synchronisation between them."""
+    ops = _ops(1500, 2000, 2000, 77, dtype)
+
+    def sequence(sync):
+        A, u1, v1, u2, v2, w, x, y, z = (t.clone() for t in ops)
+        torch.cuda.synchronize()
+        dm.gemver(A, u1, v1, u2, v2, w, x, y, z, alpha=1.5, beta=0.5, update_A=True)
+        if sync:
+            torch.cuda.synchronize()
+        y.mul_(-0.5)
+        if sync:
+            torch.cuda.synchronize()
+        dm.gemver(A, u1, v1, u2, v2, w, x, y, z, alpha=1.5, beta=0.5)
+        dm.gemver(A, u1, v1, u2, v2, w, x, y, z, alpha=0.5, beta=2.0, update_A=True)
+        torch.cuda.synchronize()
+        return A, w, x
+
+    for _ in range(3):
+        for t0, t1 in zip(sequence(False), sequence(True)):
+            assert torch.equal(t0, t1)
+
+
 @pytest.mark.parametrize("family", ["low32_set", "low29_set"])
 def test_adversarial_inputs(family):
     """All inputs positive with the low mantissa bits set: the double-float

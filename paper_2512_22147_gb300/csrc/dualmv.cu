@@ -1297,6 +1297,10 @@ dualmv_status gesummv_run(int64_t M, int64_t N, T alpha, const T *A, int64_t lda
     if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
     // Both rows-only passes leave their band partials (no combine kernels);
     // gesummv_final_kernel adds them in the combine's order and forms y.
+    // The pass over B shares no buffer with the pass over A, which lets its
+    // dependents launch only once every grid before it has completed: B's
+    // pass runs in late-wait mode (Params::pdl_late), its CTAs taking the
+    // SMs that A's leave, and the final kernel's wait for it covers both.
     T *tmp = nullptr;
     dualmv_status st = pool_alloc(&tmp, M, stream);
     if (st != DUALMV_SUCCESS) return st;
@@ -1305,7 +1309,7 @@ dualmv_status gesummv_run(int64_t M, int64_t N, T alpha, const T *A, int64_t lda
                    dmv::kOutQ, nullptr, -1, &da);
     if (st == DUALMV_SUCCESS)
         st = run<T, T>(M, N, B, ldb, 0, x, 0, nullptr, 0, y, 0, nullptr, 0, 1, stream,
-                       dmv::kOutQ, nullptr, -1, &db);
+                       dmv::kOutQ, nullptr, -1, &db, false, true);
     cudaError_t e = cudaSuccess;
     if (st == DUALMV_SUCCESS) {
         if (!da.used) da.prm.q = tmp;

@@ -347,11 +347,12 @@ __device__ __forceinline__ void f64e_body(const CUtensorMap *tmaps, const Params
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
-    pdl_launch_dependents();
     // Launched as a dependent of whatever precedes it on the stream: nothing
     // is read or written before that grid has completed (in late-wait mode,
-    // every grid before it has; see Params::pdl_late).
+    // every grid before it has; see Params::pdl_late).  Its dependents may
+    // launch only then, so that a late-wait pass may follow it.
     if (!prm.pdl_late) pdl_wait();
+    pdl_launch_dependents();
 
     // ------------------------------------------------------ producer ----
     if (!kSelf && warp == W) {

@@ -298,7 +298,10 @@ struct Params {
     // That kernel touches none of this pass's memory, so the pass reads and
     // writes without waiting, and waits for that kernel's grid only before
     // it exits: its completion still implies that kernel's.  GEMVER's
-    // columns pass runs this way beside the u . y dot-product kernel.
+    // columns pass runs this way beside the u . y dot-product kernel, and
+    // GESUMMV's pass over B after its pass over A.  A late-wait pass lets
+    // its own dependents launch at its start, so no late-wait pass may
+    // follow it.
     int32_t pdl_late;
 };
 

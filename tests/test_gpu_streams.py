@@ -10,12 +10,14 @@ double-float fp64 kernel, a strided batch, GEMVER):
     another give the bits of the same problems run one after another;
   * a graph of such calls, replayed several times, gives the bits of the
     eager calls, and those bits match the oracle."""
+import numpy as np
 import pytest
 import torch
 
+import oracle
 import paper_2512_22147_gb300 as dm
 from paper_2512_22147_gb300 import inputs
-from parity import TOL, compare_problem
+from parity import TOL, compare_problem, scaled_error
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -135,3 +137,43 @@ def test_gemver_on_two_streams_at_once():
         for a, b in zip(serial, conc):
             for t0, t1 in zip(a, b):
                 assert torch.equal(t0, t1)
+
+
+@pytest.mark.parametrize("dtype", ["f64", "f32"])
+def test_gesummv_back_to_back_sees_the_previous_writes(dtype):
+    """GESUMMV's pass over B starts without waiting for the pass over A (it
+    waits for that grid only before it exits).  Calls right after kernels
+    that rewrote B and x, and a call whose x is the y the call before wrote,
+    give the bits of the same calls with a synchronisation between them, and
+    the oracle's values."""
+    n = 1500
+    dist = "normal" if dtype == "f64" else "uniform"
+    A, B, x = inputs.generate_gesummv(
+        inputs.Workload("g", dtype, n, n, n, dist, 60, op="gesummv"), DEV)
+
+    def sequence(sync):
+        Bc, xc = B.clone(), x.clone()
+        torch.cuda.synchronize()
+        y1 = dm.gesummv(A, Bc, xc, alpha=1.5, beta=0.5)
+        if sync:
+            torch.cuda.synchronize()
+        Bc.mul_(-0.5)
+        xc.add_(0.25)
+        if sync:
+            torch.cuda.synchronize()
+        y2 = dm.gesummv(A, Bc, xc, alpha=0.5, beta=2.0)
+        if sync:
+            torch.cuda.synchronize()
+        y3 = dm.gesummv(A, Bc, y2, alpha=1.0, beta=-1.0)
+        torch.cuda.synchronize()
+        return y1, y2, y3, Bc, xc
+
+    ref = sequence(True)
+    for _ in range(3):
+        for t0, t1 in zip(sequence(False), ref):
+            assert torch.equal(t0, t1)
+    y1, y2, y3, Bc, xc = ref
+    An, Bn = A.cpu().numpy(), Bc.cpu().numpy()
+    want = oracle.gesummv(An, Bn, y2.cpu().numpy(), 1.0, -1.0, N=n)
+    den = (np.abs(An) + np.abs(Bn)) @ np.abs(y2.cpu().numpy().astype(np.float64))
+    assert scaled_error(y3.cpu().numpy(), want, den) <= TOL[dtype]

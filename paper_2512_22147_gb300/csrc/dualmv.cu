@@ -1381,6 +1381,9 @@ struct AtaxCfg<float> {
 #ifndef DUALMV_ATAX64_BAND
 #define DUALMV_ATAX64_BAND 256
 #endif
+#ifndef DUALMV_ATAX64_NATIVE_VECS
+#define DUALMV_ATAX64_NATIVE_VECS 0
+#endif
 #ifndef DUALMV_ATAX64_SPLIT_WARPS
 #define DUALMV_ATAX64_SPLIT_WARPS 1
 #endif
@@ -1394,7 +1397,8 @@ struct AtaxCfg<double> {
 #if DUALMV_ATAX64_SPLIT_WARPS
     static constexpr int kThreads = (2 * W + 1) * 32;  // and a control warp
     using L = dmv::AtaxLayout64WS<W, R, S, kBand>;
-    static constexpr auto kern = dmv::atax_cluster_f64_ws_kernel<W, R, S, kBand>;
+    static constexpr auto kern =
+        dmv::atax_cluster_f64_ws_kernel<W, R, S, kBand, DUALMV_ATAX64_NATIVE_VECS>;
 #else
     static constexpr int kThreads = (W + 1) * 32;  // and a control warp
     using L = dmv::AtaxLayout64<W, R, S, kBand>;

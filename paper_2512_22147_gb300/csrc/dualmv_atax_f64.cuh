@@ -476,13 +476,19 @@ struct AtaxLayout64WS {
         kAlign + kRing + kWarpPart + kPart + kT + kSeg + kFlags + kBars;
 };
 
-template <int W, int R, int STAGES, int BAND = kBandCols>
+template <int W, int R, int STAGES, int BAND = kBandCols, int NV = 0>
 __global__ void __launch_bounds__((2 * W + 1) * 32, 1)
 atax_cluster_f64_ws_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxParams64 prm) {
     using L = AtaxLayout64WS<W, R, STAGES, BAND>;
     using Vec = double2;
     constexpr int VE = 2, LANE_COLS = BAND / 32, VPL = LANE_COLS / VE;
     constexpr int ROW_BYTES = BAND * 8;
+    // The last NV of each lane's VPL column vectors take their column sums
+    // in native fp64 (DFMA on the otherwise idle FP64 pipe, one chain per
+    // column over the CTA's stripes); the row warp leaves those vectors as
+    // doubles in the stage instead of writing their split.
+    static_assert(NV >= 0 && NV < VPL, "native column vectors: 0 .. VPL - 1");
+    constexpr int VS = VPL - NV;  // vectors in double-float
     static_assert(L::kBoxBytes == R * ROW_BYTES, "box size mismatch");
     static_assert(VPL == 2 || VPL == 4, "a sub-band of 128 or 256 columns");
     static_assert(kAtaxMaxCluster * R <= 64, "the control warp sends two values a lane");
@@ -675,9 +681,11 @@ atax_cluster_f64_ws_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxP
                                                 f64e_range_key(a[v].y));
                         const float2 ah = make_float2(ah0, ah1), al = make_float2(al0, al1);
                         df_prod2(ah, al, xh2[v], xl2[v], qp[v].s, qp[v].c);
-                        // The column warp reads the split, not the double.
-                        reinterpret_cast<float4 *>(rowp)[v * 32 + lane] =
-                            make_float4(ah0, ah1, al0, al1);
+                        // The column warp reads the split, not the double
+                        // (except in its native vectors).
+                        if (v < VS)
+                            reinterpret_cast<float4 *>(rowp)[v * 32 + lane] =
+                                make_float4(ah0, ah1, al0, al1);
                     }
                     DF2 h;
                     if constexpr (VPL == 4)
@@ -765,6 +773,9 @@ atax_cluster_f64_ws_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxP
         DF2 grp2[VPL];
 #pragma unroll
         for (int v = 0; v < VPL; ++v) grp2[v].s = grp2[v].c = make_float2(0.f, 0.f);
+        double nacc[NV > 0 ? NV : 1][VE];  // native column sums (vectors VS ..)
+#pragma unroll
+        for (int v = 0; v < (NV > 0 ? NV : 1); ++v) nacc[v][0] = nacc[v][1] = 0.0;
         int ngrp = 0;
         uint32_t nissued = 0;
         bool ok = true;
@@ -785,8 +796,18 @@ atax_cluster_f64_ws_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxP
                     const float2 th2 = make_float2(t.x, t.x), tl2 = make_float2(t.y, t.y);
                     const float4 *rowp =
                         reinterpret_cast<const float4 *>(box + (size_t)i * ROW_BYTES);
+                    if constexpr (NV > 0) {
+                        const double td = tvec[bp * R + i];
+                        const double2 *rowd = reinterpret_cast<const double2 *>(rowp);
 #pragma unroll
-                    for (int v = 0; v < VPL; ++v) {
+                        for (int v = VS; v < VPL; ++v) {
+                            const double2 a = rowd[v * 32 + lane];
+                            nacc[v - VS][0] = fma(a.x, td, nacc[v - VS][0]);
+                            nacc[v - VS][1] = fma(a.y, td, nacc[v - VS][1]);
+                        }
+                    }
+#pragma unroll
+                    for (int v = 0; v < VS; ++v) {
                         const float4 f = rowp[v * 32 + lane];
                         float2 p0, p1;
                         df_prod2(make_float2(f.x, f.y), make_float2(f.z, f.w), th2, tl2, p0,
@@ -800,7 +821,7 @@ atax_cluster_f64_ws_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxP
                     }
                 }
 #pragma unroll
-                for (int v = 0; v < VPL; ++v) grp2[v] = df_add2(grp2[v], tacc2[v]);
+                for (int v = 0; v < VS; ++v) grp2[v] = df_add2(grp2[v], tacc2[v]);
             } else {
                 // Native fp64 from global memory (the shared copy holds the
                 // split, which is garbage for values out of range).
@@ -819,7 +840,7 @@ atax_cluster_f64_ws_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxP
             }
             if (++ngrp == kGroupTiles || jp == ns - 1) {
 #pragma unroll
-                for (int v = 0; v < VPL; ++v)
+                for (int v = 0; v < VS; ++v)
 #pragma unroll
                     for (int e = 0; e < VE; ++e) {
                         DF x;
@@ -828,7 +849,7 @@ atax_cluster_f64_ws_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxP
                         segp[lane_col<double>(v, lane, e)] += df_to_double(x);
                     }
 #pragma unroll
-                for (int v = 0; v < VPL; ++v) grp2[v].s = grp2[v].c = make_float2(0.f, 0.f);
+                for (int v = 0; v < VS; ++v) grp2[v].s = grp2[v].c = make_float2(0.f, 0.f);
                 ngrp = 0;
             }
             // The stage is free: refill it with the stripe STAGES ahead.
@@ -838,6 +859,13 @@ atax_cluster_f64_ws_kernel(const __grid_constant__ CUtensorMap tmap, const AtaxP
                 issue(jp + STAGES);
                 ++nissued;
             }
+        }
+        // The native columns' chains join their sums of the native stripes.
+        if constexpr (NV > 0) {
+#pragma unroll
+            for (int v = VS; v < VPL; ++v)
+#pragma unroll
+                for (int e = 0; e < VE; ++e) segp[lane_col<double>(v, lane, e)] += nacc[v - VS][e];
         }
         // This cluster's column sums of the sub-band.
         if (live) {

@@ -630,6 +630,7 @@ def run_native(args):
         "pct_of_peak": round(100.0 * value / (world * peak), 2),
         "trimmed_mean_ms": round(trimmed_mean(step_ms, 3) if Ki > 6 else statistics.mean(step_ms), 5),
         "median_step_ms": round(statistics.median(step_ms), 5),
+        "min_step_ms": round(min(step_ms), 5),
         "roofline": {
             "bound": "hbm",
             "kernel": kernel_name,
@@ -736,6 +737,8 @@ def measure_config(torch, dm, inputs, w, dev, stream, W, uuid, peak, ceiling, ta
                f"L2 flushed: {FLUSH_BYTES >> 20} MiB written before each call, outside its "
                "events"),
         "trimmed_mean_ms": round(trimmed_mean(step_ms, 3), 5),
+        "median_step_ms": round(statistics.median(step_ms), 5),
+        "min_step_ms": round(min(step_ms), 5),
         "kernel": kernel_name,
         "kernel_avg_ms": round(kern_avg_ms, 5),
         "kernel_frac": round(achieved / peak, 4),

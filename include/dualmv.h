@@ -115,9 +115,11 @@ dualmv_status dualmv_i32_strided_batched(
  * GESUMMV (Table 1 / Table 2, row "GESUMMV"): with A and B both M x N
  * (leading dimensions lda, ldb >= max(1, N)), x of length N and y of
  * length M:  tmp = A x;  y = B x;  y = alpha * tmp + beta * y.
- * Floating-point sums have a fixed order (deterministic).  Errors as for
- * dualmv_f32: DUALMV_ERR_INVALID_VALUE for bad sizes or NULL pointers with
- * nonzero extents; N == 0 sets y to zero. */
+ * Floating-point sums have a fixed order (deterministic).  y must not
+ * overlap A, B or x: the pass over B may start while the pass over A still
+ * reads (the two share no buffer).  Errors as for dualmv_f32:
+ * DUALMV_ERR_INVALID_VALUE for bad sizes or NULL pointers with nonzero
+ * extents; N == 0 sets y to zero. */
 dualmv_status dualmv_gesummv_f32(int64_t M, int64_t N, float alpha, const float *A,
                                  int64_t lda, float beta, const float *B, int64_t ldb,
                                  const float *x, float *y, dualmv_stream_t stream);
@@ -191,8 +193,10 @@ dualmv_status dualmv_gemver_f64(int64_t M, int64_t N, double alpha, double beta,
  * (update_A == 0).  By default it uses the factorisation
  * A_hat^T y = A^T y + v1 (u1 . y) + v2 (u2 . y) and
  * A_hat x = A x + u1 (v1 . x) + u2 (v2 . x): a columns-only and a rows-only
- * pass of the plain kernels plus four dot products (compensated, fixed
- * order), with no per-element update.  dualmv_gemver_set_onthefly(1) makes
+ * pass of the plain kernels plus four dot products (fp64 sums in a fixed
+ * order, compensated per thread when a thread adds more than 64 products;
+ * error within about 80 u of the products' magnitudes), with no
+ * per-element update.  dualmv_gemver_set_onthefly(1) makes
  * it form A_hat element by element as it streams A, as it always does with
  * update_A (tests, benchmarks).  Returns the previous setting. */
 int dualmv_gemver_set_onthefly(int onthefly);

@@ -79,8 +79,8 @@ __global__ void gemver_w_kernel(T *w, const T *t, int64_t n, T alpha) {
 //   A_hat^T y = A^T y + v1 (u1 . y) + v2 (u2 . y)
 //   A_hat x   = A x   + u1 (v1 . x) + u2 (v2 . x)
 // Two dot products per side (a . c and b . c), deterministic: kDotChunks
-// blocks per product each take one contiguous chunk (thread k: elements
-// k, k + 256, ... of the chunk, in order).  A thread with at most
+// blocks per product each take one contiguous chunk (thread k of a block of
+// T threads: elements k, k + T, ... of the chunk, in order).  A thread with at most
 // kPlainPerThread elements sums them with fp64 FMAs; one with more sums
 // them compensated (TwoProduct/TwoSum) and rounds that once.  The block
 // adds its threads' sums in a fixed tree of plain fp64 adds, and the kernel
@@ -194,8 +194,8 @@ __device__ __forceinline__ void dot_block_store2(double v1, double v2, double *h
 // that grid before reading its inputs, and only then lets its own
 // dependents launch, so that every grid before it has completed when they
 // start (GEMVER's columns pass relies on that; see Params::pdl_late).  Its
-// blocks are small (128 threads, 32 registers each) so that one fits on an
-// SM beside a CTA of that pass.
+// blocks are small (128 threads, under 48 registers each) so that one fits
+// on an SM beside a CTA of that pass.
 constexpr int kDotThreads = 128;
 
 template <typename T>

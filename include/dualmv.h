@@ -310,6 +310,19 @@ void dualmv_record_kernel_events(void *start, void *stop);
 dualmv_status dualmv_read_probe(const void *buf, int64_t bytes, uint32_t *out,
                                 dualmv_stream_t stream);
 
+/* Instrumentation for the failure-detection tests, not part of the method:
+ * enqueues on `stream` one warp that waits for an mbarrier phase that
+ * nothing completes, through the same bounded waits as the library's
+ * kernels (CTA scope if cluster_scope == 0, the cluster kernels' cluster
+ * scope otherwise).  After about 2 s the wait gives up: it sets the device
+ * fault word, so the next dualmv_device_fault returns DUALMV_ERR_TIMEOUT,
+ * and the kernel exits normally, leaving the context usable.  The device
+ * int32 *waited receives 0 when the wait ran out, 1 if it returned without
+ * running out (which nothing can make it do).  DUALMV_ERR_INVALID_VALUE for
+ * a NULL `waited`, nothing enqueued. */
+dualmv_status dualmv_selftest_wait_timeout(int cluster_scope, int32_t *waited,
+                                          dualmv_stream_t stream);
+
 /* ---- planner (pure host code, no CUDA call) ----------------------------
  * The work decomposition a call would use.  A is cut into column bands of
  * `band_cols` columns and row stripes of `tile_rows` rows; a tile is one

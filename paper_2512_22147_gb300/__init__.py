@@ -30,7 +30,8 @@ _BINDING_NAMES = {
     "dualmv_last_variant", "TuneStep", "dualmv_atax_set_two_pass",
     "dualmv_gemver_set_onthefly", "dualmv_last_kernel", "DUALMV_KERNEL_PHASED",
     "DUALMV_KERNEL_PLAIN", "dualmv_atax_last_path", "DUALMV_ATAX_ONE_READ",
-    "DUALMV_ATAX_TWO_PASS", "dualmv_read_probe", "dualmv_pool_usage", "DUALMV_KERNEL_CLUSTER",
+    "DUALMV_ATAX_TWO_PASS", "dualmv_read_probe", "dualmv_pool_usage",
+    "dualmv_selftest_wait_timeout", "DUALMV_KERNEL_CLUSTER",
     "dualmv_gemver_last_path", "DUALMV_GEMVER_FACTORED", "DUALMV_GEMVER_ONTHEFLY",
     "DUALMV_GEMVER_UPDATE_SPLIT", "dualmv_tune_f32_strided_batched",
     "dualmv_tune_f64_strided_batched", "dualmv_tune_i32_strided_batched",

@@ -63,7 +63,7 @@ EXPORTED = (
     "dualmv_tune_i32_strided_batched", "dualmv_tuned_variant_batched",
     "dualmv_atax_set_two_pass", "dualmv_gemver_set_onthefly", "dualmv_last_kernel",
     "dualmv_atax_last_path", "dualmv_read_probe", "dualmv_pool_usage",
-    "dualmv_gemver_last_path",
+    "dualmv_gemver_last_path", "dualmv_selftest_wait_timeout",
 )
 
 
@@ -170,6 +170,8 @@ def _load() -> ctypes.CDLL:
     lib.dualmv_gemver_last_path.argtypes, lib.dualmv_gemver_last_path.restype = [], i32
     lib.dualmv_read_probe.argtypes = [vp, i64, vp, vp]
     lib.dualmv_read_probe.restype = st
+    lib.dualmv_selftest_wait_timeout.argtypes = [ctypes.c_int, vp, vp]
+    lib.dualmv_selftest_wait_timeout.restype = st
     lib.dualmv_pool_usage.argtypes = [ctypes.c_int, ctypes.POINTER(i64), ctypes.POINTER(i64),
                                       ctypes.c_int]
     lib.dualmv_pool_usage.restype = st
@@ -352,6 +354,14 @@ def dualmv_read_probe(buf, nbytes: int, out, stream) -> int:
     """Benchmark instrumentation: one 16-byte-load pass over ``nbytes`` of
     device memory at ``buf`` (xor-folded into the device word ``out``)."""
     return _lib.dualmv_read_probe(buf, nbytes, out, stream)
+
+
+def dualmv_selftest_wait_timeout(cluster_scope: int, waited, stream) -> int:
+    """Failure-detection test instrumentation: one warp waits, through the
+    library's bounded mbarrier waits, on a phase nothing completes; the wait
+    runs out after about 2 s, sets the device fault word and writes 0 to the
+    device int32 ``waited``."""
+    return _lib.dualmv_selftest_wait_timeout(cluster_scope, waited, stream)
 
 
 def dualmv_pool_usage(device: int, reset_high: bool = False):

@@ -2378,6 +2378,15 @@ dualmv_status dualmv_read_probe(const void *buf, int64_t bytes, uint32_t *out,
     return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
 }
 
+dualmv_status dualmv_selftest_wait_timeout(int cluster_scope, int32_t *waited,
+                                          dualmv_stream_t stream) {
+    if (waited == nullptr) return DUALMV_ERR_INVALID_VALUE;
+    dmv::wait_selftest_kernel<<<1, 32, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+        cluster_scope != 0 ? 1 : 0, waited);
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
+}
+
 dualmv_status dualmv_pool_usage(int device, int64_t *reserved_bytes, int64_t *used_high_bytes,
                                 int reset_high) {
     if (device < 0 || device >= kMaxDevices || reserved_bytes == nullptr ||

@@ -11,6 +11,9 @@
 
 #include <cstdint>
 
+#include "dualmv_atax.cuh"
+#include "dualmv_kernels.cuh"
+
 namespace dmv {
 
 constexpr int kProbeThreads = 512;
@@ -43,6 +46,27 @@ read_probe_kernel(const uint4 *__restrict__ src, int64_t n16, uint32_t *out) {
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1) acc ^= __shfl_xor_sync(0xffffffffu, acc, off);
     if ((threadIdx.x & 31) == 0) atomicXor(out, acc);
+}
+
+// Wait self-test, for the failure-detection tests: thread 0 waits for phase
+// 0 of an mbarrier that nothing arrives on, through the bounded waits of the
+// streaming kernels (CTA scope) or of the cluster kernels (cluster scope;
+// this CTA is a cluster of one).  After kWaitTimeoutNs the wait sets the
+// device fault word and returns false, and the kernel exits as the
+// library's kernels do after a timeout.  *waited = 1 if the wait returned
+// true (nothing can make it), 0 if it ran out.
+__global__ void __launch_bounds__(32) wait_selftest_kernel(int cluster_scope, int32_t *waited) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncwarp();
+    if (threadIdx.x == 0) {
+        const bool ok = cluster_scope ? mbar_wait_cluster_bounded(smem_u32(&bar), 0u)
+                                      : mbar_wait_bounded(smem_u32(&bar), 0u);
+        *waited = ok ? 1 : 0;
+    }
 }
 
 }  // namespace dmv

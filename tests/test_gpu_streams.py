@@ -9,7 +9,12 @@ double-float fp64 kernel, a strided batch, GEMVER):
   * the same problems launched on several streams without waiting for one
     another give the bits of the same problems run one after another;
   * a graph of such calls, replayed several times, gives the bits of the
-    eager calls, and those bits match the oracle."""
+    eager calls, and those bits match the oracle;
+  * GEMVER and GESUMMV, whose kernels run as programmatic dependents of one
+    another (GEMVER's columns pass beside its u . y kernel, GESUMMV's pass
+    over B after its pass over A): GEMVER on two streams at once, GESUMMV
+    right after kernels that rewrote its inputs, and both replayed from a
+    graph give the bits of the same calls run alone."""
 import numpy as np
 import pytest
 import torch
@@ -177,3 +182,51 @@ def test_gesummv_back_to_back_sees_the_previous_writes(dtype):
     want = oracle.gesummv(An, Bn, y2.cpu().numpy(), 1.0, -1.0, N=n)
     den = (np.abs(An) + np.abs(Bn)) @ np.abs(y2.cpu().numpy().astype(np.float64))
     assert scaled_error(y3.cpu().numpy(), want, den) <= TOL[dtype]
+
+
+@pytest.mark.parametrize("dtype", ["f64", "f32"])
+def test_gemver_and_gesummv_graph_replays_give_the_eager_bits(dtype):
+    """GEMVER (its u . y kernel runs beside the columns pass, which waits for
+    it only before it exits) and GESUMMV (the pass over B after the pass
+    over A, the same way), captured in one CUDA graph: every replay gives the
+    bits of the eager calls, and GESUMMV's y matches the oracle (GEMVER's
+    parity is checked in test_gpu_ops.py)."""
+    dist = "normal" if dtype == "f64" else "uniform"
+    ops = inputs.generate_gemver(
+        inputs.Workload("gv", dtype, 1500, 2000, 2000, dist, 80, op="gemver"), DEV)
+    A, u1, v1, u2, v2, w, x, y, z = ops
+    GA, GB, gx = inputs.generate_gesummv(
+        inputs.Workload("gs", dtype, 1700, 1300, 1300, dist, 81, op="gesummv"), DEV)
+    w0, x0 = w.clone(), x.clone()
+    gy = torch.empty(1700, dtype=GA.dtype, device=DEV)
+
+    def calls():
+        dm.gemver(A, u1, v1, u2, v2, w, x, y, z, alpha=1.5, beta=0.5)
+        dm.gesummv(GA, GB, gx, alpha=0.5, beta=2.0, y=gy)
+
+    calls()
+    torch.cuda.synchronize()
+    eager = (w.clone(), x.clone(), gy.clone())
+    side = torch.cuda.Stream(DEV)
+    side.wait_stream(torch.cuda.current_stream(DEV))
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side):
+        calls()                      # warm the pool on this stream first
+        side.synchronize()
+        with torch.cuda.graph(graph, stream=side):
+            calls()
+    torch.cuda.current_stream(DEV).wait_stream(side)
+    for rep in range(3):
+        w.copy_(w0)
+        x.copy_(x0)
+        gy.zero_()
+        graph.replay()
+        torch.cuda.synchronize()
+        for t0, t1 in zip((w, x, gy), eager):
+            assert torch.equal(t0, t1), rep
+    assert dm.device_fault() == dm.DUALMV_SUCCESS
+    An, Bn, xn = GA.cpu().numpy(), GB.cpu().numpy(), gx.cpu().numpy()
+    want = oracle.gesummv(An, Bn, xn, 0.5, 2.0)
+    den = 0.5 * (np.abs(An) @ np.abs(xn)) + 2.0 * (np.abs(Bn) @ np.abs(xn))
+    assert scaled_error(gy.cpu().numpy(), want, den) <= TOL[dtype]
+    del graph

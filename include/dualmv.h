@@ -399,6 +399,11 @@ typedef struct dualmv_variant_t {
     int32_t batched;        /* 1 if the variant also runs strided batches  */
                             /* (a 3-D tensor-map instance), so that        */
                             /* dualmv_tune_*_strided_batched may choose it */
+    int32_t single_sided;   /* 1 if it also runs single-sided passes (q    */
+                            /* only, s only: GESUMMV, GEMVER, ATAX's two   */
+                            /* passes), so that dualmv_tune_pass_* may     */
+                            /* choose it                                   */
+    int32_t pad_;           /* zero                                        */
     int64_t smem_bytes;     /* dynamic shared memory per CTA              */
 } dualmv_variant_t;
 
@@ -413,9 +418,10 @@ dualmv_status dualmv_variant_info(int32_t dtype, int32_t index, dualmv_variant_t
 /* Forces variant `index` for every eligible call of `dtype` in this
  * process (-1 restores the normal choice: a tuned variant for the shape if
  * dualmv_tune_* recorded one, else entry 0).  A strided-batched call runs
- * the forced variant if it has a batched instance, else entry 0.  Returns
- * the previous setting, or -2 for an unknown dtype or an index out of
- * range.  Meant for tests. */
+ * the forced variant if it has a batched instance, and a single-sided pass
+ * (of GESUMMV, GEMVER's columns pass, ATAX's two passes) if it has
+ * single-sided instances; else entry 0.  Returns the previous setting, or
+ * -2 for an unknown dtype or an index out of range.  Meant for tests. */
 int32_t dualmv_set_variant(int32_t dtype, int32_t index);
 
 /* The variant recorded by dualmv_tune_* for this dtype and shape (one
@@ -427,13 +433,19 @@ int32_t dualmv_tuned_variant(int32_t dtype, int64_t M, int64_t N, int64_t lda);
 int32_t dualmv_tuned_variant_batched(int32_t dtype, int64_t M, int64_t N, int64_t lda,
                                      int64_t batch);
 
+/* The variant recorded by dualmv_tune_pass_* for this dtype, shape and
+ * pass (DUALMV_PASS_ROWS or DUALMV_PASS_COLS), or -1. */
+int32_t dualmv_tuned_variant_pass(int32_t dtype, int64_t M, int64_t N, int64_t lda,
+                                  int32_t pass);
+
 /* Forgets every recorded tuning result. */
 void dualmv_tune_clear(void);
 
-/* The variant the calling thread's last dual-product call launched (one
- * problem or a strided batch): its table index, or -1 if that call ran no
- * variant of the table (an empty problem, the phased, plain-load or
- * single-cluster path, a single-sided call, native fp64 by default, or an
+/* The variant the calling thread's last dual-product call or single-sided
+ * pass launched (one problem or a strided batch): its table index, or -1
+ * if that call ran no variant of the table (an empty problem, the phased,
+ * plain-load or single-cluster path, a single-sided pass on its default
+ * kernel or walking its tiles backwards, native fp64 by default, or an
  * error).  Instrumentation for tests and benchmarks. */
 int32_t dualmv_last_variant(void);
 
@@ -552,6 +564,29 @@ dualmv_status dualmv_tune_i32_strided_batched(
     int64_t strideP, const int32_t *r, int64_t strideR, int64_t *q, int64_t strideQ, int64_t *s,
     int64_t strideS, int64_t batch, const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
     dualmv_stream_t stream);
+
+/* The same loop for one single-sided pass, the building block of GESUMMV
+ * (rows: q = A x), GEMVER (its columns pass: s = A^T y) and ATAX's two-pass
+ * fallback (both): pass DUALMV_PASS_ROWS computes out = A x (x of length N,
+ * out of length M), DUALMV_PASS_COLS out = A^T x (x of length M, out of
+ * length N).  Candidates are the variants with single-sided instances
+ * (dualmv_variant_t.single_sided: every fp32 shape, the packed
+ * self-loading fp64 shapes); K^(0) is entry 0; Eq. 4 compares `out`.  The
+ * choice is recorded for (dtype, M, N, lda, pass) and used by later
+ * single-sided passes of that shape that walk their tiles forwards
+ * (dualmv_tuned_variant_pass; GEMVER's rows pass, which walks backwards to
+ * start on tiles still in L2, keeps its kernel).  The chosen variant's
+ * result is left in `out`.  DUALMV_ERR_INVALID_VALUE for an unknown pass
+ * and the argument errors of dualmv_tune_*; blocks until done. */
+enum { DUALMV_PASS_ROWS = 1, DUALMV_PASS_COLS = 2 };
+dualmv_status dualmv_tune_pass_f32(int64_t M, int64_t N, const float *A, int64_t lda,
+                                   int32_t pass, const float *x, float *out,
+                                   const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+                                   dualmv_stream_t stream);
+dualmv_status dualmv_tune_pass_f64(int64_t M, int64_t N, const double *A, int64_t lda,
+                                   int32_t pass, const double *x, double *out,
+                                   const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+                                   dualmv_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -35,9 +35,11 @@ _BINDING_NAMES = {
     "dualmv_gemver_last_path", "DUALMV_GEMVER_FACTORED", "DUALMV_GEMVER_ONTHEFLY",
     "DUALMV_GEMVER_UPDATE_SPLIT", "dualmv_tune_f32_strided_batched",
     "dualmv_tune_f64_strided_batched", "dualmv_tune_i32_strided_batched",
-    "dualmv_tuned_variant_batched",
+    "dualmv_tuned_variant_batched", "dualmv_tune_pass_f32", "dualmv_tune_pass_f64",
+    "dualmv_tuned_variant_pass", "DUALMV_PASS_ROWS", "DUALMV_PASS_COLS",
 }
-_API_NAMES = {"dualmv", "device_fault", "gesummv", "atax", "gemver", "tune", "variants"}
+_API_NAMES = {"dualmv", "device_fault", "gesummv", "atax", "gemver", "tune", "tune_pass",
+              "variants"}
 
 
 def __getattr__(name):

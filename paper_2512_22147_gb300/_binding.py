@@ -46,6 +46,8 @@ DUALMV_ATAX_ONE_READ = 1
 DUALMV_GEMVER_FACTORED = 0
 DUALMV_GEMVER_ONTHEFLY = 1
 DUALMV_GEMVER_UPDATE_SPLIT = 2
+DUALMV_PASS_ROWS = 1
+DUALMV_PASS_COLS = 2
 
 EXPORTED = (
     "dualmv_f32", "dualmv_f64", "dualmv_i32",
@@ -63,7 +65,8 @@ EXPORTED = (
     "dualmv_tune_i32_strided_batched", "dualmv_tuned_variant_batched",
     "dualmv_atax_set_two_pass", "dualmv_gemver_set_onthefly", "dualmv_last_kernel",
     "dualmv_atax_last_path", "dualmv_read_probe", "dualmv_pool_usage",
-    "dualmv_gemver_last_path", "dualmv_selftest_wait_timeout",
+    "dualmv_gemver_last_path", "dualmv_selftest_wait_timeout", "dualmv_tune_pass_f32",
+    "dualmv_tune_pass_f64", "dualmv_tuned_variant_pass",
 )
 
 
@@ -85,8 +88,8 @@ class Plan(ctypes.Structure):
 class Variant(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "index", "kernel", "warps", "rows_per_warp", "stages", "band_cols", "tile_rows",
-        "threads", "native_cols", "producer_warp", "packed", "batched")] + [
-        ("smem_bytes", ctypes.c_int64)]
+        "threads", "native_cols", "producer_warp", "packed", "batched", "single_sided",
+        "pad_")] + [("smem_bytes", ctypes.c_int64)]
 
 
 class TuneConfig(ctypes.Structure):
@@ -187,6 +190,13 @@ def _load() -> ctypes.CDLL:
         f.restype = st
     lib.dualmv_tuned_variant_batched.argtypes = [i32, i64, i64, i64, i64]
     lib.dualmv_tuned_variant_batched.restype = i32
+    for t in ("f32", "f64"):
+        f = getattr(lib, f"dualmv_tune_pass_{t}")
+        f.argtypes = [i64, i64, vp, i64, i32, vp, vp, ctypes.POINTER(TuneConfig),
+                      ctypes.POINTER(TuneResult), vp]
+        f.restype = st
+    lib.dualmv_tuned_variant_pass.argtypes = [i32, i64, i64, i64, i32]
+    lib.dualmv_tuned_variant_pass.restype = i32
     return lib
 
 
@@ -421,6 +431,26 @@ def _tune_batched(tag, M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS, batch, cfg,
         M, N, A, lda, sA, p, sP, r, sR, q, sQ, s, sS, batch,
         ctypes.byref(cfg) if cfg is not None else None,
         ctypes.byref(res) if res is not None else None, stream)
+
+
+def _tune_pass(tag, M, N, A, lda, pass_, x, out, cfg, res, stream):
+    return getattr(_lib, f"dualmv_tune_pass_{tag}")(
+        M, N, A, lda, pass_, x, out, ctypes.byref(cfg) if cfg is not None else None,
+        ctypes.byref(res) if res is not None else None, stream)
+
+
+def dualmv_tune_pass_f32(M, N, A, lda, pass_, x, out, cfg, res, stream):
+    """Tune one single-sided pass: DUALMV_PASS_ROWS (out = A x) or
+    DUALMV_PASS_COLS (out = A^T x)."""
+    return _tune_pass("f32", M, N, A, lda, pass_, x, out, cfg, res, stream)
+
+
+def dualmv_tune_pass_f64(M, N, A, lda, pass_, x, out, cfg, res, stream):
+    return _tune_pass("f64", M, N, A, lda, pass_, x, out, cfg, res, stream)
+
+
+def dualmv_tuned_variant_pass(dtype: int, M: int, N: int, lda: int, pass_: int) -> int:
+    return _lib.dualmv_tuned_variant_pass(dtype, M, N, lda, pass_)
 
 
 def dualmv_tune_f32_strided_batched(*args):

@@ -299,3 +299,43 @@ def tune(A: torch.Tensor, p: torch.Tensor, r: torch.Tensor, q: torch.Tensor | No
                      "ms": st.ms, "fe": st.fe} for st in res.trace[:res.trace_len]]
     rep["q"], rep["s"] = q, s
     return rep
+
+
+def tune_pass(A: torch.Tensor, x: torch.Tensor, pass_: str = "rows",
+              out: torch.Tensor | None = None, repeats: int = 30, trim: int = 3,
+              max_rounds: int = 4, candidates: int = 4, min_gain: float = 0.01,
+              flush_l2: bool = True, stream: torch.cuda.Stream | None = None) -> dict:
+    """Tune one single-sided pass for A's shape: ``pass_="rows"`` computes
+    ``out = A x`` (the passes of GESUMMV and GEMVER's rows side),
+    ``pass_="cols"`` computes ``out = A^T x`` (GEMVER's columns pass); later
+    forward passes of the same shape use the result.  A is one float32 or
+    float64 (M, N) problem.  Blocks until done.  Returns the tuner's report;
+    ``out`` holds the chosen variant's result."""
+    if A.dtype not in (torch.float32, torch.float64) or A.dim() != 2:
+        raise ValueError("tune_pass takes a 2-D float32 or float64 A")
+    if pass_ not in ("rows", "cols"):
+        raise ValueError('pass_ must be "rows" or "cols"')
+    M, N, lda = _matrix(A, "A")
+    rows = pass_ == "rows"
+    nx, nout = (N, M) if rows else (M, N)
+    if out is None:
+        out = torch.empty(nout, dtype=A.dtype, device=A.device)
+    for t_, n, ln in ((x, "x", nx), (out, "out", nout)):
+        if t_.dtype != A.dtype or t_.device != A.device or t_.dim() != 1 or \
+                not t_.is_contiguous() or t_.numel() != ln:
+            raise ValueError(f"{n} must be a contiguous {A.dtype} vector of length {ln} "
+                             "on A's device")
+    cfg = B.TuneConfig(repeats, trim, max_rounds, candidates, min_gain, int(flush_l2))
+    res = B.TuneResult()
+    strm = stream if stream is not None else torch.cuda.current_stream(A.device)
+    fn = getattr(B, f"dualmv_tune_pass_{_TAG[A.dtype]}")
+    rc = fn(M, N, A.data_ptr(), lda, B.DUALMV_PASS_ROWS if rows else B.DUALMV_PASS_COLS,
+            x.data_ptr(), out.data_ptr(), cfg, res, strm.cuda_stream)
+    if rc != B.DUALMV_SUCCESS:
+        raise B.DualmvError(rc, "dualmv_tune_pass")
+    rep = {f: getattr(res, f) for f, _ in res._fields_
+           if f not in ("trace", "trace_len")}
+    rep["trace"] = [{"index": st.index, "round": st.round, "feasible": bool(st.feasible),
+                     "ms": st.ms, "fe": st.fe} for st in res.trace[:res.trace_len]]
+    rep["out"] = out
+    return rep

@@ -690,6 +690,9 @@ struct Variant {
     Geometry geo;
     LaunchFn launch;
     LaunchFn launch3d;  // strided batches (3-D tensor map), or nullptr
+    // Single-sided passes (q only, s only: GESUMMV, GEMVER's forward passes,
+    // ATAX's two-pass fallback), or nullptr.
+    LaunchFn launch_q = nullptr, launch_s = nullptr;
 };
 
 template <typename T, int W, int RPW, int S, bool k3d = false>
@@ -705,9 +708,23 @@ cudaError_t launch_f64e_variant(const CUtensorMap &m, const Params &p, const dua
                                                                              st);
 }
 
+// Single-sided instances (kOut = kOutQ or kOutS) of the same shapes.
+template <typename T, int W, int RPW, int S, int kOut>
+cudaError_t launch_stream_side(const CUtensorMap &m, const Params &p, const dualmv_plan_t &pl,
+                               int dev, cudaStream_t st) {
+    return launch_stream<T, true, false, kOut, false, W, RPW, S>(m, p, pl, dev, st);
+}
+
+template <int W, int RPW, int S, int NC, bool kSelf, bool kPack, int BAND, int kOut>
+cudaError_t launch_f64e_side(const CUtensorMap &m, const Params &p, const dualmv_plan_t &pl,
+                             int dev, cudaStream_t st) {
+    return launch_f64e<false, kOut, W, RPW, S, NC, kSelf, kPack, BAND>(m, p, pl, dev, st);
+}
+
 Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind kind,
                      const Geometry &g, LaunchFn fn, int NC = 0, bool self_load = false,
-                     LaunchFn fn3d = nullptr) {
+                     LaunchFn fn3d = nullptr, LaunchFn fn_q = nullptr,
+                     LaunchFn fn_s = nullptr) {
     Variant v;
     v.info.index = index;
     v.info.kernel = kernel;
@@ -718,6 +735,8 @@ Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind 
     v.info.producer_warp = self_load ? 0 : 1;
     v.info.packed = 0;
     v.info.batched = fn3d != nullptr ? 1 : 0;
+    v.info.single_sided = (fn_q != nullptr && fn_s != nullptr) ? 1 : 0;
+    v.info.pad_ = 0;
     v.info.band_cols = (int32_t)g.band_cols;
     v.info.tile_rows = (int32_t)g.tile_rows;
     v.info.threads = (int32_t)g.threads;
@@ -726,31 +745,42 @@ Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind 
     v.geo = g;
     v.launch = fn;
     v.launch3d = fn3d;
+    v.launch_q = fn_q;
+    v.launch_s = fn_s;
     return v;
 }
 
 // kBatched: the variant also has a strided-batched instance (every shape of
 // the 4-byte tables; not the native fp64 entry, which no batched entry
-// neighbours).
+// neighbours).  fp32 shapes also have single-sided instances.
 template <typename T, int W, int RPW, int S, bool kBatched = true>
 Variant stream_variant(int32_t index) {
-    LaunchFn fn3d = nullptr;
+    LaunchFn fn3d = nullptr, fn_q = nullptr, fn_s = nullptr;
     if constexpr (kBatched) fn3d = &launch_stream_variant<T, W, RPW, S, true>;
+    if constexpr (std::is_same<T, float>::value) {
+        fn_q = &launch_stream_side<T, W, RPW, S, dmv::kOutQ>;
+        fn_s = &launch_stream_side<T, W, RPW, S, dmv::kOutS>;
+    }
     return make_variant(index, DUALMV_KERNEL_STREAM, W, RPW, S, Kind::kTma,
                         stream_geometry<T, W, RPW, S>(true),
-                        &launch_stream_variant<T, W, RPW, S>, 0, false, fn3d);
+                        &launch_stream_variant<T, W, RPW, S>, 0, false, fn3d, fn_q, fn_s);
 }
 
-// kBatched: the variant also has a strided-batched instance.
+// kBatched: the variant also has a strided-batched instance, and
+// single-sided instances (the packed self-loading 256-column shapes).
 template <int W, int RPW, int S, int NC = kF64eNativeCols, bool kSelf = kF64eSelf,
           bool kPack = kF64ePack, int BAND = kF64eBand, bool kBatched = false>
 Variant f64e_variant(int32_t index) {
-    LaunchFn fn3d = nullptr;
-    if constexpr (kBatched) fn3d = &launch_f64e_variant<W, RPW, S, NC, kSelf, kPack, BAND, true>;
+    LaunchFn fn3d = nullptr, fn_q = nullptr, fn_s = nullptr;
+    if constexpr (kBatched) {
+        fn3d = &launch_f64e_variant<W, RPW, S, NC, kSelf, kPack, BAND, true>;
+        fn_q = &launch_f64e_side<W, RPW, S, NC, kSelf, kPack, BAND, dmv::kOutQ>;
+        fn_s = &launch_f64e_side<W, RPW, S, NC, kSelf, kPack, BAND, dmv::kOutS>;
+    }
     Variant v = make_variant(index, DUALMV_KERNEL_F64E, W, RPW, S, Kind::kF64e,
                              f64e_geometry<W, RPW, S, kSelf, BAND>(),
                              &launch_f64e_variant<W, RPW, S, NC, kSelf, kPack, BAND>, NC, kSelf,
-                             fn3d);
+                             fn3d, fn_q, fn_s);
     v.info.packed = kPack ? 1 : 0;
     return v;
 }
@@ -858,14 +888,17 @@ bool neighbours(const dualmv_variant_t &a, const dualmv_variant_t &b) {
 
 std::atomic<int32_t> g_forced_variant[3] = {{-1}, {-1}, {-1}};
 std::mutex g_tuned_mu;
-// Tuned choices by (dtype, M, N, lda, batch); batch 1 for single problems.
-std::map<std::tuple<int32_t, int64_t, int64_t, int64_t, int64_t>, int32_t> g_tuned;
+// Tuned choices by (dtype, M, N, lda, batch, outputs); batch 1 for single
+// problems, outputs kOutBoth for dual products, kOutQ / kOutS for
+// single-sided passes.
+std::map<std::tuple<int32_t, int64_t, int64_t, int64_t, int64_t, uint32_t>, int32_t> g_tuned;
 std::atomic<int> g_tuned_count{0};
 
-int32_t tuned_lookup(int32_t dtype, int64_t M, int64_t N, int64_t lda, int64_t batch = 1) {
+int32_t tuned_lookup(int32_t dtype, int64_t M, int64_t N, int64_t lda, int64_t batch = 1,
+                     uint32_t outputs = dmv::kOutBoth) {
     if (g_tuned_count.load(std::memory_order_acquire) == 0) return -1;
     std::lock_guard<std::mutex> lk(g_tuned_mu);
-    auto it = g_tuned.find(std::make_tuple(dtype, M, N, lda, batch));
+    auto it = g_tuned.find(std::make_tuple(dtype, M, N, lda, batch, outputs));
     return it == g_tuned.end() ? -1 : it->second;
 }
 
@@ -883,16 +916,20 @@ int32_t default_variant(int32_t dtype, const void *A, int64_t lda_bytes) {
 // the process-wide forced one, else the tuned one for this shape, else the
 // default for the shape.  nullptr means entry 0, which the ordinary launch
 // code covers.  A strided batch (batch > 1) runs a variant only if it has a
-// batched instance; otherwise entry 0.
+// batched instance, a single-sided pass (outputs kOutQ or kOutS) only if it
+// has single-sided instances; otherwise entry 0.
 const Variant *pick_variant(int32_t dtype, int64_t M, int64_t N, const void *A, int64_t lda,
-                            int64_t es, int32_t index, int64_t batch = 1) {
+                            int64_t es, int32_t index, int64_t batch = 1,
+                            uint32_t outputs = dmv::kOutBoth) {
     const std::vector<Variant> *tab = variant_table(dtype);
     if (tab == nullptr) return nullptr;
+    const bool sided = outputs != dmv::kOutBoth;
     if (index < 0) index = g_forced_variant[dtype].load(std::memory_order_relaxed);
-    if (index < 0) index = tuned_lookup(dtype, M, N, lda, batch);
-    if (index < 0) index = batch > 1 ? 0 : default_variant(dtype, A, lda * es);
+    if (index < 0) index = tuned_lookup(dtype, M, N, lda, batch, outputs);
+    if (index < 0) index = (batch > 1 || sided) ? 0 : default_variant(dtype, A, lda * es);
     if (index <= 0 || index >= (int32_t)tab->size()) return nullptr;
     if (batch > 1 && (*tab)[index].launch3d == nullptr) return nullptr;
+    if (sided && (*tab)[index].launch_q == nullptr) return nullptr;
     return &(*tab)[index];
 }
 
@@ -1067,12 +1104,13 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                    ? Kind::kF64e
                    : Kind::kTma;
     // A compiled variant other than the default (forced, tuned or named by
-    // the tuner) for a dual product (one problem or a strided batch) on the
+    // the tuner) for a dual product (one problem or a strided batch) or a
+    // single-sided pass of one problem walking its tiles forwards, on the
     // TMA path.
     const Variant *var = nullptr;
-    if (tma && outputs == dmv::kOutBoth && rank2 == nullptr &&
-        g_path != DUALMV_PATH_TMA_NATIVE_F64)
-        var = pick_variant(dtype_code<T>(), M, N, A, lda, es, variant, batch);
+    if (tma && rank2 == nullptr && g_path != DUALMV_PATH_TMA_NATIVE_F64 &&
+        (outputs == dmv::kOutBoth || (!kIntPath && batch == 1 && !reverse)))
+        var = pick_variant(dtype_code<T>(), M, N, A, lda, es, variant, batch, outputs);
     if (var != nullptr) kind = var->kind;
     if (kind == Kind::kF64e) {
         // The double-float kernel counts tiles in 32 bits; a launch of 2^31
@@ -1159,10 +1197,8 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     prm.grid = pl.grid; prm.max_seg = pl.max_segments;
     // Late wait (Params::pdl_late) for the single-sided kernels below; the
     // caller's kernel before this call triggers its dependents after its wait.
-    prm.pdl_late = (late_wait && !kIntPath && outputs != dmv::kOutBoth && rank2 == nullptr &&
-                    var == nullptr)
-                       ? 1
-                       : 0;
+    prm.pdl_late =
+        (late_wait && !kIntPath && outputs != dmv::kOutBoth && rank2 == nullptr) ? 1 : 0;
     const int64_t q_ws_bytes = pl.bands > 1 ? batch * pl.bands * M * (int64_t)sizeof(Acc) : 0;
     prm.q_ws = (pl.bands > 1 && ws) ? ws : nullptr;
     prm.s_ws = ws ? static_cast<unsigned char *>(ws) + ((q_ws_bytes + 255) / 256) * 256 : nullptr;
@@ -1189,8 +1225,13 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                                                        : (int32_t)DUALMV_KERNEL_PLAIN;
     if (e == cudaSuccess) {
         if (var != nullptr) {
-            e = three_d ? var->launch3d(map, prm, pl, dev, stream)
-                        : var->launch(map, prm, pl, dev, stream);
+            if (outputs == dmv::kOutQ)
+                e = var->launch_q(map, prm, pl, dev, stream);
+            else if (outputs == dmv::kOutS)
+                e = var->launch_s(map, prm, pl, dev, stream);
+            else
+                e = three_d ? var->launch3d(map, prm, pl, dev, stream)
+                            : var->launch(map, prm, pl, dev, stream);
             if (e == cudaSuccess) g_last_variant = var->info.index;
         } else if (rank2 != nullptr) {
             if constexpr (!kIntPath) {
@@ -1870,13 +1911,17 @@ template <typename T> constexpr double fe_tolerance() {
 template <typename T, typename Out>
 class Tuner {
   public:
-    // One problem (batch 1) or a strided batch; strides in elements.
+    // One problem (batch 1) or a strided batch; strides in elements.  With
+    // outputs kOutQ or kOutS, single-sided passes of one problem (the
+    // other side's pointers unused).
     Tuner(int64_t M, int64_t N, int64_t batch, const T *A, int64_t lda, int64_t strideA,
           const T *p, int64_t strideP, const T *r, int64_t strideR, Out *q, int64_t strideQ,
-          Out *s, int64_t strideS, const dualmv_tune_config_t &cfg, cudaStream_t stream)
+          Out *s, int64_t strideS, const dualmv_tune_config_t &cfg, cudaStream_t stream,
+          uint32_t outputs = dmv::kOutBoth)
         : M_(M), N_(N), batch_(batch), A_(A), lda_(lda), strideA_(strideA), p_(p),
           strideP_(strideP), r_(r), strideR_(strideR), q_(q), strideQ_(strideQ), s_(s),
-          strideS_(strideS), cfg_(cfg), stream_(stream) {}
+          strideS_(strideS), cfg_(cfg), stream_(stream), outputs_(outputs),
+          want_q_((outputs & dmv::kOutQ) != 0), want_s_((outputs & dmv::kOutS) != 0) {}
 
     ~Tuner() {
         for (cudaEvent_t ev : events_) cudaEventDestroy(ev);
@@ -1887,13 +1932,14 @@ class Tuner {
     }
 
     dualmv_status setup() {
-        dualmv_status st = pool_alloc(&q_base_, batch_ * M_, stream_);
-        if (st == DUALMV_SUCCESS) st = pool_alloc(&s_base_, batch_ * N_, stream_);
+        dualmv_status st = DUALMV_SUCCESS;
+        if (want_q_) st = pool_alloc(&q_base_, batch_ * M_, stream_);
+        if (st == DUALMV_SUCCESS && want_s_) st = pool_alloc(&s_base_, batch_ * N_, stream_);
         if (st == DUALMV_SUCCESS) st = pool_alloc(&fe_word_, 1, stream_);
         constexpr bool kExact = std::is_same<T, int32_t>::value;
         if (!kExact) {
-            if (st == DUALMV_SUCCESS) st = pool_alloc(&den_q_, batch_ * M_, stream_);
-            if (st == DUALMV_SUCCESS) st = pool_alloc(&den_s_, batch_ * N_, stream_);
+            if (st == DUALMV_SUCCESS && want_q_) st = pool_alloc(&den_q_, batch_ * M_, stream_);
+            if (st == DUALMV_SUCCESS && want_s_) st = pool_alloc(&den_s_, batch_ * N_, stream_);
         }
         if (st != DUALMV_SUCCESS) return st;
         int dev = 0, l2 = 0, sms = 0;
@@ -1914,10 +1960,13 @@ class Tuner {
         if (!kExact) {  // magnitude sums for the equivalence bar, once per problem
             const int64_t bc = (N_ + 255) / 256;
             for (int64_t b = 0; b < batch_; ++b) {
-                dmv::abs_rows_kernel<T><<<4 * sms, 256, 0, stream_>>>(
-                    A_ + b * strideA_, M_, N_, lda_, p_ + b * strideP_, den_q_ + b * M_);
-                dmv::abs_cols_kernel<T><<<(unsigned)(bc < 65535 ? bc : 65535), 256, 0, stream_>>>(
-                    A_ + b * strideA_, M_, N_, lda_, r_ + b * strideR_, den_s_ + b * N_);
+                if (want_q_)
+                    dmv::abs_rows_kernel<T><<<4 * sms, 256, 0, stream_>>>(
+                        A_ + b * strideA_, M_, N_, lda_, p_ + b * strideP_, den_q_ + b * M_);
+                if (want_s_)
+                    dmv::abs_cols_kernel<T>
+                        <<<(unsigned)(bc < 65535 ? bc : 65535), 256, 0, stream_>>>(
+                            A_ + b * strideA_, M_, N_, lda_, r_ + b * strideR_, den_s_ + b * N_);
                 e = cudaGetLastError();
                 if (e != cudaSuccess) return cuda_fail(e);
             }
@@ -1930,7 +1979,7 @@ class Tuner {
         Out *q = into_base ? q_base_ : q_, *s = into_base ? s_base_ : s_;
         const int64_t sq = into_base ? M_ : strideQ_, ss = into_base ? N_ : strideS_;
         return run<T, Out>(M_, N_, A_, lda_, strideA_, p_, strideP_, r_, strideR_, q, sq, s, ss,
-                           batch_, stream_, dmv::kOutBoth, nullptr, v);
+                           batch_, stream_, outputs_, nullptr, v);
     }
 
     // Score of Eq. 3: `repeats` timed calls, trimmed mean of their times.
@@ -1965,12 +2014,14 @@ class Tuner {
         const unsigned gq = (unsigned)std::min<int64_t>((M_ + 255) / 256, 1024);
         const unsigned gs = (unsigned)std::min<int64_t>((N_ + 255) / 256, 1024);
         for (int64_t b = 0; b < batch_ && e == cudaSuccess; ++b) {
-            dmv::fe_max_kernel<Out><<<gq, 256, 0, stream_>>>(q_ + b * strideQ_, q_base_ + b * M_,
-                                                             den_q_ ? den_q_ + b * M_ : nullptr,
-                                                             M_, fe_word_);
-            dmv::fe_max_kernel<Out><<<gs, 256, 0, stream_>>>(s_ + b * strideS_, s_base_ + b * N_,
-                                                             den_s_ ? den_s_ + b * N_ : nullptr,
-                                                             N_, fe_word_);
+            if (want_q_)
+                dmv::fe_max_kernel<Out><<<gq, 256, 0, stream_>>>(
+                    q_ + b * strideQ_, q_base_ + b * M_, den_q_ ? den_q_ + b * M_ : nullptr, M_,
+                    fe_word_);
+            if (want_s_)
+                dmv::fe_max_kernel<Out><<<gs, 256, 0, stream_>>>(
+                    s_ + b * strideS_, s_base_ + b * N_, den_s_ ? den_s_ + b * N_ : nullptr, N_,
+                    fe_word_);
             e = cudaGetLastError();
         }
         unsigned long long bits = 0;
@@ -1991,7 +2042,7 @@ class Tuner {
 
     // A planted mistake in a candidate's outputs, for testing the gate.
     dualmv_status plant_mistake() {
-        cudaError_t e = cudaMemsetAsync(q_, 0x7f, sizeof(Out), stream_);
+        cudaError_t e = cudaMemsetAsync(want_q_ ? q_ : s_, 0x7f, sizeof(Out), stream_);
         return e == cudaSuccess ? DUALMV_SUCCESS : cuda_fail(e);
     }
 
@@ -2009,6 +2060,8 @@ class Tuner {
     int64_t strideS_;
     dualmv_tune_config_t cfg_;
     cudaStream_t stream_;
+    uint32_t outputs_;
+    bool want_q_, want_s_;
     Out *q_base_ = nullptr, *s_base_ = nullptr;
     double *den_q_ = nullptr, *den_s_ = nullptr;
     unsigned long long *fe_word_ = nullptr;
@@ -2018,19 +2071,23 @@ class Tuner {
 };
 
 // The loop of Section 3.2 for one problem (batch 1) or a strided batch (the
-// candidates then are the variants with a batched instance).
+// candidates then are the variants with a batched instance); with outputs
+// kOutQ or kOutS, for a single-sided pass of one problem (the candidates are
+// the variants with single-sided instances).
 template <typename T, typename Out>
 dualmv_status tune_run(int64_t M, int64_t N, int64_t batch, const T *A, int64_t lda,
                        int64_t strideA, const T *p, int64_t strideP, const T *r,
                        int64_t strideR, Out *q, int64_t strideQ, Out *s, int64_t strideS,
                        const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
-                       cudaStream_t stream) {
+                       cudaStream_t stream, uint32_t outputs = dmv::kOutBoth) {
     if (cfg == nullptr || res == nullptr) return DUALMV_ERR_INVALID_VALUE;
     if (cfg->trim < 0 || cfg->repeats <= 2 * cfg->trim || cfg->max_rounds < 0 ||
         cfg->candidates < 1 || !(cfg->min_gain >= 0.0))
         return DUALMV_ERR_INVALID_VALUE;
+    const bool sided = outputs != dmv::kOutBoth;
+    if (sided && (batch != 1 || std::is_same<T, int32_t>::value)) return DUALMV_ERR_INVALID_VALUE;
     dualmv_status st = validate(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ, s,
-                                strideS, batch);
+                                strideS, batch, outputs);
     if (st != DUALMV_SUCCESS) return st;
     std::memset(res, 0, sizeof *res);
     const int64_t es = sizeof(T);
@@ -2042,7 +2099,7 @@ dualmv_status tune_run(int64_t M, int64_t N, int64_t batch, const T *A, int64_t 
                           N < INT32_MAX && batch < INT32_MAX;
     if (!eligible)
         return run<T, Out>(M, N, A, lda, strideA, p, strideP, r, strideR, q, strideQ, s, strideS,
-                           batch, stream);
+                           batch, stream, outputs);
     if (fault_injected_alloc()) return DUALMV_ERR_ALLOC;
 
     const int32_t dtype = dtype_code<T>();
@@ -2050,13 +2107,13 @@ dualmv_status tune_run(int64_t M, int64_t N, int64_t batch, const T *A, int64_t 
     constexpr double tol = fe_tolerance<T>();
     const bool plant = fault_injected("fe");
     Tuner<T, Out> tu(M, N, batch, A, lda, strideA, p, strideP, r, strideR, q, strideQ, s,
-                     strideS, *cfg, stream);
+                     strideS, *cfg, stream, outputs);
     st = tu.setup();
     if (st != DUALMV_SUCCESS) return st;
 
     // K^(0): the variant an untuned call of this shape uses; its outputs are
     // the reference for Eq. 4.
-    int32_t base = batched ? 0 : default_variant(dtype, A, lda * es);
+    int32_t base = (batched || sided) ? 0 : default_variant(dtype, A, lda * es);
     res->initial = base;
     st = tu.call(base, true);
     if (st == DUALMV_SUCCESS) st = tu.score(base, &res->baseline_ms);
@@ -2069,7 +2126,8 @@ dualmv_status tune_run(int64_t M, int64_t N, int64_t batch, const T *A, int64_t 
         std::vector<int32_t> cands;
         for (const Variant &v : tab)
             if (!tried[v.info.index] && (!batched || v.launch3d != nullptr) &&
-                neighbours(v.info, tab[base].info) && (int32_t)cands.size() < cfg->candidates)
+                (!sided || v.launch_q != nullptr) && neighbours(v.info, tab[base].info) &&
+                (int32_t)cands.size() < cfg->candidates)
                 cands.push_back(v.info.index);
         if (cands.empty()) break;
         res->rounds = d + 1;
@@ -2118,7 +2176,7 @@ dualmv_status tune_run(int64_t M, int64_t N, int64_t batch, const T *A, int64_t 
     res->best_ms = base_ms;
     {
         std::lock_guard<std::mutex> lk(g_tuned_mu);
-        g_tuned[std::make_tuple(dtype, M, N, lda, batched ? batch : (int64_t)1)] = base;
+        g_tuned[std::make_tuple(dtype, M, N, lda, batched ? batch : (int64_t)1, outputs)] = base;
         g_tuned_count.store((int)g_tuned.size(), std::memory_order_release);
     }
     st = tu.call(base, false);  // leave the chosen variant's outputs in q, s
@@ -2229,6 +2287,22 @@ dualmv_status run_f32_noalloc(int64_t M, int64_t N, const float *A, int64_t lda,
 }  // namespace
 
 // ================================================================ C ABI ===
+
+// One single-sided pass: DUALMV_PASS_ROWS (out = A x) or DUALMV_PASS_COLS
+// (out = A^T x), through the same tuner loop.
+template <typename T>
+dualmv_status tune_pass(int64_t M, int64_t N, const T *A, int64_t lda, int32_t pass,
+                        const T *x, T *out, const dualmv_tune_config_t *cfg,
+                        dualmv_tune_result_t *res, dualmv_stream_t stream) {
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (pass == DUALMV_PASS_ROWS)
+        return tune_run<T, T>(M, N, 1, A, lda, 0, x, 0, nullptr, 0, out, 0, nullptr, 0, cfg, res,
+                              st, dmv::kOutQ);
+    if (pass == DUALMV_PASS_COLS)
+        return tune_run<T, T>(M, N, 1, A, lda, 0, nullptr, 0, x, 0, nullptr, 0, out, 0, cfg, res,
+                              st, dmv::kOutS);
+    return DUALMV_ERR_INVALID_VALUE;
+}
 
 extern "C" {
 
@@ -2471,6 +2545,12 @@ int32_t dualmv_tuned_variant_batched(int32_t dtype, int64_t M, int64_t N, int64_
     return tuned_lookup(dtype, M, N, lda, batch > 1 ? batch : 1);
 }
 
+int32_t dualmv_tuned_variant_pass(int32_t dtype, int64_t M, int64_t N, int64_t lda, int32_t pass) {
+    if (pass != DUALMV_PASS_ROWS && pass != DUALMV_PASS_COLS) return -1;
+    return tuned_lookup(dtype, M, N, lda, 1,
+                        pass == DUALMV_PASS_ROWS ? (uint32_t)dmv::kOutQ : (uint32_t)dmv::kOutS);
+}
+
 int32_t dualmv_last_variant(void) { return g_last_variant; }
 
 int32_t dualmv_last_kernel(void) { return g_last_kernel; }
@@ -2497,6 +2577,20 @@ dualmv_status dualmv_tune_f32(int64_t M, int64_t N, const float *A, int64_t lda,
                               dualmv_stream_t stream) {
     return tune_run<float, float>(M, N, 1, A, lda, 0, p, 0, r, 0, q, 0, s, 0, cfg, res,
                                   reinterpret_cast<cudaStream_t>(stream));
+}
+
+dualmv_status dualmv_tune_pass_f32(int64_t M, int64_t N, const float *A, int64_t lda,
+                                   int32_t pass, const float *x, float *out,
+                                   const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+                                   dualmv_stream_t stream) {
+    return tune_pass<float>(M, N, A, lda, pass, x, out, cfg, res, stream);
+}
+
+dualmv_status dualmv_tune_pass_f64(int64_t M, int64_t N, const double *A, int64_t lda,
+                                   int32_t pass, const double *x, double *out,
+                                   const dualmv_tune_config_t *cfg, dualmv_tune_result_t *res,
+                                   dualmv_stream_t stream) {
+    return tune_pass<double>(M, N, A, lda, pass, x, out, cfg, res, stream);
 }
 
 dualmv_status dualmv_tune_f64(int64_t M, int64_t N, const double *A, int64_t lda,

@@ -3,14 +3,18 @@ of every dtype is held to the parity bar against the oracle on shapes that
 span several tiles with ragged tails; the tuner's loop (Section 3.2) is run
 on a mid-size problem per dtype and its report, its recorded choice and its
 outputs are checked; a mistake planted in every candidate's outputs must be
-caught by the equivalence gate (Eq. 4)."""
+caught by the equivalence gate (Eq. 4).  The same for strided batches and
+for single-sided passes (the building blocks of GESUMMV, GEMVER and ATAX's
+two-pass path): every variant with single-sided instances against the
+oracle through those operations, and the pass tuner's report and choice."""
 import numpy as np
 import pytest
 import torch
 
+import oracle
 import paper_2512_22147_gb300 as dm
 from paper_2512_22147_gb300 import inputs
-from parity import TOL, compare_problem, run_and_compare
+from parity import TOL, compare_problem, run_and_compare, scaled_error
 
 pytestmark = pytest.mark.gpu
 
@@ -265,4 +269,118 @@ def test_batched_tuner_catches_a_planted_mistake(monkeypatch):
     torch.cuda.synchronize()
     assert rep["evaluated"] >= 1 and rep["rejected"] == rep["evaluated"]
     assert rep["best"] == 0
+    dm.dualmv_tune_clear()
+
+
+# ---- single-sided passes --------------------------------------------------
+
+def _sided_variants():
+    out = []
+    for tag in ("f32", "f64"):
+        code = CODE[tag]
+        for i in range(dm.dualmv_variant_count(code)):
+            if dm.dualmv_variant_info(code, i).single_sided:
+                out.append((tag, i))
+    return out
+
+
+@pytest.fixture
+def two_pass_atax():
+    old = dm.dualmv_atax_set_two_pass(1)
+    yield
+    dm.dualmv_atax_set_two_pass(old)
+
+
+@pytest.mark.parametrize("tag,index", _sided_variants())
+@pytest.mark.parametrize("M,N,pad", [(1000, 3000, 0), (3001, 257, 4), (77, 2048, 8)])
+def test_every_single_sided_variant_matches_oracle(tag, index, M, N, pad, forced,
+                                                   two_pass_atax):
+    """A forced variant with single-sided instances runs GESUMMV's two rows
+    passes, ATAX's two passes (rows, then columns) and GEMVER's columns pass:
+    each result against the oracle, and the variant reported launched (entry
+    0 is the passes' default kernel, reported as no variant; rows off the
+    16-byte grid take the plain-load path, which has no variants)."""
+    from test_gpu_ops import check_atax, check_gemver, check_gesummv
+    forced(tag, index)
+    aligned = ((N + pad) * (4 if tag == "f32" else 8)) % 16 == 0
+    launched = index if (index != 0 and aligned) else -1
+    seed = 300 + index + M
+    A, B, x = inputs.generate_gesummv(
+        inputs.Workload("g", tag, M, N, N + pad, DIST[tag], seed, op="gesummv"), DEV)
+    check_gesummv(A, B, x, N, 0.75, -1.25, tag)
+    assert dm.dualmv_last_variant() == launched
+    A, x = inputs.generate_atax(
+        inputs.Workload("a", tag, M, N, N + pad, DIST[tag], seed + 1, op="atax"), DEV)
+    check_atax(A, x, N, tag)
+    assert dm.dualmv_atax_last_path() == dm.DUALMV_ATAX_TWO_PASS
+    assert dm.dualmv_last_variant() == launched
+    ops = inputs.generate_gemver(
+        inputs.Workload("v", tag, M, N, N + pad, DIST[tag], seed + 2, op="gemver"), DEV)
+    check_gemver(ops, N, 1.5, -0.75, False, tag)
+
+
+def _pass_oracle(tag, A, x, rows):
+    An, xn = A.cpu().numpy(), x.cpu().numpy()
+    M, N = An.shape
+    if rows:
+        want, _ = oracle.dualmv(An, xn, np.zeros(M, An.dtype))
+        den, _ = oracle.absdot(An, xn, np.zeros(M, An.dtype))
+    else:
+        _, want = oracle.dualmv(An, np.zeros(N, An.dtype), xn)
+        _, den = oracle.absdot(An, np.zeros(N, An.dtype), xn)
+    return want, den
+
+
+@pytest.mark.parametrize("tag", ["f32", "f64"])
+@pytest.mark.parametrize("pass_", ["rows", "cols"])
+def test_pass_tuner_report_and_choice(tag, pass_, two_pass_atax):
+    M, N = 4096, 8192
+    A, p, r = _make(tag, M, N, N, 31)
+    rows = pass_ == "rows"
+    x = p if rows else r
+    code = CODE[tag]
+    pid = dm.DUALMV_PASS_ROWS if rows else dm.DUALMV_PASS_COLS
+    other = dm.DUALMV_PASS_COLS if rows else dm.DUALMV_PASS_ROWS
+    dm.dualmv_tune_clear()
+    rep = dm.tune_pass(A, x, pass_, repeats=9, trim=2, max_rounds=2, candidates=3,
+                       min_gain=0.0, flush_l2=True)
+    torch.cuda.synchronize()
+    assert rep["initial"] == 0
+    assert dm.dualmv_variant_info(code, rep["best"]).single_sided == 1
+    assert rep["evaluated"] >= 1 and rep["rejected"] == 0
+    assert all(dm.dualmv_variant_info(code, st["index"]).single_sided for st in rep["trace"])
+    assert 0 < rep["best_ms"] <= rep["baseline_ms"]
+    assert rep["worst_fe"] <= TOL[tag]
+    # The result the tuner left is the chosen variant's: against the oracle.
+    want, den = _pass_oracle(tag, A, x, rows)
+    assert scaled_error(rep["out"].cpu().numpy(), want, den) <= TOL[tag]
+    # Recorded for (dtype, M, N, lda, pass) only.
+    assert dm.dualmv_tuned_variant_pass(code, M, N, N, pid) == rep["best"]
+    assert dm.dualmv_tuned_variant_pass(code, M, N, N, other) == -1
+    assert dm.dualmv_tuned_variant(code, M, N, N) == -1
+    # A later forward pass of that shape runs it: GESUMMV's passes (rows),
+    # ATAX's columns pass (cols).
+    launched = rep["best"] if rep["best"] != 0 else -1
+    if rows:
+        dm.gesummv(A, A, p)
+    else:
+        dm.atax(A, p)
+    torch.cuda.synchronize()
+    assert dm.dualmv_last_variant() == launched
+    dm.dualmv_tune_clear()
+    assert dm.dualmv_tuned_variant_pass(code, M, N, N, pid) == -1
+
+
+def test_pass_tuner_catches_a_planted_mistake(monkeypatch):
+    monkeypatch.setenv("DUALMV_FAULT_INJECT", "fe")
+    A, p, r = _make("f32", 2048, 2048, 2048, 37)
+    dm.dualmv_tune_clear()
+    rep = dm.tune_pass(A, r, "cols", repeats=7, trim=1, max_rounds=2, candidates=3,
+                       min_gain=0.0, flush_l2=False)
+    torch.cuda.synchronize()
+    assert rep["evaluated"] >= 1 and rep["rejected"] == rep["evaluated"]
+    assert all(not s["feasible"] and s["fe"] > TOL["f32"] for s in rep["trace"])
+    assert rep["best"] == 0
+    want, den = _pass_oracle("f32", A, r, False)
+    assert scaled_error(rep["out"].cpu().numpy(), want, den) <= TOL["f32"]
     dm.dualmv_tune_clear()

@@ -223,3 +223,74 @@ def test_batched_tune_rejects_bad_arguments(tag):
     assert call(neg_batch) == dm.DUALMV_ERR_INVALID_VALUE
     null_a = good[:2] + (None,) + good[3:]
     assert call(null_a) == dm.DUALMV_ERR_INVALID_VALUE
+
+
+# ---- single-sided passes --------------------------------------------------
+
+def _sided_ids(tab):
+    return {i for i, v in enumerate(tab) if v.single_sided}
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_single_sided_instances(dtype):
+    """fp32: every shape has single-sided instances (the passes of GESUMMV,
+    GEMVER and ATAX's fallback); fp64: the packed self-loading 256-column
+    shapes, entry 0 among them; int32 (no single-sided calls): none.  The
+    tuner's walk over those entries reaches each of them from entry 0."""
+    tab = table(dtype)
+    ids = _sided_ids(tab)
+    for v in tab:
+        assert v.single_sided in (0, 1) and v.pad_ == 0
+    if dtype == dm.DUALMV_DTYPE_I32:
+        assert ids == set()
+        return
+    assert 0 in ids
+    if dtype == dm.DUALMV_DTYPE_F32:
+        assert ids == set(range(len(tab)))
+    else:
+        for i in ids:
+            v = tab[i]
+            assert v.kernel == dm.DUALMV_KERNEL_F64E and v.packed == 1 and \
+                v.producer_warp == 0 and v.band_cols == 256, i
+        assert len(ids) >= 4
+    seen, todo = {0}, [0]
+    while todo:
+        i = todo.pop()
+        for j in ids:
+            if j not in seen and _neighbours(tab[i], tab[j]):
+                seen.add(j)
+                todo.append(j)
+    assert seen == ids
+
+
+def test_no_pass_tuned_variant_recorded_by_default():
+    dm.dualmv_tune_clear()
+    for pass_ in (dm.DUALMV_PASS_ROWS, dm.DUALMV_PASS_COLS):
+        assert dm.dualmv_tuned_variant_pass(dm.DUALMV_DTYPE_F32, 4096, 4096, 4096, pass_) == -1
+    assert dm.dualmv_tuned_variant_pass(dm.DUALMV_DTYPE_F32, 4096, 4096, 4096, 3) == -1
+
+
+@pytest.mark.parametrize("tag", ["f32", "f64"])
+def test_pass_tune_rejects_bad_arguments(tag):
+    fn = getattr(dm, f"dualmv_tune_pass_{tag}")
+    res = dm.TuneResult()
+    rows, cols = dm.DUALMV_PASS_ROWS, dm.DUALMV_PASS_COLS
+    assert fn(64, 64, FAKE, 64, 0, FAKE, FAKE, _cfg(), res, None) == dm.DUALMV_ERR_INVALID_VALUE
+    assert fn(64, 64, FAKE, 64, 3, FAKE, FAKE, _cfg(), res, None) == dm.DUALMV_ERR_INVALID_VALUE
+    for p in (rows, cols):
+        assert fn(64, 64, FAKE, 64, p, FAKE, FAKE, None, res, None) == \
+            dm.DUALMV_ERR_INVALID_VALUE
+        assert fn(64, 64, FAKE, 64, p, FAKE, FAKE, _cfg(repeats=4, trim=2), res, None) == \
+            dm.DUALMV_ERR_INVALID_VALUE
+        assert fn(64, 64, FAKE, 64, p, FAKE, FAKE, _cfg(), None, None) == \
+            dm.DUALMV_ERR_INVALID_VALUE
+        assert fn(64, 64, FAKE, 63, p, FAKE, FAKE, _cfg(), res, None) == \
+            dm.DUALMV_ERR_INVALID_VALUE
+        assert fn(64, 64, None, 64, p, FAKE, FAKE, _cfg(), res, None) == \
+            dm.DUALMV_ERR_INVALID_VALUE
+        assert fn(64, 64, FAKE, 64, p, None, FAKE, _cfg(), res, None) == \
+            dm.DUALMV_ERR_INVALID_VALUE
+        assert fn(64, 64, FAKE, 64, p, FAKE, None, _cfg(), res, None) == \
+            dm.DUALMV_ERR_INVALID_VALUE
+        assert fn(-1, 64, FAKE, 64, p, FAKE, FAKE, _cfg(), res, None) == \
+            dm.DUALMV_ERR_INVALID_VALUE

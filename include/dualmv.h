@@ -420,7 +420,9 @@ dualmv_status dualmv_variant_info(int32_t dtype, int32_t index, dualmv_variant_t
  * dualmv_tune_* recorded one, else entry 0).  A strided-batched call runs
  * the forced variant if it has a batched instance, and a single-sided pass
  * (of GESUMMV, GEMVER's columns pass, ATAX's two passes) if it has
- * single-sided instances; else entry 0.  Returns the previous setting, or
+ * single-sided instances; else entry 0.  Without a forced or tuned variant,
+ * fp64 single-sided passes run entry 1 (8 warps x 4 rows), which their
+ * half-size arithmetic suits better than entry 0's 12 warps.  Returns the previous setting, or
  * -2 for an unknown dtype or an index out of range.  Meant for tests. */
 int32_t dualmv_set_variant(int32_t dtype, int32_t index);
 
@@ -444,9 +446,10 @@ void dualmv_tune_clear(void);
 /* The variant the calling thread's last dual-product call or single-sided
  * pass launched (one problem or a strided batch): its table index, or -1
  * if that call ran no variant of the table (an empty problem, the phased,
- * plain-load or single-cluster path, a single-sided pass on its default
- * kernel or walking its tiles backwards, native fp64 by default, or an
- * error).  Instrumentation for tests and benchmarks. */
+ * plain-load or single-cluster path, an fp32 single-sided pass on its
+ * default kernel (entry 0's shape), a pass walking its tiles backwards,
+ * native fp64 by default, or an error).  Untuned fp64 single-sided passes
+ * run entry 1 and report it.  Instrumentation for tests and benchmarks. */
 int32_t dualmv_last_variant(void);
 
 /* The kind of streaming kernel (DUALMV_KERNEL_*) that the calling thread's
@@ -571,7 +574,8 @@ dualmv_status dualmv_tune_i32_strided_batched(
  * out of length M), DUALMV_PASS_COLS out = A^T x (x of length M, out of
  * length N).  Candidates are the variants with single-sided instances
  * (dualmv_variant_t.single_sided: every fp32 shape, the packed
- * self-loading fp64 shapes); K^(0) is entry 0; Eq. 4 compares `out`.  The
+ * self-loading fp64 shapes); K^(0) is the passes' default, entry 0 for
+ * fp32 and entry 1 (8 warps x 4 rows) for fp64; Eq. 4 compares `out`.  The
  * choice is recorded for (dtype, M, N, lda, pass) and used by later
  * single-sided passes of that shape that walk their tiles forwards
  * (dualmv_tuned_variant_pass; GEMVER's rows pass, which walks backwards to

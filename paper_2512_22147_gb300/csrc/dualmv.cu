@@ -912,6 +912,15 @@ int32_t default_variant(int32_t dtype, const void *A, int64_t lda_bytes) {
     return 0;
 }
 
+// The default of a single-sided pass: fp64 entry 1 (8 warps x 4 rows, 2
+// stages), whose passes, with half the dual product's arithmetic, ran
+// 6-8% faster than entry 0's 12 warps on 8192^2 (the pass tuner's choice
+// for rows and columns); fp32 entry 0.
+constexpr int32_t kF64SidedDefault = 1;
+int32_t sided_default_variant(int32_t dtype) {
+    return dtype == DUALMV_DTYPE_F64 ? kF64SidedDefault : 0;
+}
+
 // The variant a call runs: `index` if the caller (the tuner) names one, else
 // the process-wide forced one, else the tuned one for this shape, else the
 // default for the shape.  nullptr means entry 0, which the ordinary launch
@@ -926,7 +935,10 @@ const Variant *pick_variant(int32_t dtype, int64_t M, int64_t N, const void *A, 
     const bool sided = outputs != dmv::kOutBoth;
     if (index < 0) index = g_forced_variant[dtype].load(std::memory_order_relaxed);
     if (index < 0) index = tuned_lookup(dtype, M, N, lda, batch, outputs);
-    if (index < 0) index = (batch > 1 || sided) ? 0 : default_variant(dtype, A, lda * es);
+    if (index < 0)
+        index = batch > 1 ? 0
+                : sided   ? sided_default_variant(dtype)
+                          : default_variant(dtype, A, lda * es);
     if (index <= 0 || index >= (int32_t)tab->size()) return nullptr;
     if (batch > 1 && (*tab)[index].launch3d == nullptr) return nullptr;
     if (sided && (*tab)[index].launch_q == nullptr) return nullptr;
@@ -2113,7 +2125,9 @@ dualmv_status tune_run(int64_t M, int64_t N, int64_t batch, const T *A, int64_t 
 
     // K^(0): the variant an untuned call of this shape uses; its outputs are
     // the reference for Eq. 4.
-    int32_t base = (batched || sided) ? 0 : default_variant(dtype, A, lda * es);
+    int32_t base = batched ? 0
+                   : sided ? sided_default_variant(dtype)
+                           : default_variant(dtype, A, lda * es);
     res->initial = base;
     st = tu.call(base, true);
     if (st == DUALMV_SUCCESS) st = tu.score(base, &res->baseline_ms);

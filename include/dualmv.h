@@ -447,9 +447,10 @@ void dualmv_tune_clear(void);
  * pass launched (one problem or a strided batch): its table index, or -1
  * if that call ran no variant of the table (an empty problem, the phased,
  * plain-load or single-cluster path, an fp32 single-sided pass on its
- * default kernel (entry 0's shape), a pass walking its tiles backwards,
- * native fp64 by default, or an error).  Untuned fp64 single-sided passes
- * run entry 1 and report it.  Instrumentation for tests and benchmarks. */
+ * default kernel (entry 0's shape, also walking its tiles backwards),
+ * native fp64 by default, or an error).  Untuned fp64 single-sided passes,
+ * GEMVER's backward rows pass among them, run entry 1 and report it.
+ * Instrumentation for tests and benchmarks. */
 int32_t dualmv_last_variant(void);
 
 /* The kind of streaming kernel (DUALMV_KERNEL_*) that the calling thread's
@@ -579,7 +580,8 @@ dualmv_status dualmv_tune_i32_strided_batched(
  * choice is recorded for (dtype, M, N, lda, pass) and used by later
  * single-sided passes of that shape that walk their tiles forwards
  * (dualmv_tuned_variant_pass; GEMVER's rows pass, which walks backwards to
- * start on tiles still in L2, keeps its kernel).  The chosen variant's
+ * start on tiles still in L2, runs the passes' default shape).  The chosen
+ * variant's
  * result is left in `out`.  DUALMV_ERR_INVALID_VALUE for an unknown pass
  * and the argument errors of dualmv_tune_*; blocks until done. */
 enum { DUALMV_PASS_ROWS = 1, DUALMV_PASS_COLS = 2 };

@@ -693,6 +693,9 @@ struct Variant {
     // Single-sided passes (q only, s only: GESUMMV, GEMVER's forward passes,
     // ATAX's two-pass fallback), or nullptr.
     LaunchFn launch_q = nullptr, launch_s = nullptr;
+    // A rows pass walking its tiles backwards (GEMVER's, after its columns
+    // pass), or nullptr: only the fp64 passes' default shape has one.
+    LaunchFn launch_q_rev = nullptr;
 };
 
 template <typename T, int W, int RPW, int S, bool k3d = false>
@@ -715,10 +718,11 @@ cudaError_t launch_stream_side(const CUtensorMap &m, const Params &p, const dual
     return launch_stream<T, true, false, kOut, false, W, RPW, S>(m, p, pl, dev, st);
 }
 
-template <int W, int RPW, int S, int NC, bool kSelf, bool kPack, int BAND, int kOut>
+template <int W, int RPW, int S, int NC, bool kSelf, bool kPack, int BAND, int kOut,
+          bool kRev = false>
 cudaError_t launch_f64e_side(const CUtensorMap &m, const Params &p, const dualmv_plan_t &pl,
                              int dev, cudaStream_t st) {
-    return launch_f64e<false, kOut, W, RPW, S, NC, kSelf, kPack, BAND>(m, p, pl, dev, st);
+    return launch_f64e<false, kOut, W, RPW, S, NC, kSelf, kPack, BAND, kRev>(m, p, pl, dev, st);
 }
 
 Variant make_variant(int32_t index, int32_t kernel, int W, int RPW, int S, Kind kind,
@@ -767,9 +771,11 @@ Variant stream_variant(int32_t index) {
 }
 
 // kBatched: the variant also has a strided-batched instance, and
-// single-sided instances (the packed self-loading 256-column shapes).
+// single-sided instances (the packed self-loading 256-column shapes);
+// kRevQ: a backward rows pass too (the passes' default shape).
 template <int W, int RPW, int S, int NC = kF64eNativeCols, bool kSelf = kF64eSelf,
-          bool kPack = kF64ePack, int BAND = kF64eBand, bool kBatched = false>
+          bool kPack = kF64ePack, int BAND = kF64eBand, bool kBatched = false,
+          bool kRevQ = false>
 Variant f64e_variant(int32_t index) {
     LaunchFn fn3d = nullptr, fn_q = nullptr, fn_s = nullptr;
     if constexpr (kBatched) {
@@ -782,6 +788,8 @@ Variant f64e_variant(int32_t index) {
                              &launch_f64e_variant<W, RPW, S, NC, kSelf, kPack, BAND>, NC, kSelf,
                              fn3d, fn_q, fn_s);
     v.info.packed = kPack ? 1 : 0;
+    if constexpr (kRevQ)
+        v.launch_q_rev = &launch_f64e_side<W, RPW, S, NC, kSelf, kPack, BAND, dmv::kOutQ, true>;
     return v;
 }
 
@@ -833,7 +841,7 @@ const std::vector<Variant> &i32_table() {
 const std::vector<Variant> &f64_table() {
     static const std::vector<Variant> tab = {
         f64e_variant<12, 4, 2, 0, true, true, kF64eBand, true>(0),
-        f64e_variant<8, 4, 2, 0, true, true, kF64eBand, true>(1),
+        f64e_variant<8, 4, 2, 0, true, true, kF64eBand, true, true>(1),  // fp64 passes' default
         f64e_variant<8, 4, 3, 0, true, false>(2),    // scalar FP32 instructions
         f64e_variant<8, 4, 3, 2, true, false>(3),
         f64e_variant<8, 4, 3, 3, true, false>(4),
@@ -1121,8 +1129,17 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     // TMA path.
     const Variant *var = nullptr;
     if (tma && rank2 == nullptr && g_path != DUALMV_PATH_TMA_NATIVE_F64 &&
-        (outputs == dmv::kOutBoth || (!kIntPath && batch == 1 && !reverse)))
-        var = pick_variant(dtype_code<T>(), M, N, A, lda, es, variant, batch, outputs);
+        (outputs == dmv::kOutBoth || (!kIntPath && batch == 1))) {
+        if (outputs == dmv::kOutQ && reverse) {
+            // A rows pass walking backwards: the passes' default shape, if it
+            // has a backward instance (fp64 entry 1); else the default kernel.
+            const std::vector<Variant> &tab = *variant_table(dtype_code<T>());
+            const int32_t d = sided_default_variant(dtype_code<T>());
+            if (d > 0 && tab[d].launch_q_rev != nullptr) var = &tab[d];
+        } else if (!reverse) {
+            var = pick_variant(dtype_code<T>(), M, N, A, lda, es, variant, batch, outputs);
+        }
+    }
     if (var != nullptr) kind = var->kind;
     if (kind == Kind::kF64e) {
         // The double-float kernel counts tiles in 32 bits; a launch of 2^31
@@ -1238,7 +1255,8 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
     if (e == cudaSuccess) {
         if (var != nullptr) {
             if (outputs == dmv::kOutQ)
-                e = var->launch_q(map, prm, pl, dev, stream);
+                e = reverse ? var->launch_q_rev(map, prm, pl, dev, stream)
+                            : var->launch_q(map, prm, pl, dev, stream);
             else if (outputs == dmv::kOutS)
                 e = var->launch_s(map, prm, pl, dev, stream);
             else

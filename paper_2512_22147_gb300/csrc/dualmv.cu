@@ -1281,6 +1281,8 @@ dualmv_status run(int64_t M, int64_t N, const T *A, int64_t lda, int64_t strideA
                 // A walks each CTA's tiles backwards (see Deferred).
                 const bool rev = reverse && only_q;
                 if (kind == Kind::kF64e) {
+                    // Entry 0's shape: untuned fp64 passes run entry 1 as a
+                    // variant (above); this serves a forced or tuned entry 0.
                     if constexpr (std::is_same<T, double>::value)
                         e = rev ? launch_f64e<false, dmv::kOutQ, kF64eWarps, kF64eRpw, kF64eStages,
                                               kF64eNativeCols, kF64eSelf, kF64ePack, kF64eBand,

@@ -294,3 +294,23 @@ def test_pass_tune_rejects_bad_arguments(tag):
             dm.DUALMV_ERR_INVALID_VALUE
         assert fn(-1, 64, FAKE, 64, p, FAKE, FAKE, _cfg(), res, None) == \
             dm.DUALMV_ERR_INVALID_VALUE
+
+
+def test_tune_pass_api_rejects_bad_arguments():
+    """api.tune_pass checks its tensors before any library call."""
+    torch = pytest.importorskip("torch")
+    A = torch.zeros(4, 6, dtype=torch.float32)
+    with pytest.raises(ValueError):
+        dm.tune_pass(A, torch.zeros(6), "diagonal")
+    with pytest.raises(ValueError):
+        dm.tune_pass(A.to(torch.int32), torch.zeros(6, dtype=torch.int32), "rows")
+    with pytest.raises(ValueError):
+        dm.tune_pass(A[None], torch.zeros(6), "rows")
+    with pytest.raises(ValueError):            # rows: x has N = 6 elements
+        dm.tune_pass(A, torch.zeros(4), "rows")
+    with pytest.raises(ValueError):            # cols: x has M = 4 elements
+        dm.tune_pass(A, torch.zeros(6), "cols")
+    with pytest.raises(ValueError):            # out of the wrong length
+        dm.tune_pass(A, torch.zeros(6), "rows", out=torch.zeros(6))
+    with pytest.raises(ValueError):            # x of another dtype
+        dm.tune_pass(A, torch.zeros(6, dtype=torch.float64), "rows")
